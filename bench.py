@@ -1,0 +1,380 @@
+"""Benchmark of the fuse-and-verify step on GB300.
+
+One step = one pass of the whole path over one batch: the C-ABI call
+asymspec_fuse_verify_ex in stochastic mode (row normalisers, delta fusion,
+JSD gate, acceptance tests, residual inverse-CDF draws, fused argmax and the
+per-element accept scan), which is one kernel launch.  The workload is
+B=64, K=7, V=128256 bf16 logits with the Zipf-profile recipe (512 verify
+rows, 394 MB of logits per step, larger than the 129 MB L2; two input sets
+are rotated).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl asymspec|reference]
+
+Under torchrun every rank runs its own replica of the workload on its own GPU
+(weak scaling, no collective on the data path); rank 0 prints one JSON line.
+``--impl reference`` times the float64 CPU oracle on the same workload (a
+bounded sample of batch elements per step) on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "verify rows/s (B×(K+1) vocab rows) and achieved HBM GB/s vs GB300 peak"
+WORKLOAD_CFG = 2
+FALLBACK_HBM_GBS = 6800.0
+KERNEL_SRC = os.path.join(ROOT, "paper_2608_26004_gb300", "csrc", "asymspec.cu")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_fuse_verify_B64_K7_V128256_bf16.json")
+REASON_BITS = {
+    0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
+    0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
+    0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+    0x100: "display_clock_setting",
+}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="asymspec", choices=["asymspec", "reference"])
+    ap.add_argument("--mode", default="stochastic", choices=["stochastic", "greedy"])
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="first B batch elements only (profiling a smaller case)")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_hash() -> str:
+    with open(KERNEL_SRC, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def measured_traffic(mode: str):
+    """DRAM bytes per launch from a committed ncu summary of the same kernel source."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            d = json.load(f)
+    except Exception:
+        return None
+    if d.get("kernel_sha256_16") != kernel_hash():
+        return None
+    v = d.get("dram_bytes_per_launch", {}).get(mode)
+    return float(v) if v else None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_bench_{os.getpid()}.csv")
+
+    def __enter__(self):
+        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index),
+                 "--query-gpu=index,clocks.sm,clocks.max.sm,power.draw,"
+                 "clocks_event_reasons.active", "--format=csv,noheader,nounits", "-lms", "20"],
+                stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        try:
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 5:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                    bits = int(parts[4], 16)
+                except ValueError:
+                    continue
+                for b, name in REASON_BITS.items():
+                    if bits & b and name != "gpu_idle":
+                        reasons.add(name)
+        except OSError:
+            pass
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(smax)),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def oracle_rows_per_s(batch, mode_id, seconds: float):
+    """The oracle as it stands, on consecutive batch elements, for ~`seconds`."""
+    import oracle
+    t0 = time.perf_counter()
+    rows = 0
+    b = 0
+    while True:
+        sel = slice(b % batch.B, b % batch.B + 1)
+        oracle.fuse_verify(batch.logits_full[sel], batch.logits_comp[sel], batch.logits_ver[sel],
+                           batch.draft_tokens[sel], batch.draft_probs[sel], batch.uniforms[sel],
+                           dtype=batch.dtype, mode=mode_id)
+        rows += batch.K + 1
+        b += 1
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            return rows / el, rows, el
+
+
+def run_reference(args, workload, rank, world):
+    """--impl reference: the float64 CPU oracle, timed on the host cores."""
+    from paper_2608_26004_gb300 import synth
+    if rank != 0:
+        return
+    mode_id = 1 if args.mode == "stochastic" else 0
+    sample_b = 2
+    batch = synth.make_config(WORKLOAD_CFG, nb=sample_b)
+    for _ in range(args.warmup):
+        oracle_rows_per_s(batch, mode_id, 0.0)
+    t0 = time.perf_counter()
+    rows = 0
+    for s in range(args.steps):
+        b = s % sample_b
+        import oracle
+        oracle.fuse_verify(batch.logits_full[b:b + 1], batch.logits_comp[b:b + 1],
+                           batch.logits_ver[b:b + 1], batch.draft_tokens[b:b + 1],
+                           batch.draft_probs[b:b + 1], batch.uniforms[b:b + 1],
+                           dtype=batch.dtype, mode=mode_id)
+        rows += batch.K + 1
+    el = time.perf_counter() - t0
+    value = rows / el
+    sample = (f"each step: 1 batch element (K+1={batch.K + 1} rows of V={batch.V}) of "
+              f"{workload.name}, float64 numpy oracle, single thread")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "rows/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * el / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload.name, "B": workload.B, "K": workload.K,
+                   "V": workload.V, "logits": "bf16", "mode": args.mode},
+        "cpu_baseline": {"value": value, "unit": "rows/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    rank, world, local = dist_env()
+    from paper_2608_26004_gb300 import synth
+    workload = synth.CONFIGS[WORKLOAD_CFG]
+    if args.impl == "reference":
+        run_reference(args, workload, rank, world)
+        return
+
+    import torch
+    from paper_2608_26004_gb300 import asymspec as A
+
+    assert torch.cuda.is_available(), "bench.py needs a CUDA device"
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+
+    mode = A.MODE_STOCHASTIC if args.mode == "stochastic" else A.MODE_GREEDY
+    batch = synth.make_config(WORKLOAD_CFG, nb=args.batch or None)
+    B, K, V = batch.B, batch.K, batch.V
+    rows = B * (K + 1)
+    alg_bytes = 3 * rows * V * 2 + rows * 12 + B * 8  # logits once + token/prob/uniform + outputs
+
+    def to_dev_logits(x):
+        return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    sets = []
+    for rep in range(2):  # two resident input sets, rotated (each larger than L2)
+        sets.append(dict(
+            a=to_dev_logits(batch.logits_full), b=to_dev_logits(batch.logits_comp),
+            t=to_dev_logits(batch.logits_ver),
+            tok=torch.from_numpy(batch.draft_tokens).to(dev),
+            prob=torch.from_numpy(batch.draft_probs).to(dev),
+            unif=torch.from_numpy(batch.uniforms).to(dev)))
+    L = torch.empty(B, dtype=torch.int32, device=dev)
+    N = torch.empty(B, dtype=torch.int32, device=dev)
+    nbytes = A.workspace_bytes(B, K, V)
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+    gate = A.gate_params(mode=mode)
+    stream = torch.cuda.current_stream(dev)
+    sptr = stream.cuda_stream
+    info = A.plan(B, K, V, A.BF16, gate)
+
+    def step(x):
+        st = A.fuse_verify_ex(x["a"].data_ptr(), x["b"].data_ptr(), x["t"].data_ptr(),
+                              x["tok"].data_ptr(), x["prob"].data_ptr(), x["unif"].data_ptr(),
+                              B, K, V, A.BF16, gate, L.data_ptr(), N.data_ptr(), ws.data_ptr(),
+                              nbytes, stream=sptr)
+        if st != A.OK:
+            raise A.AsymSpecError(st, "asymspec_fuse_verify_ex")
+
+    def timed(fn, steps, warmup):
+        for i in range(warmup):
+            fn(i)
+        torch.cuda.synchronize(dev)
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize(dev)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(steps):
+            fn(i)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize(dev)
+        ms = e0.elapsed_time(e1)
+        if pg:
+            t = torch.tensor([ms], device=dev)
+            pg.all_reduce(t, op=pg.ReduceOp.MAX)
+            ms = float(t.item())
+        return ms
+
+    # ---- device-resident throughput (the headline value)
+    with ClockSampler(local) as clk:
+        ms = timed(lambda i: step(sets[i % 2]), args.steps, max(args.warmup, 3))
+    clocks = clk.summary()
+    ms_step = ms / args.steps
+    value = world * rows / (ms_step * 1e-3)
+    launch_s = ms_step * 1e-3  # one launch per step
+    hbm_peak, peak_kind = peaks()
+    achieved = alg_bytes / launch_s / 1e9
+
+    # ---- the other mode, same workload (reported alongside)
+    other_mode = A.MODE_GREEDY if mode == A.MODE_STOCHASTIC else A.MODE_STOCHASTIC
+    gate_o = A.gate_params(mode=other_mode)
+
+    def step_o(x):
+        st = A.fuse_verify_ex(x["a"].data_ptr(), x["b"].data_ptr(), x["t"].data_ptr(),
+                              x["tok"].data_ptr(), x["prob"].data_ptr(), x["unif"].data_ptr(),
+                              B, K, V, A.BF16, gate_o, L.data_ptr(), N.data_ptr(), ws.data_ptr(),
+                              nbytes, stream=sptr)
+        if st != A.OK:
+            raise A.AsymSpecError(st, "asymspec_fuse_verify_ex")
+
+    ms_o = timed(lambda i: step_o(sets[i % 2]), args.steps, max(args.warmup, 3)) / args.steps
+
+    # ---- end to end through the C ABI with host buffers
+    pin = dict(
+        a=torch.from_numpy(np.ascontiguousarray(batch.logits_full).view(np.int16)).view(
+            torch.bfloat16).pin_memory(),
+        b=torch.from_numpy(np.ascontiguousarray(batch.logits_comp).view(np.int16)).view(
+            torch.bfloat16).pin_memory(),
+        t=torch.from_numpy(np.ascontiguousarray(batch.logits_ver).view(np.int16)).view(
+            torch.bfloat16).pin_memory(),
+        tok=torch.from_numpy(batch.draft_tokens).pin_memory(),
+        prob=torch.from_numpy(batch.draft_probs).pin_memory(),
+        unif=torch.from_numpy(batch.uniforms).pin_memory())
+    hL = torch.empty(B, dtype=torch.int32).pin_memory()
+    hN = torch.empty(B, dtype=torch.int32).pin_memory()
+    h2d = sum(v.numel() * v.element_size() for v in pin.values())
+    d2h = 2 * B * 4
+    x0 = sets[0]
+
+    def e2e_step(i):
+        for key in pin:
+            x0[key].copy_(pin[key], non_blocking=True)
+        step(x0)
+        hL.copy_(L, non_blocking=True)
+        hN.copy_(N, non_blocking=True)
+
+    e2e_steps = max(3, min(args.steps, 30))
+    ms_e2e = timed(e2e_step, e2e_steps, 3) / e2e_steps
+    e2e_value = world * rows / (ms_e2e * 1e-3)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": workload.name if B == workload.B else f"{workload.name}_first{B}",
+                   "B": B, "K": K, "V": V, "logits": "bf16",
+                   "mode": args.mode, "rows_per_gpu": rows, "gamma": 0.5, "beta": 1.0,
+                   "divergence": "jsd",
+                   "l2": "inputs larger than L2: 2 resident sets of 394 MB rotated",
+                   "cluster_size": info.cluster_size, "ctas": info.ctas,
+                   "parallelism": f"replicas x{world}"},
+        "hbm_gbs": achieved,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved / hbm_peak, "peak_kind": peak_kind,
+                     "traffic": measured_traffic(args.mode),
+                     "algorithmic_bytes_per_launch": alg_bytes},
+        "e2e": {"value": e2e_value, "unit": "rows/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e},
+        "gpu_launches": args.steps,
+        "clocks": clocks,
+        "other_mode": {"mode": "greedy" if other_mode == A.MODE_GREEDY else "stochastic",
+                       "ms_per_step": ms_o, "rows_per_s": world * rows / (ms_o * 1e-3),
+                       "hbm_gbs": alg_bytes / (ms_o * 1e-3) / 1e9},
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        mode_id = 1 if mode == A.MODE_STOCHASTIC else 0
+        rps, nrows, el = oracle_rows_per_s(batch, mode_id, args.cpu_seconds)
+        line["cpu_baseline"] = {
+            "value": rps, "unit": "rows/s", "cores": 1, "kind": "oracle",
+            "sample": f"{nrows} rows ({nrows // (K + 1)} batch elements) of {workload.name} "
+                      f"in {el:.1f} s, float64 numpy oracle, single thread"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,189 @@
+/*
+ * asymspec.h -- C ABI of the AsymSpec per-step fuse-and-verify path on GB300.
+ *
+ * The operation (paper: "AsymSpec: Context-Asymmetric Speculative Decoding for
+ * Agentic LLMs", Section 3 and Algorithm 1).  Each speculation step produces,
+ * for every batch element b and each of its K+1 positions k (row k predicts
+ * the token at position k+1; row K is the position after the last draft),
+ * three vocabulary-wide logit rows:
+ *   logits_full  a = drafter S on the full context        (Section 3.2, item 1)
+ *   logits_comp  b = drafter S on the compressed context  (Section 3.2, item 2)
+ *   logits_ver   t = verifier L on the compressed context (Section 3.2, item 3)
+ * and the drafter's K draft tokens d.  Per row the library computes the
+ * log-softmax normalisers of a, b, t and of the fused scores
+ * s = t + beta * (a - b) (Eqs. 1-2), the Jensen-Shannon divergence
+ * D = JSD(softmax a || softmax b) and the threshold gamma_eff = gamma exp(-D)
+ * (Eq. 3), the acceptance test of Eq. 4, and then, per batch element, the
+ * sequential accept scan of Algorithm 1:
+ *   greedy mode: accept d_k iff softmax(t_k)[d_k] > gamma_eff(k) softmax(b_k)[d_k];
+ *     the first rejected position emits argmax(s_k); if all K pass, the bonus
+ *     position emits argmax(t_K) (argmax(s_K) with fuse_bonus);
+ *   stochastic mode (an extension; the paper decodes greedily): accept d_k iff
+ *     q_k(d_k) / draft_probs[k] > u_k gamma_eff(k) with q_k = softmax(s_k); the
+ *     first rejected position draws from max(0, q_k - softmax(a_k)) normalised
+ *     (from q_k if that residual is identically zero) by inverse CDF at u_K;
+ *     if all K pass, the bonus position draws from q_K at u_K.
+ * Ties in an argmax resolve to the lowest index; inverse-CDF draws return the
+ * smallest index whose cumulative mass (in index order) exceeds the target.
+ *
+ * Conventions for every entry point below:
+ *  - Array arguments are caller-owned DEVICE pointers unless stated; the
+ *    library never frees or retains them.  Logit tensors are [B, K+1, V]
+ *    row-major in the dtype given (fp32, or bf16 as 16-bit words), with rows
+ *    16-byte aligned for the fast path (any element-aligned pointer works; a
+ *    slower path handles the rest).
+ *  - All work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream) and is asynchronous: results are valid once the stream has
+ *    completed.  Calls on different streams are independent and may run
+ *    concurrently if their workspaces differ.
+ *  - Return values are ASYMSPEC_* status codes; host-detectable errors are
+ *    reported before anything is enqueued.  Problems in the DATA (found on the
+ *    device) never trap: the affected batch element gets accept_len = -1 and
+ *    next_token = -1 and a bit is OR-ed into the optional device error word.
+ *  - Inputs must be finite.  A NaN or +inf logit is detected (the element's
+ *    normalisers become non-finite); a -inf logit is outside the contract.
+ */
+#ifndef ASYMSPEC_H
+#define ASYMSPEC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+#define ASYMSPEC_OK 0
+#define ASYMSPEC_ERR_INVALID_ARG (-1)   /* null pointer, B<1, K<1, V<2, gamma or beta out of range */
+#define ASYMSPEC_ERR_UNSUPPORTED (-2)   /* unknown dtype, mode or divergence */
+#define ASYMSPEC_ERR_MISALIGNED (-3)    /* a pointer not aligned to its element size */
+#define ASYMSPEC_ERR_WORKSPACE (-4)     /* workspace missing or smaller than asymspec_workspace_bytes() */
+#define ASYMSPEC_ERR_CUDA (-5)          /* a CUDA call failed; see asymspec_last_cuda_error() */
+#define ASYMSPEC_ERR_TOO_LARGE (-6)     /* V too large for the on-chip row slices (see asymspec_plan) */
+
+/* ---- device error-word bits (data errors, per batch element) ----------- */
+#define ASYMSPEC_DATA_BAD_TOKEN 0x1u    /* a draft token outside [0, V) */
+#define ASYMSPEC_DATA_NONFINITE 0x2u    /* a non-finite normaliser or divergence (NaN/inf logits) */
+#define ASYMSPEC_DATA_BAD_PROB 0x4u     /* stochastic: draft probability outside (0, 1] */
+#define ASYMSPEC_DATA_BAD_UNIFORM 0x8u  /* stochastic: uniform outside [0, 1) */
+
+typedef enum { ASYMSPEC_FP32 = 0, ASYMSPEC_BF16 = 1 } asymspec_dtype_t;
+
+typedef enum {
+  ASYMSPEC_MODE_GREEDY = 0,      /* Algorithm 1 (tau = 0, the paper's setting) */
+  ASYMSPEC_MODE_STOCHASTIC = 1   /* speculative sampling with the CDA-relaxed threshold */
+} asymspec_mode_t;
+
+typedef enum {
+  ASYMSPEC_DIV_JSD = 0,    /* Eq. 3: D = JSD(softmax a || softmax b), natural log (default) */
+  ASYMSPEC_DIV_NONE = 1,   /* fixed-gamma gate: gamma_eff = gamma (Appendix B baseline) */
+  ASYMSPEC_DIV_KL = 2,     /* D = KL(softmax a || softmax b) (Table "JSD vs KL") */
+  ASYMSPEC_DIV_LAMBDA = 3  /* gamma_eff = gamma exp(-lambda (log p_a(d) - log p_b(d))) (Appendix B) */
+} asymspec_div_t;
+
+/* Hyper-parameters of the step (host struct, read during the call). */
+typedef struct {
+  float gamma;         /* base threshold, in (0, 1]; paper default 0.5 (Algorithm 1, Section 4.2) */
+  float beta;          /* fusion weight, finite and >= 0; paper default 1.0 (Eq. 2) */
+  float lambda;        /* only for ASYMSPEC_DIV_LAMBDA; paper default 0.1 (Appendix B) */
+  int32_t mode;        /* asymspec_mode_t */
+  int32_t divergence;  /* asymspec_div_t */
+  int32_t fuse_bonus;  /* greedy: 0 = bonus emits argmax(t_K) as in Algorithm 1; 1 = argmax(s_K) */
+  int32_t flags;       /* reserved, must be 0 */
+} asymspec_gate_params;
+
+/* Optional launch overrides (host struct); zero fields mean "automatic". */
+typedef struct {
+  int32_t cluster_size;   /* CTAs per row triple: 1, 2, 4, 8 or 16 */
+  int32_t block_threads;  /* reserved, must be 0 (256 threads per CTA) */
+} asymspec_launch_opts;
+
+/* What a launch would use (filled by asymspec_plan). */
+typedef struct {
+  int32_t cluster_size;    /* CTAs that split one row triple, combined over DSMEM */
+  int32_t block_threads;   /* threads per CTA */
+  int32_t slice_elems;     /* vocabulary entries held on chip per CTA */
+  int32_t smem_bytes;      /* dynamic shared memory per CTA */
+  int64_t ctas;            /* CTAs in the grid = B (K+1) cluster_size */
+  int32_t vector_path;     /* 1 if rows qualify for 16-byte copies (V * element size % 16 == 0) */
+  int32_t max_active_clusters; /* clusters the device can hold at once (0 if unknown) */
+} asymspec_launch_info;
+
+/* Fills *p with the paper's defaults: gamma 0.5, beta 1.0, lambda 0.1,
+ * greedy mode, JSD gate, unfused bonus (Section 4.2, Appendix B). */
+void asymspec_default_gate_params(asymspec_gate_params* p);
+
+/* Bytes of device workspace asymspec_fuse_verify_ex needs for a batch of
+ * B elements with K drafts (independent of V).  The workspace must be zeroed
+ * once before its first use (cudaMemset or asymspec_workspace_reset); every
+ * call that completes leaves it zeroed again.  Two calls in flight at the
+ * same time must not share a workspace. */
+size_t asymspec_workspace_bytes(int B, int K, int V);
+
+/* Enqueues a zero fill of a workspace on `stream`. */
+int asymspec_workspace_reset(void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * The step with the paper's problem statement as arguments (Section 3).
+ *   logits_full, logits_comp, logits_ver: [B, K+1, V] device, dtype `dtype`
+ *   draft_tokens: [B, K] int32 device
+ *   draft_probs:  [B, K] fp32 device, the drafter's probability of each draft
+ *                 (stochastic mode; may be NULL in greedy mode)
+ *   uniforms:     [B, K+1] fp32 device in [0, 1): u[b][k] for the k-th test,
+ *                 u[b][K] for the one non-draft draw (stochastic; NULL in greedy)
+ *   gate_params:  host pointer, NULL = asymspec_default_gate_params
+ *   out_accept_len, out_next_token: [B] int32 device outputs
+ * Obtains its workspace with cudaMallocAsync/cudaFreeAsync on `stream`.
+ */
+int asymspec_fuse_verify(const void* logits_full, const void* logits_comp,
+                         const void* logits_ver, const int32_t* draft_tokens,
+                         const float* draft_probs, const float* uniforms, int B, int K,
+                         int V, int dtype, const asymspec_gate_params* gate_params,
+                         int32_t* out_accept_len, int32_t* out_next_token, void* stream);
+
+/*
+ * As asymspec_fuse_verify, with a caller-owned workspace and optional outputs:
+ *   workspace, workspace_bytes: device scratch of asymspec_workspace_bytes()
+ *       bytes, zeroed before first use (see above)
+ *   out_row_stats:  [B, K+1, 8] fp32 device or NULL: per row LSE(a), LSE(b),
+ *       LSE(t), LSE(s), D, gamma_eff, acceptance margin (greedy
+ *       1 - ratio/gamma_eff, stochastic u - ratio/gamma_eff; NaN on row K) and
+ *       the inverse-CDF mass used (stochastic) or NaN
+ *   out_row_tokens: [B, K+1, 2] int32 device or NULL: per row argmax(s) and
+ *       the token emitted if the scan stops at that row
+ *   out_fused_logprobs: [B, K+1, V] fp32 device or NULL: log softmax(s), the
+ *       fused target (a debug output that adds 4 V bytes of writes per row)
+ *   out_error_word: one uint32 device word or NULL; ASYMSPEC_DATA_* bits are
+ *       OR-ed into it (the caller clears it)
+ *   opts: NULL for automatic launch parameters
+ */
+int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
+                            const void* logits_ver, const int32_t* draft_tokens,
+                            const float* draft_probs, const float* uniforms, int B, int K,
+                            int V, int dtype, const asymspec_gate_params* gate_params,
+                            int32_t* out_accept_len, int32_t* out_next_token,
+                            void* workspace, size_t workspace_bytes, float* out_row_stats,
+                            int32_t* out_row_tokens, float* out_fused_logprobs,
+                            uint32_t* out_error_word, const asymspec_launch_opts* opts,
+                            void* stream);
+
+/* Launch parameters a call with these sizes would use, without launching.
+ * Uses the current CUDA device. */
+int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* gate_params,
+                  const asymspec_launch_opts* opts, asymspec_launch_info* out);
+
+/* Static description of a status code. */
+const char* asymspec_status_string(int status);
+
+/* The cudaError_t of the last ASYMSPEC_ERR_CUDA returned on this thread. */
+int asymspec_last_cuda_error(void);
+
+/* Library version: major * 10000 + minor * 100 + patch. */
+int asymspec_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ASYMSPEC_H */

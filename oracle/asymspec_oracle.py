@@ -305,6 +305,7 @@ class Result:
     D: np.ndarray               # [B, K+1]
     gamma_eff: np.ndarray       # [B, K+1]
     fused_argmax: np.ndarray    # [B, K+1] argmax of t + beta * delta
+    fused_gap_flag: np.ndarray  # [B, K+1] that argmax is a near-tie
     candidate: np.ndarray       # [B, K+1] token emitted if the scan stops at this row
     cand_flag: np.ndarray       # [B, K+1] the candidate's own decision is a near-tie
     accept: np.ndarray          # [B, K] per-draft decisions
@@ -343,6 +344,7 @@ def fuse_verify(logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=
         flagged=np.zeros(B, bool), error=np.zeros(B, bool),
         lse=np.full((B, K1, 4), np.nan), D=np.full((B, K1), np.nan),
         gamma_eff=np.full((B, K1), np.nan), fused_argmax=np.full((B, K1), -1, np.int64),
+        fused_gap_flag=np.zeros((B, K1), bool),
         candidate=np.full((B, K1), -1, np.int64), cand_flag=np.zeros((B, K1), bool),
         accept=np.zeros((B, K), bool), accept_margin=np.full((B, K), np.nan),
         logprobs=np.full((B, K1, V), np.nan) if want_logprobs else None)
@@ -369,6 +371,8 @@ def fuse_verify(logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=
             res.D[bi, k] = r.D
             res.gamma_eff[bi, k] = r.gamma_eff
             res.fused_argmax[bi, k] = argmax_first(r.s)
+            res.fused_gap_flag[bi, k] = (top2_gap(r.s)
+                                         < ARGMAX_BAND * max(1.0, abs(float(np.max(r.s)))))
             if want_logprobs:
                 res.logprobs[bi, k] = r.lq
         if mode == GREEDY:

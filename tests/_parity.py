@@ -1,0 +1,106 @@
+"""Shared helpers of the GPU parity tests: run the C ABI, compare with the oracle."""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle as O
+from paper_2608_26004_gb300 import asymspec as A
+from paper_2608_26004_gb300 import synth
+
+LOGPROB_TOL = {synth.FP32: 1e-5, synth.BF16: 2e-3}
+LSE_TOL = 2e-5
+D_TOL = 1e-5
+GAMMA_TOL = 1e-5
+
+
+def device_inputs(batch, torch, device="cuda"):
+    """Host arrays of a synth.Batch (or an equivalent object) as CUDA tensors."""
+    def logits(x):
+        if batch.dtype == synth.BF16:
+            t = torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16)
+        else:
+            t = torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32))
+        return t.to(device)
+    return dict(
+        a=logits(batch.logits_full), b=logits(batch.logits_comp), t=logits(batch.logits_ver),
+        tokens=torch.from_numpy(np.ascontiguousarray(batch.draft_tokens, np.int32)).to(device),
+        probs=torch.from_numpy(np.ascontiguousarray(batch.draft_probs, np.float32)).to(device),
+        unif=torch.from_numpy(np.ascontiguousarray(batch.uniforms, np.float32)).to(device))
+
+
+def run_gpu(batch, torch, *, mode, divergence=A.DIV_JSD, gamma=0.5, beta=1.0, lam=0.1,
+            fuse_bonus=False, cluster_size=0, logprobs=True, inputs=None):
+    """One call of asymspec_fuse_verify_ex through the binding; numpy results."""
+    x = inputs if inputs is not None else device_inputs(batch, torch)
+    fv = A.FuseVerify(batch.B, batch.K)
+    res = fv(x["a"], x["b"], x["t"], x["tokens"], x["probs"], x["unif"], gamma=gamma, beta=beta,
+             lam=lam, mode=mode, divergence=divergence, fuse_bonus=fuse_bonus,
+             row_stats=True, row_tokens=True, fused_logprobs=logprobs,
+             cluster_size=cluster_size)
+    torch.cuda.synchronize()
+    out = {k: v.cpu().numpy() for k, v in res.items()}
+    out["workspace_after"] = fv.workspace.cpu().numpy()
+    return out
+
+
+def run_oracle(batch, *, mode, divergence=A.DIV_JSD, gamma=0.5, beta=1.0, lam=0.1,
+               fuse_bonus=False, logprobs=True, select=None):
+    sel = slice(None) if select is None else select
+    return O.fuse_verify(batch.logits_full[sel], batch.logits_comp[sel], batch.logits_ver[sel],
+                         batch.draft_tokens[sel], batch.draft_probs[sel], batch.uniforms[sel],
+                         dtype=batch.dtype, gamma=gamma, beta=beta, mode=mode,
+                         divergence=divergence, lam=lam, fuse_bonus=fuse_bonus,
+                         want_logprobs=logprobs)
+
+
+def compare(batch, g, o, *, mode, select=None, logprobs=True, check_stats=True):
+    """Asserts GPU == oracle within the stated tolerances; returns counters.
+
+    accept_len / next_token: bit-exact except batch elements the oracle flags
+    as reaching a near-tie.  Per-row decisions and tokens: exact except rows
+    whose own decision is a near-tie.  Fused log-probs: max |error| within
+    2e-3 (bf16 inputs) or 1e-5 (fp32 inputs).
+    """
+    sel = np.arange(batch.B) if select is None else np.asarray(select)
+    L, N = g["accept_len"][sel], g["next_token"][sel]
+    err = o.error
+    assert np.array_equal(L < 0, err), "data-error elements differ"
+    assert np.array_equal(N < 0, err)
+    ok = ~o.flagged & ~err
+    bad = np.nonzero(ok & ((L != o.accept_len) | (N != o.next_token)))[0]
+    assert bad.size == 0, (
+        f"accept/next mismatch at b={sel[bad][:8]}: gpu {L[bad][:8]} {N[bad][:8]} "
+        f"oracle {o.accept_len[bad][:8]} {o.next_token[bad][:8]}")
+    K1 = batch.K + 1
+    rt = g["row_tokens"][sel]
+    rs = g["row_stats"][sel]
+    good = ~err
+    fa_ok = good[:, None] & ~o.fused_gap_flag
+    assert np.array_equal(rt[..., 0][fa_ok], o.fused_argmax[fa_ok]), "fused argmax differs"
+    c_ok = good[:, None] & ~o.cand_flag
+    cbad = np.argwhere(c_ok & (rt[..., 1] != o.candidate))
+    assert cbad.size == 0, f"row candidates differ at {cbad[:6]}"
+    acc_gpu = rs[:, :batch.K, 6] < 0
+    m_ok = good[:, None] & (np.abs(o.accept_margin) >= O.ACCEPT_BAND)
+    abad = np.argwhere(m_ok & (acc_gpu != o.accept))
+    assert abad.size == 0, f"acceptance decisions differ at {abad[:6]}"
+    if check_stats:
+        gl = rs[good][..., :4]
+        ol = o.lse[good]
+        assert np.nanmax(np.abs(gl - ol)) <= LSE_TOL * max(1.0, float(np.max(np.abs(ol)))), \
+            f"LSE error {np.nanmax(np.abs(gl - ol))}"
+        dD = np.abs(rs[good][..., 4] - o.D[good])
+        assert np.max(dD) <= D_TOL, f"D error {np.max(dD)}"
+        dg = np.abs(rs[good][..., 5] - o.gamma_eff[good])
+        assert np.max(dg) <= GAMMA_TOL, f"gamma_eff error {np.max(dg)}"
+    lp_err = None
+    if logprobs and o.logprobs is not None:
+        glp = g["fused_logprobs"][sel][good]
+        lp_err = float(np.max(np.abs(glp - o.logprobs[good]))) if good.any() else 0.0
+        assert lp_err <= LOGPROB_TOL[batch.dtype], f"fused log-prob error {lp_err}"
+    # the per-element tickets (after the 256-byte aligned row records) return to zero
+    rec_bytes = -(-batch.B * K1 * 16 // 256) * 256
+    tickets = g["workspace_after"][rec_bytes:rec_bytes + 4 * batch.B]
+    assert np.all(tickets == 0), "tickets not left zeroed"
+    return dict(compared=int(ok.sum()), flagged=int(o.flagged.sum()),
+                errors=int(err.sum()), logprob_err=lp_err, rows=int(len(sel) * K1))

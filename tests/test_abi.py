@@ -1,0 +1,120 @@
+"""The C-ABI library builds, loads and exports what include/asymspec.h declares.
+
+No compute call is made here: only entry points that return before touching
+the GPU (argument validation, sizes, strings) are exercised.
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_26004_gb300 import asymspec as A
+from paper_2608_26004_gb300 import build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build_cuda()
+    return A.lib()
+
+
+def declared_functions():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"\b(asymspec_\w+)\s*\(", src))
+    return names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert names == set(A.EXPORTED)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_library_is_built_for_sm_103a_only(lib):
+    # the build command pins one -gencode; this checks the recorded command line
+    assert build.GENCODE == "arch=compute_103a,code=sm_103a"
+
+
+def test_defaults_and_strings(lib):
+    g = A.default_gate_params()
+    assert (g.gamma, g.beta, g.mode, g.divergence, g.fuse_bonus, g.flags) == (0.5, 1.0, 0, 0, 0, 0)
+    assert g.lambda_ == pytest.approx(0.1)
+    assert A.status_string(A.OK) == "ok"
+    assert "workspace" in A.status_string(A.ERR_WORKSPACE)
+    assert A.version() == 100
+
+
+def test_workspace_size():
+    assert A.workspace_bytes(64, 7, 128256) >= 64 * 8 * 16 + 64 * 4
+    assert A.workspace_bytes(0, 7, 10) == 0
+    assert A.workspace_bytes(3, 2, 10) == A.workspace_bytes(3, 2, 10**6)
+
+
+FAKE = 0x10000  # never dereferenced: every call below fails validation first
+
+
+def call(B=2, K=2, V=64, dtype=A.FP32, gate=None, ws=FAKE, ws_bytes=1 << 20, **ptrs):
+    p = dict(a=FAKE, b=FAKE, t=FAKE, tok=FAKE, prob=FAKE, unif=FAKE, L=FAKE, N=FAKE)
+    p.update(ptrs)
+    return A.fuse_verify_ex(p["a"], p["b"], p["t"], p["tok"], p["prob"], p["unif"], B, K, V,
+                            dtype, gate, p["L"], p["N"], ws, ws_bytes)
+
+
+def test_host_validation_codes(lib):
+    assert call(B=0) == A.ERR_INVALID_ARG
+    assert call(K=0) == A.ERR_INVALID_ARG
+    assert call(V=1) == A.ERR_INVALID_ARG
+    assert call(dtype=7) == A.ERR_UNSUPPORTED
+    assert call(gate=A.gate_params(gamma=0.0)) == A.ERR_INVALID_ARG
+    assert call(gate=A.gate_params(gamma=1.5)) == A.ERR_INVALID_ARG
+    assert call(gate=A.gate_params(beta=-1.0)) == A.ERR_INVALID_ARG
+    assert call(gate=A.gate_params(beta=float("nan"))) == A.ERR_INVALID_ARG
+    assert call(gate=A.gate_params(mode=5)) == A.ERR_UNSUPPORTED
+    assert call(gate=A.gate_params(divergence=9)) == A.ERR_UNSUPPORTED
+    assert call(a=0) == A.ERR_INVALID_ARG
+    assert call(L=0) == A.ERR_INVALID_ARG
+    assert call(gate=A.gate_params(mode=A.MODE_STOCHASTIC), prob=0) == A.ERR_INVALID_ARG
+    assert call(a=FAKE + 2) == A.ERR_MISALIGNED
+    assert call(dtype=A.BF16, a=FAKE + 1) == A.ERR_MISALIGNED
+    assert call(tok=FAKE + 2) == A.ERR_MISALIGNED
+    assert call(ws=0) == A.ERR_WORKSPACE
+    assert call(ws_bytes=A.workspace_bytes(2, 2, 64) - 1) == A.ERR_WORKSPACE
+    g = A.GateParams(0.5, 1.0, 0.1, 0, 0, 0, 3)
+    assert call(gate=g) == A.ERR_INVALID_ARG          # reserved flags must be 0
+    opts = A.LaunchOpts(3, 0)
+    st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
+                          FAKE, FAKE, 1 << 20, opts=opts)
+    assert st == A.ERR_INVALID_ARG                       # cluster size must be a power of 2
+
+
+def test_plan_picks_clusters_that_fit_on_chip(lib):
+    info = A.plan(64, 7, 128256, A.BF16)
+    assert info.cluster_size == 8 and info.slice_elems == 16032 and info.vector_path == 1
+    assert info.ctas == 64 * 8 * 8 and info.smem_bytes <= 227 * 1024
+    info = A.plan(8, 5, 151936, A.BF16)
+    assert info.cluster_size == 16
+    info = A.plan(256, 4, 151936, A.FP32)
+    assert info.cluster_size == 16 and info.smem_bytes <= 227 * 1024
+    info = A.plan(1, 4, 32000, A.FP32)
+    assert info.cluster_size == 4
+    info = A.plan(2, 2, 4099, A.BF16)
+    assert info.vector_path == 0
+    with pytest.raises(A.AsymSpecError):
+        A.plan(1, 1, 2_000_000, A.FP32)
+    info = A.plan(2, 2, 100, A.FP32, opts=A.LaunchOpts(16, 0))
+    assert info.cluster_size == 16
+
+
+def test_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):
+    monkeypatch.setattr(A, "_lib", None)
+    monkeypatch.setattr(A, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError):
+        A.workspace_bytes(1, 1, 2)

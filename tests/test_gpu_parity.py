@@ -1,0 +1,265 @@
+"""GPU path (through the C ABI) against the float64 oracle on the same inputs."""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2608_26004_gb300 import asymspec as A
+from paper_2608_26004_gb300 import synth
+from tests._parity import compare, device_inputs, run_gpu, run_oracle
+
+pytestmark = pytest.mark.gpu
+
+GREEDY, STOCH = A.MODE_GREEDY, A.MODE_STOCHASTIC
+
+
+@pytest.fixture(scope="module")
+def torch():
+    import torch as _torch
+    assert _torch.cuda.is_available(), "the gpu tests need a CUDA device"
+    from paper_2608_26004_gb300 import build
+    build.build_cuda()
+    A.lib()
+    return _torch
+
+
+def small(B, K, V, dtype, seed, **kw):
+    rc = synth.Recipe(**kw) if kw else synth.Recipe()
+    return synth.generate(rc, seed, B, K, V, dtype)
+
+
+# ---------------------------------------------------------------- element by element
+
+SMALL = [
+    # B, K, V, dtype          (vector path iff V * element size % 16 == 0)
+    (3, 3, 1000, synth.FP32),     # 250 float4 per row, several CTAs per cluster
+    (2, 2, 4099, synth.BF16),     # odd V: scalar path, ragged tail
+    (4, 1, 8200, synth.BF16),     # 1025 uint4 per row
+    (2, 4, 33333, synth.FP32),    # scalar path, multi-CTA clusters
+    (5, 2, 2, synth.FP32),        # smallest vocabulary
+    (2, 2, 8, synth.BF16),        # one 16-byte vector per row
+]
+
+
+@pytest.mark.parametrize("B,K,V,dtype", SMALL)
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+def test_small_shapes_all_outputs(torch, B, K, V, dtype, mode):
+    batch = small(B, K, V, dtype, seed=1000 + V + K)
+    g = run_gpu(batch, torch, mode=mode)
+    o = run_oracle(batch, mode=mode)
+    compare(batch, g, o, mode=mode)
+
+
+@pytest.mark.parametrize("cluster", [1, 2, 4, 8, 16])
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+def test_forced_cluster_sizes(torch, cluster, mode):
+    for B, K, V, dtype in [(3, 2, 5000, synth.BF16), (2, 2, 777, synth.FP32), (2, 1, 16, synth.BF16)]:
+        batch = small(B, K, V, dtype, seed=77 + cluster + V)
+        g = run_gpu(batch, torch, mode=mode, cluster_size=cluster)
+        o = run_oracle(batch, mode=mode)
+        compare(batch, g, o, mode=mode)
+
+
+@pytest.mark.parametrize("div", [A.DIV_JSD, A.DIV_NONE, A.DIV_KL, A.DIV_LAMBDA])
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+def test_gate_variants(torch, div, mode):
+    batch = small(4, 3, 6000, synth.BF16, seed=300 + div, sigma_c=2.0, frac_lo=0.1, frac_hi=0.3)
+    g = run_gpu(batch, torch, mode=mode, divergence=div, lam=0.1)
+    o = run_oracle(batch, mode=mode, divergence=div, lam=0.1)
+    compare(batch, g, o, mode=mode)
+
+
+@pytest.mark.parametrize("gamma,beta,fuse_bonus", [(1.0, 0.0, False), (0.3, 2.0, True),
+                                                   (0.7, 0.5, False), (1.0, 1.0, True)])
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+def test_hyperparameters(torch, gamma, beta, fuse_bonus, mode):
+    batch = small(4, 3, 3000, synth.FP32, seed=int(gamma * 10 + beta * 100))
+    kw = dict(mode=mode, gamma=gamma, beta=beta, fuse_bonus=fuse_bonus)
+    g = run_gpu(batch, torch, **kw)
+    o = run_oracle(batch, **kw)
+    compare(batch, g, o, mode=mode)
+
+
+# ---------------------------------------------------------------- the five workloads
+
+@pytest.mark.parametrize("cfg", [0, 1])
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+def test_small_workloads_whole(torch, cfg, mode):
+    batch = synth.make_config(cfg)
+    g = run_gpu(batch, torch, mode=mode)
+    o = run_oracle(batch, mode=mode)
+    compare(batch, g, o, mode=mode)
+
+
+def _bench_call(batch, torch, x, mode):
+    """The call bench.py times: no debug outputs, automatic launch."""
+    fv = A.FuseVerify(batch.B, batch.K)
+    res = fv(x["a"], x["b"], x["t"], x["tokens"], x["probs"], x["unif"], mode=mode)
+    torch.cuda.synchronize()
+    return res["accept_len"].cpu().numpy(), res["next_token"].cpu().numpy()
+
+
+@pytest.mark.parametrize("cfg", [2, 3])
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+def test_large_workloads_sampled(torch, cfg, mode):
+    batch = synth.make_config(cfg)
+    x = device_inputs(batch, torch)
+    L, N = _bench_call(batch, torch, x, mode)
+    rng = np.random.default_rng(cfg * 10 + mode)
+    sel = np.sort(rng.choice(batch.B, size=8, replace=False))
+    if cfg == 3:  # both halves: z_c == z_f and high divergence
+        sel = np.unique(np.concatenate([sel, [0, batch.B // 2 - 1, batch.B // 2, batch.B - 1]]))
+    o = run_oracle(batch, mode=mode, select=sel, logprobs=True)
+    ok = ~o.flagged
+    assert np.array_equal(L[sel][ok], o.accept_len[ok])
+    assert np.array_equal(N[sel][ok], o.next_token[ok])
+    g = run_gpu(batch, torch, mode=mode, inputs=x)
+    assert np.array_equal(g["accept_len"], L) and np.array_equal(g["next_token"], N)
+    compare(batch, g, o, mode=mode, select=sel)
+
+
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+def test_divergence_sweep_gate_response(torch, mode):
+    rows = []
+    for si, s in enumerate(synth.CONFIGS[4].sweep):
+        batch = synth.make_config(4, sweep_index=si)
+        g = run_gpu(batch, torch, mode=mode, logprobs=False)
+        o = run_oracle(batch, mode=mode, logprobs=False)
+        compare(batch, g, o, mode=mode, logprobs=False)
+        hist_g = np.bincount(g["accept_len"], minlength=batch.K + 1)
+        hist_o = np.bincount(o.accept_len, minlength=batch.K + 1)
+        nflag = int(o.flagged.sum())
+        assert np.abs(hist_g - hist_o).sum() <= 2 * nflag
+        rows.append((s, float(np.mean(g["row_stats"][..., 4])),
+                     float(np.mean(g["row_stats"][..., 5]))))
+    if mode == GREEDY:
+        # the gate relaxes as the compressed context diverges: mean D rises,
+        # mean gamma_eff falls, from D = 0 at s = 0 (z_c == z_f)
+        Ds = [r[1] for r in rows]
+        gs = [r[2] for r in rows]
+        assert Ds[0] == pytest.approx(0.0, abs=1e-5)
+        assert all(np.diff(Ds) > 0) and all(np.diff(gs) < 0)
+
+
+# ---------------------------------------------------------------- edge cases
+
+def test_data_errors_never_trap(torch):
+    batch = small(6, 2, 1000, synth.FP32, seed=5)
+    batch.logits_full[1, 0, 17] = np.nan
+    batch.logits_ver[2, 2, 999] = np.inf
+    batch.draft_tokens[3, 1] = 1000
+    batch.draft_tokens[4, 0] = -3
+    for mode in (GREEDY, STOCH):
+        g = run_gpu(batch, torch, mode=mode)
+        o = run_oracle(batch, mode=mode)
+        compare(batch, g, o, mode=mode, check_stats=False, logprobs=False)
+        assert list(g["accept_len"][1:5]) == [-1] * 4 and list(g["next_token"][1:5]) == [-1] * 4
+        assert g["accept_len"][0] >= 0 and g["accept_len"][5] >= 0
+        word = int(g["error_word"][0])
+        assert word & A.DATA_NONFINITE and word & A.DATA_BAD_TOKEN
+    batch = small(3, 2, 1000, synth.FP32, seed=6)
+    batch.draft_probs[0, 1] = 0.0
+    batch.uniforms[1, 2] = 1.0
+    g = run_gpu(batch, torch, mode=STOCH)
+    assert list(g["accept_len"]) [:2] == [-1, -1] and g["accept_len"][2] >= 0
+    word = int(g["error_word"][0])
+    assert word & A.DATA_BAD_PROB and word & A.DATA_BAD_UNIFORM
+
+
+def test_exact_ties_resolve_to_lowest_index(torch):
+    B, K, V = 2, 2, 4096
+    a = np.zeros((B, K + 1, V), np.float32)
+    b = np.zeros_like(a)
+    t = np.zeros_like(a)
+    t[..., [100, 3000, 4095]] = 5.0      # three-way tie in t and in s
+    t[1, :, [5, 4000]] = 7.0
+    batch = synth.Batch(a, b, t, np.full((B, K), 7, np.int32), np.full((B, K), 0.5, np.float32),
+                        np.full((B, K + 1), 0.5, np.float32), B, K, V, synth.FP32)
+    for cluster in (0, 1, 4, 16):
+        g = run_gpu(batch, torch, mode=GREEDY, cluster_size=cluster, gamma=1.0)
+        assert list(g["row_tokens"][0, :, 0]) == [100] * (K + 1)
+        assert list(g["row_tokens"][1, :, 0]) == [5] * (K + 1)
+
+
+def test_identical_contexts_give_zero_divergence(torch):
+    batch = synth.make_config(3, b0=120, nb=4)          # b < 128: z_c == z_f
+    g = run_gpu(batch, torch, mode=GREEDY)
+    assert np.all(np.abs(g["row_stats"][:2, :, 4]) <= 1e-5)
+    assert np.all(np.abs(g["row_stats"][:2, :, 5] - 0.5) <= 1e-5)
+
+
+def test_misaligned_rows_take_the_scalar_path(torch):
+    batch = small(2, 2, 2048, synth.BF16, seed=9)
+    x = device_inputs(batch, torch)
+    for key in ("a", "b", "t"):
+        buf = torch.empty(x[key].numel() + 1, dtype=x[key].dtype, device="cuda")
+        buf[1:].copy_(x[key].reshape(-1))
+        x[key] = buf[1:].view(x[key].shape)          # 2-byte aligned, not 16
+    assert x["a"].data_ptr() % 16 != 0
+    g = run_gpu(batch, torch, mode=STOCH, inputs=x)
+    o = run_oracle(batch, mode=STOCH)
+    compare(batch, g, o, mode=STOCH)
+
+
+def test_workspace_reuse_and_allocating_entry_point(torch):
+    batch = synth.make_config(1)
+    x = device_inputs(batch, torch)
+    fv = A.FuseVerify(batch.B, batch.K)
+    outs = []
+    for _ in range(3):
+        r = fv(x["a"], x["b"], x["t"], x["tokens"], x["probs"], x["unif"], mode=STOCH)
+        outs.append((r["accept_len"].clone(), r["next_token"].clone()))
+    torch.cuda.synchronize()
+    for L, N in outs[1:]:
+        assert torch.equal(L, outs[0][0]) and torch.equal(N, outs[0][1])
+    L2 = torch.empty_like(outs[0][0])
+    N2 = torch.empty_like(outs[0][1])
+    st = A.fuse_verify(x["a"].data_ptr(), x["b"].data_ptr(), x["t"].data_ptr(),
+                       x["tokens"].data_ptr(), x["probs"].data_ptr(), x["unif"].data_ptr(),
+                       batch.B, batch.K, batch.V, batch.dtype,
+                       A.gate_params(mode=STOCH), L2.data_ptr(), N2.data_ptr(),
+                       torch.cuda.current_stream().cuda_stream)
+    assert st == A.OK
+    torch.cuda.synchronize()
+    assert torch.equal(L2, outs[0][0]) and torch.equal(N2, outs[0][1])
+
+
+def test_plan_reports_cluster_occupancy(torch):
+    info = A.plan(64, 7, 128256, A.BF16)
+    assert info.cluster_size in (8, 16) and info.vector_path == 1
+    assert info.max_active_clusters > 0
+    assert info.smem_bytes <= 227 * 1024
+
+
+# ---------------------------------------------------------------- sampling law
+
+def test_emitted_token_law_chi_square(torch):
+    from scipy.stats import chisquare
+    V, K, N = 6, 1, 1_000_000
+    rng = np.random.default_rng(42)
+    a1 = rng.normal(0, 1, (K + 1, V)).astype(np.float32)
+    b1 = (a1 + rng.normal(0, 1, (K + 1, V))).astype(np.float32)
+    t1 = rng.normal(0, 1, (K + 1, V)).astype(np.float32)
+    rows = [O.row_quantities(a1[k].astype(np.float64), b1[k].astype(np.float64),
+                             t1[k].astype(np.float64), 0.5, 1.0, O.DIV_JSD) for k in range(K + 1)]
+    p = np.exp(rows[0].la)
+    d = np.minimum(np.searchsorted(np.cumsum(p), rng.uniform(0, 1, N), side="right"), V - 1)
+    probs = p[d].astype(np.float32)
+    unif = (rng.integers(0, 1 << 24, (N, K + 1)) / float(1 << 24)).astype(np.float32)
+    batch = synth.Batch(np.broadcast_to(a1, (N, K + 1, V)), np.broadcast_to(b1, (N, K + 1, V)),
+                        np.broadcast_to(t1, (N, K + 1, V)), d[:, None].astype(np.int32),
+                        probs[:, None], unif, N, K, V, synth.FP32)
+    g = run_gpu(batch, torch, mode=STOCH, logprobs=False)
+    L, nxt = g["accept_len"], g["next_token"]
+    first = np.where(L >= 1, d, nxt)
+    # exact law of the first emitted token (see the oracle pins)
+    q = np.exp(rows[0].lq)
+    A_ = np.minimum(1.0, q / (rows[0].gamma_eff * p))
+    resid = np.maximum(q - p, 0.0)
+    law = p * A_ + (1.0 - np.sum(p * A_)) * resid / resid.sum()
+    assert chisquare(np.bincount(first, minlength=V), law * N).pvalue > 1e-3
+    # and draw for draw against the oracle on the same uniforms
+    oL, oN, oflag, _, _ = O.stochastic_scan(rows, d[:, None], probs[:, None].astype(np.float64),
+                                            unif.astype(np.float64), K)
+    ok = ~oflag
+    assert ok.mean() > 0.99
+    assert np.array_equal(L[ok], oL[ok]) and np.array_equal(nxt[ok], oN[ok])
