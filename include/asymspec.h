@@ -67,6 +67,8 @@ extern "C" {
 #define ASYMSPEC_DATA_NONFINITE 0x2u    /* a non-finite normaliser or divergence (NaN/inf logits) */
 #define ASYMSPEC_DATA_BAD_PROB 0x4u     /* stochastic: draft probability outside (0, 1] */
 #define ASYMSPEC_DATA_BAD_UNIFORM 0x8u  /* stochastic: uniform outside [0, 1) */
+#define ASYMSPEC_DATA_TIMEOUT 0x10u     /* a bulk copy into shared memory did not complete within
+                                           its time limit (the kernel gave up instead of hanging) */
 
 typedef enum { ASYMSPEC_FP32 = 0, ASYMSPEC_BF16 = 1 } asymspec_dtype_t;
 
@@ -95,9 +97,15 @@ typedef struct {
 
 /* Optional launch overrides (host struct); zero fields mean "automatic". */
 typedef struct {
-  int32_t cluster_size;   /* CTAs per row triple: 1, 2, 4, 8 or 16 */
+  int32_t cluster_size;   /* CTAs per row triple: 1 to 16 */
   int32_t block_threads;  /* reserved, must be 0 (256 threads per CTA) */
+  int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC; ASYMSPEC_KERNEL_TMA */
 } asymspec_launch_opts;
+
+/* Kernels (asymspec_launch_opts.kernel, asymspec_launch_info.kernel). */
+#define ASYMSPEC_KERNEL_GENERIC 1  /* one cluster per row; any element-aligned input */
+#define ASYMSPEC_KERNEL_TMA 2      /* one cluster per row, chunked 1-D bulk copies, per-row
+                                      programs; rows 16-byte aligned (the default when they are) */
 
 /* What a launch would use (filled by asymspec_plan). */
 typedef struct {
@@ -105,9 +113,10 @@ typedef struct {
   int32_t block_threads;   /* threads per CTA */
   int32_t slice_elems;     /* vocabulary entries held on chip per CTA */
   int32_t smem_bytes;      /* dynamic shared memory per CTA */
-  int64_t ctas;            /* CTAs in the grid = B (K+1) cluster_size */
+  int64_t ctas;            /* CTAs in the grid */
   int32_t vector_path;     /* 1 if rows qualify for 16-byte copies (V * element size % 16 == 0) */
   int32_t max_active_clusters; /* clusters the device can hold at once (0 if unknown) */
+  int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC or ASYMSPEC_KERNEL_TMA */
 } asymspec_launch_info;
 
 /* Fills *p with the paper's defaults: gamma 0.5, beta 1.0, lambda 0.1,

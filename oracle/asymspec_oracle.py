@@ -50,9 +50,10 @@ as such, so that a float32 implementation may legitimately differ there:
   boundary, or the residual mass itself below 1e-5.
 
 Inputs are required to be finite (the paper's setting); a batch element with a
-non-finite logit, a draft token outside [0, V), or (stochastic mode) a draft
-probability outside (0, 1] or a uniform outside [0, 1) is reported as a data
-error with accept_len = next_token = -1.
+non-finite logit in the data the step uses, a draft token outside [0, V), or
+(stochastic mode) a draft probability outside (0, 1] or a uniform outside
+[0, 1) is reported as a data error with accept_len = next_token = -1.  Greedy
+decoding without a fused bonus does not use a and b of the bonus row.
 """
 from __future__ import annotations
 
@@ -107,7 +108,8 @@ def jsd(la: np.ndarray, lb: np.ndarray) -> float:
     """
     p = np.exp(la)
     q = np.exp(lb)
-    lm = np.logaddexp(la, lb) - LN2
+    with np.errstate(invalid="ignore"):
+        lm = np.logaddexp(la, lb) - LN2
     tp = np.where(p > 0.0, p * (la - lm), 0.0)
     tq = np.where(q > 0.0, q * (lb - lm), 0.0)
     return float(0.5 * np.sum(tp + tq))
@@ -353,7 +355,10 @@ def fuse_verify(logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=
         a_all = widen(logits_full[bi], dtype)
         b_all = widen(logits_comp[bi], dtype)
         t_all = widen(logits_ver[bi], dtype)
-        ok = bool(np.all(np.isfinite(a_all)) and np.all(np.isfinite(b_all))
+        # greedy decoding without a fused bonus never uses a and b of the bonus
+        # row (Algorithm 1 emits argmax(t_{K+1})), so only used data is checked
+        ab_rows = K if (mode == GREEDY and not fuse_bonus) else K1
+        ok = bool(np.all(np.isfinite(a_all[:ab_rows])) and np.all(np.isfinite(b_all[:ab_rows]))
                   and np.all(np.isfinite(t_all)))
         ok = ok and bool(np.all((tokens[bi] >= 0) & (tokens[bi] < V)))
         if mode == STOCHASTIC:
@@ -370,9 +375,12 @@ def fuse_verify(logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=
             res.lse[bi, k] = (r.lse_a, r.lse_b, r.lse_t, r.lse_s)
             res.D[bi, k] = r.D
             res.gamma_eff[bi, k] = r.gamma_eff
-            res.fused_argmax[bi, k] = argmax_first(r.s)
-            res.fused_gap_flag[bi, k] = (top2_gap(r.s)
-                                         < ARGMAX_BAND * max(1.0, abs(float(np.max(r.s)))))
+            if np.all(np.isfinite(r.s)):
+                res.fused_argmax[bi, k] = argmax_first(r.s)
+                res.fused_gap_flag[bi, k] = (top2_gap(r.s)
+                                             < ARGMAX_BAND * max(1.0, abs(float(np.max(r.s)))))
+            else:  # only in rows the step does not use: undefined, not compared
+                res.fused_gap_flag[bi, k] = True
             if want_logprobs:
                 res.logprobs[bi, k] = r.lq
         if mode == GREEDY:

@@ -28,6 +28,7 @@ DATA_BAD_TOKEN = 0x1
 DATA_NONFINITE = 0x2
 DATA_BAD_PROB = 0x4
 DATA_BAD_UNIFORM = 0x8
+DATA_TIMEOUT = 0x10
 
 FP32 = 0
 BF16 = 1
@@ -59,15 +60,21 @@ class GateParams(ctypes.Structure):
                 ("flags", ctypes.c_int32)]
 
 
+KERNEL_AUTO = 0
+KERNEL_GENERIC = 1
+KERNEL_TMA = 2
+
+
 class LaunchOpts(ctypes.Structure):
-    _fields_ = [("cluster_size", ctypes.c_int32), ("block_threads", ctypes.c_int32)]
+    _fields_ = [("cluster_size", ctypes.c_int32), ("block_threads", ctypes.c_int32),
+                ("kernel", ctypes.c_int32)]
 
 
 class LaunchInfo(ctypes.Structure):
     _fields_ = [("cluster_size", ctypes.c_int32), ("block_threads", ctypes.c_int32),
                 ("slice_elems", ctypes.c_int32), ("smem_bytes", ctypes.c_int32),
                 ("ctas", ctypes.c_int64), ("vector_path", ctypes.c_int32),
-                ("max_active_clusters", ctypes.c_int32)]
+                ("max_active_clusters", ctypes.c_int32), ("kernel", ctypes.c_int32)]
 
 
 class AsymSpecError(RuntimeError):
@@ -207,7 +214,7 @@ class FuseVerify:
     def __call__(self, logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=None,
                  uniforms=None, *, gamma=0.5, beta=1.0, lam=0.1, mode=MODE_GREEDY,
                  divergence=DIV_JSD, fuse_bonus=False, row_stats=False, row_tokens=False,
-                 fused_logprobs=False, cluster_size=0, out=None):
+                 fused_logprobs=False, cluster_size=0, kernel=KERNEL_AUTO, out=None):
         import torch
         B, K1, V = logits_full.shape
         K = K1 - 1
@@ -236,7 +243,7 @@ class FuseVerify:
         if fused_logprobs and "fused_logprobs" not in res:
             res["fused_logprobs"] = torch.empty(B, K1, V, dtype=torch.float32, device=dev)
         gate = gate_params(gamma, beta, lam, mode, divergence, fuse_bonus)
-        opts = LaunchOpts(cluster_size, 0) if cluster_size else None
+        opts = LaunchOpts(cluster_size, 0, kernel) if (cluster_size or kernel) else None
         stream = torch.cuda.current_stream(dev).cuda_stream
         st = fuse_verify_ex(
             _ptr(logits_full), _ptr(logits_comp), _ptr(logits_ver), _ptr(draft_tokens),

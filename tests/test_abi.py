@@ -49,7 +49,7 @@ def test_defaults_and_strings(lib):
     assert g.lambda_ == pytest.approx(0.1)
     assert A.status_string(A.OK) == "ok"
     assert "workspace" in A.status_string(A.ERR_WORKSPACE)
-    assert A.version() == 100
+    assert A.version() == 200
 
 
 def test_workspace_size():
@@ -89,28 +89,43 @@ def test_host_validation_codes(lib):
     assert call(ws_bytes=A.workspace_bytes(2, 2, 64) - 1) == A.ERR_WORKSPACE
     g = A.GateParams(0.5, 1.0, 0.1, 0, 0, 0, 3)
     assert call(gate=g) == A.ERR_INVALID_ARG          # reserved flags must be 0
-    opts = A.LaunchOpts(3, 0)
+    opts = A.LaunchOpts(17, 0, 0)
     st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
                           FAKE, FAKE, 1 << 20, opts=opts)
-    assert st == A.ERR_INVALID_ARG                       # cluster size must be a power of 2
+    assert st == A.ERR_INVALID_ARG                       # at most 16 CTAs per cluster
+    st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
+                          FAKE, FAKE, 1 << 20, opts=A.LaunchOpts(0, 0, 7))
+    assert st == A.ERR_INVALID_ARG                       # unknown kernel
 
 
-def test_plan_picks_clusters_that_fit_on_chip(lib):
+def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
+    # the bench workload: TMA kernel, 8 CTAs of 96 KB per row, two CTAs per SM
     info = A.plan(64, 7, 128256, A.BF16)
-    assert info.cluster_size == 8 and info.slice_elems == 16032 and info.vector_path == 1
-    assert info.ctas == 64 * 8 * 8 and info.smem_bytes <= 227 * 1024
+    assert info.kernel == A.KERNEL_TMA and info.cluster_size == 8
+    assert info.slice_elems == 16032 and info.vector_path == 1
+    assert info.ctas == 64 * 8 * 8 and info.smem_bytes <= 113 * 1024
+    # Qwen3-sized bf16 rows: 8 CTAs of 112.7 KB, still two per SM
     info = A.plan(8, 5, 151936, A.BF16)
-    assert info.cluster_size == 16
+    assert info.kernel == A.KERNEL_TMA and info.cluster_size == 8
+    assert info.smem_bytes <= 113 * 1024
+    # fp32 rows of 151,936 entries: 16 CTAs of 114 KB
     info = A.plan(256, 4, 151936, A.FP32)
-    assert info.cluster_size == 16 and info.smem_bytes <= 227 * 1024
+    assert info.kernel == A.KERNEL_TMA and info.cluster_size == 16
+    assert info.smem_bytes <= 227 * 1024
     info = A.plan(1, 4, 32000, A.FP32)
-    assert info.cluster_size == 4
+    assert info.kernel == A.KERNEL_TMA and info.cluster_size == 4
     info = A.plan(2, 2, 4099, A.BF16)
-    assert info.vector_path == 0
+    assert info.vector_path == 0 and info.kernel == A.KERNEL_GENERIC
     with pytest.raises(A.AsymSpecError):
         A.plan(1, 1, 2_000_000, A.FP32)
-    info = A.plan(2, 2, 100, A.FP32, opts=A.LaunchOpts(16, 0))
+    info = A.plan(2, 2, 100, A.FP32, opts=A.LaunchOpts(16, 0, 0))
     assert info.cluster_size == 16
+    info = A.plan(2, 2, 100, A.FP32, opts=A.LaunchOpts(3, 0, 0))
+    assert info.cluster_size == 3
+    info = A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(0, 0, A.KERNEL_GENERIC))
+    assert info.kernel == A.KERNEL_GENERIC and info.cluster_size == 8
+    with pytest.raises(A.AsymSpecError):      # unaligned rows cannot use bulk copies
+        A.plan(2, 2, 4099, A.BF16, opts=A.LaunchOpts(0, 0, A.KERNEL_TMA))
 
 
 def test_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):

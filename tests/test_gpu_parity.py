@@ -1,4 +1,11 @@
-"""GPU path (through the C ABI) against the float64 oracle on the same inputs."""
+"""GPU path (through the C ABI) against the float64 oracle on the same inputs.
+
+Every case runs on the kernel the library picks (the TMA kernel for 16-byte
+aligned rows) and, where it applies, on the generic kernel; and both
+with the production program (accept/next plus row tokens, the work the
+benchmark times) and with every debug output (row statistics, fused
+log-probs), which runs the full per-row program.
+"""
 import numpy as np
 import pytest
 
@@ -10,6 +17,9 @@ from tests._parity import compare, device_inputs, run_gpu, run_oracle
 pytestmark = pytest.mark.gpu
 
 GREEDY, STOCH = A.MODE_GREEDY, A.MODE_STOCHASTIC
+AUTO, GENERIC, TMA = A.KERNEL_AUTO, A.KERNEL_GENERIC, A.KERNEL_TMA
+PATHS = [(AUTO, False), (AUTO, True), (GENERIC, True)]
+PATH_IDS = ["auto-prod", "auto-full", "generic-full"]
 
 
 @pytest.fixture(scope="module")
@@ -27,67 +37,72 @@ def small(B, K, V, dtype, seed, **kw):
     return synth.generate(rc, seed, B, K, V, dtype)
 
 
+def check(batch, torch, mode, kernel, full, **kw):
+    g = run_gpu(batch, torch, mode=mode, kernel=kernel, full=full, **kw)
+    okw = {k: v for k, v in kw.items() if k in ("divergence", "gamma", "beta", "lam", "fuse_bonus")}
+    o = run_oracle(batch, mode=mode, **okw)
+    compare(batch, g, o, mode=mode)
+    return g, o
+
+
 # ---------------------------------------------------------------- element by element
 
 SMALL = [
-    # B, K, V, dtype          (vector path iff V * element size % 16 == 0)
-    (3, 3, 1000, synth.FP32),     # 250 float4 per row, several CTAs per cluster
-    (2, 2, 4099, synth.BF16),     # odd V: scalar path, ragged tail
+    # B, K, V, dtype          (TMA kernel iff V * element size % 16 == 0)
+    (3, 3, 1000, synth.FP32),     # 250 float4 per row
+    (2, 2, 4099, synth.BF16),     # odd V: generic kernel, scalar path, ragged tail
     (4, 1, 8200, synth.BF16),     # 1025 uint4 per row
-    (2, 4, 33333, synth.FP32),    # scalar path, multi-CTA clusters
+    (2, 4, 33333, synth.FP32),    # generic kernel, scalar path, multi-CTA clusters
     (5, 2, 2, synth.FP32),        # smallest vocabulary
     (2, 2, 8, synth.BF16),        # one 16-byte vector per row
+    (3, 2, 40000, synth.BF16),    # several rounds and bulk-copy chunks per CTA
 ]
 
 
+@pytest.mark.parametrize("kernel,full", PATHS, ids=PATH_IDS)
 @pytest.mark.parametrize("B,K,V,dtype", SMALL)
 @pytest.mark.parametrize("mode", [GREEDY, STOCH])
-def test_small_shapes_all_outputs(torch, B, K, V, dtype, mode):
+def test_small_shapes(torch, B, K, V, dtype, mode, kernel, full):
     batch = small(B, K, V, dtype, seed=1000 + V + K)
-    g = run_gpu(batch, torch, mode=mode)
-    o = run_oracle(batch, mode=mode)
-    compare(batch, g, o, mode=mode)
+    check(batch, torch, mode, kernel, full)
 
 
-@pytest.mark.parametrize("cluster", [1, 2, 4, 8, 16])
+@pytest.mark.parametrize("kernel", [GENERIC, TMA])
+@pytest.mark.parametrize("cluster", [1, 2, 3, 4, 8, 16])
 @pytest.mark.parametrize("mode", [GREEDY, STOCH])
-def test_forced_cluster_sizes(torch, cluster, mode):
-    for B, K, V, dtype in [(3, 2, 5000, synth.BF16), (2, 2, 777, synth.FP32), (2, 1, 16, synth.BF16)]:
+def test_forced_cluster_sizes(torch, cluster, mode, kernel):
+    for B, K, V, dtype in [(3, 2, 5000, synth.BF16), (2, 2, 780, synth.FP32),
+                           (2, 1, 16, synth.BF16)]:
         batch = small(B, K, V, dtype, seed=77 + cluster + V)
-        g = run_gpu(batch, torch, mode=mode, cluster_size=cluster)
-        o = run_oracle(batch, mode=mode)
-        compare(batch, g, o, mode=mode)
+        for full in (False, True):
+            check(batch, torch, mode, kernel, full, cluster_size=cluster)
 
 
+@pytest.mark.parametrize("kernel,full", PATHS, ids=PATH_IDS)
 @pytest.mark.parametrize("div", [A.DIV_JSD, A.DIV_NONE, A.DIV_KL, A.DIV_LAMBDA])
 @pytest.mark.parametrize("mode", [GREEDY, STOCH])
-def test_gate_variants(torch, div, mode):
+def test_gate_variants(torch, div, mode, kernel, full):
     batch = small(4, 3, 6000, synth.BF16, seed=300 + div, sigma_c=2.0, frac_lo=0.1, frac_hi=0.3)
-    g = run_gpu(batch, torch, mode=mode, divergence=div, lam=0.1)
-    o = run_oracle(batch, mode=mode, divergence=div, lam=0.1)
-    compare(batch, g, o, mode=mode)
+    check(batch, torch, mode, kernel, full, divergence=div, lam=0.1)
 
 
+@pytest.mark.parametrize("kernel,full", PATHS, ids=PATH_IDS)
 @pytest.mark.parametrize("gamma,beta,fuse_bonus", [(1.0, 0.0, False), (0.3, 2.0, True),
                                                    (0.7, 0.5, False), (1.0, 1.0, True)])
 @pytest.mark.parametrize("mode", [GREEDY, STOCH])
-def test_hyperparameters(torch, gamma, beta, fuse_bonus, mode):
+def test_hyperparameters(torch, gamma, beta, fuse_bonus, mode, kernel, full):
     batch = small(4, 3, 3000, synth.FP32, seed=int(gamma * 10 + beta * 100))
-    kw = dict(mode=mode, gamma=gamma, beta=beta, fuse_bonus=fuse_bonus)
-    g = run_gpu(batch, torch, **kw)
-    o = run_oracle(batch, **kw)
-    compare(batch, g, o, mode=mode)
+    check(batch, torch, mode, kernel, full, gamma=gamma, beta=beta, fuse_bonus=fuse_bonus)
 
 
 # ---------------------------------------------------------------- the five workloads
 
+@pytest.mark.parametrize("kernel,full", PATHS, ids=PATH_IDS)
 @pytest.mark.parametrize("cfg", [0, 1])
 @pytest.mark.parametrize("mode", [GREEDY, STOCH])
-def test_small_workloads_whole(torch, cfg, mode):
+def test_small_workloads_whole(torch, cfg, mode, kernel, full):
     batch = synth.make_config(cfg)
-    g = run_gpu(batch, torch, mode=mode)
-    o = run_oracle(batch, mode=mode)
-    compare(batch, g, o, mode=mode)
+    check(batch, torch, mode, kernel, full)
 
 
 def _bench_call(batch, torch, x, mode):
@@ -112,9 +127,10 @@ def test_large_workloads_sampled(torch, cfg, mode):
     ok = ~o.flagged
     assert np.array_equal(L[sel][ok], o.accept_len[ok])
     assert np.array_equal(N[sel][ok], o.next_token[ok])
-    g = run_gpu(batch, torch, mode=mode, inputs=x)
-    assert np.array_equal(g["accept_len"], L) and np.array_equal(g["next_token"], N)
-    compare(batch, g, o, mode=mode, select=sel)
+    for full in (False, True):
+        g = run_gpu(batch, torch, mode=mode, inputs=x, full=full)
+        assert np.array_equal(g["accept_len"], L) and np.array_equal(g["next_token"], N)
+        compare(batch, g, o, mode=mode, select=sel)
 
 
 @pytest.mark.parametrize("mode", [GREEDY, STOCH])
@@ -122,50 +138,56 @@ def test_divergence_sweep_gate_response(torch, mode):
     rows = []
     for si, s in enumerate(synth.CONFIGS[4].sweep):
         batch = synth.make_config(4, sweep_index=si)
-        g = run_gpu(batch, torch, mode=mode, logprobs=False)
         o = run_oracle(batch, mode=mode, logprobs=False)
+        gp = run_gpu(batch, torch, mode=mode, full=False)
+        compare(batch, gp, o, mode=mode, logprobs=False)
+        g = run_gpu(batch, torch, mode=mode, logprobs=False)
         compare(batch, g, o, mode=mode, logprobs=False)
-        hist_g = np.bincount(g["accept_len"], minlength=batch.K + 1)
+        hist_g = np.bincount(gp["accept_len"], minlength=batch.K + 1)
         hist_o = np.bincount(o.accept_len, minlength=batch.K + 1)
         nflag = int(o.flagged.sum())
         assert np.abs(hist_g - hist_o).sum() <= 2 * nflag
-        rows.append((s, float(np.mean(g["row_stats"][..., 4])),
-                     float(np.mean(g["row_stats"][..., 5]))))
-    if mode == GREEDY:
-        # the gate relaxes as the compressed context diverges: mean D rises,
-        # mean gamma_eff falls, from D = 0 at s = 0 (z_c == z_f)
-        Ds = [r[1] for r in rows]
-        gs = [r[2] for r in rows]
-        assert Ds[0] == pytest.approx(0.0, abs=1e-5)
-        assert all(np.diff(Ds) > 0) and all(np.diff(gs) < 0)
+        rows.append((s, float(np.mean(g["row_stats"][:, :batch.K, 4])),
+                     float(np.mean(g["row_stats"][:, :batch.K, 5]))))
+    # the gate relaxes as the compressed context diverges: mean D rises,
+    # mean gamma_eff falls, from D = 0 at s = 0 (z_c == z_f)
+    Ds = [r[1] for r in rows]
+    gs = [r[2] for r in rows]
+    assert Ds[0] == pytest.approx(0.0, abs=1e-5)
+    assert all(np.diff(Ds) > 0) and all(np.diff(gs) < 0)
 
 
 # ---------------------------------------------------------------- edge cases
 
-def test_data_errors_never_trap(torch):
-    batch = small(6, 2, 1000, synth.FP32, seed=5)
+@pytest.mark.parametrize("kernel,full", PATHS, ids=PATH_IDS)
+def test_data_errors_never_trap(torch, kernel, full):
+    batch = small(7, 2, 1000, synth.FP32, seed=5)
     batch.logits_full[1, 0, 17] = np.nan
     batch.logits_ver[2, 2, 999] = np.inf
     batch.draft_tokens[3, 1] = 1000
     batch.draft_tokens[4, 0] = -3
+    batch.logits_comp[6, 2, 5] = np.nan      # bonus row: unused by greedy decoding
     for mode in (GREEDY, STOCH):
-        g = run_gpu(batch, torch, mode=mode)
+        g = run_gpu(batch, torch, mode=mode, kernel=kernel, full=full)
         o = run_oracle(batch, mode=mode)
         compare(batch, g, o, mode=mode, check_stats=False, logprobs=False)
         assert list(g["accept_len"][1:5]) == [-1] * 4 and list(g["next_token"][1:5]) == [-1] * 4
         assert g["accept_len"][0] >= 0 and g["accept_len"][5] >= 0
+        assert (g["accept_len"][6] >= 0) == (mode == GREEDY)
         word = int(g["error_word"][0])
         assert word & A.DATA_NONFINITE and word & A.DATA_BAD_TOKEN
+        assert not word & A.DATA_TIMEOUT
     batch = small(3, 2, 1000, synth.FP32, seed=6)
     batch.draft_probs[0, 1] = 0.0
     batch.uniforms[1, 2] = 1.0
-    g = run_gpu(batch, torch, mode=STOCH)
-    assert list(g["accept_len"]) [:2] == [-1, -1] and g["accept_len"][2] >= 0
+    g = run_gpu(batch, torch, mode=STOCH, kernel=kernel, full=full)
+    assert list(g["accept_len"])[:2] == [-1, -1] and g["accept_len"][2] >= 0
     word = int(g["error_word"][0])
     assert word & A.DATA_BAD_PROB and word & A.DATA_BAD_UNIFORM
 
 
-def test_exact_ties_resolve_to_lowest_index(torch):
+@pytest.mark.parametrize("kernel", [GENERIC, TMA])
+def test_exact_ties_resolve_to_lowest_index(torch, kernel):
     B, K, V = 2, 2, 4096
     a = np.zeros((B, K + 1, V), np.float32)
     b = np.zeros_like(a)
@@ -175,9 +197,14 @@ def test_exact_ties_resolve_to_lowest_index(torch):
     batch = synth.Batch(a, b, t, np.full((B, K), 7, np.int32), np.full((B, K), 0.5, np.float32),
                         np.full((B, K + 1), 0.5, np.float32), B, K, V, synth.FP32)
     for cluster in (0, 1, 4, 16):
-        g = run_gpu(batch, torch, mode=GREEDY, cluster_size=cluster, gamma=1.0)
-        assert list(g["row_tokens"][0, :, 0]) == [100] * (K + 1)
-        assert list(g["row_tokens"][1, :, 0]) == [5] * (K + 1)
+        for full in (False, True):
+            g = run_gpu(batch, torch, mode=GREEDY, cluster_size=cluster, gamma=1.0,
+                        kernel=kernel, full=full, fuse_bonus=True)
+            assert list(g["row_tokens"][0, :, 0]) == [100] * (K + 1)
+            assert list(g["row_tokens"][1, :, 0]) == [5] * (K + 1)
+            g = run_gpu(batch, torch, mode=GREEDY, cluster_size=cluster, gamma=1.0,
+                        kernel=kernel, full=full)
+            assert g["row_tokens"][0, K, 1] == 100 and g["row_tokens"][1, K, 1] == 5
 
 
 def test_identical_contexts_give_zero_divergence(torch):
@@ -187,7 +214,7 @@ def test_identical_contexts_give_zero_divergence(torch):
     assert np.all(np.abs(g["row_stats"][:2, :, 5] - 0.5) <= 1e-5)
 
 
-def test_misaligned_rows_take_the_scalar_path(torch):
+def test_misaligned_rows_take_the_generic_kernel(torch):
     batch = small(2, 2, 2048, synth.BF16, seed=9)
     x = device_inputs(batch, torch)
     for key in ("a", "b", "t"):
@@ -195,9 +222,10 @@ def test_misaligned_rows_take_the_scalar_path(torch):
         buf[1:].copy_(x[key].reshape(-1))
         x[key] = buf[1:].view(x[key].shape)          # 2-byte aligned, not 16
     assert x["a"].data_ptr() % 16 != 0
-    g = run_gpu(batch, torch, mode=STOCH, inputs=x)
-    o = run_oracle(batch, mode=STOCH)
-    compare(batch, g, o, mode=STOCH)
+    for full in (False, True):
+        g = run_gpu(batch, torch, mode=STOCH, inputs=x, full=full)
+        o = run_oracle(batch, mode=STOCH)
+        compare(batch, g, o, mode=STOCH)
 
 
 def test_workspace_reuse_and_allocating_entry_point(torch):
@@ -225,16 +253,19 @@ def test_workspace_reuse_and_allocating_entry_point(torch):
 
 def test_plan_reports_cluster_occupancy(torch):
     info = A.plan(64, 7, 128256, A.BF16)
-    assert info.cluster_size in (8, 16) and info.vector_path == 1
-    assert info.max_active_clusters > 0
-    assert info.smem_bytes <= 227 * 1024
+    assert info.kernel == A.KERNEL_TMA and info.cluster_size == 8 and info.vector_path == 1
+    assert info.max_active_clusters >= 30          # 2 CTAs per SM, clusters of 8
+    assert info.smem_bytes <= 113 * 1024
+    info = A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(0, 0, A.KERNEL_GENERIC))
+    assert info.kernel == A.KERNEL_GENERIC and info.max_active_clusters > 0
 
 
 # ---------------------------------------------------------------- sampling law
 
-def test_emitted_token_law_chi_square(torch):
+@pytest.mark.parametrize("kernel", [GENERIC, TMA])
+def test_emitted_token_law_chi_square(torch, kernel):
     from scipy.stats import chisquare
-    V, K, N = 6, 1, 1_000_000
+    V, K, N = 8, 1, 1_000_000
     rng = np.random.default_rng(42)
     a1 = rng.normal(0, 1, (K + 1, V)).astype(np.float32)
     b1 = (a1 + rng.normal(0, 1, (K + 1, V))).astype(np.float32)
@@ -248,7 +279,7 @@ def test_emitted_token_law_chi_square(torch):
     batch = synth.Batch(np.broadcast_to(a1, (N, K + 1, V)), np.broadcast_to(b1, (N, K + 1, V)),
                         np.broadcast_to(t1, (N, K + 1, V)), d[:, None].astype(np.int32),
                         probs[:, None], unif, N, K, V, synth.FP32)
-    g = run_gpu(batch, torch, mode=STOCH, logprobs=False)
+    g = run_gpu(batch, torch, mode=STOCH, logprobs=False, kernel=kernel, full=False)
     L, nxt = g["accept_len"], g["next_token"]
     first = np.where(L >= 1, d, nxt)
     # exact law of the first emitted token (see the oracle pins)
