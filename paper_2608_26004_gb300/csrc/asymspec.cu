@@ -66,12 +66,13 @@ bool plan_generic(int V, int elt, int VE, int forced_C, Plan* pl) {
 // TMA kernel: first C whose slice (and shared state) fits two CTAs per SM,
 // else the first that fits one; a slice holds at most kMaxRounds vectors
 // per thread.
-bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
+bool plan_tma(int V, int elt, int forced_C, bool stoch, Plan* pl) {
   const int VE = 16 / elt;
   auto fill = [&](int C) {
-    const int shared_bytes = shared_tma_bytes(C);
     const long long per = (static_cast<long long>(V) + C - 1) / C;
     const long long W = round_up_ll(per, VE);
+    const int rounds = static_cast<int>((W / VE + kTThreads - 1) / kTThreads);
+    const int shared_bytes = shared_tma_bytes(C) + (stoch ? mass_bytes(rounds) : 0);
     const long long sh_off = round_up_ll(3 * W * elt, 128);
     pl->C = C;
     pl->W = static_cast<int>(W);
@@ -88,8 +89,8 @@ bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
   return false;
 }
 
-int make_plan(int B, int K, int V, int dtype, const asymspec_launch_opts* opts, bool vec_ok,
-              Plan* pl) {
+int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_opts* opts,
+              bool vec_ok, Plan* pl) {
   const int elt = elt_size(dtype);
   const int forced_C = (opts && opts->cluster_size > 0) ? opts->cluster_size : 0;
   const int forced_kernel = opts ? opts->kernel : 0;
@@ -100,7 +101,7 @@ int make_plan(int B, int K, int V, int dtype, const asymspec_launch_opts* opts, 
   pl->rows = static_cast<long long>(B) * (K + 1);
   pl->vector_path = vec_ok;
   bool ok = false;
-  if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, pl)) {
+  if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, stoch, pl)) {
     pl->kernel = ASYMSPEC_KERNEL_TMA;
     pl->VE = 16 / elt;
     ok = true;
@@ -272,7 +273,7 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
   if (st) return st;
   const bool vec_ok = (static_cast<long long>(V) * elt_size(dtype)) % 16 == 0;
   Plan pl;
-  st = make_plan(B, K, V, dtype, opts, vec_ok, &pl);
+  st = make_plan(B, K, V, dtype, gp.mode == ASYMSPEC_MODE_STOCHASTIC, opts, vec_ok, &pl);
   if (st) return st;
   out->cluster_size = pl.C;
   out->block_threads = pl.kernel == ASYMSPEC_KERNEL_TMA ? kTThreads : kThreads;
@@ -332,7 +333,7 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   const bool vec_ok = (static_cast<long long>(V) * elt) % 16 == 0 && aligned(logits_full, 16) &&
                       aligned(logits_comp, 16) && aligned(logits_ver, 16);
   Plan pl;
-  st = make_plan(B, K, V, dtype, opts, vec_ok, &pl);
+  st = make_plan(B, K, V, dtype, stoch, opts, vec_ok, &pl);
   if (st) return st;
 
   KParams P;

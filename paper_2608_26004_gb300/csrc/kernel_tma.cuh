@@ -96,9 +96,13 @@ static_assert(sizeof(X1) % 16 == 0 && alignof(X1) == 16, "X1 must be 16-byte ali
 static_assert(sizeof(X2) % 16 == 0 && alignof(X2) == 16, "X2 must be 16-byte aligned");
 static_assert(sizeof(SharedTma) % 16 == 0, "records after SharedTma must stay 16-byte aligned");
 
-// Shared bytes after the slices for a cluster of C CTAs.
+// Shared bytes after the slices for a cluster of C CTAs (the stochastic
+// kernel adds rounds * kTThreads floats of per-vector masses).
 __host__ __device__ constexpr int shared_tma_bytes(int C) {
   return static_cast<int>(sizeof(SharedTma) + C * (sizeof(X1) + sizeof(X2)));
+}
+__host__ __device__ constexpr int mass_bytes(int rounds) {
+  return rounds * kTThreads * static_cast<int>(sizeof(float));
 }
 
 __device__ __forceinline__ X1 x1_neutral() {
@@ -168,6 +172,16 @@ __device__ __forceinline__ void warp_reduce_x1(X1& e) {
   e.bad = __reduce_or_sync(0xffffffffu, e.bad);
 }
 
+// Cluster barrier.  Only the warp that pushed records needs release
+// ordering; the others arrive relaxed.  Everyone waits with acquire.
+__device__ __forceinline__ void cluster_barrier(bool released) {
+  if (released)
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  else
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 // The record of this CTA goes into slot `rank` of every CTA of the cluster
 // (lane r of warp 0 writes to CTA r); a cluster barrier must follow.
 template <typename R>
@@ -217,45 +231,30 @@ __device__ __forceinline__ float vmax_pairs_nan(const f2 (&x)[NP]) {
   return m;
 }
 
-// Running (max m, packed sum of 2^((x - m) log2 e)) over a vector of pairs;
-// returns the vector maximum.
-template <int NP>
-__device__ __forceinline__ float online_pairs(float& m, f2& acc, const f2 (&x)[NP], f2 L2) {
-  const float cm = vmax_pairs(x);
-  if (cm > m) {
-    const float f = ex2((m - cm) * kLog2e);
-    acc = mul2(acc, pk(f, f));
-    m = cm;
-  }
-  const float nm = -m * kLog2e;
-  const f2 nm2 = pk(nm, nm);
-  f2 e[NP];
-#pragma unroll
-  for (int h = 0; h < NP; ++h) e[h] = ex2_2(fma2(x[h], L2, nm2));
-  if constexpr (NP == 4) {
-    acc = add2(acc, add2(add2(e[0], e[1]), add2(e[2], e[3])));
-  } else {
-    acc = add2(acc, add2(e[0], e[1]));
-  }
-  return cm;
+// Argmax tracking per vector, branch-free: the best vector maximum so far
+// and the index of its vector (a strict improvement wins, so the earliest
+// vector keeps a tie); a non-finite maximum is flagged.  The element inside
+// the best vector is resolved once at the end of the pass (arg_resolve).
+__device__ __forceinline__ void arg_track(float& v, int& vec, float c, int i, unsigned& bad,
+                                          unsigned bit) {
+  if (!(c <= 3.402823466e38f)) bad |= bit;
+  const bool better = c > v;
+  v = better ? c : v;
+  vec = better ? i : vec;
 }
 
-// Argmax update for one vector: the lowest index of the vector maximum wins
-// a strict improvement; a non-finite maximum is flagged.
+// Lowest index inside vector `vec` whose value equals v (INT_MAX if none).
 template <int NP>
-__device__ __forceinline__ void arg_update(float& v, int& idx, float c, const f2 (&x)[NP],
-                                           int base, unsigned& bad, unsigned bit) {
-  if (!(c <= 3.402823466e38f)) bad |= bit;
-  if (c > v) {
-    v = c;
+__device__ __forceinline__ int arg_in_vector(const f2 (&x)[NP], float v, int base) {
+  int idx = INT_MAX;
 #pragma unroll
-    for (int h = NP - 1; h >= 0; --h) {
-      float lo, hi;
-      upk(x[h], lo, hi);
-      if (hi == c) idx = base + 2 * h + 1;
-      if (lo == c) idx = base + 2 * h;
-    }
+  for (int h = NP - 1; h >= 0; --h) {
+    float lo, hi;
+    upk(x[h], lo, hi);
+    if (hi == v) idx = base + 2 * h + 1;
+    if (lo == v) idx = base + 2 * h;
   }
+  return idx;
 }
 
 // Residual max(0, q - p) and fused q masses of one vector (stochastic mode);
@@ -328,83 +327,92 @@ __device__ __forceinline__ void pass1(const T* ra, const T* rb, const T* rt, int
   constexpr bool needB = (F & (F_LB | F_LS | F_AS)) != 0;
   constexpr bool needT = (F & (F_LT | F_LS | F_AS | F_AT)) != 0;
   constexpr bool needS = (F & (F_LS | F_AS)) != 0;
+  constexpr int STEP = 2 * kTThreads * VE;  // elements per two rounds
   const f2 beta2 = pk(beta, beta);
   const f2 L2 = pk(kLog2e, kLog2e);
   f2 acc[4] = {0ull, 0ull, 0ull, 0ull};
-  int waited = -1;
-  for (int kr = 0; kr < rounds; kr += 2) {
-    const int c_hi = min(kr + 1, rounds - 1) / rc;
-    while (waited < c_hi) {
-      ++waited;
-      if (!sh->broken && !mbar_wait_bounded(&sh->bar[waited], 0, kCopyTimeoutNs))
-        atomicOr(&sh->broken, kBadTimeout);
-    }
-    const int i0 = kr * kTThreads + static_cast<int>(threadIdx.x);
-    const int i1 = i0 + kTThreads;
-    if (i0 >= nv) continue;
-    const bool has1 = i1 < nv;
-    f2 xa[NP], xb[NP], xt[NP], xs[NP], ya[NP], yb[NP], yt[NP], ys[NP];
-    if (needA) {
-      load_pairs(ra + i0 * VE, xa);
-      load_or_fill(ra + i1 * VE, has1, ya);
-    }
-    if (needB) {
-      load_pairs(rb + i0 * VE, xb);
-      load_or_fill(rb + i1 * VE, has1, yb);
-    }
-    if (needT) {
-      load_pairs(rt + i0 * VE, xt);
-      load_or_fill(rt + i1 * VE, has1, yt);
-    }
-    if (needS) {
-#pragma unroll
-      for (int h = 0; h < NP; ++h) {
-        xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
-        ys[h] = fma2(beta2, sub2(ya[h], yb[h]), yt[h]);
-      }
-    }
-    if (F & F_LA) online_pairs2(e.m[0], acc[0], xa, ya, L2);
-    if (F & F_LB) online_pairs2(e.m[1], acc[1], xb, yb, L2);
-    float ct0 = 0.f, ct1 = 0.f, cs0 = 0.f, cs1 = 0.f;
-    if (F & F_LT) {
-      online_pairs2(e.m[2], acc[2], xt, yt, L2);
-      if (F & F_AT) {
-        ct0 = vmax_pairs(xt);
-        ct1 = vmax_pairs(yt);
-      }
-    } else if (F & F_AT) {
-      ct0 = vmax_pairs_nan(xt);
-      ct1 = vmax_pairs_nan(yt);
-    }
-    if (F & F_LS) {
-      online_pairs2(e.m[3], acc[3], xs, ys, L2);
-      if (F & F_AS) {
-        cs0 = vmax_pairs(xs);
-        cs1 = vmax_pairs(ys);
-      }
-    } else if (F & F_AS) {
-      cs0 = vmax_pairs_nan(xs);
-      cs1 = vmax_pairs_nan(ys);
-    }
-    const int base0 = lo + i0 * VE, base1 = lo + i1 * VE;
-    if (F & F_AS) {
-      arg_update(e.vs, e.is, cs0, xs, base0, e.bad, kBadS);
-      if (has1) arg_update(e.vs, e.is, cs1, ys, base1, e.bad, kBadS);
-    }
-    if (F & F_AT) {
-      arg_update(e.vt, e.it, ct0, xt, base0, e.bad, kBadT);
-      if (has1) arg_update(e.vt, e.it, ct1, yt, base1, e.bad, kBadT);
-    }
-  }
-  // every chunk is waited for, even by threads that ran out of vectors
-  while (waited < kChunks - 1) {
-    ++waited;
-    if (waited * rc < rounds && !sh->broken &&
-        !mbar_wait_bounded(&sh->bar[waited], 0, kCopyTimeoutNs))
+  int vec_s = -1, vec_t = -1;  // vectors holding the best s and t so far
+  const int tid = static_cast<int>(threadIdx.x);
+  for (int c = 0, r0 = 0; c < kChunks && r0 < rounds; ++c, r0 += rc) {
+    if (!sh->broken && !mbar_wait_bounded(&sh->bar[c], 0, kCopyTimeoutNs))
       atomicOr(&sh->broken, kBadTimeout);
+    const int r1 = min(rounds, r0 + rc);
+    int i0 = r0 * kTThreads + tid;          // vector index of this thread's first vector
+    int e0 = i0 * VE;                       // its element offset in the slice
+    for (int kr = r0; kr < r1; kr += 2, i0 += 2 * kTThreads, e0 += STEP) {
+      if (i0 >= nv) break;
+      const bool has1 = (kr + 1 < r1) && (i0 + kTThreads < nv);
+      const int e1 = e0 + kTThreads * VE;
+      f2 xa[NP], xb[NP], xt[NP], xs[NP], ya[NP], yb[NP], yt[NP], ys[NP];
+      if (needA) {
+        load_pairs(ra + e0, xa);
+        load_or_fill(ra + e1, has1, ya);
+      }
+      if (needB) {
+        load_pairs(rb + e0, xb);
+        load_or_fill(rb + e1, has1, yb);
+      }
+      if (needT) {
+        load_pairs(rt + e0, xt);
+        load_or_fill(rt + e1, has1, yt);
+      }
+      if (needS) {
+#pragma unroll
+        for (int h = 0; h < NP; ++h) {
+          xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
+          ys[h] = fma2(beta2, sub2(ya[h], yb[h]), yt[h]);
+        }
+      }
+      if (F & F_LA) online_pairs2(e.m[0], acc[0], xa, ya, L2);
+      if (F & F_LB) online_pairs2(e.m[1], acc[1], xb, yb, L2);
+      float ct0 = 0.f, ct1 = 0.f, cs0 = 0.f, cs1 = 0.f;
+      if (F & F_LT) {
+        online_pairs2(e.m[2], acc[2], xt, yt, L2);
+        if (F & F_AT) {
+          ct0 = vmax_pairs(xt);
+          ct1 = vmax_pairs(yt);
+        }
+      } else if (F & F_AT) {
+        ct0 = vmax_pairs_nan(xt);
+        ct1 = vmax_pairs_nan(yt);
+      }
+      if (F & F_LS) {
+        online_pairs2(e.m[3], acc[3], xs, ys, L2);
+        if (F & F_AS) {
+          cs0 = vmax_pairs(xs);
+          cs1 = vmax_pairs(ys);
+        }
+      } else if (F & F_AS) {
+        cs0 = vmax_pairs_nan(xs);
+        cs1 = vmax_pairs_nan(ys);
+      }
+      if (F & F_AS) {
+        arg_track(e.vs, vec_s, cs0, i0, e.bad, kBadS);
+        if (has1) arg_track(e.vs, vec_s, cs1, i0 + kTThreads, e.bad, kBadS);
+      }
+      if (F & F_AT) {
+        arg_track(e.vt, vec_t, ct0, i0, e.bad, kBadT);
+        if (has1) arg_track(e.vt, vec_t, ct1, i0 + kTThreads, e.bad, kBadT);
+      }
+    }
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) e.s[q] = hsum2(acc[q]);
+  // the element of the best vector (re-read once from shared memory)
+  if ((F & F_AS) && vec_s >= 0) {
+    f2 xa[NP], xb[NP], xt[NP], xs[NP];
+    load_pairs(ra + vec_s * VE, xa);
+    load_pairs(rb + vec_s * VE, xb);
+    load_pairs(rt + vec_s * VE, xt);
+#pragma unroll
+    for (int h = 0; h < NP; ++h) xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
+    e.is = arg_in_vector(xs, e.vs, lo + vec_s * VE);
+  }
+  if ((F & F_AT) && vec_t >= 0) {
+    f2 xt[NP];
+    load_pairs(rt + vec_t * VE, xt);
+    e.it = arg_in_vector(xt, e.vt, lo + vec_t * VE);
+  }
 }
 
 // Pass 1, block combine, push to the cluster, barrier, local combine; leaves
@@ -431,7 +439,7 @@ __device__ __forceinline__ void pass1_and_combine(const T* ra, const T* rb, cons
     }
     push_record(w, sh->recv1(), rank, C, cluster);
   }
-  cluster.sync();  // B1: every CTA's pass-1 record is in every CTA
+  cluster_barrier(warp == 0);  // B1: every CTA's pass-1 record is in every CTA
   if (warp == 0) {
     X1 w = (lane < C) ? sh->recv1()[lane] : x1_neutral();
     warp_reduce_x1<F>(w);
@@ -454,101 +462,135 @@ __device__ __forceinline__ void pass1_and_combine(const T* ra, const T* rb, cons
 
 // ---------------------------------------------------------------- pass 2
 
+// Divergence terms of one vector (Eq. 3): JSD terms p (log2 p - log2 m) and
+// q (log2 q - log2 m) with m = p + q, their mass m, or KL terms.
+template <int NP, bool JSD, bool KL>
+__device__ __forceinline__ void div_terms(const f2 (&xa)[NP], const f2 (&xb)[NP], const f2 (&p)[NP],
+                                          f2 L2, f2 nA2, f2 nB2, f2 tiny2, f2& ja, f2& jb,
+                                          f2& ms2, f2& kl2) {
+#pragma unroll
+  for (int h = 0; h < NP; ++h) {
+    const f2 la2 = fma2(xa[h], L2, nA2);
+    const f2 lb2 = fma2(xb[h], L2, nB2);
+    if (JSD) {
+      const f2 q = ex2_2(lb2);
+      const f2 m = add2(add2(p[h], q), tiny2);
+      const f2 lg = lg2_2(m);
+      ja = fma2(p[h], sub2(la2, lg), ja);
+      jb = fma2(q, sub2(lb2, lg), jb);
+      ms2 = add2(ms2, m);
+    }
+    if (KL) kl2 = fma2(p[h], sub2(la2, lb2), kl2);
+  }
+}
+
+// Pass 2 over the slice, two vectors per step (an absent second vector is
+// filled with -1e30, which contributes nothing).
 template <typename T, unsigned G, bool LP>
-__device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int nv, float beta,
-                                      float A2, float B2, float S2, float lse_s, X2& x,
-                                      float (&mr)[kMaxRounds], float (&mq)[kMaxRounds],
-                                      float* lp) {
+__device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int nv, int rounds,
+                                      float beta, float A2, float B2, float S2, float lse_s, X2& x,
+                                      float* lp, float* vmass) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
   constexpr bool JSD = (G & G_JSD) != 0, KL = (G & G_KL) != 0, RES = (G & G_RES) != 0;
   constexpr bool QF = (G & G_QF) != 0;
+  constexpr bool needT = RES || QF || LP;
   const f2 beta2 = pk(beta, beta);
   const f2 L2 = pk(kLog2e, kLog2e);
   const f2 nA2 = pk(-A2, -A2), nB2 = pk(-B2, -B2), nS2 = pk(-S2, -S2);
   const f2 tiny2 = pk(kMinNormal, kMinNormal);
   const f2 nl2 = pk(-lse_s, -lse_s);
-  f2 ja = 0ull, jb = 0ull, ms2 = 0ull, kl2 = 0ull;
-  float R = 0.f, Q = 0.f;
-#pragma unroll
-  for (int jr = 0; jr < kMaxRounds; ++jr) {
-    const int i = jr * kTThreads + static_cast<int>(threadIdx.x);
-    float vr = 0.f, vq = 0.f;
-    if (i < nv) {
-      f2 xa[NP], xb[NP], xt[NP];
-      load_pairs(ra + i * VE, xa);
-      load_pairs(rb + i * VE, xb);
-      if (RES || QF || LP) load_pairs(rt + i * VE, xt);
-      f2 p[NP];
-      if (RES) {
-        f2 qf[NP], r[NP];
-        vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
-        vr = vsum(r);
-        vq = vsum(qf);
-      } else if (QF) {
-        f2 qf[NP];
-#pragma unroll
-        for (int h = 0; h < NP; ++h)
-          qf[h] = ex2_2(fma2(fma2(beta2, sub2(xa[h], xb[h]), xt[h]), L2, nS2));
-        vq = vsum(qf);
+  f2 ja = 0ull, jb = 0ull, ms2 = 0ull, kl2 = 0ull, R2 = 0ull, Q2 = 0ull;
+  for (int kr = 0; kr < rounds; kr += 2) {
+    const int i0 = kr * kTThreads + static_cast<int>(threadIdx.x);
+    const int i1 = i0 + kTThreads;
+    if (i0 >= nv) {
+      if (RES || QF) {
+        vmass[kr * kTThreads + threadIdx.x] = 0.f;
+        if (kr + 1 < rounds) vmass[(kr + 1) * kTThreads + threadIdx.x] = 0.f;
       }
-      if (!RES && (JSD || KL)) {
+      continue;
+    }
+    const bool has1 = i1 < nv;
+    f2 xa[NP], xb[NP], xt[NP], ya[NP], yb[NP], yt[NP];
+    load_pairs(ra + i0 * VE, xa);
+    load_pairs(rb + i0 * VE, xb);
+    load_or_fill(ra + i1 * VE, has1, ya);
+    load_or_fill(rb + i1 * VE, has1, yb);
+    if (needT) {
+      load_pairs(rt + i0 * VE, xt);
+      load_or_fill(rt + i1 * VE, has1, yt);
+    }
+    f2 px[NP], py[NP];
+    if (RES) {
+      f2 qx[NP], qy[NP], rx[NP], ry[NP];
+      vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, px, qx, rx);
+      vec_masses(ya, yb, yt, beta2, L2, nA2, nS2, py, qy, ry);
 #pragma unroll
-        for (int h = 0; h < NP; ++h) p[h] = ex2_2(fma2(xa[h], L2, nA2));
+      for (int h = 0; h < NP; ++h) Q2 = add2(Q2, add2(qx[h], qy[h]));
+      // residual mass of each vector, kept for the inverse-CDF walk
+      const float r0 = vsum(rx), r1 = vsum(ry);
+      R2 = add2(R2, pk(r0, r1));
+      vmass[kr * kTThreads + threadIdx.x] = r0;
+      if (kr + 1 < rounds) vmass[(kr + 1) * kTThreads + threadIdx.x] = r1;
+    } else if (QF) {
+      f2 qx[NP], qy[NP];
+#pragma unroll
+      for (int h = 0; h < NP; ++h) {
+        qx[h] = ex2_2(fma2(fma2(beta2, sub2(xa[h], xb[h]), xt[h]), L2, nS2));
+        qy[h] = ex2_2(fma2(fma2(beta2, sub2(ya[h], yb[h]), yt[h]), L2, nS2));
       }
-      if (JSD || KL) {
+      // fused mass of each vector, kept for the inverse-CDF walk
+      const float q0 = vsum(qx), q1 = vsum(qy);
+      Q2 = add2(Q2, pk(q0, q1));
+      vmass[kr * kTThreads + threadIdx.x] = q0;
+      if (kr + 1 < rounds) vmass[(kr + 1) * kTThreads + threadIdx.x] = q1;
+    } else if (JSD || KL) {
 #pragma unroll
-        for (int h = 0; h < NP; ++h) {
-          const f2 la2 = fma2(xa[h], L2, nA2);
-          const f2 lb2 = fma2(xb[h], L2, nB2);
-          if (JSD) {
-            const f2 q = ex2_2(lb2);
-            const f2 m = add2(add2(p[h], q), tiny2);
-            const f2 lg = lg2_2(m);
-            ja = fma2(p[h], sub2(la2, lg), ja);
-            jb = fma2(q, sub2(lb2, lg), jb);
-            ms2 = add2(ms2, m);
-          }
-          if (KL) kl2 = fma2(p[h], sub2(la2, lb2), kl2);
-        }
+      for (int h = 0; h < NP; ++h) {
+        px[h] = ex2_2(fma2(xa[h], L2, nA2));
+        py[h] = ex2_2(fma2(ya[h], L2, nA2));
       }
-      if (LP) {
+    }
+    if (JSD || KL) {
+      div_terms<NP, JSD, KL>(xa, xb, px, L2, nA2, nB2, tiny2, ja, jb, ms2, kl2);
+      div_terms<NP, JSD, KL>(ya, yb, py, L2, nA2, nB2, tiny2, ja, jb, ms2, kl2);
+    }
+    if (LP) {
 #pragma unroll
-        for (int h = 0; h < NP; ++h) {
-          const f2 s = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
-          float l0, l1;
-          upk(add2(s, nl2), l0, l1);
-          lp[i * VE + 2 * h] = l0;
-          lp[i * VE + 2 * h + 1] = l1;
+      for (int h = 0; h < NP; ++h) {
+        float l0, l1;
+        upk(add2(fma2(beta2, sub2(xa[h], xb[h]), xt[h]), nl2), l0, l1);
+        lp[i0 * VE + 2 * h] = l0;
+        lp[i0 * VE + 2 * h + 1] = l1;
+        if (has1) {
+          upk(add2(fma2(beta2, sub2(ya[h], yb[h]), yt[h]), nl2), l0, l1);
+          lp[i1 * VE + 2 * h] = l0;
+          lp[i1 * VE + 2 * h + 1] = l1;
         }
       }
     }
-    mr[jr] = vr;
-    mq[jr] = vq;
-    R += vr;
-    Q += vq;
   }
   x.j = hsum2(add2(ja, jb));
   x.msum = hsum2(ms2);
   x.kl = hsum2(kl2);
-  x.R = R;
-  x.Q = Q;
+  x.R = hsum2(R2);
+  x.Q = hsum2(Q2);
 }
 
-// Pass 2, block and cluster combine: divergence, inverse-CDF mass and owner.
+// Pass 2, block combine, push to the cluster, barrier, local combine:
+// divergence, inverse-CDF mass and the CTA that owns the draw.
 template <typename T, unsigned G, bool LP, bool STOCH>
 __device__ __forceinline__ void pass2_and_combine(const T* ra, const T* rb, const T* rt, int nv,
-                                                  float beta, float* lp, SharedTma* sh, int rank,
-                                                  int C,
-                                                  bool r_allowed, float u_last,
-                                                  float (&mr)[kMaxRounds],
-                                                  float (&mq)[kMaxRounds],
+                                                  int rounds, float beta, float* lp,
+                                                  SharedTma* sh, int rank, int C, bool r_allowed,
+                                                  float u_last, float* vmass,
                                                   cg::cluster_group& cluster) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
   X2 x = x2_zero();
-  pass2<T, G, LP>(ra, rb, rt, nv, beta, lse_a * kLog2e, lse_b * kLog2e, lse_s * kLog2e, lse_s, x,
-                  mr, mq, lp);
+  pass2<T, G, LP>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e, lse_s * kLog2e,
+                  lse_s, x, lp, vmass);
   warp_reduce_x2<G>(x);
   if (lane == 0) sh->w2[warp] = x;
   __syncthreads();
@@ -557,7 +599,7 @@ __device__ __forceinline__ void pass2_and_combine(const T* ra, const T* rb, cons
     warp_reduce_x2<G>(w);
     push_record(w, sh->recv2(C), rank, C, cluster);
   }
-  cluster.sync();  // B2: every CTA's pass-2 record is in every CTA
+  cluster_barrier(warp == 0);  // B2: every CTA's pass-2 record is in every CTA
   if (warp == 0) {
     const X2 w = (lane < C) ? sh->recv2(C)[lane] : x2_zero();
     X2 tot = w;
@@ -605,34 +647,54 @@ __device__ __forceinline__ void pass2_and_combine(const T* ra, const T* rb, cons
 
 // ---------------------------------------------------------------- inverse-CDF walk
 
+// Residual (use_r) or fused mass of vector i of the slice, summed.
+template <typename T>
+__device__ __forceinline__ float vec_mass(const T* ra, const T* rb, const T* rt, int i, bool use_r,
+                                          f2 beta2, f2 L2, f2 nA2, f2 nS2) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  constexpr int NP = VE / 2;
+  f2 xa[NP], xb[NP], xt[NP], p[NP], qf[NP], r[NP];
+  load_pairs(ra + i * VE, xa);
+  load_pairs(rb + i * VE, xb);
+  load_pairs(rt + i * VE, xt);
+  vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
+  return use_r ? vsum(r) : vsum(qf);
+}
+
 // In the CTA that owns the target: the smallest slice index whose cumulative
-// mass (index order: round, thread, element) exceeds tau_local.  Returns the
-// index within the row, or -1.
+// mass (index order: round, thread, element) exceeds tau_local.  The masses
+// are recomputed here exactly as pass 2 computed them.  Returns the index
+// within the row, or -1.
 template <typename T>
 __device__ int walk(SharedTma* sh, const T* ra, const T* rb, const T* rt, int nv, int rounds,
-                    int lo, float beta, const float (&mr)[kMaxRounds],
-                    const float (&mq)[kMaxRounds]) {
+                    int lo, float beta, const float* vmass, bool stored_r) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const bool use_r = sh->use_r != 0;
   const float tau = sh->tau_local;
   const float A2 = sh->lse[0] * kLog2e, S2 = sh->lse[3] * kLog2e;
-  float m[kMaxRounds];
-#pragma unroll
-  for (int j = 0; j < kMaxRounds; ++j) m[j] = use_r ? mr[j] : mq[j];
-#pragma unroll
-  for (int j = 0; j < kMaxRounds; ++j) {
-    if (j < rounds) {
-      const float v = warp_sum(m[j]);
-      if (lane == 0) sh->wr[j][warp] = v;
-    }
+  const f2 beta2 = pk(beta, beta), L2 = pk(kLog2e, kLog2e);
+  const f2 nA2 = pk(-A2, -A2), nS2 = pk(-S2, -S2);
+  // pass 2 kept the residual masses of draft rows and the fused masses of
+  // the bonus row; the other kind (a draft row whose residual is zero) is
+  // recomputed exactly as pass 2 computes it
+  const bool stored = (use_r == stored_r);
+  int last_pos = -1;  // this thread's last vector with positive mass
+  for (int j = 0; j < rounds; ++j) {
+    const int i = j * kTThreads + tid;
+    float v = 0.f;
+    if (i < nv)
+      v = stored ? vmass[j * kTThreads + tid] : vec_mass(ra, rb, rt, i, use_r, beta2, L2, nA2, nS2);
+    if (v > 0.f) last_pos = i;
+    const float ws = warp_sum(v);
+    if (lane == 0) sh->wr[j][warp] = ws;
   }
   __syncthreads();
   if (tid == 0) {
     float cum = 0.f, tj = 0.f;
     int js = -1;
-    for (int j = 0; j < rounds && j < kMaxRounds; ++j) {
+    for (int j = 0; j < rounds; ++j) {
       float tot = 0.f;
       for (int w = 0; w < kTWarps; ++w) tot += sh->wr[j][w];
       if (cum + tot > tau) {
@@ -648,13 +710,11 @@ __device__ int walk(SharedTma* sh, const T* ra, const T* rb, const T* rt, int nv
   }
   __syncthreads();
   const int js = sh->jstar;
-  const f2 beta2 = pk(beta, beta), L2 = pk(kLog2e, kLog2e);
-  const f2 nA2 = pk(-A2, -A2), nS2 = pk(-S2, -S2);
   if (js >= 0) {
+    const int i = js * kTThreads + tid;
     float x = 0.f;
-#pragma unroll
-    for (int j = 0; j < kMaxRounds; ++j)
-      if (j == js) x = m[j];
+    if (i < nv)
+      x = stored ? vmass[js * kTThreads + tid] : vec_mass(ra, rb, rt, i, use_r, beta2, L2, nA2, nS2);
     float incl = x;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
@@ -668,8 +728,7 @@ __device__ int walk(SharedTma* sh, const T* ra, const T* rb, const T* rt, int nv
     incl += woff;
     const float excl = incl - x;
     const float tj = sh->tau_j;
-    const int i = js * kTThreads + tid;
-    if (x > 0.f && i < nv && excl <= tj && tj < incl) {
+    if (x > 0.f && excl <= tj && tj < incl) {
       f2 xa[NP], xb[NP], xt[NP], p[NP], qf[NP], r[NP];
       load_pairs(ra + i * VE, xa);
       load_pairs(rb + i * VE, xb);
@@ -697,21 +756,17 @@ __device__ int walk(SharedTma* sh, const T* ra, const T* rb, const T* rt, int nv
   __syncthreads();
   if (found0 < 0) {
     // the target fell into the rounding gap at the end: last positive element
-    int key = -1;
-#pragma unroll
-    for (int j = 0; j < kMaxRounds; ++j)
-      if (m[j] > 0.f) key = j * kTThreads + tid;
-    if (key >= 0) atomicMax(&sh->found, key);
+    if (last_pos >= 0) atomicMax(&sh->found, last_pos);
     __syncthreads();
     const int kmax = sh->found;
     __syncthreads();
     if (tid == 0) sh->found = -1;
     __syncthreads();
-    if (kmax >= 0 && key == kmax) {
+    if (kmax >= 0 && last_pos == kmax) {
       f2 xa[NP], xb[NP], xt[NP], p[NP], qf[NP], r[NP];
-      load_pairs(ra + key * VE, xa);
-      load_pairs(rb + key * VE, xb);
-      load_pairs(rt + key * VE, xt);
+      load_pairs(ra + kmax * VE, xa);
+      load_pairs(rb + kmax * VE, xb);
+      load_pairs(rt + kmax * VE, xt);
       vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
       int last = -1;
 #pragma unroll
@@ -721,7 +776,7 @@ __device__ int walk(SharedTma* sh, const T* ra, const T* rb, const T* rt, int nv
         if (v0 > 0.f) last = 2 * h;
         if (v1 > 0.f) last = 2 * h + 1;
       }
-      if (last >= 0) sh->found = lo + key * VE + last;
+      if (last >= 0) sh->found = lo + kmax * VE + last;
     }
     __syncthreads();
   }
@@ -748,11 +803,15 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   const int n = max(0, min(W, V - lo));
   const int nv = n / VE;
   const int rounds = (nv + kTThreads - 1) / kTThreads;
-  const int rc = max(1, (rounds + kChunks - 1) / kChunks);  // rounds per chunk
+  // rounds per chunk, even so that pass 1's pairs of rounds never straddle a chunk
+  const int rc = max(2, ((rounds + kChunks - 1) / kChunks + 1) & ~1);
   T* sa = reinterpret_cast<T*>(smem_tma);
   T* sb = sa + W;
   T* st = sb + W;
   SharedTma* sh = reinterpret_cast<SharedTma*>(smem_tma + P.sh_off);
+  // stochastic: per-thread, per-round sampling masses after the records
+  float* vmass = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sh) +
+                                          shared_tma_bytes(C));
   const float beta = P.beta;
   const bool leader = (rank == 0 && tid == 0);
   const bool only_t = !STOCH && !P.full && bonus && !P.fuse_bonus;
@@ -825,36 +884,33 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
   const bool klg = P.divergence == ASYMSPEC_DIV_KL;
   const bool run2 = STOCH || P.full || (!bonus && (jsd || klg));
-  float mr[kMaxRounds], mq[kMaxRounds];
-#pragma unroll
-  for (int j = 0; j < kMaxRounds; ++j) mr[j] = mq[j] = 0.f;
   if (run2) {
     float* lp = P.logprobs ? P.logprobs + static_cast<size_t>(row) * V + lo : nullptr;
     const bool r_allowed = STOCH && !bonus;
     constexpr unsigned RQ = STOCH ? G_RES : 0u;
     if (STOCH && bonus && !P.full) {
-      pass2_and_combine<T, G_QF, false, STOCH>(sa, sb, st, nv, beta, nullptr, sh, rank, C, false,
-                                               u_last, mr, mq, cluster);
+      pass2_and_combine<T, G_QF, false, STOCH>(sa, sb, st, nv, rounds, beta, nullptr, sh, rank,
+                                               C, false, u_last, vmass, cluster);
     } else if (lp) {
       if (jsd)
-        pass2_and_combine<T, G_JSD | RQ, true, STOCH>(sa, sb, st, nv, beta, lp, sh, rank, C,
-                                                      r_allowed, u_last, mr, mq, cluster);
+        pass2_and_combine<T, G_JSD | RQ, true, STOCH>(sa, sb, st, nv, rounds, beta, lp, sh, rank, C,
+                                              r_allowed, u_last, vmass, cluster);
       else if (klg)
-        pass2_and_combine<T, G_KL | RQ, true, STOCH>(sa, sb, st, nv, beta, lp, sh, rank, C,
-                                                     r_allowed, u_last, mr, mq, cluster);
+        pass2_and_combine<T, G_KL | RQ, true, STOCH>(sa, sb, st, nv, rounds, beta, lp, sh, rank, C,
+                                              r_allowed, u_last, vmass, cluster);
       else
-        pass2_and_combine<T, RQ, true, STOCH>(sa, sb, st, nv, beta, lp, sh, rank, C, r_allowed,
-                                              u_last, mr, mq, cluster);
+        pass2_and_combine<T, RQ, true, STOCH>(sa, sb, st, nv, rounds, beta, lp, sh, rank, C,
+                                              r_allowed, u_last, vmass, cluster);
     } else {
       if (jsd)
-        pass2_and_combine<T, G_JSD | RQ, false, STOCH>(sa, sb, st, nv, beta, nullptr, sh, rank, C,
-                                                       r_allowed, u_last, mr, mq, cluster);
+        pass2_and_combine<T, G_JSD | RQ, false, STOCH>(sa, sb, st, nv, rounds, beta, nullptr, sh, rank, C,
+                                              r_allowed, u_last, vmass, cluster);
       else if (klg)
-        pass2_and_combine<T, G_KL | RQ, false, STOCH>(sa, sb, st, nv, beta, nullptr, sh, rank, C,
-                                                      r_allowed, u_last, mr, mq, cluster);
+        pass2_and_combine<T, G_KL | RQ, false, STOCH>(sa, sb, st, nv, rounds, beta, nullptr, sh, rank, C,
+                                              r_allowed, u_last, vmass, cluster);
       else
-        pass2_and_combine<T, RQ, false, STOCH>(sa, sb, st, nv, beta, nullptr, sh, rank, C,
-                                               r_allowed, u_last, mr, mq, cluster);
+        pass2_and_combine<T, RQ, false, STOCH>(sa, sb, st, nv, rounds, beta, nullptr, sh, rank, C,
+                                              r_allowed, u_last, vmass, cluster);
     }
   } else if (tid == 0) {
     sh->D = 0.f;
@@ -863,7 +919,7 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   // ---- stochastic: inverse-CDF draw in the owning CTA, handed to rank 0
   if constexpr (STOCH) {
     if (rank == sh->owner) {
-      const int pick = walk<T>(sh, sa, sb, st, nv, rounds, lo, beta, mr, mq);
+      const int pick = walk<T>(sh, sa, sb, st, nv, rounds, lo, beta, vmass, !bonus || P.full);
       if (tid == 0) {
         *cluster.map_shared_rank(&sh->sample, 0) = pick;
         mbar_arrive_remote(&sh->sample_bar, 0);
