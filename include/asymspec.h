@@ -61,6 +61,7 @@ extern "C" {
 #define ASYMSPEC_ERR_WORKSPACE (-4)     /* workspace missing or smaller than asymspec_workspace_bytes() */
 #define ASYMSPEC_ERR_CUDA (-5)          /* a CUDA call failed; see asymspec_last_cuda_error() */
 #define ASYMSPEC_ERR_TOO_LARGE (-6)     /* V too large for the on-chip row slices (see asymspec_plan) */
+#define ASYMSPEC_ERR_SCRATCH_LIMIT (-7) /* B*(K+1) above ASYMSPEC_STATIC_MAX_ROWS (asymspec_fuse_verify_static) */
 
 /* ---- device error-word bits (data errors, per batch element) ----------- */
 #define ASYMSPEC_DATA_BAD_TOKEN 0x1u    /* a draft token outside [0, V) */
@@ -176,6 +177,44 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
                             int32_t* out_row_tokens, float* out_fused_logprobs,
                             uint32_t* out_error_word, const asymspec_launch_opts* opts,
                             void* stream);
+
+/*
+ * The step of asymspec_fuse_verify without any allocation.  The paper has no
+ * counterpart: this is a deployment variant of the same launch.
+ *
+ * Callers that cannot allocate device memory per step use it: a serving loop
+ * that has reserved all free HBM up front for its own allocator (KV cache,
+ * activations), where a per-step cudaMallocAsync can fail or make the pool
+ * grow and trim, and plain C hosts that have no device allocator to provide
+ * the workspace asymspec_fuse_verify_ex wants.
+ *
+ * Scratch: the per-row records and per-element tickets live in one file-scope
+ * static __device__ array of the library, sized for B*(K+1) <= 8192 rows
+ * (147,456 bytes: 16 bytes per row and 4 per batch element).  Larger batches
+ * return ASYMSPEC_ERR_SCRATCH_LIMIT before anything is enqueued.  Each call
+ * enqueues on `stream` a zero fill of the B tickets (the only part that must
+ * start at zero; the records are written before they are read), then the
+ * launch of asymspec_fuse_verify_ex.  Nothing is allocated: no cudaMalloc,
+ * cudaMallocAsync, cudaFree or library call that allocates.
+ *
+ * Set-up: the first call on each device looks up the array's device address
+ * with cudaGetSymbolAddress (return code checked, ASYMSPEC_ERR_CUDA on
+ * failure) and caches it; that first call may load the module, so make it
+ * before any stream capture begins on that device.
+ *
+ * Concurrency: there is one scratch array per device.  Calls that overlap in
+ * time on one device (several streams, or several host threads) share it and
+ * race, with undefined results; order them (one stream, or events).
+ *
+ * Arguments, outputs and status codes are those of asymspec_fuse_verify.
+ */
+#define ASYMSPEC_STATIC_MAX_ROWS 8192
+int asymspec_fuse_verify_static(const void* logits_full, const void* logits_comp,
+                                const void* logits_ver, const int32_t* draft_tokens,
+                                const float* draft_probs, const float* uniforms, int B, int K,
+                                int V, int dtype, const asymspec_gate_params* gate_params,
+                                int32_t* out_accept_len, int32_t* out_next_token,
+                                void* stream);
 
 /* Launch parameters a call with these sizes would use, without launching.
  * Uses the current CUDA device. */

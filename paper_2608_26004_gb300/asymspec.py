@@ -23,6 +23,9 @@ ERR_MISALIGNED = -3
 ERR_WORKSPACE = -4
 ERR_CUDA = -5
 ERR_TOO_LARGE = -6
+ERR_SCRATCH_LIMIT = -7
+
+STATIC_MAX_ROWS = 8192  # B*(K+1) limit of fuse_verify_static
 
 DATA_BAD_TOKEN = 0x1
 DATA_NONFINITE = 0x2
@@ -46,6 +49,7 @@ EXPORTED = (
     "asymspec_workspace_reset",
     "asymspec_fuse_verify",
     "asymspec_fuse_verify_ex",
+    "asymspec_fuse_verify_static",
     "asymspec_plan",
     "asymspec_status_string",
     "asymspec_last_cuda_error",
@@ -114,6 +118,9 @@ def lib():
                                           ctypes.c_size_t, _P, _P, _P, _P,
                                           ctypes.POINTER(LaunchOpts), _P]
     L.asymspec_fuse_verify_ex.restype = _I
+    L.asymspec_fuse_verify_static.argtypes = [_P, _P, _P, _P, _P, _P, _I, _I, _I, _I,
+                                              ctypes.POINTER(GateParams), _P, _P, _P]
+    L.asymspec_fuse_verify_static.restype = _I
     L.asymspec_plan.argtypes = [_I, _I, _I, _I, ctypes.POINTER(GateParams),
                                 ctypes.POINTER(LaunchOpts), ctypes.POINTER(LaunchInfo)]
     L.asymspec_plan.restype = _I
@@ -166,6 +173,20 @@ def fuse_verify_ex(logits_full, logits_comp, logits_ver, draft_tokens, draft_pro
         logits_full, logits_comp, logits_ver, draft_tokens, draft_probs, uniforms, B, K, V,
         dtype, g, out_accept_len, out_next_token, workspace, workspace_nbytes, out_row_stats,
         out_row_tokens, out_fused_logprobs, out_error_word, o, stream)
+
+
+def fuse_verify_static(logits_full, logits_comp, logits_ver, draft_tokens, draft_probs,
+                       uniforms, B, K, V, dtype, gate, out_accept_len, out_next_token,
+                       stream=0) -> int:
+    """asymspec_fuse_verify_static with device addresses (ints); returns the status.
+
+    Allocates nothing (the scratch is a static array of the library); calls
+    that overlap in time on one device race on it.
+    """
+    g = ctypes.byref(gate) if gate is not None else None
+    return lib().asymspec_fuse_verify_static(logits_full, logits_comp, logits_ver,
+                                             draft_tokens, draft_probs, uniforms, B, K, V,
+                                             dtype, g, out_accept_len, out_next_token, stream)
 
 
 def plan(B, K, V, dtype, gate=None, opts=None) -> LaunchInfo:

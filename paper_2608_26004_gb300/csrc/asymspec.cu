@@ -232,6 +232,38 @@ int check_opts(const asymspec_launch_opts* opts) {
   return ASYMSPEC_OK;
 }
 
+// Scratch of asymspec_fuse_verify_static: records for ASYMSPEC_STATIC_MAX_ROWS
+// rows, then tickets for the largest batch that can have that many rows
+// (K >= 1, so B <= ASYMSPEC_STATIC_MAX_ROWS / 2).  The layout is the one
+// asymspec_fuse_verify_ex gives any workspace, so every batch within the limit
+// fits: records end by 16 * MAX_ROWS bytes, tickets by 4 * MAX_ROWS / 2 more.
+constexpr size_t kStaticScratchBytes =
+    static_cast<size_t>(ASYMSPEC_STATIC_MAX_ROWS) * sizeof(int4) +
+    static_cast<size_t>(ASYMSPEC_STATIC_MAX_ROWS / 2) * sizeof(unsigned);
+static_assert(kStaticScratchBytes % 256 == 0, "static scratch ends on a 256-byte boundary");
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+// Device address of g_static_scratch, looked up once per device.
+constexpr int kMaxDevices = 64;
+std::mutex g_static_mu;
+void* g_static_addr[kMaxDevices] = {};
+
+int static_scratch(void** out) {
+  int device = 0;
+  cudaError_t e = cudaGetDevice(&device);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (device < 0 || device >= kMaxDevices) return ASYMSPEC_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_addr[device]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess) return cuda_fail(e);
+    g_static_addr[device] = p;
+  }
+  *out = g_static_addr[device];
+  return ASYMSPEC_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -412,6 +444,30 @@ int asymspec_fuse_verify(const void* logits_full, const void* logits_comp,
   return ASYMSPEC_OK;
 }
 
+int asymspec_fuse_verify_static(const void* logits_full, const void* logits_comp,
+                                const void* logits_ver, const int32_t* draft_tokens,
+                                const float* draft_probs, const float* uniforms, int B, int K,
+                                int V, int dtype, const asymspec_gate_params* gate_params,
+                                int32_t* out_accept_len, int32_t* out_next_token,
+                                void* stream) {
+  if (B < 1 || K < 1 || V < 2) return ASYMSPEC_ERR_INVALID_ARG;
+  if (static_cast<long long>(B) * (K + 1) > ASYMSPEC_STATIC_MAX_ROWS)
+    return ASYMSPEC_ERR_SCRATCH_LIMIT;
+  void* scratch = nullptr;
+  int st = static_scratch(&scratch);
+  if (st) return st;
+  // the tickets must start at zero; a call that did not complete may have
+  // left some set, so they are cleared on the caller's stream every time
+  cudaError_t e = cudaMemsetAsync(static_cast<char*>(scratch) + ws_records_bytes(B, K), 0,
+                                  static_cast<size_t>(B) * sizeof(unsigned),
+                                  static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e);
+  return asymspec_fuse_verify_ex(logits_full, logits_comp, logits_ver, draft_tokens,
+                                 draft_probs, uniforms, B, K, V, dtype, gate_params,
+                                 out_accept_len, out_next_token, scratch, kStaticScratchBytes,
+                                 nullptr, nullptr, nullptr, nullptr, nullptr, stream);
+}
+
 const char* asymspec_status_string(int status) {
   switch (status) {
     case ASYMSPEC_OK: return "ok";
@@ -421,6 +477,9 @@ const char* asymspec_status_string(int status) {
     case ASYMSPEC_ERR_WORKSPACE: return "workspace missing or too small";
     case ASYMSPEC_ERR_CUDA: return "CUDA error (see asymspec_last_cuda_error)";
     case ASYMSPEC_ERR_TOO_LARGE: return "problem too large for the on-chip row slices";
+    case ASYMSPEC_ERR_SCRATCH_LIMIT:
+      return "B*(K+1) exceeds ASYMSPEC_STATIC_MAX_ROWS (8192), the static scratch of "
+             "asymspec_fuse_verify_static; use asymspec_fuse_verify_ex with a workspace";
     default: return "unknown status";
   }
 }

@@ -98,6 +98,17 @@ def test_host_validation_codes(lib):
     assert st == A.ERR_INVALID_ARG                       # unknown kernel
 
 
+def test_static_entry_point_rejects_batches_above_its_scratch(lib):
+    # returns before any CUDA call: B*(K+1) above the static scratch's rows
+    args = (FAKE, FAKE, FAKE, FAKE, FAKE, FAKE)
+    assert A.fuse_verify_static(*args, 1025, 7, 64, A.FP32, None, FAKE, FAKE) \
+        == A.ERR_SCRATCH_LIMIT
+    assert A.fuse_verify_static(*args, 1, 8192, 64, A.FP32, None, FAKE, FAKE) \
+        == A.ERR_SCRATCH_LIMIT
+    assert A.fuse_verify_static(*args, 0, 7, 64, A.FP32, None, FAKE, FAKE) == A.ERR_INVALID_ARG
+    assert "8192" in A.status_string(A.ERR_SCRATCH_LIMIT)
+
+
 def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
     # the bench workload: TMA kernel, 8 CTAs of 96 KB per row, two CTAs per SM
     info = A.plan(64, 7, 128256, A.BF16)

@@ -1,0 +1,91 @@
+"""asymspec_fuse_verify_static: the step with its scratch in a static device array.
+
+The file name sorts last so that these calls also run after every other GPU
+test has used the library in the same process; the tests must pass both
+alone and then.  Every result is compared bit for bit with
+asymspec_fuse_verify_ex (same kernel, caller-owned zeroed workspace) on the
+same inputs, over two consecutive calls, so that the second call sees the
+scratch the first one left.
+"""
+import numpy as np
+import pytest
+
+from paper_2608_26004_gb300 import asymspec as A
+from paper_2608_26004_gb300 import synth
+from tests._parity import device_inputs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch():
+    import torch as _torch
+    assert _torch.cuda.is_available(), "the gpu tests need a CUDA device"
+    from paper_2608_26004_gb300 import build
+    build.build_cuda()
+    A.lib()
+    return _torch
+
+
+def _ptr(t):
+    return int(t.data_ptr())
+
+
+def run_static(torch, x, B, K, V, dtype, gate):
+    L = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    N = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    st = A.fuse_verify_static(_ptr(x["a"]), _ptr(x["b"]), _ptr(x["t"]), _ptr(x["tokens"]),
+                              _ptr(x["probs"]), _ptr(x["unif"]), B, K, V, dtype, gate,
+                              _ptr(L), _ptr(N), stream)
+    assert st == A.OK, A.status_string(st)
+    torch.cuda.synchronize()
+    return L.cpu().numpy(), N.cpu().numpy()
+
+
+def run_ex(torch, x, B, K, V, dtype, gate):
+    L = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    N = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    nbytes = A.workspace_bytes(B, K, V)
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    st = A.fuse_verify_ex(_ptr(x["a"]), _ptr(x["b"]), _ptr(x["t"]), _ptr(x["tokens"]),
+                          _ptr(x["probs"]), _ptr(x["unif"]), B, K, V, dtype, gate, _ptr(L),
+                          _ptr(N), _ptr(ws), nbytes, stream=stream)
+    assert st == A.OK, A.status_string(st)
+    torch.cuda.synchronize()
+    return L.cpu().numpy(), N.cpu().numpy()
+
+
+CASES = [
+    # (B, K, V, dtype, mode, seed): the second call reuses the scratch the first left
+    (8, 5, 151936, synth.BF16, A.MODE_STOCHASTIC, 11),
+    (3, 2, 4099, synth.BF16, A.MODE_GREEDY, 12),          # unaligned rows: generic kernel
+    (1024, 7, 64, synth.FP32, A.MODE_STOCHASTIC, 13),     # B*(K+1) = the 8192-row limit
+    (1024, 7, 64, synth.FP32, A.MODE_GREEDY, 14),
+]
+
+
+@pytest.mark.parametrize("first,second", [(0, 1), (2, 3), (3, 0)])
+def test_two_consecutive_calls_match_the_workspace_entry_point(torch, first, second):
+    for idx in (first, second):
+        B, K, V, dtype, mode, seed = CASES[idx]
+        batch = synth.generate(synth.Recipe(), seed, B, K, V, dtype)
+        x = device_inputs(batch, torch)
+        gate = A.gate_params(mode=mode)
+        Ls, Ns = run_static(torch, x, B, K, V, dtype, gate)
+        Le, Ne = run_ex(torch, x, B, K, V, dtype, gate)
+        assert np.array_equal(Ls, Le) and np.array_equal(Ns, Ne), f"case {idx} differs"
+        assert np.all(Ls >= 0) and np.all(Ls <= K) and np.all(Ns >= 0) and np.all(Ns < V)
+
+
+def test_rows_above_the_limit_are_rejected_before_any_launch(torch):
+    B, K, V = 1025, 7, 64                                 # 8200 rows > 8192
+    x = dict(a=torch.zeros(B * (K + 1) * V, device="cuda"))
+    L = torch.full((B,), -7, dtype=torch.int32, device="cuda")
+    st = A.fuse_verify_static(_ptr(x["a"]), _ptr(x["a"]), _ptr(x["a"]), _ptr(L), 0, 0, B, K,
+                              V, synth.FP32, None, _ptr(L), _ptr(L), 0)
+    assert st == A.ERR_SCRATCH_LIMIT
+    assert "8192" in A.status_string(st)
+    torch.cuda.synchronize()
+    assert np.all(L.cpu().numpy() == -7)                  # nothing ran
