@@ -34,8 +34,9 @@ if ROOT not in sys.path:
 METRIC = "verify rows/s (B×(K+1) vocab rows) and achieved HBM GB/s vs GB300 peak"
 WORKLOAD_CFG = 2
 FALLBACK_HBM_GBS = 6800.0
-KERNEL_SRC = os.path.join(ROOT, "paper_2608_26004_gb300", "csrc", "asymspec.cu")
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_fuse_verify_B64_K7_V128256_bf16.json")
+CSRC = os.path.join(ROOT, "paper_2608_26004_gb300", "csrc")
+KERNEL_SRCS = ("asymspec.cu", "device_common.cuh", "kernel_generic.cuh", "kernel_tma.cuh")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fuse_verify_tma_B64_K7_V128256_bf16_traffic.txt")
 REASON_BITS = {
     0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
     0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
@@ -76,21 +77,43 @@ def peaks():
 
 
 def kernel_hash() -> str:
-    with open(KERNEL_SRC, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    """sha256 (first 16 hex digits) over the kernel sources, in a fixed order."""
+    h = hashlib.sha256()
+    for name in KERNEL_SRCS:
+        with open(os.path.join(CSRC, name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def measured_traffic(mode: str):
-    """DRAM bytes per launch from a committed ncu summary of the same kernel source."""
+    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from
+    the committed ncu summary, or None once the kernel sources have changed
+    since those counters were taken."""
     try:
         with open(TRAFFIC_FILE) as f:
-            d = json.load(f)
-    except Exception:
+            kv = dict(line.split(":", 1) for line in f if ":" in line and not line.startswith("#"))
+    except OSError:
         return None
-    if d.get("kernel_sha256_16") != kernel_hash():
+    kv = {k.strip(): v.strip() for k, v in kv.items()}
+    if kv.get("kernel_sources_sha256_16") != kernel_hash():
         return None
-    v = d.get("dram_bytes_per_launch", {}).get(mode)
+    v = kv.get(f"{mode}_dram_bytes_per_launch")
     return float(v) if v else None
+
+
+def algorithmic_bytes(B: int, K: int, V: int, elt: int, stochastic: bool) -> int:
+    """Bytes one launch must move: every logit row it needs read once, the
+    per-draft inputs, and the two int32 outputs per batch element.
+
+    Stochastic mode needs a, b and t on all B*(K+1) rows plus the draft
+    probabilities and the K+1 uniforms; greedy mode (unfused bonus) needs all
+    three on the B*K draft rows but only t on the B bonus rows, and no
+    probabilities or uniforms.
+    """
+    row = V * elt
+    if stochastic:
+        return 3 * row * B * (K + 1) + 4 * B * K * 2 + 4 * B * (K + 1) + 8 * B
+    return 3 * row * B * K + row * B + 4 * B * K + 8 * B
 
 
 class ClockSampler:
@@ -232,7 +255,7 @@ def main():
     batch = synth.make_config(WORKLOAD_CFG, nb=args.batch or None)
     B, K, V = batch.B, batch.K, batch.V
     rows = B * (K + 1)
-    alg_bytes = 3 * rows * V * 2 + rows * 12 + B * 8  # logits once + token/prob/uniform + outputs
+    alg_bytes = algorithmic_bytes(B, K, V, 2, mode == A.MODE_STOCHASTIC)
 
     def to_dev_logits(x):
         return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).to(dev)
@@ -309,6 +332,7 @@ def main():
             raise A.AsymSpecError(st, "asymspec_fuse_verify_ex")
 
     ms_o = timed(lambda i: step_o(sets[i % 2]), args.steps, max(args.warmup, 3)) / args.steps
+    alg_bytes_o = algorithmic_bytes(B, K, V, 2, other_mode == A.MODE_STOCHASTIC)
 
     # ---- end to end through the C ABI with host buffers
     pin = dict(
@@ -361,7 +385,10 @@ def main():
         "clocks": clocks,
         "other_mode": {"mode": "greedy" if other_mode == A.MODE_GREEDY else "stochastic",
                        "ms_per_step": ms_o, "rows_per_s": world * rows / (ms_o * 1e-3),
-                       "hbm_gbs": alg_bytes / (ms_o * 1e-3) / 1e9},
+                       "hbm_gbs": alg_bytes_o / (ms_o * 1e-3) / 1e9,
+                       "algorithmic_bytes_per_launch": alg_bytes_o,
+                       "traffic": measured_traffic(
+                           "greedy" if other_mode == A.MODE_GREEDY else "stochastic")},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         mode_id = 1 if mode == A.MODE_STOCHASTIC else 0
