@@ -100,13 +100,16 @@ typedef struct {
 typedef struct {
   int32_t cluster_size;   /* CTAs per row triple: 1 to 16 */
   int32_t block_threads;  /* reserved, must be 0 (256 threads per CTA) */
-  int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC; ASYMSPEC_KERNEL_TMA */
+  int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC, _TMA or _STREAM */
 } asymspec_launch_opts;
 
 /* Kernels (asymspec_launch_opts.kernel, asymspec_launch_info.kernel). */
 #define ASYMSPEC_KERNEL_GENERIC 1  /* one cluster per row; any element-aligned input */
 #define ASYMSPEC_KERNEL_TMA 2      /* one cluster per row, chunked 1-D bulk copies, per-row
-                                      programs; rows 16-byte aligned (the default when they are) */
+                                      programs; rows 16-byte aligned */
+#define ASYMSPEC_KERNEL_STREAM 3   /* persistent grid over row tiles: pass 1 reads each tile from
+                                      HBM, pass 2 re-reads it from L2; rows 16-byte aligned and a
+                                      workspace of asymspec_workspace_bytes(); on request only */
 
 /* What a launch would use (filled by asymspec_plan). */
 typedef struct {
@@ -117,7 +120,7 @@ typedef struct {
   int64_t ctas;            /* CTAs in the grid */
   int32_t vector_path;     /* 1 if rows qualify for 16-byte copies (V * element size % 16 == 0) */
   int32_t max_active_clusters; /* clusters the device can hold at once (0 if unknown) */
-  int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC or ASYMSPEC_KERNEL_TMA */
+  int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC, _TMA or _STREAM */
 } asymspec_launch_info;
 
 /* Fills *p with the paper's defaults: gamma 0.5, beta 1.0, lambda 0.1,
@@ -125,10 +128,12 @@ typedef struct {
 void asymspec_default_gate_params(asymspec_gate_params* p);
 
 /* Bytes of device workspace asymspec_fuse_verify_ex needs for a batch of
- * B elements with K drafts (independent of V).  The workspace must be zeroed
- * once before its first use (cudaMemset or asymspec_workspace_reset); every
- * call that completes leaves it zeroed again.  Two calls in flight at the
- * same time must not share a workspace. */
+ * B elements with K drafts and V vocabulary entries (enough for every kernel
+ * and both dtypes).  The cluster kernels (the automatic choice) need only
+ * 16 B per row plus 4 B per element, the first 256-byte aligned parts of the
+ * same layout; the rest serves ASYMSPEC_KERNEL_STREAM.  The workspace must be zeroed once before its first use (cudaMemset
+ * or asymspec_workspace_reset); every call that completes leaves it zeroed
+ * again.  Two calls in flight at the same time must not share a workspace. */
 size_t asymspec_workspace_bytes(int B, int K, int V);
 
 /* Enqueues a zero fill of a workspace on `stream`. */
@@ -194,7 +199,8 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
  * return ASYMSPEC_ERR_SCRATCH_LIMIT before anything is enqueued.  Each call
  * enqueues on `stream` a zero fill of the B tickets (the only part that must
  * start at zero; the records are written before they are read), then the
- * launch of asymspec_fuse_verify_ex.  Nothing is allocated: no cudaMalloc,
+ * launch of asymspec_fuse_verify_ex, which with this scratch runs the cluster
+ * kernels (ASYMSPEC_KERNEL_TMA for aligned rows, else _GENERIC).  Nothing is allocated: no cudaMalloc,
  * cudaMallocAsync, cudaFree or library call that allocates.
  *
  * Set-up: the first call on each device looks up the array's device address

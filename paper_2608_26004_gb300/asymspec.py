@@ -67,6 +67,7 @@ class GateParams(ctypes.Structure):
 KERNEL_AUTO = 0
 KERNEL_GENERIC = 1
 KERNEL_TMA = 2
+KERNEL_STREAM = 3
 
 
 class LaunchOpts(ctypes.Structure):
@@ -222,15 +223,28 @@ class FuseVerify:
 
     ``__call__`` takes CUDA tensors ([B, K+1, V] logits as float32 or
     bfloat16, int32 tokens, float32 probabilities and uniforms) and enqueues
-    the step on the current stream.  Outputs are returned as tensors.
+    the step on the current stream.  Outputs are returned as tensors.  The
+    workspace is sized for V_max vocabulary entries, or for the first call's
+    V when V_max is not given (and grown, zeroed, for a larger V).
     """
 
-    def __init__(self, B_max: int, K: int, device=None):
-        import torch
+    def __init__(self, B_max: int, K: int, device=None, V_max: int | None = None):
         self.B_max, self.K = B_max, K
-        self.device = torch.device(device or "cuda")
-        self.nbytes = workspace_bytes(B_max, K, 2)
-        self.workspace = torch.zeros(self.nbytes, dtype=torch.uint8, device=self.device)
+        self.device = device
+        self.V_ws = 0
+        self.nbytes = 0
+        self.workspace = None
+        if V_max is not None:
+            self._ensure(V_max)
+
+    def _ensure(self, V: int):
+        import torch
+        if self.workspace is not None and V <= self.V_ws:
+            return
+        self.V_ws = V
+        self.nbytes = workspace_bytes(self.B_max, self.K, V)
+        self.workspace = torch.zeros(self.nbytes, dtype=torch.uint8,
+                                     device=torch.device(self.device or "cuda"))
 
     def __call__(self, logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=None,
                  uniforms=None, *, gamma=0.5, beta=1.0, lam=0.1, mode=MODE_GREEDY,
@@ -241,6 +255,7 @@ class FuseVerify:
         K = K1 - 1
         if K != self.K or B > self.B_max:
             raise ValueError("batch does not fit this workspace")
+        self._ensure(V)
         if logits_full.dtype == torch.float32:
             dtype = FP32
         elif logits_full.dtype == torch.bfloat16:

@@ -14,7 +14,15 @@ from concurrent.futures import ThreadPoolExecutor
 HERE = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(HERE)
 INCLUDE = os.path.join(ROOT, "include")
-CUDA_SRC = [os.path.join(HERE, "csrc", "asymspec.cu")]
+CSRC = os.path.join(HERE, "csrc")
+# one translation unit per kernel family and dtype, compiled in parallel
+CUDA_SRC = [os.path.join(CSRC, f) for f in (
+    "asymspec.cu", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu",
+    "k_stream_bf16_greedy.cu", "k_stream_bf16_stoch.cu",
+    "k_stream_f32_greedy.cu", "k_stream_f32_stoch.cu")]
+CUDA_HEADERS = [os.path.join(CSRC, f) for f in (
+    "device_common.cuh", "kernel_generic.cuh", "kernel_tma.cuh", "kernel_stream.cuh",
+    "kernels.h")]
 CUDA_LIB = os.path.join(HERE, "libasymspec.so")
 GENCODE = "arch=compute_103a,code=sm_103a"
 
@@ -30,24 +38,40 @@ def _stale(target: str, sources) -> bool:
     if not os.path.exists(target):
         return True
     t = os.path.getmtime(target)
-    deps = list(sources) + [os.path.join(INCLUDE, "asymspec.h")]
+    deps = list(sources) + CUDA_HEADERS + [os.path.join(INCLUDE, "asymspec.h")]
     return any(os.path.getmtime(s) > t for s in deps)
+
+
+def _run(cmd):
+    res = subprocess.run(cmd, capture_output=True, text=True)
+    if res.returncode != 0:
+        raise RuntimeError(f"nvcc failed ({' '.join(cmd)}):\n{res.stdout}\n{res.stderr}")
+    return res.stderr
 
 
 def build_cuda(force: bool = False, verbose: bool = False) -> str:
     if not force and not _stale(CUDA_LIB, CUDA_SRC):
         return CUDA_LIB
-    tmp = CUDA_LIB + f".tmp{os.getpid()}"
-    cmd = [nvcc_path(), "-gencode", GENCODE, "-O3", "-lineinfo", "-std=c++17",
-           "-I" + INCLUDE, "-Xcompiler", "-fPIC", "-shared", *CUDA_SRC, "-o", tmp]
+    nvcc = nvcc_path()
+    tag = f".tmp{os.getpid()}"
+    objs = [os.path.join(CSRC, os.path.basename(src)[:-3] + tag + ".o") for src in CUDA_SRC]
+    base = [nvcc, "-gencode", GENCODE, "-O3", "-lineinfo", "-std=c++17", "-I" + INCLUDE,
+            "-Xcompiler", "-fPIC"]
     if verbose:
-        cmd.insert(1, "-Xptxas=-v")
-    res = subprocess.run(cmd, capture_output=True, text=True)
-    if res.returncode != 0:
-        raise RuntimeError(f"nvcc failed ({' '.join(cmd)}):\n{res.stdout}\n{res.stderr}")
+        base.append("-Xptxas=-v")
+    try:
+        with ThreadPoolExecutor(len(CUDA_SRC)) as ex:
+            logs = list(ex.map(_run, [base + ["-c", src, "-o", obj]
+                                      for src, obj in zip(CUDA_SRC, objs)]))
+        tmp = CUDA_LIB + tag
+        _run([nvcc, "-shared", "-gencode", GENCODE, *objs, "-o", tmp])
+        os.replace(tmp, CUDA_LIB)
+    finally:
+        for obj in objs:
+            if os.path.exists(obj):
+                os.remove(obj)
     if verbose:
-        print(res.stderr)
-    os.replace(tmp, CUDA_LIB)
+        print("".join(logs))
     return CUDA_LIB
 
 

@@ -1,20 +1,25 @@
 // AsymSpec per-step fuse-and-verify on GB300 (sm_103a): host side of the C ABI
-// declared in include/asymspec.h, and the launch of its two kernels.
+// declared in include/asymspec.h, and the launch of its three kernels.
 //
 //   fuse_verify_tma      (kernel_tma.cuh) one cluster per row, each CTA's
 //                        slice brought in by chunked 1-D bulk copies, per-row
-//                        programs; the fast path for 16-byte aligned rows.
+//                        programs; the default for 16-byte aligned rows.
+//   fuse_verify_stream   (kernel_stream.cuh) persistent grid over row tiles;
+//                        pass 1 reads each tile from HBM, pass 2 from L2;
+//                        on request.
 //   fuse_verify_generic  (kernel_generic.cuh) one cluster per row, any
 //                        element-aligned input.
 //
-// Both read every logit row from HBM once, combine the per-CTA partial
-// reductions over DSMEM, and fold Algorithm 1's sequential scan into the
-// same launch through a per-element ticket in the workspace.
+// Each reads every logit row from HBM once and folds Algorithm 1's
+// sequential scan into the same launch through a per-element ticket in the
+// workspace.
+#include <algorithm>
 #include <mutex>
 
 #include "device_common.cuh"
 #include "kernel_generic.cuh"
-#include "kernel_tma.cuh"
+#include "kernel_stream.cuh"
+#include "kernels.h"
 
 namespace {
 
@@ -89,17 +94,84 @@ bool plan_tma(int V, int elt, int forced_C, bool stoch, Plan* pl) {
   return false;
 }
 
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+size_t ws_records_bytes(int B, int K) {
+  return round_up(static_cast<size_t>(B) * (K + 1) * sizeof(int4), 256);
+}
+
+size_t cluster_ws_bytes(int B, int K) {
+  return ws_records_bytes(B, K) + round_up(static_cast<size_t>(B) * sizeof(unsigned), 256);
+}
+
+// Workspace of the streaming kernel: the cluster kernels' records and
+// tickets first (same offsets), then the per-row and per-tile state.
+struct StreamLayout {
+  int NT, TS;
+  size_t tickets, p1cnt, p2cnt, ready, tags, stat, p1rec, p2rec, groups, total;
+};
+
+StreamLayout stream_layout(int B, int K, int V, int elt) {
+  StreamLayout L;
+  const size_t R = static_cast<size_t>(B) * (K + 1);
+  L.TS = kSRounds * kSThreads * (16 / elt);
+  L.NT = (V + L.TS - 1) / L.TS;
+  const size_t NT = static_cast<size_t>(L.NT);
+  size_t off = ws_records_bytes(B, K);
+  L.tickets = off;
+  off += round_up(static_cast<size_t>(B) * sizeof(unsigned), 256);
+  L.p1cnt = off;
+  off += round_up(R * sizeof(unsigned), 256);
+  L.p2cnt = off;
+  off += round_up(R * sizeof(unsigned), 256);
+  L.ready = off;
+  off += round_up(R * sizeof(unsigned), 256);
+  L.tags = off;
+  off += round_up(R * 4 * sizeof(unsigned long long), 256);
+  L.stat = off;
+  off += round_up(R * sizeof(RowStat), 256);
+  L.p1rec = off;
+  off += round_up(R * NT * sizeof(X1), 256);
+  L.p2rec = off;
+  off += round_up(R * NT * sizeof(X2), 256);
+  L.groups = off;
+  off += round_up(R * NT * kSGroups * sizeof(float), 256);
+  L.total = off;
+  return L;
+}
+
+// The streaming kernel's tiles stay below 2^31 entries of look-ahead and
+// items; rows longer than this many tiles use the cluster kernels.
+constexpr int kMaxStreamTiles = 31;
+
 int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_opts* opts,
-              bool vec_ok, Plan* pl) {
+              bool vec_ok, size_t ws_bytes, Plan* pl) {
   const int elt = elt_size(dtype);
   const int forced_C = (opts && opts->cluster_size > 0) ? opts->cluster_size : 0;
   const int forced_kernel = opts ? opts->kernel : 0;
   if (forced_C < 0 || forced_C > 16) return ASYMSPEC_ERR_INVALID_ARG;
   if (forced_kernel != 0 && forced_kernel != ASYMSPEC_KERNEL_GENERIC &&
-      forced_kernel != ASYMSPEC_KERNEL_TMA)
+      forced_kernel != ASYMSPEC_KERNEL_TMA && forced_kernel != ASYMSPEC_KERNEL_STREAM)
     return ASYMSPEC_ERR_INVALID_ARG;
   pl->rows = static_cast<long long>(B) * (K + 1);
   pl->vector_path = vec_ok;
+  const StreamLayout L = stream_layout(B, K, V, elt);
+  const bool stream_ok = vec_ok && L.NT <= kMaxStreamTiles && ws_bytes >= L.total;
+  (void)stream_ok;  // measured slower than the cluster kernel: chosen only on request
+  if (forced_kernel == ASYMSPEC_KERNEL_STREAM) {
+    if (!vec_ok) return ASYMSPEC_ERR_UNSUPPORTED;
+    if (L.NT > kMaxStreamTiles) return ASYMSPEC_ERR_TOO_LARGE;
+    if (ws_bytes < L.total) return ASYMSPEC_ERR_WORKSPACE;
+    pl->kernel = ASYMSPEC_KERNEL_STREAM;
+    pl->VE = 16 / elt;
+    pl->C = 1;
+    pl->W = L.TS;
+    pl->sh_off = 0;
+    pl->smem = 0;
+    pl->ctas = 0;  // set at launch from the device's occupancy
+    return ASYMSPEC_OK;
+  }
+  if (ws_bytes < cluster_ws_bytes(B, K)) return ASYMSPEC_ERR_WORKSPACE;
   bool ok = false;
   if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, stoch, pl)) {
     pl->kernel = ASYMSPEC_KERNEL_TMA;
@@ -118,24 +190,12 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
   return ASYMSPEC_OK;
 }
 
-using KernelFn = void (*)(KParams);
+using KernelFn = const void*;  // a __global__ function taking KParams (or SParams)
 
 KernelFn pick_kernel(const Plan& pl, int dtype, bool stoch) {
-  if (pl.kernel == ASYMSPEC_KERNEL_TMA) {
-    if (dtype == ASYMSPEC_FP32)
-      return stoch ? fuse_verify_tma<float, true> : fuse_verify_tma<float, false>;
-    return stoch ? fuse_verify_tma<__nv_bfloat16, true> : fuse_verify_tma<__nv_bfloat16, false>;
-  }
-  if (dtype == ASYMSPEC_FP32) {
-    if (pl.vector_path)
-      return stoch ? fuse_verify_generic<float, 4, true> : fuse_verify_generic<float, 4, false>;
-    return stoch ? fuse_verify_generic<float, 1, true> : fuse_verify_generic<float, 1, false>;
-  }
-  if (pl.vector_path)
-    return stoch ? fuse_verify_generic<__nv_bfloat16, 8, true>
-                 : fuse_verify_generic<__nv_bfloat16, 8, false>;
-  return stoch ? fuse_verify_generic<__nv_bfloat16, 1, true>
-               : fuse_verify_generic<__nv_bfloat16, 1, false>;
+  if (pl.kernel == ASYMSPEC_KERNEL_TMA)
+    return dtype == ASYMSPEC_FP32 ? tma_kernel_f32(stoch) : tma_kernel_bf16(stoch);
+  return generic_kernel(dtype, pl.vector_path, stoch);
 }
 
 // Per (kernel, device): attributes set once; cluster occupancy cached per
@@ -156,7 +216,7 @@ int g_occ_count = 0;
 
 cudaError_t prepare_kernel(KernelFn fn, int device) {
   std::lock_guard<std::mutex> lock(g_mu);
-  const void* f = reinterpret_cast<const void*>(fn);
+  const void* f = fn;
   for (int i = 0; i < g_attr_count; ++i)
     if (g_attr_done[i].fn == f && g_attr_done[i].device == device) return cudaSuccess;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
@@ -185,7 +245,7 @@ cudaLaunchConfig_t launch_config(const Plan& pl, long long ctas, cudaStream_t st
 
 // Clusters of this shape the device holds at once (0 if it cannot).
 cudaError_t active_clusters(KernelFn fn, const Plan& pl, int device, int* out) {
-  const void* f = reinterpret_cast<const void*>(fn);
+  const void* f = fn;
   {
     std::lock_guard<std::mutex> lock(g_mu);
     for (int i = 0; i < g_occ_count; ++i)
@@ -206,13 +266,66 @@ cudaError_t active_clusters(KernelFn fn, const Plan& pl, int device, int* out) {
   return cudaSuccess;
 }
 
-bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+using StreamFn = const void*;  // fuse_verify_stream<T, STOCH>
 
-size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
-
-size_t ws_records_bytes(int B, int K) {
-  return round_up(static_cast<size_t>(B) * (K + 1) * sizeof(int4), 256);
+StreamFn pick_stream(int dtype, bool stoch) {
+  if (dtype == ASYMSPEC_FP32) return stoch ? stream_kernel_f32_stoch() : stream_kernel_f32_greedy();
+  return stoch ? stream_kernel_bf16_stoch() : stream_kernel_bf16_greedy();
 }
+
+// Resident CTAs of a streaming kernel on a device (cached): the persistent
+// grid, all of whose CTAs must run at once.
+struct GridEntry {
+  const void* fn;
+  int device, grid;
+};
+GridEntry g_grid[16];
+int g_grid_count = 0;
+
+cudaError_t stream_grid(StreamFn fn, int device, int* out) {
+  const void* f = fn;
+  {
+    std::lock_guard<std::mutex> lock(g_mu);
+    for (int i = 0; i < g_grid_count; ++i)
+      if (g_grid[i].fn == f && g_grid[i].device == device) {
+        *out = g_grid[i].grid;
+        return cudaSuccess;
+      }
+  }
+  int per_sm = 0, sms = 0;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
+  if (e != cudaSuccess) return e;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kSThreads, kRingBytes);
+  if (e != cudaSuccess) return e;
+  e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+  if (e != cudaSuccess) return e;
+  const int grid = per_sm * sms;
+  std::lock_guard<std::mutex> lock(g_mu);
+  if (g_grid_count < 16) g_grid[g_grid_count++] = {f, device, grid};
+  *out = grid;
+  return cudaSuccess;
+}
+
+// The row programs of the streaming kernel: [0] draft rows, [1] the bonus row.
+void stream_programs(const asymspec_gate_params& gp, bool full, bool logprobs, bool tokens,
+                     int (&prog)[2]) {
+  const bool jsd = gp.divergence == ASYMSPEC_DIV_JSD;
+  const bool kl = gp.divergence == ASYMSPEC_DIV_KL;
+  if (full) {
+    int p = jsd ? PG_FULL_JSD : kl ? PG_FULL_KL : PG_FULL_NONE;
+    if (logprobs) p += PG_FULL_JSD_LP - PG_FULL_JSD;
+    prog[0] = prog[1] = p;
+  } else if (gp.mode == ASYMSPEC_MODE_GREEDY) {
+    prog[0] = jsd ? PG_GREEDY_DRAFT_JSD : kl ? PG_GREEDY_DRAFT_KL : PG_GREEDY_DRAFT_NONE;
+    prog[1] = gp.fuse_bonus ? PG_GREEDY_BONUS_S : PG_GREEDY_BONUS_T;
+  } else {
+    const int base = jsd ? PG_STOCH_DRAFT_JSD : kl ? PG_STOCH_DRAFT_KL : PG_STOCH_DRAFT_NONE;
+    prog[0] = tokens ? base + (PG_STOCH_DRAFT_JSD_TOK - PG_STOCH_DRAFT_JSD) : base;
+    prog[1] = tokens ? PG_STOCH_BONUS_TOK : PG_STOCH_BONUS;
+  }
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 int check_params(const asymspec_gate_params* gp) {
   if (!(gp->gamma > 0.f && gp->gamma <= 1.f)) return ASYMSPEC_ERR_INVALID_ARG;
@@ -280,9 +393,16 @@ void asymspec_default_gate_params(asymspec_gate_params* p) {
 }
 
 size_t asymspec_workspace_bytes(int B, int K, int V) {
-  (void)V;
   if (B < 1 || K < 1) return 0;
-  return ws_records_bytes(B, K) + round_up(static_cast<size_t>(B) * sizeof(unsigned), 256);
+  size_t n = cluster_ws_bytes(B, K);
+  if (V >= 2) {
+    // the larger of the two dtypes' streaming layouts (fp32 has more tiles)
+    const StreamLayout L4 = stream_layout(B, K, V, 4);
+    if (L4.NT <= kMaxStreamTiles) n = std::max(n, L4.total);
+    const StreamLayout L2 = stream_layout(B, K, V, 2);
+    if (L2.NT <= kMaxStreamTiles) n = std::max(n, L2.total);
+  }
+  return n;
 }
 
 int asymspec_workspace_reset(void* workspace, size_t workspace_bytes, void* stream) {
@@ -305,8 +425,28 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
   if (st) return st;
   const bool vec_ok = (static_cast<long long>(V) * elt_size(dtype)) % 16 == 0;
   Plan pl;
-  st = make_plan(B, K, V, dtype, gp.mode == ASYMSPEC_MODE_STOCHASTIC, opts, vec_ok, &pl);
+  st = make_plan(B, K, V, dtype, gp.mode == ASYMSPEC_MODE_STOCHASTIC, opts, vec_ok,
+                 asymspec_workspace_bytes(B, K, V), &pl);
   if (st) return st;
+  if (pl.kernel == ASYMSPEC_KERNEL_STREAM) {
+    out->cluster_size = 1;
+    out->block_threads = kSThreads;
+    out->slice_elems = pl.W;
+    out->smem_bytes = kRingBytes;
+    out->ctas = 0;
+    out->vector_path = 1;
+    out->max_active_clusters = 0;
+    out->kernel = pl.kernel;
+    int device = 0, grid = 0;
+    if (cudaGetDevice(&device) == cudaSuccess &&
+        stream_grid(pick_stream(dtype, gp.mode == ASYMSPEC_MODE_STOCHASTIC), device, &grid) ==
+            cudaSuccess) {
+      out->ctas = grid;
+      out->max_active_clusters = grid;
+    }
+    cudaGetLastError();
+    return ASYMSPEC_OK;
+  }
   out->cluster_size = pl.C;
   out->block_threads = pl.kernel == ASYMSPEC_KERNEL_TMA ? kTThreads : kThreads;
   out->slice_elems = pl.W;
@@ -359,13 +499,11 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
       (out_fused_logprobs && !aligned(out_fused_logprobs, 4)) ||
       (out_error_word && !aligned(out_error_word, 4)))
     return ASYMSPEC_ERR_MISALIGNED;
-  if (!workspace || workspace_bytes < asymspec_workspace_bytes(B, K, V) ||
-      !aligned(workspace, 16))
-    return ASYMSPEC_ERR_WORKSPACE;
+  if (!workspace || !aligned(workspace, 16)) return ASYMSPEC_ERR_WORKSPACE;
   const bool vec_ok = (static_cast<long long>(V) * elt) % 16 == 0 && aligned(logits_full, 16) &&
                       aligned(logits_comp, 16) && aligned(logits_ver, 16);
   Plan pl;
-  st = make_plan(B, K, V, dtype, stoch, opts, vec_ok, &pl);
+  st = make_plan(B, K, V, dtype, stoch, opts, vec_ok, workspace_bytes, &pl);
   if (st) return st;
 
   KParams P;
@@ -408,12 +546,65 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   int device = 0;
   cudaError_t e = cudaGetDevice(&device);
   if (e != cudaSuccess) return cuda_fail(e);
+  if (pl.kernel == ASYMSPEC_KERNEL_STREAM) {
+    const StreamLayout L = stream_layout(B, K, V, elt);
+    char* base = static_cast<char*>(workspace);
+    SParams S;
+    S.P = P;
+    S.ws.recs = reinterpret_cast<int4*>(base);
+    S.ws.tickets = reinterpret_cast<unsigned*>(base + L.tickets);
+    S.ws.p1cnt = reinterpret_cast<unsigned*>(base + L.p1cnt);
+    S.ws.p2cnt = reinterpret_cast<unsigned*>(base + L.p2cnt);
+    S.ws.ready = reinterpret_cast<unsigned*>(base + L.ready);
+    S.ws.tags = reinterpret_cast<unsigned long long*>(base + L.tags);
+    S.ws.stat = reinterpret_cast<RowStat*>(base + L.stat);
+    S.ws.p1rec = reinterpret_cast<X1*>(base + L.p1rec);
+    S.ws.p2rec = reinterpret_cast<X2*>(base + L.p2rec);
+    S.ws.groups = reinterpret_cast<float*>(base + L.groups);
+    S.P.recs = S.ws.recs;
+    S.P.tickets = S.ws.tickets;
+    S.NT = L.NT;
+    S.TS = L.TS;
+    StreamFn fn = pick_stream(dtype, stoch);
+    int grid = 0;
+    e = stream_grid(fn, device, &grid);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (grid < 1) return ASYMSPEC_ERR_UNSUPPORTED;
+    // pass 2 of row r follows pass 1 of row r + D: D covers 1.5 waves of the grid
+    const long long R = pl.rows;
+    const long long per_step = 2ll * L.NT;
+    long long D = (3ll * grid + 2 * per_step - 1) / (2 * per_step);
+    D = std::max(2ll, std::min(D, R));
+    S.D = static_cast<int>(D);
+    S.NI = (R + D) * per_step;
+    stream_programs(gp, P.full != 0, out_fused_logprobs != nullptr, out_row_tokens != nullptr,
+                    S.program);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(kSThreads);
+    cfg.dynamicSmemBytes = kRingBytes;
+    cfg.stream = static_cast<cudaStream_t>(stream);
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    void* args[] = {&S};
+    e = cudaLaunchKernelExC(&cfg, fn, args);
+    if (e != cudaSuccess) return cuda_fail(e);
+    return ASYMSPEC_OK;
+  }
   KernelFn fn = pick_kernel(pl, dtype, stoch);
   e = prepare_kernel(fn, device);
   if (e != cudaSuccess) return cuda_fail(e);
+  // One cluster per row: measured faster than a persistent grid of clusters
+  // looping over rows (the kernel supports both), whose row-finishing work
+  // lands on the cluster's critical path.
+  const long long ctas = pl.ctas;
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = launch_config(pl, pl.ctas, static_cast<cudaStream_t>(stream), attr);
-  e = cudaLaunchKernelEx(&cfg, fn, P);
+  cudaLaunchConfig_t cfg = launch_config(pl, ctas, static_cast<cudaStream_t>(stream), attr);
+  void* args[] = {&P};
+  e = cudaLaunchKernelExC(&cfg, fn, args);
   if (e != cudaSuccess) return cuda_fail(e);
   return ASYMSPEC_OK;
 }

@@ -356,6 +356,21 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, unsigned b
       : "memory");
 }
 
+// As bulk_load, with an L2 cache policy (createpolicy) for the source lines.
+__device__ __forceinline__ void bulk_load_hint(void* dst, const void* src, unsigned bytes,
+                                               unsigned long long* bar, unsigned long long pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint "
+      "[%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(pol)
+      : "memory");
+}
+
+// Plain arrive (one count) on an mbarrier of this CTA.
+__device__ __forceinline__ void mbar_arrive(unsigned long long* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 struct KParams {
   const void* a;
   const void* b;
@@ -399,15 +414,32 @@ struct RowResult {
   bool have_lse_t;                   // lse_t was computed (greedy bonus rows may skip it)
 };
 
-// Runs on one thread per row (rank 0, thread 0) once the row is complete:
-// the acceptance test of Eq. 4 (or its stochastic counterpart), the optional
-// per-row outputs, the 16-byte row record and the batch element's ticket.
-// The last row of a batch element to arrive runs Algorithm 1's scan.
+// The stochastic inputs of one row: the drafter's probability of the draft
+// token, the uniform of its test, and the element's one non-draft uniform.
+struct RowScalars {
+  float dprob, u, u_last;
+};
+
+__device__ __forceinline__ RowScalars load_row_scalars(const KParams& P, int bi, int k) {
+  RowScalars sc{0.f, 0.f, 0.f};
+  const int K1 = P.K + 1;
+  sc.u_last = P.unif[static_cast<size_t>(bi) * K1 + P.K];
+  if (k < P.K) {
+    sc.dprob = P.dprobs[static_cast<size_t>(bi) * P.K + k];
+    sc.u = P.unif[static_cast<size_t>(bi) * K1 + k];
+  }
+  return sc;
+}
+
+// The decision of one complete row, on one thread: data checks, the
+// acceptance test of Eq. 4 (or its stochastic counterpart), the emitted
+// candidate, and the optional per-row outputs.  Returns the 16-byte row
+// record (accept bit, candidate, ASYMSPEC_DATA_* bits).
 // dtok/ad/bd/td: the draft token of this row and its three logits.
 template <bool STOCH>
-__device__ void finish_row(const KParams& P, long long row, int bi, int k, const RowResult& r,
-                           int dtok, float ad, float bd, float td) {
-  const int V = P.V, K = P.K, K1 = K + 1;
+__device__ int4 row_record(const KParams& P, long long row, int k, const RowResult& r, int dtok,
+                           float ad, float bd, float td, const RowScalars& sc) {
+  const int V = P.V, K = P.K;
   const bool bonus = (k == K);
   unsigned err = 0;
   if (r.bad & kBadTimeout) err |= ASYMSPEC_DATA_TIMEOUT;
@@ -432,11 +464,7 @@ __device__ void finish_row(const KParams& P, long long row, int bi, int k, const
   }
   if (P.divergence == ASYMSPEC_DIV_JSD) D = fminf(fmaxf(D, 0.f), kLn2);
   if (P.divergence == ASYMSPEC_DIV_KL) D = fmaxf(D, 0.f);
-  float u_last = 0.f;
-  if (STOCH) {
-    u_last = P.unif[static_cast<size_t>(bi) * K1 + K];
-    if (!(u_last >= 0.f && u_last < 1.f)) err |= ASYMSPEC_DATA_BAD_UNIFORM;
-  }
+  if (STOCH && !(sc.u_last >= 0.f && sc.u_last < 1.f)) err |= ASYMSPEC_DATA_BAD_UNIFORM;
   int accept = 1;
   float margin = NAN;
   float gamma_eff = P.gamma;
@@ -453,8 +481,7 @@ __device__ void finish_row(const KParams& P, long long row, int bi, int k, const
         accept = lr > ln_geff;                   // Eq. 4
         margin = 1.f - expf(lr - ln_geff);
       } else {
-        const float pd = P.dprobs[static_cast<size_t>(bi) * K + k];
-        const float u = P.unif[static_cast<size_t>(bi) * K1 + k];
+        const float pd = sc.dprob, u = sc.u;
         if (!(pd > 0.f && pd <= 1.f)) err |= ASYMSPEC_DATA_BAD_PROB;
         if (!(u >= 0.f && u < 1.f)) err |= ASYMSPEC_DATA_BAD_UNIFORM;
         const float sd = fmaf(P.beta, ad - bd, td);
@@ -489,7 +516,18 @@ __device__ void finish_row(const KParams& P, long long row, int bi, int k, const
     P.row_tokens[static_cast<size_t>(row) * 2 + 1] = cand;
   }
   if (err && P.err_word) atomicOr(P.err_word, err);
-  P.recs[row] = make_int4(accept, cand, static_cast<int>(err), 0);
+  return make_int4(accept, cand, static_cast<int>(err), 0);
+}
+
+// Runs on one thread per row once the row is complete: the row record and
+// the batch element's ticket.  The last row of a batch element to arrive
+// runs Algorithm 1's scan.
+template <bool STOCH>
+__device__ void finish_row(const KParams& P, long long row, int bi, int k, const RowResult& r,
+                           int dtok, float ad, float bd, float td) {
+  const int K = P.K, K1 = K + 1;
+  const RowScalars sc = STOCH ? load_row_scalars(P, bi, k) : RowScalars{0.f, 0.f, 0.f};
+  P.recs[row] = row_record<STOCH>(P, row, k, r, dtok, ad, bd, td, sc);
   __threadfence();
   const unsigned ticket = atomicAdd(&P.tickets[bi], 1u);
   if (ticket != static_cast<unsigned>(K)) return;
@@ -510,6 +548,54 @@ __device__ void finish_row(const KParams& P, long long row, int bi, int k, const
   P.out_len[bi] = any_err ? -1 : len;
   P.out_next[bi] = any_err ? -1 : next;
   P.tickets[bi] = 0u;
+}
+
+__device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
+  unsigned old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v)
+               : "memory");
+  return old;
+}
+
+// As finish_row, executed by a whole warp (lane 0 decides the row).  The
+// ticket's read-modify-write has acquire-release semantics, which orders this
+// row's record before it and every other row's record after it; the last
+// row reads the K+1 records 32 at a time, one per lane, and takes Algorithm
+// 1's first rejection with a ballot.
+template <bool STOCH>
+__device__ void finish_row_warp(const KParams& P, long long row, int bi, int k,
+                                const RowResult& r, int dtok, float ad, float bd, float td,
+                                const RowScalars& sc) {
+  const int lane = threadIdx.x & 31;
+  const int K = P.K, K1 = K + 1;
+  unsigned ticket = 0;
+  if (lane == 0) {
+    P.recs[row] = row_record<STOCH>(P, row, k, r, dtok, ad, bd, td, sc);
+    ticket = atom_add_acq_rel(&P.tickets[bi], 1u);
+  }
+  ticket = __shfl_sync(0xffffffffu, ticket, 0);
+  if (ticket != static_cast<unsigned>(K)) return;
+  __syncwarp();
+  const int4* recs = P.recs + static_cast<size_t>(bi) * K1;
+  bool any_err = false;
+  int len = -1, next = -1;
+  for (int base = 0; base < K1; base += 32) {
+    const int j = base + lane;
+    int4 v = make_int4(1, -1, 0, 0);
+    if (j < K1) v = __ldcg(&recs[j]);
+    any_err |= __any_sync(0xffffffffu, v.z != 0);
+    if (len < 0) {
+      const unsigned rej = __ballot_sync(0xffffffffu, j < K && v.x == 0);
+      if (rej) len = base + __ffs(rej) - 1;
+      else if (K < base + 32) len = K;
+      if (len >= 0) next = __shfl_sync(0xffffffffu, v.y, len - base);
+    }
+  }
+  if (lane == 0) {
+    P.out_len[bi] = any_err ? -1 : len;
+    P.out_next[bi] = any_err ? -1 : next;
+    P.tickets[bi] = 0u;
+  }
 }
 
 // The draft token of row (bi, k) and its three logits (rank 0, thread 0).

@@ -1,0 +1,12 @@
+// Instantiations of the cluster TMA kernel for __nv_bfloat16 logits (see kernel_tma.cuh).
+#include "kernel_tma.cuh"
+#include "kernels.h"
+
+namespace asymspec_impl {
+
+const void* tma_kernel_bf16(bool stoch) {
+  return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, true>)
+               : reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, false>);
+}
+
+}  // namespace asymspec_impl

@@ -1,0 +1,12 @@
+// Instantiations of the cluster TMA kernel for float logits (see kernel_tma.cuh).
+#include "kernel_tma.cuh"
+#include "kernels.h"
+
+namespace asymspec_impl {
+
+const void* tma_kernel_f32(bool stoch) {
+  return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<float, true>)
+               : reinterpret_cast<const void*>(&fuse_verify_tma<float, false>);
+}
+
+}  // namespace asymspec_impl

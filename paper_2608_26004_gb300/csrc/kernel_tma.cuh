@@ -20,21 +20,26 @@
 // full program.  Two fp32 values travel per add/sub/mul/fma instruction
 // (f32x2); exponentials and logarithms use ex2.approx / lg2.approx.
 //
-// Reductions: per stream, the maximum first (warp shuffles), then each lane
-// rescales its own sum once and the sums are added; warp -> CTA in shared
-// memory.  Each CTA then pushes its record into every peer's shared memory
+// Normalisers: each thread sums 2^((x - ref) log2 e) against one fixed
+// reference per stream, the maximum of its first vector, so an entry costs
+// one FMA, one ex2 and one add; partial sums are rescaled only where they
+// meet (warp, CTA, cluster).  A thread whose sum reaches 2^100 (an entry
+// more than ~69 nats above its reference, or non-finite data) makes the CTA
+// redo its slice with a running maximum (pass1_online).
+//
+// Reductions: warp maxima with redux.sync, sums with shuffles; warp -> CTA in
+// shared memory.  Each CTA pushes its record into every peer's shared memory
 // (DSMEM stores) before a cluster barrier, so after the barrier every CTA
-// combines local copies, identically, and holds bit-identical row values;
-// nothing is read remotely after a barrier, so CTAs may leave as soon as
-// they are done.  Two barriers per row (one when no pass 2 is needed); the
-// stochastic draw reaches rank 0 through a remote mbarrier arrive.  The draft
-// token's three logits come from the shared memory of the CTA whose slice
-// holds it.
+// combines local copies, identically.  Two cluster barriers per row (one
+// when no pass 2 is needed).  Once the last barrier has passed, only the
+// warp that finishes the row stays: warp 0 of rank 0 (greedy), or warp 0 of
+// the CTA whose slice holds the inverse-CDF target (stochastic), which walks
+// its slice and then decides the row itself.
 //
 // Every wait is bounded: a chunk that does not land within 200 ms marks the
 // row with ASYMSPEC_DATA_TIMEOUT; the CTA still reaches every cluster
-// barrier, so no CTA of the cluster is left waiting, and before it exits it
-// waits (bounded again) for any copy still in flight.
+// barrier, so no CTA of the cluster is left waiting, and before it exits
+// thread 0 waits (bounded again) for any copy still in flight.
 #pragma once
 
 #include "device_common.cuh"
@@ -46,12 +51,15 @@ constexpr int kTWarps = kTThreads / 32;
 constexpr int kMaxRounds = 10;  // 16-byte vectors per thread per slice
 constexpr int kChunks = 4;      // bulk-copy chunks per slice
 constexpr unsigned long long kCopyTimeoutNs = 200ull * 1000ull * 1000ull;
+constexpr float kSumLimit = 1.2676506e30f;  // 2^100: pass1_fast's overflow guard
 
 enum : unsigned { F_LA = 1, F_LB = 2, F_LT = 4, F_LS = 8, F_AS = 16, F_AT = 32 };
 enum : unsigned { G_JSD = 1, G_KL = 2, G_RES = 4, G_QF = 8 };
 
-struct __align__(16) X1 {  // pass-1 result (per thread, per warp, per CTA, per row)
-  float m[4];
+// Pass-1 result (per thread, per warp, per CTA, per row).  Stream q's
+// normaliser is ref[q] + ln s[q]: s[q] sums 2^((x - ref[q]) log2 e).
+struct __align__(16) X1 {
+  float ref[4];
   float s[4];
   float vs;
   int is;
@@ -69,24 +77,17 @@ struct __align__(16) X2 {  // pass-2 sums
 // Fixed part of the shared state; the C pass-1 and C pass-2 records pushed
 // by the cluster follow it (recv1(), recv2()).
 struct __align__(16) SharedTma {
-  unsigned long long bar[kChunks];   // one mbarrier per chunk
-  unsigned long long sample_bar;     // rank 0: the draw has arrived
-  union {                            // per-warp scratch, one use at a time
+  unsigned long long bar[kChunks];  // one mbarrier per chunk
+  union {                           // per-warp records, one pass at a time
     X1 w1[kTWarps];
     X2 w2[kTWarps];
-    float wr[kMaxRounds][kTWarps];
   };
   float lse[4];
   int is, it;
   unsigned bad;
   float da, db, dt;
-  float D, mass_total, tau_local;
-  int owner, use_r;
-  int sample;  // rank 0: written by the CTA that owns the draw
-  int found, jstar;
-  float tau_j;
-  float scan[kTWarps];
   unsigned broken;
+  unsigned pad[3];
   __device__ X1* recv1() { return reinterpret_cast<X1*>(this + 1); }
   __device__ X2* recv2(int C) { return reinterpret_cast<X2*>(recv1() + C); }
 };
@@ -109,7 +110,7 @@ __device__ __forceinline__ X1 x1_neutral() {
   X1 r;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    r.m[q] = -INFINITY;
+    r.ref[q] = -INFINITY;
     r.s[q] = 0.f;
   }
   r.vs = -INFINITY;
@@ -128,10 +129,11 @@ __device__ __forceinline__ X2 x2_zero() {
   return r;
 }
 
+// Warp maximum (NaN ignored unless every lane holds NaN).
 __device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
-  return v;
+  float r;
+  asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
+  return r;
 }
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -140,30 +142,27 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// Larger value wins, the lowest index among equal values; NaN never wins.
 __device__ __forceinline__ void warp_argmax(float& v, int& i) {
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    const float v2 = __shfl_xor_sync(0xffffffffu, v, off);
-    const int i2 = __shfl_xor_sync(0xffffffffu, i, off);
-    if (v2 > v || (v2 == v && i2 < i)) {
-      v = v2;
-      i = i2;
-    }
-  }
+  const float m = warp_max(v);
+  const int cand = (v == m) ? i : INT_MAX;
+  i = __reduce_min_sync(0xffffffffu, cand);
+  v = m;
 }
 
-// Warp-wide combine of the streams a program computes: the maximum first,
-// then every lane rescales its own sum to it and the sums are added.  Every
-// lane ends with the same (bit-identical) result.
+// Warp-wide combine of the streams a program computes: the largest
+// reference, every lane's sum rescaled to it, the sums added.  Every lane
+// ends with the same (bit-identical) result.  A NaN sum stays NaN.
 template <unsigned F>
 __device__ __forceinline__ void warp_reduce_x1(X1& e) {
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const unsigned bit = q == 0 ? F_LA : q == 1 ? F_LB : q == 2 ? F_LT : F_LS;
     if (F & bit) {
-      const float M = warp_max(e.m[q]);
-      const float s = (e.m[q] == M) ? e.s[q] : e.s[q] * ex2((e.m[q] - M) * kLog2e);
-      e.m[q] = M;
+      const float M = warp_max(e.ref[q]);
+      const float s = (e.s[q] == 0.f || e.ref[q] == M) ? e.s[q]
+                                                       : e.s[q] * ex2((e.ref[q] - M) * kLog2e);
+      e.ref[q] = M;
       e.s[q] = warp_sum(s);
     }
   }
@@ -183,7 +182,7 @@ __device__ __forceinline__ void cluster_barrier(bool released) {
 }
 
 // The record of this CTA goes into slot `rank` of every CTA of the cluster
-// (lane r of warp 0 writes to CTA r); a cluster barrier must follow.
+// (lane r of the calling warp writes to CTA r); a cluster barrier must follow.
 template <typename R>
 __device__ __forceinline__ void push_record(const R& rec, R* slots, int rank, int C,
                                             cg::cluster_group& cluster) {
@@ -315,11 +314,12 @@ __device__ __forceinline__ void load_or_fill(const T* p, bool ok, f2 (&x)[NP]) {
   }
 }
 
-// Vector i of the slice lives in round i / NT; chunk c holds rounds
-// [c rc, (c+1) rc).  Every thread waits for a chunk before its first round.
-// Rounds are taken two at a time.
+// Pass 1 with a running maximum per stream (one rescale check per two
+// vectors): the fallback for slices where pass1_fast's fixed reference
+// overflows.  Vector i of the slice lives in round i / NT; chunk c holds
+// rounds [c rc, (c+1) rc).  Rounds are taken two at a time.
 template <typename T, unsigned F>
-__device__ __forceinline__ void pass1(const T* ra, const T* rb, const T* rt, int nv, int rounds,
+__device__ __noinline__ void pass1_online(const T* ra, const T* rb, const T* rt, int nv, int rounds,
                                       int rc, int lo, float beta, SharedTma* sh, X1& e) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
@@ -363,11 +363,11 @@ __device__ __forceinline__ void pass1(const T* ra, const T* rb, const T* rt, int
           ys[h] = fma2(beta2, sub2(ya[h], yb[h]), yt[h]);
         }
       }
-      if (F & F_LA) online_pairs2(e.m[0], acc[0], xa, ya, L2);
-      if (F & F_LB) online_pairs2(e.m[1], acc[1], xb, yb, L2);
+      if (F & F_LA) online_pairs2(e.ref[0], acc[0], xa, ya, L2);
+      if (F & F_LB) online_pairs2(e.ref[1], acc[1], xb, yb, L2);
       float ct0 = 0.f, ct1 = 0.f, cs0 = 0.f, cs1 = 0.f;
       if (F & F_LT) {
-        online_pairs2(e.m[2], acc[2], xt, yt, L2);
+        online_pairs2(e.ref[2], acc[2], xt, yt, L2);
         if (F & F_AT) {
           ct0 = vmax_pairs(xt);
           ct1 = vmax_pairs(yt);
@@ -377,7 +377,7 @@ __device__ __forceinline__ void pass1(const T* ra, const T* rb, const T* rt, int
         ct1 = vmax_pairs_nan(yt);
       }
       if (F & F_LS) {
-        online_pairs2(e.m[3], acc[3], xs, ys, L2);
+        online_pairs2(e.ref[3], acc[3], xs, ys, L2);
         if (F & F_AS) {
           cs0 = vmax_pairs(xs);
           cs1 = vmax_pairs(ys);
@@ -415,19 +415,163 @@ __device__ __forceinline__ void pass1(const T* ra, const T* rb, const T* rt, int
   }
 }
 
-// Pass 1, block combine, push to the cluster, barrier, local combine; leaves
-// the row values in sh.  dtok: the row's draft token (-1 if none).
+// Adds two vectors of pairs to a packed sum of 2^((x - ref) log2 e), with
+// nm2 = -ref log2 e in both halves.
+template <int NP>
+__device__ __forceinline__ void fixed_pairs2(f2& acc, const f2 (&x)[NP], const f2 (&y)[NP], f2 L2,
+                                             f2 nm2) {
+  f2 e[NP];
+#pragma unroll
+  for (int h = 0; h < NP; ++h)
+    e[h] = add2(ex2_2(fma2(x[h], L2, nm2)), ex2_2(fma2(y[h], L2, nm2)));
+  if constexpr (NP == 4) {
+    acc = add2(acc, add2(add2(e[0], e[1]), add2(e[2], e[3])));
+  } else {
+    acc = add2(acc, add2(e[0], e[1]));
+  }
+}
+
+// Pass 1 against fixed references: every thread takes the maximum of its
+// first vector (vector tid, in chunk 0) as the reference of each normaliser
+// stream.  Returns true when one of this thread's sums reached 2^100 or is not
+// finite (the caller then redoes the slice with pass1_online).  Argmax
+// streams are tracked per vector as in pass1_online.
 template <typename T, unsigned F>
-__device__ __forceinline__ void pass1_and_combine(const T* ra, const T* rb, const T* rt, int nv,
-                                                  int rounds, int rc, int lo, int n, int W,
-                                                  float beta, int dtok, SharedTma* sh, int rank,
-                                                  int C, cg::cluster_group& cluster) {
+__device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt, int nv,
+                                           int rounds, int rc, int lo, float beta, SharedTma* sh,
+                                           X1& e) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  constexpr int NP = VE / 2;
+  constexpr bool needA = (F & (F_LA | F_LS | F_AS)) != 0;
+  constexpr bool needB = (F & (F_LB | F_LS | F_AS)) != 0;
+  constexpr bool needT = (F & (F_LT | F_LS | F_AS | F_AT)) != 0;
+  constexpr bool needS = (F & (F_LS | F_AS)) != 0;
+  constexpr int STEP = 2 * kTThreads * VE;  // elements per two rounds
+  const f2 beta2 = pk(beta, beta);
+  const f2 L2 = pk(kLog2e, kLog2e);
+  const int tid = static_cast<int>(threadIdx.x);
+  // chunk 0 holds every thread's first vector
+  if (!sh->broken && !mbar_wait_bounded(&sh->bar[0], 0, kCopyTimeoutNs))
+    atomicOr(&sh->broken, kBadTimeout);
+  float ref[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+  if (tid < nv) {
+    f2 xa[NP], xb[NP], xt[NP], xs[NP];
+    if (needA) load_pairs(ra + tid * VE, xa);
+    if (needB) load_pairs(rb + tid * VE, xb);
+    if (needT) load_pairs(rt + tid * VE, xt);
+    if (F & F_LA) ref[0] = vmax_pairs(xa);
+    if (F & F_LB) ref[1] = vmax_pairs(xb);
+    if (F & F_LT) ref[2] = vmax_pairs(xt);
+    if (F & F_LS) {
+#pragma unroll
+      for (int h = 0; h < NP; ++h) xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
+      ref[3] = vmax_pairs(xs);
+    }
+  }
+  f2 nm[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float v = -ref[q] * kLog2e;
+    nm[q] = pk(v, v);
+  }
+  f2 acc[4] = {0ull, 0ull, 0ull, 0ull};
+  int vec_s = -1, vec_t = -1;  // vectors holding the best s and t so far
+  for (int c = 0, r0 = 0; c < kChunks && r0 < rounds; ++c, r0 += rc) {
+    if (c > 0 && !sh->broken && !mbar_wait_bounded(&sh->bar[c], 0, kCopyTimeoutNs))
+      atomicOr(&sh->broken, kBadTimeout);
+    const int r1 = min(rounds, r0 + rc);
+    int i0 = r0 * kTThreads + tid;          // vector index of this thread's first vector
+    int e0 = i0 * VE;                       // its element offset in the slice
+    for (int kr = r0; kr < r1; kr += 2, i0 += 2 * kTThreads, e0 += STEP) {
+      if (i0 >= nv) break;
+      const bool has1 = (kr + 1 < r1) && (i0 + kTThreads < nv);
+      const int e1 = e0 + kTThreads * VE;
+      f2 xa[NP], xb[NP], xt[NP], xs[NP], ya[NP], yb[NP], yt[NP], ys[NP];
+      if (needA) {
+        load_pairs(ra + e0, xa);
+        load_or_fill(ra + e1, has1, ya);
+      }
+      if (needB) {
+        load_pairs(rb + e0, xb);
+        load_or_fill(rb + e1, has1, yb);
+      }
+      if (needT) {
+        load_pairs(rt + e0, xt);
+        load_or_fill(rt + e1, has1, yt);
+      }
+      if (needS) {
+#pragma unroll
+        for (int h = 0; h < NP; ++h) {
+          xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
+          ys[h] = fma2(beta2, sub2(ya[h], yb[h]), yt[h]);
+        }
+      }
+      if (F & F_LA) fixed_pairs2(acc[0], xa, ya, L2, nm[0]);
+      if (F & F_LB) fixed_pairs2(acc[1], xb, yb, L2, nm[1]);
+      if (F & F_LT) fixed_pairs2(acc[2], xt, yt, L2, nm[2]);
+      if (F & F_LS) fixed_pairs2(acc[3], xs, ys, L2, nm[3]);
+      if (F & F_AS) {
+        const float cs0 = (F & F_LS) ? vmax_pairs(xs) : vmax_pairs_nan(xs);
+        const float cs1 = (F & F_LS) ? vmax_pairs(ys) : vmax_pairs_nan(ys);
+        arg_track(e.vs, vec_s, cs0, i0, e.bad, kBadS);
+        if (has1) arg_track(e.vs, vec_s, cs1, i0 + kTThreads, e.bad, kBadS);
+      }
+      if (F & F_AT) {
+        const float ct0 = (F & F_LT) ? vmax_pairs(xt) : vmax_pairs_nan(xt);
+        const float ct1 = (F & F_LT) ? vmax_pairs(yt) : vmax_pairs_nan(yt);
+        arg_track(e.vt, vec_t, ct0, i0, e.bad, kBadT);
+        if (has1) arg_track(e.vt, vec_t, ct1, i0 + kTThreads, e.bad, kBadT);
+      }
+    }
+  }
+  bool ovf = false;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const unsigned bit = q == 0 ? F_LA : q == 1 ? F_LB : q == 2 ? F_LT : F_LS;
+    e.ref[q] = ref[q];
+    e.s[q] = hsum2(acc[q]);
+    if ((F & bit) && !(e.s[q] < kSumLimit)) ovf = true;
+  }
+  // the element of the best vector (re-read once from shared memory)
+  if ((F & F_AS) && vec_s >= 0) {
+    f2 xa[NP], xb[NP], xt[NP], xs[NP];
+    load_pairs(ra + vec_s * VE, xa);
+    load_pairs(rb + vec_s * VE, xb);
+    load_pairs(rt + vec_s * VE, xt);
+#pragma unroll
+    for (int h = 0; h < NP; ++h) xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
+    e.is = arg_in_vector(xs, e.vs, lo + vec_s * VE);
+  }
+  if ((F & F_AT) && vec_t >= 0) {
+    f2 xt[NP];
+    load_pairs(rt + vec_t * VE, xt);
+    e.it = arg_in_vector(xt, e.vt, lo + vec_t * VE);
+  }
+  return ovf;
+}
+
+// Pass 1 and the CTA combine, pushed to every CTA of the cluster, up to and
+// including cluster barrier B1.  dtok: the row's draft token (-1 if none),
+// known to warp 0.
+template <typename T, unsigned F>
+__device__ __forceinline__ void pass1_and_push(const T* ra, const T* rb, const T* rt, int nv,
+                                               int rounds, int rc, int lo, int n, float beta,
+                                               int dtok, SharedTma* sh, int rank, int C,
+                                               cg::cluster_group& cluster) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   X1 e = x1_neutral();
-  pass1<T, F>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
+  const bool ovf = pass1_fast<T, F>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
   warp_reduce_x1<F>(e);
   if (lane == 0) sh->w1[warp] = e;
-  __syncthreads();
+  if (__syncthreads_or(ovf)) {
+    // an entry far above its thread's reference (or non-finite data): redo
+    // the slice with a running maximum
+    e = x1_neutral();
+    pass1_online<T, F>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
+    warp_reduce_x1<F>(e);
+    if (lane == 0) sh->w1[warp] = e;
+    __syncthreads();
+  }
   if (warp == 0) {
     X1 w = (lane < kTWarps) ? sh->w1[lane] : x1_neutral();
     warp_reduce_x1<F>(w);
@@ -440,24 +584,59 @@ __device__ __forceinline__ void pass1_and_combine(const T* ra, const T* rb, cons
     push_record(w, sh->recv1(), rank, C, cluster);
   }
   cluster_barrier(warp == 0);  // B1: every CTA's pass-1 record is in every CTA
-  if (warp == 0) {
-    X1 w = (lane < C) ? sh->recv1()[lane] : x1_neutral();
-    warp_reduce_x1<F>(w);
-    if (lane == 0) {
+}
+
+// Thread 0: the bulk copies of a row's slice into the CTA's buffers, in
+// kChunks chunks, each completing on its own mbarrier.  only_t: copy t alone
+// (a greedy bonus row without fused bonus needs nothing else).
+template <typename T>
+__device__ __forceinline__ void issue_slice(const KParams& P, SharedTma* sh, long long row,
+                                            int lo, int nv, int rc, T* sa, T* sb, T* st,
+                                            bool only_t) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  const size_t off = static_cast<size_t>(row) * P.V + lo;
+  const T* ga = static_cast<const T*>(P.a) + off;
+  const T* gb = static_cast<const T*>(P.b) + off;
+  const T* gt = static_cast<const T*>(P.t) + off;
 #pragma unroll
-      for (int q = 0; q < 4; ++q) sh->lse[q] = w.m[q] + logf(w.s[q]);
-      sh->is = w.is;
-      sh->it = w.it;
-      sh->bad = w.bad;
-      if (dtok >= 0 && W > 0) {
-        const X1& o = sh->recv1()[dtok / W < C ? dtok / W : 0];
-        sh->da = o.da;
-        sh->db = o.db;
-        sh->dt = o.dt;
+  for (int c = 0; c < kChunks; ++c) {
+    const int v0 = min(nv, c * rc * kTThreads);
+    const int v1 = min(nv, (c + 1) * rc * kTThreads);
+    const unsigned bytes = static_cast<unsigned>(v1 - v0) * 16u;
+    mbar_arrive_expect_tx(&sh->bar[c], bytes * (only_t ? 1u : 3u));
+    if (bytes) {
+      const int e0 = v0 * VE;
+      if (!only_t) {
+        bulk_load(sa + e0, ga + e0, bytes, &sh->bar[c]);
+        bulk_load(sb + e0, gb + e0, bytes, &sh->bar[c]);
       }
+      bulk_load(st + e0, gt + e0, bytes, &sh->bar[c]);
     }
   }
-  __syncthreads();
+}
+
+// After B1, in one warp: the row values from the C pushed records (every
+// lane ends with them).  lse[q] = ln of stream q's normaliser.
+template <unsigned F>
+__device__ __forceinline__ X1 combine_pass1(SharedTma* sh, int C, float (&lse)[4]) {
+  const int lane = threadIdx.x & 31;
+  X1 w = (lane < C) ? sh->recv1()[lane] : x1_neutral();
+  warp_reduce_x1<F>(w);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) lse[q] = w.ref[q] + logf(w.s[q]);
+  return w;
+}
+
+// The draft token's a, b, t (from the record of the CTA whose slice holds it).
+__device__ __forceinline__ void draft_logits(SharedTma* sh, int dtok, int W, int C, float& ad,
+                                             float& bd, float& td) {
+  ad = bd = td = 0.f;
+  if (dtok >= 0 && W > 0) {
+    const X1& o = sh->recv1()[dtok / W < C ? dtok / W : 0];
+    ad = o.da;
+    bd = o.db;
+    td = o.dt;
+  }
 }
 
 // ---------------------------------------------------------------- pass 2
@@ -578,14 +757,13 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
   x.Q = hsum2(Q2);
 }
 
-// Pass 2, block combine, push to the cluster, barrier, local combine:
-// divergence, inverse-CDF mass and the CTA that owns the draw.
-template <typename T, unsigned G, bool LP, bool STOCH>
-__device__ __forceinline__ void pass2_and_combine(const T* ra, const T* rb, const T* rt, int nv,
-                                                  int rounds, float beta, float* lp,
-                                                  SharedTma* sh, int rank, int C, bool r_allowed,
-                                                  float u_last, float* vmass,
-                                                  cg::cluster_group& cluster) {
+// Pass 2's per-warp sums, the CTA combine, pushed to every CTA, up to and
+// including cluster barrier B2.
+template <typename T, unsigned G, bool LP>
+__device__ __forceinline__ void pass2_and_push(const T* ra, const T* rb, const T* rt, int nv,
+                                               int rounds, float beta, float* lp, SharedTma* sh,
+                                               int rank, int C, float* vmass,
+                                               cg::cluster_group& cluster) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
   X2 x = x2_zero();
@@ -600,49 +778,14 @@ __device__ __forceinline__ void pass2_and_combine(const T* ra, const T* rb, cons
     push_record(w, sh->recv2(C), rank, C, cluster);
   }
   cluster_barrier(warp == 0);  // B2: every CTA's pass-2 record is in every CTA
-  if (warp == 0) {
-    const X2 w = (lane < C) ? sh->recv2(C)[lane] : x2_zero();
-    X2 tot = w;
-    warp_reduce_x2<G>(tot);
-    float D = 0.f;
-    if (G & G_JSD) D = 0.5f * kLn2 * (tot.j + tot.msum);
-    else if (G & G_KL) D = kLn2 * tot.kl;
-    if (STOCH) {
-      // inclusive prefix of the inverse-CDF mass over ranks, in rank order
-      float incl_R = w.R, incl_Q = w.Q;
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const float vr = __shfl_up_sync(0xffffffffu, incl_R, off);
-        const float vq = __shfl_up_sync(0xffffffffu, incl_Q, off);
-        if (lane >= off) {
-          incl_R += vr;
-          incl_Q += vq;
-        }
-      }
-      const float R_all = __shfl_sync(0xffffffffu, incl_R, 31);
-      const float Q_all = __shfl_sync(0xffffffffu, incl_Q, 31);
-      const bool r_ok = r_allowed && (R_all > 0.f);
-      const float incl = r_ok ? incl_R : incl_Q;
-      const float mass = r_ok ? w.R : w.Q;
-      const float total = r_ok ? R_all : Q_all;
-      const float tau = u_last * total;
-      const unsigned over = __ballot_sync(0xffffffffu, lane < C && incl > tau);
-      const unsigned pos = __ballot_sync(0xffffffffu, lane < C && mass > 0.f);
-      int owner = -1;
-      if (over) owner = __ffs(over) - 1;
-      else if (pos) owner = 31 - __clz(pos);
-      const float incl_o = __shfl_sync(0xffffffffu, incl, owner < 0 ? 0 : owner);
-      const float mass_o = __shfl_sync(0xffffffffu, mass, owner < 0 ? 0 : owner);
-      if (lane == 0) {
-        sh->mass_total = total;
-        sh->use_r = r_ok ? 1 : 0;
-        sh->owner = owner;
-        sh->tau_local = fmaxf(tau - (incl_o - mass_o), 0.f);
-      }
-    }
-    if (lane == 0) sh->D = D;
-  }
-  __syncthreads();
+}
+
+// The divergence of Eq. 3 from the summed pass-2 records (nats).
+template <unsigned G>
+__device__ __forceinline__ float divergence_of(const X2& tot) {
+  if (G & G_JSD) return 0.5f * kLn2 * (tot.j + tot.msum);
+  if (G & G_KL) return kLn2 * tot.kl;
+  return 0.f;
 }
 
 // ---------------------------------------------------------------- inverse-CDF walk
@@ -661,129 +804,297 @@ __device__ __forceinline__ float vec_mass(const T* ra, const T* rb, const T* rt,
   return use_r ? vsum(r) : vsum(qf);
 }
 
-// In the CTA that owns the target: the smallest slice index whose cumulative
-// mass (index order: round, thread, element) exceeds tau_local.  The masses
-// are recomputed here exactly as pass 2 computed them.  Returns the index
-// within the row, or -1.
+// Mass of vector i of the slice as pass 2 left it (stored) or recomputed.
 template <typename T>
-__device__ int walk(SharedTma* sh, const T* ra, const T* rb, const T* rt, int nv, int rounds,
-                    int lo, float beta, const float* vmass, bool stored_r) {
+__device__ __forceinline__ float walk_mass(const T* ra, const T* rb, const T* rt, int i, int nv,
+                                           const float* vmass, int j, int t, bool stored,
+                                           bool use_r, f2 beta2, f2 L2, f2 nA2, f2 nS2) {
+  if (i >= nv) return 0.f;
+  if (stored) return vmass[j * kTThreads + t];
+  return vec_mass(ra, rb, rt, i, use_r, beta2, L2, nA2, nS2);
+}
+
+// The inverse-CDF draw inside the CTA that owns the target, by one warp: the
+// smallest slice index (order: round, thread, element) whose cumulative
+// residual (use_r) or fused mass exceeds tau, or the last index with positive
+// mass when rounding leaves tau at or beyond the slice's total.  Lane l covers
+// the vectors of threads 8l .. 8l+7 in every round.  Returns the index within
+// the row (every lane), or -1 when the slice holds no mass.
+template <typename T>
+__device__ int walk_warp(const T* ra, const T* rb, const T* rt, int nv, int rounds, int lo,
+                         float beta, const float* vmass, bool stored, bool use_r, float A2,
+                         float S2, float tau) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const bool use_r = sh->use_r != 0;
-  const float tau = sh->tau_local;
-  const float A2 = sh->lse[0] * kLog2e, S2 = sh->lse[3] * kLog2e;
+  constexpr int TPL = kTThreads / 32;  // threads (vectors per round) per lane
+  const int lane = threadIdx.x & 31;
   const f2 beta2 = pk(beta, beta), L2 = pk(kLog2e, kLog2e);
   const f2 nA2 = pk(-A2, -A2), nS2 = pk(-S2, -S2);
-  // pass 2 kept the residual masses of draft rows and the fused masses of
-  // the bonus row; the other kind (a draft row whose residual is zero) is
-  // recomputed exactly as pass 2 computes it
-  const bool stored = (use_r == stored_r);
-  int last_pos = -1;  // this thread's last vector with positive mass
-  for (int j = 0; j < rounds; ++j) {
-    const int i = j * kTThreads + tid;
-    float v = 0.f;
-    if (i < nv)
-      v = stored ? vmass[j * kTThreads + tid] : vec_mass(ra, rb, rt, i, use_r, beta2, L2, nA2, nS2);
-    if (v > 0.f) last_pos = i;
-    const float ws = warp_sum(v);
-    if (lane == 0) sh->wr[j][warp] = ws;
-  }
-  __syncthreads();
-  if (tid == 0) {
-    float cum = 0.f, tj = 0.f;
-    int js = -1;
-    for (int j = 0; j < rounds; ++j) {
-      float tot = 0.f;
-      for (int w = 0; w < kTWarps; ++w) tot += sh->wr[j][w];
-      if (cum + tot > tau) {
-        js = j;
-        tj = fmaxf(tau - cum, 0.f);
-        break;
-      }
-      cum += tot;
-    }
-    sh->jstar = js;
-    sh->tau_j = tj;
-    sh->found = -1;
-  }
-  __syncthreads();
-  const int js = sh->jstar;
-  if (js >= 0) {
-    const int i = js * kTThreads + tid;
-    float x = 0.f;
-    if (i < nv)
-      x = stored ? vmass[js * kTThreads + tid] : vec_mass(ra, rb, rt, i, use_r, beta2, L2, nA2, nS2);
-    float incl = x;
+  float P[kMaxRounds], Tj[kMaxRounds];
 #pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const float v = __shfl_up_sync(0xffffffffu, incl, off);
-      if (lane >= off) incl += v;
+  for (int j = 0; j < kMaxRounds; ++j) {
+    float p = 0.f;
+    if (j < rounds) {
+      if (stored) {
+        const float4 m0 = *reinterpret_cast<const float4*>(vmass + j * kTThreads + TPL * lane);
+        const float4 m1 = *reinterpret_cast<const float4*>(vmass + j * kTThreads + TPL * lane + 4);
+        p = ((((((m0.x + m0.y) + m0.z) + m0.w) + m1.x) + m1.y) + m1.z) + m1.w;
+      } else {
+#pragma unroll 1
+        for (int v = 0; v < TPL; ++v) {
+          const int t = TPL * lane + v;
+          p += walk_mass(ra, rb, rt, j * kTThreads + t, nv, vmass, j, t, false, use_r, beta2, L2,
+                         nA2, nS2);
+        }
+      }
     }
-    if (lane == 31) sh->scan[warp] = incl;
-    __syncthreads();
-    float woff = 0.f;
-    for (int w = 0; w < warp; ++w) woff += sh->scan[w];
-    incl += woff;
-    const float excl = incl - x;
-    const float tj = sh->tau_j;
-    if (x > 0.f && excl <= tj && tj < incl) {
+    P[j] = p;
+    Tj[j] = (j < rounds) ? warp_sum(p) : 0.f;
+  }
+  // the round holding the target
+  int js = -1, jlast = -1;
+  float cum = 0.f, tj = 0.f;
+#pragma unroll
+  for (int j = 0; j < kMaxRounds; ++j) {
+    if (j < rounds) {
+      if (js < 0) {
+        if (cum + Tj[j] > tau) {
+          js = j;
+          tj = fmaxf(tau - cum, 0.f);
+        } else {
+          cum += Tj[j];
+        }
+      }
+      if (Tj[j] > 0.f) jlast = j;
+    }
+  }
+  bool take_last = false;
+  if (js < 0) {
+    if (jlast < 0) return -1;
+    js = jlast;
+    take_last = true;
+  }
+  float pj = 0.f;
+#pragma unroll
+  for (int j = 0; j < kMaxRounds; ++j)
+    if (j == js) pj = P[j];
+  // the lane holding it: inclusive prefix over lanes
+  float incl = pj;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float v = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += v;
+  }
+  const float excl = incl - pj;
+  const unsigned hit = __ballot_sync(0xffffffffu, !take_last && pj > 0.f && excl <= tj && tj < incl);
+  int lc;
+  if (hit) {
+    lc = __ffs(hit) - 1;
+  } else {
+    const unsigned pos = __ballot_sync(0xffffffffu, pj > 0.f);
+    if (!pos) return -1;
+    lc = 31 - __clz(pos);
+    take_last = true;
+  }
+  int found = -1;
+  if (lane == lc) {
+    // its vector, then the element
+    float cum2 = excl, trem = 0.f;
+    int vsel = -1, vlast = -1;
+    for (int v = 0; v < TPL; ++v) {
+      const int t = TPL * lane + v;
+      const float m = walk_mass(ra, rb, rt, js * kTThreads + t, nv, vmass, js, t, stored, use_r,
+                                beta2, L2, nA2, nS2);
+      if (m > 0.f) vlast = v;
+      if (!take_last && vsel < 0) {
+        if (cum2 + m > tj) {
+          vsel = v;
+          trem = fmaxf(tj - cum2, 0.f);
+        } else {
+          cum2 += m;
+        }
+      }
+    }
+    bool last_el = take_last;
+    if (vsel < 0) {
+      vsel = vlast;
+      last_el = true;
+    }
+    if (vsel >= 0) {
+      const int i = js * kTThreads + TPL * lane + vsel;
       f2 xa[NP], xb[NP], xt[NP], p[NP], qf[NP], r[NP];
       load_pairs(ra + i * VE, xa);
       load_pairs(rb + i * VE, xb);
       load_pairs(rt + i * VE, xt);
       vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
-      float cum = excl;
+      float cum3 = 0.f;
       int pick = -1, last = -1;
 #pragma unroll
       for (int h = 0; h < NP; ++h) {
         float v0, v1;
         upk(use_r ? r[h] : qf[h], v0, v1);
         if (v0 > 0.f) last = 2 * h;
-        cum += v0;
-        if (pick < 0 && cum > tj) pick = 2 * h;
+        cum3 += v0;
+        if (!last_el && pick < 0 && cum3 > trem) pick = 2 * h;
         if (v1 > 0.f) last = 2 * h + 1;
-        cum += v1;
-        if (pick < 0 && cum > tj) pick = 2 * h + 1;
+        cum3 += v1;
+        if (!last_el && pick < 0 && cum3 > trem) pick = 2 * h + 1;
       }
       if (pick < 0) pick = last;
-      if (pick >= 0) sh->found = lo + i * VE + pick;
+      if (pick >= 0) found = lo + i * VE + pick;
     }
   }
-  __syncthreads();
-  const int found0 = sh->found;
-  __syncthreads();
-  if (found0 < 0) {
-    // the target fell into the rounding gap at the end: last positive element
-    if (last_pos >= 0) atomicMax(&sh->found, last_pos);
-    __syncthreads();
-    const int kmax = sh->found;
-    __syncthreads();
-    if (tid == 0) sh->found = -1;
-    __syncthreads();
-    if (kmax >= 0 && last_pos == kmax) {
-      f2 xa[NP], xb[NP], xt[NP], p[NP], qf[NP], r[NP];
-      load_pairs(ra + kmax * VE, xa);
-      load_pairs(rb + kmax * VE, xb);
-      load_pairs(rt + kmax * VE, xt);
-      vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
-      int last = -1;
-#pragma unroll
-      for (int h = 0; h < NP; ++h) {
-        float v0, v1;
-        upk(use_r ? r[h] : qf[h], v0, v1);
-        if (v0 > 0.f) last = 2 * h;
-        if (v1 > 0.f) last = 2 * h + 1;
-      }
-      if (last >= 0) sh->found = lo + kmax * VE + last;
-    }
-    __syncthreads();
-  }
-  return sh->found;
+  return __shfl_sync(0xffffffffu, found, lc);
 }
 
 // ---------------------------------------------------------------- the kernel
+
+// Per-row values the row programs share.
+struct RowCtx {
+  const void* sa;
+  const void* sb;
+  const void* st;
+  int nv, rounds, rc, lo, n, W, rank, C, k, bi;
+  long long row;
+  bool bonus;
+  int dtok;           // warp 0 only
+  RowScalars sc;      // warp 0 only (stochastic)
+  float* vmass;
+  SharedTma* sh;
+};
+
+// The decision of a complete row (one warp; lane 0 writes).
+template <bool STOCH>
+__device__ __forceinline__ void finish(const KParams& P, const RowCtx& c, const float (&lse)[4],
+                                       int is, int it, unsigned bad, float D, int sample,
+                                       float mass, float ad, float bd, float td) {
+  const bool has_ab = P.full || !c.bonus;
+  const bool has_t = P.full || (!STOCH && !c.bonus);
+  const bool has_s = P.full || STOCH;
+  RowResult r;
+  r.lse_a = has_ab ? lse[0] : NAN;
+  r.lse_b = has_ab ? lse[1] : NAN;
+  r.lse_t = has_t ? lse[2] : NAN;
+  r.lse_s = has_s ? lse[3] : NAN;
+  r.D = D;
+  r.is = is;
+  r.it = it;
+  r.sample = sample;
+  r.mass = mass;
+  r.bad = bad;
+  r.have_lse_t = has_t;
+  finish_row_warp<STOCH>(P, c.row, c.bi, c.k, r, c.dtok, ad, bd, td, c.sc);
+}
+
+// One row with pass-1 program F and pass-2 program G (R2: pass 2 runs; LP:
+// it writes the fused log-probs).
+template <typename T, bool STOCH, unsigned F, unsigned G, bool LP, bool R2>
+__device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
+                                        cg::cluster_group& cluster) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const T* ra = static_cast<const T*>(c.sa);
+  const T* rb = static_cast<const T*>(c.sb);
+  const T* rt = static_cast<const T*>(c.st);
+  SharedTma* sh = c.sh;
+  const float beta = P.beta;
+  pass1_and_push<T, F>(ra, rb, rt, c.nv, c.rounds, c.rc, c.lo, c.n, beta, c.dtok, sh, c.rank, c.C,
+                       cluster);
+  if constexpr (!R2) {
+    // no pass 2: the row is decided by warp 0 of rank 0; every other warp leaves
+    if (c.rank == 0 && warp == 0) {
+      float lse[4];
+      const X1 w = combine_pass1<F>(sh, c.C, lse);
+      float ad, bd, td;
+      draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td);
+      finish<STOCH>(P, c, lse, w.is, w.it, w.bad, 0.f, -1, NAN, ad, bd, td);
+    }
+    return;
+  } else {
+    if (warp == 0) {
+      float lse[4];
+      const X1 w = combine_pass1<F>(sh, c.C, lse);
+      if (lane == 0) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) sh->lse[q] = lse[q];
+        sh->is = w.is;
+        sh->it = w.it;
+        sh->bad = w.bad;
+        draft_logits(sh, c.dtok, c.W, c.C, sh->da, sh->db, sh->dt);
+      }
+    }
+    __syncthreads();
+    float* lp = LP ? P.logprobs + static_cast<size_t>(c.row) * P.V + c.lo : nullptr;
+    pass2_and_push<T, G, LP>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh, c.rank, c.C, c.vmass,
+                             cluster);
+    if (warp != 0) return;  // the rest is warp 0's
+    const X2 w = (lane < c.C) ? sh->recv2(c.C)[lane] : x2_zero();
+    const float lse[4] = {sh->lse[0], sh->lse[1], sh->lse[2], sh->lse[3]};
+    if constexpr (STOCH) {
+      // inclusive prefix of the inverse-CDF mass over ranks, in rank order
+      float incl_R = w.R, incl_Q = w.Q;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const float vr = __shfl_up_sync(0xffffffffu, incl_R, off);
+        const float vq = __shfl_up_sync(0xffffffffu, incl_Q, off);
+        if (lane >= off) {
+          incl_R += vr;
+          incl_Q += vq;
+        }
+      }
+      const float R_all = __shfl_sync(0xffffffffu, incl_R, 31);
+      const float Q_all = __shfl_sync(0xffffffffu, incl_Q, 31);
+      const bool r_ok = !c.bonus && (R_all > 0.f);
+      const float incl = r_ok ? incl_R : incl_Q;
+      const float mass = r_ok ? w.R : w.Q;
+      const float total = r_ok ? R_all : Q_all;
+      const float tau = c.sc.u_last * total;
+      const unsigned over = __ballot_sync(0xffffffffu, lane < c.C && incl > tau);
+      const unsigned pos = __ballot_sync(0xffffffffu, lane < c.C && mass > 0.f);
+      int owner = -1;
+      if (over) owner = __ffs(over) - 1;
+      else if (pos) owner = 31 - __clz(pos);
+      if (c.rank != owner && !(owner < 0 && c.rank == 0)) return;
+      X2 tot = w;
+      warp_reduce_x2<G>(tot);
+      const float D = divergence_of<G>(tot);
+      int sample = -1;
+      if (owner >= 0) {
+        const float incl_o = __shfl_sync(0xffffffffu, incl, owner);
+        const float mass_o = __shfl_sync(0xffffffffu, mass, owner);
+        const float tau_local = fmaxf(tau - (incl_o - mass_o), 0.f);
+        // pass 2 kept the residual masses of draft rows and the fused masses
+        // of the bonus row; the other kind (a draft row whose residual is
+        // zero) is recomputed exactly as pass 2 computes it
+        const bool stored_r = !c.bonus || P.full;
+        sample = walk_warp<T>(ra, rb, rt, c.nv, c.rounds, c.lo, beta, c.vmass, r_ok == stored_r,
+                              r_ok, lse[0] * kLog2e, lse[3] * kLog2e, tau_local);
+      }
+      finish<STOCH>(P, c, lse, sh->is, sh->it, sh->bad, D, sample, total, sh->da, sh->db, sh->dt);
+    } else {
+      if (c.rank != 0) return;
+      X2 tot = w;
+      warp_reduce_x2<G>(tot);
+      finish<STOCH>(P, c, lse, sh->is, sh->it, sh->bad, divergence_of<G>(tot), -1, NAN, sh->da,
+                    sh->db, sh->dt);
+    }
+  }
+}
+
+template <typename T, bool STOCH, unsigned F, unsigned RQ>
+__device__ __forceinline__ void run_full(const KParams& P, const RowCtx& c,
+                                         cg::cluster_group& cluster) {
+  const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
+  const bool klg = P.divergence == ASYMSPEC_DIV_KL;
+  if (P.logprobs) {
+    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, true, true>(P, c, cluster);
+    else if (klg) run_row<T, STOCH, F, G_KL | RQ, true, true>(P, c, cluster);
+    else run_row<T, STOCH, F, RQ, true, true>(P, c, cluster);
+  } else {
+    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, false, true>(P, c, cluster);
+    else if (klg) run_row<T, STOCH, F, G_KL | RQ, false, true>(P, c, cluster);
+    else run_row<T, STOCH, F, RQ, false, true>(P, c, cluster);
+  }
+}
 
 template <typename T, bool STOCH>
 __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P) {
@@ -812,148 +1123,81 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   // stochastic: per-thread, per-round sampling masses after the records
   float* vmass = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sh) +
                                           shared_tma_bytes(C));
-  const float beta = P.beta;
-  const bool leader = (rank == 0 && tid == 0);
   const bool only_t = !STOCH && !P.full && bonus && !P.fuse_bonus;
 
   if (tid == 0) {
 #pragma unroll
     for (int c = 0; c < kChunks; ++c) mbar_init(&sh->bar[c], 1);
-    mbar_init(&sh->sample_bar, 1);
     sh->broken = 0;
-    sh->sample = -1;
     fence_mbar_init();
+    issue_slice<T>(P, sh, row, lo, nv, rc, sa, sb, st, only_t);
   }
-  __syncthreads();
-  if (tid == 0) {
-    const size_t off = static_cast<size_t>(row) * V + lo;
-    const T* ga = static_cast<const T*>(P.a) + off;
-    const T* gb = static_cast<const T*>(P.b) + off;
-    const T* gt = static_cast<const T*>(P.t) + off;
-#pragma unroll
-    for (int c = 0; c < kChunks; ++c) {
-      const int v0 = min(nv, c * rc * kTThreads);
-      const int v1 = min(nv, (c + 1) * rc * kTThreads);
-      const unsigned bytes = static_cast<unsigned>(v1 - v0) * 16u;
-      mbar_arrive_expect_tx(&sh->bar[c], bytes * (only_t ? 1u : 3u));
-      if (bytes) {
-        const int e0 = v0 * VE;
-        if (!only_t) {
-          bulk_load(sa + e0, ga + e0, bytes, &sh->bar[c]);
-          bulk_load(sb + e0, gb + e0, bytes, &sh->bar[c]);
-        }
-        bulk_load(st + e0, gt + e0, bytes, &sh->bar[c]);
-      }
-    }
+  RowCtx c;
+  c.sa = sa;
+  c.sb = sb;
+  c.st = st;
+  c.nv = nv;
+  c.rounds = rounds;
+  c.rc = rc;
+  c.lo = lo;
+  c.n = n;
+  c.W = W;
+  c.rank = rank;
+  c.C = C;
+  c.k = k;
+  c.bi = bi;
+  c.row = row;
+  c.bonus = bonus;
+  c.vmass = vmass;
+  c.sh = sh;
+  c.dtok = -1;
+  c.sc = RowScalars{0.f, 0.f, 0.f};
+  // warp 0 keeps the row's scalar inputs, loaded while the slice is in flight
+  if ((tid >> 5) == 0) {
+    if (!bonus) c.dtok = P.tokens[static_cast<size_t>(bi) * P.K + k];
+    if (STOCH) c.sc = load_row_scalars(P, bi, k);
   }
-  // the scalars of this row, loaded while the slice is in flight
-  const int dtok = bonus ? -1 : P.tokens[static_cast<size_t>(bi) * P.K + k];
-  const float u_last = STOCH ? P.unif[static_cast<size_t>(bi) * K1 + P.K] : 0.f;
+  __syncthreads();  // the chunk barriers are initialised
 
-  // ---- pass 1 (program chosen per row; uniform over the cluster)
   if (P.full) {
-    pass1_and_combine<T, F_LA | F_LB | F_LT | F_LS | F_AS | F_AT>(
-        sa, sb, st, nv, rounds, rc, lo, n, W, beta, dtok, sh, rank, C, cluster);
+    run_full<T, STOCH, F_LA | F_LB | F_LT | F_LS | F_AS | F_AT, STOCH ? G_RES : 0u>(P, c, cluster);
   } else if (!STOCH) {
-    if (!bonus)
-      pass1_and_combine<T, F_LA | F_LB | F_LT | F_AS>(sa, sb, st, nv, rounds, rc, lo, n, W, beta,
-                                                      dtok, sh, rank, C, cluster);
-    else if (P.fuse_bonus)
-      pass1_and_combine<T, F_AS>(sa, sb, st, nv, rounds, rc, lo, n, W, beta, dtok, sh, rank, C,
-                                 cluster);
-    else
-      pass1_and_combine<T, F_AT>(sa, sb, st, nv, rounds, rc, lo, n, W, beta, dtok, sh, rank, C,
-                                 cluster);
-  } else if (!bonus) {
-    if (P.want_tokens)
-      pass1_and_combine<T, F_LA | F_LB | F_LS | F_AS>(sa, sb, st, nv, rounds, rc, lo, n, W, beta,
-                                                      dtok, sh, rank, C, cluster);
-    else
-      pass1_and_combine<T, F_LA | F_LB | F_LS>(sa, sb, st, nv, rounds, rc, lo, n, W, beta, dtok,
-                                               sh, rank, C, cluster);
-  } else {
-    if (P.want_tokens)
-      pass1_and_combine<T, F_LS | F_AS>(sa, sb, st, nv, rounds, rc, lo, n, W, beta, dtok, sh,
-                                        rank, C, cluster);
-    else
-      pass1_and_combine<T, F_LS>(sa, sb, st, nv, rounds, rc, lo, n, W, beta, dtok, sh, rank, C,
-                                 cluster);
-  }
-
-  // ---- pass 2
-  const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
-  const bool klg = P.divergence == ASYMSPEC_DIV_KL;
-  const bool run2 = STOCH || P.full || (!bonus && (jsd || klg));
-  if (run2) {
-    float* lp = P.logprobs ? P.logprobs + static_cast<size_t>(row) * V + lo : nullptr;
-    const bool r_allowed = STOCH && !bonus;
-    constexpr unsigned RQ = STOCH ? G_RES : 0u;
-    if (STOCH && bonus && !P.full) {
-      pass2_and_combine<T, G_QF, false, STOCH>(sa, sb, st, nv, rounds, beta, nullptr, sh, rank,
-                                               C, false, u_last, vmass, cluster);
-    } else if (lp) {
-      if (jsd)
-        pass2_and_combine<T, G_JSD | RQ, true, STOCH>(sa, sb, st, nv, rounds, beta, lp, sh, rank, C,
-                                              r_allowed, u_last, vmass, cluster);
-      else if (klg)
-        pass2_and_combine<T, G_KL | RQ, true, STOCH>(sa, sb, st, nv, rounds, beta, lp, sh, rank, C,
-                                              r_allowed, u_last, vmass, cluster);
-      else
-        pass2_and_combine<T, RQ, true, STOCH>(sa, sb, st, nv, rounds, beta, lp, sh, rank, C,
-                                              r_allowed, u_last, vmass, cluster);
+    const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
+    const bool klg = P.divergence == ASYMSPEC_DIV_KL;
+    constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
+    if (bonus) {
+      if (P.fuse_bonus) run_row<T, STOCH, F_AS, 0, false, false>(P, c, cluster);
+      else run_row<T, STOCH, F_AT, 0, false, false>(P, c, cluster);
+    } else if (jsd) {
+      run_row<T, STOCH, FD, G_JSD, false, true>(P, c, cluster);
+    } else if (klg) {
+      run_row<T, STOCH, FD, G_KL, false, true>(P, c, cluster);
     } else {
-      if (jsd)
-        pass2_and_combine<T, G_JSD | RQ, false, STOCH>(sa, sb, st, nv, rounds, beta, nullptr, sh, rank, C,
-                                              r_allowed, u_last, vmass, cluster);
-      else if (klg)
-        pass2_and_combine<T, G_KL | RQ, false, STOCH>(sa, sb, st, nv, rounds, beta, nullptr, sh, rank, C,
-                                              r_allowed, u_last, vmass, cluster);
-      else
-        pass2_and_combine<T, RQ, false, STOCH>(sa, sb, st, nv, rounds, beta, nullptr, sh, rank, C,
-                                              r_allowed, u_last, vmass, cluster);
+      run_row<T, STOCH, FD, 0, false, false>(P, c, cluster);
     }
-  } else if (tid == 0) {
-    sh->D = 0.f;
+  } else if (!bonus) {
+    const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
+    const bool klg = P.divergence == ASYMSPEC_DIV_KL;
+    if (P.want_tokens) {
+      constexpr unsigned FS = F_LA | F_LB | F_LS | F_AS;
+      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true>(P, c, cluster);
+      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true>(P, c, cluster);
+      else run_row<T, STOCH, FS, G_RES, false, true>(P, c, cluster);
+    } else {
+      constexpr unsigned FS = F_LA | F_LB | F_LS;
+      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true>(P, c, cluster);
+      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true>(P, c, cluster);
+      else run_row<T, STOCH, FS, G_RES, false, true>(P, c, cluster);
+    }
+  } else {
+    if (P.want_tokens) run_row<T, STOCH, F_LS | F_AS, G_QF, false, true>(P, c, cluster);
+    else run_row<T, STOCH, F_LS, G_QF, false, true>(P, c, cluster);
   }
 
-  // ---- stochastic: inverse-CDF draw in the owning CTA, handed to rank 0
-  if constexpr (STOCH) {
-    if (rank == sh->owner) {
-      const int pick = walk<T>(sh, sa, sb, st, nv, rounds, lo, beta, vmass, !bonus || P.full);
-      if (tid == 0) {
-        *cluster.map_shared_rank(&sh->sample, 0) = pick;
-        mbar_arrive_remote(&sh->sample_bar, 0);
-      }
-    }
-  }
-
-  // ---- epilogue (rank 0, thread 0)
-  if (leader) {
-    if (STOCH && sh->owner >= 0 &&
-        !mbar_wait_cluster_bounded(&sh->sample_bar, 0, kCopyTimeoutNs))
-      sh->bad |= kBadTimeout;
-    const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
-    const bool has_ab = P.full || !bonus;
-    const bool has_t = P.full || (!STOCH && !bonus);
-    const bool has_s = P.full || STOCH;
-    RowResult r;
-    r.lse_a = has_ab ? lse_a : NAN;
-    r.lse_b = has_ab ? lse_b : NAN;
-    r.lse_t = has_t ? sh->lse[2] : NAN;
-    r.lse_s = has_s ? lse_s : NAN;
-    r.D = sh->D;
-    r.is = sh->is;
-    r.it = sh->it;
-    r.sample = STOCH ? sh->sample : -1;
-    r.mass = STOCH ? sh->mass_total : NAN;
-    r.bad = sh->bad;
-    r.have_lse_t = has_t;
-    finish_row<STOCH>(P, row, bi, k, r, dtok, sh->da, sh->db, sh->dt);
-  }
   // a copy that timed out may still land: wait for it (bounded) before exit
   if (tid == 0 && sh->broken) {
 #pragma unroll
-    for (int c = 0; c < kChunks; ++c) mbar_wait_bounded(&sh->bar[c], 0, kCopyTimeoutNs);
+    for (int q = 0; q < kChunks; ++q) mbar_wait_bounded(&sh->bar[q], 0, kCopyTimeoutNs);
   }
 }
 

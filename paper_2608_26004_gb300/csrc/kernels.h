@@ -1,0 +1,19 @@
+// Host accessors of the kernels, each compiled in its own translation unit
+// (k_*.cu) so that the build compiles them in parallel.  The pointers are
+// passed to cudaLaunchKernelExC and the occupancy queries.
+#pragma once
+
+namespace asymspec_impl {
+
+// fuse_verify_generic<T, VE, STOCH> (k_generic.cu)
+const void* generic_kernel(int dtype, bool vector_path, bool stoch);
+// fuse_verify_tma<T, STOCH> (k_tma_bf16.cu, k_tma_f32.cu)
+const void* tma_kernel_bf16(bool stoch);
+const void* tma_kernel_f32(bool stoch);
+// fuse_verify_stream<T, STOCH> (k_stream_*.cu)
+const void* stream_kernel_bf16_greedy();
+const void* stream_kernel_bf16_stoch();
+const void* stream_kernel_f32_greedy();
+const void* stream_kernel_f32_stoch();
+
+}  // namespace asymspec_impl

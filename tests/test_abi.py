@@ -53,9 +53,12 @@ def test_defaults_and_strings(lib):
 
 
 def test_workspace_size():
+    # records and tickets of the cluster kernels, then the streaming kernel's state
     assert A.workspace_bytes(64, 7, 128256) >= 64 * 8 * 16 + 64 * 4
     assert A.workspace_bytes(0, 7, 10) == 0
-    assert A.workspace_bytes(3, 2, 10) == A.workspace_bytes(3, 2, 10**6)
+    # the streaming state grows with the tiles per row (fp32 rows have the most)
+    assert A.workspace_bytes(3, 2, 10) < A.workspace_bytes(3, 2, 10**5)
+    assert A.workspace_bytes(64, 7, 128256) < 8 << 20
 
 
 FAKE = 0x10000  # never dereferenced: every call below fails validation first
@@ -86,7 +89,8 @@ def test_host_validation_codes(lib):
     assert call(dtype=A.BF16, a=FAKE + 1) == A.ERR_MISALIGNED
     assert call(tok=FAKE + 2) == A.ERR_MISALIGNED
     assert call(ws=0) == A.ERR_WORKSPACE
-    assert call(ws_bytes=A.workspace_bytes(2, 2, 64) - 1) == A.ERR_WORKSPACE
+    # below even the cluster kernels' records and tickets (2 x 3 rows, 2 tickets)
+    assert call(ws_bytes=511) == A.ERR_WORKSPACE
     g = A.GateParams(0.5, 1.0, 0.1, 0, 0, 0, 3)
     assert call(gate=g) == A.ERR_INVALID_ARG          # reserved flags must be 0
     opts = A.LaunchOpts(17, 0, 0)
@@ -96,6 +100,10 @@ def test_host_validation_codes(lib):
     st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
                           FAKE, FAKE, 1 << 20, opts=A.LaunchOpts(0, 0, 7))
     assert st == A.ERR_INVALID_ARG                       # unknown kernel
+    small = A.workspace_bytes(2, 2, 64) - 1              # streaming kernel forced, workspace short
+    st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
+                          FAKE, FAKE, small, opts=A.LaunchOpts(0, 0, A.KERNEL_STREAM))
+    assert st == A.ERR_WORKSPACE
 
 
 def test_static_entry_point_rejects_batches_above_its_scratch(lib):
@@ -110,20 +118,28 @@ def test_static_entry_point_rejects_batches_above_its_scratch(lib):
 
 
 def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
-    # the bench workload: TMA kernel, 8 CTAs of 96 KB per row, two CTAs per SM
-    info = A.plan(64, 7, 128256, A.BF16)
+    # the streaming kernel on request: 16384-entry tiles (bf16), 8192 (fp32)
+    STREAM = A.LaunchOpts(0, 0, A.KERNEL_STREAM)
+    info = A.plan(64, 7, 128256, A.BF16, opts=STREAM)
+    assert info.kernel == A.KERNEL_STREAM and info.slice_elems == 16384
+    info = A.plan(1, 4, 32000, A.FP32, opts=STREAM)
+    assert info.kernel == A.KERNEL_STREAM and info.slice_elems == 8192
+    assert A.plan(64, 7, 128256, A.BF16).kernel == A.KERNEL_TMA      # the automatic choice
+    TMA = A.LaunchOpts(0, 0, A.KERNEL_TMA)
+    # the cluster kernel on the bench workload: 8 CTAs of 96 KB per row, two per SM
+    info = A.plan(64, 7, 128256, A.BF16, opts=TMA)
     assert info.kernel == A.KERNEL_TMA and info.cluster_size == 8
     assert info.slice_elems == 16032 and info.vector_path == 1
     assert info.ctas == 64 * 8 * 8 and info.smem_bytes <= 113 * 1024
     # Qwen3-sized bf16 rows: 8 CTAs of 112.7 KB, still two per SM
-    info = A.plan(8, 5, 151936, A.BF16)
+    info = A.plan(8, 5, 151936, A.BF16, opts=TMA)
     assert info.kernel == A.KERNEL_TMA and info.cluster_size == 8
     assert info.smem_bytes <= 113 * 1024
     # fp32 rows of 151,936 entries: 16 CTAs of 114 KB
-    info = A.plan(256, 4, 151936, A.FP32)
+    info = A.plan(256, 4, 151936, A.FP32, opts=TMA)
     assert info.kernel == A.KERNEL_TMA and info.cluster_size == 16
     assert info.smem_bytes <= 227 * 1024
-    info = A.plan(1, 4, 32000, A.FP32)
+    info = A.plan(1, 4, 32000, A.FP32, opts=TMA)
     assert info.kernel == A.KERNEL_TMA and info.cluster_size == 4
     info = A.plan(2, 2, 4099, A.BF16)
     assert info.vector_path == 0 and info.kernel == A.KERNEL_GENERIC

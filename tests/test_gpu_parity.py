@@ -18,8 +18,11 @@ pytestmark = pytest.mark.gpu
 
 GREEDY, STOCH = A.MODE_GREEDY, A.MODE_STOCHASTIC
 AUTO, GENERIC, TMA = A.KERNEL_AUTO, A.KERNEL_GENERIC, A.KERNEL_TMA
-PATHS = [(AUTO, False), (AUTO, True), (GENERIC, True)]
-PATH_IDS = ["auto-prod", "auto-full", "generic-full"]
+STREAM = A.KERNEL_STREAM
+# the automatic choice (the cluster TMA kernel for aligned rows), the
+# streaming kernel, and the generic cluster kernel
+PATHS = [(AUTO, False), (AUTO, True), (STREAM, False), (STREAM, True), (GENERIC, True)]
+PATH_IDS = ["auto-prod", "auto-full", "stream-prod", "stream-full", "generic-full"]
 
 
 @pytest.fixture(scope="module")
@@ -186,7 +189,7 @@ def test_data_errors_never_trap(torch, kernel, full):
     assert word & A.DATA_BAD_PROB and word & A.DATA_BAD_UNIFORM
 
 
-@pytest.mark.parametrize("kernel", [GENERIC, TMA])
+@pytest.mark.parametrize("kernel", [GENERIC, TMA, STREAM])
 def test_exact_ties_resolve_to_lowest_index(torch, kernel):
     B, K, V = 2, 2, 4096
     a = np.zeros((B, K + 1, V), np.float32)
@@ -196,7 +199,7 @@ def test_exact_ties_resolve_to_lowest_index(torch, kernel):
     t[1, :, [5, 4000]] = 7.0
     batch = synth.Batch(a, b, t, np.full((B, K), 7, np.int32), np.full((B, K), 0.5, np.float32),
                         np.full((B, K + 1), 0.5, np.float32), B, K, V, synth.FP32)
-    for cluster in (0, 1, 4, 16):
+    for cluster in ((0,) if kernel == STREAM else (0, 1, 4, 16)):
         for full in (False, True):
             g = run_gpu(batch, torch, mode=GREEDY, cluster_size=cluster, gamma=1.0,
                         kernel=kernel, full=full, fuse_bonus=True)
@@ -252,7 +255,11 @@ def test_workspace_reuse_and_allocating_entry_point(torch):
 
 
 def test_plan_reports_cluster_occupancy(torch):
-    info = A.plan(64, 7, 128256, A.BF16)
+    # streaming kernel: a persistent grid of whole SMs' worth of resident CTAs
+    info = A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(0, 0, A.KERNEL_STREAM))
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    assert info.kernel == A.KERNEL_STREAM and info.ctas >= sms and info.ctas % sms == 0
+    info = A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(0, 0, A.KERNEL_TMA))
     assert info.kernel == A.KERNEL_TMA and info.cluster_size == 8 and info.vector_path == 1
     assert info.max_active_clusters >= 30          # 2 CTAs per SM, clusters of 8
     assert info.smem_bytes <= 113 * 1024
@@ -262,7 +269,7 @@ def test_plan_reports_cluster_occupancy(torch):
 
 # ---------------------------------------------------------------- sampling law
 
-@pytest.mark.parametrize("kernel", [GENERIC, TMA])
+@pytest.mark.parametrize("kernel", [GENERIC, TMA, STREAM])
 def test_emitted_token_law_chi_square(torch, kernel):
     from scipy.stats import chisquare
     V, K, N = 8, 1, 1_000_000
@@ -294,3 +301,32 @@ def test_emitted_token_law_chi_square(torch, kernel):
     ok = ~oflag
     assert ok.mean() > 0.99
     assert np.array_equal(L[ok], oL[ok]) and np.array_equal(nxt[ok], oN[ok])
+
+
+@pytest.mark.parametrize("kernel", [AUTO, STREAM])
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+def test_entries_far_above_the_first_vector(torch, kernel, mode):
+    # a logit 150 nats above the rest, away from every thread's first vector:
+    # the fixed-reference sums overflow and the slice (or tile) is redone with
+    # a running maximum
+    batch = small(3, 2, 40000, synth.BF16, seed=91)
+    for arr in (batch.logits_full, batch.logits_comp, batch.logits_ver):
+        bits = np.zeros(1, np.float32)
+        bits[0] = 150.0
+        spike = (bits.view(np.uint32) >> 16).astype(np.uint16)[0]
+        arr[0, 1, 30001] = spike
+        arr[2, 2, 12345] = spike
+    for full in (False, True):
+        check(batch, torch, mode, kernel, full)
+
+
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+@pytest.mark.parametrize("B,K,V,dtype", [(3, 2, 16384 * 3 + 8, synth.BF16),
+                                         (2, 3, 8192 * 2 - 4, synth.FP32),
+                                         (40, 1, 16384 + 2048, synth.BF16)])
+def test_streaming_tiles_and_ragged_tail(torch, B, K, V, dtype, mode):
+    # several tiles per row, a last tile of one vector or of a partial round,
+    # and (B=40) more rows than the look-ahead of a small grid
+    batch = small(B, K, V, dtype, seed=B * 7 + V)
+    for full in (False, True):
+        check(batch, torch, mode, STREAM, full)

@@ -3,7 +3,8 @@
 The file name sorts last so that these calls also run after every other GPU
 test has used the library in the same process; the tests must pass both
 alone and then.  Every result is compared bit for bit with
-asymspec_fuse_verify_ex (same kernel, caller-owned zeroed workspace) on the
+asymspec_fuse_verify_ex on the same kernel (the scratch holds the cluster
+kernels' records and tickets) with a caller-owned zeroed workspace, on the
 same inputs, over two consecutive calls, so that the second call sees the
 scratch the first one left.
 """
@@ -44,6 +45,8 @@ def run_static(torch, x, B, K, V, dtype, gate):
 
 
 def run_ex(torch, x, B, K, V, dtype, gate):
+    """The workspace entry point on the kernel the static scratch selects: the
+    cluster kernels (TMA for aligned rows, generic otherwise)."""
     L = torch.full((B,), -7, dtype=torch.int32, device="cuda")
     N = torch.full((B,), -7, dtype=torch.int32, device="cuda")
     nbytes = A.workspace_bytes(B, K, V)
@@ -51,7 +54,9 @@ def run_ex(torch, x, B, K, V, dtype, gate):
     stream = torch.cuda.current_stream().cuda_stream
     st = A.fuse_verify_ex(_ptr(x["a"]), _ptr(x["b"]), _ptr(x["t"]), _ptr(x["tokens"]),
                           _ptr(x["probs"]), _ptr(x["unif"]), B, K, V, dtype, gate, _ptr(L),
-                          _ptr(N), _ptr(ws), nbytes, stream=stream)
+                          _ptr(N), _ptr(ws), nbytes,
+                          opts=A.LaunchOpts(0, 0, A.KERNEL_AUTO if V % 8 else A.KERNEL_TMA),
+                          stream=stream)
     assert st == A.OK, A.status_string(st)
     torch.cuda.synchronize()
     return L.cpu().numpy(), N.cpu().numpy()
