@@ -77,7 +77,7 @@ bool plan_tma(int V, int elt, int forced_C, bool stoch, Plan* pl) {
     const long long per = (static_cast<long long>(V) + C - 1) / C;
     const long long W = round_up_ll(per, VE);
     const int rounds = static_cast<int>((W / VE + kTThreads - 1) / kTThreads);
-    const int shared_bytes = shared_tma_bytes(C) + (stoch ? mass_bytes(rounds) : 0);
+    const int shared_bytes = shared_tma_bytes(C) + (stoch ? group_bytes(C) : 0);
     const long long sh_off = round_up_ll(3 * W * elt, 128);
     pl->C = C;
     pl->W = static_cast<int>(W);

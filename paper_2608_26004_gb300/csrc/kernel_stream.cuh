@@ -629,140 +629,6 @@ __device__ __forceinline__ void ring_pass2(const SParams& S, SharedStream* sh,
 
 // ---------------------------------------------------------------- inverse-CDF draw
 
-// Mass of vector v (tile-local) recomputed from global memory, as pass 2
-// computes it.
-template <typename T>
-__device__ __forceinline__ void vector_masses_g(const T* ra, const T* rb, const T* rt, int v,
-                                                f2 beta2, f2 L2, f2 nA2, f2 nS2, f2 (&p)[16 / sizeof(T) / 2],
-                                                f2 (&qf)[16 / sizeof(T) / 2],
-                                                f2 (&r)[16 / sizeof(T) / 2]) {
-  constexpr int VE = 16 / static_cast<int>(sizeof(T));
-  constexpr int NP = VE / 2;
-  const unsigned long long pol = policy_evict_first();
-  f2 xa[NP], xb[NP], xt[NP];
-  gload_pairs(ra + v * VE, pol, xa);
-  gload_pairs(rb + v * VE, pol, xb);
-  gload_pairs(rt + v * VE, pol, xt);
-  vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
-}
-
-// One warp: the row index (within the tile: entries from t0) whose cumulative
-// mass in index order first exceeds tau, or the last positive one when
-// rounding leaves tau at or beyond the total.  gm: the tile's 64 group masses
-// when `stored`, else recomputed (the rare fallback to the fused masses of a
-// draft row whose residual is zero).  Returns -1 if the tile holds no mass.
-template <typename T>
-__device__ __noinline__ int tile_walk(const T* ra, const T* rb, const T* rt, int nvec, int t0, float beta,
-                         const float* gm, bool stored, bool use_r, float A2, float S2, float tau) {
-  constexpr int VE = 16 / static_cast<int>(sizeof(T));
-  constexpr int NP = VE / 2;
-  const int lane = threadIdx.x & 31;
-  const f2 beta2 = pk(beta, beta), L2 = pk(kLog2e, kLog2e);
-  const f2 nA2 = pk(-A2, -A2), nS2 = pk(-S2, -S2);
-  // lane l holds groups 2l and 2l+1 (index order)
-  float g2[2];
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const int g = 2 * lane + h;
-    float m = 0.f;
-    if (stored) {
-      m = __ldcg(gm + g);
-    } else {
-      for (int u = 0; u < 32; ++u) {
-        const int v = 32 * g + u;
-        if (v < nvec) {
-          f2 p[NP], qf[NP], r[NP];
-          vector_masses_g(ra, rb, rt, v, beta2, L2, nA2, nS2, p, qf, r);
-          m += vsum(use_r ? r : qf);
-        }
-      }
-    }
-    g2[h] = m;
-  }
-  const float pl = g2[0] + g2[1];
-  float incl = pl;
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const float v = __shfl_up_sync(0xffffffffu, incl, off);
-    if (lane >= off) incl += v;
-  }
-  const float excl = incl - pl;
-  bool take_last = false;
-  unsigned hit = __ballot_sync(0xffffffffu, pl > 0.f && excl <= tau && tau < incl);
-  int lc;
-  if (hit) {
-    lc = __ffs(hit) - 1;
-  } else {
-    const unsigned pos = __ballot_sync(0xffffffffu, pl > 0.f);
-    if (!pos) return -1;
-    lc = 31 - __clz(pos);
-    take_last = true;
-  }
-  // the group, in lane lc
-  int gsel = -1;
-  float trem = 0.f;
-  if (lane == lc) {
-    if (!take_last && excl + g2[0] > tau) {
-      gsel = 2 * lane;
-      trem = fmaxf(tau - excl, 0.f);
-    } else if (!take_last && g2[1] > 0.f) {
-      gsel = 2 * lane + 1;
-      trem = fmaxf(tau - excl - g2[0], 0.f);
-    } else {
-      gsel = g2[1] > 0.f ? 2 * lane + 1 : 2 * lane;
-      take_last = true;
-    }
-  }
-  gsel = __shfl_sync(0xffffffffu, gsel, lc);
-  trem = __shfl_sync(0xffffffffu, trem, lc);
-  take_last = __shfl_sync(0xffffffffu, take_last ? 1 : 0, lc) != 0;
-  // the vector: lane u recomputes vector 32 gsel + u
-  const int v = 32 * gsel + lane;
-  f2 p[NP], qf[NP], r[NP];
-  float mv = 0.f;
-  if (v < nvec) {
-    vector_masses_g(ra, rb, rt, v, beta2, L2, nA2, nS2, p, qf, r);
-    mv = vsum(use_r ? r : qf);
-  }
-  float vin = mv;
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const float w = __shfl_up_sync(0xffffffffu, vin, off);
-    if (lane >= off) vin += w;
-  }
-  const float vex = vin - mv;
-  unsigned vh = __ballot_sync(0xffffffffu, !take_last && mv > 0.f && vex <= trem && trem < vin);
-  int vc;
-  if (vh) {
-    vc = __ffs(vh) - 1;
-  } else {
-    const unsigned pos = __ballot_sync(0xffffffffu, mv > 0.f);
-    if (!pos) return -1;
-    vc = 31 - __clz(pos);
-    take_last = true;
-  }
-  int found = -1;
-  if (lane == vc) {
-    const float te = fmaxf(trem - vex, 0.f);
-    float cum = 0.f;
-    int pick = -1, last = -1;
-#pragma unroll
-    for (int h = 0; h < NP; ++h) {
-      float v0, v1;
-      upk(use_r ? r[h] : qf[h], v0, v1);
-      if (v0 > 0.f) last = 2 * h;
-      cum += v0;
-      if (!take_last && pick < 0 && cum > te) pick = 2 * h;
-      if (v1 > 0.f) last = 2 * h + 1;
-      cum += v1;
-      if (!take_last && pick < 0 && cum > te) pick = 2 * h + 1;
-    }
-    if (pick < 0) pick = last;
-    if (pick >= 0) found = t0 + v * VE + pick;
-  }
-  return __shfl_sync(0xffffffffu, found, vc);
-}
-
 // ---------------------------------------------------------------- row completion
 
 // After the last pass-1 tile of a row (one warp, records acquired): the row's
@@ -913,10 +779,11 @@ __device__ __noinline__ void row_after_pass2(const SParams& S, long long row, in
       // fused masses of the bonus row; a draft row with zero residual
       // recomputes its fused masses
       const bool stored = (r_ok == (!bonus || P.full));
-      sample = tile_walk<T>(static_cast<const T*>(P.a) + off, static_cast<const T*>(P.b) + off,
-                            static_cast<const T*>(P.t) + off, nvec, t0, P.beta,
-                            S.ws.groups + (row * S.NT + owner) * kSGroups, stored, r_ok,
-                            st.lse[0] * kLog2e, st.lse[3] * kLog2e, tau_local);
+      sample = group_walk<T, true>(static_cast<const T*>(P.a) + off,
+                                   static_cast<const T*>(P.b) + off,
+                                   static_cast<const T*>(P.t) + off, nvec, t0, kSGroups, P.beta,
+                                   S.ws.groups + (row * S.NT + owner) * kSGroups, stored, r_ok,
+                                   st.lse[0] * kLog2e, st.lse[3] * kLog2e, tau_local);
     }
   }
   const bool has_ab = P.full || !bonus;

@@ -74,10 +74,12 @@ struct __align__(16) X2 {  // pass-2 sums
   float pad[3];
 };
 
-// Fixed part of the shared state; the C pass-1 and C pass-2 records pushed
-// by the cluster follow it (recv1(), recv2()).
+// Fixed part of the shared state; the C pass-1 records pushed by the
+// cluster and the C pass-2 records sent to rank 0 follow it (recv1(),
+// recv2()), then, in stochastic mode, the inverse-CDF group masses.
 struct __align__(16) SharedTma {
   unsigned long long bar[kChunks];  // one mbarrier per chunk
+  unsigned long long b2_bar;        // rank 0: every CTA's pass-2 record has arrived
   union {                           // per-warp records, one pass at a time
     X1 w1[kTWarps];
     X2 w2[kTWarps];
@@ -87,7 +89,7 @@ struct __align__(16) SharedTma {
   unsigned bad;
   float da, db, dt;
   unsigned broken;
-  unsigned pad[3];
+  unsigned pad;
   __device__ X1* recv1() { return reinterpret_cast<X1*>(this + 1); }
   __device__ X2* recv2(int C) { return reinterpret_cast<X2*>(recv1() + C); }
 };
@@ -97,13 +99,17 @@ static_assert(sizeof(X1) % 16 == 0 && alignof(X1) == 16, "X1 must be 16-byte ali
 static_assert(sizeof(X2) % 16 == 0 && alignof(X2) == 16, "X2 must be 16-byte aligned");
 static_assert(sizeof(SharedTma) % 16 == 0, "records after SharedTma must stay 16-byte aligned");
 
-// Shared bytes after the slices for a cluster of C CTAs (the stochastic
-// kernel adds rounds * kTThreads floats of per-vector masses).
+// Inverse-CDF groups: group g of a slice is the 32 vectors of warp (g % 8)
+// in round g / 8, i.e. vectors [32 g, 32 g + 32) in index order.
+constexpr int kGroupsMax = kMaxRounds * kTWarps;
+
+// Shared bytes after the slices for a cluster of C CTAs.  The stochastic
+// kernel adds this CTA's group masses and, in rank 0, every rank's.
 __host__ __device__ constexpr int shared_tma_bytes(int C) {
   return static_cast<int>(sizeof(SharedTma) + C * (sizeof(X1) + sizeof(X2)));
 }
-__host__ __device__ constexpr int mass_bytes(int rounds) {
-  return rounds * kTThreads * static_cast<int>(sizeof(float));
+__host__ __device__ constexpr int group_bytes(int C) {
+  return (C + 1) * kGroupsMax * static_cast<int>(sizeof(float));
 }
 
 __device__ __forceinline__ X1 x1_neutral() {
@@ -668,7 +674,7 @@ __device__ __forceinline__ void div_terms(const f2 (&xa)[NP], const f2 (&xb)[NP]
 template <typename T, unsigned G, bool LP>
 __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int nv, int rounds,
                                       float beta, float A2, float B2, float S2, float lse_s, X2& x,
-                                      float* lp, float* vmass) {
+                                      float* lp, float* grp) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
   constexpr bool JSD = (G & G_JSD) != 0, KL = (G & G_KL) != 0, RES = (G & G_RES) != 0;
@@ -680,16 +686,12 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
   const f2 tiny2 = pk(kMinNormal, kMinNormal);
   const f2 nl2 = pk(-lse_s, -lse_s);
   f2 ja = 0ull, jb = 0ull, ms2 = 0ull, kl2 = 0ull, R2 = 0ull, Q2 = 0ull;
+  const int warp = static_cast<int>(threadIdx.x) >> 5;
   for (int kr = 0; kr < rounds; kr += 2) {
     const int i0 = kr * kTThreads + static_cast<int>(threadIdx.x);
     const int i1 = i0 + kTThreads;
-    if (i0 >= nv) {
-      if (RES || QF) {
-        vmass[kr * kTThreads + threadIdx.x] = 0.f;
-        if (kr + 1 < rounds) vmass[(kr + 1) * kTThreads + threadIdx.x] = 0.f;
-      }
-      continue;
-    }
+    float g0 = 0.f, g1 = 0.f;  // this thread's vector masses in rounds kr and kr + 1
+    if (i0 < nv) {
     const bool has1 = i1 < nv;
     f2 xa[NP], xb[NP], xt[NP], ya[NP], yb[NP], yt[NP];
     load_pairs(ra + i0 * VE, xa);
@@ -707,11 +709,10 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
       vec_masses(ya, yb, yt, beta2, L2, nA2, nS2, py, qy, ry);
 #pragma unroll
       for (int h = 0; h < NP; ++h) Q2 = add2(Q2, add2(qx[h], qy[h]));
-      // residual mass of each vector, kept for the inverse-CDF walk
-      const float r0 = vsum(rx), r1 = vsum(ry);
-      R2 = add2(R2, pk(r0, r1));
-      vmass[kr * kTThreads + threadIdx.x] = r0;
-      if (kr + 1 < rounds) vmass[(kr + 1) * kTThreads + threadIdx.x] = r1;
+      // residual mass of each vector, summed per group for the inverse-CDF walk
+      g0 = vsum(rx);
+      g1 = vsum(ry);
+      R2 = add2(R2, pk(g0, g1));
     } else if (QF) {
       f2 qx[NP], qy[NP];
 #pragma unroll
@@ -719,11 +720,10 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
         qx[h] = ex2_2(fma2(fma2(beta2, sub2(xa[h], xb[h]), xt[h]), L2, nS2));
         qy[h] = ex2_2(fma2(fma2(beta2, sub2(ya[h], yb[h]), yt[h]), L2, nS2));
       }
-      // fused mass of each vector, kept for the inverse-CDF walk
-      const float q0 = vsum(qx), q1 = vsum(qy);
-      Q2 = add2(Q2, pk(q0, q1));
-      vmass[kr * kTThreads + threadIdx.x] = q0;
-      if (kr + 1 < rounds) vmass[(kr + 1) * kTThreads + threadIdx.x] = q1;
+      // fused mass of each vector, summed per group for the inverse-CDF walk
+      g0 = vsum(qx);
+      g1 = vsum(qy);
+      Q2 = add2(Q2, pk(g0, g1));
     } else if (JSD || KL) {
 #pragma unroll
       for (int h = 0; h < NP; ++h) {
@@ -749,6 +749,14 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
         }
       }
     }
+    }
+    if (RES || QF) {  // group masses: every lane takes part, with or without a vector
+      const float s0 = warp_sum(g0), s1 = warp_sum(g1);
+      if ((threadIdx.x & 31) == 0) {
+        grp[kr * kTWarps + warp] = s0;
+        if (kr + 1 < rounds) grp[(kr + 1) * kTWarps + warp] = s1;
+      }
+    }
   }
   x.j = hsum2(add2(ja, jb));
   x.msum = hsum2(ms2);
@@ -757,27 +765,36 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
   x.Q = hsum2(Q2);
 }
 
-// Pass 2's per-warp sums, the CTA combine, pushed to every CTA, up to and
-// including cluster barrier B2.
+// Pass 2, the CTA combine, and a one-way send to rank 0: every CTA's pass-2
+// record and group masses go into rank 0's shared memory, then each lane of
+// warp 0 arrives (release, cluster scope) on rank 0's b2_bar, whose count is
+// 32 C.  Only rank 0 waits for it; the other CTAs are done.
 template <typename T, unsigned G, bool LP>
-__device__ __forceinline__ void pass2_and_push(const T* ra, const T* rb, const T* rt, int nv,
+__device__ __forceinline__ void pass2_and_send(const T* ra, const T* rb, const T* rt, int nv,
                                                int rounds, float beta, float* lp, SharedTma* sh,
-                                               int rank, int C, float* vmass,
+                                               int rank, int C, float* groups,
                                                cg::cluster_group& cluster) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
   X2 x = x2_zero();
   pass2<T, G, LP>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e, lse_s * kLog2e,
-                  lse_s, x, lp, vmass);
+                  lse_s, x, lp, groups);
   warp_reduce_x2<G>(x);
   if (lane == 0) sh->w2[warp] = x;
   __syncthreads();
   if (warp == 0) {
     X2 w = (lane < kTWarps) ? sh->w2[lane] : x2_zero();
     warp_reduce_x2<G>(w);
-    push_record(w, sh->recv2(C), rank, C, cluster);
+    X2* rec = cluster.map_shared_rank(sh->recv2(C), 0) + rank;
+    if (lane < static_cast<int>(sizeof(X2) / 16))
+      reinterpret_cast<float4*>(rec)[lane] = reinterpret_cast<const float4*>(&w)[lane];
+    if (G & (G_RES | G_QF)) {
+      float* dst = cluster.map_shared_rank(groups, 0) + kGroupsMax * (1 + rank);
+      if (lane < kGroupsMax / 4)
+        reinterpret_cast<float4*>(dst)[lane] = reinterpret_cast<const float4*>(groups)[lane];
+    }
+    mbar_arrive_remote(&sh->b2_bar, 0);
   }
-  cluster_barrier(warp == 0);  // B2: every CTA's pass-2 record is in every CTA
 }
 
 // The divergence of Eq. 3 from the summed pass-2 records (nats).
@@ -790,161 +807,153 @@ __device__ __forceinline__ float divergence_of(const X2& tot) {
 
 // ---------------------------------------------------------------- inverse-CDF walk
 
-// Residual (use_r) or fused mass of vector i of the slice, summed.
+// Masses of vector v of a slice held in global memory, as pass 2 computes them.
 template <typename T>
-__device__ __forceinline__ float vec_mass(const T* ra, const T* rb, const T* rt, int i, bool use_r,
-                                          f2 beta2, f2 L2, f2 nA2, f2 nS2) {
+__device__ __forceinline__ void slice_vector_masses(const T* ga, const T* gb, const T* gt, int v,
+                                                    f2 beta2, f2 L2, f2 nA2, f2 nS2,
+                                                    f2 (&p)[8 / sizeof(T)],
+                                                    f2 (&qf)[8 / sizeof(T)],
+                                                    f2 (&r)[8 / sizeof(T)]) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
-  f2 xa[NP], xb[NP], xt[NP], p[NP], qf[NP], r[NP];
-  load_pairs(ra + i * VE, xa);
-  load_pairs(rb + i * VE, xb);
-  load_pairs(rt + i * VE, xt);
+  f2 xa[NP], xb[NP], xt[NP];
+  load_pairs(ga + v * VE, xa);
+  load_pairs(gb + v * VE, xb);
+  load_pairs(gt + v * VE, xt);
   vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
-  return use_r ? vsum(r) : vsum(qf);
 }
 
-// Mass of vector i of the slice as pass 2 left it (stored) or recomputed.
-template <typename T>
-__device__ __forceinline__ float walk_mass(const T* ra, const T* rb, const T* rt, int i, int nv,
-                                           const float* vmass, int j, int t, bool stored,
-                                           bool use_r, f2 beta2, f2 L2, f2 nA2, f2 nS2) {
-  if (i >= nv) return 0.f;
-  if (stored) return vmass[j * kTThreads + t];
-  return vec_mass(ra, rb, rt, i, use_r, beta2, L2, nA2, nS2);
-}
-
-// The inverse-CDF draw inside the CTA that owns the target, by one warp: the
-// smallest slice index (order: round, thread, element) whose cumulative
-// residual (use_r) or fused mass exceeds tau, or the last index with positive
-// mass when rounding leaves tau at or beyond the slice's total.  Lane l covers
-// the vectors of threads 8l .. 8l+7 in every round.  Returns the index within
-// the row (every lane), or -1 when the slice holds no mass.
-template <typename T>
-__device__ int walk_warp(const T* ra, const T* rb, const T* rt, int nv, int rounds, int lo,
-                         float beta, const float* vmass, bool stored, bool use_r, float A2,
-                         float S2, float tau) {
+// The inverse-CDF draw inside one slice, by one warp: the smallest slice
+// index (index order) whose cumulative residual (use_r) or fused mass
+// exceeds tau, or the last index with positive mass when rounding leaves tau
+// at or beyond the slice's total.  The slice (ga, gb, gt: global memory,
+// entries from lo) is cut into groups of 32 vectors; gm holds their masses
+// when `stored` (else they are recomputed: the rare fallback to the fused
+// masses of a draft row whose residual is zero).  Lane l takes groups 3l to
+// 3l+2, then the lane holding the target recomputes its group's vectors,
+// one per lane, and the element.  Returns the index within the row, or -1
+// when the slice holds no mass.
+template <typename T, bool GM_GLOBAL>
+__device__ __noinline__ int group_walk(const T* ga, const T* gb, const T* gt, int nvec, int lo,
+                                       int ngroups, float beta, const float* gm, bool stored,
+                                       bool use_r, float A2, float S2, float tau) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
-  constexpr int TPL = kTThreads / 32;  // threads (vectors per round) per lane
   const int lane = threadIdx.x & 31;
   const f2 beta2 = pk(beta, beta), L2 = pk(kLog2e, kLog2e);
   const f2 nA2 = pk(-A2, -A2), nS2 = pk(-S2, -S2);
-  float P[kMaxRounds], Tj[kMaxRounds];
+  float g3[3];
 #pragma unroll
-  for (int j = 0; j < kMaxRounds; ++j) {
-    float p = 0.f;
-    if (j < rounds) {
+  for (int h = 0; h < 3; ++h) {
+    const int g = 3 * lane + h;
+    float m = 0.f;
+    if (g < ngroups) {
       if (stored) {
-        const float4 m0 = *reinterpret_cast<const float4*>(vmass + j * kTThreads + TPL * lane);
-        const float4 m1 = *reinterpret_cast<const float4*>(vmass + j * kTThreads + TPL * lane + 4);
-        p = ((((((m0.x + m0.y) + m0.z) + m0.w) + m1.x) + m1.y) + m1.z) + m1.w;
+        m = GM_GLOBAL ? __ldcg(gm + g) : gm[g];
       } else {
-#pragma unroll 1
-        for (int v = 0; v < TPL; ++v) {
-          const int t = TPL * lane + v;
-          p += walk_mass(ra, rb, rt, j * kTThreads + t, nv, vmass, j, t, false, use_r, beta2, L2,
-                         nA2, nS2);
+        for (int u = 0; u < 32; ++u) {
+          const int v = 32 * g + u;
+          if (v < nvec) {
+            f2 p[NP], qf[NP], r[NP];
+            slice_vector_masses(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
+            m += vsum(use_r ? r : qf);
+          }
         }
       }
     }
-    P[j] = p;
-    Tj[j] = (j < rounds) ? warp_sum(p) : 0.f;
+    g3[h] = m;
   }
-  // the round holding the target
-  int js = -1, jlast = -1;
-  float cum = 0.f, tj = 0.f;
-#pragma unroll
-  for (int j = 0; j < kMaxRounds; ++j) {
-    if (j < rounds) {
-      if (js < 0) {
-        if (cum + Tj[j] > tau) {
-          js = j;
-          tj = fmaxf(tau - cum, 0.f);
-        } else {
-          cum += Tj[j];
-        }
-      }
-      if (Tj[j] > 0.f) jlast = j;
-    }
-  }
-  bool take_last = false;
-  if (js < 0) {
-    if (jlast < 0) return -1;
-    js = jlast;
-    take_last = true;
-  }
-  float pj = 0.f;
-#pragma unroll
-  for (int j = 0; j < kMaxRounds; ++j)
-    if (j == js) pj = P[j];
-  // the lane holding it: inclusive prefix over lanes
-  float incl = pj;
+  const float pl = (g3[0] + g3[1]) + g3[2];
+  float incl = pl;
 #pragma unroll
   for (int off = 1; off < 32; off <<= 1) {
     const float v = __shfl_up_sync(0xffffffffu, incl, off);
     if (lane >= off) incl += v;
   }
-  const float excl = incl - pj;
-  const unsigned hit = __ballot_sync(0xffffffffu, !take_last && pj > 0.f && excl <= tj && tj < incl);
+  const float excl = incl - pl;
+  bool take_last = false;
+  const unsigned hit = __ballot_sync(0xffffffffu, pl > 0.f && excl <= tau && tau < incl);
   int lc;
   if (hit) {
     lc = __ffs(hit) - 1;
   } else {
-    const unsigned pos = __ballot_sync(0xffffffffu, pj > 0.f);
+    const unsigned pos = __ballot_sync(0xffffffffu, pl > 0.f);
     if (!pos) return -1;
     lc = 31 - __clz(pos);
     take_last = true;
   }
-  int found = -1;
+  // the group, within lane lc
+  int gsel = -1;
+  float trem = 0.f;
   if (lane == lc) {
-    // its vector, then the element
-    float cum2 = excl, trem = 0.f;
-    int vsel = -1, vlast = -1;
-    for (int v = 0; v < TPL; ++v) {
-      const int t = TPL * lane + v;
-      const float m = walk_mass(ra, rb, rt, js * kTThreads + t, nv, vmass, js, t, stored, use_r,
-                                beta2, L2, nA2, nS2);
-      if (m > 0.f) vlast = v;
-      if (!take_last && vsel < 0) {
-        if (cum2 + m > tj) {
-          vsel = v;
-          trem = fmaxf(tj - cum2, 0.f);
+    float cum = excl;
+    int glast = -1;
+#pragma unroll
+    for (int h = 0; h < 3; ++h) {
+      if (g3[h] > 0.f) glast = 3 * lane + h;
+      if (!take_last && gsel < 0) {
+        if (cum + g3[h] > tau) {
+          gsel = 3 * lane + h;
+          trem = fmaxf(tau - cum, 0.f);
         } else {
-          cum2 += m;
+          cum += g3[h];
         }
       }
     }
-    bool last_el = take_last;
-    if (vsel < 0) {
-      vsel = vlast;
-      last_el = true;
-    }
-    if (vsel >= 0) {
-      const int i = js * kTThreads + TPL * lane + vsel;
-      f2 xa[NP], xb[NP], xt[NP], p[NP], qf[NP], r[NP];
-      load_pairs(ra + i * VE, xa);
-      load_pairs(rb + i * VE, xb);
-      load_pairs(rt + i * VE, xt);
-      vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
-      float cum3 = 0.f;
-      int pick = -1, last = -1;
-#pragma unroll
-      for (int h = 0; h < NP; ++h) {
-        float v0, v1;
-        upk(use_r ? r[h] : qf[h], v0, v1);
-        if (v0 > 0.f) last = 2 * h;
-        cum3 += v0;
-        if (!last_el && pick < 0 && cum3 > trem) pick = 2 * h;
-        if (v1 > 0.f) last = 2 * h + 1;
-        cum3 += v1;
-        if (!last_el && pick < 0 && cum3 > trem) pick = 2 * h + 1;
-      }
-      if (pick < 0) pick = last;
-      if (pick >= 0) found = lo + i * VE + pick;
+    if (gsel < 0) {
+      gsel = glast;
+      take_last = true;
     }
   }
-  return __shfl_sync(0xffffffffu, found, lc);
+  gsel = __shfl_sync(0xffffffffu, gsel, lc);
+  trem = __shfl_sync(0xffffffffu, trem, lc);
+  take_last = __shfl_sync(0xffffffffu, take_last ? 1 : 0, lc) != 0;
+  // the vector: lane u recomputes vector 32 gsel + u
+  const int v = 32 * gsel + lane;
+  f2 p[NP], qf[NP], r[NP];
+  float mv = 0.f;
+  if (v < nvec) {
+    slice_vector_masses(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
+    mv = vsum(use_r ? r : qf);
+  }
+  float vin = mv;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float w = __shfl_up_sync(0xffffffffu, vin, off);
+    if (lane >= off) vin += w;
+  }
+  const float vex = vin - mv;
+  const unsigned vh =
+      __ballot_sync(0xffffffffu, !take_last && mv > 0.f && vex <= trem && trem < vin);
+  int vc;
+  if (vh) {
+    vc = __ffs(vh) - 1;
+  } else {
+    const unsigned pos = __ballot_sync(0xffffffffu, mv > 0.f);
+    if (!pos) return -1;
+    vc = 31 - __clz(pos);
+    take_last = true;
+  }
+  int found = -1;
+  if (lane == vc) {
+    const float te = fmaxf(trem - vex, 0.f);
+    float cum = 0.f;
+    int pick = -1, last = -1;
+#pragma unroll
+    for (int h = 0; h < NP; ++h) {
+      float v0, v1;
+      upk(use_r ? r[h] : qf[h], v0, v1);
+      if (v0 > 0.f) last = 2 * h;
+      cum += v0;
+      if (!take_last && pick < 0 && cum > te) pick = 2 * h;
+      if (v1 > 0.f) last = 2 * h + 1;
+      cum += v1;
+      if (!take_last && pick < 0 && cum > te) pick = 2 * h + 1;
+    }
+    if (pick < 0) pick = last;
+    if (pick >= 0) found = lo + v * VE + pick;
+  }
+  return __shfl_sync(0xffffffffu, found, vc);
 }
 
 // ---------------------------------------------------------------- the kernel
@@ -959,7 +968,7 @@ struct RowCtx {
   bool bonus;
   int dtok;           // warp 0 only
   RowScalars sc;      // warp 0 only (stochastic)
-  float* vmass;
+  float* groups;      // stochastic: this CTA's group masses, then (rank 0) every rank's
   SharedTma* sh;
 };
 
@@ -1024,11 +1033,16 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
     }
     __syncthreads();
     float* lp = LP ? P.logprobs + static_cast<size_t>(c.row) * P.V + c.lo : nullptr;
-    pass2_and_push<T, G, LP>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh, c.rank, c.C, c.vmass,
+    pass2_and_send<T, G, LP>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh, c.rank, c.C, c.groups,
                              cluster);
-    if (warp != 0) return;  // the rest is warp 0's
+    if (c.rank != 0 || warp != 0) return;  // the rest is rank 0's warp 0
+    unsigned bad = sh->bad;
+    if (!mbar_wait_cluster_bounded(&sh->b2_bar, 0, kCopyTimeoutNs)) bad |= kBadTimeout;
     const X2 w = (lane < c.C) ? sh->recv2(c.C)[lane] : x2_zero();
     const float lse[4] = {sh->lse[0], sh->lse[1], sh->lse[2], sh->lse[3]};
+    X2 tot = w;
+    warp_reduce_x2<G>(tot);
+    const float D = divergence_of<G>(tot);
     if constexpr (STOCH) {
       // inclusive prefix of the inverse-CDF mass over ranks, in rank order
       float incl_R = w.R, incl_Q = w.Q;
@@ -1053,29 +1067,30 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
       int owner = -1;
       if (over) owner = __ffs(over) - 1;
       else if (pos) owner = 31 - __clz(pos);
-      if (c.rank != owner && !(owner < 0 && c.rank == 0)) return;
-      X2 tot = w;
-      warp_reduce_x2<G>(tot);
-      const float D = divergence_of<G>(tot);
       int sample = -1;
       if (owner >= 0) {
         const float incl_o = __shfl_sync(0xffffffffu, incl, owner);
         const float mass_o = __shfl_sync(0xffffffffu, mass, owner);
         const float tau_local = fmaxf(tau - (incl_o - mass_o), 0.f);
-        // pass 2 kept the residual masses of draft rows and the fused masses
-        // of the bonus row; the other kind (a draft row whose residual is
+        // the owner's slice, read back from global memory (L2)
+        constexpr int VE = 16 / static_cast<int>(sizeof(T));
+        const int lo_o = owner * c.W;
+        const int nv_o = max(0, min(c.W, P.V - lo_o)) / VE;
+        const int ng_o = ((nv_o + kTThreads - 1) / kTThreads) * kTWarps;
+        const size_t off = static_cast<size_t>(c.row) * P.V + lo_o;
+        // pass 2 kept the residual group masses of draft rows and the fused
+        // ones of the bonus row; the other kind (a draft row whose residual is
         // zero) is recomputed exactly as pass 2 computes it
         const bool stored_r = !c.bonus || P.full;
-        sample = walk_warp<T>(ra, rb, rt, c.nv, c.rounds, c.lo, beta, c.vmass, r_ok == stored_r,
-                              r_ok, lse[0] * kLog2e, lse[3] * kLog2e, tau_local);
+        sample = group_walk<T, false>(static_cast<const T*>(P.a) + off,
+                                      static_cast<const T*>(P.b) + off,
+                                      static_cast<const T*>(P.t) + off, nv_o, lo_o, ng_o, beta,
+                                      c.groups + kGroupsMax * (1 + owner), r_ok == stored_r, r_ok,
+                                      lse[0] * kLog2e, lse[3] * kLog2e, tau_local);
       }
-      finish<STOCH>(P, c, lse, sh->is, sh->it, sh->bad, D, sample, total, sh->da, sh->db, sh->dt);
+      finish<STOCH>(P, c, lse, sh->is, sh->it, bad, D, sample, total, sh->da, sh->db, sh->dt);
     } else {
-      if (c.rank != 0) return;
-      X2 tot = w;
-      warp_reduce_x2<G>(tot);
-      finish<STOCH>(P, c, lse, sh->is, sh->it, sh->bad, divergence_of<G>(tot), -1, NAN, sh->da,
-                    sh->db, sh->dt);
+      finish<STOCH>(P, c, lse, sh->is, sh->it, bad, D, -1, NAN, sh->da, sh->db, sh->dt);
     }
   }
 }
@@ -1120,14 +1135,16 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   T* sb = sa + W;
   T* st = sb + W;
   SharedTma* sh = reinterpret_cast<SharedTma*>(smem_tma + P.sh_off);
-  // stochastic: per-thread, per-round sampling masses after the records
-  float* vmass = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sh) +
-                                          shared_tma_bytes(C));
+  // stochastic: inverse-CDF group masses after the records
+  float* groups = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sh) +
+                                           shared_tma_bytes(C));
   const bool only_t = !STOCH && !P.full && bonus && !P.fuse_bonus;
 
   if (tid == 0) {
 #pragma unroll
     for (int c = 0; c < kChunks; ++c) mbar_init(&sh->bar[c], 1);
+    // one arrive per lane of warp 0 of every CTA; B1 orders this before any
+    mbar_init(&sh->b2_bar, 32u * static_cast<unsigned>(C));
     sh->broken = 0;
     fence_mbar_init();
     issue_slice<T>(P, sh, row, lo, nv, rc, sa, sb, st, only_t);
@@ -1148,7 +1165,7 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   c.bi = bi;
   c.row = row;
   c.bonus = bonus;
-  c.vmass = vmass;
+  c.groups = groups;
   c.sh = sh;
   c.dtok = -1;
   c.sc = RowScalars{0.f, 0.f, 0.f};
