@@ -128,12 +128,18 @@ typedef struct {
 void asymspec_default_gate_params(asymspec_gate_params* p);
 
 /* Bytes of device workspace asymspec_fuse_verify_ex needs for a batch of
- * B elements with K drafts and V vocabulary entries (enough for every kernel
- * and both dtypes).  The cluster kernels (the automatic choice) need only
- * 16 B per row plus 4 B per element, the first 256-byte aligned parts of the
- * same layout; the rest serves ASYMSPEC_KERNEL_STREAM.  The workspace must be zeroed once before its first use (cudaMemset
- * or asymspec_workspace_reset); every call that completes leaves it zeroed
- * again.  Two calls in flight at the same time must not share a workspace. */
+ * B elements with K drafts and V vocabulary entries (enough for every kernel,
+ * cluster size and dtype).  Layout, each part 256-byte aligned: 16 B of row
+ * record per row and 4 B of ticket per element (all the generic kernel
+ * needs); then, for ASYMSPEC_KERNEL_TMA with clusters of C CTAs, 48 B of
+ * pass-1 results per row and 352 B per row and CTA of pass-2 record and
+ * inverse-CDF group masses, which its decision kernel reads; or instead the
+ * streaming kernel's counters and tile records.  With less than the TMA
+ * part the automatic choice falls back to the generic kernel.  The tickets
+ * must be zero before the first use (cudaMemset or
+ * asymspec_workspace_reset); every call that completes leaves them zero
+ * again, and every other part is written before it is read.  Two calls in
+ * flight at the same time must not share a workspace. */
 size_t asymspec_workspace_bytes(int B, int K, int V);
 
 /* Enqueues a zero fill of a workspace on `stream`. */
@@ -193,15 +199,17 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
  * grow and trim, and plain C hosts that have no device allocator to provide
  * the workspace asymspec_fuse_verify_ex wants.
  *
- * Scratch: the per-row records and per-element tickets live in one file-scope
- * static __device__ array of the library, sized for B*(K+1) <= 8192 rows
- * (147,456 bytes: 16 bytes per row and 4 per batch element).  Larger batches
- * return ASYMSPEC_ERR_SCRATCH_LIMIT before anything is enqueued.  Each call
- * enqueues on `stream` a zero fill of the B tickets (the only part that must
- * start at zero; the records are written before they are read), then the
- * launch of asymspec_fuse_verify_ex, which with this scratch runs the cluster
- * kernels (ASYMSPEC_KERNEL_TMA for aligned rows, else _GENERIC).  Nothing is allocated: no cudaMalloc,
- * cudaMallocAsync, cudaFree or library call that allocates.
+ * Scratch: one file-scope static __device__ array of the library
+ * (ASYMSPEC_STATIC_SCRATCH_BYTES, 4 MiB),
+ * used as asymspec_fuse_verify_ex uses a workspace.  It holds the generic
+ * kernel's records and tickets for B*(K+1) <= 8192 rows (16 bytes per row
+ * and 4 per batch element); larger batches return ASYMSPEC_ERR_SCRATCH_LIMIT
+ * before anything is enqueued.  Aligned rows run ASYMSPEC_KERNEL_TMA when
+ * the array also holds its per-row results (about 1400 rows in clusters of
+ * 8), else the generic kernel.  Each call enqueues on `stream` a zero fill
+ * of the B tickets (the only part that must start at zero), then the
+ * launches of asymspec_fuse_verify_ex.  Nothing is allocated: no
+ * cudaMalloc, cudaMallocAsync, cudaFree or library call that allocates.
  *
  * Set-up: the first call on each device looks up the array's device address
  * with cudaGetSymbolAddress (return code checked, ASYMSPEC_ERR_CUDA on
@@ -215,6 +223,7 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
  * Arguments, outputs and status codes are those of asymspec_fuse_verify.
  */
 #define ASYMSPEC_STATIC_MAX_ROWS 8192
+#define ASYMSPEC_STATIC_SCRATCH_BYTES (4u << 20)
 int asymspec_fuse_verify_static(const void* logits_full, const void* logits_comp,
                                 const void* logits_ver, const int32_t* draft_tokens,
                                 const float* draft_probs, const float* uniforms, int B, int K,

@@ -26,6 +26,7 @@ ERR_TOO_LARGE = -6
 ERR_SCRATCH_LIMIT = -7
 
 STATIC_MAX_ROWS = 8192  # B*(K+1) limit of fuse_verify_static
+STATIC_SCRATCH_BYTES = 4 << 20  # size of fuse_verify_static's scratch array
 
 DATA_BAD_TOKEN = 0x1
 DATA_NONFINITE = 0x2

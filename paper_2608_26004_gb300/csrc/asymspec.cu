@@ -71,13 +71,13 @@ bool plan_generic(int V, int elt, int VE, int forced_C, Plan* pl) {
 // TMA kernel: first C whose slice (and shared state) fits two CTAs per SM,
 // else the first that fits one; a slice holds at most kMaxRounds vectors
 // per thread.
-bool plan_tma(int V, int elt, int forced_C, bool stoch, Plan* pl) {
+bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
   const int VE = 16 / elt;
   auto fill = [&](int C) {
     const long long per = (static_cast<long long>(V) + C - 1) / C;
     const long long W = round_up_ll(per, VE);
     const int rounds = static_cast<int>((W / VE + kTThreads - 1) / kTThreads);
-    const int shared_bytes = shared_tma_bytes(C) + (stoch ? group_bytes(C) : 0);
+    const int shared_bytes = shared_tma_bytes(C);
     const long long sh_off = round_up_ll(3 * W * elt, 128);
     pl->C = C;
     pl->W = static_cast<int>(W);
@@ -102,6 +102,28 @@ size_t ws_records_bytes(int B, int K) {
 
 size_t cluster_ws_bytes(int B, int K) {
   return ws_records_bytes(B, K) + round_up(static_cast<size_t>(B) * sizeof(unsigned), 256);
+}
+
+// Workspace of the cluster TMA kernel for clusters of C CTAs: the records
+// and tickets first (same offsets), then what each row leaves for the
+// decision kernel: the row's pass-1 results, one pass-2 record per CTA and
+// each CTA's inverse-CDF group masses.
+struct TmaLayout {
+  size_t stat, p2rec, groups, total;
+};
+
+TmaLayout tma_layout(int B, int K, int C) {
+  TmaLayout L;
+  const size_t R = static_cast<size_t>(B) * (K + 1);
+  size_t off = cluster_ws_bytes(B, K);
+  L.stat = off;
+  off += round_up(R * sizeof(RowStat), 256);
+  L.p2rec = off;
+  off += round_up(R * C * sizeof(X2), 256);
+  L.groups = off;
+  off += round_up(R * C * kGroupsMax * sizeof(float), 256);
+  L.total = off;
+  return L;
 }
 
 // Workspace of the streaming kernel: the cluster kernels' records and
@@ -173,10 +195,16 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
   }
   if (ws_bytes < cluster_ws_bytes(B, K)) return ASYMSPEC_ERR_WORKSPACE;
   bool ok = false;
-  if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, stoch, pl)) {
-    pl->kernel = ASYMSPEC_KERNEL_TMA;
-    pl->VE = 16 / elt;
-    ok = true;
+  if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, pl)) {
+    // the TMA kernel leaves each row's results in the workspace; the generic
+    // kernel, which needs only the records and tickets, runs when it is short
+    if (ws_bytes >= tma_layout(B, K, pl->C).total) {
+      pl->kernel = ASYMSPEC_KERNEL_TMA;
+      pl->VE = 16 / elt;
+      ok = true;
+    } else if (forced_kernel == ASYMSPEC_KERNEL_TMA) {
+      return ASYMSPEC_ERR_WORKSPACE;
+    }
   } else if (forced_kernel == ASYMSPEC_KERNEL_TMA) {
     return vec_ok ? ASYMSPEC_ERR_TOO_LARGE : ASYMSPEC_ERR_UNSUPPORTED;
   }
@@ -196,6 +224,10 @@ KernelFn pick_kernel(const Plan& pl, int dtype, bool stoch) {
   if (pl.kernel == ASYMSPEC_KERNEL_TMA)
     return dtype == ASYMSPEC_FP32 ? tma_kernel_f32(stoch) : tma_kernel_bf16(stoch);
   return generic_kernel(dtype, pl.vector_path, stoch);
+}
+
+KernelFn pick_decide(int dtype, bool stoch) {
+  return dtype == ASYMSPEC_FP32 ? decide_kernel_f32(stoch) : decide_kernel_bf16(stoch);
 }
 
 // Per (kernel, device): attributes set once; cluster occupancy cached per
@@ -345,15 +377,17 @@ int check_opts(const asymspec_launch_opts* opts) {
   return ASYMSPEC_OK;
 }
 
-// Scratch of asymspec_fuse_verify_static: records for ASYMSPEC_STATIC_MAX_ROWS
-// rows, then tickets for the largest batch that can have that many rows
-// (K >= 1, so B <= ASYMSPEC_STATIC_MAX_ROWS / 2).  The layout is the one
-// asymspec_fuse_verify_ex gives any workspace, so every batch within the limit
-// fits: records end by 16 * MAX_ROWS bytes, tickets by 4 * MAX_ROWS / 2 more.
-constexpr size_t kStaticScratchBytes =
-    static_cast<size_t>(ASYMSPEC_STATIC_MAX_ROWS) * sizeof(int4) +
-    static_cast<size_t>(ASYMSPEC_STATIC_MAX_ROWS / 2) * sizeof(unsigned);
-static_assert(kStaticScratchBytes % 256 == 0, "static scratch ends on a 256-byte boundary");
+// Scratch of asymspec_fuse_verify_static, used as asymspec_fuse_verify_ex
+// uses any workspace.  The generic kernel needs records for
+// ASYMSPEC_STATIC_MAX_ROWS rows and tickets for the largest batch that can
+// have that many rows (K >= 1, so B <= ASYMSPEC_STATIC_MAX_ROWS / 2): 144 KiB.
+// 4 MiB also holds the TMA kernel's per-row results for about 1400 rows in
+// clusters of 8 (2880 bytes a row); larger batches take the generic kernel.
+constexpr size_t kStaticScratchBytes = ASYMSPEC_STATIC_SCRATCH_BYTES;
+static_assert(kStaticScratchBytes >= static_cast<size_t>(ASYMSPEC_STATIC_MAX_ROWS) * sizeof(int4) +
+                                         static_cast<size_t>(ASYMSPEC_STATIC_MAX_ROWS / 2) *
+                                             sizeof(unsigned),
+              "the static scratch holds the generic kernel's records and tickets");
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
 // Device address of g_static_scratch, looked up once per device.
@@ -394,7 +428,8 @@ void asymspec_default_gate_params(asymspec_gate_params* p) {
 
 size_t asymspec_workspace_bytes(int B, int K, int V) {
   if (B < 1 || K < 1) return 0;
-  size_t n = cluster_ws_bytes(B, K);
+  // the TMA kernel's layout for the largest cluster
+  size_t n = tma_layout(B, K, 16).total;
   if (V >= 2) {
     // the larger of the two dtypes' streaming layouts (fp32 has more tiles)
     const StreamLayout L4 = stream_layout(B, K, V, 4);
@@ -540,6 +575,9 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   P.logprobs = out_fused_logprobs;
   P.err_word = out_error_word;
   P.recs = static_cast<int4*>(workspace);
+  P.row_stat = nullptr;
+  P.pass2_rec = nullptr;
+  P.group_mass = nullptr;
   P.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) +
                                               ws_records_bytes(B, K));
 
@@ -604,8 +642,22 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = launch_config(pl, ctas, static_cast<cudaStream_t>(stream), attr);
   void* args[] = {&P};
+  if (pl.kernel == ASYMSPEC_KERNEL_TMA) {
+    const TmaLayout L = tma_layout(B, K, pl.C);
+    char* base = static_cast<char*>(workspace);
+    P.row_stat = base + L.stat;
+    P.pass2_rec = reinterpret_cast<float*>(base + L.p2rec);
+    P.group_mass = reinterpret_cast<float*>(base + L.groups);
+  }
   e = cudaLaunchKernelExC(&cfg, fn, args);
   if (e != cudaSuccess) return cuda_fail(e);
+  if (pl.kernel == ASYMSPEC_KERNEL_TMA) {
+    // the rows' decisions and Algorithm 1's scan: one CTA per batch element
+    const int warps = std::min(K + 1, kDecideThreads / 32);
+    e = cudaLaunchKernel(pick_decide(dtype, stoch), dim3(static_cast<unsigned>(B)),
+                         dim3(32 * warps), args, 0, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
   return ASYMSPEC_OK;
 }
 

@@ -394,6 +394,21 @@ struct KParams {
   uint32_t* err_word;
   int4* recs;
   unsigned int* tickets;
+  // cluster TMA kernel: what its rows leave for the decision kernel
+  void* row_stat;       // [B(K+1)] RowStat (rank 0 of the row's cluster)
+  float* pass2_rec;     // [B(K+1)][C] X2 records (8 floats), one per CTA
+  float* group_mass;    // [B(K+1)][C][kGroupsMax] inverse-CDF group masses (stochastic)
+};
+
+// What pass 1 leaves for the decision of a row: the normalisers, the
+// argmaxes, the data-error bits and the draft token's three logits.
+struct __align__(16) RowStat {
+  float lse[4];
+  int is, it;
+  unsigned bad;
+  int dtok;
+  float da, db, dt;
+  float pad;
 };
 
 

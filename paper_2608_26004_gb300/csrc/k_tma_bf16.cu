@@ -1,4 +1,4 @@
-// Instantiations of the cluster TMA kernel for __nv_bfloat16 logits (see kernel_tma.cuh).
+// Instantiations of the cluster TMA kernel and its decision kernel for __nv_bfloat16 logits (see kernel_tma.cuh).
 #include "kernel_tma.cuh"
 #include "kernels.h"
 
@@ -7,6 +7,11 @@ namespace asymspec_impl {
 const void* tma_kernel_bf16(bool stoch) {
   return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, true>)
                : reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, false>);
+}
+
+const void* decide_kernel_bf16(bool stoch) {
+  return stoch ? reinterpret_cast<const void*>(&decide_rows<__nv_bfloat16, true>)
+               : reinterpret_cast<const void*>(&decide_rows<__nv_bfloat16, false>);
 }
 
 }  // namespace asymspec_impl

@@ -1,4 +1,4 @@
-// Instantiations of the cluster TMA kernel for float logits (see kernel_tma.cuh).
+// Instantiations of the cluster TMA kernel and its decision kernel for float logits (see kernel_tma.cuh).
 #include "kernel_tma.cuh"
 #include "kernels.h"
 
@@ -7,6 +7,11 @@ namespace asymspec_impl {
 const void* tma_kernel_f32(bool stoch) {
   return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<float, true>)
                : reinterpret_cast<const void*>(&fuse_verify_tma<float, false>);
+}
+
+const void* decide_kernel_f32(bool stoch) {
+  return stoch ? reinterpret_cast<const void*>(&decide_rows<float, true>)
+               : reinterpret_cast<const void*>(&decide_rows<float, false>);
 }
 
 }  // namespace asymspec_impl

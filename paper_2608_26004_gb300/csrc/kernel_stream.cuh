@@ -46,16 +46,6 @@ enum : int {
   PG_FULL_JSD, PG_FULL_KL, PG_FULL_NONE, PG_FULL_JSD_LP, PG_FULL_KL_LP, PG_FULL_NONE_LP
 };
 
-// What pass 1 publishes for pass 2 (tagged words) and for the row decision.
-struct __align__(16) RowStat {
-  float lse[4];
-  int is, it;
-  unsigned bad;
-  int dtok;
-  float da, db, dt;
-  float pad;
-};
-
 // Workspace of the streaming kernel (device pointers into one allocation).
 struct StreamWs {
   int4* recs;                   // [B(K+1)] row records (Algorithm 1's scan)

@@ -75,23 +75,17 @@ struct __align__(16) X2 {  // pass-2 sums
 };
 
 // Fixed part of the shared state; the C pass-1 records pushed by the
-// cluster and the C pass-2 records sent to rank 0 follow it (recv1(),
-// recv2()), then, in stochastic mode, the inverse-CDF group masses.
+// cluster follow it (recv1()).
 struct __align__(16) SharedTma {
   unsigned long long bar[kChunks];  // one mbarrier per chunk
-  unsigned long long b2_bar;        // rank 0: every CTA's pass-2 record has arrived
   union {                           // per-warp records, one pass at a time
     X1 w1[kTWarps];
     X2 w2[kTWarps];
   };
-  float lse[4];
-  int is, it;
-  unsigned bad;
-  float da, db, dt;
-  unsigned broken;
-  unsigned pad;
+  float lse[4];       // the row's normalisers (pass 2 reads them)
+  unsigned broken;    // a chunk copy timed out
+  unsigned pad[3];
   __device__ X1* recv1() { return reinterpret_cast<X1*>(this + 1); }
-  __device__ X2* recv2(int C) { return reinterpret_cast<X2*>(recv1() + C); }
 };
 
 // The pushed records are copied with 16-byte stores.
@@ -103,13 +97,9 @@ static_assert(sizeof(SharedTma) % 16 == 0, "records after SharedTma must stay 16
 // in round g / 8, i.e. vectors [32 g, 32 g + 32) in index order.
 constexpr int kGroupsMax = kMaxRounds * kTWarps;
 
-// Shared bytes after the slices for a cluster of C CTAs.  The stochastic
-// kernel adds this CTA's group masses and, in rank 0, every rank's.
+// Shared bytes after the slices for a cluster of C CTAs.
 __host__ __device__ constexpr int shared_tma_bytes(int C) {
-  return static_cast<int>(sizeof(SharedTma) + C * (sizeof(X1) + sizeof(X2)));
-}
-__host__ __device__ constexpr int group_bytes(int C) {
-  return (C + 1) * kGroupsMax * static_cast<int>(sizeof(float));
+  return static_cast<int>(sizeof(SharedTma) + C * sizeof(X1));
 }
 
 __device__ __forceinline__ X1 x1_neutral() {
@@ -765,15 +755,12 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
   x.Q = hsum2(Q2);
 }
 
-// Pass 2, the CTA combine, and a one-way send to rank 0: every CTA's pass-2
-// record and group masses go into rank 0's shared memory, then each lane of
-// warp 0 arrives (release, cluster scope) on rank 0's b2_bar, whose count is
-// 32 C.  Only rank 0 waits for it; the other CTAs are done.
+// Pass 2 and the CTA combine; warp 0 stores the CTA's pass-2 record in the
+// workspace (groups: this CTA's group masses there, stored by pass 2).
 template <typename T, unsigned G, bool LP>
-__device__ __forceinline__ void pass2_and_send(const T* ra, const T* rb, const T* rt, int nv,
-                                               int rounds, float beta, float* lp, SharedTma* sh,
-                                               int rank, int C, float* groups,
-                                               cg::cluster_group& cluster) {
+__device__ __forceinline__ void pass2_and_store(const T* ra, const T* rb, const T* rt, int nv,
+                                                int rounds, float beta, float* lp, SharedTma* sh,
+                                                float* rec, float* groups) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
   X2 x = x2_zero();
@@ -785,15 +772,9 @@ __device__ __forceinline__ void pass2_and_send(const T* ra, const T* rb, const T
   if (warp == 0) {
     X2 w = (lane < kTWarps) ? sh->w2[lane] : x2_zero();
     warp_reduce_x2<G>(w);
-    X2* rec = cluster.map_shared_rank(sh->recv2(C), 0) + rank;
+    if (sh->broken) w.pad[0] = __uint_as_float(kBadTimeout);
     if (lane < static_cast<int>(sizeof(X2) / 16))
       reinterpret_cast<float4*>(rec)[lane] = reinterpret_cast<const float4*>(&w)[lane];
-    if (G & (G_RES | G_QF)) {
-      float* dst = cluster.map_shared_rank(groups, 0) + kGroupsMax * (1 + rank);
-      if (lane < kGroupsMax / 4)
-        reinterpret_cast<float4*>(dst)[lane] = reinterpret_cast<const float4*>(groups)[lane];
-    }
-    mbar_arrive_remote(&sh->b2_bar, 0);
   }
 }
 
@@ -968,31 +949,26 @@ struct RowCtx {
   bool bonus;
   int dtok;           // warp 0 only
   RowScalars sc;      // warp 0 only (stochastic)
-  float* groups;      // stochastic: this CTA's group masses, then (rank 0) every rank's
   SharedTma* sh;
 };
 
-// The decision of a complete row (one warp; lane 0 writes).
-template <bool STOCH>
-__device__ __forceinline__ void finish(const KParams& P, const RowCtx& c, const float (&lse)[4],
-                                       int is, int it, unsigned bad, float D, int sample,
-                                       float mass, float ad, float bd, float td) {
-  const bool has_ab = P.full || !c.bonus;
-  const bool has_t = P.full || (!STOCH && !c.bonus);
-  const bool has_s = P.full || STOCH;
-  RowResult r;
-  r.lse_a = has_ab ? lse[0] : NAN;
-  r.lse_b = has_ab ? lse[1] : NAN;
-  r.lse_t = has_t ? lse[2] : NAN;
-  r.lse_s = has_s ? lse[3] : NAN;
-  r.D = D;
-  r.is = is;
-  r.it = it;
-  r.sample = sample;
-  r.mass = mass;
-  r.bad = bad;
-  r.have_lse_t = has_t;
-  finish_row_warp<STOCH>(P, c.row, c.bi, c.k, r, c.dtok, ad, bd, td, c.sc);
+// Rank 0: what pass 1 leaves for the row's decision.
+__device__ __forceinline__ void store_row_stat(const KParams& P, long long row,
+                                               const float (&lse)[4], int is, int it,
+                                               unsigned bad, int dtok, float ad, float bd,
+                                               float td) {
+  RowStat st;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) st.lse[q] = lse[q];
+  st.is = is;
+  st.it = it;
+  st.bad = bad;
+  st.dtok = dtok;
+  st.da = ad;
+  st.db = bd;
+  st.dt = td;
+  st.pad = 0.f;
+  static_cast<RowStat*>(P.row_stat)[row] = st;
 }
 
 // One row with pass-1 program F and pass-2 program G (R2: pass 2 runs; LP:
@@ -1009,13 +985,13 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
   pass1_and_push<T, F>(ra, rb, rt, c.nv, c.rounds, c.rc, c.lo, c.n, beta, c.dtok, sh, c.rank, c.C,
                        cluster);
   if constexpr (!R2) {
-    // no pass 2: the row is decided by warp 0 of rank 0; every other warp leaves
+    // no pass 2: rank 0 leaves the row's pass-1 results for the decision kernel
     if (c.rank == 0 && warp == 0) {
       float lse[4];
       const X1 w = combine_pass1<F>(sh, c.C, lse);
       float ad, bd, td;
       draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td);
-      finish<STOCH>(P, c, lse, w.is, w.it, w.bad, 0.f, -1, NAN, ad, bd, td);
+      if (lane == 0) store_row_stat(P, c.row, lse, w.is, w.it, w.bad, c.dtok, ad, bd, td);
     }
     return;
   } else {
@@ -1025,73 +1001,18 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
       if (lane == 0) {
 #pragma unroll
         for (int q = 0; q < 4; ++q) sh->lse[q] = lse[q];
-        sh->is = w.is;
-        sh->it = w.it;
-        sh->bad = w.bad;
-        draft_logits(sh, c.dtok, c.W, c.C, sh->da, sh->db, sh->dt);
+        if (c.rank == 0) {
+          float ad, bd, td;
+          draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td);
+          store_row_stat(P, c.row, lse, w.is, w.it, w.bad, c.dtok, ad, bd, td);
+        }
       }
     }
     __syncthreads();
     float* lp = LP ? P.logprobs + static_cast<size_t>(c.row) * P.V + c.lo : nullptr;
-    pass2_and_send<T, G, LP>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh, c.rank, c.C, c.groups,
-                             cluster);
-    if (c.rank != 0 || warp != 0) return;  // the rest is rank 0's warp 0
-    unsigned bad = sh->bad;
-    if (!mbar_wait_cluster_bounded(&sh->b2_bar, 0, kCopyTimeoutNs)) bad |= kBadTimeout;
-    const X2 w = (lane < c.C) ? sh->recv2(c.C)[lane] : x2_zero();
-    const float lse[4] = {sh->lse[0], sh->lse[1], sh->lse[2], sh->lse[3]};
-    X2 tot = w;
-    warp_reduce_x2<G>(tot);
-    const float D = divergence_of<G>(tot);
-    if constexpr (STOCH) {
-      // inclusive prefix of the inverse-CDF mass over ranks, in rank order
-      float incl_R = w.R, incl_Q = w.Q;
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const float vr = __shfl_up_sync(0xffffffffu, incl_R, off);
-        const float vq = __shfl_up_sync(0xffffffffu, incl_Q, off);
-        if (lane >= off) {
-          incl_R += vr;
-          incl_Q += vq;
-        }
-      }
-      const float R_all = __shfl_sync(0xffffffffu, incl_R, 31);
-      const float Q_all = __shfl_sync(0xffffffffu, incl_Q, 31);
-      const bool r_ok = !c.bonus && (R_all > 0.f);
-      const float incl = r_ok ? incl_R : incl_Q;
-      const float mass = r_ok ? w.R : w.Q;
-      const float total = r_ok ? R_all : Q_all;
-      const float tau = c.sc.u_last * total;
-      const unsigned over = __ballot_sync(0xffffffffu, lane < c.C && incl > tau);
-      const unsigned pos = __ballot_sync(0xffffffffu, lane < c.C && mass > 0.f);
-      int owner = -1;
-      if (over) owner = __ffs(over) - 1;
-      else if (pos) owner = 31 - __clz(pos);
-      int sample = -1;
-      if (owner >= 0) {
-        const float incl_o = __shfl_sync(0xffffffffu, incl, owner);
-        const float mass_o = __shfl_sync(0xffffffffu, mass, owner);
-        const float tau_local = fmaxf(tau - (incl_o - mass_o), 0.f);
-        // the owner's slice, read back from global memory (L2)
-        constexpr int VE = 16 / static_cast<int>(sizeof(T));
-        const int lo_o = owner * c.W;
-        const int nv_o = max(0, min(c.W, P.V - lo_o)) / VE;
-        const int ng_o = ((nv_o + kTThreads - 1) / kTThreads) * kTWarps;
-        const size_t off = static_cast<size_t>(c.row) * P.V + lo_o;
-        // pass 2 kept the residual group masses of draft rows and the fused
-        // ones of the bonus row; the other kind (a draft row whose residual is
-        // zero) is recomputed exactly as pass 2 computes it
-        const bool stored_r = !c.bonus || P.full;
-        sample = group_walk<T, false>(static_cast<const T*>(P.a) + off,
-                                      static_cast<const T*>(P.b) + off,
-                                      static_cast<const T*>(P.t) + off, nv_o, lo_o, ng_o, beta,
-                                      c.groups + kGroupsMax * (1 + owner), r_ok == stored_r, r_ok,
-                                      lse[0] * kLog2e, lse[3] * kLog2e, tau_local);
-      }
-      finish<STOCH>(P, c, lse, sh->is, sh->it, bad, D, sample, total, sh->da, sh->db, sh->dt);
-    } else {
-      finish<STOCH>(P, c, lse, sh->is, sh->it, bad, D, -1, NAN, sh->da, sh->db, sh->dt);
-    }
+    const size_t slot = static_cast<size_t>(c.row) * c.C + c.rank;
+    pass2_and_store<T, G, LP>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh, P.pass2_rec + slot * 8,
+                              P.group_mass + slot * kGroupsMax);
   }
 }
 
@@ -1135,16 +1056,11 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   T* sb = sa + W;
   T* st = sb + W;
   SharedTma* sh = reinterpret_cast<SharedTma*>(smem_tma + P.sh_off);
-  // stochastic: inverse-CDF group masses after the records
-  float* groups = reinterpret_cast<float*>(reinterpret_cast<unsigned char*>(sh) +
-                                           shared_tma_bytes(C));
   const bool only_t = !STOCH && !P.full && bonus && !P.fuse_bonus;
 
   if (tid == 0) {
 #pragma unroll
     for (int c = 0; c < kChunks; ++c) mbar_init(&sh->bar[c], 1);
-    // one arrive per lane of warp 0 of every CTA; B1 orders this before any
-    mbar_init(&sh->b2_bar, 32u * static_cast<unsigned>(C));
     sh->broken = 0;
     fence_mbar_init();
     issue_slice<T>(P, sh, row, lo, nv, rc, sa, sb, st, only_t);
@@ -1165,7 +1081,6 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   c.bi = bi;
   c.row = row;
   c.bonus = bonus;
-  c.groups = groups;
   c.sh = sh;
   c.dtok = -1;
   c.sc = RowScalars{0.f, 0.f, 0.f};
@@ -1215,6 +1130,127 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   if (tid == 0 && sh->broken) {
 #pragma unroll
     for (int q = 0; q < kChunks; ++q) mbar_wait_bounded(&sh->bar[q], 0, kCopyTimeoutNs);
+  }
+}
+
+// ---------------------------------------------------------------- row decisions
+
+constexpr int kDecideThreads = 256;  // at most 8 warps; each takes rows k, k + 8, ...
+
+// The decisions of one batch element's K+1 rows (one CTA per element, one
+// warp per row) from what fuse_verify_tma left in the workspace, then
+// Algorithm 1's scan over them in shared memory.  Per row: the divergence
+// (Eq. 3) from the C pass-2 records; in stochastic mode the CTA whose slice
+// holds the inverse-CDF target (prefix over ranks) and the draw inside it
+// (group_walk, reading that slice back from L2); the acceptance test and
+// the emitted candidate (row_record, kept in the workspace's records).
+template <typename T, bool STOCH>
+__global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  const int bi = blockIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const int K = P.K, K1 = K + 1, C = P.C;
+  const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
+  const bool klg = P.divergence == ASYMSPEC_DIV_KL;
+  for (int k = warp; k < K1; k += nw) {
+    const long long row = static_cast<long long>(bi) * K1 + k;
+    const bool bonus = (k == K);
+    const bool pass2 = STOCH || P.full || (!bonus && (jsd || klg));
+    RowStat st = static_cast<const RowStat*>(P.row_stat)[row];
+    X2 w = x2_zero();
+    if (pass2 && lane < C) w = reinterpret_cast<const X2*>(P.pass2_rec)[row * C + lane];
+    const unsigned late = __ballot_sync(0xffffffffu, pass2 && lane < C &&
+                                                         __float_as_uint(w.pad[0]) != 0u);
+    if (late) st.bad |= kBadTimeout;
+    const float j = warp_sum(w.j), msum = warp_sum(w.msum), kl = warp_sum(w.kl);
+    float D = 0.f;
+    if (pass2 && jsd) D = 0.5f * kLn2 * (j + msum);
+    else if (pass2 && klg) D = kLn2 * kl;
+    int sample = -1;
+    float mass_total = NAN;
+    const RowScalars sc = STOCH ? load_row_scalars(P, bi, k) : RowScalars{0.f, 0.f, 0.f};
+    if constexpr (STOCH) {
+      // inclusive prefix of the inverse-CDF mass over ranks, in rank order
+      float incl_R = w.R, incl_Q = w.Q;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const float vr = __shfl_up_sync(0xffffffffu, incl_R, off);
+        const float vq = __shfl_up_sync(0xffffffffu, incl_Q, off);
+        if (lane >= off) {
+          incl_R += vr;
+          incl_Q += vq;
+        }
+      }
+      const float R_all = __shfl_sync(0xffffffffu, incl_R, 31);
+      const float Q_all = __shfl_sync(0xffffffffu, incl_Q, 31);
+      const bool r_ok = !bonus && (R_all > 0.f);
+      const float incl = r_ok ? incl_R : incl_Q;
+      const float mass = r_ok ? w.R : w.Q;
+      const float total = r_ok ? R_all : Q_all;
+      mass_total = total;
+      const float tau = sc.u_last * total;
+      const unsigned over = __ballot_sync(0xffffffffu, lane < C && incl > tau);
+      const unsigned pos = __ballot_sync(0xffffffffu, lane < C && mass > 0.f);
+      int owner = -1;
+      if (over) owner = __ffs(over) - 1;
+      else if (pos) owner = 31 - __clz(pos);
+      if (owner >= 0) {
+        const float incl_o = __shfl_sync(0xffffffffu, incl, owner);
+        const float mass_o = __shfl_sync(0xffffffffu, mass, owner);
+        const float tau_local = fmaxf(tau - (incl_o - mass_o), 0.f);
+        const int lo_o = owner * P.W;
+        const int nv_o = max(0, min(P.W, P.V - lo_o)) / VE;
+        const int ng_o = ((nv_o + kTThreads - 1) / kTThreads) * kTWarps;
+        const size_t off = static_cast<size_t>(row) * P.V + lo_o;
+        // the group masses are residual ones for draft rows and fused ones for
+        // the bonus row; the other kind (a draft row whose residual is zero)
+        // is recomputed exactly as pass 2 computes it
+        const bool stored_r = !bonus || P.full;
+        sample = group_walk<T, true>(static_cast<const T*>(P.a) + off,
+                                     static_cast<const T*>(P.b) + off,
+                                     static_cast<const T*>(P.t) + off, nv_o, lo_o, ng_o, P.beta,
+                                     P.group_mass + (row * C + owner) * kGroupsMax,
+                                     r_ok == stored_r, r_ok, st.lse[0] * kLog2e,
+                                     st.lse[3] * kLog2e, tau_local);
+      }
+    }
+    const bool has_ab = P.full || !bonus;
+    const bool has_t = P.full || (!STOCH && !bonus);
+    RowResult r;
+    r.lse_a = has_ab ? st.lse[0] : NAN;
+    r.lse_b = has_ab ? st.lse[1] : NAN;
+    r.lse_t = has_t ? st.lse[2] : NAN;
+    r.lse_s = (P.full || STOCH) ? st.lse[3] : NAN;
+    r.D = D;
+    r.is = st.is;
+    r.it = st.it;
+    r.sample = sample;
+    r.mass = mass_total;
+    r.bad = st.bad;
+    r.have_lse_t = has_t;
+    if (lane == 0) P.recs[row] = row_record<STOCH>(P, row, k, r, st.dtok, st.da, st.db, st.dt, sc);
+  }
+  __syncthreads();  // the element's records are visible to the block
+  const int4* recs = P.recs + static_cast<size_t>(bi) * K1;
+  if (warp != 0) return;
+  // Algorithm 1: the first rejected draft, or K if none; any data error voids the element
+  bool any_err = false;
+  int len = -1, next = -1;
+  for (int base = 0; base < K1; base += 32) {
+    const int j = base + lane;
+    int4 v = make_int4(1, -1, 0, 0);
+    if (j < K1) v = __ldcg(&recs[j]);
+    any_err |= __any_sync(0xffffffffu, v.z != 0);
+    if (len < 0) {
+      const unsigned rej = __ballot_sync(0xffffffffu, j < K && v.x == 0);
+      if (rej) len = base + __ffs(rej) - 1;
+      else if (K < base + 32) len = K;
+      if (len >= 0) next = __shfl_sync(0xffffffffu, v.y, len - base);
+    }
+  }
+  if (lane == 0) {
+    P.out_len[bi] = any_err ? -1 : len;
+    P.out_next[bi] = any_err ? -1 : next;
   }
 }
 

@@ -10,6 +10,9 @@ const void* generic_kernel(int dtype, bool vector_path, bool stoch);
 // fuse_verify_tma<T, STOCH> (k_tma_bf16.cu, k_tma_f32.cu)
 const void* tma_kernel_bf16(bool stoch);
 const void* tma_kernel_f32(bool stoch);
+// decide_rows<T, STOCH>, launched after fuse_verify_tma (same files)
+const void* decide_kernel_bf16(bool stoch);
+const void* decide_kernel_f32(bool stoch);
 // fuse_verify_stream<T, STOCH> (k_stream_*.cu)
 const void* stream_kernel_bf16_greedy();
 const void* stream_kernel_bf16_stoch();

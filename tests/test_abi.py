@@ -52,12 +52,27 @@ def test_defaults_and_strings(lib):
     assert A.version() == 200
 
 
+def _up(n):
+    return (n + 255) // 256 * 256
+
+
+def tma_bytes(B, K, C):
+    """Records and tickets, then the TMA kernel's per-row results: a 48-byte
+    row record of pass 1, and per CTA a 32-byte pass-2 record and 80 group
+    masses."""
+    R = B * (K + 1)
+    return _up(R * 16) + _up(B * 4) + _up(R * 48) + _up(R * C * 32) + _up(R * C * 80 * 4)
+
+
 def test_workspace_size():
-    # records and tickets of the cluster kernels, then the streaming kernel's state
-    assert A.workspace_bytes(64, 7, 128256) >= 64 * 8 * 16 + 64 * 4
+    # the TMA kernel's layout for clusters of up to 16 CTAs, independent of V,
+    # unless the streaming kernel's is larger (fp32 rows of 16 or more tiles)
+    assert A.workspace_bytes(64, 7, 128256) >= tma_bytes(64, 7, 16)
+    assert A.workspace_bytes(3, 2, 10) == A.workspace_bytes(3, 2, 10**5) == tma_bytes(3, 2, 16)
     assert A.workspace_bytes(0, 7, 10) == 0
-    # the streaming state grows with the tiles per row (fp32 rows have the most)
-    assert A.workspace_bytes(3, 2, 10) < A.workspace_bytes(3, 2, 10**5)
+    # the streaming state grows with the tiles per row and passes it for fp32
+    # rows of 31 tiles of 8192 entries
+    assert A.workspace_bytes(3, 2, 250000) > tma_bytes(3, 2, 16)
     assert A.workspace_bytes(64, 7, 128256) < 8 << 20
 
 
@@ -100,9 +115,13 @@ def test_host_validation_codes(lib):
     st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
                           FAKE, FAKE, 1 << 20, opts=A.LaunchOpts(0, 0, 7))
     assert st == A.ERR_INVALID_ARG                       # unknown kernel
-    small = A.workspace_bytes(2, 2, 64) - 1              # streaming kernel forced, workspace short
-    st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
+    small = A.workspace_bytes(2, 2, 250000) - 1          # streaming kernel forced, workspace short
+    st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 250000, A.FP32, None, FAKE,
                           FAKE, FAKE, small, opts=A.LaunchOpts(0, 0, A.KERNEL_STREAM))
+    assert st == A.ERR_WORKSPACE
+    small = tma_bytes(2, 2, 4) - 1                       # TMA kernel forced (clusters of 4), short
+    st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
+                          FAKE, FAKE, small, opts=A.LaunchOpts(4, 0, A.KERNEL_TMA))
     assert st == A.ERR_WORKSPACE
 
 

@@ -3,9 +3,8 @@
 The file name sorts last so that these calls also run after every other GPU
 test has used the library in the same process; the tests must pass both
 alone and then.  Every result is compared bit for bit with
-asymspec_fuse_verify_ex on the same kernel (the scratch holds the cluster
-kernels' records and tickets) with a caller-owned zeroed workspace, on the
-same inputs, over two consecutive calls, so that the second call sees the
+asymspec_fuse_verify_ex given a caller-owned zeroed workspace of the static
+scratch's size, which selects the same kernel, on the same inputs, over two consecutive calls, so that the second call sees the
 scratch the first one left.
 """
 import numpy as np
@@ -45,18 +44,16 @@ def run_static(torch, x, B, K, V, dtype, gate):
 
 
 def run_ex(torch, x, B, K, V, dtype, gate):
-    """The workspace entry point on the kernel the static scratch selects: the
-    cluster kernels (TMA for aligned rows, generic otherwise)."""
+    """The workspace entry point with a workspace of the static scratch's size:
+    the automatic choice then takes the kernel the static entry takes."""
     L = torch.full((B,), -7, dtype=torch.int32, device="cuda")
     N = torch.full((B,), -7, dtype=torch.int32, device="cuda")
-    nbytes = A.workspace_bytes(B, K, V)
+    nbytes = A.STATIC_SCRATCH_BYTES
     ws = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
     stream = torch.cuda.current_stream().cuda_stream
     st = A.fuse_verify_ex(_ptr(x["a"]), _ptr(x["b"]), _ptr(x["t"]), _ptr(x["tokens"]),
                           _ptr(x["probs"]), _ptr(x["unif"]), B, K, V, dtype, gate, _ptr(L),
-                          _ptr(N), _ptr(ws), nbytes,
-                          opts=A.LaunchOpts(0, 0, A.KERNEL_AUTO if V % 8 else A.KERNEL_TMA),
-                          stream=stream)
+                          _ptr(N), _ptr(ws), nbytes, stream=stream)
     assert st == A.OK, A.status_string(st)
     torch.cuda.synchronize()
     return L.cpu().numpy(), N.cpu().numpy()
@@ -68,10 +65,12 @@ CASES = [
     (3, 2, 4099, synth.BF16, A.MODE_GREEDY, 12),          # unaligned rows: generic kernel
     (1024, 7, 64, synth.FP32, A.MODE_STOCHASTIC, 13),     # B*(K+1) = the 8192-row limit
     (1024, 7, 64, synth.FP32, A.MODE_GREEDY, 14),
+    (64, 7, 128256, synth.BF16, A.MODE_STOCHASTIC, 15),   # 512 rows: the TMA kernel
+    (700, 7, 12288, synth.FP32, A.MODE_GREEDY, 16),       # TMA part too large: generic
 ]
 
 
-@pytest.mark.parametrize("first,second", [(0, 1), (2, 3), (3, 0)])
+@pytest.mark.parametrize("first,second", [(0, 1), (2, 3), (3, 0), (4, 5), (5, 4)])
 def test_two_consecutive_calls_match_the_workspace_entry_point(torch, first, second):
     for idx in (first, second):
         B, K, V, dtype, mode, seed = CASES[idx]
@@ -94,3 +93,21 @@ def test_rows_above_the_limit_are_rejected_before_any_launch(torch):
     assert "8192" in A.status_string(st)
     torch.cuda.synchronize()
     assert np.all(L.cpu().numpy() == -7)                  # nothing ran
+
+
+def _up(n):
+    return (n + 255) // 256 * 256
+
+
+def test_the_cases_cover_both_kernels_the_scratch_selects(torch):
+    # the TMA kernel needs, beyond records and tickets, 48 bytes per row and
+    # 352 per row and CTA; the static scratch takes it when they fit
+    fits = []
+    for B, K, V, dtype, mode, seed in CASES:
+        info = A.plan(B, K, V, dtype, A.gate_params(mode=mode))
+        R = B * (K + 1)
+        need = (_up(R * 16) + _up(B * 4) + _up(R * 48) + _up(R * info.cluster_size * 32)
+                + _up(R * info.cluster_size * 320))
+        if info.kernel == A.KERNEL_TMA:
+            fits.append(need <= A.STATIC_SCRATCH_BYTES)
+    assert True in fits and False in fits
