@@ -318,7 +318,7 @@ def main():
     value = world * rows / (ms_step * 1e-3)
     # the cluster kernel and its decision kernel: the whole step is charged to
     # the cluster kernel (its share of the step is in the ncu launch list)
-    launches_per_step = 2 if info.kernel == A.KERNEL_TMA else 1
+    launches_per_step = 2 if info.kernel in (A.KERNEL_TMA, A.KERNEL_RING) else 1
     launch_s = ms_step * 1e-3
     hbm_peak, peak_kind = peaks()
     achieved = alg_bytes / launch_s / 1e9

@@ -100,16 +100,19 @@ typedef struct {
 typedef struct {
   int32_t cluster_size;   /* CTAs per row triple: 1 to 16 */
   int32_t block_threads;  /* reserved, must be 0 (256 threads per CTA) */
-  int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC, _TMA or _STREAM */
+  int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC, _TMA, _STREAM or _RING */
 } asymspec_launch_opts;
 
 /* Kernels (asymspec_launch_opts.kernel, asymspec_launch_info.kernel). */
 #define ASYMSPEC_KERNEL_GENERIC 1  /* one cluster per row; any element-aligned input */
 #define ASYMSPEC_KERNEL_TMA 2      /* one cluster per row, chunked 1-D bulk copies, per-row
-                                      programs; rows 16-byte aligned */
+                                      programs; rows 16-byte aligned; debug outputs */
 #define ASYMSPEC_KERNEL_STREAM 3   /* persistent grid over row tiles: pass 1 reads each tile from
                                       HBM, pass 2 re-reads it from L2; rows 16-byte aligned and a
                                       workspace of asymspec_workspace_bytes(); on request only */
+#define ASYMSPEC_KERNEL_RING 4     /* persistent clusters: pass 1 through a ring of bulk copies,
+                                      pass 2 from L2; rows 16-byte aligned; no debug outputs;
+                                      on request only */
 
 /* What a launch would use (filled by asymspec_plan). */
 typedef struct {
@@ -120,7 +123,7 @@ typedef struct {
   int64_t ctas;            /* CTAs in the grid */
   int32_t vector_path;     /* 1 if rows qualify for 16-byte copies (V * element size % 16 == 0) */
   int32_t max_active_clusters; /* clusters the device can hold at once (0 if unknown) */
-  int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC, _TMA or _STREAM */
+  int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC, _TMA, _STREAM or _RING */
 } asymspec_launch_info;
 
 /* Fills *p with the paper's defaults: gamma 0.5, beta 1.0, lambda 0.1,

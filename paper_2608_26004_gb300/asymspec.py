@@ -69,6 +69,7 @@ KERNEL_AUTO = 0
 KERNEL_GENERIC = 1
 KERNEL_TMA = 2
 KERNEL_STREAM = 3
+KERNEL_RING = 4
 
 
 class LaunchOpts(ctypes.Structure):

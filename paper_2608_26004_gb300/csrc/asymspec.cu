@@ -18,6 +18,7 @@
 
 #include "device_common.cuh"
 #include "kernel_generic.cuh"
+#include "kernel_ring.cuh"
 #include "kernel_stream.cuh"
 #include "kernels.h"
 
@@ -94,6 +95,23 @@ bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
   return false;
 }
 
+// Persistent ring kernel: clusters of 8 (16 when a slice of 8 would take
+// more than kMaxRounds rounds); the slice is not held in shared memory.
+bool plan_ring(int V, int elt, int forced_C, Plan* pl) {
+  const int VE = 16 / elt;
+  auto fill = [&](int C) {
+    const long long per = (static_cast<long long>(V) + C - 1) / C;
+    const long long W = round_up_ll(per, VE);
+    pl->C = C;
+    pl->W = static_cast<int>(W);
+    pl->sh_off = 0;
+    pl->smem = ring_smem_bytes(C);
+    return pl->smem <= kMaxSmem && W / VE <= static_cast<long long>(kMaxRounds) * kTThreads;
+  };
+  if (forced_C > 0) return fill(forced_C);
+  return fill(8) || fill(16);
+}
+
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 size_t ws_records_bytes(int B, int K) {
@@ -166,14 +184,17 @@ StreamLayout stream_layout(int B, int K, int V, int elt) {
 // items; rows longer than this many tiles use the cluster kernels.
 constexpr int kMaxStreamTiles = 31;
 
+// debug_out: the call asks for row statistics or fused log-probs, which only
+// the one-shot kernels produce.
 int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_opts* opts,
-              bool vec_ok, size_t ws_bytes, Plan* pl) {
+              bool vec_ok, size_t ws_bytes, bool debug_out, Plan* pl) {
   const int elt = elt_size(dtype);
   const int forced_C = (opts && opts->cluster_size > 0) ? opts->cluster_size : 0;
   const int forced_kernel = opts ? opts->kernel : 0;
   if (forced_C < 0 || forced_C > 16) return ASYMSPEC_ERR_INVALID_ARG;
   if (forced_kernel != 0 && forced_kernel != ASYMSPEC_KERNEL_GENERIC &&
-      forced_kernel != ASYMSPEC_KERNEL_TMA && forced_kernel != ASYMSPEC_KERNEL_STREAM)
+      forced_kernel != ASYMSPEC_KERNEL_TMA && forced_kernel != ASYMSPEC_KERNEL_STREAM &&
+      forced_kernel != ASYMSPEC_KERNEL_RING)
     return ASYMSPEC_ERR_INVALID_ARG;
   pl->rows = static_cast<long long>(B) * (K + 1);
   pl->vector_path = vec_ok;
@@ -194,6 +215,25 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
     return ASYMSPEC_OK;
   }
   if (ws_bytes < cluster_ws_bytes(B, K)) return ASYMSPEC_ERR_WORKSPACE;
+  // the persistent ring kernel on request only: measured slower than the
+  // one-shot kernel on the headline workload (pass 2 misses L2 at this reuse
+  // distance, and warps wait on warp 0's producer and combine work)
+  if (forced_kernel == ASYMSPEC_KERNEL_RING) {
+    Plan r = *pl;
+    if (vec_ok && !debug_out && plan_ring(V, elt, forced_C, &r) &&
+        ws_bytes >= tma_layout(B, K, r.C).total) {
+      *pl = r;
+      pl->kernel = ASYMSPEC_KERNEL_RING;
+      pl->VE = 16 / elt;
+      pl->ctas = 0;  // set at launch from the device's cluster occupancy
+      return ASYMSPEC_OK;
+    }
+    if (forced_kernel == ASYMSPEC_KERNEL_RING) {
+      if (!vec_ok || debug_out) return ASYMSPEC_ERR_UNSUPPORTED;
+      return (r.C > 0 && ws_bytes < tma_layout(B, K, r.C).total) ? ASYMSPEC_ERR_WORKSPACE
+                                                                : ASYMSPEC_ERR_TOO_LARGE;
+    }
+  }
   bool ok = false;
   if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, pl)) {
     // the TMA kernel leaves each row's results in the workspace; the generic
@@ -220,10 +260,17 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
 
 using KernelFn = const void*;  // a __global__ function taking KParams (or SParams)
 
+KernelFn pick_ring(int dtype, bool stoch);
+
 KernelFn pick_kernel(const Plan& pl, int dtype, bool stoch) {
+  if (pl.kernel == ASYMSPEC_KERNEL_RING) return pick_ring(dtype, stoch);
   if (pl.kernel == ASYMSPEC_KERNEL_TMA)
     return dtype == ASYMSPEC_FP32 ? tma_kernel_f32(stoch) : tma_kernel_bf16(stoch);
   return generic_kernel(dtype, pl.vector_path, stoch);
+}
+
+KernelFn pick_ring(int dtype, bool stoch) {
+  return dtype == ASYMSPEC_FP32 ? ring_kernel_f32(stoch) : ring_kernel_bf16(stoch);
 }
 
 KernelFn pick_decide(int dtype, bool stoch) {
@@ -267,7 +314,7 @@ cudaLaunchConfig_t launch_config(const Plan& pl, long long ctas, cudaStream_t st
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.gridDim = dim3(static_cast<unsigned>(ctas));
-  cfg.blockDim = dim3(pl.kernel == ASYMSPEC_KERNEL_TMA ? kTThreads : kThreads);
+  cfg.blockDim = dim3(pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : kTThreads);
   cfg.dynamicSmemBytes = pl.smem;
   cfg.stream = stream;
   cfg.attrs = attr;
@@ -459,9 +506,9 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
   st = check_params(&gp);
   if (st) return st;
   const bool vec_ok = (static_cast<long long>(V) * elt_size(dtype)) % 16 == 0;
-  Plan pl;
+  Plan pl = {};
   st = make_plan(B, K, V, dtype, gp.mode == ASYMSPEC_MODE_STOCHASTIC, opts, vec_ok,
-                 asymspec_workspace_bytes(B, K, V), &pl);
+                 asymspec_workspace_bytes(B, K, V), false, &pl);
   if (st) return st;
   if (pl.kernel == ASYMSPEC_KERNEL_STREAM) {
     out->cluster_size = 1;
@@ -483,7 +530,7 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
     return ASYMSPEC_OK;
   }
   out->cluster_size = pl.C;
-  out->block_threads = pl.kernel == ASYMSPEC_KERNEL_TMA ? kTThreads : kThreads;
+  out->block_threads = pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : kTThreads;
   out->slice_elems = pl.W;
   out->smem_bytes = pl.smem;
   out->ctas = pl.ctas;
@@ -497,6 +544,9 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
     if (prepare_kernel(fn, device) == cudaSuccess &&
         active_clusters(fn, pl, device, &ncl) == cudaSuccess)
       out->max_active_clusters = ncl;
+    // the persistent kernel launches the clusters the device holds, at most one per row
+    if (pl.kernel == ASYMSPEC_KERNEL_RING)
+      out->ctas = std::min(static_cast<long long>(ncl), pl.rows) * pl.C;
   }
   cudaGetLastError();
   return ASYMSPEC_OK;
@@ -537,8 +587,9 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   if (!workspace || !aligned(workspace, 16)) return ASYMSPEC_ERR_WORKSPACE;
   const bool vec_ok = (static_cast<long long>(V) * elt) % 16 == 0 && aligned(logits_full, 16) &&
                       aligned(logits_comp, 16) && aligned(logits_ver, 16);
-  Plan pl;
-  st = make_plan(B, K, V, dtype, stoch, opts, vec_ok, workspace_bytes, &pl);
+  Plan pl = {};
+  st = make_plan(B, K, V, dtype, stoch, opts, vec_ok, workspace_bytes,
+                 out_row_stats || out_fused_logprobs, &pl);
   if (st) return st;
 
   KParams P;
@@ -635,14 +686,20 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   KernelFn fn = pick_kernel(pl, dtype, stoch);
   e = prepare_kernel(fn, device);
   if (e != cudaSuccess) return cuda_fail(e);
-  // One cluster per row: measured faster than a persistent grid of clusters
-  // looping over rows (the kernel supports both), whose row-finishing work
-  // lands on the cluster's critical path.
-  const long long ctas = pl.ctas;
+  // The one-shot kernels launch one cluster per row; the persistent ring
+  // kernel as many clusters as the device holds at once (at most one per row).
+  long long ctas = pl.ctas;
+  if (pl.kernel == ASYMSPEC_KERNEL_RING) {
+    int ncl = 0;
+    e = active_clusters(fn, pl, device, &ncl);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (ncl < 1) return ASYMSPEC_ERR_UNSUPPORTED;
+    ctas = std::min(static_cast<long long>(ncl), pl.rows) * pl.C;
+  }
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = launch_config(pl, ctas, static_cast<cudaStream_t>(stream), attr);
   void* args[] = {&P};
-  if (pl.kernel == ASYMSPEC_KERNEL_TMA) {
+  if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING) {
     const TmaLayout L = tma_layout(B, K, pl.C);
     char* base = static_cast<char*>(workspace);
     P.row_stat = base + L.stat;
@@ -651,7 +708,7 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   }
   e = cudaLaunchKernelExC(&cfg, fn, args);
   if (e != cudaSuccess) return cuda_fail(e);
-  if (pl.kernel == ASYMSPEC_KERNEL_TMA) {
+  if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING) {
     // the rows' decisions and Algorithm 1's scan: one CTA per batch element
     const int warps = std::min(K + 1, kDecideThreads / 32);
     e = cudaLaunchKernel(pick_decide(dtype, stoch), dim3(static_cast<unsigned>(B)),

@@ -314,7 +314,9 @@ __device__ __forceinline__ void load_or_fill(const T* p, bool ok, f2 (&x)[NP]) {
 // vectors): the fallback for slices where pass1_fast's fixed reference
 // overflows.  Vector i of the slice lives in round i / NT; chunk c holds
 // rounds [c rc, (c+1) rc).  Rounds are taken two at a time.
-template <typename T, unsigned F>
+// WAIT: the slice is in shared memory behind the chunk barriers of sh (false:
+// it is in global memory and sh is not used).
+template <typename T, unsigned F, bool WAIT = true>
 __device__ __noinline__ void pass1_online(const T* ra, const T* rb, const T* rt, int nv, int rounds,
                                       int rc, int lo, float beta, SharedTma* sh, X1& e) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
@@ -330,7 +332,7 @@ __device__ __noinline__ void pass1_online(const T* ra, const T* rb, const T* rt,
   int vec_s = -1, vec_t = -1;  // vectors holding the best s and t so far
   const int tid = static_cast<int>(threadIdx.x);
   for (int c = 0, r0 = 0; c < kChunks && r0 < rounds; ++c, r0 += rc) {
-    if (!sh->broken && !mbar_wait_bounded(&sh->bar[c], 0, kCopyTimeoutNs))
+    if (WAIT && !sh->broken && !mbar_wait_bounded(&sh->bar[c], 0, kCopyTimeoutNs))
       atomicOr(&sh->broken, kBadTimeout);
     const int r1 = min(rounds, r0 + rc);
     int i0 = r0 * kTThreads + tid;          // vector index of this thread's first vector
@@ -741,11 +743,14 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
     }
     }
     if (RES || QF) {  // group masses: every lane takes part, with or without a vector
-      const float s0 = warp_sum(g0), s1 = warp_sum(g1);
-      if ((threadIdx.x & 31) == 0) {
-        grp[kr * kTWarps + warp] = s0;
-        if (kr + 1 < rounds) grp[(kr + 1) * kTWarps + warp] = s1;
-      }
+      // both rounds' sums in one butterfly: lanes 0-15 carry round kr, 16-31 round kr + 1
+      const int lane = static_cast<int>(threadIdx.x & 31);
+      const bool upper = lane >= 16;
+      float g = (upper ? g1 : g0) + __shfl_xor_sync(0xffffffffu, upper ? g0 : g1, 16);
+#pragma unroll
+      for (int off = 8; off > 0; off >>= 1) g += __shfl_xor_sync(0xffffffffu, g, off);
+      if (lane == 0) grp[kr * kTWarps + warp] = g;
+      if (lane == 16 && kr + 1 < rounds) grp[(kr + 1) * kTWarps + warp] = g;
     }
   }
   x.j = hsum2(add2(ja, jb));
@@ -1040,10 +1045,12 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   const int rank = static_cast<int>(cluster.block_rank());
   const int tid = threadIdx.x;
   const int C = P.C;
-  const long long row = blockIdx.x / C;
-  const int K1 = P.K + 1;
-  const int bi = static_cast<int>(row / K1);
-  const int k = static_cast<int>(row % K1);
+  // 32-bit row arithmetic: the host keeps rows x C below 2^31
+  const unsigned row32 = blockIdx.x / static_cast<unsigned>(C);
+  const long long row = row32;
+  const unsigned K1 = static_cast<unsigned>(P.K) + 1u;
+  const int bi = static_cast<int>(row32 / K1);
+  const int k = static_cast<int>(row32 - static_cast<unsigned>(bi) * K1);
   const bool bonus = (k == P.K);
   const int V = P.V, W = P.W;
   const int lo = rank * W;

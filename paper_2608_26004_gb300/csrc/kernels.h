@@ -10,7 +10,10 @@ const void* generic_kernel(int dtype, bool vector_path, bool stoch);
 // fuse_verify_tma<T, STOCH> (k_tma_bf16.cu, k_tma_f32.cu)
 const void* tma_kernel_bf16(bool stoch);
 const void* tma_kernel_f32(bool stoch);
-// decide_rows<T, STOCH>, launched after fuse_verify_tma (same files)
+// fuse_verify_ring<T, STOCH> (k_ring_bf16.cu, k_ring_f32.cu)
+const void* ring_kernel_bf16(bool stoch);
+const void* ring_kernel_f32(bool stoch);
+// decide_rows<T, STOCH>, launched after fuse_verify_tma or fuse_verify_ring (k_tma_*.cu)
 const void* decide_kernel_bf16(bool stoch);
 const void* decide_kernel_f32(bool stoch);
 // fuse_verify_stream<T, STOCH> (k_stream_*.cu)

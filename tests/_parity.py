@@ -38,7 +38,7 @@ def run_gpu(batch, torch, *, mode, divergence=A.DIV_JSD, gamma=0.5, beta=1.0, la
     """
     x = inputs if inputs is not None else device_inputs(batch, torch)
     elt = 4 if batch.dtype == synth.FP32 else 2
-    if kernel in (A.KERNEL_TMA, A.KERNEL_STREAM) and (batch.V * elt) % 16:
+    if kernel in (A.KERNEL_TMA, A.KERNEL_STREAM, A.KERNEL_RING) and (batch.V * elt) % 16:
         kernel = A.KERNEL_AUTO  # rows not 16-byte aligned: only the generic kernel applies
     fv = A.FuseVerify(batch.B, batch.K)
     res = fv(x["a"], x["b"], x["t"], x["tokens"], x["probs"], x["unif"], gamma=gamma, beta=beta,

@@ -144,6 +144,15 @@ def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
     info = A.plan(1, 4, 32000, A.FP32, opts=STREAM)
     assert info.kernel == A.KERNEL_STREAM and info.slice_elems == 8192
     assert A.plan(64, 7, 128256, A.BF16).kernel == A.KERNEL_TMA      # the automatic choice
+    RING = A.LaunchOpts(0, 0, A.KERNEL_RING)
+    # the ring kernel keeps no slice in shared memory: clusters of 8 while a
+    # slice takes at most 10 rounds of 256 vectors, else 16
+    info = A.plan(64, 7, 128256, A.BF16, opts=RING)
+    assert info.kernel == A.KERNEL_RING and info.cluster_size == 8 and info.slice_elems == 16032
+    info = A.plan(256, 4, 151936, A.FP32, opts=RING)
+    assert info.kernel == A.KERNEL_RING and info.cluster_size == 16
+    with pytest.raises(A.AsymSpecError):      # unaligned rows cannot use bulk copies
+        A.plan(2, 2, 4099, A.BF16, opts=RING)
     TMA = A.LaunchOpts(0, 0, A.KERNEL_TMA)
     # the cluster kernel on the bench workload: 8 CTAs of 96 KB per row, two per SM
     info = A.plan(64, 7, 128256, A.BF16, opts=TMA)

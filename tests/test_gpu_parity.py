@@ -1,10 +1,11 @@
 """GPU path (through the C ABI) against the float64 oracle on the same inputs.
 
-Every case runs on the kernel the library picks (the TMA kernel for 16-byte
-aligned rows) and, where it applies, on the generic kernel; and both
-with the production program (accept/next plus row tokens, the work the
-benchmark times) and with every debug output (row statistics, fused
-log-probs), which runs the full per-row program.
+Every case runs on the kernel the library picks (the one-shot TMA kernel
+for 16-byte aligned rows, the generic kernel otherwise) and on the ring,
+streaming and generic kernels where they apply; with the production program
+(accept/next plus row tokens, the work the benchmark times) and with every
+debug output (row statistics, fused log-probs), which runs the full per-row
+program.
 """
 import numpy as np
 import pytest
@@ -18,11 +19,12 @@ pytestmark = pytest.mark.gpu
 
 GREEDY, STOCH = A.MODE_GREEDY, A.MODE_STOCHASTIC
 AUTO, GENERIC, TMA = A.KERNEL_AUTO, A.KERNEL_GENERIC, A.KERNEL_TMA
-STREAM = A.KERNEL_STREAM
-# the automatic choice (the cluster TMA kernel for aligned rows), the
-# streaming kernel, and the generic cluster kernel
-PATHS = [(AUTO, False), (AUTO, True), (STREAM, False), (STREAM, True), (GENERIC, True)]
-PATH_IDS = ["auto-prod", "auto-full", "stream-prod", "stream-full", "generic-full"]
+STREAM, RING = A.KERNEL_STREAM, A.KERNEL_RING
+# the automatic choice (the one-shot TMA kernel for aligned rows), the
+# persistent ring kernel, the streaming kernel, and the generic cluster kernel
+PATHS = [(AUTO, False), (AUTO, True), (RING, False), (STREAM, False), (STREAM, True),
+         (GENERIC, True)]
+PATH_IDS = ["auto-prod", "auto-full", "ring-prod", "stream-prod", "stream-full", "generic-full"]
 
 
 @pytest.fixture(scope="module")
@@ -189,7 +191,7 @@ def test_data_errors_never_trap(torch, kernel, full):
     assert word & A.DATA_BAD_PROB and word & A.DATA_BAD_UNIFORM
 
 
-@pytest.mark.parametrize("kernel", [GENERIC, TMA, STREAM])
+@pytest.mark.parametrize("kernel", [GENERIC, TMA, STREAM, RING])
 def test_exact_ties_resolve_to_lowest_index(torch, kernel):
     B, K, V = 2, 2, 4096
     a = np.zeros((B, K + 1, V), np.float32)
@@ -200,7 +202,7 @@ def test_exact_ties_resolve_to_lowest_index(torch, kernel):
     batch = synth.Batch(a, b, t, np.full((B, K), 7, np.int32), np.full((B, K), 0.5, np.float32),
                         np.full((B, K + 1), 0.5, np.float32), B, K, V, synth.FP32)
     for cluster in ((0,) if kernel == STREAM else (0, 1, 4, 16)):
-        for full in (False, True):
+        for full in ((False,) if kernel == RING else (False, True)):  # RING: no debug outputs
             g = run_gpu(batch, torch, mode=GREEDY, cluster_size=cluster, gamma=1.0,
                         kernel=kernel, full=full, fuse_bonus=True)
             assert list(g["row_tokens"][0, :, 0]) == [100] * (K + 1)
@@ -265,11 +267,19 @@ def test_plan_reports_cluster_occupancy(torch):
     assert info.smem_bytes <= 113 * 1024
     info = A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(0, 0, A.KERNEL_GENERIC))
     assert info.kernel == A.KERNEL_GENERIC and info.max_active_clusters > 0
+    # the persistent ring kernel: every resident cluster of 8 (two CTAs per SM)
+    RING_OPTS = A.LaunchOpts(0, 0, A.KERNEL_RING)
+    info = A.plan(64, 7, 128256, A.BF16, opts=RING_OPTS)
+    assert info.kernel == A.KERNEL_RING and info.cluster_size == 8
+    assert info.max_active_clusters >= 30
+    assert info.ctas == min(info.max_active_clusters, 64 * 8) * 8
+    info = A.plan(1, 1, 128256, A.BF16, opts=RING_OPTS)  # fewer rows than resident clusters
+    assert info.kernel == A.KERNEL_RING and info.ctas == 2 * 8
 
 
 # ---------------------------------------------------------------- sampling law
 
-@pytest.mark.parametrize("kernel", [GENERIC, TMA, STREAM])
+@pytest.mark.parametrize("kernel", [GENERIC, TMA, STREAM, RING])
 def test_emitted_token_law_chi_square(torch, kernel):
     from scipy.stats import chisquare
     V, K, N = 8, 1, 1_000_000
