@@ -314,7 +314,9 @@ cudaLaunchConfig_t launch_config(const Plan& pl, long long ctas, cudaStream_t st
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.gridDim = dim3(static_cast<unsigned>(ctas));
-  cfg.blockDim = dim3(pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : kTThreads);
+  cfg.blockDim = dim3(pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads
+                      : pl.kernel == ASYMSPEC_KERNEL_RING  ? kRThreads
+                                                            : kTThreads);
   cfg.dynamicSmemBytes = pl.smem;
   cfg.stream = stream;
   cfg.attrs = attr;
@@ -530,7 +532,9 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
     return ASYMSPEC_OK;
   }
   out->cluster_size = pl.C;
-  out->block_threads = pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : kTThreads;
+  out->block_threads = pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads
+                       : pl.kernel == ASYMSPEC_KERNEL_RING  ? kRThreads
+                                                             : kTThreads;
   out->slice_elems = pl.W;
   out->smem_bytes = pl.smem;
   out->ctas = pl.ctas;

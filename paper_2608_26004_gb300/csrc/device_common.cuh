@@ -301,17 +301,44 @@ __device__ __forceinline__ bool mbar_try_wait(unsigned long long* bar, unsigned 
       : "memory");
   return ok != 0;
 }
+// Non-blocking test of the phase with the given parity (try_wait may suspend
+// the thread for a while; test_wait returns at once).
+__device__ __forceinline__ bool mbar_test_wait(unsigned long long* bar, unsigned parity) {
+  unsigned ok;
+  asm volatile(
+      "{ .reg .pred p; mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 __device__ __forceinline__ unsigned long long global_ns() {
   unsigned long long t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
+// As mbar_try_wait, suspending the thread for up to hint_ns while the phase
+// is incomplete (the thread resumes as soon as it completes), so a waiting
+// warp takes no issue slots.
+__device__ __forceinline__ bool mbar_try_wait_hint(unsigned long long* bar, unsigned parity,
+                                                   unsigned hint_ns) {
+  unsigned ok;
+  asm volatile(
+      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; "
+      "selp.u32 %0, 1, 0, p; }"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+constexpr unsigned kSuspendHintNs = 100000;  // 0.1 ms per suspension
+
 // Waits for the phase with the given parity, giving up after limit_ns.
 __device__ __forceinline__ bool mbar_wait_bounded(unsigned long long* bar, unsigned parity,
                                                   unsigned long long limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = global_ns();
-  while (!mbar_try_wait(bar, parity)) {
+  while (!mbar_try_wait_hint(bar, parity, kSuspendHintNs)) {
     if (global_ns() - t0 > limit_ns) return false;
   }
   return true;

@@ -6,20 +6,18 @@
 // cluster kernel (kernel_tma.cuh), whose per-entry arithmetic this kernel
 // shares.  What differs is where the slice lives:
 //
-//   pass 1  streams the slice through a ring of kRStages shared-memory stages,
-//           one round (256 vectors of each of a, b, t) per stage, filled by
-//           1-D bulk copies that thread 0 keeps issuing ahead of the
-//           consumers, across row boundaries (L2 policy evict_last);
-//   pass 2  reads the slice again from global memory, where pass 1 has just
-//           brought it into L2.
+// both passes stream the slice through a ring of kRStages shared-memory
+// stages, one round (256 vectors of each of a, b, t) per stage, filled by
+// 1-D bulk copies that thread 0 keeps issuing ahead of the consumers, across
+// pass and row boundaries: for each row the ring carries the slice's rounds
+// for pass 1 (from HBM), then the same rounds again for pass 2, which finds
+// them in L2 one slice later (L2 policy evict_first on the second copy).
+// A row without pass 2 still takes its ring positions, with no copies.
 //
-// Rows are processed with a lag of one: pass 1 of row i + 1 runs between
-// pass 1 and pass 2 of row i, so the exchange of pass-1 records inside the
-// cluster (DSMEM stores plus a remote mbarrier arrive into each peer) has a
-// whole pass to land, and the ring keeps prefetching the next rows while
-// pass 2 runs.  Each CTA keeps four record slots: a peer can push row i as
-// soon as it has taken this CTA's push of row i - 2, when this CTA may not
-// have read row i - 3 yet.  No cluster-wide barrier is
+// Between the passes each CTA pushes its pass-1 record to every CTA of the
+// cluster (DSMEM stores plus a remote mbarrier arrive) and waits for the
+// others', while the ring keeps loading.  Each CTA keeps kRSlots record
+// slots, so a peer that is ahead never overwrites a record not yet read.  No cluster-wide barrier is
 // taken per row; each row's decision is left to decide_rows, from the same
 // workspace records the one-shot kernel writes.
 //
@@ -37,6 +35,7 @@
 namespace asymspec_impl {
 
 constexpr int kRStages = 8;                             // ring stages (rounds in flight)
+constexpr int kRThreads = kTThreads + 32;               // 8 consumer warps + 1 producer warp
 constexpr int kRSlots = 4;                              // pass-1 record slots per peer
 constexpr int kRStreamBytes = kTThreads * 16;           // one round of one stream
 constexpr int kRStageBytes = 3 * kRStreamBytes;         // one round of a, b and t
@@ -69,8 +68,9 @@ struct RingCtx {
   int W, lo, n, nv, rounds;    // this CTA's slice
   unsigned seq;                // next ring sequence number to consume
   unsigned issued;             // next to issue (thread 0)
-  unsigned total;              // nrows * rounds
-  unsigned long long pol;      // L2 policy of the pass-1 copies
+  unsigned total;              // nrows * 2 * rounds
+  unsigned long long pol1;     // L2 policy of the pass-1 copies
+  unsigned long long pol2;     // L2 policy of the pass-2 copies
 };
 
 __device__ __forceinline__ long long ring_row(const RingCtx& c, int i) {
@@ -83,41 +83,59 @@ __device__ __forceinline__ bool ring_only_t(const KParams& P, long long row) {
   return !STOCH && !P.fuse_bonus && static_cast<int>(row % (P.K + 1)) == P.K;
 }
 
+// Rows with a pass 2: every stochastic row; greedy draft rows with a JSD or KL gate.
+template <bool STOCH>
+__device__ __forceinline__ bool ring_has_pass2(const KParams& P, long long row) {
+  if (STOCH) return true;
+  return static_cast<int>(row % (P.K + 1)) != P.K &&
+         (P.divergence == ASYMSPEC_DIV_JSD || P.divergence == ASYMSPEC_DIV_KL);
+}
+
 // What thread 0 needs to issue copies (passed by value).
 struct RingIssue {
   SharedRing* sh;
   unsigned char* ring;
   int q, ncl, rounds, nv, lo;
   unsigned total;
-  unsigned long long pol;
+  unsigned long long pol1, pol2;
 };
 
 __device__ __forceinline__ RingIssue ring_issue_of(const RingCtx& c) {
-  return RingIssue{c.sh, c.ring, c.q, c.ncl, c.rounds, c.nv, c.lo, c.total, c.pol};
+  return RingIssue{c.sh, c.ring, c.q, c.ncl, c.rounds, c.nv, c.lo, c.total, c.pol1, c.pol2};
 }
 
-// Thread 0: the copies of ring sequence number n (local row n / rounds,
-// round n % rounds) into stage n % kRStages.
+// Thread 0: the copies of ring sequence number n into stage n % kRStages.
+// Local row i takes sequence numbers [2 i R, 2 i R + R) for pass 1 and the
+// next R for pass 2 (R = rounds); round kr of a pass is vectors
+// [256 kr, 256 kr + 256) of the slice.
 template <typename T, bool STOCH>
 __device__ __forceinline__ void ring_issue(const KParams& P, const RingIssue& c, unsigned n) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   const int s = static_cast<int>(n % kRStages);
-  const int i = static_cast<int>(n / c.rounds);
-  const int kr = static_cast<int>(n % c.rounds);
+  const unsigned R = static_cast<unsigned>(c.rounds);
+  const int i = static_cast<int>(n / (2u * R));
+  const unsigned w = n - static_cast<unsigned>(i) * 2u * R;
+  const bool second = w >= R;
+  const int kr = static_cast<int>(second ? w - R : w);
   const long long row = static_cast<long long>(c.q) + static_cast<long long>(i) * c.ncl;
+  unsigned long long* bar = &c.sh->full[s];
+  if (second && !ring_has_pass2<STOCH>(P, row)) {
+    mbar_arrive(bar);  // an empty position: nothing to copy
+    return;
+  }
+  const unsigned long long pol = second ? c.pol2 : c.pol1;
   const bool only_t = ring_only_t<STOCH>(P, row);
   const int v0 = kr * kTThreads;
   const int v1 = min(c.nv, v0 + kTThreads);
   const unsigned bytes = static_cast<unsigned>(v1 - v0) * 16u;
   unsigned char* st = c.ring + s * kRStageBytes;
-  unsigned long long* bar = &c.sh->full[s];
   mbar_arrive_expect_tx(bar, bytes * (only_t ? 1u : 3u));
   const size_t off = static_cast<size_t>(row) * P.V + c.lo + static_cast<size_t>(v0) * VE;
   if (!only_t) {
-    bulk_load_hint(st, static_cast<const T*>(P.a) + off, bytes, bar, c.pol);
-    bulk_load_hint(st + kRStreamBytes, static_cast<const T*>(P.b) + off, bytes, bar, c.pol);
+    bulk_load_hint(st, static_cast<const T*>(P.a) + off, bytes, bar, pol);
+    bulk_load_hint(st + kRStreamBytes, static_cast<const T*>(P.b) + off, bytes, bar, pol);
   }
-  bulk_load_hint(st + 2 * kRStreamBytes, static_cast<const T*>(P.t) + off, bytes, bar, c.pol);
+  bulk_load_hint(st + 2 * kRStreamBytes, static_cast<const T*>(P.t) + off, bytes, bar, pol);
 }
 
 // Thread 0: issues every sequence number from `issued` on whose stage is
@@ -133,7 +151,7 @@ __device__ __noinline__ unsigned ring_top_up_impl(const KParams& P, RingIssue c,
       // the stage's previous use, sequence n - kRStages, must be released
       unsigned long long* e = &c.sh->empty[n % kRStages];
       const unsigned par = ((n / kRStages) + 1u) & 1u;
-      if (!mbar_try_wait(e, par)) {
+      if (!mbar_test_wait(e, par)) {
         if (!block || n > upto) break;
         if (!mbar_wait_bounded(e, par, kCopyTimeoutNs)) {
           atomicOr(&c.sh->broken, kBadTimeout);
@@ -147,9 +165,11 @@ __device__ __noinline__ unsigned ring_top_up_impl(const KParams& P, RingIssue c,
   return issued;
 }
 
+// The producer warp's lane 0: every sequence number in order, each once its
+// stage's previous use has been released (bounded waits).
 template <typename T, bool STOCH>
-__device__ __forceinline__ void ring_top_up(const KParams& P, RingCtx& c, unsigned upto, bool block) {
-  c.issued = ring_top_up_impl<T, STOCH>(P, ring_issue_of(c), c.issued, upto, block);
+__device__ __forceinline__ void ring_produce(const KParams& P, RingCtx& c) {
+  c.issued = ring_top_up_impl<T, STOCH>(P, ring_issue_of(c), 0u, c.total, true);
 }
 
 // Waits (bounded) for the stage of sequence number n; false on a timeout.
@@ -164,6 +184,21 @@ __device__ __forceinline__ bool ring_wait(RingCtx& c, unsigned n) {
 __device__ __forceinline__ void ring_release(RingCtx& c, unsigned n) {
   __syncwarp();
   if ((threadIdx.x & 31) == 0) mbar_arrive(&c.sh->empty[n % kRStages]);
+}
+
+// Barrier over the 256 consumer threads (named barrier 1; the producer warp
+// never takes part), and its OR-reduction form.
+__device__ __forceinline__ void consumer_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kTThreads) : "memory");
+}
+__device__ __forceinline__ bool consumer_sync_or(bool v) {
+  unsigned r;
+  asm volatile(
+      "{ .reg .pred p, q; setp.ne.u32 p, %1, 0; bar.red.or.pred q, 1, %2, p; selp.u32 %0, 1, 0, q; }"
+      : "=r"(r)
+      : "r"(v ? 1u : 0u), "n"(kTThreads)
+      : "memory");
+  return r != 0;
 }
 
 // Vector `slot` (0 .. 255) of stream q (0 a, 1 b, 2 t) in the stage of n.
@@ -200,7 +235,6 @@ __device__ __forceinline__ bool ring_pass1(const KParams& P, RingCtx& c, const T
     for (int q = 0; q < 4; ++q) e.s[q] = 0.f;
     return false;
   }
-  if (tid == 0) ring_top_up<T, STOCH>(P, c, s0 + (c.rounds > 1 ? 1u : 0u), true);
   ring_wait(c, s0);
   float ref[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
   if (tid < c.nv) {
@@ -228,10 +262,7 @@ __device__ __forceinline__ bool ring_pass1(const KParams& P, RingCtx& c, const T
   for (int kr = 0; kr < c.rounds; kr += 2) {
     const unsigned n0 = s0 + static_cast<unsigned>(kr);
     const bool two = kr + 1 < c.rounds;
-    if (kr > 0) {
-      if (tid == 0) ring_top_up<T, STOCH>(P, c, two ? n0 + 1 : n0, true);
-      ring_wait(c, n0);
-    }
+    if (kr > 0) ring_wait(c, n0);
     if (two) ring_wait(c, n0 + 1);
     const int i0 = kr * kTThreads + tid;
     const bool has0 = i0 < c.nv;
@@ -301,6 +332,61 @@ __device__ __forceinline__ bool ring_pass1(const KParams& P, RingCtx& c, const T
   return ovf;
 }
 
+// ---------------------------------------------------------------- pass 2
+
+// Pass 2 of one row from the ring (the second R sequence numbers of the row),
+// two rounds per step; as pass2 in kernel_tma.cuh, with the slice's rounds in
+// ring stages instead of a resident slice.
+template <typename T, bool STOCH, unsigned G>
+__device__ __forceinline__ void ring_pass2(const KParams& P, RingCtx& c, float A2, float B2,
+                                           float S2, float lse_s, X2& x, float* grp) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  constexpr int NP = VE / 2;
+  constexpr bool needT = (G & (G_RES | G_QF)) != 0;
+  const int tid = static_cast<int>(threadIdx.x);
+  const unsigned s0 = c.seq;
+  c.seq = s0 + static_cast<unsigned>(c.rounds);
+  const P2Const k = p2_const(P.beta, A2, B2, S2, lse_s);
+  P2Acc acc = {0ull, 0ull, 0ull, 0ull, 0ull, 0ull};
+  for (int kr = 0; kr < c.rounds; kr += 2) {
+    const unsigned n0 = s0 + static_cast<unsigned>(kr);
+    const bool two = kr + 1 < c.rounds;
+    ring_wait(c, n0);
+    if (two) ring_wait(c, n0 + 1);
+    const int i0 = kr * kTThreads + tid;
+    const bool has1 = two && i0 + kTThreads < c.nv;
+    float g0 = 0.f, g1 = 0.f;
+    if (i0 < c.nv) {
+      f2 xa[NP], xb[NP], xt[NP], ya[NP], yb[NP], yt[NP];
+      load_pairs(ring_vec<T>(c, n0, 0, tid), xa);
+      load_pairs(ring_vec<T>(c, n0, 1, tid), xb);
+      load_or_fill(ring_vec<T>(c, n0 + 1, 0, tid), has1, ya);
+      load_or_fill(ring_vec<T>(c, n0 + 1, 1, tid), has1, yb);
+      if (needT) {
+        load_pairs(ring_vec<T>(c, n0, 2, tid), xt);
+        load_or_fill(ring_vec<T>(c, n0 + 1, 2, tid), has1, yt);
+      }
+      p2_pair<NP, G, false>(xa, xb, xt, ya, yb, yt, has1, k, acc, g0, g1, nullptr, nullptr);
+    }
+    if (G & (G_RES | G_QF)) p2_groups(g0, g1, grp, kr, c.rounds);
+    ring_release(c, n0);
+    if (two) ring_release(c, n0 + 1);
+  }
+  p2_finish(acc, x);
+}
+
+// The ring positions of a row without pass 2 (no copies behind them).
+template <typename T, bool STOCH>
+__device__ __forceinline__ void ring_skip(const KParams& P, RingCtx& c) {
+  const unsigned s0 = c.seq;
+  c.seq = s0 + static_cast<unsigned>(c.rounds);
+  for (int kr = 0; kr < c.rounds; ++kr) {
+    const unsigned n = s0 + static_cast<unsigned>(kr);
+    ring_wait(c, n);
+    ring_release(c, n);
+  }
+}
+
 // The CTA's pass-1 record of row i goes into slot i % kRSlots of every CTA
 // of the cluster (lane r of warp 0 stores into CTA r and arrives, with
 // cluster-scope release, on that CTA's row barrier).
@@ -321,7 +407,7 @@ __device__ __forceinline__ void ring_row_pass1(const KParams& P, RingCtx& c, int
   warp_reduce_x1<F>(e);
   X1* w1 = sh->w1[i & 1];
   if (lane == 0) w1[warp] = e;
-  if (__syncthreads_or(ovf)) {
+  if (consumer_sync_or(ovf)) {
     // an entry far above its thread's reference (or non-finite data): redo
     // the slice, from global memory, with a running maximum
     e = x1_neutral();
@@ -329,7 +415,7 @@ __device__ __forceinline__ void ring_row_pass1(const KParams& P, RingCtx& c, int
                               nullptr, e);
     warp_reduce_x1<F>(e);
     if (lane == 0) w1[warp] = e;
-    __syncthreads();
+    consumer_sync();
   }
   if (warp == 0) {
     X1 w = (lane < kTWarps) ? w1[lane] : x1_neutral();
@@ -359,13 +445,13 @@ __device__ __forceinline__ void ring_row_pass1(const KParams& P, RingCtx& c, int
 
 // Row i once every CTA's pass-1 record is in: its normalisers (rank 0
 // leaves the row's pass-1 results for decide_rows) and, with R2, pass 2 from
-// global memory and this CTA's pass-2 record and group masses.
+// the ring and this CTA's pass-2 record and group masses (else the row's
+// empty pass-2 positions are passed over).
 template <typename T, bool STOCH, unsigned F, unsigned G, bool R2>
 __device__ __forceinline__ void ring_row_finish(const KParams& P, RingCtx& c, int i) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const long long row = ring_row(c, i);
   SharedRing* sh = c.sh;
-  if (threadIdx.x == 0) ring_top_up<T, STOCH>(P, c, 0, false);
   if (warp == 0) {
     const int slot = i % kRSlots;
     const bool ok =
@@ -402,19 +488,15 @@ __device__ __forceinline__ void ring_row_finish(const KParams& P, RingCtx& c, in
     }
   }
   if constexpr (R2) {
-    __syncthreads();
-    const size_t off = static_cast<size_t>(row) * P.V + c.lo;
-    const T* ga = static_cast<const T*>(P.a) + off;
-    const T* gb = static_cast<const T*>(P.b) + off;
-    const T* gt = static_cast<const T*>(P.t) + off;
+    consumer_sync();
     const size_t slot = static_cast<size_t>(row) * c.C + c.rank;
     const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
     X2 x = x2_zero();
-    pass2<T, G, false>(ga, gb, gt, c.nv, c.rounds, P.beta, lse_a * kLog2e, lse_b * kLog2e,
-                       lse_s * kLog2e, lse_s, x, nullptr, P.group_mass + slot * kGroupsMax);
+    ring_pass2<T, STOCH, G>(P, c, lse_a * kLog2e, lse_b * kLog2e, lse_s * kLog2e, lse_s, x,
+                            P.group_mass + slot * kGroupsMax);
     warp_reduce_x2<G>(x);
     if (lane == 0) sh->w2[warp] = x;
-    __syncthreads();
+    consumer_sync();
     if (warp == 0) {
       X2 w = (lane < kTWarps) ? sh->w2[lane] : x2_zero();
       warp_reduce_x2<G>(w);
@@ -423,6 +505,8 @@ __device__ __forceinline__ void ring_row_finish(const KParams& P, RingCtx& c, in
         reinterpret_cast<float4*>(P.pass2_rec + slot * 8)[lane] =
             reinterpret_cast<const float4*>(&w)[lane];
     }
+  } else {
+    ring_skip<T, STOCH>(P, c);
   }
 }
 
@@ -482,7 +566,7 @@ __device__ __forceinline__ void ring_dispatch_finish(const KParams& P, RingCtx& 
 // ---------------------------------------------------------------- the kernel
 
 template <typename T, bool STOCH>
-__global__ void __launch_bounds__(kTThreads, 2) fuse_verify_ring(const __grid_constant__ KParams P) {
+__global__ void __launch_bounds__(kRThreads, 2) fuse_verify_ring(const __grid_constant__ KParams P) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   extern __shared__ __align__(128) unsigned char smem_ring[];
   cg::cluster_group cluster = cg::this_cluster();
@@ -501,8 +585,9 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_ring(const __grid_co
   c.rounds = (c.nv + kTThreads - 1) / kTThreads;
   c.seq = 0;
   c.issued = 0;
-  c.total = static_cast<unsigned>(c.nrows) * static_cast<unsigned>(c.rounds);
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(c.pol));
+  c.total = static_cast<unsigned>(c.nrows) * 2u * static_cast<unsigned>(c.rounds);
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(c.pol1));
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(c.pol2));
   SharedRing* sh = c.sh;
   if (threadIdx.x == 0) {
 #pragma unroll
@@ -515,21 +600,25 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_ring(const __grid_co
     sh->broken = 0;
     fence_mbar_init();
   }
+  __syncwarp();
   cluster.sync();  // every CTA's barriers are initialised before any remote arrive
-  if (threadIdx.x == 0) ring_top_up<T, STOCH>(P, c, 0, false);
-  if (c.nrows > 0) {
-    ring_dispatch_pass1<T, STOCH>(P, c, 0, cluster);
+  if (threadIdx.x >= kTThreads) {
+    // the producer warp: lane 0 keeps the ring full
+    if (threadIdx.x == kTThreads) ring_produce<T, STOCH>(P, c);
+    __syncwarp();
+  } else {
     for (int i = 0; i < c.nrows; ++i) {
-      if (i + 1 < c.nrows) ring_dispatch_pass1<T, STOCH>(P, c, i + 1, cluster);
+      ring_dispatch_pass1<T, STOCH>(P, c, i, cluster);
       ring_dispatch_finish<T, STOCH>(P, c, i);
     }
   }
   // after a timeout, copies still in flight land before the CTA exits
-  if (threadIdx.x == 0 && sh->broken) {
+  if (threadIdx.x == kTThreads && sh->broken) {
     for (unsigned n = c.issued > static_cast<unsigned>(kRStages) ? c.issued - kRStages : 0u;
          n < c.issued; ++n)
       mbar_wait_bounded(&sh->full[n % kRStages], (n / kRStages) & 1u, kCopyTimeoutNs);
   }
+  __syncwarp();
   cluster.sync();  // no CTA leaves while a peer may still push into it
 }
 

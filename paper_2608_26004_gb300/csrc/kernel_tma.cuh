@@ -661,103 +661,140 @@ __device__ __forceinline__ void div_terms(const f2 (&xa)[NP], const f2 (&xb)[NP]
   }
 }
 
-// Pass 2 over the slice, two vectors per step (an absent second vector is
-// filled with -1e30, which contributes nothing).
+// Pass-2 constants and running sums of one thread.
+struct P2Const {
+  f2 beta2, L2, nA2, nB2, nS2, tiny2, nl2;
+};
+struct P2Acc {
+  f2 ja, jb, ms2, kl2, R2, Q2;
+};
+
+__device__ __forceinline__ P2Const p2_const(float beta, float A2, float B2, float S2,
+                                            float lse_s) {
+  P2Const k;
+  k.beta2 = pk(beta, beta);
+  k.L2 = pk(kLog2e, kLog2e);
+  k.nA2 = pk(-A2, -A2);
+  k.nB2 = pk(-B2, -B2);
+  k.nS2 = pk(-S2, -S2);
+  k.tiny2 = pk(kMinNormal, kMinNormal);
+  k.nl2 = pk(-lse_s, -lse_s);
+  return k;
+}
+
+// Pass 2 on two vectors x, y of a thread (y absent unless has1: filled with
+// -1e30, which contributes nothing); g0, g1 receive their inverse-CDF masses
+// (residual, or fused for G_QF).  LP: fused log-probs go to lpx, lpy.
+template <int NP, unsigned G, bool LP>
+__device__ __forceinline__ void p2_pair(const f2 (&xa)[NP], const f2 (&xb)[NP], const f2 (&xt)[NP],
+                                        const f2 (&ya)[NP], const f2 (&yb)[NP], const f2 (&yt)[NP],
+                                        bool has1, const P2Const& k, P2Acc& acc, float& g0,
+                                        float& g1, float* lpx, float* lpy) {
+  constexpr bool JSD = (G & G_JSD) != 0, KL = (G & G_KL) != 0, RES = (G & G_RES) != 0;
+  constexpr bool QF = (G & G_QF) != 0;
+  f2 px[NP], py[NP];
+  if (RES) {
+    f2 qx[NP], qy[NP], rx[NP], ry[NP];
+    vec_masses(xa, xb, xt, k.beta2, k.L2, k.nA2, k.nS2, px, qx, rx);
+    vec_masses(ya, yb, yt, k.beta2, k.L2, k.nA2, k.nS2, py, qy, ry);
+#pragma unroll
+    for (int h = 0; h < NP; ++h) acc.Q2 = add2(acc.Q2, add2(qx[h], qy[h]));
+    // residual mass of each vector, summed per group for the inverse-CDF walk
+    g0 = vsum(rx);
+    g1 = vsum(ry);
+    acc.R2 = add2(acc.R2, pk(g0, g1));
+  } else if (QF) {
+    f2 qx[NP], qy[NP];
+#pragma unroll
+    for (int h = 0; h < NP; ++h) {
+      qx[h] = ex2_2(fma2(fma2(k.beta2, sub2(xa[h], xb[h]), xt[h]), k.L2, k.nS2));
+      qy[h] = ex2_2(fma2(fma2(k.beta2, sub2(ya[h], yb[h]), yt[h]), k.L2, k.nS2));
+    }
+    // fused mass of each vector, summed per group for the inverse-CDF walk
+    g0 = vsum(qx);
+    g1 = vsum(qy);
+    acc.Q2 = add2(acc.Q2, pk(g0, g1));
+  } else if (JSD || KL) {
+#pragma unroll
+    for (int h = 0; h < NP; ++h) {
+      px[h] = ex2_2(fma2(xa[h], k.L2, k.nA2));
+      py[h] = ex2_2(fma2(ya[h], k.L2, k.nA2));
+    }
+  }
+  if (JSD || KL) {
+    div_terms<NP, JSD, KL>(xa, xb, px, k.L2, k.nA2, k.nB2, k.tiny2, acc.ja, acc.jb, acc.ms2,
+                           acc.kl2);
+    div_terms<NP, JSD, KL>(ya, yb, py, k.L2, k.nA2, k.nB2, k.tiny2, acc.ja, acc.jb, acc.ms2,
+                           acc.kl2);
+  }
+  if (LP) {
+#pragma unroll
+    for (int h = 0; h < NP; ++h) {
+      float l0, l1;
+      upk(add2(fma2(k.beta2, sub2(xa[h], xb[h]), xt[h]), k.nl2), l0, l1);
+      lpx[2 * h] = l0;
+      lpx[2 * h + 1] = l1;
+      if (has1) {
+        upk(add2(fma2(k.beta2, sub2(ya[h], yb[h]), yt[h]), k.nl2), l0, l1);
+        lpy[2 * h] = l0;
+        lpy[2 * h + 1] = l1;
+      }
+    }
+  }
+}
+
+// The inverse-CDF group masses of rounds kr and kr + 1 of one warp (every
+// lane takes part, with or without a vector): one butterfly, lanes 0-15
+// carrying round kr and lanes 16-31 round kr + 1.
+__device__ __forceinline__ void p2_groups(float g0, float g1, float* grp, int kr, int rounds) {
+  const int lane = static_cast<int>(threadIdx.x & 31), warp = static_cast<int>(threadIdx.x >> 5);
+  const bool upper = lane >= 16;
+  float g = (upper ? g1 : g0) + __shfl_xor_sync(0xffffffffu, upper ? g0 : g1, 16);
+#pragma unroll
+  for (int off = 8; off > 0; off >>= 1) g += __shfl_xor_sync(0xffffffffu, g, off);
+  if (lane == 0) grp[kr * kTWarps + warp] = g;
+  if (lane == 16 && kr + 1 < rounds) grp[(kr + 1) * kTWarps + warp] = g;
+}
+
+__device__ __forceinline__ void p2_finish(const P2Acc& acc, X2& x) {
+  x.j = hsum2(add2(acc.ja, acc.jb));
+  x.msum = hsum2(acc.ms2);
+  x.kl = hsum2(acc.kl2);
+  x.R = hsum2(acc.R2);
+  x.Q = hsum2(acc.Q2);
+}
+
+// Pass 2 over the slice, two vectors per step.
 template <typename T, unsigned G, bool LP>
 __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int nv, int rounds,
                                       float beta, float A2, float B2, float S2, float lse_s, X2& x,
                                       float* lp, float* grp) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
-  constexpr bool JSD = (G & G_JSD) != 0, KL = (G & G_KL) != 0, RES = (G & G_RES) != 0;
-  constexpr bool QF = (G & G_QF) != 0;
-  constexpr bool needT = RES || QF || LP;
-  const f2 beta2 = pk(beta, beta);
-  const f2 L2 = pk(kLog2e, kLog2e);
-  const f2 nA2 = pk(-A2, -A2), nB2 = pk(-B2, -B2), nS2 = pk(-S2, -S2);
-  const f2 tiny2 = pk(kMinNormal, kMinNormal);
-  const f2 nl2 = pk(-lse_s, -lse_s);
-  f2 ja = 0ull, jb = 0ull, ms2 = 0ull, kl2 = 0ull, R2 = 0ull, Q2 = 0ull;
-  const int warp = static_cast<int>(threadIdx.x) >> 5;
+  constexpr bool needT = (G & (G_RES | G_QF)) != 0 || LP;
+  const P2Const k = p2_const(beta, A2, B2, S2, lse_s);
+  P2Acc acc = {0ull, 0ull, 0ull, 0ull, 0ull, 0ull};
   for (int kr = 0; kr < rounds; kr += 2) {
     const int i0 = kr * kTThreads + static_cast<int>(threadIdx.x);
     const int i1 = i0 + kTThreads;
     float g0 = 0.f, g1 = 0.f;  // this thread's vector masses in rounds kr and kr + 1
     if (i0 < nv) {
-    const bool has1 = i1 < nv;
-    f2 xa[NP], xb[NP], xt[NP], ya[NP], yb[NP], yt[NP];
-    load_pairs(ra + i0 * VE, xa);
-    load_pairs(rb + i0 * VE, xb);
-    load_or_fill(ra + i1 * VE, has1, ya);
-    load_or_fill(rb + i1 * VE, has1, yb);
-    if (needT) {
-      load_pairs(rt + i0 * VE, xt);
-      load_or_fill(rt + i1 * VE, has1, yt);
-    }
-    f2 px[NP], py[NP];
-    if (RES) {
-      f2 qx[NP], qy[NP], rx[NP], ry[NP];
-      vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, px, qx, rx);
-      vec_masses(ya, yb, yt, beta2, L2, nA2, nS2, py, qy, ry);
-#pragma unroll
-      for (int h = 0; h < NP; ++h) Q2 = add2(Q2, add2(qx[h], qy[h]));
-      // residual mass of each vector, summed per group for the inverse-CDF walk
-      g0 = vsum(rx);
-      g1 = vsum(ry);
-      R2 = add2(R2, pk(g0, g1));
-    } else if (QF) {
-      f2 qx[NP], qy[NP];
-#pragma unroll
-      for (int h = 0; h < NP; ++h) {
-        qx[h] = ex2_2(fma2(fma2(beta2, sub2(xa[h], xb[h]), xt[h]), L2, nS2));
-        qy[h] = ex2_2(fma2(fma2(beta2, sub2(ya[h], yb[h]), yt[h]), L2, nS2));
+      const bool has1 = i1 < nv;
+      f2 xa[NP], xb[NP], xt[NP], ya[NP], yb[NP], yt[NP];
+      load_pairs(ra + i0 * VE, xa);
+      load_pairs(rb + i0 * VE, xb);
+      load_or_fill(ra + i1 * VE, has1, ya);
+      load_or_fill(rb + i1 * VE, has1, yb);
+      if (needT) {
+        load_pairs(rt + i0 * VE, xt);
+        load_or_fill(rt + i1 * VE, has1, yt);
       }
-      // fused mass of each vector, summed per group for the inverse-CDF walk
-      g0 = vsum(qx);
-      g1 = vsum(qy);
-      Q2 = add2(Q2, pk(g0, g1));
-    } else if (JSD || KL) {
-#pragma unroll
-      for (int h = 0; h < NP; ++h) {
-        px[h] = ex2_2(fma2(xa[h], L2, nA2));
-        py[h] = ex2_2(fma2(ya[h], L2, nA2));
-      }
+      p2_pair<NP, G, LP>(xa, xb, xt, ya, yb, yt, has1, k, acc, g0, g1,
+                         LP ? lp + i0 * VE : nullptr, LP ? lp + i1 * VE : nullptr);
     }
-    if (JSD || KL) {
-      div_terms<NP, JSD, KL>(xa, xb, px, L2, nA2, nB2, tiny2, ja, jb, ms2, kl2);
-      div_terms<NP, JSD, KL>(ya, yb, py, L2, nA2, nB2, tiny2, ja, jb, ms2, kl2);
-    }
-    if (LP) {
-#pragma unroll
-      for (int h = 0; h < NP; ++h) {
-        float l0, l1;
-        upk(add2(fma2(beta2, sub2(xa[h], xb[h]), xt[h]), nl2), l0, l1);
-        lp[i0 * VE + 2 * h] = l0;
-        lp[i0 * VE + 2 * h + 1] = l1;
-        if (has1) {
-          upk(add2(fma2(beta2, sub2(ya[h], yb[h]), yt[h]), nl2), l0, l1);
-          lp[i1 * VE + 2 * h] = l0;
-          lp[i1 * VE + 2 * h + 1] = l1;
-        }
-      }
-    }
-    }
-    if (RES || QF) {  // group masses: every lane takes part, with or without a vector
-      // both rounds' sums in one butterfly: lanes 0-15 carry round kr, 16-31 round kr + 1
-      const int lane = static_cast<int>(threadIdx.x & 31);
-      const bool upper = lane >= 16;
-      float g = (upper ? g1 : g0) + __shfl_xor_sync(0xffffffffu, upper ? g0 : g1, 16);
-#pragma unroll
-      for (int off = 8; off > 0; off >>= 1) g += __shfl_xor_sync(0xffffffffu, g, off);
-      if (lane == 0) grp[kr * kTWarps + warp] = g;
-      if (lane == 16 && kr + 1 < rounds) grp[(kr + 1) * kTWarps + warp] = g;
-    }
+    if (G & (G_RES | G_QF)) p2_groups(g0, g1, grp, kr, rounds);
   }
-  x.j = hsum2(add2(ja, jb));
-  x.msum = hsum2(ms2);
-  x.kl = hsum2(kl2);
-  x.R = hsum2(R2);
-  x.Q = hsum2(Q2);
+  p2_finish(acc, x);
 }
 
 // Pass 2 and the CTA combine; warp 0 stores the CTA's pass-2 record in the
