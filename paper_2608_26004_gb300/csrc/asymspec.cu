@@ -38,6 +38,7 @@ constexpr int kTmaPreferredSmem = 113 * 1024;  // two CTAs per SM
 struct Plan {
   int kernel;  // ASYMSPEC_KERNEL_*
   int C, W, VE, sh_off, smem;
+  int group_stride;  // TMA and ring kernels: floats per row and CTA of group masses
   long long rows;
   long long ctas;  // grid size
   bool vector_path;
@@ -84,6 +85,7 @@ bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
     pl->W = static_cast<int>(W);
     pl->sh_off = static_cast<int>(sh_off);
     pl->smem = static_cast<int>(sh_off + shared_bytes);
+    pl->group_stride = kGroupsMax;
     return sh_off + shared_bytes <= kMaxSmem &&
            W / VE <= static_cast<long long>(kMaxRounds) * kTThreads;
   };
@@ -96,17 +98,20 @@ bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
 }
 
 // Persistent ring kernel: clusters of 8 (16 when a slice of 8 would take
-// more than kMaxRounds rounds); the slice is not held in shared memory.
+// more than kRMaxRounds rounds); the slice is not held in shared memory, so
+// smaller clusters (more entries per thread) work too.
 bool plan_ring(int V, int elt, int forced_C, Plan* pl) {
   const int VE = 16 / elt;
   auto fill = [&](int C) {
     const long long per = (static_cast<long long>(V) + C - 1) / C;
     const long long W = round_up_ll(per, VE);
+    const long long rounds = (W / VE + kTThreads - 1) / kTThreads;
     pl->C = C;
     pl->W = static_cast<int>(W);
     pl->sh_off = 0;
     pl->smem = ring_smem_bytes(C);
-    return pl->smem <= kMaxSmem && W / VE <= static_cast<long long>(kMaxRounds) * kTThreads;
+    pl->group_stride = static_cast<int>(rounds) * kTWarps;
+    return pl->smem <= kMaxSmem && rounds <= kRMaxRounds;
   };
   if (forced_C > 0) return fill(forced_C);
   return fill(8) || fill(16);
@@ -130,7 +135,9 @@ struct TmaLayout {
   size_t stat, p2rec, groups, total;
 };
 
-TmaLayout tma_layout(int B, int K, int C) {
+// group_stride: floats of group masses per row and CTA (kGroupsMax for the
+// one-shot kernel, 8 per round for the ring kernel).
+TmaLayout tma_layout(int B, int K, int C, int group_stride = kGroupsMax) {
   TmaLayout L;
   const size_t R = static_cast<size_t>(B) * (K + 1);
   size_t off = cluster_ws_bytes(B, K);
@@ -139,7 +146,7 @@ TmaLayout tma_layout(int B, int K, int C) {
   L.p2rec = off;
   off += round_up(R * C * sizeof(X2), 256);
   L.groups = off;
-  off += round_up(R * C * kGroupsMax * sizeof(float), 256);
+  off += round_up(R * C * static_cast<size_t>(group_stride) * sizeof(float), 256);
   L.total = off;
   return L;
 }
@@ -221,7 +228,7 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
   if (forced_kernel == ASYMSPEC_KERNEL_RING) {
     Plan r = *pl;
     if (vec_ok && !debug_out && plan_ring(V, elt, forced_C, &r) &&
-        ws_bytes >= tma_layout(B, K, r.C).total) {
+        ws_bytes >= tma_layout(B, K, r.C, r.group_stride).total) {
       *pl = r;
       pl->kernel = ASYMSPEC_KERNEL_RING;
       pl->VE = 16 / elt;
@@ -230,8 +237,10 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
     }
     if (forced_kernel == ASYMSPEC_KERNEL_RING) {
       if (!vec_ok || debug_out) return ASYMSPEC_ERR_UNSUPPORTED;
-      return (r.C > 0 && ws_bytes < tma_layout(B, K, r.C).total) ? ASYMSPEC_ERR_WORKSPACE
-                                                                : ASYMSPEC_ERR_TOO_LARGE;
+      return (r.C > 0 && r.group_stride > 0 &&
+              ws_bytes < tma_layout(B, K, r.C, r.group_stride).total)
+                 ? ASYMSPEC_ERR_WORKSPACE
+                 : ASYMSPEC_ERR_TOO_LARGE;
     }
   }
   bool ok = false;
@@ -477,8 +486,16 @@ void asymspec_default_gate_params(asymspec_gate_params* p) {
 
 size_t asymspec_workspace_bytes(int B, int K, int V) {
   if (B < 1 || K < 1) return 0;
-  // the TMA kernel's layout for the largest cluster
+  // the TMA kernel's layout for the largest cluster, and the ring kernel's
+  // for every cluster size it may take
   size_t n = tma_layout(B, K, 16).total;
+  if (V >= 2) {
+    for (int elt : {2, 4})
+      for (int C : {1, 2, 4, 8, 16}) {
+        Plan r = {};
+        if (plan_ring(V, elt, C, &r)) n = std::max(n, tma_layout(B, K, C, r.group_stride).total);
+      }
+  }
   if (V >= 2) {
     // the larger of the two dtypes' streaming layouts (fp32 has more tiles)
     const StreamLayout L4 = stream_layout(B, K, V, 4);
@@ -703,8 +720,9 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = launch_config(pl, ctas, static_cast<cudaStream_t>(stream), attr);
   void* args[] = {&P};
+  P.group_stride = pl.group_stride;
   if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING) {
-    const TmaLayout L = tma_layout(B, K, pl.C);
+    const TmaLayout L = tma_layout(B, K, pl.C, pl.group_stride);
     char* base = static_cast<char*>(workspace);
     P.row_stat = base + L.stat;
     P.pass2_rec = reinterpret_cast<float*>(base + L.p2rec);

@@ -424,7 +424,8 @@ struct KParams {
   // cluster TMA kernel: what its rows leave for the decision kernel
   void* row_stat;       // [B(K+1)] RowStat (rank 0 of the row's cluster)
   float* pass2_rec;     // [B(K+1)][C] X2 records (8 floats), one per CTA
-  float* group_mass;    // [B(K+1)][C][kGroupsMax] inverse-CDF group masses (stochastic)
+  float* group_mass;    // [B(K+1)][C][group_stride] inverse-CDF group masses (stochastic)
+  int group_stride;     // floats per row and CTA in group_mass (8 per round of the slice)
 };
 
 // What pass 1 leaves for the decision of a row: the normalisers, the

@@ -36,6 +36,7 @@ namespace asymspec_impl {
 
 constexpr int kRStages = 8;                             // ring stages (rounds in flight)
 constexpr int kRThreads = kTThreads + 32;               // 8 consumer warps + 1 producer warp
+constexpr int kRMaxRounds = 32;                         // rounds per slice (group walk: 256 groups)
 constexpr int kRSlots = 4;                              // pass-1 record slots per peer
 constexpr int kRStreamBytes = kTThreads * 16;           // one round of one stream
 constexpr int kRStageBytes = 3 * kRStreamBytes;         // one round of a, b and t
@@ -493,7 +494,7 @@ __device__ __forceinline__ void ring_row_finish(const KParams& P, RingCtx& c, in
     const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
     X2 x = x2_zero();
     ring_pass2<T, STOCH, G>(P, c, lse_a * kLog2e, lse_b * kLog2e, lse_s * kLog2e, lse_s, x,
-                            P.group_mass + slot * kGroupsMax);
+                            P.group_mass + slot * P.group_stride);
     warp_reduce_x2<G>(x);
     if (lane == 0) sh->w2[warp] = x;
     consumer_sync();

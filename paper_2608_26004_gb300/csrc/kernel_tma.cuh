@@ -852,25 +852,30 @@ __device__ __forceinline__ void slice_vector_masses(const T* ga, const T* gb, co
 // at or beyond the slice's total.  The slice (ga, gb, gt: global memory,
 // entries from lo) is cut into groups of 32 vectors; gm holds their masses
 // when `stored` (else they are recomputed: the rare fallback to the fused
-// masses of a draft row whose residual is zero).  Lane l takes groups 3l to
-// 3l+2, then the lane holding the target recomputes its group's vectors,
-// one per lane, and the element.  Returns the index within the row, or -1
-// when the slice holds no mass.
+// masses of a draft row whose residual is zero).  Lane l takes groups
+// [l P, l P + P) (P = ceil(ngroups / 32) <= kWalkGroupsPerLane), then the lane
+// holding the target recomputes its group's vectors, one per lane, and the
+// element.  Returns the index within the row, or -1 when the slice holds no
+// mass.
+constexpr int kWalkGroupsPerLane = 8;  // slices of up to 256 groups (32 rounds)
+
 template <typename T, bool GM_GLOBAL>
 __device__ __noinline__ int group_walk(const T* ga, const T* gb, const T* gt, int nvec, int lo,
                                        int ngroups, float beta, const float* gm, bool stored,
                                        bool use_r, float A2, float S2, float tau) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
+  constexpr int GP = kWalkGroupsPerLane;
   const int lane = threadIdx.x & 31;
+  const int gpl = (ngroups + 31) / 32;
   const f2 beta2 = pk(beta, beta), L2 = pk(kLog2e, kLog2e);
   const f2 nA2 = pk(-A2, -A2), nS2 = pk(-S2, -S2);
-  float g3[3];
+  float gl[GP];
 #pragma unroll
-  for (int h = 0; h < 3; ++h) {
-    const int g = 3 * lane + h;
+  for (int h = 0; h < GP; ++h) {
+    const int g = gpl * lane + h;
     float m = 0.f;
-    if (g < ngroups) {
+    if (h < gpl && g < ngroups) {
       if (stored) {
         m = GM_GLOBAL ? __ldcg(gm + g) : gm[g];
       } else {
@@ -884,9 +889,11 @@ __device__ __noinline__ int group_walk(const T* ga, const T* gb, const T* gt, in
         }
       }
     }
-    g3[h] = m;
+    gl[h] = m;
   }
-  const float pl = (g3[0] + g3[1]) + g3[2];
+  float pl = 0.f;
+#pragma unroll
+  for (int h = 0; h < GP; ++h) pl += gl[h];
   float incl = pl;
 #pragma unroll
   for (int off = 1; off < 32; off <<= 1) {
@@ -912,14 +919,14 @@ __device__ __noinline__ int group_walk(const T* ga, const T* gb, const T* gt, in
     float cum = excl;
     int glast = -1;
 #pragma unroll
-    for (int h = 0; h < 3; ++h) {
-      if (g3[h] > 0.f) glast = 3 * lane + h;
-      if (!take_last && gsel < 0) {
-        if (cum + g3[h] > tau) {
-          gsel = 3 * lane + h;
+    for (int h = 0; h < GP; ++h) {
+      if (gl[h] > 0.f) glast = gpl * lane + h;
+      if (h < gpl && !take_last && gsel < 0) {
+        if (cum + gl[h] > tau) {
+          gsel = gpl * lane + h;
           trem = fmaxf(tau - cum, 0.f);
         } else {
-          cum += g3[h];
+          cum += gl[h];
         }
       }
     }
@@ -1054,7 +1061,7 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
     float* lp = LP ? P.logprobs + static_cast<size_t>(c.row) * P.V + c.lo : nullptr;
     const size_t slot = static_cast<size_t>(c.row) * c.C + c.rank;
     pass2_and_store<T, G, LP>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh, P.pass2_rec + slot * 8,
-                              P.group_mass + slot * kGroupsMax);
+                              P.group_mass + slot * P.group_stride);
   }
 }
 
@@ -1253,7 +1260,7 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
         sample = group_walk<T, true>(static_cast<const T*>(P.a) + off,
                                      static_cast<const T*>(P.b) + off,
                                      static_cast<const T*>(P.t) + off, nv_o, lo_o, ng_o, P.beta,
-                                     P.group_mass + (row * C + owner) * kGroupsMax,
+                                     P.group_mass + (row * C + owner) * P.group_stride,
                                      r_ok == stored_r, r_ok, st.lse[0] * kLog2e,
                                      st.lse[3] * kLog2e, tau_local);
       }

@@ -146,11 +146,16 @@ def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
     assert A.plan(64, 7, 128256, A.BF16).kernel == A.KERNEL_TMA      # the automatic choice
     RING = A.LaunchOpts(0, 0, A.KERNEL_RING)
     # the ring kernel keeps no slice in shared memory: clusters of 8 while a
-    # slice takes at most 10 rounds of 256 vectors, else 16
+    # slice takes at most 32 rounds of 256 vectors, else 16; smaller clusters
+    # on request (more entries per thread)
     info = A.plan(64, 7, 128256, A.BF16, opts=RING)
     assert info.kernel == A.KERNEL_RING and info.cluster_size == 8 and info.slice_elems == 16032
     info = A.plan(256, 4, 151936, A.FP32, opts=RING)
-    assert info.kernel == A.KERNEL_RING and info.cluster_size == 16
+    assert info.kernel == A.KERNEL_RING and info.cluster_size == 8
+    info = A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(2, 0, A.KERNEL_RING))
+    assert info.kernel == A.KERNEL_RING and info.cluster_size == 2 and info.slice_elems == 64128
+    with pytest.raises(A.AsymSpecError):      # a single CTA's slice would take 63 rounds
+        A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(1, 0, A.KERNEL_RING))
     with pytest.raises(A.AsymSpecError):      # unaligned rows cannot use bulk copies
         A.plan(2, 2, 4099, A.BF16, opts=RING)
     TMA = A.LaunchOpts(0, 0, A.KERNEL_TMA)

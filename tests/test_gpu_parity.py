@@ -191,6 +191,16 @@ def test_data_errors_never_trap(torch, kernel, full):
     assert word & A.DATA_BAD_PROB and word & A.DATA_BAD_UNIFORM
 
 
+@pytest.mark.parametrize("cluster", [1, 2, 4])
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+def test_ring_kernel_small_clusters(torch, cluster, mode):
+    # the ring kernel keeps no slice in shared memory: clusters of 1 to 4 give
+    # slices of up to 32 rounds (256 inverse-CDF groups per CTA)
+    for B, K, V in ((3, 2, 40000), (2, 3, min(128256, 65536 * cluster))):  # up to 32 rounds
+        batch = small(B, K, V, synth.BF16, 31 + cluster)
+        check(batch, torch, mode, RING, False, cluster_size=cluster)
+
+
 @pytest.mark.parametrize("kernel", [GENERIC, TMA, STREAM, RING])
 def test_exact_ties_resolve_to_lowest_index(torch, kernel):
     B, K, V = 2, 2, 4096
