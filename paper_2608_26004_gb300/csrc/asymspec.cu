@@ -271,10 +271,11 @@ using KernelFn = const void*;  // a __global__ function taking KParams (or SPara
 
 KernelFn pick_ring(int dtype, bool stoch);
 
-KernelFn pick_kernel(const Plan& pl, int dtype, bool stoch) {
+// sel: the TMA kernel's program set (tma_program_set; 0 = run-time dispatch)
+KernelFn pick_kernel(const Plan& pl, int dtype, bool stoch, int sel = 0) {
   if (pl.kernel == ASYMSPEC_KERNEL_RING) return pick_ring(dtype, stoch);
   if (pl.kernel == ASYMSPEC_KERNEL_TMA)
-    return dtype == ASYMSPEC_FP32 ? tma_kernel_f32(stoch) : tma_kernel_bf16(stoch);
+    return dtype == ASYMSPEC_FP32 ? tma_kernel_f32(stoch, sel) : tma_kernel_bf16(stoch, sel);
   return generic_kernel(dtype, pl.vector_path, stoch);
 }
 
@@ -560,7 +561,10 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
   out->kernel = pl.kernel;
   int device = 0;
   if (cudaGetDevice(&device) == cudaSuccess) {
-    KernelFn fn = pick_kernel(pl, dtype, gp.mode == ASYMSPEC_MODE_STOCHASTIC);
+    const bool st_mode = gp.mode == ASYMSPEC_MODE_STOCHASTIC;
+    KernelFn fn = pick_kernel(pl, dtype, st_mode,
+                              tma_program_set(st_mode, gp.divergence, gp.fuse_bonus != 0, false,
+                                              false));
     int ncl = 0;
     if (prepare_kernel(fn, device) == cudaSuccess &&
         active_clusters(fn, pl, device, &ncl) == cudaSuccess)
@@ -704,7 +708,9 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
     if (e != cudaSuccess) return cuda_fail(e);
     return ASYMSPEC_OK;
   }
-  KernelFn fn = pick_kernel(pl, dtype, stoch);
+  KernelFn fn = pick_kernel(pl, dtype, stoch,
+                            tma_program_set(stoch, gp.divergence, gp.fuse_bonus != 0, P.full != 0,
+                                            P.want_tokens != 0));
   e = prepare_kernel(fn, device);
   if (e != cudaSuccess) return cuda_fail(e);
   // The one-shot kernels launch one cluster per row; the persistent ring

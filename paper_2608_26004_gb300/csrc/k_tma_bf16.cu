@@ -4,9 +4,10 @@
 
 namespace asymspec_impl {
 
-const void* tma_kernel_bf16(bool stoch) {
-  return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, true>)
-               : reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, false>);
+// Program set 0 (run-time dispatch); the production sets are in k_tma_bf16_prod.cu.
+const void* tma_kernel_bf16_any(bool stoch) {
+  return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, true, 0>)
+               : reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, false, 0>);
 }
 
 const void* decide_kernel_bf16(bool stoch) {

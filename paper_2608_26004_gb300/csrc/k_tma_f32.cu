@@ -4,9 +4,10 @@
 
 namespace asymspec_impl {
 
-const void* tma_kernel_f32(bool stoch) {
-  return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<float, true>)
-               : reinterpret_cast<const void*>(&fuse_verify_tma<float, false>);
+// Program set 0 (run-time dispatch); the production sets are in k_tma_f32_prod.cu.
+const void* tma_kernel_f32_any(bool stoch) {
+  return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<float, true, 0>)
+               : reinterpret_cast<const void*>(&fuse_verify_tma<float, false, 0>);
 }
 
 const void* decide_kernel_f32(bool stoch) {

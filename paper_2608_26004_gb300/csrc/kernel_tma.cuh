@@ -1081,7 +1081,24 @@ __device__ __forceinline__ void run_full(const KParams& P, const RowCtx& c,
   }
 }
 
-template <typename T, bool STOCH>
+// Program sets.  SEL 0 chooses among every row program at run time (debug
+// outputs, per-row tokens, any gate).  SEL > 0 compiles only the two
+// programs of one production configuration (draft rows, bonus row), which
+// keeps the instruction footprint of the two CTAs an SM runs small:
+//   stochastic  SEL = 1 + d
+//   greedy      SEL = 1 + d + 3 fuse_bonus
+// with d = 0 for the JSD gate, 1 for KL, 2 for none or lambda.
+constexpr int kTmaProgramSets = 7;
+
+__host__ __device__ constexpr int tma_program_set(bool stoch, int divergence, bool fuse_bonus,
+                                                  bool full, bool want_tokens) {
+  return (full || (stoch && want_tokens))
+             ? 0
+             : 1 + (divergence == ASYMSPEC_DIV_JSD ? 0 : divergence == ASYMSPEC_DIV_KL ? 1 : 2) +
+                   ((!stoch && fuse_bonus) ? 3 : 0);
+}
+
+template <typename T, bool STOCH, int SEL>
 __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   extern __shared__ __align__(128) unsigned char smem_tma[];
@@ -1142,7 +1159,26 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   }
   __syncthreads();  // the chunk barriers are initialised
 
-  if (P.full) {
+  if constexpr (SEL > 0 && STOCH) {
+    constexpr int d = SEL - 1;
+    constexpr unsigned GD = d == 0 ? G_JSD : d == 1 ? G_KL : 0u;
+    if (!bonus) run_row<T, STOCH, F_LA | F_LB | F_LS, GD | G_RES, false, true>(P, c, cluster);
+    else run_row<T, STOCH, F_LS, G_QF, false, true>(P, c, cluster);
+  } else if constexpr (SEL > 0) {
+    constexpr int d = (SEL - 1) % 3;
+    constexpr bool fused_bonus = SEL > 3;
+    constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
+    if (bonus) {
+      if (fused_bonus) run_row<T, STOCH, F_AS, 0, false, false>(P, c, cluster);
+      else run_row<T, STOCH, F_AT, 0, false, false>(P, c, cluster);
+    } else if (d == 0) {
+      run_row<T, STOCH, FD, G_JSD, false, true>(P, c, cluster);
+    } else if (d == 1) {
+      run_row<T, STOCH, FD, G_KL, false, true>(P, c, cluster);
+    } else {
+      run_row<T, STOCH, FD, 0, false, false>(P, c, cluster);
+    }
+  } else if (P.full) {
     run_full<T, STOCH, F_LA | F_LB | F_LT | F_LS | F_AS | F_AT, STOCH ? G_RES : 0u>(P, c, cluster);
   } else if (!STOCH) {
     const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;

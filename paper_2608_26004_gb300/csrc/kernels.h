@@ -7,9 +7,13 @@ namespace asymspec_impl {
 
 // fuse_verify_generic<T, VE, STOCH> (k_generic.cu)
 const void* generic_kernel(int dtype, bool vector_path, bool stoch);
-// fuse_verify_tma<T, STOCH> (k_tma_bf16.cu, k_tma_f32.cu)
-const void* tma_kernel_bf16(bool stoch);
-const void* tma_kernel_f32(bool stoch);
+// fuse_verify_tma<T, STOCH, SEL>: program set 0 (k_tma_bf16.cu, k_tma_f32.cu) and the
+// production sets 1..6 (k_tma_bf16_prod.cu, k_tma_f32_prod.cu); tma_kernel_* falls
+// back to set 0 for any other sel
+const void* tma_kernel_bf16_any(bool stoch);
+const void* tma_kernel_f32_any(bool stoch);
+const void* tma_kernel_bf16(bool stoch, int sel);
+const void* tma_kernel_f32(bool stoch, int sel);
 // fuse_verify_ring<T, STOCH> (k_ring_bf16.cu, k_ring_f32.cu)
 const void* ring_kernel_bf16(bool stoch);
 const void* ring_kernel_f32(bool stoch);

@@ -191,6 +191,29 @@ def test_data_errors_never_trap(torch, kernel, full):
     assert word & A.DATA_BAD_PROB and word & A.DATA_BAD_UNIFORM
 
 
+@pytest.mark.parametrize("div", [A.DIV_JSD, A.DIV_KL, A.DIV_NONE, A.DIV_LAMBDA])
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+@pytest.mark.parametrize("kernel", [AUTO, RING])
+def test_accept_and_next_only(torch, div, mode, kernel):
+    # no per-row outputs: the program sets the benchmark runs (one production
+    # configuration per kernel); accepted length and next token against the
+    # oracle, bit-exact except near-ties the oracle flags
+    for B, K, V, dtype, seed in ((6, 3, 40000, synth.BF16, 41), (4, 2, 8200, synth.FP32, 42)):
+        batch = small(B, K, V, dtype, seed)
+        for fuse_bonus in ((False, True) if mode == GREEDY else (False,)):
+            x = device_inputs(batch, torch)
+            fv = A.FuseVerify(batch.B, batch.K)
+            res = fv(x["a"], x["b"], x["t"], x["tokens"], x["probs"], x["unif"], mode=mode,
+                     divergence=div, fuse_bonus=fuse_bonus, kernel=kernel)
+            torch.cuda.synchronize()
+            L, N = res["accept_len"].cpu().numpy(), res["next_token"].cpu().numpy()
+            o = run_oracle(batch, mode=mode, divergence=div, fuse_bonus=fuse_bonus)
+            ok = ~o.flagged & ~o.error
+            assert np.array_equal(L < 0, o.error) and np.array_equal(N < 0, o.error)
+            assert np.array_equal(L[ok], o.accept_len[ok]) and np.array_equal(N[ok], o.next_token[ok])
+            assert ok.any()
+
+
 @pytest.mark.parametrize("cluster", [1, 2, 4])
 @pytest.mark.parametrize("mode", [GREEDY, STOCH])
 def test_ring_kernel_small_clusters(torch, cluster, mode):
