@@ -167,6 +167,45 @@ __device__ __forceinline__ void warp_reduce_x1(X1& e) {
   e.bad = __reduce_or_sync(0xffffffffu, e.bad);
 }
 
+// Sums of four values over a warp in one transposed butterfly (9 shuffles
+// instead of 20); every lane ends with the four totals.
+__device__ __forceinline__ void warp_sum4(float& v0, float& v1, float& v2, float& v3) {
+  const int lane = threadIdx.x & 31;
+  const bool up16 = (lane & 16) != 0, up8 = (lane & 8) != 0;
+  // lanes 0-15 carry v0, v1 on; lanes 16-31 carry v2, v3
+  const float a = (up16 ? v2 : v0) + __shfl_xor_sync(0xffffffffu, up16 ? v0 : v2, 16);
+  const float b = (up16 ? v3 : v1) + __shfl_xor_sync(0xffffffffu, up16 ? v1 : v3, 16);
+  // lanes with bit 3 clear carry a (v0 or v2) on, the others b (v1 or v3)
+  float c = (up8 ? b : a) + __shfl_xor_sync(0xffffffffu, up8 ? a : b, 8);
+#pragma unroll
+  for (int off = 4; off > 0; off >>= 1) c += __shfl_xor_sync(0xffffffffu, c, off);
+  // lane 0: v0, lane 8: v1, lane 16: v2, lane 24: v3
+  v0 = __shfl_sync(0xffffffffu, c, 0);
+  v1 = __shfl_sync(0xffffffffu, c, 8);
+  v2 = __shfl_sync(0xffffffffu, c, 16);
+  v3 = __shfl_sync(0xffffffffu, c, 24);
+}
+
+// As warp_reduce_x1 for records whose references are already equal across
+// the warp (pass1_fast takes the warp maximum of the first vectors): the
+// sums are added without rescaling.
+template <unsigned F>
+__device__ __forceinline__ void warp_reduce_x1_uniform(X1& e) {
+  constexpr int nsum = ((F & F_LA) != 0) + ((F & F_LB) != 0) + ((F & F_LT) != 0) + ((F & F_LS) != 0);
+  if constexpr (nsum >= 2) {
+    warp_sum4(e.s[0], e.s[1], e.s[2], e.s[3]);
+  } else {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const unsigned bit = q == 0 ? F_LA : q == 1 ? F_LB : q == 2 ? F_LT : F_LS;
+      if (F & bit) e.s[q] = warp_sum(e.s[q]);
+    }
+  }
+  if (F & F_AS) warp_argmax(e.vs, e.is);
+  if (F & F_AT) warp_argmax(e.vt, e.it);
+  e.bad = __reduce_or_sync(0xffffffffu, e.bad);
+}
+
 // Cluster barrier.  Only the warp that pushed records needs release
 // ordering; the others arrive relaxed.  Everyone waits with acquire.
 __device__ __forceinline__ void cluster_barrier(bool released) {
@@ -194,13 +233,28 @@ __device__ __forceinline__ void push_record(const R& rec, R* slots, int rank, in
 
 template <unsigned G>
 __device__ __forceinline__ void warp_reduce_x2(X2& x) {
-  if (G & G_JSD) {
-    x.j = warp_sum(x.j);
-    x.msum = warp_sum(x.msum);
+  constexpr int nsum = ((G & G_JSD) ? 2 : 0) + ((G & G_KL) ? 1 : 0) + ((G & G_RES) ? 2 : 0) +
+                       ((!(G & G_RES) && (G & G_QF)) ? 1 : 0);
+  if constexpr (nsum >= 2 && !((G & G_JSD) && (G & G_KL))) {
+    // the (at most four) sums of the gate in one butterfly
+    float v0 = (G & G_JSD) ? x.j : x.kl, v1 = x.msum, v2 = x.R, v3 = x.Q;
+    warp_sum4(v0, v1, v2, v3);
+    if (G & G_JSD) {
+      x.j = v0;
+      x.msum = v1;
+    }
+    if (G & G_KL) x.kl = v0;
+    if (G & G_RES) x.R = v2;
+    if (G & (G_RES | G_QF)) x.Q = v3;
+  } else {
+    if (G & G_JSD) {
+      x.j = warp_sum(x.j);
+      x.msum = warp_sum(x.msum);
+    }
+    if (G & G_KL) x.kl = warp_sum(x.kl);
+    if (G & G_RES) x.R = warp_sum(x.R);
+    if (G & (G_RES | G_QF)) x.Q = warp_sum(x.Q);
   }
-  if (G & G_KL) x.kl = warp_sum(x.kl);
-  if (G & G_RES) x.R = warp_sum(x.R);
-  if (G & (G_RES | G_QF)) x.Q = warp_sum(x.Q);
 }
 
 // Maximum of the 2*NP values of a vector (NaN ignored / NaN propagated).
@@ -429,9 +483,9 @@ __device__ __forceinline__ void fixed_pairs2(f2& acc, const f2 (&x)[NP], const f
   }
 }
 
-// Pass 1 against fixed references: every thread takes the maximum of its
-// first vector (vector tid, in chunk 0) as the reference of each normaliser
-// stream.  Returns true when one of this thread's sums reached 2^100 or is not
+// Pass 1 against fixed references: each warp takes the largest of its
+// threads' first-vector maxima (vector tid, in chunk 0) as the reference of
+// each normaliser stream.  Returns true when one of this thread's sums reached 2^100 or is not
 // finite (the caller then redoes the slice with pass1_online).  Argmax
 // streams are tracked per vector as in pass1_online.
 template <typename T, unsigned F>
@@ -465,6 +519,12 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
       for (int h = 0; h < NP; ++h) xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
       ref[3] = vmax_pairs(xs);
     }
+  }
+  // one reference per warp: the largest of its threads' first-vector maxima
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const unsigned bit = q == 0 ? F_LA : q == 1 ? F_LB : q == 2 ? F_LT : F_LS;
+    if (F & bit) ref[q] = warp_max(ref[q]);
   }
   f2 nm[4];
 #pragma unroll
@@ -559,7 +619,7 @@ __device__ __forceinline__ void pass1_and_push(const T* ra, const T* rb, const T
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   X1 e = x1_neutral();
   const bool ovf = pass1_fast<T, F>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
-  warp_reduce_x1<F>(e);
+  warp_reduce_x1_uniform<F>(e);  // the warp's references are equal
   if (lane == 0) sh->w1[warp] = e;
   if (__syncthreads_or(ovf)) {
     // an entry far above its thread's reference (or non-finite data): redo
