@@ -353,14 +353,18 @@ def main():
     hN = torch.empty(B, dtype=torch.int32).pin_memory()
     h2d = sum(v.numel() * v.element_size() for v in pin.values())
     d2h = 2 * B * 4
-    x0 = sets[0]
+    # asymspec_fuse_verify_host: the public call with host buffers, its copies
+    # pipelined with the kernels in chunks of batch elements
+    sbytes = A.host_scratch_bytes(B, K, V, A.BF16)
+    scratch = torch.empty(sbytes, dtype=torch.uint8, device=dev)
 
     def e2e_step(i):
-        for key in pin:
-            x0[key].copy_(pin[key], non_blocking=True)
-        step(x0)
-        hL.copy_(L, non_blocking=True)
-        hN.copy_(N, non_blocking=True)
+        st = A.fuse_verify_host(pin["a"].data_ptr(), pin["b"].data_ptr(), pin["t"].data_ptr(),
+                                pin["tok"].data_ptr(), pin["prob"].data_ptr(),
+                                pin["unif"].data_ptr(), B, K, V, A.BF16, gate, hL.data_ptr(),
+                                hN.data_ptr(), scratch.data_ptr(), sbytes, sptr)
+        if st != A.OK:
+            raise A.AsymSpecError(st, "asymspec_fuse_verify_host")
 
     e2e_steps = max(3, min(args.steps, 30))
     ms_e2e = timed(e2e_step, e2e_steps, 3) / e2e_steps

@@ -234,6 +234,46 @@ int asymspec_fuse_verify_static(const void* logits_full, const void* logits_comp
                                 int32_t* out_accept_len, int32_t* out_next_token,
                                 void* stream);
 
+/*
+ * The step from host memory: asymspec_fuse_verify_ex's computation for
+ * callers whose logits are in host memory (no counterpart in the paper: a
+ * deployment variant).  The batch is cut into at most ASYMSPEC_HOST_CHUNKS
+ * chunks of whole batch elements.  Every chunk's inputs are copied host to
+ * device on a copy stream the library keeps per device; the step of chunk c
+ * runs on `stream` as soon as chunk c's copies have landed, while later
+ * chunks are still being copied, and each chunk's two outputs are copied
+ * back on `stream`.
+ *   h_logits_full, h_logits_comp, h_logits_ver: [B, K+1, V] host, dtype `dtype`
+ *   h_draft_tokens [B, K] int32, h_draft_probs [B, K] fp32 and
+ *   h_uniforms [B, K+1] fp32: host (probabilities and uniforms may be NULL in
+ *       greedy mode), laid out as for asymspec_fuse_verify
+ *   h_out_accept_len, h_out_next_token: [B] int32 host, written once `stream`
+ *       reaches the end of the call (synchronise on it before reading them)
+ *   d_scratch, scratch_bytes: device memory of at least
+ *       asymspec_host_scratch_bytes(B, K, V, dtype) bytes, 256-byte aligned:
+ *       device copies of the inputs and outputs, then one workspace per
+ *       chunk.  It needs no zeroing (each chunk's tickets are cleared on
+ *       `stream` before its step).
+ * Host buffers should be page-locked (cudaMallocHost or cudaHostRegister)
+ * for the copies to run asynchronously and overlap the kernels; pageable
+ * buffers give the same results with the copies staged by the driver.
+ * Calls that overlap in time must not share a scratch, and calls from
+ * several host threads on one device must be serialised by the caller
+ * (they share the copy stream's events).  Status codes are those of
+ * asymspec_fuse_verify_ex; ASYMSPEC_ERR_WORKSPACE when the scratch is
+ * missing, unaligned or too small.  On a status other than ASYMSPEC_OK
+ * returned after copies were enqueued, the call waits for the copy stream
+ * before returning.
+ */
+#define ASYMSPEC_HOST_CHUNKS 8
+size_t asymspec_host_scratch_bytes(int B, int K, int V, int dtype);
+int asymspec_fuse_verify_host(const void* h_logits_full, const void* h_logits_comp,
+                              const void* h_logits_ver, const int32_t* h_draft_tokens,
+                              const float* h_draft_probs, const float* h_uniforms, int B, int K,
+                              int V, int dtype, const asymspec_gate_params* gate_params,
+                              int32_t* h_out_accept_len, int32_t* h_out_next_token,
+                              void* d_scratch, size_t scratch_bytes, void* stream);
+
 /* Launch parameters a call with these sizes would use, without launching.
  * Uses the current CUDA device. */
 int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* gate_params,

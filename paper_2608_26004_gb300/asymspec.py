@@ -51,6 +51,8 @@ EXPORTED = (
     "asymspec_fuse_verify",
     "asymspec_fuse_verify_ex",
     "asymspec_fuse_verify_static",
+    "asymspec_host_scratch_bytes",
+    "asymspec_fuse_verify_host",
     "asymspec_plan",
     "asymspec_status_string",
     "asymspec_last_cuda_error",
@@ -124,6 +126,12 @@ def lib():
     L.asymspec_fuse_verify_static.argtypes = [_P, _P, _P, _P, _P, _P, _I, _I, _I, _I,
                                               ctypes.POINTER(GateParams), _P, _P, _P]
     L.asymspec_fuse_verify_static.restype = _I
+    L.asymspec_host_scratch_bytes.argtypes = [_I, _I, _I, _I]
+    L.asymspec_host_scratch_bytes.restype = ctypes.c_size_t
+    L.asymspec_fuse_verify_host.argtypes = [_P, _P, _P, _P, _P, _P, _I, _I, _I, _I,
+                                            ctypes.POINTER(GateParams), _P, _P, _P,
+                                            ctypes.c_size_t, _P]
+    L.asymspec_fuse_verify_host.restype = _I
     L.asymspec_plan.argtypes = [_I, _I, _I, _I, ctypes.POINTER(GateParams),
                                 ctypes.POINTER(LaunchOpts), ctypes.POINTER(LaunchInfo)]
     L.asymspec_plan.restype = _I
@@ -190,6 +198,26 @@ def fuse_verify_static(logits_full, logits_comp, logits_ver, draft_tokens, draft
     return lib().asymspec_fuse_verify_static(logits_full, logits_comp, logits_ver,
                                              draft_tokens, draft_probs, uniforms, B, K, V,
                                              dtype, g, out_accept_len, out_next_token, stream)
+
+
+HOST_CHUNKS = 8  # chunks of batch elements asymspec_fuse_verify_host pipelines
+
+
+def host_scratch_bytes(B, K, V, dtype) -> int:
+    return lib().asymspec_host_scratch_bytes(B, K, V, dtype)
+
+
+def fuse_verify_host(h_logits_full, h_logits_comp, h_logits_ver, h_draft_tokens, h_draft_probs,
+                     h_uniforms, B, K, V, dtype, gate, h_out_accept_len, h_out_next_token,
+                     d_scratch, scratch_bytes, stream=0) -> int:
+    """asymspec_fuse_verify_host with host addresses (ints) for the inputs and
+    outputs and a device scratch address; returns the status.  The outputs
+    are written once `stream` has reached the end of the call."""
+    g = ctypes.byref(gate) if gate is not None else None
+    return lib().asymspec_fuse_verify_host(h_logits_full, h_logits_comp, h_logits_ver,
+                                           h_draft_tokens, h_draft_probs, h_uniforms, B, K, V,
+                                           dtype, g, h_out_accept_len, h_out_next_token,
+                                           d_scratch, scratch_bytes, stream)
 
 
 def plan(B, K, V, dtype, gate=None, opts=None) -> LaunchInfo:

@@ -470,6 +470,71 @@ int static_scratch(void** out) {
   return ASYMSPEC_OK;
 }
 
+// asymspec_fuse_verify_host: the scratch layout (each part 256-byte aligned)
+// and the chunking of the batch.
+struct HostLayout {
+  int P, Bc;  // chunks, batch elements per chunk (the last may have fewer)
+  size_t a, b, t, tok, prob, unif, len, next, ws, ws_each, total;
+};
+
+HostLayout host_layout(int B, int K, int V, int dtype) {
+  HostLayout L;
+  L.Bc = (B + ASYMSPEC_HOST_CHUNKS - 1) / ASYMSPEC_HOST_CHUNKS;
+  L.P = (B + L.Bc - 1) / L.Bc;
+  const size_t R = static_cast<size_t>(B) * (K + 1);
+  const size_t row = static_cast<size_t>(V) * elt_size(dtype);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += round_up(bytes, 256);
+    return o;
+  };
+  L.a = take(R * row);
+  L.b = take(R * row);
+  L.t = take(R * row);
+  L.tok = take(static_cast<size_t>(B) * K * sizeof(int32_t));
+  L.prob = take(static_cast<size_t>(B) * K * sizeof(float));
+  L.unif = take(R * sizeof(float));
+  L.len = take(static_cast<size_t>(B) * sizeof(int32_t));
+  L.next = take(static_cast<size_t>(B) * sizeof(int32_t));
+  L.ws_each = round_up(asymspec_workspace_bytes(L.Bc, K, V), 256);
+  L.ws = take(L.ws_each * L.P);
+  L.total = off;
+  return L;
+}
+
+// Per device: the copy stream and its per-chunk events (created on first use).
+struct HostRes {
+  cudaStream_t copy;
+  cudaEvent_t start;
+  cudaEvent_t chunk[ASYMSPEC_HOST_CHUNKS];
+  bool ready;
+};
+std::mutex g_host_mu;
+HostRes g_host[kMaxDevices] = {};
+
+int host_resources(HostRes** out) {
+  int device = 0;
+  cudaError_t e = cudaGetDevice(&device);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (device < 0 || device >= kMaxDevices) return ASYMSPEC_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_host_mu);
+  HostRes& r = g_host[device];
+  if (!r.ready) {
+    e = cudaStreamCreateWithFlags(&r.copy, cudaStreamNonBlocking);
+    if (e != cudaSuccess) return cuda_fail(e);
+    e = cudaEventCreateWithFlags(&r.start, cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(e);
+    for (int c = 0; c < ASYMSPEC_HOST_CHUNKS; ++c) {
+      e = cudaEventCreateWithFlags(&r.chunk[c], cudaEventDisableTiming);
+      if (e != cudaSuccess) return cuda_fail(e);
+    }
+    r.ready = true;
+  }
+  *out = &r;
+  return ASYMSPEC_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -794,6 +859,103 @@ int asymspec_fuse_verify_static(const void* logits_full, const void* logits_comp
                                  draft_probs, uniforms, B, K, V, dtype, gate_params,
                                  out_accept_len, out_next_token, scratch, kStaticScratchBytes,
                                  nullptr, nullptr, nullptr, nullptr, nullptr, stream);
+}
+
+size_t asymspec_host_scratch_bytes(int B, int K, int V, int dtype) {
+  if (B < 1 || K < 1 || V < 2) return 0;
+  if (dtype != ASYMSPEC_FP32 && dtype != ASYMSPEC_BF16) return 0;
+  return host_layout(B, K, V, dtype).total;
+}
+
+int asymspec_fuse_verify_host(const void* h_logits_full, const void* h_logits_comp,
+                              const void* h_logits_ver, const int32_t* h_draft_tokens,
+                              const float* h_draft_probs, const float* h_uniforms, int B, int K,
+                              int V, int dtype, const asymspec_gate_params* gate_params,
+                              int32_t* h_out_accept_len, int32_t* h_out_next_token,
+                              void* d_scratch, size_t scratch_bytes, void* stream) {
+  if (B < 1 || K < 1 || V < 2) return ASYMSPEC_ERR_INVALID_ARG;
+  if (dtype != ASYMSPEC_FP32 && dtype != ASYMSPEC_BF16) return ASYMSPEC_ERR_UNSUPPORTED;
+  asymspec_gate_params gp;
+  asymspec_default_gate_params(&gp);
+  if (gate_params) gp = *gate_params;
+  int st = check_params(&gp);
+  if (st) return st;
+  const bool stoch = gp.mode == ASYMSPEC_MODE_STOCHASTIC;
+  if (!h_logits_full || !h_logits_comp || !h_logits_ver || !h_draft_tokens ||
+      !h_out_accept_len || !h_out_next_token)
+    return ASYMSPEC_ERR_INVALID_ARG;
+  if (stoch && (!h_draft_probs || !h_uniforms)) return ASYMSPEC_ERR_INVALID_ARG;
+  const HostLayout L = host_layout(B, K, V, dtype);
+  if (!d_scratch || !aligned(d_scratch, 256) || scratch_bytes < L.total)
+    return ASYMSPEC_ERR_WORKSPACE;
+  HostRes* r = nullptr;
+  st = host_resources(&r);
+  if (st) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* base = static_cast<char*>(d_scratch);
+  const size_t row = static_cast<size_t>(V) * elt_size(dtype);
+  const int K1 = K + 1;
+  // the copies start after everything already on `stream` (which may still
+  // read this scratch), then run back to back on the copy stream
+  cudaError_t e = cudaEventRecord(r->start, s);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(r->copy, r->start, 0);
+  if (e != cudaSuccess) return cuda_fail(e);
+  auto h2d = [&](size_t dst, const void* src, size_t off, size_t bytes) {
+    return cudaMemcpyAsync(base + dst + off, static_cast<const char*>(src) + off, bytes,
+                           cudaMemcpyHostToDevice, r->copy);
+  };
+  for (int c = 0; c < L.P && e == cudaSuccess; ++c) {
+    const int b0 = c * L.Bc, nb = std::min(L.Bc, B - b0);
+    const size_t r0 = static_cast<size_t>(b0) * K1, nr = static_cast<size_t>(nb) * K1;
+    e = h2d(L.a, h_logits_full, r0 * row, nr * row);
+    if (e == cudaSuccess) e = h2d(L.b, h_logits_comp, r0 * row, nr * row);
+    if (e == cudaSuccess) e = h2d(L.t, h_logits_ver, r0 * row, nr * row);
+    if (e == cudaSuccess)
+      e = h2d(L.tok, h_draft_tokens, static_cast<size_t>(b0) * K * 4, static_cast<size_t>(nb) * K * 4);
+    if (stoch && e == cudaSuccess)
+      e = h2d(L.prob, h_draft_probs, static_cast<size_t>(b0) * K * 4, static_cast<size_t>(nb) * K * 4);
+    if (stoch && e == cudaSuccess) e = h2d(L.unif, h_uniforms, r0 * 4, nr * 4);
+    if (e == cudaSuccess) e = cudaEventRecord(r->chunk[c], r->copy);
+  }
+  if (e != cudaSuccess) {
+    cudaStreamSynchronize(r->copy);
+    return cuda_fail(e);
+  }
+  // each chunk's step on `stream` once its copies have landed
+  for (int c = 0; c < L.P; ++c) {
+    const int b0 = c * L.Bc, nb = std::min(L.Bc, B - b0);
+    const size_t r0 = static_cast<size_t>(b0) * K1;
+    char* ws = base + L.ws + static_cast<size_t>(c) * L.ws_each;
+    e = cudaStreamWaitEvent(s, r->chunk[c], 0);
+    if (e == cudaSuccess)
+      e = cudaMemsetAsync(ws + ws_records_bytes(nb, K), 0, static_cast<size_t>(nb) * sizeof(unsigned), s);
+    if (e != cudaSuccess) {
+      cudaStreamSynchronize(r->copy);
+      return cuda_fail(e);
+    }
+    int32_t* d_len = reinterpret_cast<int32_t*>(base + L.len) + b0;
+    int32_t* d_next = reinterpret_cast<int32_t*>(base + L.next) + b0;
+    st = asymspec_fuse_verify_ex(
+        base + L.a + r0 * row, base + L.b + r0 * row, base + L.t + r0 * row,
+        reinterpret_cast<const int32_t*>(base + L.tok) + static_cast<size_t>(b0) * K,
+        stoch ? reinterpret_cast<const float*>(base + L.prob) + static_cast<size_t>(b0) * K : nullptr,
+        stoch ? reinterpret_cast<const float*>(base + L.unif) + r0 : nullptr, nb, K, V, dtype, &gp,
+        d_len, d_next, ws, L.ws_each, nullptr, nullptr, nullptr, nullptr, nullptr, stream);
+    if (st != ASYMSPEC_OK) {
+      cudaStreamSynchronize(r->copy);
+      return st;
+    }
+    e = cudaMemcpyAsync(h_out_accept_len + b0, d_len, static_cast<size_t>(nb) * 4,
+                        cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(h_out_next_token + b0, d_next, static_cast<size_t>(nb) * 4,
+                          cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) {
+      cudaStreamSynchronize(r->copy);
+      return cuda_fail(e);
+    }
+  }
+  return ASYMSPEC_OK;
 }
 
 const char* asymspec_status_string(int status) {

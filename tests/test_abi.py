@@ -125,6 +125,38 @@ def test_host_validation_codes(lib):
     assert st == A.ERR_WORKSPACE
 
 
+def test_host_entry_point_scratch_layout_and_validation(lib):
+    # the device copies of the inputs and outputs, then one workspace per chunk of
+    # ceil(B / 8) batch elements, each part 256-byte aligned
+    for B, K, V, dtype, elt in ((64, 7, 128256, A.BF16, 2), (13, 3, 4099, A.FP32, 4),
+                                (1, 1, 2, A.FP32, 4)):
+        R = B * (K + 1)
+        Bc = -(-B // A.HOST_CHUNKS)
+        P = -(-B // Bc)
+        want = (3 * _up(R * V * elt) + 2 * _up(B * K * 4) + _up(R * 4) + 2 * _up(B * 4)
+                + _up(_up(A.workspace_bytes(Bc, K, V)) * P))
+        assert A.host_scratch_bytes(B, K, V, dtype) == want
+    assert A.host_scratch_bytes(0, 7, 10, A.BF16) == 0
+    assert A.host_scratch_bytes(2, 2, 10, 7) == 0
+    # validation before any CUDA call
+    args = (FAKE, FAKE, FAKE, FAKE, FAKE, FAKE)
+    need = A.host_scratch_bytes(2, 2, 64, A.FP32)
+    assert A.fuse_verify_host(*args, 0, 2, 64, A.FP32, None, FAKE, FAKE, FAKE, need) \
+        == A.ERR_INVALID_ARG
+    assert A.fuse_verify_host(*args, 2, 2, 64, 9, None, FAKE, FAKE, FAKE, need) == A.ERR_UNSUPPORTED
+    assert A.fuse_verify_host(*args, 2, 2, 64, A.FP32, None, 0, FAKE, FAKE, need) \
+        == A.ERR_INVALID_ARG
+    stoch = A.gate_params(mode=A.MODE_STOCHASTIC)
+    assert A.fuse_verify_host(FAKE, FAKE, FAKE, FAKE, 0, FAKE, 2, 2, 64, A.FP32, stoch, FAKE,
+                              FAKE, FAKE, need) == A.ERR_INVALID_ARG
+    assert A.fuse_verify_host(*args, 2, 2, 64, A.FP32, None, FAKE, FAKE, 0, need) \
+        == A.ERR_WORKSPACE
+    assert A.fuse_verify_host(*args, 2, 2, 64, A.FP32, None, FAKE, FAKE, FAKE + 16, need) \
+        == A.ERR_WORKSPACE                               # not 256-byte aligned
+    assert A.fuse_verify_host(*args, 2, 2, 64, A.FP32, None, FAKE, FAKE, FAKE, need - 1) \
+        == A.ERR_WORKSPACE
+
+
 def test_static_entry_point_rejects_batches_above_its_scratch(lib):
     # returns before any CUDA call: B*(K+1) above the static scratch's rows
     args = (FAKE, FAKE, FAKE, FAKE, FAKE, FAKE)
