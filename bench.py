@@ -278,13 +278,23 @@ def main():
     sptr = stream.cuda_stream
     info = A.plan(B, K, V, A.BF16, gate)
 
-    def step(x):
+    def step(x, opts=None):
         st = A.fuse_verify_ex(x["a"].data_ptr(), x["b"].data_ptr(), x["t"].data_ptr(),
                               x["tok"].data_ptr(), x["prob"].data_ptr(), x["unif"].data_ptr(),
                               B, K, V, A.BF16, gate, L.data_ptr(), N.data_ptr(), ws.data_ptr(),
-                              nbytes, stream=sptr)
+                              nbytes, opts=opts, stream=sptr)
         if st != A.OK:
             raise A.AsymSpecError(st, "asymspec_fuse_verify_ex")
+
+    # events the library records around the fused row kernel of every timed
+    # step (asymspec_launch_opts.timing_begin / timing_end), on its stream
+    kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    for b, e in kev:  # torch creates an event at its first record: before taking handles
+        b.record(stream)
+        e.record(stream)
+    kopts = [A.LaunchOpts(0, 0, 0, 0, b.cuda_event, e.cuda_event) for b, e in kev]
+    assert all(o.timing_begin and o.timing_end for o in kopts)
 
     def timed(fn, steps, warmup):
         for i in range(warmup):
@@ -313,13 +323,19 @@ def main():
     # ---- device-resident throughput (the headline value)
     with ClockSampler(local) as clk:
         ms = timed(lambda i: step(sets[i % 2]), args.steps, max(args.warmup, 3))
+        # the same K steps again with the library's events around the fused row
+        # kernel (kept out of the headline loop: two records add ~3 us a step)
+        timed(lambda i: step(sets[i % 2], kopts[i] if i < args.steps else None),
+              args.steps, max(args.warmup, 3))
     clocks = clk.summary()
     ms_step = ms / args.steps
     value = world * rows / (ms_step * 1e-3)
-    # the cluster kernel and its decision kernel: the whole step is charged to
-    # the cluster kernel (its share of the step is in the ncu launch list)
+    # a step is the fused row kernel and its decision kernel; the roofline is
+    # the fused row kernel's own: its mean duration between the events the
+    # library recorded around it in every timed step
     launches_per_step = 2 if info.kernel in (A.KERNEL_TMA, A.KERNEL_RING) else 1
-    launch_s = ms_step * 1e-3
+    kernel_ms = float(np.mean([b.elapsed_time(e) for b, e in kev]))
+    launch_s = kernel_ms * 1e-3
     hbm_peak, peak_kind = peaks()
     achieved = alg_bytes / launch_s / 1e9
 
@@ -386,7 +402,12 @@ def main():
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                      "frac": achieved / hbm_peak, "peak_kind": peak_kind,
                      "traffic": measured_traffic(args.mode),
-                     "algorithmic_bytes_per_launch": alg_bytes},
+                     "algorithmic_bytes_per_launch": alg_bytes,
+                     "kernel": "fuse_verify_tma" if info.kernel == A.KERNEL_TMA else str(info.kernel),
+                     "launch_us": kernel_ms * 1e3,
+                     "timing": "CUDA events the library records around the fused row kernel "
+                               "on its stream, in every step of a second timed loop of the same "
+                               "K steps"},
         "e2e": {"value": e2e_value, "unit": "rows/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e},
         "gpu_launches": launches_per_step * args.steps,

@@ -101,6 +101,13 @@ typedef struct {
   int32_t cluster_size;   /* CTAs per row triple: 1 to 16 */
   int32_t block_threads;  /* reserved, must be 0 (256 threads per CTA) */
   int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC, _TMA, _STREAM or _RING */
+  int32_t pad;            /* reserved, must be 0 */
+  /* Optional cudaEvent_t handles (or NULL): recorded on the call's stream
+   * immediately before and after the launch of the fused row kernel (not
+   * around the decision kernel that follows it), so that a caller can time
+   * that kernel alone with cudaEventElapsedTime.  Both or neither. */
+  void* timing_begin;
+  void* timing_end;
 } asymspec_launch_opts;
 
 /* Kernels (asymspec_launch_opts.kernel, asymspec_launch_info.kernel). */

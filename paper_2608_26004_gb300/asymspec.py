@@ -76,7 +76,8 @@ KERNEL_RING = 4
 
 class LaunchOpts(ctypes.Structure):
     _fields_ = [("cluster_size", ctypes.c_int32), ("block_threads", ctypes.c_int32),
-                ("kernel", ctypes.c_int32)]
+                ("kernel", ctypes.c_int32), ("pad", ctypes.c_int32),
+                ("timing_begin", ctypes.c_void_p), ("timing_end", ctypes.c_void_p)]
 
 
 class LaunchInfo(ctypes.Structure):

@@ -432,8 +432,16 @@ int check_params(const asymspec_gate_params* gp) {
 }
 
 int check_opts(const asymspec_launch_opts* opts) {
-  if (opts && opts->block_threads != 0) return ASYMSPEC_ERR_INVALID_ARG;
+  if (opts && (opts->block_threads != 0 || opts->pad != 0)) return ASYMSPEC_ERR_INVALID_ARG;
+  if (opts && ((opts->timing_begin == nullptr) != (opts->timing_end == nullptr)))
+    return ASYMSPEC_ERR_INVALID_ARG;
   return ASYMSPEC_OK;
+}
+
+// The caller's timing events around the fused row kernel (asymspec_launch_opts).
+cudaError_t record_timing(const asymspec_launch_opts* opts, bool begin, cudaStream_t s) {
+  if (!opts || !opts->timing_begin) return cudaSuccess;
+  return cudaEventRecord(static_cast<cudaEvent_t>(begin ? opts->timing_begin : opts->timing_end), s);
 }
 
 // Scratch of asymspec_fuse_verify_static, used as asymspec_fuse_verify_ex
@@ -769,7 +777,9 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     void* args[] = {&S};
-    e = cudaLaunchKernelExC(&cfg, fn, args);
+    e = record_timing(opts, true, cfg.stream);
+    if (e == cudaSuccess) e = cudaLaunchKernelExC(&cfg, fn, args);
+    if (e == cudaSuccess) e = record_timing(opts, false, cfg.stream);
     if (e != cudaSuccess) return cuda_fail(e);
     return ASYMSPEC_OK;
   }
@@ -799,7 +809,9 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
     P.pass2_rec = reinterpret_cast<float*>(base + L.p2rec);
     P.group_mass = reinterpret_cast<float*>(base + L.groups);
   }
-  e = cudaLaunchKernelExC(&cfg, fn, args);
+  e = record_timing(opts, true, cfg.stream);
+  if (e == cudaSuccess) e = cudaLaunchKernelExC(&cfg, fn, args);
+  if (e == cudaSuccess) e = record_timing(opts, false, cfg.stream);
   if (e != cudaSuccess) return cuda_fail(e);
   if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING) {
     // the rows' decisions and Algorithm 1's scan: one CTA per batch element

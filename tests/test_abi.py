@@ -115,6 +115,12 @@ def test_host_validation_codes(lib):
     st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
                           FAKE, FAKE, 1 << 20, opts=A.LaunchOpts(0, 0, 7))
     assert st == A.ERR_INVALID_ARG                       # unknown kernel
+    half = A.LaunchOpts(0, 0, 0, 0, FAKE, 0)             # one timing event without the other
+    assert A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
+                            FAKE, FAKE, 1 << 20, opts=half) == A.ERR_INVALID_ARG
+    padded = A.LaunchOpts(0, 0, 0, 1)                    # reserved field set
+    assert A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
+                            FAKE, FAKE, 1 << 20, opts=padded) == A.ERR_INVALID_ARG
     small = A.workspace_bytes(2, 2, 250000) - 1          # streaming kernel forced, workspace short
     st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 250000, A.FP32, None, FAKE,
                           FAKE, FAKE, small, opts=A.LaunchOpts(0, 0, A.KERNEL_STREAM))

@@ -289,6 +289,40 @@ def test_workspace_reuse_and_allocating_entry_point(torch):
     assert torch.equal(L2, outs[0][0]) and torch.equal(N2, outs[0][1])
 
 
+def test_timing_events_bracket_the_fused_row_kernel(torch):
+    # the library records the caller's events around the fused row kernel only:
+    # the results are unchanged and the bracketed time is positive and below the step's
+    batch = small(4, 3, 40000, synth.BF16, 81)
+    x = device_inputs(batch, torch)
+    B, K, V = batch.B, batch.K, batch.V
+    L = torch.empty(B, dtype=torch.int32, device="cuda")
+    N = torch.empty_like(L)
+    nbytes = A.workspace_bytes(B, K, V)
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
+    s = torch.cuda.current_stream()
+    gate = A.gate_params(mode=STOCH)
+    outs = []
+    for timed in (False, True):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        for e in ev:
+            e.record(s)
+        opts = A.LaunchOpts(0, 0, 0, 0, ev[1].cuda_event, ev[2].cuda_event) if timed else None
+        assert not timed or (opts.timing_begin and opts.timing_end)
+        ev[0].record(s)
+        st = A.fuse_verify_ex(x["a"].data_ptr(), x["b"].data_ptr(), x["t"].data_ptr(),
+                              x["tokens"].data_ptr(), x["probs"].data_ptr(), x["unif"].data_ptr(),
+                              B, K, V, synth.BF16, gate, L.data_ptr(), N.data_ptr(),
+                              ws.data_ptr(), nbytes, opts=opts, stream=s.cuda_stream)
+        ev[3].record(s)
+        assert st == A.OK
+        torch.cuda.synchronize()
+        outs.append((L.cpu().numpy().copy(), N.cpu().numpy().copy()))
+        if timed:
+            kernel_ms, step_ms = ev[1].elapsed_time(ev[2]), ev[0].elapsed_time(ev[3])
+            assert 0.25 * step_ms < kernel_ms <= step_ms  # a real kernel, not two adjacent records
+    assert np.array_equal(outs[0][0], outs[1][0]) and np.array_equal(outs[0][1], outs[1][1])
+
+
 def test_plan_reports_cluster_occupancy(torch):
     # streaming kernel: a persistent grid of whole SMs' worth of resident CTAs
     info = A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(0, 0, A.KERNEL_STREAM))
