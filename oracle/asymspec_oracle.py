@@ -36,6 +36,11 @@ the paper's position i = k+1; row K is the position after the last draft):
   the JSD (Table "JSD vs KL"), and the tuned-lambda gate
   gamma * exp(-lambda * Delta) with Delta = log softmax(a_i)[d_i] -
   log softmax(b_i)[d_i] evaluated at the draft token (Appendix B).
+* delta sources the paper's mechanism ablation (Section 5, "Mechanism
+  ablation" table) compares with its own a - b: raw-augmented, delta = a (the
+  drafter's full-context logits alone), and SCD-style, delta = t - b (the
+  verifier against the compressed drafter).  Only the fused scores change;
+  the gate and the acceptance test of Eq. 4 keep their own a, b and t.
 
 Near-ties.  Every decision the step takes from floating-point values (an
 acceptance test, an argmax, an inverse-CDF boundary) is also measured here in
@@ -68,6 +73,10 @@ DIV_JSD = 0
 DIV_NONE = 1
 DIV_KL = 2
 DIV_LAMBDA = 3
+
+DELTA_AB = 0   # delta = a - b (Eq. 1, the paper's)
+DELTA_A = 1    # delta = a (raw-augmented, mechanism ablation)
+DELTA_TB = 2   # delta = t - b (SCD-style, mechanism ablation)
 
 FP32 = 0
 BF16 = 1
@@ -172,9 +181,17 @@ class Row:
     gamma_eff: float
 
 
-def row_quantities(a, b, t, gamma, beta, divergence, lam=0.1, draft_token=None) -> Row:
+def row_quantities(a, b, t, gamma, beta, divergence, lam=0.1, draft_token=None,
+                   delta_source=DELTA_AB) -> Row:
     """Eqs. 1-3 for one position (a, b, t are float64 logit rows)."""
-    delta = a - b                                   # Eq. 1
+    if delta_source == DELTA_AB:
+        delta = a - b                               # Eq. 1
+    elif delta_source == DELTA_A:
+        delta = a                                   # raw-augmented (ablation)
+    elif delta_source == DELTA_TB:
+        delta = t - b                               # SCD-style (ablation)
+    else:
+        raise ValueError(f"unknown delta source {delta_source}")
     s = t + beta * delta                            # Eq. 2 (argument of argmax)
     lse_a, lse_b, lse_t, lse_s = logsumexp(a), logsumexp(b), logsumexp(t), logsumexp(s)
     la, lb, lt, lq = a - lse_a, b - lse_b, t - lse_t, s - lse_s
@@ -318,7 +335,7 @@ class Result:
 def fuse_verify(logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=None,
                 uniforms=None, *, dtype=FP32, gamma=0.5, beta=1.0, mode=GREEDY,
                 divergence=DIV_JSD, lam=0.1, fuse_bonus=False,
-                want_logprobs=False) -> Result:
+                want_logprobs=False, delta_source=DELTA_AB) -> Result:
     """Runs the step over a batch.
 
     logits_*: [B, K+1, V] in the stored dtype (float32, or uint16 bf16 bits);
@@ -370,7 +387,8 @@ def fuse_verify(logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=
         rows = []
         for k in range(K1):
             d = int(tokens[bi, k]) if k < K else None
-            r = row_quantities(a_all[k], b_all[k], t_all[k], gamma, beta, divergence, lam, d)
+            r = row_quantities(a_all[k], b_all[k], t_all[k], gamma, beta, divergence, lam, d,
+                               delta_source)
             rows.append(r)
             res.lse[bi, k] = (r.lse_a, r.lse_b, r.lse_t, r.lse_s)
             res.D[bi, k] = r.D

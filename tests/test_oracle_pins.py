@@ -18,12 +18,13 @@ from scipy.stats import chisquare
 import oracle as O
 
 
-def rows_of(a, b, t, gamma=0.5, beta=1.0, div=O.DIV_JSD, lam=0.1, tokens=None):
+def rows_of(a, b, t, gamma=0.5, beta=1.0, div=O.DIV_JSD, lam=0.1, tokens=None,
+            delta=O.DELTA_AB):
     K1 = a.shape[0]
     out = []
     for k in range(K1):
         d = int(tokens[k]) if tokens is not None and k < len(tokens) else None
-        out.append(O.row_quantities(a[k], b[k], t[k], gamma, beta, div, lam, d))
+        out.append(O.row_quantities(a[k], b[k], t[k], gamma, beta, div, lam, d, delta))
     return out
 
 
@@ -152,6 +153,62 @@ def test_zero_delta_or_zero_beta_gives_verifier_distribution(rng):
     b = a + rng.normal(0, 3, (1, V))
     r = rows_of(a, b, t, beta=0.0)[0]
     assert np.allclose(r.lq, sp_log_softmax(t[0]), atol=1e-12, rtol=0)
+
+
+def test_delta_sources_probability_space_routes(rng):
+    # raw-augmented: softmax(t + beta a) is proportional to softmax(t) softmax(a)^beta;
+    # SCD-style: softmax(t + beta (t - b)) to softmax(t)^(1 + beta) / softmax(b)^beta
+    V = 64
+    for beta in (0.0, 0.5, 1.0, 2.0):
+        a, b, t = (rng.normal(0, 2, (1, V)) for _ in range(3))
+        r = rows_of(a, b, t, beta=beta, delta=O.DELTA_A)[0]
+        w = sp_softmax(t[0]) * sp_softmax(a[0]) ** beta
+        assert np.allclose(np.exp(r.lq), w / w.sum(), atol=1e-15, rtol=1e-12)
+        r = rows_of(a, b, t, beta=beta, delta=O.DELTA_TB)[0]
+        w = sp_softmax(t[0]) ** (1.0 + beta) / sp_softmax(b[0]) ** beta
+        assert np.allclose(np.exp(r.lq), w / w.sum(), atol=1e-15, rtol=1e-12)
+
+
+def test_delta_sources_coincide_where_the_definitions_do(rng):
+    B, K, V = 4, 3, 300
+    a, b, t = (rng.normal(0, 2, (B, K + 1, V)).astype(np.float32) for _ in range(3))
+    tokens = rng.integers(0, V, (B, K))
+    # b constant along each row: a - b and a differ by a per-row constant
+    flat = np.broadcast_to(b[..., :1], b.shape).copy()
+    for mode in (O.GREEDY, O.STOCHASTIC):
+        probs = np.full((B, K), 0.3, np.float32)
+        unif = rng.random((B, K + 1)).astype(np.float32)
+        kw = dict(mode=mode, want_logprobs=True, draft_probs=probs, uniforms=unif)
+        r_ab = O.fuse_verify(a, flat, t, tokens, delta_source=O.DELTA_AB, **kw)
+        r_a = O.fuse_verify(a, flat, t, tokens, delta_source=O.DELTA_A, **kw)
+        assert np.allclose(r_ab.logprobs, r_a.logprobs, atol=1e-12, rtol=0)
+        assert np.array_equal(r_ab.accept_len, r_a.accept_len)
+        assert np.array_equal(r_ab.next_token, r_a.next_token)
+        # a == t: a - b and t - b are the same signal
+        r_ab = O.fuse_verify(t, b, t, tokens, delta_source=O.DELTA_AB, **kw)
+        r_tb = O.fuse_verify(t, b, t, tokens, delta_source=O.DELTA_TB, **kw)
+        assert np.array_equal(r_ab.logprobs, r_tb.logprobs)
+        assert np.array_equal(r_ab.next_token, r_tb.next_token)
+
+
+def test_delta_source_leaves_the_gate_and_greedy_acceptance_alone(rng):
+    # Eq. 4 and Eq. 3 use a, b and t themselves: per-draft decisions, D and
+    # gamma_eff are the same whatever delta fuses the emission; beta = 0
+    # removes delta altogether
+    B, K, V = 6, 3, 200
+    a, b, t = (rng.normal(0, 2, (B, K + 1, V)).astype(np.float32) for _ in range(3))
+    tokens = rng.integers(0, V, (B, K))
+    base = O.fuse_verify(a, b, t, tokens)
+    for src in (O.DELTA_A, O.DELTA_TB):
+        r = O.fuse_verify(a, b, t, tokens, delta_source=src)
+        assert np.array_equal(r.accept, base.accept)
+        assert np.array_equal(r.D, base.D) and np.array_equal(r.gamma_eff, base.gamma_eff)
+        assert np.array_equal(r.accept_len, base.accept_len)
+        z = O.fuse_verify(a, b, t, tokens, delta_source=src, beta=0.0)
+        z0 = O.fuse_verify(a, b, t, tokens, beta=0.0)
+        assert np.array_equal(z.next_token, z0.next_token)
+    with pytest.raises(ValueError):
+        O.row_quantities(a[0, 0], b[0, 0], t[0, 0], 0.5, 1.0, O.DIV_JSD, delta_source=3)
 
 
 def test_row_constant_shifts_change_nothing(rng):
