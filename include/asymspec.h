@@ -93,8 +93,20 @@ typedef struct {
   int32_t mode;        /* asymspec_mode_t */
   int32_t divergence;  /* asymspec_div_t */
   int32_t fuse_bonus;  /* greedy: 0 = bonus emits argmax(t_K) as in Algorithm 1; 1 = argmax(s_K) */
-  int32_t flags;       /* reserved, must be 0 */
+  int32_t flags;       /* bits 0-1: the delta source (ASYMSPEC_DELTA_*); other bits reserved, 0 */
 } asymspec_gate_params;
+
+/* The signal fused into the emission, s = t + beta * delta (Eq. 2), in
+ * gate_params.flags & ASYMSPEC_FLAG_DELTA_MASK: the paper's delta = a - b
+ * (Eq. 1), or one of the alternatives its mechanism ablation compares,
+ * delta = a (raw-augmented) and delta = t - b (SCD-style).  Only the fused
+ * scores change: the gate (Eq. 3) and the acceptance test (Eq. 4) keep their
+ * own a, b and t.  The ring and streaming kernels implement a - b only
+ * (ASYMSPEC_ERR_UNSUPPORTED when forced with another source). */
+#define ASYMSPEC_DELTA_AB 0
+#define ASYMSPEC_DELTA_A 1
+#define ASYMSPEC_DELTA_TB 2
+#define ASYMSPEC_FLAG_DELTA_MASK 3
 
 /* Optional launch overrides (host struct); zero fields mean "automatic". */
 typedef struct {

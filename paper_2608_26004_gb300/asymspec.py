@@ -67,6 +67,10 @@ class GateParams(ctypes.Structure):
                 ("flags", ctypes.c_int32)]
 
 
+DELTA_AB = 0   # delta = a - b (Eq. 1)
+DELTA_A = 1    # delta = a (raw-augmented)
+DELTA_TB = 2   # delta = t - b (SCD-style)
+
 KERNEL_AUTO = 0
 KERNEL_GENERIC = 1
 KERNEL_TMA = 2
@@ -153,8 +157,10 @@ def default_gate_params() -> GateParams:
 
 
 def gate_params(gamma=0.5, beta=1.0, lam=0.1, mode=MODE_GREEDY, divergence=DIV_JSD,
-                fuse_bonus=False) -> GateParams:
-    return GateParams(gamma, beta, lam, mode, divergence, int(bool(fuse_bonus)), 0)
+                fuse_bonus=False, delta_source=DELTA_AB) -> GateParams:
+    """Gate parameters; delta_source goes into the flags (bits 0-1)."""
+    return GateParams(gamma, beta, lam, mode, divergence, int(bool(fuse_bonus)),
+                      int(delta_source))
 
 
 def workspace_bytes(B: int, K: int, V: int) -> int:
@@ -280,7 +286,8 @@ class FuseVerify:
     def __call__(self, logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=None,
                  uniforms=None, *, gamma=0.5, beta=1.0, lam=0.1, mode=MODE_GREEDY,
                  divergence=DIV_JSD, fuse_bonus=False, row_stats=False, row_tokens=False,
-                 fused_logprobs=False, cluster_size=0, kernel=KERNEL_AUTO, out=None):
+                 fused_logprobs=False, cluster_size=0, kernel=KERNEL_AUTO, out=None,
+                 delta_source=DELTA_AB):
         import torch
         B, K1, V = logits_full.shape
         K = K1 - 1
@@ -309,7 +316,7 @@ class FuseVerify:
             res["row_tokens"] = torch.empty(B, K1, 2, dtype=torch.int32, device=dev)
         if fused_logprobs and "fused_logprobs" not in res:
             res["fused_logprobs"] = torch.empty(B, K1, V, dtype=torch.float32, device=dev)
-        gate = gate_params(gamma, beta, lam, mode, divergence, fuse_bonus)
+        gate = gate_params(gamma, beta, lam, mode, divergence, fuse_bonus, delta_source)
         opts = LaunchOpts(cluster_size, 0, kernel) if (cluster_size or kernel) else None
         stream = torch.cuda.current_stream(dev).cuda_stream
         st = fuse_verify_ex(

@@ -17,7 +17,8 @@ INCLUDE = os.path.join(ROOT, "include")
 CSRC = os.path.join(HERE, "csrc")
 # one translation unit per kernel family and dtype, compiled in parallel
 CUDA_SRC = [os.path.join(CSRC, f) for f in (
-    "asymspec.cu", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu", "k_tma_bf16_prod.cu", "k_tma_f32_prod.cu", "k_ring_bf16.cu", "k_ring_f32.cu",
+    "asymspec.cu", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu", "k_tma_bf16_prod.cu", "k_tma_f32_prod.cu",
+    "k_tma_bf16_any_s.cu", "k_tma_f32_any_s.cu", "k_ring_bf16.cu", "k_ring_f32.cu",
     "k_stream_bf16_greedy.cu", "k_stream_bf16_stoch.cu",
     "k_stream_f32_greedy.cu", "k_stream_f32_stoch.cu")]
 CUDA_HEADERS = [os.path.join(CSRC, f) for f in (

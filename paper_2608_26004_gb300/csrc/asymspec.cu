@@ -192,9 +192,10 @@ StreamLayout stream_layout(int B, int K, int V, int elt) {
 constexpr int kMaxStreamTiles = 31;
 
 // debug_out: the call asks for row statistics or fused log-probs, which only
-// the one-shot kernels produce.
+// the one-shot kernels produce; delta_ab: the delta source is a - b, the only
+// one the ring and streaming kernels implement.
 int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_opts* opts,
-              bool vec_ok, size_t ws_bytes, bool debug_out, Plan* pl) {
+              bool vec_ok, size_t ws_bytes, bool debug_out, bool delta_ab, Plan* pl) {
   const int elt = elt_size(dtype);
   const int forced_C = (opts && opts->cluster_size > 0) ? opts->cluster_size : 0;
   const int forced_kernel = opts ? opts->kernel : 0;
@@ -209,7 +210,7 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
   const bool stream_ok = vec_ok && L.NT <= kMaxStreamTiles && ws_bytes >= L.total;
   (void)stream_ok;  // measured slower than the cluster kernel: chosen only on request
   if (forced_kernel == ASYMSPEC_KERNEL_STREAM) {
-    if (!vec_ok) return ASYMSPEC_ERR_UNSUPPORTED;
+    if (!vec_ok || !delta_ab) return ASYMSPEC_ERR_UNSUPPORTED;
     if (L.NT > kMaxStreamTiles) return ASYMSPEC_ERR_TOO_LARGE;
     if (ws_bytes < L.total) return ASYMSPEC_ERR_WORKSPACE;
     pl->kernel = ASYMSPEC_KERNEL_STREAM;
@@ -227,7 +228,7 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
   // distance, and warps wait on warp 0's producer and combine work)
   if (forced_kernel == ASYMSPEC_KERNEL_RING) {
     Plan r = *pl;
-    if (vec_ok && !debug_out && plan_ring(V, elt, forced_C, &r) &&
+    if (vec_ok && !debug_out && delta_ab && plan_ring(V, elt, forced_C, &r) &&
         ws_bytes >= tma_layout(B, K, r.C, r.group_stride).total) {
       *pl = r;
       pl->kernel = ASYMSPEC_KERNEL_RING;
@@ -236,7 +237,7 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
       return ASYMSPEC_OK;
     }
     if (forced_kernel == ASYMSPEC_KERNEL_RING) {
-      if (!vec_ok || debug_out) return ASYMSPEC_ERR_UNSUPPORTED;
+      if (!vec_ok || debug_out || !delta_ab) return ASYMSPEC_ERR_UNSUPPORTED;
       return (r.C > 0 && r.group_stride > 0 &&
               ws_bytes < tma_layout(B, K, r.C, r.group_stride).total)
                  ? ASYMSPEC_ERR_WORKSPACE
@@ -427,7 +428,11 @@ int check_params(const asymspec_gate_params* gp) {
     return ASYMSPEC_ERR_UNSUPPORTED;
   if (gp->divergence == ASYMSPEC_DIV_LAMBDA && !std::isfinite(gp->lambda))
     return ASYMSPEC_ERR_INVALID_ARG;
-  if (gp->flags != 0) return ASYMSPEC_ERR_INVALID_ARG;
+  // flags: bits 0-1 the delta source, every other bit reserved
+  if ((gp->flags & ~ASYMSPEC_FLAG_DELTA_MASK) != 0) return ASYMSPEC_ERR_INVALID_ARG;
+  const int ds = gp->flags & ASYMSPEC_FLAG_DELTA_MASK;
+  if (ds != ASYMSPEC_DELTA_AB && ds != ASYMSPEC_DELTA_A && ds != ASYMSPEC_DELTA_TB)
+    return ASYMSPEC_ERR_INVALID_ARG;
   return ASYMSPEC_OK;
 }
 
@@ -601,7 +606,8 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
   const bool vec_ok = (static_cast<long long>(V) * elt_size(dtype)) % 16 == 0;
   Plan pl = {};
   st = make_plan(B, K, V, dtype, gp.mode == ASYMSPEC_MODE_STOCHASTIC, opts, vec_ok,
-                 asymspec_workspace_bytes(B, K, V), false, &pl);
+                 asymspec_workspace_bytes(B, K, V), false,
+                 (gp.flags & ASYMSPEC_FLAG_DELTA_MASK) == ASYMSPEC_DELTA_AB, &pl);
   if (st) return st;
   if (pl.kernel == ASYMSPEC_KERNEL_STREAM) {
     out->cluster_size = 1;
@@ -637,7 +643,7 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
     const bool st_mode = gp.mode == ASYMSPEC_MODE_STOCHASTIC;
     KernelFn fn = pick_kernel(pl, dtype, st_mode,
                               tma_program_set(st_mode, gp.divergence, gp.fuse_bonus != 0, false,
-                                              false));
+                                              false, gp.flags & ASYMSPEC_FLAG_DELTA_MASK));
     int ncl = 0;
     if (prepare_kernel(fn, device) == cudaSuccess &&
         active_clusters(fn, pl, device, &ncl) == cudaSuccess)
@@ -687,7 +693,8 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
                       aligned(logits_comp, 16) && aligned(logits_ver, 16);
   Plan pl = {};
   st = make_plan(B, K, V, dtype, stoch, opts, vec_ok, workspace_bytes,
-                 out_row_stats || out_fused_logprobs, &pl);
+                 out_row_stats || out_fused_logprobs,
+                 (gp.flags & ASYMSPEC_FLAG_DELTA_MASK) == ASYMSPEC_DELTA_AB, &pl);
   if (st) return st;
 
   KParams P;
@@ -708,6 +715,7 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   P.lambda = gp.lambda;
   P.ln_gamma = logf(gp.gamma);
   P.divergence = gp.divergence;
+  P.delta_src = gp.flags & ASYMSPEC_FLAG_DELTA_MASK;
   P.fuse_bonus = gp.fuse_bonus ? 1 : 0;
   P.need_lse_s = (stoch || out_fused_logprobs || out_row_stats) ? 1 : 0;
   P.need_pass2 = (stoch || out_fused_logprobs || gp.divergence == ASYMSPEC_DIV_JSD ||
@@ -785,7 +793,7 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   }
   KernelFn fn = pick_kernel(pl, dtype, stoch,
                             tma_program_set(stoch, gp.divergence, gp.fuse_bonus != 0, P.full != 0,
-                                            P.want_tokens != 0));
+                                            P.want_tokens != 0, P.delta_src));
   e = prepare_kernel(fn, device);
   if (e != cudaSuccess) return cuda_fail(e);
   // The one-shot kernels launch one cluster per row; the persistent ring

@@ -51,6 +51,14 @@ __device__ __forceinline__ void cp_async_wait_all() {
 __device__ __forceinline__ float to_f32(float x) { return x; }
 __device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
 
+// The fused score t + beta delta of one entry (Eq. 2) for delta source ds
+// (ASYMSPEC_DELTA_*: a - b, a, or t - b).
+__device__ __forceinline__ float fuse1(float beta, float a, float b, float t, int ds) {
+  return ds == ASYMSPEC_DELTA_A    ? fmaf(beta, a, t)
+         : ds == ASYMSPEC_DELTA_TB ? fmaf(beta, t - b, t)
+                                   : fmaf(beta, a - b, t);
+}
+
 // Vector of VE consecutive elements from shared memory, widened to fp32.
 __device__ __forceinline__ void load_vec(const float* p, float (&x)[4]) {
   const float4 v = *reinterpret_cast<const float4*>(p);
@@ -409,6 +417,7 @@ struct KParams {
   int C, W, sh_off;
   float gamma, beta, lambda, ln_gamma;
   int divergence, fuse_bonus;
+  int delta_src;               // ASYMSPEC_DELTA_*: the signal fused into the emission (Eq. 1)
   int need_lse_s, need_pass2;  // generic kernel: compute LSE(s); run pass 2
   int full;                    // streaming kernel: compute every row quantity (debug outputs)
   int want_tokens;             // streaming kernel: also track argmax(s) in stochastic rows
@@ -527,7 +536,10 @@ __device__ int4 row_record(const KParams& P, long long row, int k, const RowResu
         const float pd = sc.dprob, u = sc.u;
         if (!(pd > 0.f && pd <= 1.f)) err |= ASYMSPEC_DATA_BAD_PROB;
         if (!(u >= 0.f && u < 1.f)) err |= ASYMSPEC_DATA_BAD_UNIFORM;
-        const float sd = fmaf(P.beta, ad - bd, td);
+        // the draft token's fused score, for the delta source in use
+        const float sd = P.delta_src == ASYMSPEC_DELTA_A    ? fmaf(P.beta, ad, td)
+                         : P.delta_src == ASYMSPEC_DELTA_TB ? fmaf(P.beta, td - bd, td)
+                                                            : fmaf(P.beta, ad - bd, td);
         const float qd = expf(sd - r.lse_s);
         accept = qd > u * gamma_eff * pd;
         margin = u - (qd / pd) / gamma_eff;

@@ -5,8 +5,9 @@
 namespace asymspec_impl {
 
 // Program set 0 (run-time dispatch); the production sets are in k_tma_bf16_prod.cu.
+// (the stochastic one in k_tma_bf16_any_s.cu, built in parallel)
 const void* tma_kernel_bf16_any(bool stoch) {
-  return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, true, 0>)
+  return stoch ? tma_kernel_bf16_any_stoch()
                : reinterpret_cast<const void*>(&fuse_verify_tma<__nv_bfloat16, false, 0>);
 }
 

@@ -5,8 +5,9 @@
 namespace asymspec_impl {
 
 // Program set 0 (run-time dispatch); the production sets are in k_tma_f32_prod.cu.
+// (the stochastic one in k_tma_f32_any_s.cu, built in parallel)
 const void* tma_kernel_f32_any(bool stoch) {
-  return stoch ? reinterpret_cast<const void*>(&fuse_verify_tma<float, true, 0>)
+  return stoch ? tma_kernel_f32_any_stoch()
                : reinterpret_cast<const void*>(&fuse_verify_tma<float, false, 0>);
 }
 

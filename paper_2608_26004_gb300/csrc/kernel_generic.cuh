@@ -36,8 +36,8 @@ struct SharedGeneric {
 // The residual / fused mass of one element (stochastic mode).  Pass 2 and the
 // inverse-CDF walk both call this, so they see identical values.
 __device__ __forceinline__ float sample_mass(float xa, float xb, float xt, float beta, float A2,
-                                             float S2, bool use_r) {
-  const float xs = fmaf(beta, xa - xb, xt);
+                                             float S2, bool use_r, int ds) {
+  const float xs = fuse1(beta, xa, xb, xt, ds);
   const float qf = ex2(fmaf(xs, kLog2e, -S2));
   if (!use_r) return qf;
   const float p = ex2(fmaf(xa, kLog2e, -A2));
@@ -107,7 +107,7 @@ __global__ void __launch_bounds__(kThreads, 1) fuse_verify_generic(const KParams
     load_vec(sb + i * VE, xb);
     load_vec(st + i * VE, xt);
 #pragma unroll
-    for (int e = 0; e < VE; ++e) xs[e] = fmaf(beta, xa[e] - xb[e], xt[e]);
+    for (int e = 0; e < VE; ++e) xs[e] = fuse1(beta, xa[e], xb[e], xt[e], P.delta_src);
     online_add(r1.m[0], r1.s[0], xa);
     online_add(r1.m[1], r1.s[1], xb);
     const float ct = online_add(r1.m[2], r1.s[2], xt);
@@ -175,12 +175,12 @@ __global__ void __launch_bounds__(kThreads, 1) fuse_verify_generic(const KParams
         }
         if (do_kl) r2.kl += p * (la2 - lb2);
         if (STOCH) {
-          const float xs = fmaf(beta, xa[e] - xb[e], xt[e]);
+          const float xs = fuse1(beta, xa[e], xb[e], xt[e], P.delta_src);
           const float qf = ex2(fmaf(xs, kLog2e, -S2));
           r2.R += fmaxf(qf - p, 0.f);
           r2.Q += qf;
         }
-        if (lp) lp[i * VE + e] = fmaf(beta, xa[e] - xb[e], xt[e]) - lse_s;
+        if (lp) lp[i * VE + e] = fuse1(beta, xa[e], xb[e], xt[e], P.delta_src) - lse_s;
       }
     }
   }
@@ -263,7 +263,7 @@ __global__ void __launch_bounds__(kThreads, 1) fuse_verify_generic(const KParams
       load_vec(st + i * VE, xt);
 #pragma unroll
       for (int e = 0; e < VE; ++e) {
-        const float mm = sample_mass(xa[e], xb[e], xt[e], beta, A2, S2, use_r);
+        const float mm = sample_mass(xa[e], xb[e], xt[e], beta, A2, S2, use_r, P.delta_src);
         tsum += mm;
         if (mm > 0.f) last_pos = i * VE + e;
       }
@@ -292,7 +292,7 @@ __global__ void __launch_bounds__(kThreads, 1) fuse_verify_generic(const KParams
         load_vec(st + i * VE, xt);
 #pragma unroll
         for (int e = 0; e < VE; ++e) {
-          const float mm = sample_mass(xa[e], xb[e], xt[e], beta, A2, S2, use_r);
+          const float mm = sample_mass(xa[e], xb[e], xt[e], beta, A2, S2, use_r, P.delta_src);
           cum += mm;
           if (pick < 0 && cum > tau) pick = i * VE + e;
         }

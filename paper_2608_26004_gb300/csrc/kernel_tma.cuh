@@ -306,16 +306,25 @@ __device__ __forceinline__ int arg_in_vector(const f2 (&x)[NP], float v, int bas
   return idx;
 }
 
+// The fused score s = t + beta delta of a pair (Eq. 2) for delta source DS:
+// a - b (Eq. 1, ASYMSPEC_DELTA_AB), a (raw-augmented) or t - b (SCD-style).
+template <int DS>
+__device__ __forceinline__ f2 fuse2(f2 beta2, f2 a, f2 b, f2 t) {
+  if constexpr (DS == ASYMSPEC_DELTA_A) return fma2(beta2, a, t);
+  else if constexpr (DS == ASYMSPEC_DELTA_TB) return fma2(beta2, sub2(t, b), t);
+  else return fma2(beta2, sub2(a, b), t);
+}
+
 // Residual max(0, q - p) and fused q masses of one vector (stochastic mode);
 // pass 2 and the inverse-CDF walk share this, so they see identical values.
-template <int NP>
+template <int NP, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void vec_masses(const f2 (&xa)[NP], const f2 (&xb)[NP],
                                            const f2 (&xt)[NP], f2 beta2, f2 L2, f2 nA2, f2 nS2,
                                            f2 (&p)[NP], f2 (&qf)[NP], f2 (&r)[NP]) {
 #pragma unroll
   for (int h = 0; h < NP; ++h) {
     p[h] = ex2_2(fma2(xa[h], L2, nA2));
-    const f2 s = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
+    const f2 s = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
     qf[h] = ex2_2(fma2(s, L2, nS2));
     r[h] = relu2(sub2(qf[h], p[h]));
   }
@@ -370,7 +379,7 @@ __device__ __forceinline__ void load_or_fill(const T* p, bool ok, f2 (&x)[NP]) {
 // rounds [c rc, (c+1) rc).  Rounds are taken two at a time.
 // WAIT: the slice is in shared memory behind the chunk barriers of sh (false:
 // it is in global memory and sh is not used).
-template <typename T, unsigned F, bool WAIT = true>
+template <typename T, unsigned F, bool WAIT = true, int DS = ASYMSPEC_DELTA_AB>
 __device__ __noinline__ void pass1_online(const T* ra, const T* rb, const T* rt, int nv, int rounds,
                                       int rc, int lo, float beta, SharedTma* sh, X1& e) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
@@ -411,8 +420,8 @@ __device__ __noinline__ void pass1_online(const T* ra, const T* rb, const T* rt,
       if (needS) {
 #pragma unroll
         for (int h = 0; h < NP; ++h) {
-          xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
-          ys[h] = fma2(beta2, sub2(ya[h], yb[h]), yt[h]);
+          xs[h] = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
+          ys[h] = fuse2<DS>(beta2, ya[h], yb[h], yt[h]);
         }
       }
       if (F & F_LA) online_pairs2(e.ref[0], acc[0], xa, ya, L2);
@@ -457,7 +466,7 @@ __device__ __noinline__ void pass1_online(const T* ra, const T* rb, const T* rt,
     load_pairs(rb + vec_s * VE, xb);
     load_pairs(rt + vec_s * VE, xt);
 #pragma unroll
-    for (int h = 0; h < NP; ++h) xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
+    for (int h = 0; h < NP; ++h) xs[h] = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
     e.is = arg_in_vector(xs, e.vs, lo + vec_s * VE);
   }
   if ((F & F_AT) && vec_t >= 0) {
@@ -488,7 +497,7 @@ __device__ __forceinline__ void fixed_pairs2(f2& acc, const f2 (&x)[NP], const f
 // each normaliser stream.  Returns true when one of this thread's sums reached 2^100 or is not
 // finite (the caller then redoes the slice with pass1_online).  Argmax
 // streams are tracked per vector as in pass1_online.
-template <typename T, unsigned F>
+template <typename T, unsigned F, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt, int nv,
                                            int rounds, int rc, int lo, float beta, SharedTma* sh,
                                            X1& e) {
@@ -516,7 +525,7 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
     if (F & F_LT) ref[2] = vmax_pairs(xt);
     if (F & F_LS) {
 #pragma unroll
-      for (int h = 0; h < NP; ++h) xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
+      for (int h = 0; h < NP; ++h) xs[h] = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
       ref[3] = vmax_pairs(xs);
     }
   }
@@ -560,8 +569,8 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
       if (needS) {
 #pragma unroll
         for (int h = 0; h < NP; ++h) {
-          xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
-          ys[h] = fma2(beta2, sub2(ya[h], yb[h]), yt[h]);
+          xs[h] = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
+          ys[h] = fuse2<DS>(beta2, ya[h], yb[h], yt[h]);
         }
       }
       if (F & F_LA) fixed_pairs2(acc[0], xa, ya, L2, nm[0]);
@@ -597,7 +606,7 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
     load_pairs(rb + vec_s * VE, xb);
     load_pairs(rt + vec_s * VE, xt);
 #pragma unroll
-    for (int h = 0; h < NP; ++h) xs[h] = fma2(beta2, sub2(xa[h], xb[h]), xt[h]);
+    for (int h = 0; h < NP; ++h) xs[h] = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
     e.is = arg_in_vector(xs, e.vs, lo + vec_s * VE);
   }
   if ((F & F_AT) && vec_t >= 0) {
@@ -611,21 +620,21 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
 // Pass 1 and the CTA combine, pushed to every CTA of the cluster, up to and
 // including cluster barrier B1.  dtok: the row's draft token (-1 if none),
 // known to warp 0.
-template <typename T, unsigned F>
+template <typename T, unsigned F, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void pass1_and_push(const T* ra, const T* rb, const T* rt, int nv,
                                                int rounds, int rc, int lo, int n, float beta,
                                                int dtok, SharedTma* sh, int rank, int C,
                                                cg::cluster_group& cluster) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   X1 e = x1_neutral();
-  const bool ovf = pass1_fast<T, F>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
+  const bool ovf = pass1_fast<T, F, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
   warp_reduce_x1_uniform<F>(e);  // the warp's references are equal
   if (lane == 0) sh->w1[warp] = e;
   if (__syncthreads_or(ovf)) {
     // an entry far above its thread's reference (or non-finite data): redo
     // the slice with a running maximum
     e = x1_neutral();
-    pass1_online<T, F>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
+    pass1_online<T, F, true, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
     warp_reduce_x1<F>(e);
     if (lane == 0) sh->w1[warp] = e;
     __syncthreads();
@@ -745,7 +754,7 @@ __device__ __forceinline__ P2Const p2_const(float beta, float A2, float B2, floa
 // Pass 2 on two vectors x, y of a thread (y absent unless has1: filled with
 // -1e30, which contributes nothing); g0, g1 receive their inverse-CDF masses
 // (residual, or fused for G_QF).  LP: fused log-probs go to lpx, lpy.
-template <int NP, unsigned G, bool LP>
+template <int NP, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void p2_pair(const f2 (&xa)[NP], const f2 (&xb)[NP], const f2 (&xt)[NP],
                                         const f2 (&ya)[NP], const f2 (&yb)[NP], const f2 (&yt)[NP],
                                         bool has1, const P2Const& k, P2Acc& acc, float& g0,
@@ -755,8 +764,8 @@ __device__ __forceinline__ void p2_pair(const f2 (&xa)[NP], const f2 (&xb)[NP], 
   f2 px[NP], py[NP];
   if (RES) {
     f2 qx[NP], qy[NP], rx[NP], ry[NP];
-    vec_masses(xa, xb, xt, k.beta2, k.L2, k.nA2, k.nS2, px, qx, rx);
-    vec_masses(ya, yb, yt, k.beta2, k.L2, k.nA2, k.nS2, py, qy, ry);
+    vec_masses<NP, DS>(xa, xb, xt, k.beta2, k.L2, k.nA2, k.nS2, px, qx, rx);
+    vec_masses<NP, DS>(ya, yb, yt, k.beta2, k.L2, k.nA2, k.nS2, py, qy, ry);
 #pragma unroll
     for (int h = 0; h < NP; ++h) acc.Q2 = add2(acc.Q2, add2(qx[h], qy[h]));
     // residual mass of each vector, summed per group for the inverse-CDF walk
@@ -767,8 +776,8 @@ __device__ __forceinline__ void p2_pair(const f2 (&xa)[NP], const f2 (&xb)[NP], 
     f2 qx[NP], qy[NP];
 #pragma unroll
     for (int h = 0; h < NP; ++h) {
-      qx[h] = ex2_2(fma2(fma2(k.beta2, sub2(xa[h], xb[h]), xt[h]), k.L2, k.nS2));
-      qy[h] = ex2_2(fma2(fma2(k.beta2, sub2(ya[h], yb[h]), yt[h]), k.L2, k.nS2));
+      qx[h] = ex2_2(fma2(fuse2<DS>(k.beta2, xa[h], xb[h], xt[h]), k.L2, k.nS2));
+      qy[h] = ex2_2(fma2(fuse2<DS>(k.beta2, ya[h], yb[h], yt[h]), k.L2, k.nS2));
     }
     // fused mass of each vector, summed per group for the inverse-CDF walk
     g0 = vsum(qx);
@@ -791,11 +800,11 @@ __device__ __forceinline__ void p2_pair(const f2 (&xa)[NP], const f2 (&xb)[NP], 
 #pragma unroll
     for (int h = 0; h < NP; ++h) {
       float l0, l1;
-      upk(add2(fma2(k.beta2, sub2(xa[h], xb[h]), xt[h]), k.nl2), l0, l1);
+      upk(add2(fuse2<DS>(k.beta2, xa[h], xb[h], xt[h]), k.nl2), l0, l1);
       lpx[2 * h] = l0;
       lpx[2 * h + 1] = l1;
       if (has1) {
-        upk(add2(fma2(k.beta2, sub2(ya[h], yb[h]), yt[h]), k.nl2), l0, l1);
+        upk(add2(fuse2<DS>(k.beta2, ya[h], yb[h], yt[h]), k.nl2), l0, l1);
         lpy[2 * h] = l0;
         lpy[2 * h + 1] = l1;
       }
@@ -825,7 +834,7 @@ __device__ __forceinline__ void p2_finish(const P2Acc& acc, X2& x) {
 }
 
 // Pass 2 over the slice, two vectors per step.
-template <typename T, unsigned G, bool LP>
+template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int nv, int rounds,
                                       float beta, float A2, float B2, float S2, float lse_s, X2& x,
                                       float* lp, float* grp) {
@@ -849,7 +858,7 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
         load_pairs(rt + i0 * VE, xt);
         load_or_fill(rt + i1 * VE, has1, yt);
       }
-      p2_pair<NP, G, LP>(xa, xb, xt, ya, yb, yt, has1, k, acc, g0, g1,
+      p2_pair<NP, G, LP, DS>(xa, xb, xt, ya, yb, yt, has1, k, acc, g0, g1,
                          LP ? lp + i0 * VE : nullptr, LP ? lp + i1 * VE : nullptr);
     }
     if (G & (G_RES | G_QF)) p2_groups(g0, g1, grp, kr, rounds);
@@ -859,14 +868,14 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
 
 // Pass 2 and the CTA combine; warp 0 stores the CTA's pass-2 record in the
 // workspace (groups: this CTA's group masses there, stored by pass 2).
-template <typename T, unsigned G, bool LP>
+template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void pass2_and_store(const T* ra, const T* rb, const T* rt, int nv,
                                                 int rounds, float beta, float* lp, SharedTma* sh,
                                                 float* rec, float* groups) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
   X2 x = x2_zero();
-  pass2<T, G, LP>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e, lse_s * kLog2e,
+  pass2<T, G, LP, DS>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e, lse_s * kLog2e,
                   lse_s, x, lp, groups);
   warp_reduce_x2<G>(x);
   if (lane == 0) sh->w2[warp] = x;
@@ -891,7 +900,7 @@ __device__ __forceinline__ float divergence_of(const X2& tot) {
 // ---------------------------------------------------------------- inverse-CDF walk
 
 // Masses of vector v of a slice held in global memory, as pass 2 computes them.
-template <typename T>
+template <typename T, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void slice_vector_masses(const T* ga, const T* gb, const T* gt, int v,
                                                     f2 beta2, f2 L2, f2 nA2, f2 nS2,
                                                     f2 (&p)[8 / sizeof(T)],
@@ -903,7 +912,7 @@ __device__ __forceinline__ void slice_vector_masses(const T* ga, const T* gb, co
   load_pairs(ga + v * VE, xa);
   load_pairs(gb + v * VE, xb);
   load_pairs(gt + v * VE, xt);
-  vec_masses(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
+  vec_masses<NP, DS>(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r);
 }
 
 // The inverse-CDF draw inside one slice, by one warp: the smallest slice
@@ -919,7 +928,7 @@ __device__ __forceinline__ void slice_vector_masses(const T* ga, const T* gb, co
 // mass.
 constexpr int kWalkGroupsPerLane = 8;  // slices of up to 256 groups (32 rounds)
 
-template <typename T, bool GM_GLOBAL>
+template <typename T, bool GM_GLOBAL, int DS = ASYMSPEC_DELTA_AB>
 __device__ __noinline__ int group_walk(const T* ga, const T* gb, const T* gt, int nvec, int lo,
                                        int ngroups, float beta, const float* gm, bool stored,
                                        bool use_r, float A2, float S2, float tau) {
@@ -943,7 +952,7 @@ __device__ __noinline__ int group_walk(const T* ga, const T* gb, const T* gt, in
           const int v = 32 * g + u;
           if (v < nvec) {
             f2 p[NP], qf[NP], r[NP];
-            slice_vector_masses(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
+            slice_vector_masses<T, DS>(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
             m += vsum(use_r ? r : qf);
           }
         }
@@ -1003,7 +1012,7 @@ __device__ __noinline__ int group_walk(const T* ga, const T* gb, const T* gt, in
   f2 p[NP], qf[NP], r[NP];
   float mv = 0.f;
   if (v < nvec) {
-    slice_vector_masses(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
+    slice_vector_masses<T, DS>(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
     mv = vsum(use_r ? r : qf);
   }
   float vin = mv;
@@ -1082,7 +1091,8 @@ __device__ __forceinline__ void store_row_stat(const KParams& P, long long row,
 
 // One row with pass-1 program F and pass-2 program G (R2: pass 2 runs; LP:
 // it writes the fused log-probs).
-template <typename T, bool STOCH, unsigned F, unsigned G, bool LP, bool R2>
+template <typename T, bool STOCH, unsigned F, unsigned G, bool LP, bool R2,
+          int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
                                         cg::cluster_group& cluster) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -1091,7 +1101,7 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
   const T* rt = static_cast<const T*>(c.st);
   SharedTma* sh = c.sh;
   const float beta = P.beta;
-  pass1_and_push<T, F>(ra, rb, rt, c.nv, c.rounds, c.rc, c.lo, c.n, beta, c.dtok, sh, c.rank, c.C,
+  pass1_and_push<T, F, DS>(ra, rb, rt, c.nv, c.rounds, c.rc, c.lo, c.n, beta, c.dtok, sh, c.rank, c.C,
                        cluster);
   if constexpr (!R2) {
     // no pass 2: rank 0 leaves the row's pass-1 results for the decision kernel
@@ -1120,29 +1130,71 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
     __syncthreads();
     float* lp = LP ? P.logprobs + static_cast<size_t>(c.row) * P.V + c.lo : nullptr;
     const size_t slot = static_cast<size_t>(c.row) * c.C + c.rank;
-    pass2_and_store<T, G, LP>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh, P.pass2_rec + slot * 8,
+    pass2_and_store<T, G, LP, DS>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh, P.pass2_rec + slot * 8,
                               P.group_mass + slot * P.group_stride);
   }
 }
 
-template <typename T, bool STOCH, unsigned F, unsigned RQ>
+template <typename T, bool STOCH, unsigned F, unsigned RQ, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void run_full(const KParams& P, const RowCtx& c,
                                          cg::cluster_group& cluster) {
   const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
   const bool klg = P.divergence == ASYMSPEC_DIV_KL;
   if (P.logprobs) {
-    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, true, true>(P, c, cluster);
-    else if (klg) run_row<T, STOCH, F, G_KL | RQ, true, true>(P, c, cluster);
-    else run_row<T, STOCH, F, RQ, true, true>(P, c, cluster);
+    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, true, true, DS>(P, c, cluster);
+    else if (klg) run_row<T, STOCH, F, G_KL | RQ, true, true, DS>(P, c, cluster);
+    else run_row<T, STOCH, F, RQ, true, true, DS>(P, c, cluster);
   } else {
-    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, false, true>(P, c, cluster);
-    else if (klg) run_row<T, STOCH, F, G_KL | RQ, false, true>(P, c, cluster);
-    else run_row<T, STOCH, F, RQ, false, true>(P, c, cluster);
+    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, false, true, DS>(P, c, cluster);
+    else if (klg) run_row<T, STOCH, F, G_KL | RQ, false, true, DS>(P, c, cluster);
+    else run_row<T, STOCH, F, RQ, false, true, DS>(P, c, cluster);
   }
 }
 
+// Program set 0: every row program, chosen at run time, for delta source DS.
+template <typename T, bool STOCH, int DS>
+__device__ __forceinline__ void run_any(const KParams& P, const RowCtx& c, bool bonus,
+                                        cg::cluster_group& cluster) {
+  if (P.full) {
+    run_full<T, STOCH, F_LA | F_LB | F_LT | F_LS | F_AS | F_AT, STOCH ? G_RES : 0u, DS>(P, c, cluster);
+  } else if (!STOCH) {
+    const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
+    const bool klg = P.divergence == ASYMSPEC_DIV_KL;
+    constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
+    if (bonus) {
+      if (P.fuse_bonus) run_row<T, STOCH, F_AS, 0, false, false, DS>(P, c, cluster);
+      else run_row<T, STOCH, F_AT, 0, false, false, DS>(P, c, cluster);
+    } else if (jsd) {
+      run_row<T, STOCH, FD, G_JSD, false, true, DS>(P, c, cluster);
+    } else if (klg) {
+      run_row<T, STOCH, FD, G_KL, false, true, DS>(P, c, cluster);
+    } else {
+      run_row<T, STOCH, FD, 0, false, false, DS>(P, c, cluster);
+    }
+  } else if (!bonus) {
+    const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
+    const bool klg = P.divergence == ASYMSPEC_DIV_KL;
+    if (P.want_tokens) {
+      constexpr unsigned FS = F_LA | F_LB | F_LS | F_AS;
+      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS>(P, c, cluster);
+      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS>(P, c, cluster);
+      else run_row<T, STOCH, FS, G_RES, false, true, DS>(P, c, cluster);
+    } else {
+      constexpr unsigned FS = F_LA | F_LB | F_LS;
+      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS>(P, c, cluster);
+      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS>(P, c, cluster);
+      else run_row<T, STOCH, FS, G_RES, false, true, DS>(P, c, cluster);
+    }
+  } else {
+    if (P.want_tokens) run_row<T, STOCH, F_LS | F_AS, G_QF, false, true, DS>(P, c, cluster);
+    else run_row<T, STOCH, F_LS, G_QF, false, true, DS>(P, c, cluster);
+  }
+
+}
+
 // Program sets.  SEL 0 chooses among every row program at run time (debug
-// outputs, per-row tokens, any gate).  SEL > 0 compiles only the two
+// outputs, per-row tokens, any gate, any delta source).  SEL > 0 compiles
+// only the two
 // programs of one production configuration (draft rows, bonus row), which
 // keeps the instruction footprint of the two CTAs an SM runs small:
 //   stochastic  SEL = 1 + d
@@ -1151,8 +1203,8 @@ __device__ __forceinline__ void run_full(const KParams& P, const RowCtx& c,
 constexpr int kTmaProgramSets = 7;
 
 __host__ __device__ constexpr int tma_program_set(bool stoch, int divergence, bool fuse_bonus,
-                                                  bool full, bool want_tokens) {
-  return (full || (stoch && want_tokens))
+                                                  bool full, bool want_tokens, int delta_src) {
+  return (full || (stoch && want_tokens) || delta_src != ASYMSPEC_DELTA_AB)
              ? 0
              : 1 + (divergence == ASYMSPEC_DIV_JSD ? 0 : divergence == ASYMSPEC_DIV_KL ? 1 : 2) +
                    ((!stoch && fuse_bonus) ? 3 : 0);
@@ -1238,39 +1290,12 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
     } else {
       run_row<T, STOCH, FD, 0, false, false>(P, c, cluster);
     }
-  } else if (P.full) {
-    run_full<T, STOCH, F_LA | F_LB | F_LT | F_LS | F_AS | F_AT, STOCH ? G_RES : 0u>(P, c, cluster);
-  } else if (!STOCH) {
-    const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
-    const bool klg = P.divergence == ASYMSPEC_DIV_KL;
-    constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
-    if (bonus) {
-      if (P.fuse_bonus) run_row<T, STOCH, F_AS, 0, false, false>(P, c, cluster);
-      else run_row<T, STOCH, F_AT, 0, false, false>(P, c, cluster);
-    } else if (jsd) {
-      run_row<T, STOCH, FD, G_JSD, false, true>(P, c, cluster);
-    } else if (klg) {
-      run_row<T, STOCH, FD, G_KL, false, true>(P, c, cluster);
-    } else {
-      run_row<T, STOCH, FD, 0, false, false>(P, c, cluster);
-    }
-  } else if (!bonus) {
-    const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
-    const bool klg = P.divergence == ASYMSPEC_DIV_KL;
-    if (P.want_tokens) {
-      constexpr unsigned FS = F_LA | F_LB | F_LS | F_AS;
-      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true>(P, c, cluster);
-      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true>(P, c, cluster);
-      else run_row<T, STOCH, FS, G_RES, false, true>(P, c, cluster);
-    } else {
-      constexpr unsigned FS = F_LA | F_LB | F_LS;
-      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true>(P, c, cluster);
-      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true>(P, c, cluster);
-      else run_row<T, STOCH, FS, G_RES, false, true>(P, c, cluster);
-    }
+  } else if (P.delta_src == ASYMSPEC_DELTA_A) {
+    run_any<T, STOCH, ASYMSPEC_DELTA_A>(P, c, bonus, cluster);
+  } else if (P.delta_src == ASYMSPEC_DELTA_TB) {
+    run_any<T, STOCH, ASYMSPEC_DELTA_TB>(P, c, bonus, cluster);
   } else {
-    if (P.want_tokens) run_row<T, STOCH, F_LS | F_AS, G_QF, false, true>(P, c, cluster);
-    else run_row<T, STOCH, F_LS, G_QF, false, true>(P, c, cluster);
+    run_any<T, STOCH, ASYMSPEC_DELTA_AB>(P, c, bonus, cluster);
   }
 
   // a copy that timed out may still land: wait for it (bounded) before exit
@@ -1353,12 +1378,21 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
         // the bonus row; the other kind (a draft row whose residual is zero)
         // is recomputed exactly as pass 2 computes it
         const bool stored_r = !bonus || P.full;
-        sample = group_walk<T, true>(static_cast<const T*>(P.a) + off,
-                                     static_cast<const T*>(P.b) + off,
-                                     static_cast<const T*>(P.t) + off, nv_o, lo_o, ng_o, P.beta,
-                                     P.group_mass + (row * C + owner) * P.group_stride,
-                                     r_ok == stored_r, r_ok, st.lse[0] * kLog2e,
-                                     st.lse[3] * kLog2e, tau_local);
+        const T* ga = static_cast<const T*>(P.a) + off;
+        const T* gb = static_cast<const T*>(P.b) + off;
+        const T* gt = static_cast<const T*>(P.t) + off;
+        const float* gm = P.group_mass + (row * C + owner) * P.group_stride;
+        const float A2 = st.lse[0] * kLog2e, S2 = st.lse[3] * kLog2e;
+        const bool stored = r_ok == stored_r;
+        if (P.delta_src == ASYMSPEC_DELTA_A)
+          sample = group_walk<T, true, ASYMSPEC_DELTA_A>(ga, gb, gt, nv_o, lo_o, ng_o, P.beta, gm,
+                                                         stored, r_ok, A2, S2, tau_local);
+        else if (P.delta_src == ASYMSPEC_DELTA_TB)
+          sample = group_walk<T, true, ASYMSPEC_DELTA_TB>(ga, gb, gt, nv_o, lo_o, ng_o, P.beta, gm,
+                                                          stored, r_ok, A2, S2, tau_local);
+        else
+          sample = group_walk<T, true>(ga, gb, gt, nv_o, lo_o, ng_o, P.beta, gm, stored, r_ok, A2,
+                                       S2, tau_local);
       }
     }
     const bool has_ab = P.full || !bonus;

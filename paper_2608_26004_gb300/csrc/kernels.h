@@ -12,6 +12,8 @@ const void* generic_kernel(int dtype, bool vector_path, bool stoch);
 // back to set 0 for any other sel
 const void* tma_kernel_bf16_any(bool stoch);
 const void* tma_kernel_f32_any(bool stoch);
+const void* tma_kernel_bf16_any_stoch();  // k_tma_bf16_any_s.cu
+const void* tma_kernel_f32_any_stoch();   // k_tma_f32_any_s.cu
 const void* tma_kernel_bf16(bool stoch, int sel);
 const void* tma_kernel_f32(bool stoch, int sel);
 // fuse_verify_ring<T, STOCH> (k_ring_bf16.cu, k_ring_f32.cu)

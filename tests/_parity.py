@@ -29,7 +29,8 @@ def device_inputs(batch, torch, device="cuda"):
 
 
 def run_gpu(batch, torch, *, mode, divergence=A.DIV_JSD, gamma=0.5, beta=1.0, lam=0.1,
-            fuse_bonus=False, cluster_size=0, logprobs=True, inputs=None, kernel=0, full=True):
+            fuse_bonus=False, cluster_size=0, logprobs=True, inputs=None, kernel=0, full=True,
+            delta_source=A.DELTA_AB):
     """One call of asymspec_fuse_verify_ex through the binding; numpy results.
 
     full=True asks for every debug output (row statistics, fused log-probs),
@@ -44,7 +45,7 @@ def run_gpu(batch, torch, *, mode, divergence=A.DIV_JSD, gamma=0.5, beta=1.0, la
     res = fv(x["a"], x["b"], x["t"], x["tokens"], x["probs"], x["unif"], gamma=gamma, beta=beta,
              lam=lam, mode=mode, divergence=divergence, fuse_bonus=fuse_bonus,
              row_stats=full, row_tokens=True, fused_logprobs=full and logprobs,
-             cluster_size=cluster_size, kernel=kernel)
+             cluster_size=cluster_size, kernel=kernel, delta_source=delta_source)
     torch.cuda.synchronize()
     out = {k: v.cpu().numpy() for k, v in res.items()}
     out["workspace_after"] = fv.workspace.cpu().numpy()
@@ -52,13 +53,13 @@ def run_gpu(batch, torch, *, mode, divergence=A.DIV_JSD, gamma=0.5, beta=1.0, la
 
 
 def run_oracle(batch, *, mode, divergence=A.DIV_JSD, gamma=0.5, beta=1.0, lam=0.1,
-               fuse_bonus=False, logprobs=True, select=None):
+               fuse_bonus=False, logprobs=True, select=None, delta_source=A.DELTA_AB):
     sel = slice(None) if select is None else select
     return O.fuse_verify(batch.logits_full[sel], batch.logits_comp[sel], batch.logits_ver[sel],
                          batch.draft_tokens[sel], batch.draft_probs[sel], batch.uniforms[sel],
                          dtype=batch.dtype, gamma=gamma, beta=beta, mode=mode,
                          divergence=divergence, lam=lam, fuse_bonus=fuse_bonus,
-                         want_logprobs=logprobs)
+                         want_logprobs=logprobs, delta_source=delta_source)
 
 
 def compare(batch, g, o, *, mode, select=None, logprobs=True, check_stats=True):

@@ -107,7 +107,9 @@ def test_host_validation_codes(lib):
     # below even the cluster kernels' records and tickets (2 x 3 rows, 2 tickets)
     assert call(ws_bytes=511) == A.ERR_WORKSPACE
     g = A.GateParams(0.5, 1.0, 0.1, 0, 0, 0, 3)
-    assert call(gate=g) == A.ERR_INVALID_ARG          # reserved flags must be 0
+    assert call(gate=g) == A.ERR_INVALID_ARG          # delta source 3 does not exist
+    g = A.GateParams(0.5, 1.0, 0.1, 0, 0, 0, 4)
+    assert call(gate=g) == A.ERR_INVALID_ARG          # reserved flag bits must be 0
     opts = A.LaunchOpts(17, 0, 0)
     st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
                           FAKE, FAKE, 1 << 20, opts=opts)

@@ -44,7 +44,8 @@ def small(B, K, V, dtype, seed, **kw):
 
 def check(batch, torch, mode, kernel, full, **kw):
     g = run_gpu(batch, torch, mode=mode, kernel=kernel, full=full, **kw)
-    okw = {k: v for k, v in kw.items() if k in ("divergence", "gamma", "beta", "lam", "fuse_bonus")}
+    okw = {k: v for k, v in kw.items()
+           if k in ("divergence", "gamma", "beta", "lam", "fuse_bonus", "delta_source")}
     o = run_oracle(batch, mode=mode, **okw)
     compare(batch, g, o, mode=mode)
     return g, o
@@ -189,6 +190,28 @@ def test_data_errors_never_trap(torch, kernel, full):
     assert list(g["accept_len"])[:2] == [-1, -1] and g["accept_len"][2] >= 0
     word = int(g["error_word"][0])
     assert word & A.DATA_BAD_PROB and word & A.DATA_BAD_UNIFORM
+
+
+@pytest.mark.parametrize("delta", [A.DELTA_A, A.DELTA_TB])
+@pytest.mark.parametrize("mode", [GREEDY, STOCH])
+@pytest.mark.parametrize("kernel,full", [(AUTO, False), (AUTO, True), (GENERIC, True)],
+                         ids=["auto-prod", "auto-full", "generic-full"])
+def test_delta_sources(torch, delta, mode, kernel, full):
+    # the mechanism ablation's alternatives to a - b (raw-augmented a, SCD-style
+    # t - b): every row quantity and decision against the oracle, aligned and
+    # unaligned rows, greedy with and without the fused bonus
+    for B, K, V, dtype, seed in ((3, 3, 40000, synth.BF16, 91), (2, 2, 4099, synth.FP32, 92)):
+        batch = small(B, K, V, dtype, seed)
+        for fuse_bonus in ((False, True) if mode == GREEDY else (False,)):
+            check(batch, torch, mode, kernel, full, delta_source=delta, fuse_bonus=fuse_bonus)
+
+
+def test_delta_sources_rejected_where_not_implemented(torch):
+    batch = small(2, 2, 8200, synth.BF16, 93)
+    for kernel in (RING, STREAM):
+        with pytest.raises(A.AsymSpecError):
+            run_gpu(batch, torch, mode=STOCH, kernel=kernel, full=False,
+                    delta_source=A.DELTA_TB)
 
 
 @pytest.mark.parametrize("div", [A.DIV_JSD, A.DIV_KL, A.DIV_NONE, A.DIV_LAMBDA])
