@@ -417,3 +417,54 @@ def fuse_verify(logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=
         res.accept[bi] = out[3][0]
         res.accept_margin[bi] = out[4][0]
     return res
+
+
+# ----------------------------------------------------------- the drafter's draw
+
+@dataclass
+class DraftResult:
+    tokens: np.ndarray     # [rows] int, -1 on data error
+    probs: np.ndarray      # [rows] softmax(a)[token], NaN on data error
+    flagged: np.ndarray    # [rows] bool: the draw is a near-tie
+    error: np.ndarray      # [rows] bool
+
+
+def draft_sample(logits, uniforms=None, *, dtype=FP32, mode=GREEDY) -> DraftResult:
+    """The augmented drafter's draw at each position (Section 3.2, item 1 of
+    the three forward passes; the drafting line of Algorithm 1): from the
+    drafter's full-context logits a, greedy decoding takes d = argmax a (the
+    lowest index among ties) and sampling takes the inverse CDF of softmax(a)
+    at the position's uniform u (index order, strict >).  Also returns the
+    drafter's probability of its draw, softmax(a)[d], which the stochastic
+    verification divides by.
+
+    logits: [rows, V] in the stored dtype; uniforms: [rows] float32 (sampling
+    only).  A row with a non-finite logit, or (sampling) a uniform outside
+    [0, 1), is a data error.  Near-ties: an argmax whose top-2 gap is below
+    ARGMAX_BAND * max(1, |top|), or an inverse-CDF target within CDF_BAND of
+    a cumulative boundary, is flagged.
+    """
+    rows, V = np.shape(logits)
+    out = DraftResult(tokens=np.full(rows, -1, np.int64), probs=np.full(rows, np.nan),
+                      flagged=np.zeros(rows, bool), error=np.zeros(rows, bool))
+    if mode == STOCHASTIC:
+        unif = np.asarray(uniforms, np.float32).astype(np.float64).reshape(rows)
+    elif mode != GREEDY:
+        raise ValueError(f"unknown mode {mode}")
+    for r in range(rows):
+        a = widen(np.asarray(logits)[r], dtype)
+        if not np.all(np.isfinite(a)) or (mode == STOCHASTIC and not 0.0 <= unif[r] < 1.0):
+            out.error[r] = True
+            continue
+        la = log_softmax(a)
+        if mode == GREEDY:
+            d = argmax_first(a)
+            out.flagged[r] = top2_gap(a) < ARGMAX_BAND * max(1.0, abs(float(a[d])))
+        else:
+            p = np.exp(la)
+            idx, dist = inverse_cdf(p, unif[r])
+            d = int(idx[0])
+            out.flagged[r] = bool(dist[0] < CDF_BAND)
+        out.tokens[r] = d
+        out.probs[r] = float(np.exp(la[d]))
+    return out

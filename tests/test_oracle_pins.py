@@ -430,3 +430,60 @@ def test_data_errors_are_reported_not_raised(rng):
     unif[1, 2] = 1.0
     res = O.fuse_verify(a, b, t, tokens, probs, unif, mode=O.STOCHASTIC)
     assert list(res.error) == [True, True, False, False]
+
+
+# ------------------------------------------------------------ the drafter's draw
+
+def test_draft_sample_greedy_ties_and_probability():
+    # argmax with the lowest index among ties, and the closed-form probability
+    a = np.array([[0.0, 2.0, 2.0, 1.0], [5.0, 5.0, 5.0, 5.0], [-1.0, -3.0, -2.0, -1.0]])
+    r = O.draft_sample(a, mode=O.GREEDY)
+    assert list(r.tokens) == [1, 0, 0]
+    z = np.exp(2.0) * 2 + 1.0 + np.exp(1.0)
+    assert r.probs[0] == pytest.approx(np.exp(2.0) / z, rel=1e-15)
+    assert r.probs[1] == pytest.approx(0.25, rel=1e-15)
+    assert list(r.flagged) == [True, True, True]   # every row here is an exact tie
+
+
+def test_draft_sample_inverse_cdf_boundaries():
+    # softmax = (0.1, 0.2, 0.3, 0.4): cumulative 0.1, 0.3, 0.6, 1.0; the draw is
+    # the smallest index whose cumulative mass exceeds u
+    a = np.log(np.array([[0.1, 0.2, 0.3, 0.4]] * 6))
+    u = np.array([0.0, 0.05, 0.1 + 1e-3, 0.299, 0.6 + 1e-3, 0.999], np.float32)
+    r = O.draft_sample(a, u, mode=O.STOCHASTIC)
+    assert list(r.tokens) == [0, 0, 1, 1, 3, 3]
+    # (the logits are stored as float32, so the probabilities are exact to ~1e-7)
+    assert np.allclose(r.probs, [0.1, 0.1, 0.2, 0.2, 0.4, 0.4], rtol=1e-6, atol=0)
+    assert not r.flagged[[1, 3, 5]].any() and r.flagged[0]   # u = 0 sits on the boundary 0
+
+
+def test_draft_sample_law_chi_square(rng):
+    V, N = 8, 1_000_000
+    a = rng.normal(0, 1, (1, V))
+    p = sp_softmax(a[0])
+    u = rng.random(N).astype(np.float32)
+    # the oracle's rule on one row, vectorised through inverse_cdf's targets
+    idx, _ = O.inverse_cdf(np.exp(O.log_softmax(a[0])), u.astype(np.float64))
+    counts = np.bincount(idx, minlength=V)
+    assert chisquare(counts, N * p).pvalue > 1e-3
+    r = O.draft_sample(np.repeat(a, 100, axis=0), u[:100], mode=O.STOCHASTIC)
+    assert np.array_equal(r.tokens, idx[:100])
+
+
+def test_draft_sample_shift_invariance_and_errors(rng):
+    a = rng.normal(0, 2, (5, 300))
+    u = rng.random(5).astype(np.float32)
+    for mode in (O.GREEDY, O.STOCHASTIC):
+        r0 = O.draft_sample(a, u, mode=mode)
+        r1 = O.draft_sample(a + 7.25, u, mode=mode)
+        assert np.array_equal(r0.tokens, r1.tokens)
+        # the shifted logits are stored as float32 again: equal to its rounding
+        assert np.allclose(r0.probs, r1.probs, rtol=1e-5, atol=0)
+    bad = a.copy()
+    bad[2, 7] = np.nan
+    r = O.draft_sample(bad, u, mode=O.GREEDY)
+    assert list(r.error) == [False, False, True, False, False] and r.tokens[2] == -1
+    ub = u.copy()
+    ub[4] = 1.0
+    r = O.draft_sample(a, ub, mode=O.STOCHASTIC)
+    assert r.error[4] and not r.error[:4].any()
