@@ -293,6 +293,44 @@ int asymspec_fuse_verify_host(const void* h_logits_full, const void* h_logits_co
                               int32_t* h_out_accept_len, int32_t* h_out_next_token,
                               void* d_scratch, size_t scratch_bytes, void* stream);
 
+/* ---- the drafter's draw ---------------------------------------------------
+ * The step upstream of fuse-and-verify (Section 3.2, item 1: the augmented
+ * drafter S run on the full context; the drafting step of Algorithm 1): for
+ * each of `rows` positions, the draft token d drawn from the drafter's
+ * full-context logits a, and the drafter's probability of it, softmax(a)[d]
+ * (the draft_probs that the stochastic acceptance test of Eq. 4 divides by).
+ *   mode ASYMSPEC_MODE_GREEDY:     d = argmax a, the lowest index on ties;
+ *                                  uniforms is not read (may be NULL).
+ *   mode ASYMSPEC_MODE_STOCHASTIC: d = the smallest index whose cumulative
+ *                                  softmax(a) mass, in index order, exceeds
+ *                                  uniforms[r] (inverse CDF); if rounding
+ *                                  leaves no such index, the last index of
+ *                                  positive mass.
+ * Arguments (device pointers, caller-owned, not retained):
+ *   logits      [rows, V] row-major, fp32 or bf16 (dtype), element-aligned;
+ *               16-byte aligned with V * element size a multiple of 16 takes
+ *               the vector path (same results)
+ *   uniforms    [rows] float32, stochastic mode only
+ *   out_tokens  [rows] int32; out_probs [rows] float32
+ *   cluster_size  CTAs that share a row (1, 2, 4 or 8; each reads one
+ *               contiguous slice of it), or 0 for the library's choice: the
+ *               smallest that gives at least 4 CTAs per SM, up to 8, while a
+ *               slice keeps at least 512 vectors.  Results do not depend on it
+ *               beyond fp32 rounding of the sums.
+ * One kernel launch on `stream` (rows x cluster_size CTAs), no workspace,
+ * nothing allocated.  rows = 0 is a no-op.  Host-detectable errors, returned
+ * before anything is enqueued: ASYMSPEC_ERR_INVALID_ARG (a null pointer,
+ * rows < 0, V < 2, a cluster_size other than 0, 1, 2, 4, 8),
+ * ASYMSPEC_ERR_UNSUPPORTED (dtype or mode), ASYMSPEC_ERR_MISALIGNED,
+ * ASYMSPEC_ERR_TOO_LARGE (V > ASYMSPEC_DRAFT_MAX_V or rows above 2^27).  In the data: a row with
+ * a non-finite logit (NaN, +inf or -inf) or, stochastic, a uniform outside
+ * [0, 1) gets token -1 and probability NaN; the other rows are unaffected.
+ */
+#define ASYMSPEC_DRAFT_MAX_V (1 << 20)
+int asymspec_draft_sample(const void* logits, int rows, int V, int dtype, int mode,
+                          const float* uniforms, int32_t* out_tokens, float* out_probs,
+                          int cluster_size, void* stream);
+
 /* Launch parameters a call with these sizes would use, without launching.
  * Uses the current CUDA device. */
 int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* gate_params,

@@ -27,6 +27,7 @@ ERR_SCRATCH_LIMIT = -7
 
 STATIC_MAX_ROWS = 8192  # B*(K+1) limit of fuse_verify_static
 STATIC_SCRATCH_BYTES = 4 << 20  # size of fuse_verify_static's scratch array
+DRAFT_MAX_V = 1 << 20  # largest V draft_sample takes
 
 DATA_BAD_TOKEN = 0x1
 DATA_NONFINITE = 0x2
@@ -53,6 +54,7 @@ EXPORTED = (
     "asymspec_fuse_verify_static",
     "asymspec_host_scratch_bytes",
     "asymspec_fuse_verify_host",
+    "asymspec_draft_sample",
     "asymspec_plan",
     "asymspec_status_string",
     "asymspec_last_cuda_error",
@@ -137,6 +139,8 @@ def lib():
                                             ctypes.POINTER(GateParams), _P, _P, _P,
                                             ctypes.c_size_t, _P]
     L.asymspec_fuse_verify_host.restype = _I
+    L.asymspec_draft_sample.argtypes = [_P, _I, _I, _I, _I, _P, _P, _P, _I, _P]
+    L.asymspec_draft_sample.restype = _I
     L.asymspec_plan.argtypes = [_I, _I, _I, _I, ctypes.POINTER(GateParams),
                                 ctypes.POINTER(LaunchOpts), ctypes.POINTER(LaunchInfo)]
     L.asymspec_plan.restype = _I
@@ -225,6 +229,13 @@ def fuse_verify_host(h_logits_full, h_logits_comp, h_logits_ver, h_draft_tokens,
                                            h_draft_tokens, h_draft_probs, h_uniforms, B, K, V,
                                            dtype, g, h_out_accept_len, h_out_next_token,
                                            d_scratch, scratch_bytes, stream)
+
+
+def draft_sample(logits, rows, V, dtype, mode, uniforms, out_tokens, out_probs, cluster_size=0,
+                 stream=0) -> int:
+    """asymspec_draft_sample with device addresses (ints); returns the status."""
+    return lib().asymspec_draft_sample(logits, rows, V, dtype, mode, uniforms, out_tokens,
+                                       out_probs, cluster_size, stream)
 
 
 def plan(B, K, V, dtype, gate=None, opts=None) -> LaunchInfo:
@@ -330,3 +341,38 @@ class FuseVerify:
         if st != OK:
             raise AsymSpecError(st, "asymspec_fuse_verify_ex")
         return res
+
+
+def draft_tokens(logits, uniforms=None, *, mode=MODE_GREEDY, cluster_size=0, out=None):
+    """The drafter's draw for CUDA tensors: logits [..., V] (float32 or
+    bfloat16, contiguous), uniforms [...] float32 for sampling.  Returns
+    (tokens int32, probs float32) of the leading shape, enqueued on the
+    current stream; ``out`` may pass the two tensors to fill."""
+    import torch
+    if logits.dtype == torch.float32:
+        dtype = FP32
+    elif logits.dtype == torch.bfloat16:
+        dtype = BF16
+    else:
+        raise TypeError("logits must be float32 or bfloat16")
+    if not logits.is_cuda or not logits.is_contiguous():
+        raise ValueError("logits must be a contiguous CUDA tensor")
+    lead, V = tuple(logits.shape[:-1]), int(logits.shape[-1])
+    rows = 1
+    for n in lead:
+        rows *= n
+    if mode == MODE_STOCHASTIC:
+        if uniforms is None or uniforms.dtype != torch.float32 or not uniforms.is_cuda \
+                or not uniforms.is_contiguous() or uniforms.numel() != rows:
+            raise ValueError("sampling takes one contiguous float32 CUDA uniform per row")
+    dev = logits.device
+    tokens, probs = out if out is not None else (
+        torch.empty(lead, dtype=torch.int32, device=dev),
+        torch.empty(lead, dtype=torch.float32, device=dev))
+    stream = torch.cuda.current_stream(dev).cuda_stream
+    st = draft_sample(_ptr(logits), rows, V, dtype, mode,
+                      _ptr(uniforms) if mode == MODE_STOCHASTIC else 0,
+                      _ptr(tokens), _ptr(probs), cluster_size, stream)
+    if st != OK:
+        raise AsymSpecError(st, "asymspec_draft_sample")
+    return tokens, probs

@@ -19,6 +19,7 @@
 #include "device_common.cuh"
 #include "kernel_generic.cuh"
 #include "kernel_ring.cuh"
+#include "kernel_draft.cuh"
 #include "kernel_stream.cuh"
 #include "kernels.h"
 
@@ -78,7 +79,6 @@ bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
   auto fill = [&](int C) {
     const long long per = (static_cast<long long>(V) + C - 1) / C;
     const long long W = round_up_ll(per, VE);
-    const int rounds = static_cast<int>((W / VE + kTThreads - 1) / kTThreads);
     const int shared_bytes = shared_tma_bytes(C);
     const long long sh_off = round_up_ll(3 * W * elt, 128);
     pl->C = C;
@@ -976,6 +976,72 @@ int asymspec_fuse_verify_host(const void* h_logits_full, const void* h_logits_co
     }
   }
   return ASYMSPEC_OK;
+}
+
+int asymspec_draft_sample(const void* logits, int rows, int V, int dtype, int mode,
+                          const float* uniforms, int32_t* out_tokens, float* out_probs,
+                          int cluster_size, void* stream) {
+  if (dtype != ASYMSPEC_FP32 && dtype != ASYMSPEC_BF16) return ASYMSPEC_ERR_UNSUPPORTED;
+  if (mode != ASYMSPEC_MODE_GREEDY && mode != ASYMSPEC_MODE_STOCHASTIC)
+    return ASYMSPEC_ERR_UNSUPPORTED;
+  if (rows < 0 || V < 2) return ASYMSPEC_ERR_INVALID_ARG;
+  if (cluster_size != 0 && cluster_size != 1 && cluster_size != 2 && cluster_size != 4 &&
+      cluster_size != kDMaxCluster)
+    return ASYMSPEC_ERR_INVALID_ARG;
+  if (V > ASYMSPEC_DRAFT_MAX_V || rows > (1 << 27)) return ASYMSPEC_ERR_TOO_LARGE;
+  if (rows == 0) return ASYMSPEC_OK;
+  const bool stoch = mode == ASYMSPEC_MODE_STOCHASTIC;
+  if (!logits || !out_tokens || !out_probs || (stoch && !uniforms)) return ASYMSPEC_ERR_INVALID_ARG;
+  const int elt = elt_size(dtype);
+  if (!aligned(logits, elt) || !aligned(out_tokens, 4) || !aligned(out_probs, 4) ||
+      (stoch && !aligned(uniforms, 4)))
+    return ASYMSPEC_ERR_MISALIGNED;
+  const bool vec = (static_cast<long long>(V) * elt) % 16 == 0 && aligned(logits, 16);
+  const int VE = vec ? 16 / elt : 1;
+  const int nv = V / VE;
+  int C = cluster_size;
+  if (C == 0) {
+    int device = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+    if (e != cudaSuccess) return cuda_fail(e);
+    C = 1;
+    while (C < kDMaxCluster && static_cast<long long>(rows) * C < 4LL * sms &&
+           (nv + 2 * C - 1) / (2 * C) >= 512)
+      C *= 2;
+  }
+  DParams P;
+  P.logits = logits;
+  P.unif = stoch ? uniforms : nullptr;
+  P.tokens = out_tokens;
+  P.probs = out_probs;
+  P.rows = rows;
+  P.V = V;
+  P.nv = nv;
+  P.W = (nv + C - 1) / C;
+  // sampling: one float of group mass per warp and round of a slice
+  const size_t smem =
+      stoch ? static_cast<size_t>((P.W + kDThreads - 1) / kDThreads) * kDWarps * sizeof(float) : 0;
+  const void* fn = draft_kernel_ptr(dtype, vec, stoch);
+  cudaError_t e = cudaSuccess;
+  if (smem > 48 * 1024)
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return cuda_fail(e);
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(static_cast<unsigned>(static_cast<long long>(rows) * C));
+  cfg.blockDim = dim3(kDThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = static_cast<cudaStream_t>(stream);
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  void* args[] = {&P};
+  e = cudaLaunchKernelExC(&cfg, fn, args);
+  return e == cudaSuccess ? ASYMSPEC_OK : cuda_fail(e);
 }
 
 const char* asymspec_status_string(int status) {

@@ -27,5 +27,7 @@ const void* stream_kernel_bf16_greedy();
 const void* stream_kernel_bf16_stoch();
 const void* stream_kernel_f32_greedy();
 const void* stream_kernel_f32_stoch();
+// draft_kernel<T, VE, STOCH>, the drafter's draw (k_draft.cu)
+const void* draft_kernel_ptr(int dtype, bool vector_path, bool stoch);
 
 }  // namespace asymspec_impl

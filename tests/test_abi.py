@@ -176,6 +176,29 @@ def test_static_entry_point_rejects_batches_above_its_scratch(lib):
     assert "8192" in A.status_string(A.ERR_SCRATCH_LIMIT)
 
 
+def test_draft_sample_validation_codes(lib):
+    # every case returns before any CUDA call
+    G, S = A.MODE_GREEDY, A.MODE_STOCHASTIC
+    d = A.draft_sample
+    assert d(FAKE, 4, 64, 7, G, 0, FAKE, FAKE) == A.ERR_UNSUPPORTED        # dtype
+    assert d(FAKE, 4, 64, A.BF16, 2, FAKE, FAKE, FAKE) == A.ERR_UNSUPPORTED  # mode
+    assert d(FAKE, -1, 64, A.BF16, G, 0, FAKE, FAKE) == A.ERR_INVALID_ARG
+    assert d(FAKE, 4, 1, A.BF16, G, 0, FAKE, FAKE) == A.ERR_INVALID_ARG     # V < 2
+    assert d(FAKE, 4, A.DRAFT_MAX_V + 1, A.FP32, G, 0, FAKE, FAKE) == A.ERR_TOO_LARGE
+    assert d(FAKE, (1 << 27) + 1, 64, A.FP32, G, 0, FAKE, FAKE) == A.ERR_TOO_LARGE
+    for c in (-1, 3, 5, 16):
+        assert d(FAKE, 4, 64, A.FP32, G, 0, FAKE, FAKE, c) == A.ERR_INVALID_ARG
+    assert d(0, 0, 64, A.FP32, S, 0, 0, 0) == A.OK                          # no rows: no-op
+    assert d(0, 4, 64, A.FP32, G, 0, FAKE, FAKE) == A.ERR_INVALID_ARG
+    assert d(FAKE, 4, 64, A.FP32, G, 0, 0, FAKE) == A.ERR_INVALID_ARG
+    assert d(FAKE, 4, 64, A.FP32, G, 0, FAKE, 0) == A.ERR_INVALID_ARG
+    assert d(FAKE, 4, 64, A.FP32, S, 0, FAKE, FAKE) == A.ERR_INVALID_ARG     # sampling: uniforms
+    assert d(FAKE + 2, 4, 64, A.FP32, G, 0, FAKE, FAKE) == A.ERR_MISALIGNED
+    assert d(FAKE + 1, 4, 64, A.BF16, G, 0, FAKE, FAKE) == A.ERR_MISALIGNED
+    assert d(FAKE, 4, 64, A.FP32, G, 0, FAKE + 2, FAKE) == A.ERR_MISALIGNED
+    assert d(FAKE, 4, 64, A.FP32, S, FAKE + 1, FAKE, FAKE) == A.ERR_MISALIGNED
+
+
 def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
     # the streaming kernel on request: 16384-entry tiles (bf16), 8192 (fp32)
     STREAM = A.LaunchOpts(0, 0, A.KERNEL_STREAM)
