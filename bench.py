@@ -191,6 +191,70 @@ def oracle_rows_per_s(batch, mode_id, seconds: float):
             return rows / el, rows, el
 
 
+def draft_timing(torch, A, sets, B, K, V, mode, dev, steps):
+    """Per-launch time of asymspec_draft_sample on the workload's drafter rows:
+    launches of B rows (one drafted position of every batch element) and one
+    launch of all B (K+1) rows, each captured K+1 (resp. 1) times per input
+    set into a CUDA graph that is replayed; CUDA events around the replays."""
+    rows_all = B * (K + 1)
+    flat = [x["a"].view(rows_all, V) for x in sets]
+    unif = [x["unif"].view(rows_all) for x in sets]
+    tok = torch.empty(rows_all, dtype=torch.int32, device=dev)
+    prob = torch.empty(rows_all, dtype=torch.float32, device=dev)
+
+    def launches(rows):
+        out = []
+        for f, u in zip(flat, unif):
+            for r0 in range(0, rows_all, rows):
+                out.append((f[r0:r0 + rows], u[r0:r0 + rows]))
+        return out
+
+    def time_graph(items, rows):
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(torch.cuda.current_stream(dev))
+
+        def issue(stream_ptr):
+            for f, u in items:
+                st = A.draft_sample(f.data_ptr(), rows, V, A.BF16, mode, u.data_ptr(),
+                                    tok.data_ptr(), prob.data_ptr(), 0, stream_ptr)
+                if st != A.OK:
+                    raise A.AsymSpecError(st, "asymspec_draft_sample")
+
+        with torch.cuda.stream(side):
+            issue(side.cuda_stream)  # warm-up, outside the graph
+        torch.cuda.synchronize(dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            issue(side.cuda_stream)
+        reps = max(3, min(200, steps))
+        with torch.cuda.stream(side):
+            for _ in range(3):
+                g.replay()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(side)
+            for _ in range(reps):
+                g.replay()
+            e1.record(side)
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) * 1e3 / (reps * len(items))
+
+    hbm_peak, peak_kind = peaks()
+    res = {"mode": "stochastic" if mode == A.MODE_STOCHASTIC else "greedy", "kernel": "draft_kernel",
+           "peak_kind": peak_kind,
+           "algorithmic_bytes": "rows x V x 2 (the bf16 logits, read once) + rows x 12 "
+                                "(uniform in, token and probability out)",
+           "timing": "CUDA graph of the launches over both resident input sets, replayed; "
+                     "CUDA events on the replay stream"}
+    for key, rows in (("per_position", B), ("all_rows", rows_all)):
+        us = time_graph(launches(rows), rows)
+        alg = rows * V * 2 + rows * 12
+        gbs = alg / (us * 1e-6) / 1e9
+        res[key] = {"rows": rows, "us_per_launch": us, "hbm_gbs": gbs, "frac": gbs / hbm_peak,
+                    "rows_per_s": rows / (us * 1e-6)}
+    return res
+
+
 def run_reference(args, workload, rank, world):
     """--impl reference: the float64 CPU oracle, timed on the host cores."""
     from paper_2608_26004_gb300 import synth
@@ -354,6 +418,13 @@ def main():
     ms_o = timed(lambda i: step_o(sets[i % 2]), args.steps, max(args.warmup, 3)) / args.steps
     alg_bytes_o = algorithmic_bytes(B, K, V, 2, other_mode == A.MODE_STOCHASTIC)
 
+    # ---- the drafter's draw (asymspec_draft_sample), the step upstream of
+    # fuse-and-verify: per drafted position one launch over the B rows of the
+    # drafter's full-context logits, and once over all B (K+1) rows.  Timed as
+    # CUDA graph replays (host launch overhead would exceed a 64-row launch);
+    # the launches read the rows of both resident sets in turn (262 MB > L2).
+    draft = draft_timing(torch, A, sets, B, K, V, mode, dev, args.steps)
+
     # ---- end to end through the C ABI with host buffers
     pin = dict(
         a=torch.from_numpy(np.ascontiguousarray(batch.logits_full).view(np.int16)).view(
@@ -412,6 +483,7 @@ def main():
                 "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
+        "draft": draft,
         "other_mode": {"mode": "greedy" if other_mode == A.MODE_GREEDY else "stochastic",
                        "ms_per_step": ms_o, "rows_per_s": world * rows / (ms_o * 1e-3),
                        "hbm_gbs": alg_bytes_o / (ms_o * 1e-3) / 1e9,
