@@ -36,7 +36,9 @@ WORKLOAD_CFG = 2
 FALLBACK_HBM_GBS = 6800.0
 CSRC = os.path.join(ROOT, "paper_2608_26004_gb300", "csrc")
 KERNEL_SRCS = ("asymspec.cu", "device_common.cuh", "kernel_generic.cuh", "kernel_tma.cuh",
-               "kernel_stream.cuh", "kernels.h", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu")
+               "kernel_stream.cuh", "kernels.h", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu",
+               "k_tma_bf16_prod.cu", "k_tma_f32_prod.cu", "k_tma_bf16_any_s.cu",
+               "k_tma_f32_any_s.cu")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fuse_verify_tma_B64_K7_V128256_bf16_traffic.txt")
 REASON_BITS = {
     0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
