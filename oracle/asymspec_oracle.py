@@ -42,6 +42,17 @@ the paper's position i = k+1; row K is the position after the last draft):
   verifier against the compressed drafter).  Only the fused scores change;
   the gate and the acceptance test of Eq. 4 keep their own a, b and t.
 
+* Cross-family vocabularies (Section 4, "Cross-family portability", and the
+  appendix of the same name): drafter and verifier with different
+  vocabularies share S string-identical tokens, the pairs (map_d[j],
+  map_v[j]).  delta is computed in the drafter vocabulary and carried to the
+  verifier token of each pair, and committed tokens are restricted to the
+  shared set.  Read here as: the step above run on the rows restricted to
+  the pairs, a'_j = a[map_d[j]], b'_j = b[map_d[j]], t'_j = t[map_v[j]]
+  (every softmax, the divergence, the acceptance test and the emission
+  renormalised over the shared set, index order = pair order), drafts given
+  as pair indices, and the emitted pair index reported as its verifier token.
+
 Near-ties.  Every decision the step takes from floating-point values (an
 acceptance test, an argmax, an inverse-CDF boundary) is also measured here in
 float64; a decision closer to its boundary than the bands below is "flagged"
@@ -416,6 +427,54 @@ def fuse_verify(logits_full, logits_comp, logits_ver, draft_tokens, draft_probs=
         res.flagged[bi] = out[2][0]
         res.accept[bi] = out[3][0]
         res.accept_margin[bi] = out[4][0]
+    return res
+
+
+# ------------------------------------------------- cross-family vocabularies
+
+def check_vocab_map(map_d, map_v, V_d: int, V_v: int):
+    """The shared-token pairs as int64 arrays; raises ValueError unless they
+    are two 1-D arrays of one length S >= 2, in range, each without repeats."""
+    md = np.asarray(map_d, np.int64)
+    mv = np.asarray(map_v, np.int64)
+    if md.ndim != 1 or mv.shape != md.shape or md.size < 2:
+        raise ValueError("map_d and map_v must be 1-D of one length S >= 2")
+    if md.min() < 0 or md.max() >= V_d or mv.min() < 0 or mv.max() >= V_v:
+        raise ValueError("a map entry lies outside its vocabulary")
+    if np.unique(md).size != md.size or np.unique(mv).size != mv.size:
+        raise ValueError("a vocabulary token appears in two pairs")
+    return md, mv
+
+
+def fuse_verify_xvocab(logits_full, logits_comp, logits_ver, map_d, map_v, draft_index,
+                       draft_probs=None, uniforms=None, **kw) -> Result:
+    """The step for a drafter and a verifier with different vocabularies
+    (Section 4, "Cross-family portability"; appendix "Cross-family
+    portability"): logits_full and logits_comp are [B, K+1, V_d] (drafter
+    vocabulary), logits_ver [B, K+1, V_v] (verifier vocabulary), the S pairs
+    (map_d[j], map_v[j]) the string-identical tokens, draft_index [B, K] pair
+    indices in [0, S).  The rows are restricted to the pairs and the step runs
+    on them unchanged; the emitted pair index j is committed as the verifier
+    token map_v[j].  Returns fuse_verify's Result with next_token, candidate
+    and fused_argmax as verifier tokens, the pair index of the next token in
+    an extra field next_index, and logprobs (if asked for) over the pairs.
+    """
+    V_d = np.shape(logits_full)[-1]
+    V_v = np.shape(logits_ver)[-1]
+    md, mv = check_vocab_map(map_d, map_v, V_d, V_v)
+    a = np.asarray(logits_full)[..., md]
+    b = np.asarray(logits_comp)[..., md]
+    t = np.asarray(logits_ver)[..., mv]
+    res = fuse_verify(a, b, t, draft_index, draft_probs, uniforms, **kw)
+
+    def to_verifier(j):
+        j = np.asarray(j)
+        return np.where(j >= 0, mv[np.maximum(j, 0)], -1)
+
+    res.next_index = res.next_token.copy()
+    res.next_token = to_verifier(res.next_token)
+    res.candidate = to_verifier(res.candidate)
+    res.fused_argmax = to_verifier(res.fused_argmax)
     return res
 
 

@@ -487,3 +487,125 @@ def test_draft_sample_shift_invariance_and_errors(rng):
     ub[4] = 1.0
     r = O.draft_sample(a, ub, mode=O.STOCHASTIC)
     assert r.error[4] and not r.error[:4].any()
+
+
+# ------------------------------------------------- cross-family vocabularies
+
+def _xcase(rng, B, K, V_d, V_v, S, scale=2.0):
+    a = rng.normal(0, scale, (B, K + 1, V_d)).astype(np.float32)
+    b = (a + rng.normal(0, 1.0, a.shape)).astype(np.float32)
+    t = rng.normal(0, scale, (B, K + 1, V_v)).astype(np.float32)
+    md = rng.choice(V_d, S, replace=False)
+    mv = rng.choice(V_v, S, replace=False)
+    draft = rng.integers(0, S, (B, K))
+    probs = rng.uniform(0.05, 1.0, (B, K)).astype(np.float32)
+    unif = rng.random((B, K + 1)).astype(np.float32)
+    return a, b, t, md, mv, draft, probs, unif
+
+
+def _same(r0, r1, next_map=None):
+    assert np.array_equal(r0.accept_len, r1.accept_len)
+    nt = r0.next_token if next_map is None else np.where(r0.next_token >= 0,
+                                                          next_map[np.maximum(r0.next_token, 0)], -1)
+    assert np.array_equal(nt, r1.next_token)
+    assert np.array_equal(r0.flagged, r1.flagged) and np.array_equal(r0.error, r1.error)
+    np.testing.assert_allclose(r0.D, r1.D, rtol=1e-12, atol=1e-15)
+
+
+@pytest.mark.parametrize("mode", [O.GREEDY, O.STOCHASTIC])
+def test_xvocab_identity_map_is_the_plain_step(rng, mode):
+    # one shared vocabulary, every token paired with itself
+    a, b, t, _, _, draft, probs, unif = _xcase(rng, 3, 3, 40, 40, 40)
+    ident = np.arange(40)
+    r0 = O.fuse_verify(a, b, t, draft, probs, unif, mode=mode)
+    r1 = O.fuse_verify_xvocab(a, b, t, ident, ident, draft, probs, unif, mode=mode)
+    _same(r0, r1)
+    assert np.array_equal(r1.next_index, r0.next_token)
+    np.testing.assert_allclose(r0.lse, r1.lse, rtol=1e-12)
+
+
+@pytest.mark.parametrize("mode", [O.GREEDY, O.STOCHASTIC])
+def test_xvocab_tokens_outside_the_shared_set_do_not_matter(rng, mode):
+    # committed tokens are restricted to the pairs: changing (even poisoning)
+    # unpaired logits of either vocabulary changes nothing
+    a, b, t, md, mv, draft, probs, unif = _xcase(rng, 4, 2, 70, 55, 30)
+    r0 = O.fuse_verify_xvocab(a, b, t, md, mv, draft, probs, unif, mode=mode)
+    free_d = np.setdiff1d(np.arange(70), md)
+    free_v = np.setdiff1d(np.arange(55), mv)
+    a2, b2, t2 = a.copy(), b.copy(), t.copy()
+    a2[..., free_d] = 60.0
+    b2[..., free_d] = np.nan
+    t2[..., free_v] = rng.normal(30, 5, t2[..., free_v].shape)
+    r1 = O.fuse_verify_xvocab(a2, b2, t2, md, mv, draft, probs, unif, mode=mode)
+    _same(r0, r1)
+    assert not r1.error.any()
+
+
+@pytest.mark.parametrize("mode", [O.GREEDY, O.STOCHASTIC])
+def test_xvocab_relabelling_either_vocabulary(rng, mode):
+    # renaming the verifier's tokens renames the committed token and nothing
+    # else; renaming the drafter's tokens changes nothing
+    a, b, t, md, mv, draft, probs, unif = _xcase(rng, 4, 3, 64, 48, 36)
+    r0 = O.fuse_verify_xvocab(a, b, t, md, mv, draft, probs, unif, mode=mode)
+    pv = rng.permutation(48)
+    t2 = np.empty_like(t)
+    t2[..., pv] = t
+    r1 = O.fuse_verify_xvocab(a, b, t2, md, pv[mv], draft, probs, unif, mode=mode)
+    _same(r0, r1, next_map=pv)
+    pd = rng.permutation(64)
+    a2, b2 = np.empty_like(a), np.empty_like(b)
+    a2[..., pd] = a
+    b2[..., pd] = b
+    r2 = O.fuse_verify_xvocab(a2, b2, t, pd[md], mv, draft, probs, unif, mode=mode)
+    _same(r0, r2)
+
+
+def test_xvocab_restricted_normalisation_closed_form():
+    # two pairs, K = 1, greedy.  Over the pairs: p_a' = (1/2, 1/2),
+    # p_b' = (0.8, 0.2), p_t' = (e^2, 1) / (e^2 + 1).  The unpaired verifier
+    # tokens 0 and 3 carry almost all of the full verifier vocabulary's mass:
+    # normalised over the full vocabulary the draft would be rejected
+    # (p_t = 1 / (2 e^35 + e^2 + 1) against gamma_eff p_b ~ 0.1); over the pairs
+    # it is accepted (1 / (1 + e^2) = 0.119 > gamma_eff 0.2).
+    V_d, V_v = 3, 4
+    md, mv = np.array([1, 0]), np.array([2, 1])
+    a = np.zeros((1, 2, V_d), np.float32)
+    a[..., 2] = -30.0
+    b = np.zeros((1, 2, V_d), np.float32)
+    b[..., 1], b[..., 0], b[..., 2] = np.log(0.8), np.log(0.2), -30.0
+    t = np.zeros((1, 2, V_v), np.float32)
+    t[..., 0] = t[..., 3] = 35.0
+    t[0, :, 2], t[0, :, 1] = 2.0, 0.0          # t' = (2, 0)
+    draft = np.array([[1]])                     # pair 1: drafter token 0, verifier token 1
+    r = O.fuse_verify_xvocab(a, b, t, md, mv, draft, gamma=0.5, beta=1.0)
+    p = np.array([0.5, 0.5])
+    q = np.array([np.float32(np.log(0.8)), np.float32(np.log(0.2))], np.float64)
+    q = np.exp(q) / np.exp(q).sum()
+    m = (p + q) / 2
+    D = 0.5 * np.sum(p * np.log(p / m)) + 0.5 * np.sum(q * np.log(q / m))
+    assert r.D[0, 0] == pytest.approx(D, rel=1e-9)
+    gamma_eff = 0.5 * np.exp(-D)
+    assert r.gamma_eff[0, 0] == pytest.approx(gamma_eff, rel=1e-7)
+    pt = 1.0 / (1.0 + np.exp(2.0))
+    assert pt > gamma_eff * q[1] and r.accept_len[0] == 1
+    assert 1.0 / (2 * np.exp(35.0) + np.exp(2.0) + 1.0) < gamma_eff * q[1]
+    # all K drafts accepted: the bonus row emits argmax t' = pair 0 = verifier token 2
+    assert r.next_index[0] == 0 and r.next_token[0] == 2
+
+
+def test_xvocab_maps_and_draft_indices_are_validated(rng):
+    a, b, t, md, mv, draft, probs, unif = _xcase(rng, 2, 2, 30, 20, 10)
+    with pytest.raises(ValueError):
+        O.fuse_verify_xvocab(a, b, t, md, mv[:-1], draft)
+    bad = md.copy()
+    bad[3] = bad[4]
+    with pytest.raises(ValueError):
+        O.fuse_verify_xvocab(a, b, t, bad, mv, draft)
+    bad = mv.copy()
+    bad[0] = 20
+    with pytest.raises(ValueError):
+        O.fuse_verify_xvocab(a, b, t, md, bad, draft)
+    d2 = draft.copy()
+    d2[1, 0] = 10                                # a pair index outside [0, S)
+    r = O.fuse_verify_xvocab(a, b, t, md, mv, d2)
+    assert list(r.error) == [False, True] and r.next_token[1] == -1
