@@ -257,6 +257,77 @@ def draft_timing(torch, A, sets, B, K, V, mode, dev, steps):
     return res
 
 
+def xvocab_timing(torch, A, synth, mode, dev, steps, timed, stream):
+    """The cross-family step (asymspec_fuse_verify_xvocab: gather, step,
+    emission) on the bench workload's batch shape over a Qwen3-sized drafter
+    vocabulary, a Llama-3-sized verifier vocabulary and the paper's shared set,
+    and its gather (asymspec_xvocab_gather) alone; CUDA events on the stream."""
+    w = synth.CONFIGS[WORKLOAD_CFG]
+    x = synth.make_xvocab(w.recipe, w.seed, w.B, w.K, synth.XVOCAB_S, synth.XVOCAB_V_D,
+                          synth.XVOCAB_V_V, synth.BF16)
+    B, K, S, V_d, V_v = x.B, x.K, x.S, x.V_d, x.V_v
+    rows = B * (K + 1)
+
+    def bf(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    a, b, t = bf(x.logits_full), bf(x.logits_comp), bf(x.logits_ver)
+    md = torch.from_numpy(x.map_d).to(dev)
+    mv = torch.from_numpy(x.map_v).to(dev)
+    d = torch.from_numpy(x.draft_tokens).to(dev)
+    pr = torch.from_numpy(x.draft_probs).to(dev)
+    u = torch.from_numpy(x.uniforms).to(dev)
+    nbytes = A.xvocab_workspace_bytes(B, K, S, A.BF16)
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+    L = torch.empty(B, dtype=torch.int32, device=dev)
+    N = torch.empty(B, dtype=torch.int32, device=dev)
+    gate = A.gate_params(mode=mode)
+    sptr = stream.cuda_stream
+
+    def step(i):
+        st = A.fuse_verify_xvocab(a.data_ptr(), b.data_ptr(), V_d, t.data_ptr(), V_v,
+                                  md.data_ptr(), mv.data_ptr(), S, d.data_ptr(), pr.data_ptr(),
+                                  u.data_ptr(), B, K, A.BF16, gate, L.data_ptr(), N.data_ptr(),
+                                  0, ws.data_ptr(), nbytes, None, sptr)
+        if st != A.OK:
+            raise A.AsymSpecError(st, "asymspec_fuse_verify_xvocab")
+
+    g_out = torch.empty(3, rows, S, dtype=torch.bfloat16, device=dev)
+
+    def gather(i):
+        st = A.xvocab_gather(a.data_ptr(), b.data_ptr(), V_d, t.data_ptr(), V_v, md.data_ptr(),
+                             mv.data_ptr(), S, rows, A.BF16, g_out[0].data_ptr(),
+                             g_out[1].data_ptr(), g_out[2].data_ptr(), None, sptr)
+        if st != A.OK:
+            raise A.AsymSpecError(st, "asymspec_xvocab_gather")
+
+    n = max(3, min(steps, 50))
+    ms_step = timed(step, n, 3) / n
+    ms_gather = timed(gather, n, 3) / n
+    del g_out, ws
+
+    # the gather must bring in every 32-byte DRAM sector holding a paired entry
+    # and write the restricted rows densely
+    def sectors(m):
+        return int(np.unique(m.astype(np.int64) * 2 // 32).size)
+
+    touched = rows * 32 * (2 * sectors(x.map_d) + sectors(x.map_v))
+    written = rows * 3 * S * 2
+    hbm_peak, peak_kind = peaks()
+    g_gbs = (touched + written) / (ms_gather * 1e-3) / 1e9
+    return {"mode": "stochastic" if mode == A.MODE_STOCHASTIC else "greedy",
+            "B": B, "K": K, "S": S, "V_d": V_d, "V_v": V_v, "rows": rows,
+            "ms_per_step": ms_step, "rows_per_s": rows / (ms_step * 1e-3),
+            "launches_per_step": 4,
+            "gather": {"kernel": "xvocab_gather", "us_per_launch": ms_gather * 1e3,
+                       "algorithmic_bytes_per_launch": touched + written,
+                       "algorithmic_bytes": "the 32-byte sectors of a, b and t holding paired "
+                                            "entries, read once, plus the restricted rows "
+                                            "written once",
+                       "hbm_gbs": g_gbs, "frac": g_gbs / hbm_peak, "peak_kind": peak_kind},
+            "timing": "CUDA events around the timed calls on the launching stream"}
+
+
 def run_reference(args, workload, rank, world):
     """--impl reference: the float64 CPU oracle, timed on the host cores."""
     from paper_2608_26004_gb300 import synth
@@ -427,6 +498,10 @@ def main():
     # the launches read the rows of both resident sets in turn (262 MB > L2).
     draft = draft_timing(torch, A, sets, B, K, V, mode, dev, args.steps)
 
+    # ---- the cross-family step (drafter and verifier vocabularies that
+    # differ, restricted to their shared tokens): reported alongside
+    xvocab = xvocab_timing(torch, A, synth, mode, dev, args.steps, timed, stream)
+
     # ---- end to end through the C ABI with host buffers
     pin = dict(
         a=torch.from_numpy(np.ascontiguousarray(batch.logits_full).view(np.int16)).view(
@@ -486,6 +561,7 @@ def main():
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
         "draft": draft,
+        "xvocab": xvocab,
         "other_mode": {"mode": "greedy" if other_mode == A.MODE_GREEDY else "stochastic",
                        "ms_per_step": ms_o, "rows_per_s": world * rows / (ms_o * 1e-3),
                        "hbm_gbs": alg_bytes_o / (ms_o * 1e-3) / 1e9,

@@ -70,6 +70,7 @@ extern "C" {
 #define ASYMSPEC_DATA_BAD_UNIFORM 0x8u  /* stochastic: uniform outside [0, 1) */
 #define ASYMSPEC_DATA_TIMEOUT 0x10u     /* a bulk copy into shared memory did not complete within
                                            its time limit (the kernel gave up instead of hanging) */
+#define ASYMSPEC_DATA_BAD_MAP 0x20u     /* cross-family step: a map entry outside its vocabulary */
 
 typedef enum { ASYMSPEC_FP32 = 0, ASYMSPEC_BF16 = 1 } asymspec_dtype_t;
 
@@ -330,6 +331,66 @@ int asymspec_fuse_verify_host(const void* h_logits_full, const void* h_logits_co
 int asymspec_draft_sample(const void* logits, int rows, int V, int dtype, int mode,
                           const float* uniforms, int32_t* out_tokens, float* out_probs,
                           int cluster_size, void* stream);
+
+/* ---- cross-family vocabularies -------------------------------------------
+ * The step for a drafter and a verifier that tokenise differently (Section 4,
+ * "Cross-family portability", and the appendix of the same name: delta is
+ * computed in the drafter's vocabulary and carried to the verifier through
+ * the S string-identical tokens; committed tokens are restricted to that
+ * shared set).  The S pairs are (map_d[j], map_v[j]): drafter token map_d[j]
+ * and verifier token map_v[j] spell the same string.  The step runs, exactly
+ * as asymspec_fuse_verify_ex defines it, on the rows restricted to the pairs
+ * in pair order, a'_j = a[map_d[j]], b'_j = b[map_d[j]], t'_j = t[map_v[j]]:
+ * every softmax, the divergence of Eq. 3, the acceptance test of Eq. 4 and
+ * the emission are taken over the S pairs.  Draft tokens are given as pair
+ * indices in [0, S); the emitted pair index j is committed as the verifier
+ * token map_v[j].
+ *
+ * asymspec_xvocab_gather: the restriction alone.  For each of `rows` rows,
+ *   out_full[r][j] = logits_full[r][map_d[j]], out_comp likewise, and
+ *   out_ver[r][j] = logits_ver[r][map_v[j]]; outputs [rows, S] row-major in
+ *   `dtype`, caller-owned device memory.  logits_full and logits_comp are
+ *   [rows, V_d], logits_ver [rows, V_v], all device, element-aligned.
+ *   map_d, map_v: [S] int32 device.  A map entry outside [0, V_d) or
+ *   [0, V_v) is not dereferenced: the gathered values become NaN and
+ *   ASYMSPEC_DATA_BAD_MAP is OR-ed into *out_error_word (device, may be
+ *   NULL).  Maps with a token in two pairs are not detected (the library
+ *   computes over them as given; the paper's maps pair each token once).
+ *   One launch on `stream`, nothing allocated.  Host-detectable errors:
+ *   ASYMSPEC_ERR_INVALID_ARG (a null pointer, rows < 0, S < 2, V_d < 1,
+ *   V_v < 1), ASYMSPEC_ERR_UNSUPPORTED (dtype), ASYMSPEC_ERR_MISALIGNED.
+ *
+ * asymspec_fuse_verify_xvocab: gather, step and emission, three or four
+ *   launches on `stream` (the gather, the step's one or two, the emission):
+ *   logits_full, logits_comp [B, K+1, V_d]; logits_ver [B, K+1, V_v];
+ *   draft_index [B, K] int32 pair indices; draft_probs, uniforms, gate_params
+ *   as for asymspec_fuse_verify (draft_probs[b][k] is the drafter's
+ *   probability of pair draft_index[b][k] under the restricted softmax);
+ *   out_accept_len, out_next_token [B] int32 (verifier tokens);
+ *   out_next_index [B] int32 or NULL: the emitted pair index;
+ *   workspace of asymspec_xvocab_workspace_bytes(B, K, S, dtype) bytes,
+ *   16-byte aligned and zeroed before its first use (asymspec_workspace_reset;
+ *   every call that completes leaves it fit for the next); out_error_word as
+ *   for asymspec_fuse_verify_ex.  The restricted rows are laid out with a
+ *   stride of S entries, so the fast kernel runs when S * element size is a
+ *   multiple of 16 and the generic one otherwise.  Status codes are those of
+ *   asymspec_fuse_verify_ex and asymspec_xvocab_gather; a pair index outside
+ *   [0, S) is the data error ASYMSPEC_DATA_BAD_TOKEN of that element.
+ */
+size_t asymspec_xvocab_workspace_bytes(int B, int K, int S, int dtype);
+int asymspec_xvocab_gather(const void* logits_full, const void* logits_comp, int V_d,
+                           const void* logits_ver, int V_v, const int32_t* map_d,
+                           const int32_t* map_v, int S, int rows, int dtype, void* out_full,
+                           void* out_comp, void* out_ver, uint32_t* out_error_word,
+                           void* stream);
+int asymspec_fuse_verify_xvocab(const void* logits_full, const void* logits_comp, int V_d,
+                                const void* logits_ver, int V_v, const int32_t* map_d,
+                                const int32_t* map_v, int S, const int32_t* draft_index,
+                                const float* draft_probs, const float* uniforms, int B, int K,
+                                int dtype, const asymspec_gate_params* gate_params,
+                                int32_t* out_accept_len, int32_t* out_next_token,
+                                int32_t* out_next_index, void* workspace,
+                                size_t workspace_bytes, uint32_t* out_error_word, void* stream);
 
 /* Launch parameters a call with these sizes would use, without launching.
  * Uses the current CUDA device. */

@@ -34,6 +34,7 @@ DATA_NONFINITE = 0x2
 DATA_BAD_PROB = 0x4
 DATA_BAD_UNIFORM = 0x8
 DATA_TIMEOUT = 0x10
+DATA_BAD_MAP = 0x20
 
 FP32 = 0
 BF16 = 1
@@ -55,6 +56,9 @@ EXPORTED = (
     "asymspec_host_scratch_bytes",
     "asymspec_fuse_verify_host",
     "asymspec_draft_sample",
+    "asymspec_xvocab_workspace_bytes",
+    "asymspec_xvocab_gather",
+    "asymspec_fuse_verify_xvocab",
     "asymspec_plan",
     "asymspec_status_string",
     "asymspec_last_cuda_error",
@@ -141,6 +145,15 @@ def lib():
     L.asymspec_fuse_verify_host.restype = _I
     L.asymspec_draft_sample.argtypes = [_P, _I, _I, _I, _I, _P, _P, _P, _I, _P]
     L.asymspec_draft_sample.restype = _I
+    L.asymspec_xvocab_workspace_bytes.argtypes = [_I, _I, _I, _I]
+    L.asymspec_xvocab_workspace_bytes.restype = ctypes.c_size_t
+    L.asymspec_xvocab_gather.argtypes = [_P, _P, _I, _P, _I, _P, _P, _I, _I, _I, _P, _P, _P,
+                                         _P, _P]
+    L.asymspec_xvocab_gather.restype = _I
+    L.asymspec_fuse_verify_xvocab.argtypes = [_P, _P, _I, _P, _I, _P, _P, _I, _P, _P, _P, _I,
+                                              _I, _I, ctypes.POINTER(GateParams), _P, _P, _P,
+                                              _P, ctypes.c_size_t, _P, _P]
+    L.asymspec_fuse_verify_xvocab.restype = _I
     L.asymspec_plan.argtypes = [_I, _I, _I, _I, ctypes.POINTER(GateParams),
                                 ctypes.POINTER(LaunchOpts), ctypes.POINTER(LaunchInfo)]
     L.asymspec_plan.restype = _I
@@ -236,6 +249,30 @@ def draft_sample(logits, rows, V, dtype, mode, uniforms, out_tokens, out_probs, 
     """asymspec_draft_sample with device addresses (ints); returns the status."""
     return lib().asymspec_draft_sample(logits, rows, V, dtype, mode, uniforms, out_tokens,
                                        out_probs, cluster_size, stream)
+
+
+def xvocab_workspace_bytes(B, K, S, dtype) -> int:
+    return int(lib().asymspec_xvocab_workspace_bytes(B, K, S, dtype))
+
+
+def xvocab_gather(logits_full, logits_comp, V_d, logits_ver, V_v, map_d, map_v, S, rows, dtype,
+                  out_full, out_comp, out_ver, out_error_word=None, stream=0) -> int:
+    """asymspec_xvocab_gather with device addresses (ints); returns the status."""
+    return lib().asymspec_xvocab_gather(logits_full, logits_comp, V_d, logits_ver, V_v, map_d,
+                                        map_v, S, rows, dtype, out_full, out_comp, out_ver,
+                                        out_error_word, stream)
+
+
+def fuse_verify_xvocab(logits_full, logits_comp, V_d, logits_ver, V_v, map_d, map_v, S,
+                       draft_index, draft_probs, uniforms, B, K, dtype, gate, out_accept_len,
+                       out_next_token, out_next_index, workspace, workspace_nbytes,
+                       out_error_word=None, stream=0) -> int:
+    """asymspec_fuse_verify_xvocab with device addresses (ints); returns the status."""
+    g = ctypes.byref(gate) if gate is not None else None
+    return lib().asymspec_fuse_verify_xvocab(
+        logits_full, logits_comp, V_d, logits_ver, V_v, map_d, map_v, S, draft_index,
+        draft_probs, uniforms, B, K, dtype, g, out_accept_len, out_next_token, out_next_index,
+        workspace, workspace_nbytes, out_error_word, stream)
 
 
 def plan(B, K, V, dtype, gate=None, opts=None) -> LaunchInfo:

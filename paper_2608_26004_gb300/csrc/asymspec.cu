@@ -21,6 +21,7 @@
 #include "kernel_ring.cuh"
 #include "kernel_draft.cuh"
 #include "kernel_stream.cuh"
+#include "kernel_xvocab.cuh"
 #include "kernels.h"
 
 namespace {
@@ -1041,6 +1042,125 @@ int asymspec_draft_sample(const void* logits, int rows, int V, int dtype, int mo
   cfg.numAttrs = 1;
   void* args[] = {&P};
   e = cudaLaunchKernelExC(&cfg, fn, args);
+  return e == cudaSuccess ? ASYMSPEC_OK : cuda_fail(e);
+}
+
+}  // extern "C"
+
+// ------------------------------------------------- cross-family vocabularies
+
+namespace {
+
+// Workspace of asymspec_fuse_verify_xvocab, each part 256-byte aligned: the
+// restricted rows a', b', t' ([B, K+1, S] each), the emitted pair indices
+// ([B] int32), then the step's own workspace for a vocabulary of S entries.
+struct XLayout {
+  size_t ga, gb, gt, idx, step, step_bytes, total;
+};
+
+XLayout xvocab_layout(int B, int K, int S, int dtype) {
+  XLayout L;
+  const size_t plane = round_up(static_cast<size_t>(B) * (K + 1) * S * elt_size(dtype), 256);
+  L.ga = 0;
+  L.gb = plane;
+  L.gt = 2 * plane;
+  L.idx = 3 * plane;
+  L.step = L.idx + round_up(static_cast<size_t>(B) * sizeof(int32_t), 256);
+  L.step_bytes = asymspec_workspace_bytes(B, K, S);
+  L.total = L.step + L.step_bytes;
+  return L;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t asymspec_xvocab_workspace_bytes(int B, int K, int S, int dtype) {
+  if (B < 1 || K < 1 || S < 2) return 0;
+  if (dtype != ASYMSPEC_FP32 && dtype != ASYMSPEC_BF16) return 0;
+  return xvocab_layout(B, K, S, dtype).total;
+}
+
+int asymspec_xvocab_gather(const void* logits_full, const void* logits_comp, int V_d,
+                           const void* logits_ver, int V_v, const int32_t* map_d,
+                           const int32_t* map_v, int S, int rows, int dtype, void* out_full,
+                           void* out_comp, void* out_ver, uint32_t* out_error_word,
+                           void* stream) {
+  if (dtype != ASYMSPEC_FP32 && dtype != ASYMSPEC_BF16) return ASYMSPEC_ERR_UNSUPPORTED;
+  if (rows < 0 || S < 2 || V_d < 1 || V_v < 1) return ASYMSPEC_ERR_INVALID_ARG;
+  if (rows == 0) return ASYMSPEC_OK;
+  if (!logits_full || !logits_comp || !logits_ver || !map_d || !map_v || !out_full ||
+      !out_comp || !out_ver)
+    return ASYMSPEC_ERR_INVALID_ARG;
+  const int elt = elt_size(dtype);
+  if (!aligned(logits_full, elt) || !aligned(logits_comp, elt) || !aligned(logits_ver, elt) ||
+      !aligned(out_full, elt) || !aligned(out_comp, elt) || !aligned(out_ver, elt) ||
+      !aligned(map_d, 4) || !aligned(map_v, 4) || (out_error_word && !aligned(out_error_word, 4)))
+    return ASYMSPEC_ERR_MISALIGNED;
+  const long long ycount = (static_cast<long long>(rows) + kXRows - 1) / kXRows;
+  if (ycount > 65535) return ASYMSPEC_ERR_TOO_LARGE;
+  XGatherParams P;
+  P.a = logits_full;
+  P.b = logits_comp;
+  P.t = logits_ver;
+  P.map_d = map_d;
+  P.map_v = map_v;
+  P.ga = out_full;
+  P.gb = out_comp;
+  P.gt = out_ver;
+  P.err_word = out_error_word;
+  P.rows = rows;
+  P.V_d = V_d;
+  P.V_v = V_v;
+  P.S = S;
+  const dim3 grid(static_cast<unsigned>((S + kXThreads * kXJ - 1) / (kXThreads * kXJ)),
+                  static_cast<unsigned>(ycount));
+  void* args[] = {&P};
+  const cudaError_t e = cudaLaunchKernel(xvocab_gather_ptr(dtype), grid, dim3(kXThreads), args,
+                                         0, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? ASYMSPEC_OK : cuda_fail(e);
+}
+
+int asymspec_fuse_verify_xvocab(const void* logits_full, const void* logits_comp, int V_d,
+                                const void* logits_ver, int V_v, const int32_t* map_d,
+                                const int32_t* map_v, int S, const int32_t* draft_index,
+                                const float* draft_probs, const float* uniforms, int B, int K,
+                                int dtype, const asymspec_gate_params* gate_params,
+                                int32_t* out_accept_len, int32_t* out_next_token,
+                                int32_t* out_next_index, void* workspace,
+                                size_t workspace_bytes, uint32_t* out_error_word, void* stream) {
+  if (B < 1 || K < 1 || S < 2 || V_d < 1 || V_v < 1) return ASYMSPEC_ERR_INVALID_ARG;
+  if (dtype != ASYMSPEC_FP32 && dtype != ASYMSPEC_BF16) return ASYMSPEC_ERR_UNSUPPORTED;
+  asymspec_gate_params gp;
+  asymspec_default_gate_params(&gp);
+  if (gate_params) gp = *gate_params;
+  int st = check_params(&gp);
+  if (st) return st;
+  if (!draft_index || !out_accept_len || !out_next_token) return ASYMSPEC_ERR_INVALID_ARG;
+  if (gp.mode == ASYMSPEC_MODE_STOCHASTIC && (!draft_probs || !uniforms))
+    return ASYMSPEC_ERR_INVALID_ARG;
+  if (!aligned(out_next_token, 4) || (out_next_index && !aligned(out_next_index, 4)))
+    return ASYMSPEC_ERR_MISALIGNED;
+  const XLayout L = xvocab_layout(B, K, S, dtype);
+  if (!workspace || !aligned(workspace, 16) || workspace_bytes < L.total)
+    return ASYMSPEC_ERR_WORKSPACE;
+  char* base = static_cast<char*>(workspace);
+  st = asymspec_xvocab_gather(logits_full, logits_comp, V_d, logits_ver, V_v, map_d, map_v, S,
+                              B * (K + 1), dtype, base + L.ga, base + L.gb, base + L.gt,
+                              out_error_word, stream);
+  if (st) return st;
+  int32_t* idx = out_next_index ? out_next_index : reinterpret_cast<int32_t*>(base + L.idx);
+  st = asymspec_fuse_verify_ex(base + L.ga, base + L.gb, base + L.gt, draft_index, draft_probs,
+                               uniforms, B, K, S, dtype, &gp, out_accept_len, idx,
+                               base + L.step, L.step_bytes, nullptr, nullptr, nullptr,
+                               out_error_word, nullptr, stream);
+  if (st) return st;
+  int32_t* next = out_next_token;
+  const int32_t* mv = map_v;
+  int S_ = S, B_ = B;
+  void* args[] = {&idx, &mv, &S_, &B_, &next};
+  const cudaError_t e = cudaLaunchKernel(xvocab_emit_ptr(), dim3((B + 255) / 256), dim3(256),
+                                         args, 0, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? ASYMSPEC_OK : cuda_fail(e);
 }
 

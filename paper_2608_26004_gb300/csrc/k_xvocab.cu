@@ -1,0 +1,14 @@
+// Instantiations of the cross-family gather and emission (see kernel_xvocab.cuh).
+#include "kernel_xvocab.cuh"
+#include "kernels.h"
+
+namespace asymspec_impl {
+
+const void* xvocab_gather_ptr(int dtype) {
+  return dtype == ASYMSPEC_FP32 ? reinterpret_cast<const void*>(&xvocab_gather<float>)
+                                : reinterpret_cast<const void*>(&xvocab_gather<__nv_bfloat16>);
+}
+
+const void* xvocab_emit_ptr() { return reinterpret_cast<const void*>(&xvocab_emit<int32_t>); }
+
+}  // namespace asymspec_impl

@@ -29,5 +29,8 @@ const void* stream_kernel_f32_greedy();
 const void* stream_kernel_f32_stoch();
 // draft_kernel<T, VE, STOCH>, the drafter's draw (k_draft.cu)
 const void* draft_kernel_ptr(int dtype, bool vector_path, bool stoch);
+// xvocab_gather<T> and xvocab_emit, the cross-family vocabulary map (k_xvocab.cu)
+const void* xvocab_gather_ptr(int dtype);
+const void* xvocab_emit_ptr();
 
 }  // namespace asymspec_impl

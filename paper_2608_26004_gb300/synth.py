@@ -212,3 +212,71 @@ def make_config(cfg_id: int, sweep_index: int = 0, b0: int = 0, nb: int | None =
         nb = w.B - b0
     return generate(rc, w.seed, w.B, w.K, w.V, w.dtype, b0=b0, nb=nb, B_total=w.B,
                     nthreads=nthreads)
+
+
+# ------------------------------------------------- cross-family vocabularies
+
+# The paper's heterogeneous pairings (Section 4, "Cross-family portability")
+# share 109,566 string-identical tokens plus paired special tokens between a
+# Qwen3 (151,936) and a Llama-3 (128,256) vocabulary; two special pairs are
+# taken here, which makes S = 109,568.
+XVOCAB_S = 109_568
+XVOCAB_V_D = 151_936
+XVOCAB_V_V = 128_256
+
+
+@dataclass
+class XBatch:
+    """A step whose drafter (vocabulary V_d) and verifier (vocabulary V_v)
+    share S tokens, the pairs (map_d[j], map_v[j]).  logits_full and
+    logits_comp are [B, K+1, V_d], logits_ver [B, K+1, V_v]; draft_tokens are
+    pair indices in [0, S) and draft_probs their probabilities under the
+    drafter's softmax over the pairs."""
+
+    logits_full: np.ndarray
+    logits_comp: np.ndarray
+    logits_ver: np.ndarray
+    map_d: np.ndarray
+    map_v: np.ndarray
+    draft_tokens: np.ndarray
+    draft_probs: np.ndarray
+    uniforms: np.ndarray
+    B: int
+    K: int
+    S: int
+    V_d: int
+    V_v: int
+    dtype: int
+
+
+def _f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round-to-nearest-even bf16 bit patterns of finite float32 values."""
+    u = np.ascontiguousarray(x, np.float32).view(np.uint32)
+    return ((u + (((u >> 16) & 1) + 0x7FFF)) >> 16).astype(np.uint16)
+
+
+def make_xvocab(recipe: Recipe, seed: int, B: int, K: int, S: int, V_d: int, V_v: int,
+                dtype: int, unpaired_mean: float = 3.0, nthreads: int = 0) -> XBatch:
+    """Cross-family inputs: the workload recipe generated over the S shared
+    tokens (so the drafts and their probabilities are those of the shared
+    set), scattered into the two vocabularies through a seeded map.  map_d
+    is an increasing subset of the drafter's tokens, map_v a random
+    injection into the verifier's; the unpaired logits are N(unpaired_mean,
+    2^2), above the paired ones on average, so that a path that read them
+    would visibly change every normaliser."""
+    if not (2 <= S <= min(V_d, V_v)):
+        raise ValueError("need 2 <= S <= min(V_d, V_v)")
+    inner = generate(recipe, seed, B, K, S, dtype, nthreads=nthreads)
+    rng = np.random.default_rng(seed)
+    map_d = np.sort(rng.choice(V_d, S, replace=False)).astype(np.int32)
+    map_v = rng.choice(V_v, S, replace=False).astype(np.int32)
+
+    def scatter(rows, V, idx):
+        fill = rng.normal(unpaired_mean, 2.0, (B, K + 1, V)).astype(np.float32)
+        out = fill if dtype == FP32 else _f32_to_bf16_bits(fill)
+        out[..., idx] = rows
+        return out
+
+    return XBatch(scatter(inner.logits_full, V_d, map_d), scatter(inner.logits_comp, V_d, map_d),
+                  scatter(inner.logits_ver, V_v, map_v), map_d, map_v, inner.draft_tokens,
+                  inner.draft_probs, inner.uniforms, B, K, S, V_d, V_v, dtype)

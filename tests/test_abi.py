@@ -256,3 +256,50 @@ def test_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):
     monkeypatch.setattr(A, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError):
         A.workspace_bytes(1, 1, 2)
+
+
+def test_xvocab_workspace_layout_and_validation(lib):
+    # the restricted rows a', b', t' ([B, K+1, S] each), the emitted pair
+    # indices, then the step's workspace for a vocabulary of S entries
+    for B, K, S, dtype, elt in ((64, 7, 109568, A.BF16, 2), (3, 2, 37, A.FP32, 4)):
+        R = B * (K + 1)
+        want = 3 * _up(R * S * elt) + _up(B * 4) + A.workspace_bytes(B, K, S)
+        assert A.xvocab_workspace_bytes(B, K, S, dtype) == want
+    assert A.xvocab_workspace_bytes(0, 2, 10, A.FP32) == 0
+    assert A.xvocab_workspace_bytes(2, 2, 1, A.FP32) == 0
+    assert A.xvocab_workspace_bytes(2, 2, 10, 5) == 0
+    need = A.xvocab_workspace_bytes(2, 2, 10, A.FP32)
+
+    def fv(B=2, K=2, S=10, V_d=30, V_v=20, dtype=A.FP32, gate=None, ws=FAKE, n=need, **p):
+        x = dict(a=FAKE, b=FAKE, t=FAKE, md=FAKE, mv=FAKE, d=FAKE, pr=FAKE, u=FAKE, L=FAKE,
+                 N=FAKE, I=0)
+        x.update(p)
+        return A.fuse_verify_xvocab(x["a"], x["b"], V_d, x["t"], V_v, x["md"], x["mv"], S,
+                                    x["d"], x["pr"], x["u"], B, K, dtype, gate, x["L"], x["N"],
+                                    x["I"], ws, n)
+
+    # every case returns before any CUDA call
+    assert fv(B=0) == A.ERR_INVALID_ARG
+    assert fv(S=1) == A.ERR_INVALID_ARG
+    assert fv(V_v=0) == A.ERR_INVALID_ARG
+    assert fv(dtype=3) == A.ERR_UNSUPPORTED
+    assert fv(gate=A.gate_params(gamma=2.0)) == A.ERR_INVALID_ARG
+    assert fv(d=0) == A.ERR_INVALID_ARG
+    assert fv(gate=A.gate_params(mode=A.MODE_STOCHASTIC), u=0) == A.ERR_INVALID_ARG
+    assert fv(N=FAKE + 2) == A.ERR_MISALIGNED
+    assert fv(ws=0) == A.ERR_WORKSPACE
+    assert fv(ws=FAKE + 8) == A.ERR_WORKSPACE
+    assert fv(n=need - 1) == A.ERR_WORKSPACE
+    assert fv(md=0) == A.ERR_INVALID_ARG                 # the gather's own checks
+    assert fv(a=FAKE + 2) == A.ERR_MISALIGNED
+    assert fv(mv=FAKE + 1) == A.ERR_MISALIGNED
+    g = A.xvocab_gather
+    assert g(FAKE, FAKE, 30, FAKE, 20, FAKE, FAKE, 10, -1, A.FP32, FAKE, FAKE, FAKE) \
+        == A.ERR_INVALID_ARG
+    assert g(0, 0, 30, 0, 20, 0, 0, 10, 0, A.FP32, 0, 0, 0) == A.OK  # no rows: no-op
+    assert g(FAKE, FAKE, 30, FAKE, 20, FAKE, FAKE, 10, 4, 9, FAKE, FAKE, FAKE) \
+        == A.ERR_UNSUPPORTED
+    assert g(FAKE, FAKE, 30, FAKE, 20, FAKE, FAKE, 10, 4, A.BF16, FAKE + 1, FAKE, FAKE) \
+        == A.ERR_MISALIGNED
+    assert g(FAKE, FAKE, 30, FAKE, 20, FAKE, FAKE, 10, 8 * 65536, A.FP32, FAKE, FAKE, FAKE) \
+        == A.ERR_TOO_LARGE

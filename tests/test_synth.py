@@ -81,3 +81,25 @@ def test_draft_probs_are_drafter_probabilities_of_drafts():
         z = a[k] - a[k].max()
         p = np.exp(z) / np.exp(z).sum()
         assert b.draft_probs[0, k] == pytest.approx(p[b.draft_tokens[0, k]], rel=1e-6)
+
+
+def test_xvocab_inputs_embed_the_shared_set():
+    # the recipe generated over the S shared tokens, scattered through a map
+    # whose two sides are injective and in range
+    w = synth.CONFIGS[1]
+    x = synth.make_xvocab(w.recipe, w.seed, 2, 3, 200, 300, 250, synth.BF16)
+    inner = synth.generate(w.recipe, w.seed, 2, 3, 200, synth.BF16)
+    assert np.unique(x.map_d).size == 200 and np.all(np.diff(x.map_d) > 0)
+    assert np.unique(x.map_v).size == 200 and 0 <= x.map_v.min() and x.map_v.max() < 250
+    assert x.map_d.max() < 300
+    assert np.array_equal(x.logits_full[..., x.map_d], inner.logits_full)
+    assert np.array_equal(x.logits_comp[..., x.map_d], inner.logits_comp)
+    assert np.array_equal(x.logits_ver[..., x.map_v], inner.logits_ver)
+    assert np.array_equal(x.draft_tokens, inner.draft_tokens)
+    assert np.array_equal(x.draft_probs, inner.draft_probs)
+    # reproducible from the seed
+    y = synth.make_xvocab(w.recipe, w.seed, 2, 3, 200, 300, 250, synth.BF16)
+    assert np.array_equal(x.logits_ver, y.logits_ver) and np.array_equal(x.map_v, y.map_v)
+    # bf16 rounding of the unpaired fill is round-to-nearest-even
+    bits = synth._f32_to_bf16_bits(np.array([1.0, 1 + 2**-8, 1 + 3 * 2**-8, -2.5], np.float32))
+    assert list(bits) == [0x3F80, 0x3F80, 0x3F82, 0xC020]
