@@ -38,7 +38,7 @@ CSRC = os.path.join(ROOT, "paper_2608_26004_gb300", "csrc")
 KERNEL_SRCS = ("asymspec.cu", "device_common.cuh", "kernel_generic.cuh", "kernel_tma.cuh",
                "kernel_stream.cuh", "kernels.h", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu",
                "k_tma_bf16_prod.cu", "k_tma_f32_prod.cu", "k_tma_bf16_any_s.cu",
-               "k_tma_f32_any_s.cu")
+               "k_tma_f32_any_s.cu", "k_tmap_bf16.cu", "k_tmap_f32.cu")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fuse_verify_tma_B64_K7_V128256_bf16_traffic.txt")
 REASON_BITS = {
     0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
@@ -277,7 +277,7 @@ def xvocab_timing(torch, A, synth, mode, dev, steps, timed, stream):
     d = torch.from_numpy(x.draft_tokens).to(dev)
     pr = torch.from_numpy(x.draft_probs).to(dev)
     u = torch.from_numpy(x.uniforms).to(dev)
-    nbytes = A.xvocab_workspace_bytes(B, K, S, A.BF16)
+    nbytes = A.xvocab_workspace_bytes(B, K, S, V_d, V_v, A.BF16)
     ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
     L = torch.empty(B, dtype=torch.int32, device=dev)
     N = torch.empty(B, dtype=torch.int32, device=dev)
@@ -293,11 +293,14 @@ def xvocab_timing(torch, A, synth, mode, dev, steps, timed, stream):
             raise A.AsymSpecError(st, "asymspec_fuse_verify_xvocab")
 
     g_out = torch.empty(3, rows, S, dtype=torch.bfloat16, device=dev)
+    sc_n = A.xvocab_gather_scratch_bytes(V_d, V_v)
+    sc = torch.empty(sc_n, dtype=torch.uint8, device=dev)
 
     def gather(i):
         st = A.xvocab_gather(a.data_ptr(), b.data_ptr(), V_d, t.data_ptr(), V_v, md.data_ptr(),
                              mv.data_ptr(), S, rows, A.BF16, g_out[0].data_ptr(),
-                             g_out[1].data_ptr(), g_out[2].data_ptr(), None, sptr)
+                             g_out[1].data_ptr(), g_out[2].data_ptr(), None, sc.data_ptr(), sc_n,
+                             sptr)
         if st != A.OK:
             raise A.AsymSpecError(st, "asymspec_xvocab_gather")
 
@@ -318,12 +321,14 @@ def xvocab_timing(torch, A, synth, mode, dev, steps, timed, stream):
     return {"mode": "stochastic" if mode == A.MODE_STOCHASTIC else "greedy",
             "B": B, "K": K, "S": S, "V_d": V_d, "V_v": V_v, "rows": rows,
             "ms_per_step": ms_step, "rows_per_s": rows / (ms_step * 1e-3),
-            "launches_per_step": 4,
+            "launches_per_step": 6,
             "gather": {"kernel": "xvocab_gather", "us_per_launch": ms_gather * 1e3,
                        "algorithmic_bytes_per_launch": touched + written,
                        "algorithmic_bytes": "the 32-byte sectors of a, b and t holding paired "
                                             "entries, read once, plus the restricted rows "
-                                            "written once",
+                                            "written once (the inverse maps the launch builds "
+                                            "and reads are not counted)",
+                       "launches": "the map check (inverse-map fill and build), then the gather",
                        "hbm_gbs": g_gbs, "frac": g_gbs / hbm_peak, "peak_kind": peak_kind},
             "timing": "CUDA events around the timed calls on the launching stream"}
 
@@ -489,6 +494,22 @@ def main():
             raise A.AsymSpecError(st, "asymspec_fuse_verify_ex")
 
     ms_o = timed(lambda i: step_o(sets[i % 2]), args.steps, max(args.warmup, 3)) / args.steps
+
+    # ---- the persistent form of the cluster kernel (asymspec_launch_opts.kernel
+    # = ASYMSPEC_KERNEL_PERSIST), same workload and mode, reported alongside
+    popts = [A.LaunchOpts(0, 0, A.KERNEL_PERSIST, 0, b.cuda_event, e.cuda_event) for b, e in kev]
+    popts_plain = A.LaunchOpts(0, 0, A.KERNEL_PERSIST)
+    pinfo = A.plan(B, K, V, A.BF16, gate, popts_plain)
+    ms_p = timed(lambda i: step(sets[i % 2], popts_plain), args.steps,
+                 max(args.warmup, 3)) / args.steps
+    timed(lambda i: step(sets[i % 2], popts[i] if i < args.steps else popts_plain), args.steps,
+          max(args.warmup, 3))
+    kernel_ms_p = float(np.mean([b.elapsed_time(e) for b, e in kev]))
+    persistent = {"kernel": "fuse_verify_tma<T, STOCH, SEL, true>", "ctas": pinfo.ctas,
+                  "cluster_size": pinfo.cluster_size, "ms_per_step": ms_p,
+                  "rows_per_s": world * rows / (ms_p * 1e-3), "launch_us": kernel_ms_p * 1e3,
+                  "hbm_gbs": alg_bytes / (kernel_ms_p * 1e-3) / 1e9,
+                  "frac": alg_bytes / (kernel_ms_p * 1e-3) / 1e9 / hbm_peak}
     alg_bytes_o = algorithmic_bytes(B, K, V, 2, other_mode == A.MODE_STOCHASTIC)
 
     # ---- the drafter's draw (asymspec_draft_sample), the step upstream of
@@ -562,6 +583,7 @@ def main():
         "clocks": clocks,
         "draft": draft,
         "xvocab": xvocab,
+        "persistent": persistent,
         "other_mode": {"mode": "greedy" if other_mode == A.MODE_GREEDY else "stochastic",
                        "ms_per_step": ms_o, "rows_per_s": world * rows / (ms_o * 1e-3),
                        "hbm_gbs": alg_bytes_o / (ms_o * 1e-3) / 1e9,

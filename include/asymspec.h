@@ -113,7 +113,7 @@ typedef struct {
 typedef struct {
   int32_t cluster_size;   /* CTAs per row triple: 1 to 16 */
   int32_t block_threads;  /* reserved, must be 0 (256 threads per CTA) */
-  int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC, _TMA, _STREAM or _RING */
+  int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC, _TMA, _STREAM, _RING or _PERSIST */
   int32_t pad;            /* reserved, must be 0 */
   /* Optional cudaEvent_t handles (or NULL): recorded on the call's stream
    * immediately before and after the launch of the fused row kernel (not
@@ -133,6 +133,11 @@ typedef struct {
 #define ASYMSPEC_KERNEL_RING 4     /* persistent clusters: pass 1 through a ring of bulk copies,
                                       pass 2 from L2; rows 16-byte aligned; no debug outputs;
                                       on request only */
+#define ASYMSPEC_KERNEL_PERSIST 5  /* persistent form of ASYMSPEC_KERNEL_TMA: as many clusters
+                                      as the device holds, each taking every G-th row; each
+                                      CTA's slice buffer is refilled with the cluster's next
+                                      row chunk by chunk as pass 2 finishes with it; rows
+                                      16-byte aligned; debug outputs */
 
 /* What a launch would use (filled by asymspec_plan). */
 typedef struct {
@@ -143,7 +148,7 @@ typedef struct {
   int64_t ctas;            /* CTAs in the grid */
   int32_t vector_path;     /* 1 if rows qualify for 16-byte copies (V * element size % 16 == 0) */
   int32_t max_active_clusters; /* clusters the device can hold at once (0 if unknown) */
-  int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC, _TMA, _STREAM or _RING */
+  int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC, _TMA, _STREAM, _RING or _PERSIST */
 } asymspec_launch_info;
 
 /* Fills *p with the paper's defaults: gamma 0.5, beta 1.0, lambda 0.1,
@@ -351,38 +356,50 @@ int asymspec_draft_sample(const void* logits, int rows, int V, int dtype, int mo
  *   out_ver[r][j] = logits_ver[r][map_v[j]]; outputs [rows, S] row-major in
  *   `dtype`, caller-owned device memory.  logits_full and logits_comp are
  *   [rows, V_d], logits_ver [rows, V_v], all device, element-aligned.
- *   map_d, map_v: [S] int32 device.  A map entry outside [0, V_d) or
- *   [0, V_v) is not dereferenced: the gathered values become NaN and
- *   ASYMSPEC_DATA_BAD_MAP is OR-ed into *out_error_word (device, may be
- *   NULL).  Maps with a token in two pairs are not detected (the library
- *   computes over them as given; the paper's maps pair each token once).
- *   One launch on `stream`, nothing allocated.  Host-detectable errors:
+ *   map_d, map_v: [S] int32 device.  out_error_word: device word or NULL.
+ *   scratch, scratch_bytes: device memory of at least
+ *   asymspec_xvocab_gather_scratch_bytes(V_d, V_v) bytes, 256-byte aligned,
+ *   no zeroing needed, or NULL.  With a scratch the maps are checked: the
+ *   inverse maps of the pairs are built in it (atomicCAS), and a map entry
+ *   outside its vocabulary or a token that appears in two pairs sets
+ *   ASYMSPEC_DATA_BAD_MAP in *out_error_word and a map-error word in the
+ *   scratch.  Without one, an entry outside its vocabulary is still never
+ *   dereferenced (its values read NaN, and ASYMSPEC_DATA_BAD_MAP is set) but
+ *   a repeated token is not detected.  Each pair is read through the maps
+ *   (one thread per pair and row).  One launch on `stream` (three with a
+ *   scratch), nothing allocated.  Host-detectable errors:
  *   ASYMSPEC_ERR_INVALID_ARG (a null pointer, rows < 0, S < 2, V_d < 1,
- *   V_v < 1), ASYMSPEC_ERR_UNSUPPORTED (dtype), ASYMSPEC_ERR_MISALIGNED.
+ *   V_v < 1), ASYMSPEC_ERR_UNSUPPORTED (dtype), ASYMSPEC_ERR_MISALIGNED,
+ *   ASYMSPEC_ERR_WORKSPACE (scratch unaligned or too small),
+ *   ASYMSPEC_ERR_TOO_LARGE (rows above 524,280).
  *
- * asymspec_fuse_verify_xvocab: gather, step and emission, three or four
- *   launches on `stream` (the gather, the step's one or two, the emission):
- *   logits_full, logits_comp [B, K+1, V_d]; logits_ver [B, K+1, V_v];
- *   draft_index [B, K] int32 pair indices; draft_probs, uniforms, gate_params
- *   as for asymspec_fuse_verify (draft_probs[b][k] is the drafter's
- *   probability of pair draft_index[b][k] under the restricted softmax);
- *   out_accept_len, out_next_token [B] int32 (verifier tokens);
- *   out_next_index [B] int32 or NULL: the emitted pair index;
- *   workspace of asymspec_xvocab_workspace_bytes(B, K, S, dtype) bytes,
- *   16-byte aligned and zeroed before its first use (asymspec_workspace_reset;
- *   every call that completes leaves it fit for the next); out_error_word as
- *   for asymspec_fuse_verify_ex.  The restricted rows are laid out with a
- *   stride of S entries, so the fast kernel runs when S * element size is a
- *   multiple of 16 and the generic one otherwise.  Status codes are those of
+ * asymspec_fuse_verify_xvocab: map check, gather, step and emission, five
+ *   or six launches on `stream` (two for the map check, the gather, the
+ *   step's one or two, the emission): logits_full, logits_comp
+ *   [B, K+1, V_d]; logits_ver [B, K+1, V_v]; draft_index [B, K] int32 pair indices; draft_probs,
+ *   uniforms, gate_params as for asymspec_fuse_verify (draft_probs[b][k] is
+ *   the drafter's probability of pair draft_index[b][k] under the restricted
+ *   softmax); out_accept_len, out_next_token [B] int32 (verifier tokens);
+ *   out_next_index [B] int32 or NULL: the emitted pair index; workspace of
+ *   asymspec_xvocab_workspace_bytes(B, K, S, V_d, V_v, dtype) bytes,
+ *   256-byte aligned and zeroed before its first use
+ *   (asymspec_workspace_reset; every call that completes leaves it fit for
+ *   the next); out_error_word as for asymspec_fuse_verify_ex.  A map entry
+ *   outside its vocabulary or a token in two pairs makes every batch element
+ *   a data error (accept_len = next_token = -1, ASYMSPEC_DATA_BAD_MAP).  The
+ *   restricted rows are laid out with a stride of S entries, so the fast
+ *   step kernel runs when S * element size is a multiple of 16 and the
+ *   generic one otherwise.  Status codes are those of
  *   asymspec_fuse_verify_ex and asymspec_xvocab_gather; a pair index outside
  *   [0, S) is the data error ASYMSPEC_DATA_BAD_TOKEN of that element.
  */
-size_t asymspec_xvocab_workspace_bytes(int B, int K, int S, int dtype);
+size_t asymspec_xvocab_gather_scratch_bytes(int V_d, int V_v);
+size_t asymspec_xvocab_workspace_bytes(int B, int K, int S, int V_d, int V_v, int dtype);
 int asymspec_xvocab_gather(const void* logits_full, const void* logits_comp, int V_d,
                            const void* logits_ver, int V_v, const int32_t* map_d,
                            const int32_t* map_v, int S, int rows, int dtype, void* out_full,
                            void* out_comp, void* out_ver, uint32_t* out_error_word,
-                           void* stream);
+                           void* scratch, size_t scratch_bytes, void* stream);
 int asymspec_fuse_verify_xvocab(const void* logits_full, const void* logits_comp, int V_d,
                                 const void* logits_ver, int V_v, const int32_t* map_d,
                                 const int32_t* map_v, int S, const int32_t* draft_index,

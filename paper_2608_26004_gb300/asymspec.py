@@ -56,6 +56,7 @@ EXPORTED = (
     "asymspec_host_scratch_bytes",
     "asymspec_fuse_verify_host",
     "asymspec_draft_sample",
+    "asymspec_xvocab_gather_scratch_bytes",
     "asymspec_xvocab_workspace_bytes",
     "asymspec_xvocab_gather",
     "asymspec_fuse_verify_xvocab",
@@ -82,6 +83,7 @@ KERNEL_GENERIC = 1
 KERNEL_TMA = 2
 KERNEL_STREAM = 3
 KERNEL_RING = 4
+KERNEL_PERSIST = 5
 
 
 class LaunchOpts(ctypes.Structure):
@@ -145,10 +147,12 @@ def lib():
     L.asymspec_fuse_verify_host.restype = _I
     L.asymspec_draft_sample.argtypes = [_P, _I, _I, _I, _I, _P, _P, _P, _I, _P]
     L.asymspec_draft_sample.restype = _I
-    L.asymspec_xvocab_workspace_bytes.argtypes = [_I, _I, _I, _I]
+    L.asymspec_xvocab_gather_scratch_bytes.argtypes = [_I, _I]
+    L.asymspec_xvocab_gather_scratch_bytes.restype = ctypes.c_size_t
+    L.asymspec_xvocab_workspace_bytes.argtypes = [_I, _I, _I, _I, _I, _I]
     L.asymspec_xvocab_workspace_bytes.restype = ctypes.c_size_t
     L.asymspec_xvocab_gather.argtypes = [_P, _P, _I, _P, _I, _P, _P, _I, _I, _I, _P, _P, _P,
-                                         _P, _P]
+                                         _P, _P, ctypes.c_size_t, _P]
     L.asymspec_xvocab_gather.restype = _I
     L.asymspec_fuse_verify_xvocab.argtypes = [_P, _P, _I, _P, _I, _P, _P, _I, _P, _P, _P, _I,
                                               _I, _I, ctypes.POINTER(GateParams), _P, _P, _P,
@@ -251,16 +255,21 @@ def draft_sample(logits, rows, V, dtype, mode, uniforms, out_tokens, out_probs, 
                                        out_probs, cluster_size, stream)
 
 
-def xvocab_workspace_bytes(B, K, S, dtype) -> int:
-    return int(lib().asymspec_xvocab_workspace_bytes(B, K, S, dtype))
+def xvocab_gather_scratch_bytes(V_d, V_v) -> int:
+    return int(lib().asymspec_xvocab_gather_scratch_bytes(V_d, V_v))
+
+
+def xvocab_workspace_bytes(B, K, S, V_d, V_v, dtype) -> int:
+    return int(lib().asymspec_xvocab_workspace_bytes(B, K, S, V_d, V_v, dtype))
 
 
 def xvocab_gather(logits_full, logits_comp, V_d, logits_ver, V_v, map_d, map_v, S, rows, dtype,
-                  out_full, out_comp, out_ver, out_error_word=None, stream=0) -> int:
+                  out_full, out_comp, out_ver, out_error_word=None, scratch=None,
+                  scratch_nbytes=0, stream=0) -> int:
     """asymspec_xvocab_gather with device addresses (ints); returns the status."""
     return lib().asymspec_xvocab_gather(logits_full, logits_comp, V_d, logits_ver, V_v, map_d,
                                         map_v, S, rows, dtype, out_full, out_comp, out_ver,
-                                        out_error_word, stream)
+                                        out_error_word, scratch, scratch_nbytes, stream)
 
 
 def fuse_verify_xvocab(logits_full, logits_comp, V_d, logits_ver, V_v, map_d, map_v, S,

@@ -75,12 +75,12 @@ bool plan_generic(int V, int elt, int VE, int forced_C, Plan* pl) {
 // TMA kernel: first C whose slice (and shared state) fits two CTAs per SM,
 // else the first that fits one; a slice holds at most kMaxRounds vectors
 // per thread.
-bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
+bool plan_tma(int V, int elt, int forced_C, Plan* pl, bool persistent = false) {
   const int VE = 16 / elt;
   auto fill = [&](int C) {
     const long long per = (static_cast<long long>(V) + C - 1) / C;
     const long long W = round_up_ll(per, VE);
-    const int shared_bytes = shared_tma_bytes(C);
+    const int shared_bytes = shared_tma_bytes(C, persistent);
     const long long sh_off = round_up_ll(3 * W * elt, 128);
     pl->C = C;
     pl->W = static_cast<int>(W);
@@ -203,7 +203,7 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
   if (forced_C < 0 || forced_C > 16) return ASYMSPEC_ERR_INVALID_ARG;
   if (forced_kernel != 0 && forced_kernel != ASYMSPEC_KERNEL_GENERIC &&
       forced_kernel != ASYMSPEC_KERNEL_TMA && forced_kernel != ASYMSPEC_KERNEL_STREAM &&
-      forced_kernel != ASYMSPEC_KERNEL_RING)
+      forced_kernel != ASYMSPEC_KERNEL_RING && forced_kernel != ASYMSPEC_KERNEL_PERSIST)
     return ASYMSPEC_ERR_INVALID_ARG;
   pl->rows = static_cast<long long>(B) * (K + 1);
   pl->vector_path = vec_ok;
@@ -245,6 +245,16 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
                  : ASYMSPEC_ERR_TOO_LARGE;
     }
   }
+  if (forced_kernel == ASYMSPEC_KERNEL_PERSIST) {
+    // the persistent form of the cluster kernel: same slices, on request
+    if (!vec_ok) return ASYMSPEC_ERR_UNSUPPORTED;
+    if (!plan_tma(V, elt, forced_C, pl, true)) return ASYMSPEC_ERR_TOO_LARGE;
+    if (ws_bytes < tma_layout(B, K, pl->C).total) return ASYMSPEC_ERR_WORKSPACE;
+    pl->kernel = ASYMSPEC_KERNEL_PERSIST;
+    pl->VE = 16 / elt;
+    pl->ctas = 0;  // set at launch from the device's cluster occupancy
+    return ASYMSPEC_OK;
+  }
   bool ok = false;
   if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, pl)) {
     // the TMA kernel leaves each row's results in the workspace; the generic
@@ -278,6 +288,8 @@ KernelFn pick_kernel(const Plan& pl, int dtype, bool stoch, int sel = 0) {
   if (pl.kernel == ASYMSPEC_KERNEL_RING) return pick_ring(dtype, stoch);
   if (pl.kernel == ASYMSPEC_KERNEL_TMA)
     return dtype == ASYMSPEC_FP32 ? tma_kernel_f32(stoch, sel) : tma_kernel_bf16(stoch, sel);
+  if (pl.kernel == ASYMSPEC_KERNEL_PERSIST)
+    return dtype == ASYMSPEC_FP32 ? tmap_kernel_f32(stoch, sel) : tmap_kernel_bf16(stoch, sel);
   return generic_kernel(dtype, pl.vector_path, stoch);
 }
 
@@ -646,11 +658,11 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
                               tma_program_set(st_mode, gp.divergence, gp.fuse_bonus != 0, false,
                                               false, gp.flags & ASYMSPEC_FLAG_DELTA_MASK));
     int ncl = 0;
-    if (prepare_kernel(fn, device) == cudaSuccess &&
+    if (fn && prepare_kernel(fn, device) == cudaSuccess &&
         active_clusters(fn, pl, device, &ncl) == cudaSuccess)
       out->max_active_clusters = ncl;
-    // the persistent kernel launches the clusters the device holds, at most one per row
-    if (pl.kernel == ASYMSPEC_KERNEL_RING)
+    // the persistent kernels launch the clusters the device holds, at most one per row
+    if (pl.kernel == ASYMSPEC_KERNEL_RING || pl.kernel == ASYMSPEC_KERNEL_PERSIST)
       out->ctas = std::min(static_cast<long long>(ncl), pl.rows) * pl.C;
   }
   cudaGetLastError();
@@ -795,12 +807,15 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   KernelFn fn = pick_kernel(pl, dtype, stoch,
                             tma_program_set(stoch, gp.divergence, gp.fuse_bonus != 0, P.full != 0,
                                             P.want_tokens != 0, P.delta_src));
+  // the persistent kernel exists for the production program sets only (no
+  // debug outputs, no per-row tokens in stochastic mode, delta = a - b)
+  if (!fn) return ASYMSPEC_ERR_UNSUPPORTED;
   e = prepare_kernel(fn, device);
   if (e != cudaSuccess) return cuda_fail(e);
   // The one-shot kernels launch one cluster per row; the persistent ring
   // kernel as many clusters as the device holds at once (at most one per row).
   long long ctas = pl.ctas;
-  if (pl.kernel == ASYMSPEC_KERNEL_RING) {
+  if (pl.kernel == ASYMSPEC_KERNEL_RING || pl.kernel == ASYMSPEC_KERNEL_PERSIST) {
     int ncl = 0;
     e = active_clusters(fn, pl, device, &ncl);
     if (e != cudaSuccess) return cuda_fail(e);
@@ -811,7 +826,8 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   cudaLaunchConfig_t cfg = launch_config(pl, ctas, static_cast<cudaStream_t>(stream), attr);
   void* args[] = {&P};
   P.group_stride = pl.group_stride;
-  if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING) {
+  if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING ||
+      pl.kernel == ASYMSPEC_KERNEL_PERSIST) {
     const TmaLayout L = tma_layout(B, K, pl.C, pl.group_stride);
     char* base = static_cast<char*>(workspace);
     P.row_stat = base + L.stat;
@@ -822,11 +838,23 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   if (e == cudaSuccess) e = cudaLaunchKernelExC(&cfg, fn, args);
   if (e == cudaSuccess) e = record_timing(opts, false, cfg.stream);
   if (e != cudaSuccess) return cuda_fail(e);
-  if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING) {
+  if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING ||
+      pl.kernel == ASYMSPEC_KERNEL_PERSIST) {
     // the rows' decisions and Algorithm 1's scan: one CTA per batch element
+    // as a programmatic dependent launch: its launch overlaps the row
+    // kernel's last CTAs, and it waits (griddepcontrol.wait) for that kernel
     const int warps = std::min(K + 1, kDecideThreads / 32);
-    e = cudaLaunchKernel(pick_decide(dtype, stoch), dim3(static_cast<unsigned>(B)),
-                         dim3(32 * warps), args, 0, static_cast<cudaStream_t>(stream));
+    cudaLaunchConfig_t dcfg = {};
+    cudaLaunchAttribute dattr[1];
+    dattr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    dattr[0].val.programmaticStreamSerializationAllowed = 1;
+    dcfg.gridDim = dim3(static_cast<unsigned>(B));
+    dcfg.blockDim = dim3(32 * warps);
+    dcfg.dynamicSmemBytes = 0;
+    dcfg.stream = static_cast<cudaStream_t>(stream);
+    dcfg.attrs = dattr;
+    dcfg.numAttrs = 1;
+    e = cudaLaunchKernelExC(&dcfg, pick_decide(dtype, stoch), args);
     if (e != cudaSuccess) return cuda_fail(e);
   }
   return ASYMSPEC_OK;
@@ -1051,21 +1079,39 @@ int asymspec_draft_sample(const void* logits, int rows, int V, int dtype, int mo
 
 namespace {
 
-// Workspace of asymspec_fuse_verify_xvocab, each part 256-byte aligned: the
-// restricted rows a', b', t' ([B, K+1, S] each), the emitted pair indices
-// ([B] int32), then the step's own workspace for a vocabulary of S entries.
-struct XLayout {
-  size_t ga, gb, gt, idx, step, step_bytes, total;
+// Scratch of asymspec_xvocab_gather, each part 256-byte aligned: inv_d[V_d],
+// inv_v[V_v] (int32) and the map-error word.
+struct XScratch {
+  size_t inv_d, inv_v, err, total;
 };
 
-XLayout xvocab_layout(int B, int K, int S, int dtype) {
+XScratch xvocab_scratch_layout(int V_d, int V_v) {
+  XScratch L;
+  L.inv_d = 0;
+  L.inv_v = round_up(static_cast<size_t>(V_d) * sizeof(int32_t), 256);
+  L.err = L.inv_v + round_up(static_cast<size_t>(V_v) * sizeof(int32_t), 256);
+  L.total = L.err + 256;
+  return L;
+}
+
+// Workspace of asymspec_fuse_verify_xvocab, each part 256-byte aligned: the
+// restricted rows a', b', t' ([B, K+1, S] each), the emitted pair indices
+// ([B] int32), the gather's scratch, then the step's own workspace for a
+// vocabulary of S entries.
+struct XLayout {
+  size_t ga, gb, gt, idx, scratch, scratch_bytes, step, step_bytes, total;
+};
+
+XLayout xvocab_layout(int B, int K, int S, int V_d, int V_v, int dtype) {
   XLayout L;
   const size_t plane = round_up(static_cast<size_t>(B) * (K + 1) * S * elt_size(dtype), 256);
   L.ga = 0;
   L.gb = plane;
   L.gt = 2 * plane;
   L.idx = 3 * plane;
-  L.step = L.idx + round_up(static_cast<size_t>(B) * sizeof(int32_t), 256);
+  L.scratch = L.idx + round_up(static_cast<size_t>(B) * sizeof(int32_t), 256);
+  L.scratch_bytes = xvocab_scratch_layout(V_d, V_v).total;
+  L.step = L.scratch + L.scratch_bytes;
   L.step_bytes = asymspec_workspace_bytes(B, K, S);
   L.total = L.step + L.step_bytes;
   return L;
@@ -1075,17 +1121,22 @@ XLayout xvocab_layout(int B, int K, int S, int dtype) {
 
 extern "C" {
 
-size_t asymspec_xvocab_workspace_bytes(int B, int K, int S, int dtype) {
-  if (B < 1 || K < 1 || S < 2) return 0;
+size_t asymspec_xvocab_gather_scratch_bytes(int V_d, int V_v) {
+  if (V_d < 1 || V_v < 1) return 0;
+  return xvocab_scratch_layout(V_d, V_v).total;
+}
+
+size_t asymspec_xvocab_workspace_bytes(int B, int K, int S, int V_d, int V_v, int dtype) {
+  if (B < 1 || K < 1 || S < 2 || V_d < 1 || V_v < 1) return 0;
   if (dtype != ASYMSPEC_FP32 && dtype != ASYMSPEC_BF16) return 0;
-  return xvocab_layout(B, K, S, dtype).total;
+  return xvocab_layout(B, K, S, V_d, V_v, dtype).total;
 }
 
 int asymspec_xvocab_gather(const void* logits_full, const void* logits_comp, int V_d,
                            const void* logits_ver, int V_v, const int32_t* map_d,
                            const int32_t* map_v, int S, int rows, int dtype, void* out_full,
                            void* out_comp, void* out_ver, uint32_t* out_error_word,
-                           void* stream) {
+                           void* scratch, size_t scratch_bytes, void* stream) {
   if (dtype != ASYMSPEC_FP32 && dtype != ASYMSPEC_BF16) return ASYMSPEC_ERR_UNSUPPORTED;
   if (rows < 0 || S < 2 || V_d < 1 || V_v < 1) return ASYMSPEC_ERR_INVALID_ARG;
   if (rows == 0) return ASYMSPEC_OK;
@@ -1097,8 +1148,30 @@ int asymspec_xvocab_gather(const void* logits_full, const void* logits_comp, int
       !aligned(out_full, elt) || !aligned(out_comp, elt) || !aligned(out_ver, elt) ||
       !aligned(map_d, 4) || !aligned(map_v, 4) || (out_error_word && !aligned(out_error_word, 4)))
     return ASYMSPEC_ERR_MISALIGNED;
+  const XScratch XL = xvocab_scratch_layout(V_d, V_v);
+  if (scratch && (!aligned(scratch, 256) || scratch_bytes < XL.total)) return ASYMSPEC_ERR_WORKSPACE;
   const long long ycount = (static_cast<long long>(rows) + kXRows - 1) / kXRows;
   if (ycount > 65535) return ASYMSPEC_ERR_TOO_LARGE;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaSuccess;
+  if (scratch) {
+    // the map check: inverse maps built with atomicCAS, the map-error word
+    char* base = static_cast<char*>(scratch);
+    int* inv_d = reinterpret_cast<int*>(base + XL.inv_d);
+    int* inv_v = reinterpret_cast<int*>(base + XL.inv_v);
+    unsigned* merr = reinterpret_cast<unsigned*>(base + XL.err);
+    int Vd = V_d, Vv = V_v, S_ = S;
+    void* fargs[] = {&inv_d, &Vd, &inv_v, &Vv, &merr};
+    const int vmax = std::max(V_d, V_v);
+    e = cudaLaunchKernel(xvocab_inv_fill_ptr(), dim3((vmax + 255) / 256), dim3(256), fargs, 0, st);
+    if (e != cudaSuccess) return cuda_fail(e);
+    const int32_t* md = map_d;
+    const int32_t* mv = map_v;
+    uint32_t* ew = out_error_word;
+    void* bargs[] = {&md, &mv, &S_, &inv_d, &Vd, &inv_v, &Vv, &merr, &ew};
+    e = cudaLaunchKernel(xvocab_inv_build_ptr(), dim3((S + 255) / 256), dim3(256), bargs, 0, st);
+    if (e != cudaSuccess) return cuda_fail(e);
+  }
   XGatherParams P;
   P.a = logits_full;
   P.b = logits_comp;
@@ -1116,8 +1189,7 @@ int asymspec_xvocab_gather(const void* logits_full, const void* logits_comp, int
   const dim3 grid(static_cast<unsigned>((S + kXThreads * kXJ - 1) / (kXThreads * kXJ)),
                   static_cast<unsigned>(ycount));
   void* args[] = {&P};
-  const cudaError_t e = cudaLaunchKernel(xvocab_gather_ptr(dtype), grid, dim3(kXThreads), args,
-                                         0, static_cast<cudaStream_t>(stream));
+  e = cudaLaunchKernel(xvocab_gather_ptr(dtype), grid, dim3(kXThreads), args, 0, st);
   return e == cudaSuccess ? ASYMSPEC_OK : cuda_fail(e);
 }
 
@@ -1139,15 +1211,16 @@ int asymspec_fuse_verify_xvocab(const void* logits_full, const void* logits_comp
   if (!draft_index || !out_accept_len || !out_next_token) return ASYMSPEC_ERR_INVALID_ARG;
   if (gp.mode == ASYMSPEC_MODE_STOCHASTIC && (!draft_probs || !uniforms))
     return ASYMSPEC_ERR_INVALID_ARG;
-  if (!aligned(out_next_token, 4) || (out_next_index && !aligned(out_next_index, 4)))
+  if (!aligned(out_next_token, 4) || !aligned(out_accept_len, 4) ||
+      (out_next_index && !aligned(out_next_index, 4)))
     return ASYMSPEC_ERR_MISALIGNED;
-  const XLayout L = xvocab_layout(B, K, S, dtype);
-  if (!workspace || !aligned(workspace, 16) || workspace_bytes < L.total)
+  const XLayout L = xvocab_layout(B, K, S, V_d, V_v, dtype);
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < L.total)
     return ASYMSPEC_ERR_WORKSPACE;
   char* base = static_cast<char*>(workspace);
   st = asymspec_xvocab_gather(logits_full, logits_comp, V_d, logits_ver, V_v, map_d, map_v, S,
                               B * (K + 1), dtype, base + L.ga, base + L.gb, base + L.gt,
-                              out_error_word, stream);
+                              out_error_word, base + L.scratch, L.scratch_bytes, stream);
   if (st) return st;
   int32_t* idx = out_next_index ? out_next_index : reinterpret_cast<int32_t*>(base + L.idx);
   st = asymspec_fuse_verify_ex(base + L.ga, base + L.gb, base + L.gt, draft_index, draft_probs,
@@ -1156,9 +1229,12 @@ int asymspec_fuse_verify_xvocab(const void* logits_full, const void* logits_comp
                                out_error_word, nullptr, stream);
   if (st) return st;
   int32_t* next = out_next_token;
+  int32_t* len = out_accept_len;
   const int32_t* mv = map_v;
+  const unsigned* merr =
+      reinterpret_cast<const unsigned*>(base + L.scratch + xvocab_scratch_layout(V_d, V_v).err);
   int S_ = S, B_ = B;
-  void* args[] = {&idx, &mv, &S_, &B_, &next};
+  void* args[] = {&idx, &mv, &S_, &B_, &merr, &len, &next};
   const cudaError_t e = cudaLaunchKernel(xvocab_emit_ptr(), dim3((B + 255) / 256), dim3(256),
                                          args, 0, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? ASYMSPEC_OK : cuda_fail(e);

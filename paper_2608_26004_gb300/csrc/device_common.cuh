@@ -381,6 +381,12 @@ __device__ __forceinline__ void mbar_arrive_remote(unsigned long long* bar, unsi
                : "memory");
 }
 
+// Orders this thread's earlier generic-proxy accesses to shared memory before
+// later async-proxy ones (a bulk copy into a buffer that was just read).
+__device__ __forceinline__ void fence_proxy_async_shared() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // 1-D bulk copy global -> this CTA's shared memory, completing on `bar`.
 __device__ __forceinline__ void bulk_load(void* dst, const void* src, unsigned bytes,
                                           unsigned long long* bar) {

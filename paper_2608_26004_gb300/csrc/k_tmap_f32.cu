@@ -1,0 +1,29 @@
+// The production program sets 1..6 of the persistent cluster kernel,
+// fuse_verify_tma<T, STOCH, SEL, true>, for float logits (see kernel_tma.cuh).
+// There is no persistent form of program set 0 (run-time dispatch).
+#include "kernel_tma.cuh"
+#include "kernels.h"
+
+namespace asymspec_impl {
+
+const void* tmap_kernel_f32(bool stoch, int sel) {
+  if (sel <= 0 || sel >= kTmaProgramSets || (stoch && sel > 3)) return nullptr;
+  if (stoch) {
+    switch (sel) {
+      case 1: return reinterpret_cast<const void*>(&fuse_verify_tma<float, true, 1, true>);
+      case 2: return reinterpret_cast<const void*>(&fuse_verify_tma<float, true, 2, true>);
+      case 3: return reinterpret_cast<const void*>(&fuse_verify_tma<float, true, 3, true>);
+    }
+  }
+  switch (sel) {
+    case 1: return reinterpret_cast<const void*>(&fuse_verify_tma<float, false, 1, true>);
+    case 2: return reinterpret_cast<const void*>(&fuse_verify_tma<float, false, 2, true>);
+    case 3: return reinterpret_cast<const void*>(&fuse_verify_tma<float, false, 3, true>);
+    case 4: return reinterpret_cast<const void*>(&fuse_verify_tma<float, false, 4, true>);
+    case 5: return reinterpret_cast<const void*>(&fuse_verify_tma<float, false, 5, true>);
+    case 6: return reinterpret_cast<const void*>(&fuse_verify_tma<float, false, 6, true>);
+  }
+  return nullptr;
+}
+
+}  // namespace asymspec_impl

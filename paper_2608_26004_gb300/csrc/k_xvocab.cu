@@ -11,4 +11,8 @@ const void* xvocab_gather_ptr(int dtype) {
 
 const void* xvocab_emit_ptr() { return reinterpret_cast<const void*>(&xvocab_emit<int32_t>); }
 
+const void* xvocab_inv_fill_ptr() { return reinterpret_cast<const void*>(&xvocab_inv_fill<int>); }
+
+const void* xvocab_inv_build_ptr() { return reinterpret_cast<const void*>(&xvocab_inv_build<int>); }
+
 }  // namespace asymspec_impl

@@ -78,14 +78,14 @@ struct __align__(16) X2 {  // pass-2 sums
 // cluster follow it (recv1()).
 struct __align__(16) SharedTma {
   unsigned long long bar[kChunks];  // one mbarrier per chunk
-  union {                           // per-warp records, one pass at a time
-    X1 w1[kTWarps];
-    X2 w2[kTWarps];
-  };
+  X1 w1[kTWarps];                   // per-warp pass-1 records
+  X2 w2[kTWarps];                   // per-warp pass-2 records
   float lse[4];       // the row's normalisers (pass 2 reads them)
   unsigned broken;    // a chunk copy timed out
+  int rel[kChunks];   // persistent kernel: warps done with each chunk of the row
   unsigned pad[3];
-  __device__ X1* recv1() { return reinterpret_cast<X1*>(this + 1); }
+  // slot s (0, or the row's parity in the persistent kernel) of the C pushed records
+  __device__ X1* recv1(int slot = 0, int C = 0) { return reinterpret_cast<X1*>(this + 1) + slot * C; }
 };
 
 // The pushed records are copied with 16-byte stores.
@@ -97,9 +97,10 @@ static_assert(sizeof(SharedTma) % 16 == 0, "records after SharedTma must stay 16
 // in round g / 8, i.e. vectors [32 g, 32 g + 32) in index order.
 constexpr int kGroupsMax = kMaxRounds * kTWarps;
 
-// Shared bytes after the slices for a cluster of C CTAs.
-__host__ __device__ constexpr int shared_tma_bytes(int C) {
-  return static_cast<int>(sizeof(SharedTma) + C * sizeof(X1));
+// Shared bytes after the slices for a cluster of C CTAs (the persistent
+// kernel keeps two slots of pushed records, by row parity).
+__host__ __device__ constexpr int shared_tma_bytes(int C, bool persistent = false) {
+  return static_cast<int>(sizeof(SharedTma) + (persistent ? 2 : 1) * C * sizeof(X1));
 }
 
 __device__ __forceinline__ X1 x1_neutral() {
@@ -320,14 +321,24 @@ __device__ __forceinline__ f2 fuse2(f2 beta2, f2 a, f2 b, f2 t) {
 template <int NP, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void vec_masses(const f2 (&xa)[NP], const f2 (&xb)[NP],
                                            const f2 (&xt)[NP], f2 beta2, f2 L2, f2 nA2, f2 nS2,
-                                           f2 (&p)[NP], f2 (&qf)[NP], f2 (&r)[NP]) {
+                                           f2 (&p)[NP], f2 (&qf)[NP], f2 (&r)[NP],
+                                           f2 (&la2)[NP]) {
 #pragma unroll
   for (int h = 0; h < NP; ++h) {
-    p[h] = ex2_2(fma2(xa[h], L2, nA2));
+    la2[h] = fma2(xa[h], L2, nA2);  // log2 softmax(a), which the divergence terms reuse
+    p[h] = ex2_2(la2[h]);
     const f2 s = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
     qf[h] = ex2_2(fma2(s, L2, nS2));
     r[h] = relu2(sub2(qf[h], p[h]));
   }
+}
+
+template <int NP, int DS = ASYMSPEC_DELTA_AB>
+__device__ __forceinline__ void vec_masses(const f2 (&xa)[NP], const f2 (&xb)[NP],
+                                           const f2 (&xt)[NP], f2 beta2, f2 L2, f2 nA2, f2 nS2,
+                                           f2 (&p)[NP], f2 (&qf)[NP], f2 (&r)[NP]) {
+  f2 la2[NP];
+  vec_masses<NP, DS>(xa, xb, xt, beta2, L2, nA2, nS2, p, qf, r, la2);
 }
 
 template <int NP>
@@ -381,7 +392,8 @@ __device__ __forceinline__ void load_or_fill(const T* p, bool ok, f2 (&x)[NP]) {
 // it is in global memory and sh is not used).
 template <typename T, unsigned F, bool WAIT = true, int DS = ASYMSPEC_DELTA_AB>
 __device__ __noinline__ void pass1_online(const T* ra, const T* rb, const T* rt, int nv, int rounds,
-                                      int rc, int lo, float beta, SharedTma* sh, X1& e) {
+                                      int rc, int lo, float beta, SharedTma* sh, X1& e,
+                                      unsigned ph = 0) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
   constexpr bool needA = (F & (F_LA | F_LS | F_AS)) != 0;
@@ -395,7 +407,7 @@ __device__ __noinline__ void pass1_online(const T* ra, const T* rb, const T* rt,
   int vec_s = -1, vec_t = -1;  // vectors holding the best s and t so far
   const int tid = static_cast<int>(threadIdx.x);
   for (int c = 0, r0 = 0; c < kChunks && r0 < rounds; ++c, r0 += rc) {
-    if (WAIT && !sh->broken && !mbar_wait_bounded(&sh->bar[c], 0, kCopyTimeoutNs))
+    if (WAIT && !sh->broken && !mbar_wait_bounded(&sh->bar[c], ph, kCopyTimeoutNs))
       atomicOr(&sh->broken, kBadTimeout);
     const int r1 = min(rounds, r0 + rc);
     int i0 = r0 * kTThreads + tid;          // vector index of this thread's first vector
@@ -500,7 +512,7 @@ __device__ __forceinline__ void fixed_pairs2(f2& acc, const f2 (&x)[NP], const f
 template <typename T, unsigned F, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt, int nv,
                                            int rounds, int rc, int lo, float beta, SharedTma* sh,
-                                           X1& e) {
+                                           X1& e, unsigned ph = 0) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
   constexpr bool needA = (F & (F_LA | F_LS | F_AS)) != 0;
@@ -512,7 +524,7 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
   const f2 L2 = pk(kLog2e, kLog2e);
   const int tid = static_cast<int>(threadIdx.x);
   // chunk 0 holds every thread's first vector
-  if (!sh->broken && !mbar_wait_bounded(&sh->bar[0], 0, kCopyTimeoutNs))
+  if (!sh->broken && !mbar_wait_bounded(&sh->bar[0], ph, kCopyTimeoutNs))
     atomicOr(&sh->broken, kBadTimeout);
   float ref[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
   if (tid < nv) {
@@ -544,7 +556,7 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
   f2 acc[4] = {0ull, 0ull, 0ull, 0ull};
   int vec_s = -1, vec_t = -1;  // vectors holding the best s and t so far
   for (int c = 0, r0 = 0; c < kChunks && r0 < rounds; ++c, r0 += rc) {
-    if (c > 0 && !sh->broken && !mbar_wait_bounded(&sh->bar[c], 0, kCopyTimeoutNs))
+    if (c > 0 && !sh->broken && !mbar_wait_bounded(&sh->bar[c], ph, kCopyTimeoutNs))
       atomicOr(&sh->broken, kBadTimeout);
     const int r1 = min(rounds, r0 + rc);
     int i0 = r0 * kTThreads + tid;          // vector index of this thread's first vector
@@ -624,17 +636,18 @@ template <typename T, unsigned F, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void pass1_and_push(const T* ra, const T* rb, const T* rt, int nv,
                                                int rounds, int rc, int lo, int n, float beta,
                                                int dtok, SharedTma* sh, int rank, int C,
-                                               cg::cluster_group& cluster) {
+                                               cg::cluster_group& cluster, unsigned ph = 0,
+                                               int slot = 0) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   X1 e = x1_neutral();
-  const bool ovf = pass1_fast<T, F, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
+  const bool ovf = pass1_fast<T, F, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e, ph);
   warp_reduce_x1_uniform<F>(e);  // the warp's references are equal
   if (lane == 0) sh->w1[warp] = e;
   if (__syncthreads_or(ovf)) {
     // an entry far above its thread's reference (or non-finite data): redo
     // the slice with a running maximum
     e = x1_neutral();
-    pass1_online<T, F, true, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
+    pass1_online<T, F, true, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e, ph);
     warp_reduce_x1<F>(e);
     if (lane == 0) sh->w1[warp] = e;
     __syncthreads();
@@ -648,7 +661,7 @@ __device__ __forceinline__ void pass1_and_push(const T* ra, const T* rb, const T
       w.db = to_f32(rb[dtok - lo]);
       w.dt = to_f32(rt[dtok - lo]);
     }
-    push_record(w, sh->recv1(), rank, C, cluster);
+    push_record(w, sh->recv1(slot, C), rank, C, cluster);
   }
   cluster_barrier(warp == 0);  // B1: every CTA's pass-1 record is in every CTA
 }
@@ -657,37 +670,68 @@ __device__ __forceinline__ void pass1_and_push(const T* ra, const T* rb, const T
 // kChunks chunks, each completing on its own mbarrier.  only_t: copy t alone
 // (a greedy bonus row without fused bonus needs nothing else).
 template <typename T>
+__device__ __forceinline__ void issue_chunk(const KParams& P, SharedTma* sh, long long row,
+                                            int lo, int nv, int rc, T* sa, T* sb, T* st,
+                                            bool only_t, int c) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  const size_t off = static_cast<size_t>(row) * P.V + lo;
+  const int v0 = min(nv, c * rc * kTThreads);
+  const int v1 = min(nv, (c + 1) * rc * kTThreads);
+  const unsigned bytes = static_cast<unsigned>(v1 - v0) * 16u;
+  mbar_arrive_expect_tx(&sh->bar[c], bytes * (only_t ? 1u : 3u));
+  if (bytes) {
+    const int e0 = v0 * VE;
+    if (!only_t) {
+      bulk_load(sa + e0, static_cast<const T*>(P.a) + off + e0, bytes, &sh->bar[c]);
+      bulk_load(sb + e0, static_cast<const T*>(P.b) + off + e0, bytes, &sh->bar[c]);
+    }
+    bulk_load(st + e0, static_cast<const T*>(P.t) + off + e0, bytes, &sh->bar[c]);
+  }
+}
+template <typename T>
 __device__ __forceinline__ void issue_slice(const KParams& P, SharedTma* sh, long long row,
                                             int lo, int nv, int rc, T* sa, T* sb, T* st,
                                             bool only_t) {
-  constexpr int VE = 16 / static_cast<int>(sizeof(T));
-  const size_t off = static_cast<size_t>(row) * P.V + lo;
-  const T* ga = static_cast<const T*>(P.a) + off;
-  const T* gb = static_cast<const T*>(P.b) + off;
-  const T* gt = static_cast<const T*>(P.t) + off;
 #pragma unroll
-  for (int c = 0; c < kChunks; ++c) {
-    const int v0 = min(nv, c * rc * kTThreads);
-    const int v1 = min(nv, (c + 1) * rc * kTThreads);
-    const unsigned bytes = static_cast<unsigned>(v1 - v0) * 16u;
-    mbar_arrive_expect_tx(&sh->bar[c], bytes * (only_t ? 1u : 3u));
-    if (bytes) {
-      const int e0 = v0 * VE;
-      if (!only_t) {
-        bulk_load(sa + e0, ga + e0, bytes, &sh->bar[c]);
-        bulk_load(sb + e0, gb + e0, bytes, &sh->bar[c]);
-      }
-      bulk_load(st + e0, gt + e0, bytes, &sh->bar[c]);
-    }
-  }
+  for (int c = 0; c < kChunks; ++c) issue_chunk<T>(P, sh, row, lo, nv, rc, sa, sb, st, only_t, c);
 }
+
+// Persistent kernel: once all kTWarps warps have read chunk c of the slice
+// in pass 2, the last of them copies chunk c of the cluster's next row into
+// it (mbarrier c completes once per row, so the waits take the row's parity).
+template <typename T>
+struct ChunkRefill {
+  static constexpr bool kActive = true;
+  int rc;
+  const KParams* P;
+  SharedTma* sh;
+  long long next;  // the next row, or -1
+  int lo, nv;
+  T* sa;
+  T* sb;
+  T* st;
+  bool only_t;
+  __device__ __forceinline__ void operator()(int c) const {
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) {
+      __threadfence_block();  // this warp's reads of the chunk come first
+      if (atomicAdd(&sh->rel[c], 1) == kTWarps - 1) {
+        sh->rel[c] = 0;
+        __threadfence_block();
+        fence_proxy_async_shared();
+        if (next >= 0 && !sh->broken) issue_chunk<T>(*P, sh, next, lo, nv, rc, sa, sb, st, only_t, c);
+      }
+    }
+    __syncwarp();
+  }
+};
 
 // After B1, in one warp: the row values from the C pushed records (every
 // lane ends with them).  lse[q] = ln of stream q's normaliser.
 template <unsigned F>
-__device__ __forceinline__ X1 combine_pass1(SharedTma* sh, int C, float (&lse)[4]) {
+__device__ __forceinline__ X1 combine_pass1(SharedTma* sh, int C, float (&lse)[4], int slot = 0) {
   const int lane = threadIdx.x & 31;
-  X1 w = (lane < C) ? sh->recv1()[lane] : x1_neutral();
+  X1 w = (lane < C) ? sh->recv1(slot, C)[lane] : x1_neutral();
   warp_reduce_x1<F>(w);
 #pragma unroll
   for (int q = 0; q < 4; ++q) lse[q] = w.ref[q] + logf(w.s[q]);
@@ -696,10 +740,10 @@ __device__ __forceinline__ X1 combine_pass1(SharedTma* sh, int C, float (&lse)[4
 
 // The draft token's a, b, t (from the record of the CTA whose slice holds it).
 __device__ __forceinline__ void draft_logits(SharedTma* sh, int dtok, int W, int C, float& ad,
-                                             float& bd, float& td) {
+                                             float& bd, float& td, int slot = 0) {
   ad = bd = td = 0.f;
   if (dtok >= 0 && W > 0) {
-    const X1& o = sh->recv1()[dtok / W < C ? dtok / W : 0];
+    const X1& o = sh->recv1(slot, C)[dtok / W < C ? dtok / W : 0];
     ad = o.da;
     bd = o.db;
     td = o.dt;
@@ -709,14 +753,14 @@ __device__ __forceinline__ void draft_logits(SharedTma* sh, int dtok, int W, int
 // ---------------------------------------------------------------- pass 2
 
 // Divergence terms of one vector (Eq. 3): JSD terms p (log2 p - log2 m) and
-// q (log2 q - log2 m) with m = p + q, their mass m, or KL terms.
+// q (log2 q - log2 m) with m = p + q, their mass m, or KL terms; la: log2 p.
 template <int NP, bool JSD, bool KL>
-__device__ __forceinline__ void div_terms(const f2 (&xa)[NP], const f2 (&xb)[NP], const f2 (&p)[NP],
-                                          f2 L2, f2 nA2, f2 nB2, f2 tiny2, f2& ja, f2& jb,
+__device__ __forceinline__ void div_terms(const f2 (&la)[NP], const f2 (&xb)[NP], const f2 (&p)[NP],
+                                          f2 L2, f2 nB2, f2 tiny2, f2& ja, f2& jb,
                                           f2& ms2, f2& kl2) {
 #pragma unroll
   for (int h = 0; h < NP; ++h) {
-    const f2 la2 = fma2(xa[h], L2, nA2);
+    const f2 la2 = la[h];
     const f2 lb2 = fma2(xb[h], L2, nB2);
     if (JSD) {
       const f2 q = ex2_2(lb2);
@@ -728,6 +772,17 @@ __device__ __forceinline__ void div_terms(const f2 (&xa)[NP], const f2 (&xb)[NP]
     }
     if (KL) kl2 = fma2(p[h], sub2(la2, lb2), kl2);
   }
+}
+
+// As above from the logits a (log2 p = a log2 e - nA2).
+template <int NP, bool JSD, bool KL>
+__device__ __forceinline__ void div_terms(const f2 (&xa)[NP], const f2 (&xb)[NP], const f2 (&p)[NP],
+                                          f2 L2, f2 nA2, f2 nB2, f2 tiny2, f2& ja, f2& jb,
+                                          f2& ms2, f2& kl2) {
+  f2 la[NP];
+#pragma unroll
+  for (int h = 0; h < NP; ++h) la[h] = fma2(xa[h], L2, nA2);
+  div_terms<NP, JSD, KL>(la, xb, p, L2, nB2, tiny2, ja, jb, ms2, kl2);
 }
 
 // Pass-2 constants and running sums of one thread.
@@ -761,11 +816,11 @@ __device__ __forceinline__ void p2_pair(const f2 (&xa)[NP], const f2 (&xb)[NP], 
                                         float& g1, float* lpx, float* lpy) {
   constexpr bool JSD = (G & G_JSD) != 0, KL = (G & G_KL) != 0, RES = (G & G_RES) != 0;
   constexpr bool QF = (G & G_QF) != 0;
-  f2 px[NP], py[NP];
+  f2 px[NP], py[NP], lax[NP], lay[NP];
   if (RES) {
     f2 qx[NP], qy[NP], rx[NP], ry[NP];
-    vec_masses<NP, DS>(xa, xb, xt, k.beta2, k.L2, k.nA2, k.nS2, px, qx, rx);
-    vec_masses<NP, DS>(ya, yb, yt, k.beta2, k.L2, k.nA2, k.nS2, py, qy, ry);
+    vec_masses<NP, DS>(xa, xb, xt, k.beta2, k.L2, k.nA2, k.nS2, px, qx, rx, lax);
+    vec_masses<NP, DS>(ya, yb, yt, k.beta2, k.L2, k.nA2, k.nS2, py, qy, ry, lay);
 #pragma unroll
     for (int h = 0; h < NP; ++h) acc.Q2 = add2(acc.Q2, add2(qx[h], qy[h]));
     // residual mass of each vector, summed per group for the inverse-CDF walk
@@ -786,15 +841,15 @@ __device__ __forceinline__ void p2_pair(const f2 (&xa)[NP], const f2 (&xb)[NP], 
   } else if (JSD || KL) {
 #pragma unroll
     for (int h = 0; h < NP; ++h) {
-      px[h] = ex2_2(fma2(xa[h], k.L2, k.nA2));
-      py[h] = ex2_2(fma2(ya[h], k.L2, k.nA2));
+      lax[h] = fma2(xa[h], k.L2, k.nA2);
+      lay[h] = fma2(ya[h], k.L2, k.nA2);
+      px[h] = ex2_2(lax[h]);
+      py[h] = ex2_2(lay[h]);
     }
   }
   if (JSD || KL) {
-    div_terms<NP, JSD, KL>(xa, xb, px, k.L2, k.nA2, k.nB2, k.tiny2, acc.ja, acc.jb, acc.ms2,
-                           acc.kl2);
-    div_terms<NP, JSD, KL>(ya, yb, py, k.L2, k.nA2, k.nB2, k.tiny2, acc.ja, acc.jb, acc.ms2,
-                           acc.kl2);
+    div_terms<NP, JSD, KL>(lax, xb, px, k.L2, k.nB2, k.tiny2, acc.ja, acc.jb, acc.ms2, acc.kl2);
+    div_terms<NP, JSD, KL>(lay, yb, py, k.L2, k.nB2, k.tiny2, acc.ja, acc.jb, acc.ms2, acc.kl2);
   }
   if (LP) {
 #pragma unroll
@@ -833,16 +888,26 @@ __device__ __forceinline__ void p2_finish(const P2Acc& acc, X2& x) {
   x.Q = hsum2(acc.Q2);
 }
 
-// Pass 2 over the slice, two vectors per step.
-template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB>
+// What pass 2 does with a chunk of the slice once a warp has read it: nothing
+// in the one-shot kernel; the persistent kernel refills it with the next row.
+struct NoRelease {
+  static constexpr bool kActive = false;
+  int rc = 0;
+  __device__ __forceinline__ void operator()(int) const {}
+};
+
+// Pass 2 over the slice, two vectors per step.  Rel::kActive: after the last
+// step that reads chunk c (rounds [c rc, (c+1) rc)), every warp calls rel(c).
+template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, class Rel = NoRelease>
 __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int nv, int rounds,
                                       float beta, float A2, float B2, float S2, float lse_s, X2& x,
-                                      float* lp, float* grp) {
+                                      float* lp, float* grp, const Rel& rel = Rel()) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
   constexpr bool needT = (G & (G_RES | G_QF)) != 0 || LP;
   const P2Const k = p2_const(beta, A2, B2, S2, lse_s);
   P2Acc acc = {0ull, 0ull, 0ull, 0ull, 0ull, 0ull};
+  int next_c = 0;  // chunks this warp has released
   for (int kr = 0; kr < rounds; kr += 2) {
     const int i0 = kr * kTThreads + static_cast<int>(threadIdx.x);
     const int i1 = i0 + kTThreads;
@@ -862,21 +927,29 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
                          LP ? lp + i0 * VE : nullptr, LP ? lp + i1 * VE : nullptr);
     }
     if (G & (G_RES | G_QF)) p2_groups(g0, g1, grp, kr, rounds);
+    if constexpr (Rel::kActive) {
+      const int done = kr + 2;  // rounds this warp has finished
+      while (next_c < kChunks && (done >= (next_c + 1) * rel.rc || done >= rounds)) rel(next_c++);
+    }
+  }
+  if constexpr (Rel::kActive) {
+    while (next_c < kChunks) rel(next_c++);
   }
   p2_finish(acc, x);
 }
 
 // Pass 2 and the CTA combine; warp 0 stores the CTA's pass-2 record in the
 // workspace (groups: this CTA's group masses there, stored by pass 2).
-template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB>
+template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, class Rel = NoRelease>
 __device__ __forceinline__ void pass2_and_store(const T* ra, const T* rb, const T* rt, int nv,
                                                 int rounds, float beta, float* lp, SharedTma* sh,
-                                                float* rec, float* groups) {
+                                                float* rec, float* groups,
+                                                const Rel& rel = Rel()) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
   X2 x = x2_zero();
-  pass2<T, G, LP, DS>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e, lse_s * kLog2e,
-                  lse_s, x, lp, groups);
+  pass2<T, G, LP, DS, Rel>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e,
+                           lse_s * kLog2e, lse_s, x, lp, groups, rel);
   warp_reduce_x2<G>(x);
   if (lane == 0) sh->w2[warp] = x;
   __syncthreads();
@@ -1065,9 +1138,14 @@ struct RowCtx {
   int nv, rounds, rc, lo, n, W, rank, C, k, bi;
   long long row;
   bool bonus;
-  int dtok;           // warp 0 only
-  RowScalars sc;      // warp 0 only (stochastic)
+  int dtok;           // warp 0 only: the row's draft token (-1 on the bonus row)
   SharedTma* sh;
+  // persistent kernel: the parity of the row's chunk barriers and record
+  // slot, and the cluster's next row (-1 if none) with its copy kind
+  unsigned ph;
+  int slot;
+  long long next;
+  bool next_only_t;
 };
 
 // Rank 0: what pass 1 leaves for the row's decision.
@@ -1091,8 +1169,9 @@ __device__ __forceinline__ void store_row_stat(const KParams& P, long long row,
 
 // One row with pass-1 program F and pass-2 program G (R2: pass 2 runs; LP:
 // it writes the fused log-probs).
+// PER: the persistent kernel (the slice is refilled with the next row).
 template <typename T, bool STOCH, unsigned F, unsigned G, bool LP, bool R2,
-          int DS = ASYMSPEC_DELTA_AB>
+          int DS = ASYMSPEC_DELTA_AB, bool PER = false>
 __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
                                         cg::cluster_group& cluster) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -1102,27 +1181,35 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
   SharedTma* sh = c.sh;
   const float beta = P.beta;
   pass1_and_push<T, F, DS>(ra, rb, rt, c.nv, c.rounds, c.rc, c.lo, c.n, beta, c.dtok, sh, c.rank, c.C,
-                       cluster);
+                       cluster, c.ph, c.slot);
   if constexpr (!R2) {
     // no pass 2: rank 0 leaves the row's pass-1 results for the decision kernel
+    if constexpr (PER) {
+      // after B1 no thread reads the slice again: refill it with the next row
+      if (threadIdx.x == 0 && c.next >= 0 && !sh->broken) {
+        fence_proxy_async_shared();
+        issue_slice<T>(P, sh, c.next, c.lo, c.nv, c.rc, const_cast<T*>(ra), const_cast<T*>(rb),
+                       const_cast<T*>(rt), c.next_only_t);
+      }
+    }
     if (c.rank == 0 && warp == 0) {
       float lse[4];
-      const X1 w = combine_pass1<F>(sh, c.C, lse);
+      const X1 w = combine_pass1<F>(sh, c.C, lse, c.slot);
       float ad, bd, td;
-      draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td);
+      draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td, c.slot);
       if (lane == 0) store_row_stat(P, c.row, lse, w.is, w.it, w.bad, c.dtok, ad, bd, td);
     }
     return;
   } else {
     if (warp == 0) {
       float lse[4];
-      const X1 w = combine_pass1<F>(sh, c.C, lse);
+      const X1 w = combine_pass1<F>(sh, c.C, lse, c.slot);
       if (lane == 0) {
 #pragma unroll
         for (int q = 0; q < 4; ++q) sh->lse[q] = lse[q];
         if (c.rank == 0) {
           float ad, bd, td;
-          draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td);
+          draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td, c.slot);
           store_row_stat(P, c.row, lse, w.is, w.it, w.bad, c.dtok, ad, bd, td);
         }
       }
@@ -1130,64 +1217,73 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
     __syncthreads();
     float* lp = LP ? P.logprobs + static_cast<size_t>(c.row) * P.V + c.lo : nullptr;
     const size_t slot = static_cast<size_t>(c.row) * c.C + c.rank;
-    pass2_and_store<T, G, LP, DS>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh, P.pass2_rec + slot * 8,
-                              P.group_mass + slot * P.group_stride);
+    if constexpr (PER) {
+      const ChunkRefill<T> rel{c.rc, &P, sh, c.next, c.lo, c.nv, const_cast<T*>(ra),
+                               const_cast<T*>(rb), const_cast<T*>(rt), c.next_only_t};
+      pass2_and_store<T, G, LP, DS, ChunkRefill<T>>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh,
+                                                    P.pass2_rec + slot * 8,
+                                                    P.group_mass + slot * P.group_stride, rel);
+    } else {
+      pass2_and_store<T, G, LP, DS>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh,
+                                    P.pass2_rec + slot * 8, P.group_mass + slot * P.group_stride);
+    }
   }
 }
 
-template <typename T, bool STOCH, unsigned F, unsigned RQ, int DS = ASYMSPEC_DELTA_AB>
+template <typename T, bool STOCH, unsigned F, unsigned RQ, int DS = ASYMSPEC_DELTA_AB,
+          bool PER = false>
 __device__ __forceinline__ void run_full(const KParams& P, const RowCtx& c,
                                          cg::cluster_group& cluster) {
   const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
   const bool klg = P.divergence == ASYMSPEC_DIV_KL;
   if (P.logprobs) {
-    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, true, true, DS>(P, c, cluster);
-    else if (klg) run_row<T, STOCH, F, G_KL | RQ, true, true, DS>(P, c, cluster);
-    else run_row<T, STOCH, F, RQ, true, true, DS>(P, c, cluster);
+    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, true, true, DS, PER>(P, c, cluster);
+    else if (klg) run_row<T, STOCH, F, G_KL | RQ, true, true, DS, PER>(P, c, cluster);
+    else run_row<T, STOCH, F, RQ, true, true, DS, PER>(P, c, cluster);
   } else {
-    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, false, true, DS>(P, c, cluster);
-    else if (klg) run_row<T, STOCH, F, G_KL | RQ, false, true, DS>(P, c, cluster);
-    else run_row<T, STOCH, F, RQ, false, true, DS>(P, c, cluster);
+    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, false, true, DS, PER>(P, c, cluster);
+    else if (klg) run_row<T, STOCH, F, G_KL | RQ, false, true, DS, PER>(P, c, cluster);
+    else run_row<T, STOCH, F, RQ, false, true, DS, PER>(P, c, cluster);
   }
 }
 
 // Program set 0: every row program, chosen at run time, for delta source DS.
-template <typename T, bool STOCH, int DS>
+template <typename T, bool STOCH, int DS, bool PER = false>
 __device__ __forceinline__ void run_any(const KParams& P, const RowCtx& c, bool bonus,
                                         cg::cluster_group& cluster) {
   if (P.full) {
-    run_full<T, STOCH, F_LA | F_LB | F_LT | F_LS | F_AS | F_AT, STOCH ? G_RES : 0u, DS>(P, c, cluster);
+    run_full<T, STOCH, F_LA | F_LB | F_LT | F_LS | F_AS | F_AT, STOCH ? G_RES : 0u, DS, PER>(P, c, cluster);
   } else if (!STOCH) {
     const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
     const bool klg = P.divergence == ASYMSPEC_DIV_KL;
     constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
     if (bonus) {
-      if (P.fuse_bonus) run_row<T, STOCH, F_AS, 0, false, false, DS>(P, c, cluster);
-      else run_row<T, STOCH, F_AT, 0, false, false, DS>(P, c, cluster);
+      if (P.fuse_bonus) run_row<T, STOCH, F_AS, 0, false, false, DS, PER>(P, c, cluster);
+      else run_row<T, STOCH, F_AT, 0, false, false, DS, PER>(P, c, cluster);
     } else if (jsd) {
-      run_row<T, STOCH, FD, G_JSD, false, true, DS>(P, c, cluster);
+      run_row<T, STOCH, FD, G_JSD, false, true, DS, PER>(P, c, cluster);
     } else if (klg) {
-      run_row<T, STOCH, FD, G_KL, false, true, DS>(P, c, cluster);
+      run_row<T, STOCH, FD, G_KL, false, true, DS, PER>(P, c, cluster);
     } else {
-      run_row<T, STOCH, FD, 0, false, false, DS>(P, c, cluster);
+      run_row<T, STOCH, FD, 0, false, false, DS, PER>(P, c, cluster);
     }
   } else if (!bonus) {
     const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
     const bool klg = P.divergence == ASYMSPEC_DIV_KL;
     if (P.want_tokens) {
       constexpr unsigned FS = F_LA | F_LB | F_LS | F_AS;
-      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS>(P, c, cluster);
-      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS>(P, c, cluster);
-      else run_row<T, STOCH, FS, G_RES, false, true, DS>(P, c, cluster);
+      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS, PER>(P, c, cluster);
+      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS, PER>(P, c, cluster);
+      else run_row<T, STOCH, FS, G_RES, false, true, DS, PER>(P, c, cluster);
     } else {
       constexpr unsigned FS = F_LA | F_LB | F_LS;
-      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS>(P, c, cluster);
-      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS>(P, c, cluster);
-      else run_row<T, STOCH, FS, G_RES, false, true, DS>(P, c, cluster);
+      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS, PER>(P, c, cluster);
+      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS, PER>(P, c, cluster);
+      else run_row<T, STOCH, FS, G_RES, false, true, DS, PER>(P, c, cluster);
     }
   } else {
-    if (P.want_tokens) run_row<T, STOCH, F_LS | F_AS, G_QF, false, true, DS>(P, c, cluster);
-    else run_row<T, STOCH, F_LS, G_QF, false, true, DS>(P, c, cluster);
+    if (P.want_tokens) run_row<T, STOCH, F_LS | F_AS, G_QF, false, true, DS, PER>(P, c, cluster);
+    else run_row<T, STOCH, F_LS, G_QF, false, true, DS, PER>(P, c, cluster);
   }
 
 }
@@ -1210,7 +1306,13 @@ __host__ __device__ constexpr int tma_program_set(bool stoch, int divergence, bo
                    ((!stoch && fuse_bonus) ? 3 : 0);
 }
 
-template <typename T, bool STOCH, int SEL>
+// PER = false: one row per cluster (grid = rows x C).  PER = true: the
+// persistent form, grid = G clusters (as many as the device holds), cluster q
+// taking rows q, q + G, q + 2G, ...; each CTA keeps one slice buffer, and as
+// pass 2 of a row finishes with a chunk of it, that chunk is refilled with
+// the cluster's next row, so the copies of row r + G overlap pass 2 of row r
+// and pass 1 of row r + G starts on data already in shared memory.
+template <typename T, bool STOCH, int SEL, bool PER = false>
 __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   extern __shared__ __align__(128) unsigned char smem_tma[];
@@ -1219,12 +1321,10 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   const int tid = threadIdx.x;
   const int C = P.C;
   // 32-bit row arithmetic: the host keeps rows x C below 2^31
-  const unsigned row32 = blockIdx.x / static_cast<unsigned>(C);
-  const long long row = row32;
+  const unsigned rows32 = static_cast<unsigned>(P.rows);
+  const unsigned G = PER ? gridDim.x / static_cast<unsigned>(C) : 1u;
+  unsigned row32 = blockIdx.x / static_cast<unsigned>(C);
   const unsigned K1 = static_cast<unsigned>(P.K) + 1u;
-  const int bi = static_cast<int>(row32 / K1);
-  const int k = static_cast<int>(row32 - static_cast<unsigned>(bi) * K1);
-  const bool bonus = (k == P.K);
   const int V = P.V, W = P.W;
   const int lo = rank * W;
   const int n = max(0, min(W, V - lo));
@@ -1236,14 +1336,20 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   T* sb = sa + W;
   T* st = sb + W;
   SharedTma* sh = reinterpret_cast<SharedTma*>(smem_tma + P.sh_off);
-  const bool only_t = !STOCH && !P.full && bonus && !P.fuse_bonus;
+  auto t_only = [&](unsigned r) {
+    const unsigned kk = r - (r / K1) * K1;
+    return !STOCH && !P.full && kk == static_cast<unsigned>(P.K) && !P.fuse_bonus;
+  };
 
   if (tid == 0) {
 #pragma unroll
-    for (int c = 0; c < kChunks; ++c) mbar_init(&sh->bar[c], 1);
+    for (int c = 0; c < kChunks; ++c) {
+      mbar_init(&sh->bar[c], 1);
+      sh->rel[c] = 0;
+    }
     sh->broken = 0;
     fence_mbar_init();
-    issue_slice<T>(P, sh, row, lo, nv, rc, sa, sb, st, only_t);
+    issue_slice<T>(P, sh, row32, lo, nv, rc, sa, sb, st, t_only(row32));
   }
   RowCtx c;
   c.sa = sa;
@@ -1257,51 +1363,68 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   c.W = W;
   c.rank = rank;
   c.C = C;
-  c.k = k;
-  c.bi = bi;
-  c.row = row;
-  c.bonus = bonus;
   c.sh = sh;
-  c.dtok = -1;
-  c.sc = RowScalars{0.f, 0.f, 0.f};
-  // warp 0 keeps the row's scalar inputs, loaded while the slice is in flight
-  if ((tid >> 5) == 0) {
-    if (!bonus) c.dtok = P.tokens[static_cast<size_t>(bi) * P.K + k];
-    if (STOCH) c.sc = load_row_scalars(P, bi, k);
-  }
-  __syncthreads();  // the chunk barriers are initialised
+  unsigned it = 0;
+  for (;;) {
+    const int bi = static_cast<int>(row32 / K1);
+    const int k = static_cast<int>(row32 - static_cast<unsigned>(bi) * K1);
+    const bool bonus = (k == P.K);
+    c.k = k;
+    c.bi = bi;
+    c.row = row32;
+    c.bonus = bonus;
+    c.ph = it & 1u;
+    c.slot = PER ? static_cast<int>(it & 1u) : 0;
+    c.next = (PER && row32 + G < rows32) ? static_cast<long long>(row32 + G) : -1;
+    c.next_only_t = c.next >= 0 && t_only(row32 + G);
+    // warp 0 keeps the row's draft token, loaded while the slice is in flight
+    c.dtok = -1;
+    if ((tid >> 5) == 0 && !bonus) c.dtok = P.tokens[static_cast<size_t>(bi) * P.K + k];
+    if (it == 0) __syncthreads();  // the chunk barriers are initialised
 
-  if constexpr (SEL > 0 && STOCH) {
-    constexpr int d = SEL - 1;
-    constexpr unsigned GD = d == 0 ? G_JSD : d == 1 ? G_KL : 0u;
-    if (!bonus) run_row<T, STOCH, F_LA | F_LB | F_LS, GD | G_RES, false, true>(P, c, cluster);
-    else run_row<T, STOCH, F_LS, G_QF, false, true>(P, c, cluster);
-  } else if constexpr (SEL > 0) {
-    constexpr int d = (SEL - 1) % 3;
-    constexpr bool fused_bonus = SEL > 3;
-    constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
-    if (bonus) {
-      if (fused_bonus) run_row<T, STOCH, F_AS, 0, false, false>(P, c, cluster);
-      else run_row<T, STOCH, F_AT, 0, false, false>(P, c, cluster);
-    } else if (d == 0) {
-      run_row<T, STOCH, FD, G_JSD, false, true>(P, c, cluster);
-    } else if (d == 1) {
-      run_row<T, STOCH, FD, G_KL, false, true>(P, c, cluster);
+    if constexpr (SEL > 0 && STOCH) {
+      constexpr int d = SEL - 1;
+      constexpr unsigned GD = d == 0 ? G_JSD : d == 1 ? G_KL : 0u;
+      if (!bonus)
+        run_row<T, STOCH, F_LA | F_LB | F_LS, GD | G_RES, false, true, ASYMSPEC_DELTA_AB, PER>(
+            P, c, cluster);
+      else
+        run_row<T, STOCH, F_LS, G_QF, false, true, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
+    } else if constexpr (SEL > 0) {
+      constexpr int d = (SEL - 1) % 3;
+      constexpr bool fused_bonus = SEL > 3;
+      constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
+      if (bonus) {
+        if (fused_bonus) run_row<T, STOCH, F_AS, 0, false, false, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
+        else run_row<T, STOCH, F_AT, 0, false, false, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
+      } else if (d == 0) {
+        run_row<T, STOCH, FD, G_JSD, false, true, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
+      } else if (d == 1) {
+        run_row<T, STOCH, FD, G_KL, false, true, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
+      } else {
+        run_row<T, STOCH, FD, 0, false, false, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
+      }
+    } else if (P.delta_src == ASYMSPEC_DELTA_A) {
+      run_any<T, STOCH, ASYMSPEC_DELTA_A, PER>(P, c, bonus, cluster);
+    } else if (P.delta_src == ASYMSPEC_DELTA_TB) {
+      run_any<T, STOCH, ASYMSPEC_DELTA_TB, PER>(P, c, bonus, cluster);
     } else {
-      run_row<T, STOCH, FD, 0, false, false>(P, c, cluster);
+      run_any<T, STOCH, ASYMSPEC_DELTA_AB, PER>(P, c, bonus, cluster);
     }
-  } else if (P.delta_src == ASYMSPEC_DELTA_A) {
-    run_any<T, STOCH, ASYMSPEC_DELTA_A>(P, c, bonus, cluster);
-  } else if (P.delta_src == ASYMSPEC_DELTA_TB) {
-    run_any<T, STOCH, ASYMSPEC_DELTA_TB>(P, c, bonus, cluster);
-  } else {
-    run_any<T, STOCH, ASYMSPEC_DELTA_AB>(P, c, bonus, cluster);
+    if (!PER || c.next < 0) break;
+    row32 += G;
+    ++it;
   }
 
-  // a copy that timed out may still land: wait for it (bounded) before exit
+  // a copy that timed out may still land: wait for it (bounded) before exit.
+  // No copy of a later row is issued once a copy has timed out, but the
+  // persistent kernel may have moved on by then, so both parities are waited.
   if (tid == 0 && sh->broken) {
 #pragma unroll
-    for (int q = 0; q < kChunks; ++q) mbar_wait_bounded(&sh->bar[q], 0, kCopyTimeoutNs);
+    for (int q = 0; q < kChunks; ++q) {
+      mbar_wait_bounded(&sh->bar[q], 0u, kCopyTimeoutNs);
+      if (PER) mbar_wait_bounded(&sh->bar[q], 1u, kCopyTimeoutNs);
+    }
   }
 }
 
@@ -1319,6 +1442,9 @@ constexpr int kDecideThreads = 256;  // at most 8 warps; each takes rows k, k + 
 template <typename T, bool STOCH>
 __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  // launched as a programmatic dependent of the row kernel: its CTAs may
+  // start early; nothing of the workspace is read before that kernel is done
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int bi = blockIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
   const int K = P.K, K1 = K + 1, C = P.C;

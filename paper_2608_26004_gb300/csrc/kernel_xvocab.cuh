@@ -7,19 +7,24 @@
 // t'_j = t[map_v[j]] (verifier vocabulary); the emitted pair index j is
 // committed as the verifier token map_v[j].
 //
+//   xvocab_inv_fill, xvocab_inv_build
+//                  the map check: inverse maps inv_d[V_d], inv_v[V_v] (the
+//                  pair of each token, -1 if unpaired) built with atomicCAS,
+//                  and a map-error word that an entry outside its vocabulary
+//                  or a token claimed by two pairs sets.
 //   xvocab_gather  restricts every row of a, b and t to the pairs, in pair
 //                  order, into dense [rows, S] arrays the fuse-and-verify
 //                  kernels then read as rows of a vocabulary of S entries.
 //   xvocab_emit    turns the emitted pair index of each batch element into
-//                  its verifier token.
+//                  its verifier token (every element is a data error if the
+//                  map-error word is set).
 //
 // HBM-bound, no contraction: per row the gather reads the 3 S paired
-// entries (scattered through the maps) and writes them densely.  A CTA
-// takes kXJ pair indices per thread for kXRows rows, so each map entry is
-// read once per CTA and reused across the rows.  A map entry outside its
-// vocabulary is never dereferenced: the gathered value becomes NaN (which
-// the step reports as a non-finite row, ASYMSPEC_DATA_NONFINITE, on every
-// batch element) and ASYMSPEC_DATA_BAD_MAP is OR-ed into the error word.
+// entries through the maps and writes them densely.  A warp reading through
+// a random map asks L2 for a sector per entry (a sequential read of the
+// source row scattered through the inverse map into a shared-memory copy of
+// the restricted row was measured no faster: the int32 inverse map doubles
+// the bytes each source row brings from L2).
 #pragma once
 
 #include "device_common.cuh"
@@ -106,14 +111,62 @@ __global__ void __launch_bounds__(kXThreads) xvocab_gather(XGatherParams P) {
   }
 }
 
-// out_next[b] = map_v[next_index[b]] (-1 stays -1: a data error).
+// inv[v] = -1 for every token of both vocabularies; the map-error word is
+// cleared.  (I = int; a template so that the header can be included twice.)
 template <typename I>
-__global__ void __launch_bounds__(256) xvocab_emit(const I* __restrict__ next_index,
+__global__ void __launch_bounds__(256) xvocab_inv_fill(I* __restrict__ inv_d, int V_d,
+                                                       I* __restrict__ inv_v, int V_v,
+                                                       unsigned* __restrict__ map_err) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < V_d) inv_d[i] = -1;
+  if (i < V_v) inv_v[i] = -1;
+  if (i == 0) *map_err = 0u;
+}
+
+// inv_d[map_d[j]] = j and inv_v[map_v[j]] = j; an entry outside its
+// vocabulary, or a token that a second pair claims, sets the error word.
+template <typename I>
+__global__ void __launch_bounds__(256) xvocab_inv_build(const I* __restrict__ map_d,
+                                                        const I* __restrict__ map_v, int S,
+                                                        I* __restrict__ inv_d, int V_d,
+                                                        I* __restrict__ inv_v, int V_v,
+                                                        unsigned* __restrict__ map_err,
+                                                        uint32_t* __restrict__ err_word) {
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= S) return;
+  const I md = map_d[j], mv = map_v[j];
+  bool bad = false;
+  if (static_cast<unsigned>(md) < static_cast<unsigned>(V_d))
+    bad |= atomicCAS(inv_d + md, I(-1), I(j)) != I(-1);
+  else
+    bad = true;
+  if (static_cast<unsigned>(mv) < static_cast<unsigned>(V_v))
+    bad |= atomicCAS(inv_v + mv, I(-1), I(j)) != I(-1);
+  else
+    bad = true;
+  if (bad) {
+    atomicOr(map_err, 1u);
+    if (err_word) atomicOr(err_word, ASYMSPEC_DATA_BAD_MAP);
+  }
+}
+
+// out_next[b] = map_v[next_index[b]] (-1 stays -1: a data error); with the
+// map-error word set, every element is a data error (its pair index too).
+template <typename I>
+__global__ void __launch_bounds__(256) xvocab_emit(I* __restrict__ next_index,
                                                    const I* __restrict__ map_v, int S, int B,
+                                                   const unsigned* __restrict__ map_err,
+                                                   I* __restrict__ out_len,
                                                    I* __restrict__ out_next) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= B) return;
   const I j = next_index[i];
+  if (*map_err) {
+    out_len[i] = -1;
+    out_next[i] = -1;
+    next_index[i] = -1;
+    return;
+  }
   out_next[i] = (j >= 0 && j < S) ? map_v[j] : -1;
 }
 

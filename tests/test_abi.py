@@ -260,15 +260,21 @@ def test_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):
 
 def test_xvocab_workspace_layout_and_validation(lib):
     # the restricted rows a', b', t' ([B, K+1, S] each), the emitted pair
-    # indices, then the step's workspace for a vocabulary of S entries
-    for B, K, S, dtype, elt in ((64, 7, 109568, A.BF16, 2), (3, 2, 37, A.FP32, 4)):
+    # indices, the gather's scratch (inverse maps and the map-error word),
+    # then the step's workspace for a vocabulary of S entries
+    for B, K, S, V_d, V_v, dtype, elt in ((64, 7, 109568, 151936, 128256, A.BF16, 2),
+                                          (3, 2, 37, 50, 41, A.FP32, 4)):
         R = B * (K + 1)
-        want = 3 * _up(R * S * elt) + _up(B * 4) + A.workspace_bytes(B, K, S)
-        assert A.xvocab_workspace_bytes(B, K, S, dtype) == want
-    assert A.xvocab_workspace_bytes(0, 2, 10, A.FP32) == 0
-    assert A.xvocab_workspace_bytes(2, 2, 1, A.FP32) == 0
-    assert A.xvocab_workspace_bytes(2, 2, 10, 5) == 0
-    need = A.xvocab_workspace_bytes(2, 2, 10, A.FP32)
+        scratch = _up(V_d * 4) + _up(V_v * 4) + 256
+        assert A.xvocab_gather_scratch_bytes(V_d, V_v) == scratch
+        want = 3 * _up(R * S * elt) + _up(B * 4) + scratch + A.workspace_bytes(B, K, S)
+        assert A.xvocab_workspace_bytes(B, K, S, V_d, V_v, dtype) == want
+    assert A.xvocab_workspace_bytes(0, 2, 10, 30, 20, A.FP32) == 0
+    assert A.xvocab_workspace_bytes(2, 2, 1, 30, 20, A.FP32) == 0
+    assert A.xvocab_workspace_bytes(2, 2, 10, 0, 20, A.FP32) == 0
+    assert A.xvocab_workspace_bytes(2, 2, 10, 30, 20, 5) == 0
+    assert A.xvocab_gather_scratch_bytes(0, 5) == 0
+    need = A.xvocab_workspace_bytes(2, 2, 10, 30, 20, A.FP32)
 
     def fv(B=2, K=2, S=10, V_d=30, V_v=20, dtype=A.FP32, gate=None, ws=FAKE, n=need, **p):
         x = dict(a=FAKE, b=FAKE, t=FAKE, md=FAKE, mv=FAKE, d=FAKE, pr=FAKE, u=FAKE, L=FAKE,
@@ -288,7 +294,7 @@ def test_xvocab_workspace_layout_and_validation(lib):
     assert fv(gate=A.gate_params(mode=A.MODE_STOCHASTIC), u=0) == A.ERR_INVALID_ARG
     assert fv(N=FAKE + 2) == A.ERR_MISALIGNED
     assert fv(ws=0) == A.ERR_WORKSPACE
-    assert fv(ws=FAKE + 8) == A.ERR_WORKSPACE
+    assert fv(ws=FAKE + 16) == A.ERR_WORKSPACE           # not 256-byte aligned
     assert fv(n=need - 1) == A.ERR_WORKSPACE
     assert fv(md=0) == A.ERR_INVALID_ARG                 # the gather's own checks
     assert fv(a=FAKE + 2) == A.ERR_MISALIGNED
@@ -303,3 +309,8 @@ def test_xvocab_workspace_layout_and_validation(lib):
         == A.ERR_MISALIGNED
     assert g(FAKE, FAKE, 30, FAKE, 20, FAKE, FAKE, 10, 8 * 65536, A.FP32, FAKE, FAKE, FAKE) \
         == A.ERR_TOO_LARGE
+    small = A.xvocab_gather_scratch_bytes(30, 20) - 1
+    assert g(FAKE, FAKE, 30, FAKE, 20, FAKE, FAKE, 10, 4, A.FP32, FAKE, FAKE, FAKE, None,
+             FAKE, small) == A.ERR_WORKSPACE
+    assert g(FAKE, FAKE, 30, FAKE, 20, FAKE, FAKE, 10, 4, A.FP32, FAKE, FAKE, FAKE, None,
+             FAKE + 16, small + 1) == A.ERR_WORKSPACE

@@ -49,7 +49,7 @@ def run(torch, x, mode, *, gamma=0.5, beta=1.0, map_d=None, map_v=None, draft=No
     t = dev(torch, x.logits_ver, x.dtype)
     d = dev(torch, np.asarray(x.draft_tokens if draft is None else draft, np.int32))
     pr, u = dev(torch, x.draft_probs.astype(np.float32)), dev(torch, x.uniforms.astype(np.float32))
-    nbytes = A.xvocab_workspace_bytes(x.B, x.K, x.S, x.dtype)
+    nbytes = A.xvocab_workspace_bytes(x.B, x.K, x.S, x.V_d, x.V_v, x.dtype)
     ws = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
     L = torch.empty(x.B, dtype=torch.int32, device="cuda")
     N = torch.empty_like(L)
@@ -158,30 +158,80 @@ def test_identity_map_is_the_plain_step(torch):
         assert np.array_equal(I, N) and err == 0
 
 
-@pytest.mark.parametrize("dtype", [synth.FP32, synth.BF16])
-def test_gather_is_exact(torch, dtype):
-    x = small(dtype, 203, seed=5, B=3, K=2, V_d=1000, V_v=777)
+def gather(torch, x, md, mv, with_scratch):
+    """asymspec_xvocab_gather on a synth.XBatch; the three restricted arrays as
+    bit patterns and the error word."""
     rows = x.B * (x.K + 1)
-    a, b = dev(torch, x.logits_full, dtype), dev(torch, x.logits_comp, dtype)
-    t = dev(torch, x.logits_ver, dtype)
-    md, mv = dev(torch, x.map_d), dev(torch, x.map_v)
-    tdt = torch.float32 if dtype == synth.FP32 else torch.bfloat16
+    a, b = dev(torch, x.logits_full, x.dtype), dev(torch, x.logits_comp, x.dtype)
+    t = dev(torch, x.logits_ver, x.dtype)
+    mdd, mvd = dev(torch, np.asarray(md, np.int32)), dev(torch, np.asarray(mv, np.int32))
+    tdt = torch.float32 if x.dtype == synth.FP32 else torch.bfloat16
     outs = [torch.empty(rows, x.S, dtype=tdt, device="cuda") for _ in range(3)]
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
-    st = A.xvocab_gather(a.data_ptr(), b.data_ptr(), x.V_d, t.data_ptr(), x.V_v, md.data_ptr(),
-                         mv.data_ptr(), x.S, rows, dtype, *[o.data_ptr() for o in outs],
-                         err.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    n = A.xvocab_gather_scratch_bytes(x.V_d, x.V_v)
+    scratch = torch.full((n,), 0x5A, dtype=torch.uint8, device="cuda") if with_scratch else None
+    st = A.xvocab_gather(a.data_ptr(), b.data_ptr(), x.V_d, t.data_ptr(), x.V_v, mdd.data_ptr(),
+                         mvd.data_ptr(), x.S, rows, x.dtype, *[o.data_ptr() for o in outs],
+                         err.data_ptr(), scratch.data_ptr() if with_scratch else None,
+                         n if with_scratch else 0, torch.cuda.current_stream().cuda_stream)
     assert st == A.OK
     torch.cuda.synchronize()
-    view = np.float32 if dtype == synth.FP32 else np.uint16
-    got = [o.view(torch.int32 if dtype == synth.FP32 else torch.int16).cpu().numpy().view(view)
+    bits = np.uint32 if x.dtype == synth.FP32 else np.uint16
+    got = [o.view(torch.int32 if x.dtype == synth.FP32 else torch.int16).cpu().numpy().view(bits)
            for o in outs]
+    return got, int(err.item()) & 0xFFFFFFFF
+
+
+@pytest.mark.parametrize("with_scratch", [True, False])
+@pytest.mark.parametrize("S", [200, 203])
+@pytest.mark.parametrize("dtype", [synth.FP32, synth.BF16])
+def test_gather_is_exact(torch, dtype, S, with_scratch):
+    # with and without the map check, 16-byte and unaligned restricted rows
+    x = small(dtype, S, seed=5, B=3, K=2, V_d=1000, V_v=776)
+    rows = x.B * (x.K + 1)
+    got, err = gather(torch, x, x.map_d, x.map_v, with_scratch)
+    bits = np.uint32 if dtype == synth.FP32 else np.uint16
     want = [x.logits_full.reshape(rows, -1)[:, x.map_d], x.logits_comp.reshape(rows, -1)[:, x.map_d],
             x.logits_ver.reshape(rows, -1)[:, x.map_v]]
     for g, w_ in zip(got, want):
-        assert np.array_equal(g.view(np.uint32 if dtype == synth.FP32 else np.uint16),
-                              w_.view(np.uint32 if dtype == synth.FP32 else np.uint16))
-    assert int(err.item()) == 0
+        assert np.array_equal(g, w_.view(bits))
+    assert err == 0
+
+
+def test_gather_of_full_size_rows(torch):
+    # Qwen3 / Llama-3 sized rows and the paper's shared set
+    x = full_size(1, 8, 5)
+    rows = x.B * (x.K + 1)
+    got, err = gather(torch, x, x.map_d, x.map_v, True)
+    assert np.array_equal(got[0], x.logits_full.reshape(rows, -1)[:, x.map_d])
+    assert np.array_equal(got[1], x.logits_comp.reshape(rows, -1)[:, x.map_d])
+    assert np.array_equal(got[2], x.logits_ver.reshape(rows, -1)[:, x.map_v])
+    assert err == 0
+
+
+@pytest.mark.parametrize("side", ["d", "v"])
+def test_a_token_in_two_pairs_is_a_data_error(torch, side):
+    # the map check finds the token claimed twice: the map bit is set and
+    # every batch element is a data error (pair index included); the gather
+    # itself still copies what the maps name
+    x = small(synth.BF16, 200, V_d=304, V_v=256)
+    md, mv = x.map_d.copy(), x.map_v.copy()
+    if side == "d":
+        md[40] = md[41]
+    else:
+        mv[7] = mv[150]
+    with pytest.raises(ValueError):
+        O.check_vocab_map(md, mv, x.V_d, x.V_v)
+    got, err = gather(torch, x, md, mv, True)
+    assert err & A.DATA_BAD_MAP
+    rows = x.B * (x.K + 1)
+    assert np.array_equal(got[0], x.logits_full.reshape(rows, -1)[:, md])
+    assert np.array_equal(got[2], x.logits_ver.reshape(rows, -1)[:, mv])
+    _, err = gather(torch, x, md, mv, False)           # without the check: not detected
+    assert err == 0
+    for mode in (GREEDY, STOCH):
+        L, N, I, e = run(torch, x, mode, map_d=md, map_v=mv)
+        assert np.all(L == -1) and np.all(N == -1) and np.all(I == -1) and e & A.DATA_BAD_MAP
 
 
 @pytest.mark.parametrize("side", ["d", "v"])
