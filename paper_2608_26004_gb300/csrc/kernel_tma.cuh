@@ -42,6 +42,8 @@
 // thread 0 waits (bounded again) for any copy still in flight.
 #pragma once
 
+#include <type_traits>
+
 #include "device_common.cuh"
 
 namespace asymspec_impl {
@@ -563,20 +565,24 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
     int e0 = i0 * VE;                       // its element offset in the slice
     for (int kr = r0; kr < r1; kr += 2, i0 += 2 * kTThreads, e0 += STEP) {
       if (i0 >= nv) break;
-      const bool has1 = (kr + 1 < r1) && (i0 + kTThreads < nv);
+      // TWO: the thread has both vectors of the step (all but the slice's
+      // last step); the other form fills the missing one (one copy each)
+      auto step = [&](auto two) {
+      constexpr bool TWO = decltype(two)::value;
+      const bool has1 = TWO;
       const int e1 = e0 + kTThreads * VE;
       f2 xa[NP], xb[NP], xt[NP], xs[NP], ya[NP], yb[NP], yt[NP], ys[NP];
       if (needA) {
         load_pairs(ra + e0, xa);
-        load_or_fill(ra + e1, has1, ya);
+        if (TWO) load_pairs(ra + e1, ya); else load_or_fill(ra + e1, false, ya);
       }
       if (needB) {
         load_pairs(rb + e0, xb);
-        load_or_fill(rb + e1, has1, yb);
+        if (TWO) load_pairs(rb + e1, yb); else load_or_fill(rb + e1, false, yb);
       }
       if (needT) {
         load_pairs(rt + e0, xt);
-        load_or_fill(rt + e1, has1, yt);
+        if (TWO) load_pairs(rt + e1, yt); else load_or_fill(rt + e1, false, yt);
       }
       if (needS) {
 #pragma unroll
@@ -601,6 +607,9 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
         arg_track(e.vt, vec_t, ct0, i0, e.bad, kBadT);
         if (has1) arg_track(e.vt, vec_t, ct1, i0 + kTThreads, e.bad, kBadT);
       }
+      };
+      if ((kr + 1 < r1) && (i0 + kTThreads < nv)) step(std::true_type{});
+      else step(std::false_type{});
     }
   }
   bool ovf = false;
@@ -913,18 +922,28 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
     const int i1 = i0 + kTThreads;
     float g0 = 0.f, g1 = 0.f;  // this thread's vector masses in rounds kr and kr + 1
     if (i0 < nv) {
-      const bool has1 = i1 < nv;
-      f2 xa[NP], xb[NP], xt[NP], ya[NP], yb[NP], yt[NP];
-      load_pairs(ra + i0 * VE, xa);
-      load_pairs(rb + i0 * VE, xb);
-      load_or_fill(ra + i1 * VE, has1, ya);
-      load_or_fill(rb + i1 * VE, has1, yb);
-      if (needT) {
-        load_pairs(rt + i0 * VE, xt);
-        load_or_fill(rt + i1 * VE, has1, yt);
-      }
-      p2_pair<NP, G, LP, DS>(xa, xb, xt, ya, yb, yt, has1, k, acc, g0, g1,
-                         LP ? lp + i0 * VE : nullptr, LP ? lp + i1 * VE : nullptr);
+      // TWO: both vectors present (all but the slice's last step)
+      auto step = [&](auto two) {
+        constexpr bool TWO = decltype(two)::value;
+        f2 xa[NP], xb[NP], xt[NP], ya[NP], yb[NP], yt[NP];
+        load_pairs(ra + i0 * VE, xa);
+        load_pairs(rb + i0 * VE, xb);
+        if (TWO) {
+          load_pairs(ra + i1 * VE, ya);
+          load_pairs(rb + i1 * VE, yb);
+        } else {
+          load_or_fill(ra + i1 * VE, false, ya);
+          load_or_fill(rb + i1 * VE, false, yb);
+        }
+        if (needT) {
+          load_pairs(rt + i0 * VE, xt);
+          if (TWO) load_pairs(rt + i1 * VE, yt); else load_or_fill(rt + i1 * VE, false, yt);
+        }
+        p2_pair<NP, G, LP, DS>(xa, xb, xt, ya, yb, yt, TWO, k, acc, g0, g1,
+                               LP ? lp + i0 * VE : nullptr, LP ? lp + i1 * VE : nullptr);
+      };
+      if (i1 < nv) step(std::true_type{});
+      else step(std::false_type{});
     }
     if (G & (G_RES | G_QF)) p2_groups(g0, g1, grp, kr, rounds);
     if constexpr (Rel::kActive) {
