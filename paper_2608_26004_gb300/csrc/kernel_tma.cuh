@@ -309,6 +309,15 @@ __device__ __forceinline__ int arg_in_vector(const f2 (&x)[NP], float v, int bas
   return idx;
 }
 
+// The first two entries of a 16-byte vector in shared memory, widened.
+__device__ __forceinline__ f2 first_pair(const __nv_bfloat16* p) {
+  const unsigned w = *reinterpret_cast<const unsigned*>(p);
+  return pk(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+}
+__device__ __forceinline__ f2 first_pair(const float* p) {
+  return *reinterpret_cast<const f2*>(p);
+}
+
 // The fused score s = t + beta delta of a pair (Eq. 2) for delta source DS:
 // a - b (Eq. 1, ASYMSPEC_DELTA_AB), a (raw-augmented) or t - b (SCD-style).
 template <int DS>
@@ -530,20 +539,21 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
     atomicOr(&sh->broken, kBadTimeout);
   float ref[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
   if (tid < nv) {
-    f2 xa[NP], xb[NP], xt[NP], xs[NP];
-    if (needA) load_pairs(ra + tid * VE, xa);
-    if (needB) load_pairs(rb + tid * VE, xb);
-    if (needT) load_pairs(rt + tid * VE, xt);
-    if (F & F_LA) ref[0] = vmax_pairs(xa);
-    if (F & F_LB) ref[1] = vmax_pairs(xb);
-    if (F & F_LT) ref[2] = vmax_pairs(xt);
+    // the first two entries of the thread's first vector: any entries do as
+    // references (a sum that reaches 2^100 sends the CTA to pass1_online)
+    f2 xa = 0ull, xb = 0ull, xt = 0ull;
+    if (needA) xa = first_pair(ra + tid * VE);
+    if (needB) xb = first_pair(rb + tid * VE);
+    if (needT) xt = first_pair(rt + tid * VE);
+    if (F & F_LA) ref[0] = fmaxf(lo_of(xa), hi_of(xa));
+    if (F & F_LB) ref[1] = fmaxf(lo_of(xb), hi_of(xb));
+    if (F & F_LT) ref[2] = fmaxf(lo_of(xt), hi_of(xt));
     if (F & F_LS) {
-#pragma unroll
-      for (int h = 0; h < NP; ++h) xs[h] = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
-      ref[3] = vmax_pairs(xs);
+      const f2 xs = fuse2<DS>(beta2, xa, xb, xt);
+      ref[3] = fmaxf(lo_of(xs), hi_of(xs));
     }
   }
-  // one reference per warp: the largest of its threads' first-vector maxima
+  // one reference per warp: the largest of its threads' first-pair maxima
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const unsigned bit = q == 0 ? F_LA : q == 1 ? F_LB : q == 2 ? F_LT : F_LS;
