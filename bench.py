@@ -512,17 +512,6 @@ def main():
                   "frac": alg_bytes / (kernel_ms_p * 1e-3) / 1e9 / hbm_peak}
     alg_bytes_o = algorithmic_bytes(B, K, V, 2, other_mode == A.MODE_STOCHASTIC)
 
-    # ---- the drafter's draw (asymspec_draft_sample), the step upstream of
-    # fuse-and-verify: per drafted position one launch over the B rows of the
-    # drafter's full-context logits, and once over all B (K+1) rows.  Timed as
-    # CUDA graph replays (host launch overhead would exceed a 64-row launch);
-    # the launches read the rows of both resident sets in turn (262 MB > L2).
-    draft = draft_timing(torch, A, sets, B, K, V, mode, dev, args.steps)
-
-    # ---- the cross-family step (drafter and verifier vocabularies that
-    # differ, restricted to their shared tokens): reported alongside
-    xvocab = xvocab_timing(torch, A, synth, mode, dev, args.steps, timed, stream)
-
     # ---- end to end through the C ABI with host buffers
     pin = dict(
         a=torch.from_numpy(np.ascontiguousarray(batch.logits_full).view(np.int16)).view(
@@ -554,6 +543,18 @@ def main():
     e2e_steps = max(3, min(args.steps, 30))
     ms_e2e = timed(e2e_step, e2e_steps, 3) / e2e_steps
     e2e_value = world * rows / (ms_e2e * 1e-3)
+
+    # ---- the drafter's draw (asymspec_draft_sample), the step upstream of
+    # fuse-and-verify: per drafted position one launch over the B rows of the
+    # drafter's full-context logits, and once over all B (K+1) rows.  Timed as
+    # CUDA graph replays (host launch overhead would exceed a 64-row launch);
+    # the launches read the rows of both resident sets in turn (262 MB > L2).
+    draft = draft_timing(torch, A, sets, B, K, V, mode, dev, args.steps)
+
+    # ---- the cross-family step (drafter and verifier vocabularies that
+    # differ, restricted to their shared tokens): reported alongside
+    xvocab = xvocab_timing(torch, A, synth, mode, dev, args.steps, timed, stream)
+
 
     line = {
         "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": world,
