@@ -85,7 +85,8 @@ struct __align__(16) SharedTma {
   float lse[4];       // the row's normalisers (pass 2 reads them)
   unsigned broken;    // a chunk copy timed out
   int rel[kChunks];   // persistent kernel: warps done with each chunk of the row
-  unsigned pad[3];
+  float qown;         // production draft rows: this slice's fused mass, from pass 1
+  unsigned pad[2];
   // slot s (0, or the row's parity in the persistent kernel) of the C pushed records
   __device__ X1* recv1(int slot = 0, int C = 0) { return reinterpret_cast<X1*>(this + 1) + slot * C; }
 };
@@ -828,7 +829,7 @@ __device__ __forceinline__ P2Const p2_const(float beta, float A2, float B2, floa
 // Pass 2 on two vectors x, y of a thread (y absent unless has1: filled with
 // -1e30, which contributes nothing); g0, g1 receive their inverse-CDF masses
 // (residual, or fused for G_QF).  LP: fused log-probs go to lpx, lpy.
-template <int NP, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB>
+template <int NP, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, bool QSUM = true>
 __device__ __forceinline__ void p2_pair(const f2 (&xa)[NP], const f2 (&xb)[NP], const f2 (&xt)[NP],
                                         const f2 (&ya)[NP], const f2 (&yb)[NP], const f2 (&yt)[NP],
                                         bool has1, const P2Const& k, P2Acc& acc, float& g0,
@@ -840,8 +841,12 @@ __device__ __forceinline__ void p2_pair(const f2 (&xa)[NP], const f2 (&xb)[NP], 
     f2 qx[NP], qy[NP], rx[NP], ry[NP];
     vec_masses<NP, DS>(xa, xb, xt, k.beta2, k.L2, k.nA2, k.nS2, px, qx, rx, lax);
     vec_masses<NP, DS>(ya, yb, yt, k.beta2, k.L2, k.nA2, k.nS2, py, qy, ry, lay);
+    // the fused mass, used only when the whole residual is zero (QSUM false:
+    // the caller takes the slice's fused mass from its pass-1 sum instead)
+    if constexpr (QSUM) {
 #pragma unroll
-    for (int h = 0; h < NP; ++h) acc.Q2 = add2(acc.Q2, add2(qx[h], qy[h]));
+      for (int h = 0; h < NP; ++h) acc.Q2 = add2(acc.Q2, add2(qx[h], qy[h]));
+    }
     // residual mass of each vector, summed per group for the inverse-CDF walk
     g0 = vsum(rx);
     g1 = vsum(ry);
@@ -899,6 +904,21 @@ __device__ __forceinline__ void p2_groups(float g0, float g1, float* grp, int kr
   if (lane == 16 && kr + 1 < rounds) grp[(kr + 1) * kTWarps + warp] = g;
 }
 
+// As p2_groups for four rounds kr .. kr + 3 (v0 .. v3) in one transposed
+// butterfly: lanes 0, 8, 16 and 24 end with the four group masses.
+__device__ __forceinline__ void p2_groups4(float v0, float v1, float v2, float v3, float* grp,
+                                           int kr, int rounds) {
+  const int lane = static_cast<int>(threadIdx.x & 31), warp = static_cast<int>(threadIdx.x >> 5);
+  const bool up16 = (lane & 16) != 0, up8 = (lane & 8) != 0;
+  const float a = (up16 ? v2 : v0) + __shfl_xor_sync(0xffffffffu, up16 ? v0 : v2, 16);
+  const float b = (up16 ? v3 : v1) + __shfl_xor_sync(0xffffffffu, up16 ? v1 : v3, 16);
+  float c = (up8 ? b : a) + __shfl_xor_sync(0xffffffffu, up8 ? a : b, 8);
+#pragma unroll
+  for (int off = 4; off > 0; off >>= 1) c += __shfl_xor_sync(0xffffffffu, c, off);
+  const int r = kr + (lane >> 3);
+  if ((lane & 7) == 0 && r < rounds) grp[r * kTWarps + warp] = c;
+}
+
 __device__ __forceinline__ void p2_finish(const P2Acc& acc, X2& x) {
   x.j = hsum2(add2(acc.ja, acc.jb));
   x.msum = hsum2(acc.ms2);
@@ -917,7 +937,8 @@ struct NoRelease {
 
 // Pass 2 over the slice, two vectors per step.  Rel::kActive: after the last
 // step that reads chunk c (rounds [c rc, (c+1) rc)), every warp calls rel(c).
-template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, class Rel = NoRelease>
+template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, class Rel = NoRelease,
+          bool QSUM = true>
 __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int nv, int rounds,
                                       float beta, float A2, float B2, float S2, float lse_s, X2& x,
                                       float* lp, float* grp, const Rel& rel = Rel()) {
@@ -927,6 +948,8 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
   const P2Const k = p2_const(beta, A2, B2, S2, lse_s);
   P2Acc acc = {0ull, 0ull, 0ull, 0ull, 0ull, 0ull};
   int next_c = 0;  // chunks this warp has released
+  float gp0 = 0.f, gp1 = 0.f;  // the previous step's masses, reduced with this step's
+  bool pending = false;
   for (int kr = 0; kr < rounds; kr += 2) {
     const int i0 = kr * kTThreads + static_cast<int>(threadIdx.x);
     const int i1 = i0 + kTThreads;
@@ -949,18 +972,25 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
           load_pairs(rt + i0 * VE, xt);
           if (TWO) load_pairs(rt + i1 * VE, yt); else load_or_fill(rt + i1 * VE, false, yt);
         }
-        p2_pair<NP, G, LP, DS>(xa, xb, xt, ya, yb, yt, TWO, k, acc, g0, g1,
+        p2_pair<NP, G, LP, DS, QSUM>(xa, xb, xt, ya, yb, yt, TWO, k, acc, g0, g1,
                                LP ? lp + i0 * VE : nullptr, LP ? lp + i1 * VE : nullptr);
       };
       if (i1 < nv) step(std::true_type{});
       else step(std::false_type{});
     }
-    if (G & (G_RES | G_QF)) p2_groups(g0, g1, grp, kr, rounds);
+    if (G & (G_RES | G_QF)) {
+      // group masses leave the warp four rounds at a time
+      if (pending) p2_groups4(gp0, gp1, g0, g1, grp, kr - 2, rounds);
+      gp0 = g0;
+      gp1 = g1;
+      pending = !pending;
+    }
     if constexpr (Rel::kActive) {
       const int done = kr + 2;  // rounds this warp has finished
       while (next_c < kChunks && (done >= (next_c + 1) * rel.rc || done >= rounds)) rel(next_c++);
     }
   }
+  if ((G & (G_RES | G_QF)) && pending) p2_groups(gp0, gp1, grp, ((rounds - 1) & ~1), rounds);
   if constexpr (Rel::kActive) {
     while (next_c < kChunks) rel(next_c++);
   }
@@ -969,7 +999,8 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
 
 // Pass 2 and the CTA combine; warp 0 stores the CTA's pass-2 record in the
 // workspace (groups: this CTA's group masses there, stored by pass 2).
-template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, class Rel = NoRelease>
+template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, class Rel = NoRelease,
+          bool QSUM = true>
 __device__ __forceinline__ void pass2_and_store(const T* ra, const T* rb, const T* rt, int nv,
                                                 int rounds, float beta, float* lp, SharedTma* sh,
                                                 float* rec, float* groups,
@@ -977,14 +1008,15 @@ __device__ __forceinline__ void pass2_and_store(const T* ra, const T* rb, const 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
   X2 x = x2_zero();
-  pass2<T, G, LP, DS, Rel>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e,
-                           lse_s * kLog2e, lse_s, x, lp, groups, rel);
+  pass2<T, G, LP, DS, Rel, QSUM>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e,
+                                 lse_s * kLog2e, lse_s, x, lp, groups, rel);
   warp_reduce_x2<G>(x);
   if (lane == 0) sh->w2[warp] = x;
   __syncthreads();
   if (warp == 0) {
     X2 w = (lane < kTWarps) ? sh->w2[lane] : x2_zero();
     warp_reduce_x2<G>(w);
+    if (!QSUM && (G & G_RES)) w.Q = sh->qown;
     if (sh->broken) w.pad[0] = __uint_as_float(kBadTimeout);
     if (lane < static_cast<int>(sizeof(X2) / 16))
       reinterpret_cast<float4*>(rec)[lane] = reinterpret_cast<const float4*>(&w)[lane];
@@ -1209,6 +1241,10 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
   const T* rt = static_cast<const T*>(c.st);
   SharedTma* sh = c.sh;
   const float beta = P.beta;
+  // the residual rows of the production programs take their fused mass (used
+  // only when the whole residual is zero) from pass 1; the full program (the
+  // only one with F_AT and pass 2) sums it in pass 2, for every row alike
+  constexpr bool QSUM = !((G & G_RES) && !(F & F_AT) && (F & F_LS));
   pass1_and_push<T, F, DS>(ra, rb, rt, c.nv, c.rounds, c.rc, c.lo, c.n, beta, c.dtok, sh, c.rank, c.C,
                        cluster, c.ph, c.slot);
   if constexpr (!R2) {
@@ -1236,6 +1272,11 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
       if (lane == 0) {
 #pragma unroll
         for (int q = 0; q < 4; ++q) sh->lse[q] = lse[q];
+        if (!QSUM) {
+          // this slice's fused mass sum exp(s - LSE(s)), from its own pass-1 record
+          const X1& own = sh->recv1(c.slot, c.C)[c.rank];
+          sh->qown = own.s[3] * ex2((own.ref[3] - lse[3]) * kLog2e);
+        }
         if (c.rank == 0) {
           float ad, bd, td;
           draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td, c.slot);
@@ -1249,11 +1290,11 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
     if constexpr (PER) {
       const ChunkRefill<T> rel{c.rc, &P, sh, c.next, c.lo, c.nv, const_cast<T*>(ra),
                                const_cast<T*>(rb), const_cast<T*>(rt), c.next_only_t};
-      pass2_and_store<T, G, LP, DS, ChunkRefill<T>>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh,
+      pass2_and_store<T, G, LP, DS, ChunkRefill<T>, QSUM>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh,
                                                     P.pass2_rec + slot * 8,
                                                     P.group_mass + slot * P.group_stride, rel);
     } else {
-      pass2_and_store<T, G, LP, DS>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh,
+      pass2_and_store<T, G, LP, DS, NoRelease, QSUM>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh,
                                     P.pass2_rec + slot * 8, P.group_mass + slot * P.group_stride);
     }
   }
