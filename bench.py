@@ -2,11 +2,11 @@
 
 One step = one pass of the whole path over one batch: the C-ABI call
 asymspec_fuse_verify_ex in stochastic mode (row normalisers, delta fusion,
-JSD gate, acceptance tests, residual inverse-CDF draws, fused argmax and the
-per-element accept scan), which is one kernel launch.  The workload is
-B=64, K=7, V=128256 bf16 logits with the Zipf-profile recipe (512 verify
-rows, 394 MB of logits per step, larger than the 129 MB L2; two input sets
-are rotated).
+JSD gate, acceptance tests, residual inverse-CDF draws and the per-element
+accept scan), which is two kernel launches: the fused row kernel and the
+decision kernel.  The workload is B=64, K=7, V=128256 bf16 logits with the
+Zipf-profile recipe (512 verify rows, 394 MB of logits per step, larger than
+the 129 MB L2; two input sets are rotated).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl asymspec|reference]
 
