@@ -314,3 +314,22 @@ def test_xvocab_workspace_layout_and_validation(lib):
              FAKE, small) == A.ERR_WORKSPACE
     assert g(FAKE, FAKE, 30, FAKE, 20, FAKE, FAKE, 10, 4, A.FP32, FAKE, FAKE, FAKE, None,
              FAKE + 16, small + 1) == A.ERR_WORKSPACE
+
+
+def test_plan_of_the_persistent_kernel(lib):
+    # the persistent form keeps the one-shot kernel's slices and one more slot
+    # of pushed pass-1 records (64 bytes per CTA of the cluster)
+    PER = A.LaunchOpts(0, 0, A.KERNEL_PERSIST)
+    TMA = A.LaunchOpts(0, 0, A.KERNEL_TMA)
+    for B, K, V, dtype in ((64, 7, 128256, A.BF16), (1, 4, 32000, A.FP32)):
+        p, t = A.plan(B, K, V, dtype, opts=PER), A.plan(B, K, V, dtype, opts=TMA)
+        assert p.kernel == A.KERNEL_PERSIST and p.cluster_size == t.cluster_size
+        assert p.slice_elems == t.slice_elems
+        assert p.smem_bytes == t.smem_bytes + 64 * t.cluster_size
+    # Qwen3-sized bf16 rows: clusters of 8 leave no room for the second slot
+    # within two CTAs per SM, so the persistent form takes clusters of 10
+    p, t = A.plan(8, 5, 151936, A.BF16, opts=PER), A.plan(8, 5, 151936, A.BF16, opts=TMA)
+    assert (t.cluster_size, p.cluster_size) == (8, 10) and p.smem_bytes <= 113 * 1024
+    with pytest.raises(A.AsymSpecError) as e:      # unaligned rows: no bulk copies
+        A.plan(2, 2, 4099, A.BF16, opts=PER)
+    assert e.value.status == A.ERR_UNSUPPORTED
