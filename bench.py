@@ -333,6 +333,23 @@ def xvocab_timing(torch, A, synth, mode, dev, steps, timed, stream):
             "timing": "CUDA events around the timed calls on the launching stream"}
 
 
+def max_over_ranks(ms: float, dist=None, device="cpu") -> float:
+    """The slowest rank's time: an all-reduce MAX over the process group (the
+    value itself with a single process)."""
+    if dist is None:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_rows_per_s(world: int, rows_per_rank: int, ms_per_step: float) -> float:
+    """Whole-job throughput: every rank verifies its own rows_per_rank rows per
+    step (replicas, weak scaling), in the slowest rank's step time."""
+    return world * rows_per_rank / (ms_per_step * 1e-3)
+
+
 def run_reference(args, workload, rank, world):
     """--impl reference: the float64 CPU oracle, timed on the host cores."""
     from paper_2608_26004_gb300 import synth
@@ -455,12 +472,7 @@ def main():
         if pg:
             pg.barrier()
         torch.cuda.synchronize(dev)
-        ms = e0.elapsed_time(e1)
-        if pg:
-            t = torch.tensor([ms], device=dev)
-            pg.all_reduce(t, op=pg.ReduceOp.MAX)
-            ms = float(t.item())
-        return ms
+        return max_over_ranks(e0.elapsed_time(e1), pg, dev)
 
     # ---- device-resident throughput (the headline value)
     with ClockSampler(local) as clk:
@@ -471,7 +483,7 @@ def main():
               args.steps, max(args.warmup, 3))
     clocks = clk.summary()
     ms_step = ms / args.steps
-    value = world * rows / (ms_step * 1e-3)
+    value = aggregate_rows_per_s(world, rows, ms_step)
     # a step is the fused row kernel and its decision kernel; the roofline is
     # the fused row kernel's own: its mean duration between the events the
     # library recorded around it in every timed step
@@ -542,7 +554,7 @@ def main():
 
     e2e_steps = max(3, min(args.steps, 30))
     ms_e2e = timed(e2e_step, e2e_steps, 3) / e2e_steps
-    e2e_value = world * rows / (ms_e2e * 1e-3)
+    e2e_value = aggregate_rows_per_s(world, rows, ms_e2e)
 
     # ---- the drafter's draw (asymspec_draft_sample), the step upstream of
     # fuse-and-verify: per drafted position one launch over the B rows of the
