@@ -80,8 +80,10 @@ struct __align__(16) X2 {  // pass-2 sums
 // cluster follow it (recv1()).
 struct __align__(16) SharedTma {
   unsigned long long bar[kChunks];  // one mbarrier per chunk
-  X1 w1[kTWarps];                   // per-warp pass-1 records
-  X2 w2[kTWarps];                   // per-warp pass-2 records
+  union {                           // per-warp records, one pass at a time
+    X1 w1[kTWarps];
+    X2 w2[kTWarps];
+  };
   float lse[4];       // the row's normalisers (pass 2 reads them)
   unsigned broken;    // a chunk copy timed out
   int rel[kChunks];   // persistent kernel: warps done with each chunk of the row
@@ -1450,7 +1452,9 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
     // warp 0 keeps the row's draft token, loaded while the slice is in flight
     c.dtok = -1;
     if ((tid >> 5) == 0 && !bonus) c.dtok = P.tokens[static_cast<size_t>(bi) * P.K + k];
-    if (it == 0) __syncthreads();  // the chunk barriers are initialised
+    // the chunk barriers are initialised (first row); warp 0 has read the
+    // previous row's pass-2 records out of w2, which pass 1 reuses as w1
+    __syncthreads();
 
     if constexpr (SEL > 0 && STOCH) {
       constexpr int d = SEL - 1;

@@ -231,10 +231,10 @@ def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
     info = A.plan(8, 5, 151936, A.BF16, opts=TMA)
     assert info.kernel == A.KERNEL_TMA and info.cluster_size == 8
     assert info.smem_bytes <= 113 * 1024
-    # fp32 rows of 151,936 entries: 16 CTAs of 114 KB
+    # fp32 rows of 151,936 entries: 16 CTAs of 113 KB, two per SM
     info = A.plan(256, 4, 151936, A.FP32, opts=TMA)
     assert info.kernel == A.KERNEL_TMA and info.cluster_size == 16
-    assert info.smem_bytes <= 227 * 1024
+    assert info.smem_bytes <= 113 * 1024
     info = A.plan(1, 4, 32000, A.FP32, opts=TMA)
     assert info.kernel == A.KERNEL_TMA and info.cluster_size == 4
     info = A.plan(2, 2, 4099, A.BF16)
@@ -321,15 +321,13 @@ def test_plan_of_the_persistent_kernel(lib):
     # of pushed pass-1 records (64 bytes per CTA of the cluster)
     PER = A.LaunchOpts(0, 0, A.KERNEL_PERSIST)
     TMA = A.LaunchOpts(0, 0, A.KERNEL_TMA)
-    for B, K, V, dtype in ((64, 7, 128256, A.BF16), (1, 4, 32000, A.FP32)):
+    for B, K, V, dtype in ((64, 7, 128256, A.BF16), (8, 5, 151936, A.BF16),
+                           (1, 4, 32000, A.FP32)):
         p, t = A.plan(B, K, V, dtype, opts=PER), A.plan(B, K, V, dtype, opts=TMA)
         assert p.kernel == A.KERNEL_PERSIST and p.cluster_size == t.cluster_size
         assert p.slice_elems == t.slice_elems
         assert p.smem_bytes == t.smem_bytes + 64 * t.cluster_size
-    # Qwen3-sized bf16 rows: clusters of 8 leave no room for the second slot
-    # within two CTAs per SM, so the persistent form takes clusters of 10
-    p, t = A.plan(8, 5, 151936, A.BF16, opts=PER), A.plan(8, 5, 151936, A.BF16, opts=TMA)
-    assert (t.cluster_size, p.cluster_size) == (8, 10) and p.smem_bytes <= 113 * 1024
+        assert p.smem_bytes <= 113 * 1024          # still two CTAs per SM
     with pytest.raises(A.AsymSpecError) as e:      # unaligned rows: no bulk copies
         A.plan(2, 2, 4099, A.BF16, opts=PER)
     assert e.value.status == A.ERR_UNSUPPORTED
