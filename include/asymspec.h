@@ -380,7 +380,8 @@ int asymspec_draft_sample(const void* logits, int rows, int V, int dtype, int mo
  *   uniforms, gate_params as for asymspec_fuse_verify (draft_probs[b][k] is
  *   the drafter's probability of pair draft_index[b][k] under the restricted
  *   softmax); out_accept_len, out_next_token [B] int32 (verifier tokens);
- *   out_next_index [B] int32 or NULL: the emitted pair index; workspace of
+ *   out_next_index [B] int32 or NULL: the emitted pair index (-1 on a data
+ *   error); workspace of
  *   asymspec_xvocab_workspace_bytes(B, K, S, V_d, V_v, dtype) bytes,
  *   256-byte aligned and zeroed before its first use
  *   (asymspec_workspace_reset; every call that completes leaves it fit for
