@@ -6,14 +6,14 @@ JSD gate, acceptance tests, residual inverse-CDF draws and the per-element
 accept scan), which is two kernel launches: the fused row kernel and the
 decision kernel.  The workload is B=64, K=7, V=128256 bf16 logits with the
 Zipf-profile recipe (512 verify rows, 394 MB of logits per step, larger than
-the 129 MB L2; two input sets are rotated).
+the 129 MB L2; four resident input sets are rotated).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl asymspec|reference]
 
 Under torchrun every rank runs its own replica of the workload on its own GPU
 (weak scaling, no collective on the data path); rank 0 prints one JSON line.
 ``--impl reference`` times the float64 CPU oracle on the same workload (a
-bounded sample of batch elements per step) on the host cores.
+bounded sample of batch elements per step) on all the host cores.
 """
 from __future__ import annotations
 
@@ -37,9 +37,11 @@ WORKLOAD_CFG = 2
 FALLBACK_HBM_GBS = 6800.0
 CSRC = os.path.join(ROOT, "paper_2608_26004_gb300", "csrc")
 KERNEL_SRCS = ("asymspec.cu", "device_common.cuh", "kernel_generic.cuh", "kernel_tma.cuh",
-               "kernel_stream.cuh", "kernels.h", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu",
+               "kernels.h", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu",
                "k_tma_bf16_prod.cu", "k_tma_f32_prod.cu", "k_tma_bf16_any_s.cu",
-               "k_tma_f32_any_s.cu", "k_tmap_bf16.cu", "k_tmap_f32.cu")
+               "k_tma_f32_any_s.cu")
+N_SETS = 4          # resident input sets rotated between steps (4 x 394 MB, each > L2)
+DIST_MIN_S = 1.0    # the per-step distribution loop runs at least this long
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fuse_verify_tma_B64_K7_V128256_bf16_traffic.txt")
 REASON_BITS = {
     0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
@@ -178,6 +180,72 @@ class ClockSampler:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
         return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(smax)),
                 "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def percentiles(us):
+    """p10 / p50 / p90 of a list of durations (microseconds)."""
+    q = np.percentile(np.asarray(us, np.float64), [10, 50, 90])
+    return {"p10": float(q[0]), "p50": float(q[1]), "p90": float(q[2]), "n": len(us)}
+
+
+# ---- the oracle over all host cores: one process per core (spawned), each
+# generating its own copy of a bounded sample of the workload's batch elements
+# at start-up, outside the timed region
+_W = {}
+
+
+def _oracle_init(cfg_id: int, nsample: int):
+    from paper_2608_26004_gb300 import synth
+    _W["batch"] = synth.make_config(cfg_id, nb=nsample)
+
+
+def _oracle_element(args):
+    import oracle
+    b, mode_id = args
+    bt = _W["batch"]
+    b = b % bt.B
+    sel = slice(b, b + 1)
+    oracle.fuse_verify(bt.logits_full[sel], bt.logits_comp[sel], bt.logits_ver[sel],
+                       bt.draft_tokens[sel], bt.draft_probs[sel], bt.uniforms[sel],
+                       dtype=bt.dtype, mode=mode_id)
+    return bt.K + 1
+
+
+class OraclePool:
+    """The float64 oracle, as it stands, run over batch elements on every host
+    core (os.cpu_count() spawned processes)."""
+
+    def __init__(self, cfg_id: int, nsample: int):
+        import multiprocessing as mp
+        self.cores = os.cpu_count() or 1
+        self.pool = mp.get_context("spawn").Pool(self.cores, _oracle_init, (cfg_id, nsample))
+        self.next = 0
+
+    def run(self, n_elements: int, mode_id: int) -> int:
+        """n_elements batch elements (cycling over the sample); returns rows done."""
+        items = [(self.next + i, mode_id) for i in range(n_elements)]
+        self.next += n_elements
+        return sum(self.pool.map(_oracle_element, items, chunksize=1))
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+
+
+def oracle_all_cores(cfg_id: int, mode_id: int, seconds: float):
+    """rows/s of the oracle on all host cores for ~`seconds` (after one warm-up
+    element per core)."""
+    pool = OraclePool(cfg_id, nsample=16)
+    try:
+        pool.run(pool.cores, mode_id)
+        t0 = time.perf_counter()
+        rows = 0
+        while time.perf_counter() - t0 < seconds:
+            rows += pool.run(pool.cores, mode_id)
+        el = time.perf_counter() - t0
+        return rows / el, rows, el, pool.cores
+    finally:
+        pool.close()
 
 
 def oracle_rows_per_s(batch, mode_id, seconds: float):
@@ -356,29 +424,26 @@ def aggregate_rows_per_s(world: int, rows_per_rank: int, ms_per_step: float) -> 
 
 
 def run_reference(args, workload, rank, world):
-    """--impl reference: the float64 CPU oracle, timed on the host cores."""
-    from paper_2608_26004_gb300 import synth
+    """--impl reference: the float64 CPU oracle, timed on all the host cores
+    (one batch element per core per step)."""
     if rank != 0:
         return
     mode_id = 1 if args.mode == "stochastic" else 0
-    sample_b = 2
-    batch = synth.make_config(WORKLOAD_CFG, nb=sample_b)
-    for _ in range(args.warmup):
-        oracle_rows_per_s(batch, mode_id, 0.0)
-    t0 = time.perf_counter()
-    rows = 0
-    for s in range(args.steps):
-        b = s % sample_b
-        import oracle
-        oracle.fuse_verify(batch.logits_full[b:b + 1], batch.logits_comp[b:b + 1],
-                           batch.logits_ver[b:b + 1], batch.draft_tokens[b:b + 1],
-                           batch.draft_probs[b:b + 1], batch.uniforms[b:b + 1],
-                           dtype=batch.dtype, mode=mode_id)
-        rows += batch.K + 1
-    el = time.perf_counter() - t0
+    pool = OraclePool(WORKLOAD_CFG, nsample=16)
+    try:
+        for _ in range(max(args.warmup, 1)):
+            pool.run(pool.cores, mode_id)
+        t0 = time.perf_counter()
+        rows = 0
+        for _ in range(args.steps):
+            rows += pool.run(pool.cores, mode_id)
+        el = time.perf_counter() - t0
+    finally:
+        pool.close()
     value = rows / el
-    sample = (f"each step: 1 batch element (K+1={batch.K + 1} rows of V={batch.V}) of "
-              f"{workload.name}, float64 numpy oracle, single thread")
+    sample = (f"each step: {pool.cores} batch elements (one per host core; K+1={workload.K + 1} "
+              f"rows of V={workload.V} each) cycling over the first 16 elements of "
+              f"{workload.name}, float64 numpy oracle, {pool.cores} processes")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "rows/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -386,7 +451,7 @@ def run_reference(args, workload, rank, world):
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": workload.name, "B": workload.B, "K": workload.K,
                    "V": workload.V, "logits": "bf16", "mode": args.mode},
-        "cpu_baseline": {"value": value, "unit": "rows/s", "cores": 1, "kind": "oracle",
+        "cpu_baseline": {"value": value, "unit": "rows/s", "cores": pool.cores, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "rows/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
@@ -426,7 +491,7 @@ def main():
         return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).to(dev)
 
     sets = []
-    for rep in range(2):  # two resident input sets, rotated (each larger than L2)
+    for rep in range(N_SETS):  # resident input sets, rotated (each larger than L2)
         sets.append(dict(
             a=to_dev_logits(batch.logits_full), b=to_dev_logits(batch.logits_comp),
             t=to_dev_logits(batch.logits_ver),
@@ -450,11 +515,16 @@ def main():
         if st != A.OK:
             raise A.AsymSpecError(st, "asymspec_fuse_verify_ex")
 
-    # events the library records around the fused row kernel of every timed
-    # step (asymspec_launch_opts.timing_begin / timing_end), on its stream
+    # the per-step distribution loop: events around every step, and the events
+    # the library records around the fused row kernel of every step
+    # (asymspec_launch_opts.timing_begin / timing_end), all on the one stream.
+    # It runs at least DIST_MIN_S seconds (so that the clock sampler sees it).
+    n_dist = max(args.steps, 64)
+    sev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(n_dist)]
     kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(args.steps)]
-    for b, e in kev:  # torch creates an event at its first record: before taking handles
+           for _ in range(n_dist)]
+    for b, e in kev + sev:  # torch creates an event at its first record: before taking handles
         b.record(stream)
         e.record(stream)
     kopts = [A.LaunchOpts(0, 0, 0, 0, b.cuda_event, e.cuda_event) for b, e in kev]
@@ -479,21 +549,33 @@ def main():
         torch.cuda.synchronize(dev)
         return max_over_ranks(e0.elapsed_time(e1), pg, dev)
 
+    def dist_step(i):
+        j = i % n_dist
+        sev[j][0].record(stream)
+        step(sets[i % N_SETS], kopts[j])
+        sev[j][1].record(stream)
+
     # ---- device-resident throughput (the headline value)
     with ClockSampler(local) as clk:
-        ms = timed(lambda i: step(sets[i % 2]), args.steps, max(args.warmup, 3))
-        # the same K steps again with the library's events around the fused row
-        # kernel (kept out of the headline loop: two records add ~3 us a step)
-        timed(lambda i: step(sets[i % 2], kopts[i] if i < args.steps else None),
-              args.steps, max(args.warmup, 3))
+        ms = timed(lambda i: step(sets[i % N_SETS]), args.steps, max(args.warmup, 3))
+        # the distribution loop (kept out of the headline loop: the records add
+        # a few us a step): per-step and per-kernel events, repeated until it
+        # has run DIST_MIN_S seconds; the last pass's events are kept
+        step_us, kern_us, t0 = [], [], time.time()
+        while True:
+            timed(dist_step, n_dist, max(args.warmup, 3))
+            step_us = [1e3 * b.elapsed_time(e) for b, e in sev]
+            kern_us = [1e3 * b.elapsed_time(e) for b, e in kev]
+            if time.time() - t0 >= DIST_MIN_S:
+                break
     clocks = clk.summary()
     ms_step = ms / args.steps
     value = aggregate_rows_per_s(world, rows, ms_step)
     # a step is the fused row kernel and its decision kernel; the roofline is
     # the fused row kernel's own: its mean duration between the events the
-    # library recorded around it in every timed step
-    launches_per_step = 2 if info.kernel in (A.KERNEL_TMA, A.KERNEL_RING) else 1
-    kernel_ms = float(np.mean([b.elapsed_time(e) for b, e in kev]))
+    # library recorded around it in every step of the distribution loop
+    launches_per_step = 2 if info.kernel == A.KERNEL_TMA else 1
+    kernel_ms = float(np.mean(kern_us)) * 1e-3
     launch_s = kernel_ms * 1e-3
     hbm_peak, peak_kind = peaks()
     achieved = alg_bytes / launch_s / 1e9
@@ -510,23 +592,8 @@ def main():
         if st != A.OK:
             raise A.AsymSpecError(st, "asymspec_fuse_verify_ex")
 
-    ms_o = timed(lambda i: step_o(sets[i % 2]), args.steps, max(args.warmup, 3)) / args.steps
+    ms_o = timed(lambda i: step_o(sets[i % N_SETS]), args.steps, max(args.warmup, 3)) / args.steps
 
-    # ---- the persistent form of the cluster kernel (asymspec_launch_opts.kernel
-    # = ASYMSPEC_KERNEL_PERSIST), same workload and mode, reported alongside
-    popts = [A.LaunchOpts(0, 0, A.KERNEL_PERSIST, 0, b.cuda_event, e.cuda_event) for b, e in kev]
-    popts_plain = A.LaunchOpts(0, 0, A.KERNEL_PERSIST)
-    pinfo = A.plan(B, K, V, A.BF16, gate, popts_plain)
-    ms_p = timed(lambda i: step(sets[i % 2], popts_plain), args.steps,
-                 max(args.warmup, 3)) / args.steps
-    timed(lambda i: step(sets[i % 2], popts[i] if i < args.steps else popts_plain), args.steps,
-          max(args.warmup, 3))
-    kernel_ms_p = float(np.mean([b.elapsed_time(e) for b, e in kev]))
-    persistent = {"kernel": "fuse_verify_tma<T, STOCH, SEL, true>", "ctas": pinfo.ctas,
-                  "cluster_size": pinfo.cluster_size, "ms_per_step": ms_p,
-                  "rows_per_s": world * rows / (ms_p * 1e-3), "launch_us": kernel_ms_p * 1e3,
-                  "hbm_gbs": alg_bytes / (kernel_ms_p * 1e-3) / 1e9,
-                  "frac": alg_bytes / (kernel_ms_p * 1e-3) / 1e9 / hbm_peak}
     alg_bytes_o = algorithmic_bytes(B, K, V, 2, other_mode == A.MODE_STOCHASTIC)
 
     # ---- end to end through the C ABI with host buffers
@@ -582,7 +649,8 @@ def main():
                    "B": B, "K": K, "V": V, "logits": "bf16",
                    "mode": args.mode, "rows_per_gpu": rows, "gamma": 0.5, "beta": 1.0,
                    "divergence": "jsd",
-                   "l2": "inputs larger than L2: 2 resident sets of 394 MB rotated",
+                   "l2": f"inputs larger than L2: {N_SETS} resident sets of "
+                         f"{3 * rows * V * 2 / 1e6:.0f} MB rotated",
                    "cluster_size": info.cluster_size, "ctas": info.ctas,
                    "parallelism": f"replicas x{world}"},
         "hbm_gbs": achieved,
@@ -592,16 +660,18 @@ def main():
                      "algorithmic_bytes_per_launch": alg_bytes,
                      "kernel": "fuse_verify_tma" if info.kernel == A.KERNEL_TMA else str(info.kernel),
                      "launch_us": kernel_ms * 1e3,
+                     "launch_us_pct": percentiles(kern_us),
                      "timing": "CUDA events the library records around the fused row kernel "
-                               "on its stream, in every step of a second timed loop of the same "
-                               "K steps"},
+                               f"on its stream, in every step of a loop of {n_dist} steps "
+                               "(repeated until it has run 1 s; the last pass is kept), "
+                               "separate from the headline loop"},
+        "step_us_pct": percentiles(step_us),
         "e2e": {"value": e2e_value, "unit": "rows/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
         "draft": draft,
         "xvocab": xvocab,
-        "persistent": persistent,
         "other_mode": {"mode": "greedy" if other_mode == A.MODE_GREEDY else "stochastic",
                        "ms_per_step": ms_o, "rows_per_s": world * rows / (ms_o * 1e-3),
                        "hbm_gbs": alg_bytes_o / (ms_o * 1e-3) / 1e9,
@@ -611,11 +681,17 @@ def main():
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         mode_id = 1 if mode == A.MODE_STOCHASTIC else 0
-        rps, nrows, el = oracle_rows_per_s(batch, mode_id, args.cpu_seconds)
+        rps, nrows, el, cores = oracle_all_cores(WORKLOAD_CFG, mode_id, args.cpu_seconds)
+        rps1, nrows1, el1 = oracle_rows_per_s(batch, mode_id, args.cpu_seconds)
         line["cpu_baseline"] = {
-            "value": rps, "unit": "rows/s", "cores": 1, "kind": "oracle",
-            "sample": f"{nrows} rows ({nrows // (K + 1)} batch elements) of {workload.name} "
-                      f"in {el:.1f} s, float64 numpy oracle, single thread"}
+            "value": rps, "unit": "rows/s", "cores": cores, "kind": "oracle",
+            "sample": f"{nrows} rows ({nrows // (K + 1)} batch elements, cycling over the first "
+                      f"16) of {workload.name} in {el:.1f} s, float64 numpy oracle, one "
+                      f"process per host core ({cores})",
+            "single_thread": {
+                "value": rps1, "unit": "rows/s", "cores": 1,
+                "sample": f"{nrows1} rows ({nrows1 // (K + 1)} batch elements) of "
+                          f"{workload.name} in {el1:.1f} s, float64 numpy oracle, one thread"}}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if pg:

@@ -102,8 +102,7 @@ typedef struct {
  * (Eq. 1), or one of the alternatives its mechanism ablation compares,
  * delta = a (raw-augmented) and delta = t - b (SCD-style).  Only the fused
  * scores change: the gate (Eq. 3) and the acceptance test (Eq. 4) keep their
- * own a, b and t.  The ring and streaming kernels implement a - b only
- * (ASYMSPEC_ERR_UNSUPPORTED when forced with another source). */
+ * own a, b and t. */
 #define ASYMSPEC_DELTA_AB 0
 #define ASYMSPEC_DELTA_A 1
 #define ASYMSPEC_DELTA_TB 2
@@ -113,8 +112,8 @@ typedef struct {
 typedef struct {
   int32_t cluster_size;   /* CTAs per row triple: 1 to 16 */
   int32_t block_threads;  /* reserved, must be 0 (256 threads per CTA) */
-  int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC, _TMA, _STREAM, _RING or _PERSIST */
-  int32_t pad;            /* reserved, must be 0 */
+  int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC or ASYMSPEC_KERNEL_TMA */
+  int32_t test_flags;     /* 0, or test hooks (ASYMSPEC_TEST_*); other bits reserved, 0 */
   /* Optional cudaEvent_t handles (or NULL): recorded on the call's stream
    * immediately before and after the launch of the fused row kernel (not
    * around the decision kernel that follows it), so that a caller can time
@@ -123,21 +122,20 @@ typedef struct {
   void* timing_end;
 } asymspec_launch_opts;
 
+/* Test hook (asymspec_launch_opts.test_flags), for tests of the timeout
+ * path only: every bulk-copy wait of ASYMSPEC_KERNEL_TMA gives up at once,
+ * as if its time limit (200 ms) had passed, while the copies still land.
+ * Each CTA then takes its timeout branch: it marks its row, still reaches
+ * every cluster barrier, and before it exits waits (with the normal limit)
+ * for its copies in flight; every batch element comes back as a data error
+ * (accept_len = next_token = -1) with ASYMSPEC_DATA_TIMEOUT in the error
+ * word.  The generic kernel has no bounded waits and ignores it. */
+#define ASYMSPEC_TEST_COPY_GIVE_UP 1
+
 /* Kernels (asymspec_launch_opts.kernel, asymspec_launch_info.kernel). */
 #define ASYMSPEC_KERNEL_GENERIC 1  /* one cluster per row; any element-aligned input */
 #define ASYMSPEC_KERNEL_TMA 2      /* one cluster per row, chunked 1-D bulk copies, per-row
-                                      programs; rows 16-byte aligned; debug outputs */
-#define ASYMSPEC_KERNEL_STREAM 3   /* persistent grid over row tiles: pass 1 reads each tile from
-                                      HBM, pass 2 re-reads it from L2; rows 16-byte aligned and a
-                                      workspace of asymspec_workspace_bytes(); on request only */
-#define ASYMSPEC_KERNEL_RING 4     /* persistent clusters: pass 1 through a ring of bulk copies,
-                                      pass 2 from L2; rows 16-byte aligned; no debug outputs;
-                                      on request only */
-#define ASYMSPEC_KERNEL_PERSIST 5  /* persistent form of ASYMSPEC_KERNEL_TMA: as many clusters
-                                      as the device holds, each taking every G-th row; each
-                                      CTA's slice buffer is refilled with the cluster's next
-                                      row chunk by chunk as pass 2 finishes with it; rows
-                                      16-byte aligned; debug outputs */
+                                      programs, then a decision kernel; rows 16-byte aligned */
 
 /* What a launch would use (filled by asymspec_plan). */
 typedef struct {
@@ -148,7 +146,7 @@ typedef struct {
   int64_t ctas;            /* CTAs in the grid */
   int32_t vector_path;     /* 1 if rows qualify for 16-byte copies (V * element size % 16 == 0) */
   int32_t max_active_clusters; /* clusters the device can hold at once (0 if unknown) */
-  int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC, _TMA, _STREAM, _RING or _PERSIST */
+  int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC or ASYMSPEC_KERNEL_TMA */
 } asymspec_launch_info;
 
 /* Fills *p with the paper's defaults: gamma 0.5, beta 1.0, lambda 0.1,
@@ -161,9 +159,8 @@ void asymspec_default_gate_params(asymspec_gate_params* p);
  * record per row and 4 B of ticket per element (all the generic kernel
  * needs); then, for ASYMSPEC_KERNEL_TMA with clusters of C CTAs, 48 B of
  * pass-1 results per row and 352 B per row and CTA of pass-2 record and
- * inverse-CDF group masses, which its decision kernel reads; or instead the
- * streaming kernel's counters and tile records.  With less than the TMA
- * part the automatic choice falls back to the generic kernel.  The tickets
+ * inverse-CDF group masses, which its decision kernel reads.  With less than
+ * the TMA part the automatic choice falls back to the generic kernel.  The tickets
  * must be zero before the first use (cudaMemset or
  * asymspec_workspace_reset); every call that completes leaves them zero
  * again, and every other part is written before it is read.  Two calls in
@@ -239,9 +236,10 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
  * launches of asymspec_fuse_verify_ex.  Nothing is allocated: no
  * cudaMalloc, cudaMallocAsync, cudaFree or library call that allocates.
  *
- * Set-up: the first call on each device looks up the array's device address
- * with cudaGetSymbolAddress (return code checked, ASYMSPEC_ERR_CUDA on
- * failure) and caches it; that first call may load the module, so make it
+ * Set-up: every call looks up the array's device address in the current
+ * device's context with cudaGetSymbolAddress (return code checked,
+ * ASYMSPEC_ERR_CUDA on failure), so the address stays right after a
+ * cudaDeviceReset.  The first call in a context may load the module: make it
  * before any stream capture begins on that device.
  *
  * Concurrency: there is one scratch array per device.  Calls that overlap in

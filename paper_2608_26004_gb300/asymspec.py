@@ -78,17 +78,16 @@ DELTA_AB = 0   # delta = a - b (Eq. 1)
 DELTA_A = 1    # delta = a (raw-augmented)
 DELTA_TB = 2   # delta = t - b (SCD-style)
 
+TEST_COPY_GIVE_UP = 1  # asymspec_launch_opts.test_flags: the copy waits give up at once
+
 KERNEL_AUTO = 0
 KERNEL_GENERIC = 1
 KERNEL_TMA = 2
-KERNEL_STREAM = 3
-KERNEL_RING = 4
-KERNEL_PERSIST = 5
 
 
 class LaunchOpts(ctypes.Structure):
     _fields_ = [("cluster_size", ctypes.c_int32), ("block_threads", ctypes.c_int32),
-                ("kernel", ctypes.c_int32), ("pad", ctypes.c_int32),
+                ("kernel", ctypes.c_int32), ("test_flags", ctypes.c_int32),
                 ("timing_begin", ctypes.c_void_p), ("timing_end", ctypes.c_void_p)]
 
 
@@ -344,7 +343,7 @@ class FuseVerify:
                  uniforms=None, *, gamma=0.5, beta=1.0, lam=0.1, mode=MODE_GREEDY,
                  divergence=DIV_JSD, fuse_bonus=False, row_stats=False, row_tokens=False,
                  fused_logprobs=False, cluster_size=0, kernel=KERNEL_AUTO, out=None,
-                 delta_source=DELTA_AB):
+                 delta_source=DELTA_AB, test_flags=0):
         import torch
         B, K1, V = logits_full.shape
         K = K1 - 1
@@ -374,7 +373,8 @@ class FuseVerify:
         if fused_logprobs and "fused_logprobs" not in res:
             res["fused_logprobs"] = torch.empty(B, K1, V, dtype=torch.float32, device=dev)
         gate = gate_params(gamma, beta, lam, mode, divergence, fuse_bonus, delta_source)
-        opts = LaunchOpts(cluster_size, 0, kernel) if (cluster_size or kernel) else None
+        opts = (LaunchOpts(cluster_size, 0, kernel, test_flags)
+                if (cluster_size or kernel or test_flags) else None)
         stream = torch.cuda.current_stream(dev).cuda_stream
         st = fuse_verify_ex(
             _ptr(logits_full), _ptr(logits_comp), _ptr(logits_ver), _ptr(draft_tokens),

@@ -1,26 +1,23 @@
 // AsymSpec per-step fuse-and-verify on GB300 (sm_103a): host side of the C ABI
-// declared in include/asymspec.h, and the launch of its three kernels.
+// declared in include/asymspec.h, and the launch of its kernels.
 //
 //   fuse_verify_tma      (kernel_tma.cuh) one cluster per row, each CTA's
 //                        slice brought in by chunked 1-D bulk copies, per-row
-//                        programs; the default for 16-byte aligned rows.
-//   fuse_verify_stream   (kernel_stream.cuh) persistent grid over row tiles;
-//                        pass 1 reads each tile from HBM, pass 2 from L2;
-//                        on request.
+//                        programs; the default for 16-byte aligned rows.  Its
+//                        rows are decided, and Algorithm 1's scan run, by
+//                        decide_rows, a second launch.
 //   fuse_verify_generic  (kernel_generic.cuh) one cluster per row, any
-//                        element-aligned input.
+//                        element-aligned input; folds the scan into the same
+//                        launch through a per-element ticket in the workspace.
 //
-// Each reads every logit row from HBM once and folds Algorithm 1's
-// sequential scan into the same launch through a per-element ticket in the
-// workspace.
+// Each reads every logit row from HBM once.
 #include <algorithm>
 #include <mutex>
 
 #include "device_common.cuh"
 #include "kernel_generic.cuh"
-#include "kernel_ring.cuh"
+#include "kernel_tma.cuh"
 #include "kernel_draft.cuh"
-#include "kernel_stream.cuh"
 #include "kernel_xvocab.cuh"
 #include "kernels.h"
 
@@ -75,12 +72,12 @@ bool plan_generic(int V, int elt, int VE, int forced_C, Plan* pl) {
 // TMA kernel: first C whose slice (and shared state) fits two CTAs per SM,
 // else the first that fits one; a slice holds at most kMaxRounds vectors
 // per thread.
-bool plan_tma(int V, int elt, int forced_C, Plan* pl, bool persistent = false) {
+bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
   const int VE = 16 / elt;
   auto fill = [&](int C) {
     const long long per = (static_cast<long long>(V) + C - 1) / C;
     const long long W = round_up_ll(per, VE);
-    const int shared_bytes = shared_tma_bytes(C, persistent);
+    const int shared_bytes = shared_tma_bytes(C);
     const long long sh_off = round_up_ll(3 * W * elt, 128);
     pl->C = C;
     pl->W = static_cast<int>(W);
@@ -96,26 +93,6 @@ bool plan_tma(int V, int elt, int forced_C, Plan* pl, bool persistent = false) {
   for (int C : kClusterOrder)
     if (fill(C)) return true;
   return false;
-}
-
-// Persistent ring kernel: clusters of 8 (16 when a slice of 8 would take
-// more than kRMaxRounds rounds); the slice is not held in shared memory, so
-// smaller clusters (more entries per thread) work too.
-bool plan_ring(int V, int elt, int forced_C, Plan* pl) {
-  const int VE = 16 / elt;
-  auto fill = [&](int C) {
-    const long long per = (static_cast<long long>(V) + C - 1) / C;
-    const long long W = round_up_ll(per, VE);
-    const long long rounds = (W / VE + kTThreads - 1) / kTThreads;
-    pl->C = C;
-    pl->W = static_cast<int>(W);
-    pl->sh_off = 0;
-    pl->smem = ring_smem_bytes(C);
-    pl->group_stride = static_cast<int>(rounds) * kTWarps;
-    return pl->smem <= kMaxSmem && rounds <= kRMaxRounds;
-  };
-  if (forced_C > 0) return fill(forced_C);
-  return fill(8) || fill(16);
 }
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -136,8 +113,7 @@ struct TmaLayout {
   size_t stat, p2rec, groups, total;
 };
 
-// group_stride: floats of group masses per row and CTA (kGroupsMax for the
-// one-shot kernel, 8 per round for the ring kernel).
+// group_stride: floats of group masses per row and CTA.
 TmaLayout tma_layout(int B, int K, int C, int group_stride = kGroupsMax) {
   TmaLayout L;
   const size_t R = static_cast<size_t>(B) * (K + 1);
@@ -152,109 +128,18 @@ TmaLayout tma_layout(int B, int K, int C, int group_stride = kGroupsMax) {
   return L;
 }
 
-// Workspace of the streaming kernel: the cluster kernels' records and
-// tickets first (same offsets), then the per-row and per-tile state.
-struct StreamLayout {
-  int NT, TS;
-  size_t tickets, p1cnt, p2cnt, ready, tags, stat, p1rec, p2rec, groups, total;
-};
-
-StreamLayout stream_layout(int B, int K, int V, int elt) {
-  StreamLayout L;
-  const size_t R = static_cast<size_t>(B) * (K + 1);
-  L.TS = kSRounds * kSThreads * (16 / elt);
-  L.NT = (V + L.TS - 1) / L.TS;
-  const size_t NT = static_cast<size_t>(L.NT);
-  size_t off = ws_records_bytes(B, K);
-  L.tickets = off;
-  off += round_up(static_cast<size_t>(B) * sizeof(unsigned), 256);
-  L.p1cnt = off;
-  off += round_up(R * sizeof(unsigned), 256);
-  L.p2cnt = off;
-  off += round_up(R * sizeof(unsigned), 256);
-  L.ready = off;
-  off += round_up(R * sizeof(unsigned), 256);
-  L.tags = off;
-  off += round_up(R * 4 * sizeof(unsigned long long), 256);
-  L.stat = off;
-  off += round_up(R * sizeof(RowStat), 256);
-  L.p1rec = off;
-  off += round_up(R * NT * sizeof(X1), 256);
-  L.p2rec = off;
-  off += round_up(R * NT * sizeof(X2), 256);
-  L.groups = off;
-  off += round_up(R * NT * kSGroups * sizeof(float), 256);
-  L.total = off;
-  return L;
-}
-
-// The streaming kernel's tiles stay below 2^31 entries of look-ahead and
-// items; rows longer than this many tiles use the cluster kernels.
-constexpr int kMaxStreamTiles = 31;
-
-// debug_out: the call asks for row statistics or fused log-probs, which only
-// the one-shot kernels produce; delta_ab: the delta source is a - b, the only
-// one the ring and streaming kernels implement.
-int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_opts* opts,
-              bool vec_ok, size_t ws_bytes, bool debug_out, bool delta_ab, Plan* pl) {
+int make_plan(int B, int K, int V, int dtype, const asymspec_launch_opts* opts, bool vec_ok,
+              size_t ws_bytes, Plan* pl) {
   const int elt = elt_size(dtype);
   const int forced_C = (opts && opts->cluster_size > 0) ? opts->cluster_size : 0;
   const int forced_kernel = opts ? opts->kernel : 0;
   if (forced_C < 0 || forced_C > 16) return ASYMSPEC_ERR_INVALID_ARG;
   if (forced_kernel != 0 && forced_kernel != ASYMSPEC_KERNEL_GENERIC &&
-      forced_kernel != ASYMSPEC_KERNEL_TMA && forced_kernel != ASYMSPEC_KERNEL_STREAM &&
-      forced_kernel != ASYMSPEC_KERNEL_RING && forced_kernel != ASYMSPEC_KERNEL_PERSIST)
+      forced_kernel != ASYMSPEC_KERNEL_TMA)
     return ASYMSPEC_ERR_INVALID_ARG;
   pl->rows = static_cast<long long>(B) * (K + 1);
   pl->vector_path = vec_ok;
-  const StreamLayout L = stream_layout(B, K, V, elt);
-  const bool stream_ok = vec_ok && L.NT <= kMaxStreamTiles && ws_bytes >= L.total;
-  (void)stream_ok;  // measured slower than the cluster kernel: chosen only on request
-  if (forced_kernel == ASYMSPEC_KERNEL_STREAM) {
-    if (!vec_ok || !delta_ab) return ASYMSPEC_ERR_UNSUPPORTED;
-    if (L.NT > kMaxStreamTiles) return ASYMSPEC_ERR_TOO_LARGE;
-    if (ws_bytes < L.total) return ASYMSPEC_ERR_WORKSPACE;
-    pl->kernel = ASYMSPEC_KERNEL_STREAM;
-    pl->VE = 16 / elt;
-    pl->C = 1;
-    pl->W = L.TS;
-    pl->sh_off = 0;
-    pl->smem = 0;
-    pl->ctas = 0;  // set at launch from the device's occupancy
-    return ASYMSPEC_OK;
-  }
   if (ws_bytes < cluster_ws_bytes(B, K)) return ASYMSPEC_ERR_WORKSPACE;
-  // the persistent ring kernel on request only: measured slower than the
-  // one-shot kernel on the headline workload (pass 2 misses L2 at this reuse
-  // distance, and warps wait on warp 0's producer and combine work)
-  if (forced_kernel == ASYMSPEC_KERNEL_RING) {
-    Plan r = *pl;
-    if (vec_ok && !debug_out && delta_ab && plan_ring(V, elt, forced_C, &r) &&
-        ws_bytes >= tma_layout(B, K, r.C, r.group_stride).total) {
-      *pl = r;
-      pl->kernel = ASYMSPEC_KERNEL_RING;
-      pl->VE = 16 / elt;
-      pl->ctas = 0;  // set at launch from the device's cluster occupancy
-      return ASYMSPEC_OK;
-    }
-    if (forced_kernel == ASYMSPEC_KERNEL_RING) {
-      if (!vec_ok || debug_out || !delta_ab) return ASYMSPEC_ERR_UNSUPPORTED;
-      return (r.C > 0 && r.group_stride > 0 &&
-              ws_bytes < tma_layout(B, K, r.C, r.group_stride).total)
-                 ? ASYMSPEC_ERR_WORKSPACE
-                 : ASYMSPEC_ERR_TOO_LARGE;
-    }
-  }
-  if (forced_kernel == ASYMSPEC_KERNEL_PERSIST) {
-    // the persistent form of the cluster kernel: same slices, on request
-    if (!vec_ok) return ASYMSPEC_ERR_UNSUPPORTED;
-    if (!plan_tma(V, elt, forced_C, pl, true)) return ASYMSPEC_ERR_TOO_LARGE;
-    if (ws_bytes < tma_layout(B, K, pl->C).total) return ASYMSPEC_ERR_WORKSPACE;
-    pl->kernel = ASYMSPEC_KERNEL_PERSIST;
-    pl->VE = 16 / elt;
-    pl->ctas = 0;  // set at launch from the device's cluster occupancy
-    return ASYMSPEC_OK;
-  }
   bool ok = false;
   if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, pl)) {
     // the TMA kernel leaves each row's results in the workspace; the generic
@@ -281,20 +166,11 @@ int make_plan(int B, int K, int V, int dtype, bool stoch, const asymspec_launch_
 
 using KernelFn = const void*;  // a __global__ function taking KParams (or SParams)
 
-KernelFn pick_ring(int dtype, bool stoch);
-
 // sel: the TMA kernel's program set (tma_program_set; 0 = run-time dispatch)
 KernelFn pick_kernel(const Plan& pl, int dtype, bool stoch, int sel = 0) {
-  if (pl.kernel == ASYMSPEC_KERNEL_RING) return pick_ring(dtype, stoch);
   if (pl.kernel == ASYMSPEC_KERNEL_TMA)
     return dtype == ASYMSPEC_FP32 ? tma_kernel_f32(stoch, sel) : tma_kernel_bf16(stoch, sel);
-  if (pl.kernel == ASYMSPEC_KERNEL_PERSIST)
-    return dtype == ASYMSPEC_FP32 ? tmap_kernel_f32(stoch, sel) : tmap_kernel_bf16(stoch, sel);
   return generic_kernel(dtype, pl.vector_path, stoch);
-}
-
-KernelFn pick_ring(int dtype, bool stoch) {
-  return dtype == ASYMSPEC_FP32 ? ring_kernel_f32(stoch) : ring_kernel_bf16(stoch);
 }
 
 KernelFn pick_decide(int dtype, bool stoch) {
@@ -338,9 +214,7 @@ cudaLaunchConfig_t launch_config(const Plan& pl, long long ctas, cudaStream_t st
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.gridDim = dim3(static_cast<unsigned>(ctas));
-  cfg.blockDim = dim3(pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads
-                      : pl.kernel == ASYMSPEC_KERNEL_RING  ? kRThreads
-                                                            : kTThreads);
+  cfg.blockDim = dim3(pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : kTThreads);
   cfg.dynamicSmemBytes = pl.smem;
   cfg.stream = stream;
   cfg.attrs = attr;
@@ -371,65 +245,6 @@ cudaError_t active_clusters(KernelFn fn, const Plan& pl, int device, int* out) {
   return cudaSuccess;
 }
 
-using StreamFn = const void*;  // fuse_verify_stream<T, STOCH>
-
-StreamFn pick_stream(int dtype, bool stoch) {
-  if (dtype == ASYMSPEC_FP32) return stoch ? stream_kernel_f32_stoch() : stream_kernel_f32_greedy();
-  return stoch ? stream_kernel_bf16_stoch() : stream_kernel_bf16_greedy();
-}
-
-// Resident CTAs of a streaming kernel on a device (cached): the persistent
-// grid, all of whose CTAs must run at once.
-struct GridEntry {
-  const void* fn;
-  int device, grid;
-};
-GridEntry g_grid[16];
-int g_grid_count = 0;
-
-cudaError_t stream_grid(StreamFn fn, int device, int* out) {
-  const void* f = fn;
-  {
-    std::lock_guard<std::mutex> lock(g_mu);
-    for (int i = 0; i < g_grid_count; ++i)
-      if (g_grid[i].fn == f && g_grid[i].device == device) {
-        *out = g_grid[i].grid;
-        return cudaSuccess;
-      }
-  }
-  int per_sm = 0, sms = 0;
-  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kRingBytes);
-  if (e != cudaSuccess) return e;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kSThreads, kRingBytes);
-  if (e != cudaSuccess) return e;
-  e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
-  if (e != cudaSuccess) return e;
-  const int grid = per_sm * sms;
-  std::lock_guard<std::mutex> lock(g_mu);
-  if (g_grid_count < 16) g_grid[g_grid_count++] = {f, device, grid};
-  *out = grid;
-  return cudaSuccess;
-}
-
-// The row programs of the streaming kernel: [0] draft rows, [1] the bonus row.
-void stream_programs(const asymspec_gate_params& gp, bool full, bool logprobs, bool tokens,
-                     int (&prog)[2]) {
-  const bool jsd = gp.divergence == ASYMSPEC_DIV_JSD;
-  const bool kl = gp.divergence == ASYMSPEC_DIV_KL;
-  if (full) {
-    int p = jsd ? PG_FULL_JSD : kl ? PG_FULL_KL : PG_FULL_NONE;
-    if (logprobs) p += PG_FULL_JSD_LP - PG_FULL_JSD;
-    prog[0] = prog[1] = p;
-  } else if (gp.mode == ASYMSPEC_MODE_GREEDY) {
-    prog[0] = jsd ? PG_GREEDY_DRAFT_JSD : kl ? PG_GREEDY_DRAFT_KL : PG_GREEDY_DRAFT_NONE;
-    prog[1] = gp.fuse_bonus ? PG_GREEDY_BONUS_S : PG_GREEDY_BONUS_T;
-  } else {
-    const int base = jsd ? PG_STOCH_DRAFT_JSD : kl ? PG_STOCH_DRAFT_KL : PG_STOCH_DRAFT_NONE;
-    prog[0] = tokens ? base + (PG_STOCH_DRAFT_JSD_TOK - PG_STOCH_DRAFT_JSD) : base;
-    prog[1] = tokens ? PG_STOCH_BONUS_TOK : PG_STOCH_BONUS;
-  }
-}
-
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 int check_params(const asymspec_gate_params* gp) {
@@ -450,7 +265,8 @@ int check_params(const asymspec_gate_params* gp) {
 }
 
 int check_opts(const asymspec_launch_opts* opts) {
-  if (opts && (opts->block_threads != 0 || opts->pad != 0)) return ASYMSPEC_ERR_INVALID_ARG;
+  if (opts && opts->block_threads != 0) return ASYMSPEC_ERR_INVALID_ARG;
+  if (opts && (opts->test_flags & ~ASYMSPEC_TEST_COPY_GIVE_UP) != 0) return ASYMSPEC_ERR_INVALID_ARG;
   if (opts && ((opts->timing_begin == nullptr) != (opts->timing_end == nullptr)))
     return ASYMSPEC_ERR_INVALID_ARG;
   return ASYMSPEC_OK;
@@ -475,24 +291,18 @@ static_assert(kStaticScratchBytes >= static_cast<size_t>(ASYMSPEC_STATIC_MAX_ROW
               "the static scratch holds the generic kernel's records and tickets");
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-// Device address of g_static_scratch, looked up once per device.
+// Device address of g_static_scratch in the current device's context, looked
+// up on every call: a cached address would outlive a context that
+// cudaDeviceReset tore down (the module, and the array, are loaded again in
+// the next context).  Once the module is loaded the lookup is a host-side
+// table read; the first lookup in a context may load the module.
 constexpr int kMaxDevices = 64;
-std::mutex g_static_mu;
-void* g_static_addr[kMaxDevices] = {};
 
 int static_scratch(void** out) {
-  int device = 0;
-  cudaError_t e = cudaGetDevice(&device);
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
   if (e != cudaSuccess) return cuda_fail(e);
-  if (device < 0 || device >= kMaxDevices) return ASYMSPEC_ERR_UNSUPPORTED;
-  std::lock_guard<std::mutex> lock(g_static_mu);
-  if (!g_static_addr[device]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_static_scratch);
-    if (e != cudaSuccess) return cuda_fail(e);
-    g_static_addr[device] = p;
-  }
-  *out = g_static_addr[device];
+  *out = p;
   return ASYMSPEC_OK;
 }
 
@@ -577,25 +387,10 @@ void asymspec_default_gate_params(asymspec_gate_params* p) {
 }
 
 size_t asymspec_workspace_bytes(int B, int K, int V) {
+  (void)V;
   if (B < 1 || K < 1) return 0;
-  // the TMA kernel's layout for the largest cluster, and the ring kernel's
-  // for every cluster size it may take
-  size_t n = tma_layout(B, K, 16).total;
-  if (V >= 2) {
-    for (int elt : {2, 4})
-      for (int C : {1, 2, 4, 8, 16}) {
-        Plan r = {};
-        if (plan_ring(V, elt, C, &r)) n = std::max(n, tma_layout(B, K, C, r.group_stride).total);
-      }
-  }
-  if (V >= 2) {
-    // the larger of the two dtypes' streaming layouts (fp32 has more tiles)
-    const StreamLayout L4 = stream_layout(B, K, V, 4);
-    if (L4.NT <= kMaxStreamTiles) n = std::max(n, L4.total);
-    const StreamLayout L2 = stream_layout(B, K, V, 2);
-    if (L2.NT <= kMaxStreamTiles) n = std::max(n, L2.total);
-  }
-  return n;
+  // the TMA kernel's layout for the largest cluster
+  return tma_layout(B, K, 16).total;
 }
 
 int asymspec_workspace_reset(void* workspace, size_t workspace_bytes, void* stream) {
@@ -618,33 +413,10 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
   if (st) return st;
   const bool vec_ok = (static_cast<long long>(V) * elt_size(dtype)) % 16 == 0;
   Plan pl = {};
-  st = make_plan(B, K, V, dtype, gp.mode == ASYMSPEC_MODE_STOCHASTIC, opts, vec_ok,
-                 asymspec_workspace_bytes(B, K, V), false,
-                 (gp.flags & ASYMSPEC_FLAG_DELTA_MASK) == ASYMSPEC_DELTA_AB, &pl);
+  st = make_plan(B, K, V, dtype, opts, vec_ok, asymspec_workspace_bytes(B, K, V), &pl);
   if (st) return st;
-  if (pl.kernel == ASYMSPEC_KERNEL_STREAM) {
-    out->cluster_size = 1;
-    out->block_threads = kSThreads;
-    out->slice_elems = pl.W;
-    out->smem_bytes = kRingBytes;
-    out->ctas = 0;
-    out->vector_path = 1;
-    out->max_active_clusters = 0;
-    out->kernel = pl.kernel;
-    int device = 0, grid = 0;
-    if (cudaGetDevice(&device) == cudaSuccess &&
-        stream_grid(pick_stream(dtype, gp.mode == ASYMSPEC_MODE_STOCHASTIC), device, &grid) ==
-            cudaSuccess) {
-      out->ctas = grid;
-      out->max_active_clusters = grid;
-    }
-    cudaGetLastError();
-    return ASYMSPEC_OK;
-  }
   out->cluster_size = pl.C;
-  out->block_threads = pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads
-                       : pl.kernel == ASYMSPEC_KERNEL_RING  ? kRThreads
-                                                             : kTThreads;
+  out->block_threads = pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : kTThreads;
   out->slice_elems = pl.W;
   out->smem_bytes = pl.smem;
   out->ctas = pl.ctas;
@@ -661,9 +433,6 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
     if (fn && prepare_kernel(fn, device) == cudaSuccess &&
         active_clusters(fn, pl, device, &ncl) == cudaSuccess)
       out->max_active_clusters = ncl;
-    // the persistent kernels launch the clusters the device holds, at most one per row
-    if (pl.kernel == ASYMSPEC_KERNEL_RING || pl.kernel == ASYMSPEC_KERNEL_PERSIST)
-      out->ctas = std::min(static_cast<long long>(ncl), pl.rows) * pl.C;
   }
   cudaGetLastError();
   return ASYMSPEC_OK;
@@ -705,9 +474,7 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   const bool vec_ok = (static_cast<long long>(V) * elt) % 16 == 0 && aligned(logits_full, 16) &&
                       aligned(logits_comp, 16) && aligned(logits_ver, 16);
   Plan pl = {};
-  st = make_plan(B, K, V, dtype, stoch, opts, vec_ok, workspace_bytes,
-                 out_row_stats || out_fused_logprobs,
-                 (gp.flags & ASYMSPEC_FLAG_DELTA_MASK) == ASYMSPEC_DELTA_AB, &pl);
+  st = make_plan(B, K, V, dtype, opts, vec_ok, workspace_bytes, &pl);
   if (st) return st;
 
   KParams P;
@@ -748,86 +515,27 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   P.row_stat = nullptr;
   P.pass2_rec = nullptr;
   P.group_mass = nullptr;
+  // the chunk waits of the TMA kernel: bounded, or (test hook) giving up at once
+  P.copy_wait_ns =
+      (opts && (opts->test_flags & ASYMSPEC_TEST_COPY_GIVE_UP)) ? 0ull : kCopyTimeoutNs;
   P.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) +
                                               ws_records_bytes(B, K));
 
   int device = 0;
   cudaError_t e = cudaGetDevice(&device);
   if (e != cudaSuccess) return cuda_fail(e);
-  if (pl.kernel == ASYMSPEC_KERNEL_STREAM) {
-    const StreamLayout L = stream_layout(B, K, V, elt);
-    char* base = static_cast<char*>(workspace);
-    SParams S;
-    S.P = P;
-    S.ws.recs = reinterpret_cast<int4*>(base);
-    S.ws.tickets = reinterpret_cast<unsigned*>(base + L.tickets);
-    S.ws.p1cnt = reinterpret_cast<unsigned*>(base + L.p1cnt);
-    S.ws.p2cnt = reinterpret_cast<unsigned*>(base + L.p2cnt);
-    S.ws.ready = reinterpret_cast<unsigned*>(base + L.ready);
-    S.ws.tags = reinterpret_cast<unsigned long long*>(base + L.tags);
-    S.ws.stat = reinterpret_cast<RowStat*>(base + L.stat);
-    S.ws.p1rec = reinterpret_cast<X1*>(base + L.p1rec);
-    S.ws.p2rec = reinterpret_cast<X2*>(base + L.p2rec);
-    S.ws.groups = reinterpret_cast<float*>(base + L.groups);
-    S.P.recs = S.ws.recs;
-    S.P.tickets = S.ws.tickets;
-    S.NT = L.NT;
-    S.TS = L.TS;
-    StreamFn fn = pick_stream(dtype, stoch);
-    int grid = 0;
-    e = stream_grid(fn, device, &grid);
-    if (e != cudaSuccess) return cuda_fail(e);
-    if (grid < 1) return ASYMSPEC_ERR_UNSUPPORTED;
-    // pass 2 of row r follows pass 1 of row r + D: D covers 1.5 waves of the grid
-    const long long R = pl.rows;
-    const long long per_step = 2ll * L.NT;
-    long long D = (3ll * grid + 2 * per_step - 1) / (2 * per_step);
-    D = std::max(2ll, std::min(D, R));
-    S.D = static_cast<int>(D);
-    S.NI = (R + D) * per_step;
-    stream_programs(gp, P.full != 0, out_fused_logprobs != nullptr, out_row_tokens != nullptr,
-                    S.program);
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeCooperative;
-    attr[0].val.cooperative = 1;
-    cfg.gridDim = dim3(static_cast<unsigned>(grid));
-    cfg.blockDim = dim3(kSThreads);
-    cfg.dynamicSmemBytes = kRingBytes;
-    cfg.stream = static_cast<cudaStream_t>(stream);
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    void* args[] = {&S};
-    e = record_timing(opts, true, cfg.stream);
-    if (e == cudaSuccess) e = cudaLaunchKernelExC(&cfg, fn, args);
-    if (e == cudaSuccess) e = record_timing(opts, false, cfg.stream);
-    if (e != cudaSuccess) return cuda_fail(e);
-    return ASYMSPEC_OK;
-  }
   KernelFn fn = pick_kernel(pl, dtype, stoch,
                             tma_program_set(stoch, gp.divergence, gp.fuse_bonus != 0, P.full != 0,
                                             P.want_tokens != 0, P.delta_src));
-  // the persistent kernel exists for the production program sets only (no
-  // debug outputs, no per-row tokens in stochastic mode, delta = a - b)
   if (!fn) return ASYMSPEC_ERR_UNSUPPORTED;
   e = prepare_kernel(fn, device);
   if (e != cudaSuccess) return cuda_fail(e);
-  // The one-shot kernels launch one cluster per row; the persistent ring
-  // kernel as many clusters as the device holds at once (at most one per row).
-  long long ctas = pl.ctas;
-  if (pl.kernel == ASYMSPEC_KERNEL_RING || pl.kernel == ASYMSPEC_KERNEL_PERSIST) {
-    int ncl = 0;
-    e = active_clusters(fn, pl, device, &ncl);
-    if (e != cudaSuccess) return cuda_fail(e);
-    if (ncl < 1) return ASYMSPEC_ERR_UNSUPPORTED;
-    ctas = std::min(static_cast<long long>(ncl), pl.rows) * pl.C;
-  }
+  const long long ctas = pl.ctas;  // one cluster of C CTAs per row
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = launch_config(pl, ctas, static_cast<cudaStream_t>(stream), attr);
   void* args[] = {&P};
   P.group_stride = pl.group_stride;
-  if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING ||
-      pl.kernel == ASYMSPEC_KERNEL_PERSIST) {
+  if (pl.kernel == ASYMSPEC_KERNEL_TMA) {
     const TmaLayout L = tma_layout(B, K, pl.C, pl.group_stride);
     char* base = static_cast<char*>(workspace);
     P.row_stat = base + L.stat;
@@ -838,8 +546,7 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   if (e == cudaSuccess) e = cudaLaunchKernelExC(&cfg, fn, args);
   if (e == cudaSuccess) e = record_timing(opts, false, cfg.stream);
   if (e != cudaSuccess) return cuda_fail(e);
-  if (pl.kernel == ASYMSPEC_KERNEL_TMA || pl.kernel == ASYMSPEC_KERNEL_RING ||
-      pl.kernel == ASYMSPEC_KERNEL_PERSIST) {
+  if (pl.kernel == ASYMSPEC_KERNEL_TMA) {
     // the rows' decisions and Algorithm 1's scan: one CTA per batch element
     // as a programmatic dependent launch: its launch overlaps the row
     // kernel's last CTAs, and it waits (griddepcontrol.wait) for that kernel

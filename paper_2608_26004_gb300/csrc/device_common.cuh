@@ -341,9 +341,12 @@ __device__ __forceinline__ bool mbar_try_wait_hint(unsigned long long* bar, unsi
 }
 constexpr unsigned kSuspendHintNs = 100000;  // 0.1 ms per suspension
 
-// Waits for the phase with the given parity, giving up after limit_ns.
+// Waits for the phase with the given parity, giving up after limit_ns.  A
+// limit of 0 gives up at once, without looking at the barrier (the test hook
+// ASYMSPEC_TEST_COPY_GIVE_UP: a wait that times out, with no fault needed).
 __device__ __forceinline__ bool mbar_wait_bounded(unsigned long long* bar, unsigned parity,
                                                   unsigned long long limit_ns) {
+  if (limit_ns == 0) return false;
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = global_ns();
   while (!mbar_try_wait_hint(bar, parity, kSuspendHintNs)) {
@@ -425,8 +428,8 @@ struct KParams {
   int divergence, fuse_bonus;
   int delta_src;               // ASYMSPEC_DELTA_*: the signal fused into the emission (Eq. 1)
   int need_lse_s, need_pass2;  // generic kernel: compute LSE(s); run pass 2
-  int full;                    // streaming kernel: compute every row quantity (debug outputs)
-  int want_tokens;             // streaming kernel: also track argmax(s) in stochastic rows
+  int full;                    // compute every row quantity (debug outputs)
+  int want_tokens;             // also track argmax(s) in stochastic rows (per-row tokens)
   long long rows;              // B (K+1)
   int32_t* out_len;
   int32_t* out_next;
@@ -441,6 +444,7 @@ struct KParams {
   float* pass2_rec;     // [B(K+1)][C] X2 records (8 floats), one per CTA
   float* group_mass;    // [B(K+1)][C][group_stride] inverse-CDF group masses (stochastic)
   int group_stride;     // floats per row and CTA in group_mass (8 per round of the slice)
+  unsigned long long copy_wait_ns;  // limit of each bulk-copy wait (0: give up at once)
 };
 
 // What pass 1 leaves for the decision of a row: the normalisers, the

@@ -86,11 +86,11 @@ struct __align__(16) SharedTma {
   };
   float lse[4];       // the row's normalisers (pass 2 reads them)
   unsigned broken;    // a chunk copy timed out
-  int rel[kChunks];   // persistent kernel: warps done with each chunk of the row
   float qown;         // production draft rows: this slice's fused mass, from pass 1
-  unsigned pad[2];
-  // slot s (0, or the row's parity in the persistent kernel) of the C pushed records
-  __device__ X1* recv1(int slot = 0, int C = 0) { return reinterpret_cast<X1*>(this + 1) + slot * C; }
+  unsigned long long wait_ns;  // limit of each chunk wait (KParams::copy_wait_ns)
+  unsigned pad[kChunks];
+  // the C pushed records
+  __device__ X1* recv1() { return reinterpret_cast<X1*>(this + 1); }
 };
 
 // The pushed records are copied with 16-byte stores.
@@ -102,10 +102,9 @@ static_assert(sizeof(SharedTma) % 16 == 0, "records after SharedTma must stay 16
 // in round g / 8, i.e. vectors [32 g, 32 g + 32) in index order.
 constexpr int kGroupsMax = kMaxRounds * kTWarps;
 
-// Shared bytes after the slices for a cluster of C CTAs (the persistent
-// kernel keeps two slots of pushed records, by row parity).
-__host__ __device__ constexpr int shared_tma_bytes(int C, bool persistent = false) {
-  return static_cast<int>(sizeof(SharedTma) + (persistent ? 2 : 1) * C * sizeof(X1));
+// Shared bytes after the slices for a cluster of C CTAs.
+__host__ __device__ constexpr int shared_tma_bytes(int C) {
+  return static_cast<int>(sizeof(SharedTma) + C * sizeof(X1));
 }
 
 __device__ __forceinline__ X1 x1_neutral() {
@@ -421,7 +420,7 @@ __device__ __noinline__ void pass1_online(const T* ra, const T* rb, const T* rt,
   int vec_s = -1, vec_t = -1;  // vectors holding the best s and t so far
   const int tid = static_cast<int>(threadIdx.x);
   for (int c = 0, r0 = 0; c < kChunks && r0 < rounds; ++c, r0 += rc) {
-    if (WAIT && !sh->broken && !mbar_wait_bounded(&sh->bar[c], ph, kCopyTimeoutNs))
+    if (WAIT && !sh->broken && !mbar_wait_bounded(&sh->bar[c], ph, sh->wait_ns))
       atomicOr(&sh->broken, kBadTimeout);
     const int r1 = min(rounds, r0 + rc);
     int i0 = r0 * kTThreads + tid;          // vector index of this thread's first vector
@@ -538,7 +537,7 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
   const f2 L2 = pk(kLog2e, kLog2e);
   const int tid = static_cast<int>(threadIdx.x);
   // chunk 0 holds every thread's first vector
-  if (!sh->broken && !mbar_wait_bounded(&sh->bar[0], ph, kCopyTimeoutNs))
+  if (!sh->broken && !mbar_wait_bounded(&sh->bar[0], ph, sh->wait_ns))
     atomicOr(&sh->broken, kBadTimeout);
   float ref[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
   if (tid < nv) {
@@ -571,7 +570,7 @@ __device__ __forceinline__ bool pass1_fast(const T* ra, const T* rb, const T* rt
   f2 acc[4] = {0ull, 0ull, 0ull, 0ull};
   int vec_s = -1, vec_t = -1;  // vectors holding the best s and t so far
   for (int c = 0, r0 = 0; c < kChunks && r0 < rounds; ++c, r0 += rc) {
-    if (c > 0 && !sh->broken && !mbar_wait_bounded(&sh->bar[c], ph, kCopyTimeoutNs))
+    if (c > 0 && !sh->broken && !mbar_wait_bounded(&sh->bar[c], ph, sh->wait_ns))
       atomicOr(&sh->broken, kBadTimeout);
     const int r1 = min(rounds, r0 + rc);
     int i0 = r0 * kTThreads + tid;          // vector index of this thread's first vector
@@ -658,18 +657,17 @@ template <typename T, unsigned F, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void pass1_and_push(const T* ra, const T* rb, const T* rt, int nv,
                                                int rounds, int rc, int lo, int n, float beta,
                                                int dtok, SharedTma* sh, int rank, int C,
-                                               cg::cluster_group& cluster, unsigned ph = 0,
-                                               int slot = 0) {
+                                               cg::cluster_group& cluster) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   X1 e = x1_neutral();
-  const bool ovf = pass1_fast<T, F, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e, ph);
+  const bool ovf = pass1_fast<T, F, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
   warp_reduce_x1_uniform<F>(e);  // the warp's references are equal
   if (lane == 0) sh->w1[warp] = e;
   if (__syncthreads_or(ovf)) {
     // an entry far above its thread's reference (or non-finite data): redo
     // the slice with a running maximum
     e = x1_neutral();
-    pass1_online<T, F, true, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e, ph);
+    pass1_online<T, F, true, DS>(ra, rb, rt, nv, rounds, rc, lo, beta, sh, e);
     warp_reduce_x1<F>(e);
     if (lane == 0) sh->w1[warp] = e;
     __syncthreads();
@@ -683,7 +681,7 @@ __device__ __forceinline__ void pass1_and_push(const T* ra, const T* rb, const T
       w.db = to_f32(rb[dtok - lo]);
       w.dt = to_f32(rt[dtok - lo]);
     }
-    push_record(w, sh->recv1(slot, C), rank, C, cluster);
+    push_record(w, sh->recv1(), rank, C, cluster);
   }
   cluster_barrier(warp == 0);  // B1: every CTA's pass-1 record is in every CTA
 }
@@ -718,42 +716,12 @@ __device__ __forceinline__ void issue_slice(const KParams& P, SharedTma* sh, lon
   for (int c = 0; c < kChunks; ++c) issue_chunk<T>(P, sh, row, lo, nv, rc, sa, sb, st, only_t, c);
 }
 
-// Persistent kernel: once all kTWarps warps have read chunk c of the slice
-// in pass 2, the last of them copies chunk c of the cluster's next row into
-// it (mbarrier c completes once per row, so the waits take the row's parity).
-template <typename T>
-struct ChunkRefill {
-  static constexpr bool kActive = true;
-  int rc;
-  const KParams* P;
-  SharedTma* sh;
-  long long next;  // the next row, or -1
-  int lo, nv;
-  T* sa;
-  T* sb;
-  T* st;
-  bool only_t;
-  __device__ __forceinline__ void operator()(int c) const {
-    __syncwarp();
-    if ((threadIdx.x & 31) == 0) {
-      __threadfence_block();  // this warp's reads of the chunk come first
-      if (atomicAdd(&sh->rel[c], 1) == kTWarps - 1) {
-        sh->rel[c] = 0;
-        __threadfence_block();
-        fence_proxy_async_shared();
-        if (next >= 0 && !sh->broken) issue_chunk<T>(*P, sh, next, lo, nv, rc, sa, sb, st, only_t, c);
-      }
-    }
-    __syncwarp();
-  }
-};
-
 // After B1, in one warp: the row values from the C pushed records (every
 // lane ends with them).  lse[q] = ln of stream q's normaliser.
 template <unsigned F>
-__device__ __forceinline__ X1 combine_pass1(SharedTma* sh, int C, float (&lse)[4], int slot = 0) {
+__device__ __forceinline__ X1 combine_pass1(SharedTma* sh, int C, float (&lse)[4]) {
   const int lane = threadIdx.x & 31;
-  X1 w = (lane < C) ? sh->recv1(slot, C)[lane] : x1_neutral();
+  X1 w = (lane < C) ? sh->recv1()[lane] : x1_neutral();
   warp_reduce_x1<F>(w);
 #pragma unroll
   for (int q = 0; q < 4; ++q) lse[q] = w.ref[q] + logf(w.s[q]);
@@ -762,10 +730,10 @@ __device__ __forceinline__ X1 combine_pass1(SharedTma* sh, int C, float (&lse)[4
 
 // The draft token's a, b, t (from the record of the CTA whose slice holds it).
 __device__ __forceinline__ void draft_logits(SharedTma* sh, int dtok, int W, int C, float& ad,
-                                             float& bd, float& td, int slot = 0) {
+                                             float& bd, float& td) {
   ad = bd = td = 0.f;
   if (dtok >= 0 && W > 0) {
-    const X1& o = sh->recv1(slot, C)[dtok / W < C ? dtok / W : 0];
+    const X1& o = sh->recv1()[dtok / W < C ? dtok / W : 0];
     ad = o.da;
     bd = o.db;
     td = o.dt;
@@ -929,27 +897,16 @@ __device__ __forceinline__ void p2_finish(const P2Acc& acc, X2& x) {
   x.Q = hsum2(acc.Q2);
 }
 
-// What pass 2 does with a chunk of the slice once a warp has read it: nothing
-// in the one-shot kernel; the persistent kernel refills it with the next row.
-struct NoRelease {
-  static constexpr bool kActive = false;
-  int rc = 0;
-  __device__ __forceinline__ void operator()(int) const {}
-};
-
-// Pass 2 over the slice, two vectors per step.  Rel::kActive: after the last
-// step that reads chunk c (rounds [c rc, (c+1) rc)), every warp calls rel(c).
-template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, class Rel = NoRelease,
-          bool QSUM = true>
+// Pass 2 over the slice, two vectors per step.
+template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, bool QSUM = true>
 __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int nv, int rounds,
                                       float beta, float A2, float B2, float S2, float lse_s, X2& x,
-                                      float* lp, float* grp, const Rel& rel = Rel()) {
+                                      float* lp, float* grp) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
   constexpr bool needT = (G & (G_RES | G_QF)) != 0 || LP;
   const P2Const k = p2_const(beta, A2, B2, S2, lse_s);
   P2Acc acc = {0ull, 0ull, 0ull, 0ull, 0ull, 0ull};
-  int next_c = 0;  // chunks this warp has released
   float gp0 = 0.f, gp1 = 0.f;  // the previous step's masses, reduced with this step's
   bool pending = false;
   for (int kr = 0; kr < rounds; kr += 2) {
@@ -987,31 +944,22 @@ __device__ __forceinline__ void pass2(const T* ra, const T* rb, const T* rt, int
       gp1 = g1;
       pending = !pending;
     }
-    if constexpr (Rel::kActive) {
-      const int done = kr + 2;  // rounds this warp has finished
-      while (next_c < kChunks && (done >= (next_c + 1) * rel.rc || done >= rounds)) rel(next_c++);
-    }
   }
   if ((G & (G_RES | G_QF)) && pending) p2_groups(gp0, gp1, grp, ((rounds - 1) & ~1), rounds);
-  if constexpr (Rel::kActive) {
-    while (next_c < kChunks) rel(next_c++);
-  }
   p2_finish(acc, x);
 }
 
 // Pass 2 and the CTA combine; warp 0 stores the CTA's pass-2 record in the
 // workspace (groups: this CTA's group masses there, stored by pass 2).
-template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, class Rel = NoRelease,
-          bool QSUM = true>
+template <typename T, unsigned G, bool LP, int DS = ASYMSPEC_DELTA_AB, bool QSUM = true>
 __device__ __forceinline__ void pass2_and_store(const T* ra, const T* rb, const T* rt, int nv,
                                                 int rounds, float beta, float* lp, SharedTma* sh,
-                                                float* rec, float* groups,
-                                                const Rel& rel = Rel()) {
+                                                float* rec, float* groups) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const float lse_a = sh->lse[0], lse_b = sh->lse[1], lse_s = sh->lse[3];
   X2 x = x2_zero();
-  pass2<T, G, LP, DS, Rel, QSUM>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e,
-                                 lse_s * kLog2e, lse_s, x, lp, groups, rel);
+  pass2<T, G, LP, DS, QSUM>(ra, rb, rt, nv, rounds, beta, lse_a * kLog2e, lse_b * kLog2e,
+                            lse_s * kLog2e, lse_s, x, lp, groups);
   warp_reduce_x2<G>(x);
   if (lane == 0) sh->w2[warp] = x;
   __syncthreads();
@@ -1203,12 +1151,6 @@ struct RowCtx {
   bool bonus;
   int dtok;           // warp 0 only: the row's draft token (-1 on the bonus row)
   SharedTma* sh;
-  // persistent kernel: the parity of the row's chunk barriers and record
-  // slot, and the cluster's next row (-1 if none) with its copy kind
-  unsigned ph;
-  int slot;
-  long long next;
-  bool next_only_t;
 };
 
 // Rank 0: what pass 1 leaves for the row's decision.
@@ -1232,9 +1174,8 @@ __device__ __forceinline__ void store_row_stat(const KParams& P, long long row,
 
 // One row with pass-1 program F and pass-2 program G (R2: pass 2 runs; LP:
 // it writes the fused log-probs).
-// PER: the persistent kernel (the slice is refilled with the next row).
 template <typename T, bool STOCH, unsigned F, unsigned G, bool LP, bool R2,
-          int DS = ASYMSPEC_DELTA_AB, bool PER = false>
+          int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
                                         cg::cluster_group& cluster) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -1247,41 +1188,33 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
   // only when the whole residual is zero) from pass 1; the full program (the
   // only one with F_AT and pass 2) sums it in pass 2, for every row alike
   constexpr bool QSUM = !((G & G_RES) && !(F & F_AT) && (F & F_LS));
-  pass1_and_push<T, F, DS>(ra, rb, rt, c.nv, c.rounds, c.rc, c.lo, c.n, beta, c.dtok, sh, c.rank, c.C,
-                       cluster, c.ph, c.slot);
+  pass1_and_push<T, F, DS>(ra, rb, rt, c.nv, c.rounds, c.rc, c.lo, c.n, beta, c.dtok, sh, c.rank,
+                           c.C, cluster);
   if constexpr (!R2) {
     // no pass 2: rank 0 leaves the row's pass-1 results for the decision kernel
-    if constexpr (PER) {
-      // after B1 no thread reads the slice again: refill it with the next row
-      if (threadIdx.x == 0 && c.next >= 0 && !sh->broken) {
-        fence_proxy_async_shared();
-        issue_slice<T>(P, sh, c.next, c.lo, c.nv, c.rc, const_cast<T*>(ra), const_cast<T*>(rb),
-                       const_cast<T*>(rt), c.next_only_t);
-      }
-    }
     if (c.rank == 0 && warp == 0) {
       float lse[4];
-      const X1 w = combine_pass1<F>(sh, c.C, lse, c.slot);
+      const X1 w = combine_pass1<F>(sh, c.C, lse);
       float ad, bd, td;
-      draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td, c.slot);
+      draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td);
       if (lane == 0) store_row_stat(P, c.row, lse, w.is, w.it, w.bad, c.dtok, ad, bd, td);
     }
     return;
   } else {
     if (warp == 0) {
       float lse[4];
-      const X1 w = combine_pass1<F>(sh, c.C, lse, c.slot);
+      const X1 w = combine_pass1<F>(sh, c.C, lse);
       if (lane == 0) {
 #pragma unroll
         for (int q = 0; q < 4; ++q) sh->lse[q] = lse[q];
         if (!QSUM) {
           // this slice's fused mass sum exp(s - LSE(s)), from its own pass-1 record
-          const X1& own = sh->recv1(c.slot, c.C)[c.rank];
+          const X1& own = sh->recv1()[c.rank];
           sh->qown = own.s[3] * ex2((own.ref[3] - lse[3]) * kLog2e);
         }
         if (c.rank == 0) {
           float ad, bd, td;
-          draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td, c.slot);
+          draft_logits(sh, c.dtok, c.W, c.C, ad, bd, td);
           store_row_stat(P, c.row, lse, w.is, w.it, w.bad, c.dtok, ad, bd, td);
         }
       }
@@ -1289,73 +1222,65 @@ __device__ __forceinline__ void run_row(const KParams& P, const RowCtx& c,
     __syncthreads();
     float* lp = LP ? P.logprobs + static_cast<size_t>(c.row) * P.V + c.lo : nullptr;
     const size_t slot = static_cast<size_t>(c.row) * c.C + c.rank;
-    if constexpr (PER) {
-      const ChunkRefill<T> rel{c.rc, &P, sh, c.next, c.lo, c.nv, const_cast<T*>(ra),
-                               const_cast<T*>(rb), const_cast<T*>(rt), c.next_only_t};
-      pass2_and_store<T, G, LP, DS, ChunkRefill<T>, QSUM>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh,
-                                                    P.pass2_rec + slot * 8,
-                                                    P.group_mass + slot * P.group_stride, rel);
-    } else {
-      pass2_and_store<T, G, LP, DS, NoRelease, QSUM>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh,
-                                    P.pass2_rec + slot * 8, P.group_mass + slot * P.group_stride);
-    }
+    pass2_and_store<T, G, LP, DS, QSUM>(ra, rb, rt, c.nv, c.rounds, beta, lp, sh,
+                                        P.pass2_rec + slot * 8,
+                                        P.group_mass + slot * P.group_stride);
   }
 }
 
-template <typename T, bool STOCH, unsigned F, unsigned RQ, int DS = ASYMSPEC_DELTA_AB,
-          bool PER = false>
+template <typename T, bool STOCH, unsigned F, unsigned RQ, int DS = ASYMSPEC_DELTA_AB>
 __device__ __forceinline__ void run_full(const KParams& P, const RowCtx& c,
                                          cg::cluster_group& cluster) {
   const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
   const bool klg = P.divergence == ASYMSPEC_DIV_KL;
   if (P.logprobs) {
-    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, true, true, DS, PER>(P, c, cluster);
-    else if (klg) run_row<T, STOCH, F, G_KL | RQ, true, true, DS, PER>(P, c, cluster);
-    else run_row<T, STOCH, F, RQ, true, true, DS, PER>(P, c, cluster);
+    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, true, true, DS>(P, c, cluster);
+    else if (klg) run_row<T, STOCH, F, G_KL | RQ, true, true, DS>(P, c, cluster);
+    else run_row<T, STOCH, F, RQ, true, true, DS>(P, c, cluster);
   } else {
-    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, false, true, DS, PER>(P, c, cluster);
-    else if (klg) run_row<T, STOCH, F, G_KL | RQ, false, true, DS, PER>(P, c, cluster);
-    else run_row<T, STOCH, F, RQ, false, true, DS, PER>(P, c, cluster);
+    if (jsd) run_row<T, STOCH, F, G_JSD | RQ, false, true, DS>(P, c, cluster);
+    else if (klg) run_row<T, STOCH, F, G_KL | RQ, false, true, DS>(P, c, cluster);
+    else run_row<T, STOCH, F, RQ, false, true, DS>(P, c, cluster);
   }
 }
 
 // Program set 0: every row program, chosen at run time, for delta source DS.
-template <typename T, bool STOCH, int DS, bool PER = false>
+template <typename T, bool STOCH, int DS>
 __device__ __forceinline__ void run_any(const KParams& P, const RowCtx& c, bool bonus,
                                         cg::cluster_group& cluster) {
   if (P.full) {
-    run_full<T, STOCH, F_LA | F_LB | F_LT | F_LS | F_AS | F_AT, STOCH ? G_RES : 0u, DS, PER>(P, c, cluster);
+    run_full<T, STOCH, F_LA | F_LB | F_LT | F_LS | F_AS | F_AT, STOCH ? G_RES : 0u, DS>(P, c, cluster);
   } else if (!STOCH) {
     const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
     const bool klg = P.divergence == ASYMSPEC_DIV_KL;
     constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
     if (bonus) {
-      if (P.fuse_bonus) run_row<T, STOCH, F_AS, 0, false, false, DS, PER>(P, c, cluster);
-      else run_row<T, STOCH, F_AT, 0, false, false, DS, PER>(P, c, cluster);
+      if (P.fuse_bonus) run_row<T, STOCH, F_AS, 0, false, false, DS>(P, c, cluster);
+      else run_row<T, STOCH, F_AT, 0, false, false, DS>(P, c, cluster);
     } else if (jsd) {
-      run_row<T, STOCH, FD, G_JSD, false, true, DS, PER>(P, c, cluster);
+      run_row<T, STOCH, FD, G_JSD, false, true, DS>(P, c, cluster);
     } else if (klg) {
-      run_row<T, STOCH, FD, G_KL, false, true, DS, PER>(P, c, cluster);
+      run_row<T, STOCH, FD, G_KL, false, true, DS>(P, c, cluster);
     } else {
-      run_row<T, STOCH, FD, 0, false, false, DS, PER>(P, c, cluster);
+      run_row<T, STOCH, FD, 0, false, false, DS>(P, c, cluster);
     }
   } else if (!bonus) {
     const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
     const bool klg = P.divergence == ASYMSPEC_DIV_KL;
     if (P.want_tokens) {
       constexpr unsigned FS = F_LA | F_LB | F_LS | F_AS;
-      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS, PER>(P, c, cluster);
-      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS, PER>(P, c, cluster);
-      else run_row<T, STOCH, FS, G_RES, false, true, DS, PER>(P, c, cluster);
+      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS>(P, c, cluster);
+      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS>(P, c, cluster);
+      else run_row<T, STOCH, FS, G_RES, false, true, DS>(P, c, cluster);
     } else {
       constexpr unsigned FS = F_LA | F_LB | F_LS;
-      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS, PER>(P, c, cluster);
-      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS, PER>(P, c, cluster);
-      else run_row<T, STOCH, FS, G_RES, false, true, DS, PER>(P, c, cluster);
+      if (jsd) run_row<T, STOCH, FS, G_JSD | G_RES, false, true, DS>(P, c, cluster);
+      else if (klg) run_row<T, STOCH, FS, G_KL | G_RES, false, true, DS>(P, c, cluster);
+      else run_row<T, STOCH, FS, G_RES, false, true, DS>(P, c, cluster);
     }
   } else {
-    if (P.want_tokens) run_row<T, STOCH, F_LS | F_AS, G_QF, false, true, DS, PER>(P, c, cluster);
-    else run_row<T, STOCH, F_LS, G_QF, false, true, DS, PER>(P, c, cluster);
+    if (P.want_tokens) run_row<T, STOCH, F_LS | F_AS, G_QF, false, true, DS>(P, c, cluster);
+    else run_row<T, STOCH, F_LS, G_QF, false, true, DS>(P, c, cluster);
   }
 
 }
@@ -1378,25 +1303,19 @@ __host__ __device__ constexpr int tma_program_set(bool stoch, int divergence, bo
                    ((!stoch && fuse_bonus) ? 3 : 0);
 }
 
-// PER = false: one row per cluster (grid = rows x C).  PER = true: the
-// persistent form, grid = G clusters (as many as the device holds), cluster q
-// taking rows q, q + G, q + 2G, ...; each CTA keeps one slice buffer, and as
-// pass 2 of a row finishes with a chunk of it, that chunk is refilled with
-// the cluster's next row, so the copies of row r + G overlap pass 2 of row r
-// and pass 1 of row r + G starts on data already in shared memory.
-template <typename T, bool STOCH, int SEL, bool PER = false>
+// One cluster of C CTAs per row (grid = rows x C); CTA r of the cluster
+// takes entries [r W, (r+1) W) of the row.
+template <typename T, bool STOCH, int SEL>
 __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P) {
-  constexpr int VE = 16 / static_cast<int>(sizeof(T));
   extern __shared__ __align__(128) unsigned char smem_tma[];
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
   const int tid = threadIdx.x;
   const int C = P.C;
   // 32-bit row arithmetic: the host keeps rows x C below 2^31
-  const unsigned rows32 = static_cast<unsigned>(P.rows);
-  const unsigned G = PER ? gridDim.x / static_cast<unsigned>(C) : 1u;
-  unsigned row32 = blockIdx.x / static_cast<unsigned>(C);
+  const unsigned row32 = blockIdx.x / static_cast<unsigned>(C);
   const unsigned K1 = static_cast<unsigned>(P.K) + 1u;
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
   const int V = P.V, W = P.W;
   const int lo = rank * W;
   const int n = max(0, min(W, V - lo));
@@ -1408,20 +1327,19 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   T* sb = sa + W;
   T* st = sb + W;
   SharedTma* sh = reinterpret_cast<SharedTma*>(smem_tma + P.sh_off);
-  auto t_only = [&](unsigned r) {
-    const unsigned kk = r - (r / K1) * K1;
-    return !STOCH && !P.full && kk == static_cast<unsigned>(P.K) && !P.fuse_bonus;
-  };
+  const int bi = static_cast<int>(row32 / K1);
+  const int k = static_cast<int>(row32 - static_cast<unsigned>(bi) * K1);
+  const bool bonus = (k == P.K);
 
   if (tid == 0) {
 #pragma unroll
-    for (int c = 0; c < kChunks; ++c) {
-      mbar_init(&sh->bar[c], 1);
-      sh->rel[c] = 0;
-    }
+    for (int q = 0; q < kChunks; ++q) mbar_init(&sh->bar[q], 1);
     sh->broken = 0;
+    sh->wait_ns = P.copy_wait_ns;
     fence_mbar_init();
-    issue_slice<T>(P, sh, row32, lo, nv, rc, sa, sb, st, t_only(row32));
+    // a greedy bonus row without fused bonus needs t alone (Algorithm 1 emits argmax t)
+    const bool only_t = !STOCH && !P.full && bonus && !P.fuse_bonus;
+    issue_slice<T>(P, sh, row32, lo, nv, rc, sa, sb, st, only_t);
   }
   RowCtx c;
   c.sa = sa;
@@ -1436,69 +1354,50 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
   c.rank = rank;
   c.C = C;
   c.sh = sh;
-  unsigned it = 0;
-  for (;;) {
-    const int bi = static_cast<int>(row32 / K1);
-    const int k = static_cast<int>(row32 - static_cast<unsigned>(bi) * K1);
-    const bool bonus = (k == P.K);
-    c.k = k;
-    c.bi = bi;
-    c.row = row32;
-    c.bonus = bonus;
-    c.ph = it & 1u;
-    c.slot = PER ? static_cast<int>(it & 1u) : 0;
-    c.next = (PER && row32 + G < rows32) ? static_cast<long long>(row32 + G) : -1;
-    c.next_only_t = c.next >= 0 && t_only(row32 + G);
-    // warp 0 keeps the row's draft token, loaded while the slice is in flight
-    c.dtok = -1;
-    if ((tid >> 5) == 0 && !bonus) c.dtok = P.tokens[static_cast<size_t>(bi) * P.K + k];
-    // the chunk barriers are initialised (first row); warp 0 has read the
-    // previous row's pass-2 records out of w2, which pass 1 reuses as w1
-    __syncthreads();
+  c.k = k;
+  c.bi = bi;
+  c.row = row32;
+  c.bonus = bonus;
+  // warp 0 keeps the row's draft token, loaded while the slice is in flight
+  c.dtok = -1;
+  if ((tid >> 5) == 0 && !bonus) c.dtok = P.tokens[static_cast<size_t>(bi) * P.K + k];
+  __syncthreads();  // the chunk barriers are initialised
 
-    if constexpr (SEL > 0 && STOCH) {
-      constexpr int d = SEL - 1;
-      constexpr unsigned GD = d == 0 ? G_JSD : d == 1 ? G_KL : 0u;
-      if (!bonus)
-        run_row<T, STOCH, F_LA | F_LB | F_LS, GD | G_RES, false, true, ASYMSPEC_DELTA_AB, PER>(
-            P, c, cluster);
-      else
-        run_row<T, STOCH, F_LS, G_QF, false, true, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
-    } else if constexpr (SEL > 0) {
-      constexpr int d = (SEL - 1) % 3;
-      constexpr bool fused_bonus = SEL > 3;
-      constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
-      if (bonus) {
-        if (fused_bonus) run_row<T, STOCH, F_AS, 0, false, false, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
-        else run_row<T, STOCH, F_AT, 0, false, false, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
-      } else if (d == 0) {
-        run_row<T, STOCH, FD, G_JSD, false, true, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
-      } else if (d == 1) {
-        run_row<T, STOCH, FD, G_KL, false, true, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
-      } else {
-        run_row<T, STOCH, FD, 0, false, false, ASYMSPEC_DELTA_AB, PER>(P, c, cluster);
-      }
-    } else if (P.delta_src == ASYMSPEC_DELTA_A) {
-      run_any<T, STOCH, ASYMSPEC_DELTA_A, PER>(P, c, bonus, cluster);
-    } else if (P.delta_src == ASYMSPEC_DELTA_TB) {
-      run_any<T, STOCH, ASYMSPEC_DELTA_TB, PER>(P, c, bonus, cluster);
+  if constexpr (SEL > 0 && STOCH) {
+    constexpr int d = SEL - 1;
+    constexpr unsigned GD = d == 0 ? G_JSD : d == 1 ? G_KL : 0u;
+    if (!bonus)
+      run_row<T, STOCH, F_LA | F_LB | F_LS, GD | G_RES, false, true, ASYMSPEC_DELTA_AB>(P, c,
+                                                                                     cluster);
+    else
+      run_row<T, STOCH, F_LS, G_QF, false, true, ASYMSPEC_DELTA_AB>(P, c, cluster);
+  } else if constexpr (SEL > 0) {
+    constexpr int d = (SEL - 1) % 3;
+    constexpr bool fused_bonus = SEL > 3;
+    constexpr unsigned FD = F_LA | F_LB | F_LT | F_AS;
+    if (bonus) {
+      if (fused_bonus) run_row<T, STOCH, F_AS, 0, false, false, ASYMSPEC_DELTA_AB>(P, c, cluster);
+      else run_row<T, STOCH, F_AT, 0, false, false, ASYMSPEC_DELTA_AB>(P, c, cluster);
+    } else if (d == 0) {
+      run_row<T, STOCH, FD, G_JSD, false, true, ASYMSPEC_DELTA_AB>(P, c, cluster);
+    } else if (d == 1) {
+      run_row<T, STOCH, FD, G_KL, false, true, ASYMSPEC_DELTA_AB>(P, c, cluster);
     } else {
-      run_any<T, STOCH, ASYMSPEC_DELTA_AB, PER>(P, c, bonus, cluster);
+      run_row<T, STOCH, FD, 0, false, false, ASYMSPEC_DELTA_AB>(P, c, cluster);
     }
-    if (!PER || c.next < 0) break;
-    row32 += G;
-    ++it;
+  } else if (P.delta_src == ASYMSPEC_DELTA_A) {
+    run_any<T, STOCH, ASYMSPEC_DELTA_A>(P, c, bonus, cluster);
+  } else if (P.delta_src == ASYMSPEC_DELTA_TB) {
+    run_any<T, STOCH, ASYMSPEC_DELTA_TB>(P, c, bonus, cluster);
+  } else {
+    run_any<T, STOCH, ASYMSPEC_DELTA_AB>(P, c, bonus, cluster);
   }
 
-  // a copy that timed out may still land: wait for it (bounded) before exit.
-  // No copy of a later row is issued once a copy has timed out, but the
-  // persistent kernel may have moved on by then, so both parities are waited.
+  // a copy that timed out may still land: wait for it (bounded, always with
+  // the normal limit) before exit
   if (tid == 0 && sh->broken) {
 #pragma unroll
-    for (int q = 0; q < kChunks; ++q) {
-      mbar_wait_bounded(&sh->bar[q], 0u, kCopyTimeoutNs);
-      if (PER) mbar_wait_bounded(&sh->bar[q], 1u, kCopyTimeoutNs);
-    }
+    for (int q = 0; q < kChunks; ++q) mbar_wait_bounded(&sh->bar[q], 0u, kCopyTimeoutNs);
   }
 }
 

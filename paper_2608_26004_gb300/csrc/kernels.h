@@ -16,21 +16,9 @@ const void* tma_kernel_bf16_any_stoch();  // k_tma_bf16_any_s.cu
 const void* tma_kernel_f32_any_stoch();   // k_tma_f32_any_s.cu
 const void* tma_kernel_bf16(bool stoch, int sel);
 const void* tma_kernel_f32(bool stoch, int sel);
-// fuse_verify_tma<T, STOCH, SEL, true>, the persistent form: the production
-// sets 1..6 only (k_tmap_bf16.cu, k_tmap_f32.cu); nullptr for any other set
-const void* tmap_kernel_bf16(bool stoch, int sel);
-const void* tmap_kernel_f32(bool stoch, int sel);
-// fuse_verify_ring<T, STOCH> (k_ring_bf16.cu, k_ring_f32.cu)
-const void* ring_kernel_bf16(bool stoch);
-const void* ring_kernel_f32(bool stoch);
-// decide_rows<T, STOCH>, launched after fuse_verify_tma or fuse_verify_ring (k_tma_*.cu)
+// decide_rows<T, STOCH>, launched after fuse_verify_tma (k_tma_*.cu)
 const void* decide_kernel_bf16(bool stoch);
 const void* decide_kernel_f32(bool stoch);
-// fuse_verify_stream<T, STOCH> (k_stream_*.cu)
-const void* stream_kernel_bf16_greedy();
-const void* stream_kernel_bf16_stoch();
-const void* stream_kernel_f32_greedy();
-const void* stream_kernel_f32_stoch();
 // draft_kernel<T, VE, STOCH>, the drafter's draw (k_draft.cu)
 const void* draft_kernel_ptr(int dtype, bool vector_path, bool stoch);
 // the cross-family vocabulary map (k_xvocab.cu): xvocab_gather<T>, xvocab_inv_fill,

@@ -65,14 +65,11 @@ def tma_bytes(B, K, C):
 
 
 def test_workspace_size():
-    # the TMA kernel's layout for clusters of up to 16 CTAs, independent of V,
-    # unless the streaming kernel's is larger (fp32 rows of 16 or more tiles)
-    assert A.workspace_bytes(64, 7, 128256) >= tma_bytes(64, 7, 16)
+    # the TMA kernel's layout for clusters of up to 16 CTAs, independent of V
+    assert A.workspace_bytes(64, 7, 128256) == tma_bytes(64, 7, 16)
     assert A.workspace_bytes(3, 2, 10) == A.workspace_bytes(3, 2, 10**5) == tma_bytes(3, 2, 16)
+    assert A.workspace_bytes(3, 2, 250000) == tma_bytes(3, 2, 16)
     assert A.workspace_bytes(0, 7, 10) == 0
-    # the streaming state grows with the tiles per row and passes it for fp32
-    # rows of 31 tiles of 8192 entries
-    assert A.workspace_bytes(3, 2, 250000) > tma_bytes(3, 2, 16)
     assert A.workspace_bytes(64, 7, 128256) < 8 << 20
 
 
@@ -117,16 +114,17 @@ def test_host_validation_codes(lib):
     st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
                           FAKE, FAKE, 1 << 20, opts=A.LaunchOpts(0, 0, 7))
     assert st == A.ERR_INVALID_ARG                       # unknown kernel
+    for removed in (3, 4, 5):                            # numbers of no kernel
+        st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
+                              FAKE, FAKE, 1 << 20, opts=A.LaunchOpts(0, 0, removed))
+        assert st == A.ERR_INVALID_ARG
     half = A.LaunchOpts(0, 0, 0, 0, FAKE, 0)             # one timing event without the other
     assert A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
                             FAKE, FAKE, 1 << 20, opts=half) == A.ERR_INVALID_ARG
-    padded = A.LaunchOpts(0, 0, 0, 1)                    # reserved field set
-    assert A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
-                            FAKE, FAKE, 1 << 20, opts=padded) == A.ERR_INVALID_ARG
-    small = A.workspace_bytes(2, 2, 250000) - 1          # streaming kernel forced, workspace short
-    st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 250000, A.FP32, None, FAKE,
-                          FAKE, FAKE, small, opts=A.LaunchOpts(0, 0, A.KERNEL_STREAM))
-    assert st == A.ERR_WORKSPACE
+    for bits in (2, 4, -1):                              # reserved test-flag bits set
+        assert A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
+                                FAKE, FAKE, 1 << 20, opts=A.LaunchOpts(0, 0, 0, bits)) \
+            == A.ERR_INVALID_ARG
     small = tma_bytes(2, 2, 4) - 1                       # TMA kernel forced (clusters of 4), short
     st = A.fuse_verify_ex(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 2, 2, 64, A.FP32, None, FAKE,
                           FAKE, FAKE, small, opts=A.LaunchOpts(4, 0, A.KERNEL_TMA))
@@ -200,27 +198,7 @@ def test_draft_sample_validation_codes(lib):
 
 
 def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
-    # the streaming kernel on request: 16384-entry tiles (bf16), 8192 (fp32)
-    STREAM = A.LaunchOpts(0, 0, A.KERNEL_STREAM)
-    info = A.plan(64, 7, 128256, A.BF16, opts=STREAM)
-    assert info.kernel == A.KERNEL_STREAM and info.slice_elems == 16384
-    info = A.plan(1, 4, 32000, A.FP32, opts=STREAM)
-    assert info.kernel == A.KERNEL_STREAM and info.slice_elems == 8192
     assert A.plan(64, 7, 128256, A.BF16).kernel == A.KERNEL_TMA      # the automatic choice
-    RING = A.LaunchOpts(0, 0, A.KERNEL_RING)
-    # the ring kernel keeps no slice in shared memory: clusters of 8 while a
-    # slice takes at most 32 rounds of 256 vectors, else 16; smaller clusters
-    # on request (more entries per thread)
-    info = A.plan(64, 7, 128256, A.BF16, opts=RING)
-    assert info.kernel == A.KERNEL_RING and info.cluster_size == 8 and info.slice_elems == 16032
-    info = A.plan(256, 4, 151936, A.FP32, opts=RING)
-    assert info.kernel == A.KERNEL_RING and info.cluster_size == 8
-    info = A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(2, 0, A.KERNEL_RING))
-    assert info.kernel == A.KERNEL_RING and info.cluster_size == 2 and info.slice_elems == 64128
-    with pytest.raises(A.AsymSpecError):      # a single CTA's slice would take 63 rounds
-        A.plan(64, 7, 128256, A.BF16, opts=A.LaunchOpts(1, 0, A.KERNEL_RING))
-    with pytest.raises(A.AsymSpecError):      # unaligned rows cannot use bulk copies
-        A.plan(2, 2, 4099, A.BF16, opts=RING)
     TMA = A.LaunchOpts(0, 0, A.KERNEL_TMA)
     # the cluster kernel on the bench workload: 8 CTAs of 96 KB per row, two per SM
     info = A.plan(64, 7, 128256, A.BF16, opts=TMA)
@@ -314,20 +292,3 @@ def test_xvocab_workspace_layout_and_validation(lib):
              FAKE, small) == A.ERR_WORKSPACE
     assert g(FAKE, FAKE, 30, FAKE, 20, FAKE, FAKE, 10, 4, A.FP32, FAKE, FAKE, FAKE, None,
              FAKE + 16, small + 1) == A.ERR_WORKSPACE
-
-
-def test_plan_of_the_persistent_kernel(lib):
-    # the persistent form keeps the one-shot kernel's slices and one more slot
-    # of pushed pass-1 records (64 bytes per CTA of the cluster)
-    PER = A.LaunchOpts(0, 0, A.KERNEL_PERSIST)
-    TMA = A.LaunchOpts(0, 0, A.KERNEL_TMA)
-    for B, K, V, dtype in ((64, 7, 128256, A.BF16), (8, 5, 151936, A.BF16),
-                           (1, 4, 32000, A.FP32)):
-        p, t = A.plan(B, K, V, dtype, opts=PER), A.plan(B, K, V, dtype, opts=TMA)
-        assert p.kernel == A.KERNEL_PERSIST and p.cluster_size == t.cluster_size
-        assert p.slice_elems == t.slice_elems
-        assert p.smem_bytes == t.smem_bytes + 64 * t.cluster_size
-        assert p.smem_bytes <= 113 * 1024          # still two CTAs per SM
-    with pytest.raises(A.AsymSpecError) as e:      # unaligned rows: no bulk copies
-        A.plan(2, 2, 4099, A.BF16, opts=PER)
-    assert e.value.status == A.ERR_UNSUPPORTED

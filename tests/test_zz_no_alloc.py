@@ -4,15 +4,16 @@ The file name sorts last so that these calls also run after every other GPU
 test has used the library in the same process; the tests must pass both
 alone and then.  Every result is compared bit for bit with
 asymspec_fuse_verify_ex given a caller-owned zeroed workspace of the static
-scratch's size, which selects the same kernel, on the same inputs, over two consecutive calls, so that the second call sees the
-scratch the first one left.
+scratch's size, which selects the same kernel, on the same inputs, over two
+consecutive calls, so that the second call sees the scratch the first one
+left; and, on a sample of batch elements, with the float64 oracle.
 """
 import numpy as np
 import pytest
 
 from paper_2608_26004_gb300 import asymspec as A
 from paper_2608_26004_gb300 import synth
-from tests._parity import device_inputs
+from tests._parity import check_decisions, device_inputs, run_oracle
 
 pytestmark = pytest.mark.gpu
 
@@ -81,6 +82,11 @@ def test_two_consecutive_calls_match_the_workspace_entry_point(torch, first, sec
         Le, Ne = run_ex(torch, x, B, K, V, dtype, gate)
         assert np.array_equal(Ls, Le) and np.array_equal(Ns, Ne), f"case {idx} differs"
         assert np.all(Ls >= 0) and np.all(Ls <= K) and np.all(Ns >= 0) and np.all(Ns < V)
+        # a sample of the elements against the oracle: first, last, and six more
+        rng = np.random.default_rng(seed)
+        sel = np.unique(np.concatenate([[0, B - 1], rng.choice(B, size=min(B, 6), replace=False)]))
+        o = run_oracle(batch, mode=mode, select=sel, logprobs=False)
+        check_decisions(batch, sel, Ls[sel], Ns[sel], o, mode)
 
 
 def test_rows_above_the_limit_are_rejected_before_any_launch(torch):
@@ -108,6 +114,6 @@ def test_the_cases_cover_both_kernels_the_scratch_selects(torch):
         R = B * (K + 1)
         need = (_up(R * 16) + _up(B * 4) + _up(R * 48) + _up(R * info.cluster_size * 32)
                 + _up(R * info.cluster_size * 320))
-        if info.kernel in (A.KERNEL_TMA, A.KERNEL_RING):
+        if info.kernel == A.KERNEL_TMA:
             fits.append(need <= A.STATIC_SCRATCH_BYTES)
     assert True in fits and False in fits
