@@ -62,8 +62,16 @@ as such, so that a float32 implementation may legitimately differ there:
 * acceptance: |u - ratio / gamma_eff| < 1e-6, with u = 1 in greedy mode and
   ratio = softmax(t)[d] / softmax(b)[d] (greedy) or q(d) / p_draft (stochastic);
 * argmax: gap between the two largest scores < 1e-6 * max(1, |largest|);
-* inverse CDF: the target u * mass within 1e-5 of either neighbouring cumulative
-  boundary, or the residual mass itself below 1e-5.
+* inverse CDF: the target u * mass within CDF_BAND = 5e-7 (in units of
+  probability mass) of either neighbouring cumulative boundary, or the
+  residual mass itself below CDF_BAND.  An fp32 implementation's cumulative
+  position error is dominated by the float32 rounding of the two
+  normalisers the residual max(0, q - p) is built from: each (in log2 units,
+  of magnitude below 32) carries at most 2^-20 of rounding, a relative mass
+  error of at most 2^-20 ln 2 = 6.6e-7, and the position error is their
+  difference times the part of the fused mass between the boundary and the
+  target, a fraction of the total; the blocked float32 prefix adds about
+  2^-24 per level of the summation tree.
 
 Inputs are required to be finite (the paper's setting); a batch element with a
 non-finite logit in the data the step uses, a draft token outside [0, V), or
@@ -94,7 +102,7 @@ BF16 = 1
 
 ACCEPT_BAND = 1e-6
 ARGMAX_BAND = 1e-6
-CDF_BAND = 1e-5
+CDF_BAND = 5e-7
 LN2 = float(np.log(2.0))
 
 

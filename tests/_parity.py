@@ -177,7 +177,9 @@ def compare(batch, g, o, *, mode, select=None, logprobs=True, check_stats=True,
     assert np.all(computed[good][:, :batch.K]), "fused argmax missing on draft rows"
     fa_ok = good[:, None] & ~o.fused_gap_flag & computed
     assert np.array_equal(rt[..., 0][fa_ok], o.fused_argmax[fa_ok]), "fused argmax differs"
-    for i, k in np.argwhere(good[:, None] & o.fused_gap_flag & computed):
+    # (rows whose fused scores are not all finite, which the step does not
+    # use, have no defined argmax: the oracle reports -1 there)
+    for i, k in np.argwhere(good[:, None] & o.fused_gap_flag & computed & (o.fused_argmax >= 0)):
         assert argmax_valid(batch, sel[i], k, int(rt[i, k, 0]), params), \
             f"fused argmax of b={sel[i]} row {k} is not within the near-tie band"
     # the token each row would emit: exact, or valid where the row's own

@@ -137,11 +137,14 @@ def test_large_workloads_sampled(torch, cfg, mode):
 @pytest.mark.parametrize("mode", [GREEDY, STOCH])
 def test_divergence_sweep_gate_response(torch, mode):
     rows = []
+    flagged = total = 0
     for si, s in enumerate(synth.CONFIGS[4].sweep):
         batch = synth.make_config(4, sweep_index=si)
         o = run_oracle(batch, mode=mode, logprobs=False)
         gp = run_gpu(batch, torch, mode=mode, full=False)
-        compare(batch, gp, o, mode=mode, logprobs=False)
+        c = compare(batch, gp, o, mode=mode, logprobs=False, max_flagged=0.125)
+        flagged += c["flagged"]
+        total += batch.B
         g = run_gpu(batch, torch, mode=mode, logprobs=False)
         compare(batch, g, o, mode=mode, logprobs=False)
         hist_g = np.bincount(gp["accept_len"], minlength=batch.K + 1)
@@ -150,6 +153,9 @@ def test_divergence_sweep_gate_response(torch, mode):
         assert np.abs(hist_g - hist_o).sum() <= 2 * nflag
         rows.append((s, float(np.mean(g["row_stats"][:, :batch.K, 4])),
                      float(np.mean(g["row_stats"][:, :batch.K, 5]))))
+    # near-ties over the six points (the oracle flags 9 of 192 stochastic
+    # elements and none of the greedy ones; each is checked for validity)
+    assert flagged <= 0.06 * total, f"{flagged} of {total} elements flagged"
     # the gate relaxes as the compressed context diverges: mean D rises,
     # mean gamma_eff falls, from D = 0 at s = 0 (z_c == z_f)
     Ds = [r[1] for r in rows]
