@@ -343,7 +343,7 @@ class FuseVerify:
                  uniforms=None, *, gamma=0.5, beta=1.0, lam=0.1, mode=MODE_GREEDY,
                  divergence=DIV_JSD, fuse_bonus=False, row_stats=False, row_tokens=False,
                  fused_logprobs=False, cluster_size=0, kernel=KERNEL_AUTO, out=None,
-                 delta_source=DELTA_AB, test_flags=0):
+                 delta_source=DELTA_AB, test_flags=0, block_threads=0):
         import torch
         B, K1, V = logits_full.shape
         K = K1 - 1
@@ -373,8 +373,8 @@ class FuseVerify:
         if fused_logprobs and "fused_logprobs" not in res:
             res["fused_logprobs"] = torch.empty(B, K1, V, dtype=torch.float32, device=dev)
         gate = gate_params(gamma, beta, lam, mode, divergence, fuse_bonus, delta_source)
-        opts = (LaunchOpts(cluster_size, 0, kernel, test_flags)
-                if (cluster_size or kernel or test_flags) else None)
+        opts = (LaunchOpts(cluster_size, block_threads, kernel, test_flags)
+                if (cluster_size or kernel or test_flags or block_threads) else None)
         stream = torch.cuda.current_stream(dev).cuda_stream
         st = fuse_verify_ex(
             _ptr(logits_full), _ptr(logits_comp), _ptr(logits_ver), _ptr(draft_tokens),

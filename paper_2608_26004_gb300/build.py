@@ -18,10 +18,11 @@ CSRC = os.path.join(HERE, "csrc")
 # one translation unit per kernel family and dtype, compiled in parallel
 CUDA_SRC = [os.path.join(CSRC, f) for f in (
     "asymspec.cu", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu", "k_tma_bf16_prod.cu",
-    "k_tma_f32_prod.cu", "k_tma_bf16_any_s.cu", "k_tma_f32_any_s.cu", "k_draft.cu", "k_xvocab.cu")]
+    "k_tma_f32_prod.cu", "k_tma_bf16_any_s.cu", "k_tma_f32_any_s.cu", "k_row_bf16.cu",
+    "k_row_f32.cu", "k_draft.cu", "k_xvocab.cu")]
 CUDA_HEADERS = [os.path.join(CSRC, f) for f in (
-    "device_common.cuh", "kernel_generic.cuh", "kernel_tma.cuh", "kernel_draft.cuh",
-    "kernel_xvocab.cuh", "kernels.h")]
+    "device_common.cuh", "kernel_generic.cuh", "kernel_tma.cuh", "kernel_row.cuh",
+    "kernel_draft.cuh", "kernel_xvocab.cuh", "kernels.h")]
 CUDA_LIB = os.path.join(HERE, "libasymspec.so")
 GENCODE = "arch=compute_103a,code=sm_103a"
 

@@ -6,6 +6,10 @@
 //                        programs; the default for 16-byte aligned rows.  Its
 //                        rows are decided, and Algorithm 1's scan run, by
 //                        decide_rows, a second launch.
+//   fuse_verify_row      (kernel_row.cuh) the same decomposition with a CTA
+//                        shape chosen per workload and the lean per-entry
+//                        arithmetic: the production program of the
+//                        stochastic JSD step (no debug outputs, delta = a - b).
 //   fuse_verify_generic  (kernel_generic.cuh) one cluster per row, any
 //                        element-aligned input; folds the scan into the same
 //                        launch through a per-element ticket in the workspace.
@@ -17,6 +21,7 @@
 #include "device_common.cuh"
 #include "kernel_generic.cuh"
 #include "kernel_tma.cuh"
+#include "kernel_row.cuh"
 #include "kernel_draft.cuh"
 #include "kernel_xvocab.cuh"
 #include "kernels.h"
@@ -37,11 +42,23 @@ constexpr int kTmaPreferredSmem = 113 * 1024;  // two CTAs per SM
 struct Plan {
   int kernel;  // ASYMSPEC_KERNEL_*
   int C, W, VE, sh_off, smem;
-  int group_stride;  // TMA and ring kernels: floats per row and CTA of group masses
+  int group_stride;  // TMA kernels: floats per row and CTA of group masses
   long long rows;
   long long ctas;  // grid size
   bool vector_path;
+  bool row;          // the production row kernel (fuse_verify_row) runs
+  int nt, minb;      // its CTA shape: threads, CTAs per SM (kTThreads, 2 otherwise)
 };
+
+// Shared memory one SM offers its CTAs, and what each CTA costs beyond its
+// own allocation.
+constexpr int kSmemPerSm = 228 * 1024;
+constexpr int kSmemPerCta = 1024;
+
+const void* row_kernel(int dtype, int nt, int minb) {
+  return dtype == ASYMSPEC_FP32 ? row_kernel_f32(nt, minb) : row_kernel_bf16(nt, minb);
+}
+
 
 int elt_size(int dtype) { return dtype == ASYMSPEC_FP32 ? 4 : 2; }
 
@@ -95,6 +112,48 @@ bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
   return false;
 }
 
+// The production row kernel: CTA shapes in order of preference (bf16: 224
+// threads three to an SM, else 256 threads two to an SM; fp32: 256 threads
+// two to an SM), each with the smallest cluster (1, 2, 4, 8, 10, 12, 16)
+// whose slice and shared state fit that many CTAs per SM and whose slice
+// takes at most kMaxRounds vectors per thread.  forced_nt, forced_C: the
+// caller's asymspec_launch_opts.
+bool plan_row(int V, int dtype, int forced_C, int forced_nt, Plan* pl) {
+  const int elt = elt_size(dtype);
+  const int VE = 16 / elt;
+  struct Shape {
+    int nt, minb;
+  };
+  const Shape shapes_bf16[] = {{224, 3}, {256, 3}, {256, 2}};
+  const Shape shapes_f32[] = {{256, 2}};
+  const Shape* shapes = dtype == ASYMSPEC_FP32 ? shapes_f32 : shapes_bf16;
+  const int nshapes = dtype == ASYMSPEC_FP32 ? 1 : 3;
+  for (int si = 0; si < nshapes; ++si) {
+    const Shape sh = shapes[si];
+    if (forced_nt && sh.nt != forced_nt) continue;
+    if (!row_kernel(dtype, sh.nt, sh.minb)) continue;
+    for (int C : kClusterOrder) {
+      if (forced_C && C != forced_C) continue;
+      const long long per = (static_cast<long long>(V) + C - 1) / C;
+      const long long W = round_up_ll(per, VE);
+      const long long sh_off = round_up_ll(3 * W * elt, 128);
+      const long long smem = sh_off + row_shared_bytes(C);
+      if (W / VE > static_cast<long long>(kMaxRounds) * sh.nt) continue;
+      if (sh.minb * (smem + kSmemPerCta) > kSmemPerSm) continue;
+      if (sh.minb == 2 && smem > kTmaPreferredSmem) continue;
+      pl->C = C;
+      pl->W = static_cast<int>(W);
+      pl->sh_off = static_cast<int>(sh_off);
+      pl->smem = static_cast<int>(smem);
+      pl->group_stride = kGroupsMax;
+      pl->nt = sh.nt;
+      pl->minb = sh.minb;
+      return true;
+    }
+  }
+  return false;
+}
+
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 size_t ws_records_bytes(int B, int K) {
@@ -128,20 +187,41 @@ TmaLayout tma_layout(int B, int K, int C, int group_stride = kGroupsMax) {
   return L;
 }
 
+// prod_row: the call is the production stochastic JSD step (no debug
+// outputs, no per-row tokens, delta = a - b), which fuse_verify_row runs.
 int make_plan(int B, int K, int V, int dtype, const asymspec_launch_opts* opts, bool vec_ok,
-              size_t ws_bytes, Plan* pl) {
+              size_t ws_bytes, bool prod_row, Plan* pl) {
   const int elt = elt_size(dtype);
   const int forced_C = (opts && opts->cluster_size > 0) ? opts->cluster_size : 0;
   const int forced_kernel = opts ? opts->kernel : 0;
+  const int forced_nt = opts ? opts->block_threads : 0;
   if (forced_C < 0 || forced_C > 16) return ASYMSPEC_ERR_INVALID_ARG;
   if (forced_kernel != 0 && forced_kernel != ASYMSPEC_KERNEL_GENERIC &&
       forced_kernel != ASYMSPEC_KERNEL_TMA)
     return ASYMSPEC_ERR_INVALID_ARG;
   pl->rows = static_cast<long long>(B) * (K + 1);
   pl->vector_path = vec_ok;
+  pl->row = false;
+  pl->nt = kTThreads;
+  pl->minb = 2;
   if (ws_bytes < cluster_ws_bytes(B, K)) return ASYMSPEC_ERR_WORKSPACE;
   bool ok = false;
-  if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, pl)) {
+  if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && prod_row &&
+      plan_row(V, dtype, forced_C, forced_nt, pl)) {
+    if (ws_bytes >= tma_layout(B, K, pl->C).total) {
+      pl->kernel = ASYMSPEC_KERNEL_TMA;
+      pl->VE = 16 / elt;
+      pl->row = true;
+      ok = true;
+    } else if (forced_kernel == ASYMSPEC_KERNEL_TMA) {
+      return ASYMSPEC_ERR_WORKSPACE;
+    }
+  }
+  // other shapes than 256 threads exist for the production row kernel only
+  if (!ok && forced_nt != 0 && forced_nt != kTThreads) return ASYMSPEC_ERR_UNSUPPORTED;
+  if (ok) {
+    // the production row kernel
+  } else if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, pl)) {
     // the TMA kernel leaves each row's results in the workspace; the generic
     // kernel, which needs only the records and tickets, runs when it is short
     if (ws_bytes >= tma_layout(B, K, pl->C).total) {
@@ -168,6 +248,7 @@ using KernelFn = const void*;  // a __global__ function taking KParams (or SPara
 
 // sel: the TMA kernel's program set (tma_program_set; 0 = run-time dispatch)
 KernelFn pick_kernel(const Plan& pl, int dtype, bool stoch, int sel = 0) {
+  if (pl.row) return row_kernel(dtype, pl.nt, pl.minb);
   if (pl.kernel == ASYMSPEC_KERNEL_TMA)
     return dtype == ASYMSPEC_FP32 ? tma_kernel_f32(stoch, sel) : tma_kernel_bf16(stoch, sel);
   return generic_kernel(dtype, pl.vector_path, stoch);
@@ -214,7 +295,7 @@ cudaLaunchConfig_t launch_config(const Plan& pl, long long ctas, cudaStream_t st
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.gridDim = dim3(static_cast<unsigned>(ctas));
-  cfg.blockDim = dim3(pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : kTThreads);
+  cfg.blockDim = dim3(pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : pl.nt);
   cfg.dynamicSmemBytes = pl.smem;
   cfg.stream = stream;
   cfg.attrs = attr;
@@ -265,7 +346,9 @@ int check_params(const asymspec_gate_params* gp) {
 }
 
 int check_opts(const asymspec_launch_opts* opts) {
-  if (opts && opts->block_threads != 0) return ASYMSPEC_ERR_INVALID_ARG;
+  if (opts && opts->block_threads != 0 && opts->block_threads != 224 &&
+      opts->block_threads != 256)
+    return ASYMSPEC_ERR_INVALID_ARG;
   if (opts && (opts->test_flags & ~ASYMSPEC_TEST_COPY_GIVE_UP) != 0) return ASYMSPEC_ERR_INVALID_ARG;
   if (opts && ((opts->timing_begin == nullptr) != (opts->timing_end == nullptr)))
     return ASYMSPEC_ERR_INVALID_ARG;
@@ -413,10 +496,14 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
   if (st) return st;
   const bool vec_ok = (static_cast<long long>(V) * elt_size(dtype)) % 16 == 0;
   Plan pl = {};
-  st = make_plan(B, K, V, dtype, opts, vec_ok, asymspec_workspace_bytes(B, K, V), &pl);
+  const bool stoch_p = gp.mode == ASYMSPEC_MODE_STOCHASTIC;
+  st = make_plan(B, K, V, dtype, opts, vec_ok, asymspec_workspace_bytes(B, K, V),
+                 stoch_p && gp.divergence == ASYMSPEC_DIV_JSD &&
+                     (gp.flags & ASYMSPEC_FLAG_DELTA_MASK) == ASYMSPEC_DELTA_AB,
+                 &pl);
   if (st) return st;
   out->cluster_size = pl.C;
-  out->block_threads = pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : kTThreads;
+  out->block_threads = pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : pl.nt;
   out->slice_elems = pl.W;
   out->smem_bytes = pl.smem;
   out->ctas = pl.ctas;
@@ -474,7 +561,10 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   const bool vec_ok = (static_cast<long long>(V) * elt) % 16 == 0 && aligned(logits_full, 16) &&
                       aligned(logits_comp, 16) && aligned(logits_ver, 16);
   Plan pl = {};
-  st = make_plan(B, K, V, dtype, opts, vec_ok, workspace_bytes, &pl);
+  const bool prod_row = stoch && gp.divergence == ASYMSPEC_DIV_JSD && !out_row_stats &&
+                        !out_fused_logprobs && !out_row_tokens &&
+                        (gp.flags & ASYMSPEC_FLAG_DELTA_MASK) == ASYMSPEC_DELTA_AB;
+  st = make_plan(B, K, V, dtype, opts, vec_ok, workspace_bytes, prod_row, &pl);
   if (st) return st;
 
   KParams P;
@@ -515,6 +605,8 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   P.row_stat = nullptr;
   P.pass2_rec = nullptr;
   P.group_mass = nullptr;
+  P.tma_threads = pl.nt;
+  P.row_blocks = pl.row ? 1 : 0;
   // the chunk waits of the TMA kernel: bounded, or (test hook) giving up at once
   P.copy_wait_ns =
       (opts && (opts->test_flags & ASYMSPEC_TEST_COPY_GIVE_UP)) ? 0ull : kCopyTimeoutNs;

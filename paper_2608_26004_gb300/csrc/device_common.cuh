@@ -443,7 +443,9 @@ struct KParams {
   void* row_stat;       // [B(K+1)] RowStat (rank 0 of the row's cluster)
   float* pass2_rec;     // [B(K+1)][C] X2 records (8 floats), one per CTA
   float* group_mass;    // [B(K+1)][C][group_stride] inverse-CDF group masses (stochastic)
-  int group_stride;     // floats per row and CTA in group_mass (8 per round of the slice)
+  int group_stride;     // floats per row and CTA in group_mass (one per warp and round)
+  int tma_threads;      // threads per CTA of the row kernel (its group layout)
+  int row_blocks;       // 1: fuse_verify_row's layout, one inverse-CDF group per warp block
   unsigned long long copy_wait_ns;  // limit of each bulk-copy wait (0: give up at once)
 };
 

@@ -1,0 +1,495 @@
+// Production kernel of the stochastic step (JSD gate, delta = a - b, no
+// debug outputs): the program bench workloads and serving run.
+//
+// Same decomposition as fuse_verify_tma (kernel_tma.cuh), whose records it
+// leaves for the same decision kernel: one cluster of C CTAs per row triple
+// (a_k, b_k, t_k); CTA r brings entries [r W, (r+1) W) of the three rows
+// into shared memory with 1-D bulk copies in kChunks chunks, each on its own
+// mbarrier; pass 1 (the normalisers of Eqs. 1-3) streams the slice as the
+// chunks land; the CTAs exchange pass-1 records through distributed shared
+// memory and one cluster barrier; pass 2 reads the slice again from shared
+// memory.  Each logit row is read from HBM once.
+//
+// What differs from fuse_verify_tma is the shape of the work, chosen for
+// the instruction budget (the arithmetic alone is about 27 instructions per
+// vocabulary entry against 6 bytes read, so every instruction a CTA spends
+// once per row counts):
+//   * the CTA shape is a template parameter: NT threads, MINB CTAs per SM
+//     (the register cap of __launch_bounds__);
+//   * each warp owns a contiguous block of the slice: its lane 0 issues the
+//     block's bulk copies (two chunks, each on the warp's own mbarrier), the
+//     warp waits for its own data only, and each step reads 32 consecutive
+//     16-byte vectors per stream (no bank conflicts);
+//   * the block of a warp is one inverse-CDF group: its mass is the warp's
+//     residual (or fused) sum, which the warp reduces anyway, so pass 2 needs
+//     no per-step group reductions (the decision kernel walks the group's
+//     vectors);
+//   * one 16-byte vector per stream per step, unpacked pair by pair from the
+//     raw words (bf16 -> fp32 is a shift or a mask), two fp32 lanes per
+//     add/sub/mul/fma instruction;
+//   * the divergence of Eq. 3 in one product per pair.  With p = softmax(a),
+//     q = softmax(b) in log2 units, e = q/p = 2^d (d = log2 q - log2 p) and
+//     w = 1 + e, each entry contributes to 2 JSD (in bits)
+//         p log2(2p/(p+q)) + q log2(2q/(p+q)) = p [w (1 - log2 w) + e d],
+//     a sum of small non-negative terms with no cancellation at the end;
+//   * the residual max(0, q_f - p) and fused score (t + beta (a - b)) log2 e
+//     are formed exactly as the decision kernel's inverse-CDF walk forms
+//     them (res_pair), so the group masses and the walk agree bit for bit.
+//
+// Every wait is bounded as in fuse_verify_tma: a chunk that does not land in
+// time (KParams::copy_wait_ns) marks the row ASYMSPEC_DATA_TIMEOUT, the CTA
+// still reaches the cluster barrier, and thread 0 drains its copies
+// (bounded) before the CTA exits.
+#pragma once
+
+#include "kernel_tma.cuh"
+
+namespace asymspec_impl {
+
+// A 16-byte vector of the slice, as raw words; pair(h) widens entries
+// 2h, 2h + 1 to fp32.
+template <typename T>
+struct RawVec;
+template <>
+struct RawVec<__nv_bfloat16> {
+  static constexpr int NP = 4;
+  uint4 v;
+  __device__ __forceinline__ f2 pair(int h) const {
+    const unsigned w = h == 0 ? v.x : h == 1 ? v.y : h == 2 ? v.z : v.w;
+    return pk(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+  }
+};
+template <>
+struct RawVec<float> {
+  static constexpr int NP = 2;
+  float4 v;
+  __device__ __forceinline__ f2 pair(int h) const { return h == 0 ? pk(v.x, v.y) : pk(v.z, v.w); }
+};
+template <typename T>
+__device__ __forceinline__ RawVec<T> raw_load(const T* p) {
+  RawVec<T> r;
+  r.v = *reinterpret_cast<const decltype(r.v)*>(p);
+  return r;
+}
+
+// Constants of a row's pass 2 (log2 units): L2 = log2 e, bL2 = beta log2 e,
+// nA2 = -LSE(a) log2 e, nS2 = -LSE(s) log2 e, cAB2 = (LSE(a) - LSE(b)) log2 e.
+struct ResConst {
+  f2 L2, nL2, bL2, nA2, nS2, cAB2, one2;
+};
+
+__device__ __forceinline__ ResConst res_const(float beta, float A2, float B2, float S2) {
+  ResConst k;
+  k.L2 = pk(kLog2e, kLog2e);
+  k.nL2 = pk(-kLog2e, -kLog2e);
+  const float bl = beta * kLog2e;
+  k.bL2 = pk(bl, bl);
+  k.nA2 = pk(-A2, -A2);
+  k.nS2 = pk(-S2, -S2);
+  const float c = A2 - B2;
+  k.cAB2 = pk(c, c);
+  k.one2 = pk(1.f, 1.f);
+  return k;
+}
+
+// The masses of one pair of entries: p = softmax(a), the fused q_f =
+// softmax(t + beta (a - b)) and the residual r = max(0, q_f - p); amb = a - b.
+// The row kernel's pass 2 and the decision kernel's walk both use this.
+__device__ __forceinline__ void res_pair(f2 a2, f2 b2, f2 t2, const ResConst& k, f2& amb, f2& p,
+                                         f2& qf, f2& r) {
+  amb = sub2(a2, b2);
+  p = ex2_2(fma2(a2, k.L2, k.nA2));
+  qf = ex2_2(fma2(t2, k.L2, fma2(k.bL2, amb, k.nS2)));
+  r = relu2(sub2(qf, p));
+}
+
+// The JSD term of a pair (see the header): p [w (1 - log2 w) + e d] with
+// d = log2 q - log2 p = -(a - b) log2 e + (LSE(a) - LSE(b)) log2 e.
+__device__ __forceinline__ f2 jsd_pair(f2 amb, f2 p, const ResConst& k, f2 jacc) {
+  const f2 d = fma2(amb, k.nL2, k.cAB2);
+  const f2 e = ex2_2(d);
+  const f2 w = add2(e, k.one2);
+  const f2 x = sub2(k.one2, lg2_2(w));
+  return fma2(p, fma2(w, x, mul2(e, d)), jacc);
+}
+
+
+// ---------------------------------------------------------------- layout
+
+constexpr int kRowMaxWarps = 8;
+constexpr int kRowChunks = 2;  // bulk-copy chunks per warp block
+
+// A warp's pass-1 record: the references (nats) and sums of
+// 2^((x - ref) log2 e) of a, b and the fused score, and its data-error bits.
+struct __align__(16) W1 {
+  float ref[3], s[3];
+  unsigned bad;
+  float pad;
+};
+
+// Fixed shared state of the row kernel; the C pass-1 records pushed by the
+// cluster follow it (recv()).
+struct __align__(16) RowShared {
+  unsigned long long bar[kRowMaxWarps][kRowChunks];  // per warp and chunk
+  union {                                            // per-warp records, one pass at a time
+    W1 w1[kRowMaxWarps];
+    X2 w2[kRowMaxWarps];
+  };
+  float lse[4];                 // the row's normalisers (a, b, -, s)
+  unsigned broken;              // a chunk copy timed out
+  float qown;                   // this slice's fused mass (draft rows), from pass 1
+  unsigned long long wait_ns;   // limit of each chunk wait (KParams::copy_wait_ns)
+  __device__ X1* recv() { return reinterpret_cast<X1*>(this + 1); }
+};
+static_assert(sizeof(W1) == 32 && sizeof(X2) == 32, "warp records share storage");
+static_assert(sizeof(RowShared) % 16 == 0, "records after RowShared stay 16-byte aligned");
+
+__host__ __device__ constexpr int row_shared_bytes(int C) {
+  return static_cast<int>(sizeof(RowShared) + C * sizeof(X1));
+}
+
+// Lane 0 of warp w: the bulk copies of the warp's block [v0, v1) of the
+// slice (vectors), in two chunks (the first ceil(R/2) steps, then the rest),
+// each completing on the warp's own mbarrier.
+template <typename T>
+__device__ __forceinline__ void issue_block(const KParams& P, RowShared* sh, int w, size_t off,
+                                            int v0, int v1, int split, T* sa, T* sb, T* st) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+#pragma unroll
+  for (int q = 0; q < kRowChunks; ++q) {
+    const int c0 = q == 0 ? v0 : min(v1, split), c1 = q == 0 ? min(v1, split) : v1;
+    const unsigned bytes = static_cast<unsigned>(max(0, c1 - c0)) * 16u;
+    mbar_arrive_expect_tx(&sh->bar[w][q], 3u * bytes);
+    if (bytes) {
+      const int e0 = c0 * VE;
+      bulk_load(sa + e0, static_cast<const T*>(P.a) + off + e0, bytes, &sh->bar[w][q]);
+      bulk_load(sb + e0, static_cast<const T*>(P.b) + off + e0, bytes, &sh->bar[w][q]);
+      bulk_load(st + e0, static_cast<const T*>(P.t) + off + e0, bytes, &sh->bar[w][q]);
+    }
+  }
+}
+
+// ---------------------------------------------------------------- pass 1
+
+// Pass 1 over the warp's block [v0, v1) (R steps, chunk 1 from step R1 on)
+// with one fixed reference per warp and stream.  DRAFT: the normalisers of
+// a, b and the fused score s; the bonus row needs s only.  Returns true when
+// a lane's sum reached 2^100 or is not finite (the CTA then redoes its slice
+// with a running maximum).  Every lane ends with the warp's record.
+template <typename T, bool DRAFT>
+__device__ __forceinline__ bool row_pass1(const T* ra, const T* rb, const T* rt, int v0, int v1,
+                                          int R, int R1, float beta, RowShared* sh, int w,
+                                          W1& e) {
+  constexpr int NP = RawVec<T>::NP;
+  constexpr int VE = 2 * NP;
+  const int lane = static_cast<int>(threadIdx.x & 31);
+  if (!sh->broken && !mbar_wait_bounded(&sh->bar[w][0], 0u, sh->wait_ns))
+    atomicOr(&sh->broken, kBadTimeout);
+  const f2 L2 = pk(kLog2e, kLog2e);
+  const float bl = beta * kLog2e;
+  const f2 bL2 = pk(bl, bl);
+  // references (nats): the largest of the warp's first pairs of a, b and the
+  // fused score (every lane's first vector is in chunk 0)
+  float ra0 = -INFINITY, rb0 = -INFINITY, rs0 = -INFINITY;
+  const int i0 = v0 + lane;
+  if (i0 < v1) {
+    const f2 a2 = first_pair(ra + i0 * VE), b2 = first_pair(rb + i0 * VE);
+    const f2 t2 = first_pair(rt + i0 * VE);
+    const f2 s2 = fma2(pk(beta, beta), sub2(a2, b2), t2);
+    ra0 = fmaxf(lo_of(a2), hi_of(a2));
+    rb0 = fmaxf(lo_of(b2), hi_of(b2));
+    rs0 = fmaxf(lo_of(s2), hi_of(s2));
+  }
+  if (DRAFT) {
+    ra0 = warp_max(ra0);
+    rb0 = warp_max(rb0);
+  }
+  rs0 = warp_max(rs0);
+  const float nA = -ra0 * kLog2e, nB = -rb0 * kLog2e, nS = -rs0 * kLog2e;
+  const f2 nA2 = pk(nA, nA), nB2 = pk(nB, nB), nS2 = pk(nS, nS);
+  f2 acc_a = 0ull, acc_b = 0ull, acc_s = 0ull;
+  auto step = [&](int i) {
+    const RawVec<T> va = raw_load(ra + i * VE), vb = raw_load(rb + i * VE);
+    const RawVec<T> vt = raw_load(rt + i * VE);
+#pragma unroll
+    for (int h = 0; h < NP; ++h) {
+      const f2 a2 = va.pair(h), b2 = vb.pair(h), t2 = vt.pair(h);
+      if (DRAFT) {
+        acc_a = add2(acc_a, ex2_2(fma2(a2, L2, nA2)));
+        acc_b = add2(acc_b, ex2_2(fma2(b2, L2, nB2)));
+      }
+      acc_s = add2(acc_s, ex2_2(fma2(t2, L2, fma2(bL2, sub2(a2, b2), nS2))));
+    }
+  };
+  int r = 0;
+#pragma unroll 2
+  for (; r < R1; ++r) {
+    const int i = i0 + 32 * r;
+    if (i < v1) step(i);
+  }
+  if (!sh->broken && !mbar_wait_bounded(&sh->bar[w][1], 0u, sh->wait_ns))
+    atomicOr(&sh->broken, kBadTimeout);
+#pragma unroll 2
+  for (; r < R; ++r) {
+    const int i = i0 + 32 * r;
+    if (i < v1) step(i);
+  }
+  float sa = DRAFT ? hsum2(acc_a) : 0.f, sb = DRAFT ? hsum2(acc_b) : 0.f, ss = hsum2(acc_s);
+  const bool ovf = !(ss < kSumLimit) || (DRAFT && (!(sa < kSumLimit) || !(sb < kSumLimit)));
+  // the warp's sums (its references are equal across lanes)
+  float z = 0.f;
+  warp_sum4(sa, sb, ss, z);
+  e.ref[0] = ra0;
+  e.ref[1] = rb0;
+  e.ref[2] = rs0;
+  e.s[0] = sa;
+  e.s[1] = sb;
+  e.s[2] = ss;
+  e.bad = 0u;
+  e.pad = 0.f;
+  return ovf;
+}
+
+// Fallback of row_pass1 (a sum reached 2^100, or non-finite data): each lane
+// keeps a running maximum per stream over its vectors of the warp's block,
+// rescaling its sum when the maximum rises; the lanes then merge.  The block
+// is in shared memory (its chunks have landed, or the warp gave up waiting).
+template <typename T, bool DRAFT>
+__device__ __forceinline__ void row_pass1_online(const T* ra, const T* rb, const T* rt, int v0,
+                                                 int v1, float beta, W1& e) {
+  constexpr int NP = RawVec<T>::NP;
+  constexpr int VE = 2 * NP;
+  const int lane = static_cast<int>(threadIdx.x & 31);
+  float m[3] = {-INFINITY, -INFINITY, -INFINITY};  // running maxima of a, b, s (nats)
+  float s[3] = {0.f, 0.f, 0.f};                    // sums of 2^((x - m) log2 e)
+  for (int i = v0 + lane; i < v1; i += 32) {
+    const RawVec<T> va = raw_load(ra + i * VE), vb = raw_load(rb + i * VE);
+    const RawVec<T> vt = raw_load(rt + i * VE);
+#pragma unroll
+    for (int h = 0; h < NP; ++h) {
+      const f2 a2 = va.pair(h), b2 = vb.pair(h), t2 = vt.pair(h);
+      const f2 s2 = fma2(pk(beta, beta), sub2(a2, b2), t2);
+      float x[3][2];
+      upk(a2, x[0][0], x[0][1]);
+      upk(b2, x[1][0], x[1][1]);
+      upk(s2, x[2][0], x[2][1]);
+#pragma unroll
+      for (int q = 0; q < 3; ++q) {
+        if (!DRAFT && q < 2) continue;
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          const float v = x[q][j];
+          if (v > m[q]) {
+            s[q] = s[q] * ex2((m[q] - v) * kLog2e);
+            m[q] = v;
+          }
+          s[q] += ex2((v - m[q]) * kLog2e);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < 3; ++q) {
+    const float M = warp_max(m[q]);
+    const float sc = (s[q] == 0.f || m[q] == M) ? s[q] : s[q] * ex2((m[q] - M) * kLog2e);
+    e.ref[q] = M;
+    e.s[q] = warp_sum(sc);
+  }
+  if (!DRAFT) {
+    e.ref[0] = e.ref[1] = -INFINITY;
+    e.s[0] = e.s[1] = 0.f;
+  }
+}
+
+// ---------------------------------------------------------------- pass 2
+
+// Pass 2 over the warp's block: DRAFT, the JSD terms (see the header) and
+// the residual masses; the bonus row, the fused masses.  Returns through
+// jsum / msum the warp's sums (every lane ends with them): msum is the mass
+// of the warp's inverse-CDF group.
+template <typename T, bool DRAFT>
+__device__ __forceinline__ void row_pass2(const T* ra, const T* rb, const T* rt, int v0, int v1,
+                                          int R, const ResConst& k, float& jsum, float& msum) {
+  constexpr int NP = RawVec<T>::NP;
+  constexpr int VE = 2 * NP;
+  const int lane = static_cast<int>(threadIdx.x & 31);
+  f2 jacc = 0ull, macc = 0ull;
+  const int i0 = v0 + lane;
+#pragma unroll 2
+  for (int r = 0; r < R; ++r) {
+    const int i = i0 + 32 * r;
+    if (i < v1) {
+      const RawVec<T> va = raw_load(ra + i * VE), vb = raw_load(rb + i * VE);
+      const RawVec<T> vt = raw_load(rt + i * VE);
+#pragma unroll
+      for (int h = 0; h < NP; ++h) {
+        f2 amb, p, qf, rr;
+        res_pair(va.pair(h), vb.pair(h), vt.pair(h), k, amb, p, qf, rr);
+        if (DRAFT) {
+          macc = add2(macc, rr);
+          jacc = jsd_pair(amb, p, k, jacc);
+        } else {
+          macc = add2(macc, qf);
+        }
+      }
+    }
+  }
+  float j = hsum2(jacc), m = hsum2(macc), z0 = 0.f, z1 = 0.f;
+  warp_sum4(j, m, z0, z1);
+  jsum = j;
+  msum = m;
+}
+
+// ---------------------------------------------------------------- the kernel
+
+template <typename T, int NT, int MINB>
+__global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
+  static_assert(NT % 32 == 0 && NT / 32 <= kRowMaxWarps, "at most kRowMaxWarps warps");
+  constexpr int NW = NT / 32;
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  constexpr unsigned FD = F_LA | F_LB | F_LS;
+  extern __shared__ __align__(128) unsigned char smem_row[];
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int tid = static_cast<int>(threadIdx.x);
+  const int lane = tid & 31, warp = tid >> 5;
+  const int C = P.C;
+  const unsigned row32 = blockIdx.x / static_cast<unsigned>(C);
+  const unsigned K1 = static_cast<unsigned>(P.K) + 1u;
+  const int W = P.W;
+  const int lo = rank * W;
+  const int n = max(0, min(W, P.V - lo));
+  const int nv = n / VE;
+  // this warp's block of the slice, its steps, and the step chunk 1 starts at
+  const int bw = row_block_vectors(nv, NW);
+  const int v0 = min(nv, warp * bw), v1 = min(nv, v0 + bw);
+  const int R = (v1 - v0 + 31) / 32, R1 = (R + 1) / 2;
+  T* sa = reinterpret_cast<T*>(smem_row);
+  T* sb = sa + W;
+  T* st = sb + W;
+  RowShared* sh = reinterpret_cast<RowShared*>(smem_row + P.sh_off);
+  const int bi = static_cast<int>(row32 / K1);
+  const int k = static_cast<int>(row32 - static_cast<unsigned>(bi) * K1);
+  const bool draft = k < P.K;
+
+  // each warp brings in its own block: no CTA barrier before the copies
+  if (lane == 0) {
+    mbar_init(&sh->bar[warp][0], 1);
+    mbar_init(&sh->bar[warp][1], 1);
+    fence_mbar_init();
+    issue_block<T>(P, sh, warp, static_cast<size_t>(row32) * P.V + lo, v0, v1, v0 + 32 * R1, sa,
+                   sb, st);
+  }
+  if (tid == 0) {
+    sh->broken = 0;
+    sh->wait_ns = P.copy_wait_ns;
+  }
+  // warp 0 keeps the row's draft token, loaded while the slice is in flight
+  int dtok = -1;
+  if (warp == 0 && draft) dtok = P.tokens[static_cast<size_t>(bi) * P.K + k];
+  __syncthreads();  // every warp's barriers and the shared flags are initialised
+
+  // ---- pass 1: the row normalisers, combined over the cluster
+  W1 e;
+  const bool ovf = draft ? row_pass1<T, true>(sa, sb, st, v0, v1, R, R1, P.beta, sh, warp, e)
+                         : row_pass1<T, false>(sa, sb, st, v0, v1, R, R1, P.beta, sh, warp, e);
+  if (lane == 0) sh->w1[warp] = e;
+  if (__syncthreads_or(ovf)) {
+    // an entry far above its warp's reference (or non-finite data): redo the
+    // slice with running maxima
+    if (draft) row_pass1_online<T, true>(sa, sb, st, v0, v1, P.beta, e);
+    else row_pass1_online<T, false>(sa, sb, st, v0, v1, P.beta, e);
+    e.bad = 0u;
+    e.pad = 0.f;
+    if (lane == 0) sh->w1[warp] = e;
+    __syncthreads();
+  }
+  if (warp == 0) {
+    // the CTA's record: the warps' records merged (their references differ)
+    X1 x = x1_neutral();
+    if (lane < NW) {
+      const W1 r = sh->w1[lane];
+      x.ref[0] = r.ref[0];
+      x.ref[1] = r.ref[1];
+      x.ref[3] = r.ref[2];
+      x.s[0] = r.s[0];
+      x.s[1] = r.s[1];
+      x.s[3] = r.s[2];
+    }
+    if (draft) warp_reduce_x1<FD>(x);
+    else warp_reduce_x1<F_LS>(x);
+    x.bad = sh->broken;
+    if (dtok >= lo && dtok < lo + n) {  // this CTA's slice holds the draft token
+      x.da = to_f32(sa[dtok - lo]);
+      x.db = to_f32(sb[dtok - lo]);
+      x.dt = to_f32(st[dtok - lo]);
+    }
+    push_record(x, sh->recv(), rank, C, cluster);
+  }
+  cluster_barrier(warp == 0);  // every CTA's pass-1 record is in every CTA
+
+  if (warp == 0) {
+    float lse[4];
+    X1 x = (lane < C) ? sh->recv()[lane] : x1_neutral();
+    if (draft) warp_reduce_x1<FD>(x);
+    else warp_reduce_x1<F_LS>(x);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) lse[q] = x.ref[q] + logf(x.s[q]);
+    if (lane == 0) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) sh->lse[q] = lse[q];
+      // this slice's fused mass, from its own pass-1 record (the draw falls
+      // back to the fused masses when the row's whole residual is zero)
+      const X1& own = sh->recv()[rank];
+      sh->qown = own.s[3] * ex2((own.ref[3] - lse[3]) * kLog2e);
+      if (rank == 0) {
+        float ad = 0.f, bd = 0.f, td = 0.f;
+        if (dtok >= 0 && W > 0) {
+          const X1& o = sh->recv()[dtok / W < C ? dtok / W : 0];
+          ad = o.da;
+          bd = o.db;
+          td = o.dt;
+        }
+        store_row_stat(P, row32, lse, INT_MAX, INT_MAX, x.bad, dtok, ad, bd, td);
+      }
+    }
+  }
+  __syncthreads();
+
+  // ---- pass 2: divergence terms and inverse-CDF masses
+  const float A2 = sh->lse[0] * kLog2e, B2 = sh->lse[1] * kLog2e, S2 = sh->lse[3] * kLog2e;
+  const ResConst kc = res_const(P.beta, A2, B2, S2);
+  float jsum, msum;
+  if (draft) row_pass2<T, true>(sa, sb, st, v0, v1, R, kc, jsum, msum);
+  else row_pass2<T, false>(sa, sb, st, v0, v1, R, kc, jsum, msum);
+  const size_t slot = static_cast<size_t>(row32) * C + rank;
+  if (lane == 0) {
+    // the warp's block is group `warp` of this CTA's slice
+    P.group_mass[slot * P.group_stride + warp] = msum;
+    X2 x = x2_zero();
+    x.j = jsum;  // 2 JSD in bits (the decision kernel adds msum = 0)
+    if (draft) x.R = msum;
+    else x.Q = msum;
+    sh->w2[warp] = x;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    X2 x = (lane < NW) ? sh->w2[lane] : x2_zero();
+    warp_reduce_x2<G_JSD | G_RES>(x);
+    x.msum = 0.f;
+    if (draft) x.Q = sh->qown;
+    if (sh->broken) x.pad[0] = __uint_as_float(kBadTimeout);
+    float4* rec = reinterpret_cast<float4*>(P.pass2_rec + slot * 8);
+    if (lane == 0) rec[0] = make_float4(x.j, x.msum, x.kl, x.R);
+    if (lane == 1) rec[1] = make_float4(x.Q, x.pad[0], x.pad[1], x.pad[2]);
+  }
+
+  // a copy that timed out may still land: wait for it (bounded, always with
+  // the normal limit) before the CTA exits
+  if (lane == 0 && sh->broken) {
+    mbar_wait_bounded(&sh->bar[warp][0], 0u, kCopyTimeoutNs);
+    mbar_wait_bounded(&sh->bar[warp][1], 0u, kCopyTimeoutNs);
+  }
+}
+
+}  // namespace asymspec_impl

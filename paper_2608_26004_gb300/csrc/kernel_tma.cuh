@@ -336,12 +336,20 @@ __device__ __forceinline__ void vec_masses(const f2 (&xa)[NP], const f2 (&xb)[NP
                                            const f2 (&xt)[NP], f2 beta2, f2 L2, f2 nA2, f2 nS2,
                                            f2 (&p)[NP], f2 (&qf)[NP], f2 (&r)[NP],
                                            f2 (&la2)[NP]) {
+  // delta = a - b: the fused score in log2 units as t log2 e + (beta log2 e)(a - b),
+  // the form the production kernel (kernel_row.cuh) uses, so that a walk over
+  // either kernel's group masses sees identical vector masses
+  const f2 bL2 = mul2(beta2, L2);
 #pragma unroll
   for (int h = 0; h < NP; ++h) {
     la2[h] = fma2(xa[h], L2, nA2);  // log2 softmax(a), which the divergence terms reuse
     p[h] = ex2_2(la2[h]);
-    const f2 s = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
-    qf[h] = ex2_2(fma2(s, L2, nS2));
+    if constexpr (DS == ASYMSPEC_DELTA_AB) {
+      qf[h] = ex2_2(fma2(xt[h], L2, fma2(bL2, sub2(xa[h], xb[h]), nS2)));
+    } else {
+      const f2 s = fuse2<DS>(beta2, xa[h], xb[h], xt[h]);
+      qf[h] = ex2_2(fma2(s, L2, nS2));
+    }
     r[h] = relu2(sub2(qf[h], p[h]));
   }
 }
@@ -875,7 +883,9 @@ __device__ __forceinline__ void p2_groups(float g0, float g1, float* grp, int kr
 }
 
 // As p2_groups for four rounds kr .. kr + 3 (v0 .. v3) in one transposed
-// butterfly: lanes 0, 8, 16 and 24 end with the four group masses.
+// butterfly: lanes 0, 8, 16 and 24 end with the four group masses.  NW: warps
+// per CTA (group r NW + w is warp w's 32 vectors of round r).
+template <int NW = kTWarps>
 __device__ __forceinline__ void p2_groups4(float v0, float v1, float v2, float v3, float* grp,
                                            int kr, int rounds) {
   const int lane = static_cast<int>(threadIdx.x & 31), warp = static_cast<int>(threadIdx.x >> 5);
@@ -886,7 +896,7 @@ __device__ __forceinline__ void p2_groups4(float v0, float v1, float v2, float v
 #pragma unroll
   for (int off = 4; off > 0; off >>= 1) c += __shfl_xor_sync(0xffffffffu, c, off);
   const int r = kr + (lane >> 3);
-  if ((lane & 7) == 0 && r < rounds) grp[r * kTWarps + warp] = c;
+  if ((lane & 7) == 0 && r < rounds) grp[r * NW + warp] = c;
 }
 
 __device__ __forceinline__ void p2_finish(const P2Acc& acc, X2& x) {
@@ -1137,6 +1147,124 @@ __device__ __noinline__ int group_walk(const T* ga, const T* gb, const T* gt, in
     if (pick >= 0) found = lo + v * VE + pick;
   }
   return __shfl_sync(0xffffffffu, found, vc);
+}
+
+// The block of warp w in fuse_verify_row (kernel_row.cuh): vectors
+// [w bw, min(nv, (w + 1) bw)) of the slice, bw = ceil(nv / NW); the warp's
+// lane l takes vector w bw + 32 r + l in step r.
+__host__ __device__ __forceinline__ int row_block_vectors(int nv, int nw) {
+  return (nv + nw - 1) / nw;
+}
+
+// The inverse-CDF draw inside one slice whose groups are warp blocks (the
+// layout of fuse_verify_row): group g is vectors [g bw, min(nvec, (g+1) bw))
+// of the slice, its mass gm[g] (stored: pass 2's sums; else recomputed here,
+// the rare fallback to the fused masses of a draft row whose residual is
+// zero).  One warp: lane g takes group g (ngroups <= 32), the lane holding
+// the target walks its group 32 vectors per step (recomputed from global
+// memory exactly as pass 2 forms them), then the element inside the vector.
+// Same conventions as group_walk: the smallest index whose cumulative mass
+// exceeds tau, else the last index with positive mass; -1 when the slice
+// holds no mass.
+template <typename T, int DS = ASYMSPEC_DELTA_AB>
+__device__ __noinline__ int block_walk(const T* ga, const T* gb, const T* gt, int nvec, int lo,
+                                       int ngroups, int bw, float beta, const float* gm,
+                                       bool stored, bool use_r, float A2, float S2, float tau) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  constexpr int NP = VE / 2;
+  const int lane = threadIdx.x & 31;
+  const f2 beta2 = pk(beta, beta), L2 = pk(kLog2e, kLog2e);
+  const f2 nA2 = pk(-A2, -A2), nS2 = pk(-S2, -S2);
+  auto vmass = [&](int v) {
+    f2 p[NP], qf[NP], r[NP];
+    slice_vector_masses<T, DS>(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
+    return vsum(use_r ? r : qf);
+  };
+  // the group masses, one per lane
+  float gmass = 0.f;
+  if (stored) {
+    if (lane < ngroups) gmass = __ldcg(gm + lane);
+  } else {
+    for (int g = 0; g < ngroups; ++g) {
+      const int b0 = g * bw, b1 = min(nvec, b0 + bw);
+      float m = 0.f;
+      for (int v = b0 + lane; v < b1; v += 32) m += vmass(v);
+      m = warp_sum(m);
+      if (lane == g) gmass = m;
+    }
+  }
+  float incl = gmass;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float v = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += v;
+  }
+  const float excl = incl - gmass;
+  bool take_last = false;
+  const unsigned hit = __ballot_sync(0xffffffffu, gmass > 0.f && excl <= tau && tau < incl);
+  int gc;
+  if (hit) {
+    gc = __ffs(hit) - 1;
+  } else {
+    const unsigned pos = __ballot_sync(0xffffffffu, gmass > 0.f);
+    if (!pos) return -1;
+    gc = 31 - __clz(pos);
+    take_last = true;
+  }
+  const float trem = fmaxf(tau - __shfl_sync(0xffffffffu, excl, gc), 0.f);
+  // the vector, 32 at a time in index order
+  const int b0 = gc * bw, b1 = min(nvec, b0 + bw);
+  float run = 0.f;
+  int vsel = -1, vlast = -1;
+  float tin = 0.f;  // the target's offset inside the selected vector
+  for (int base = b0; base < b1 && vsel < 0; base += 32) {
+    const int v = base + lane;
+    const float mv = v < b1 ? vmass(v) : 0.f;
+    float vin = mv;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const float w = __shfl_up_sync(0xffffffffu, vin, off);
+      if (lane >= off) vin += w;
+    }
+    const float vex = vin - mv;
+    const unsigned pos = __ballot_sync(0xffffffffu, mv > 0.f);
+    if (pos) vlast = base + 31 - __clz(pos);
+    const unsigned vh = __ballot_sync(0xffffffffu, !take_last && mv > 0.f && run + vex <= trem &&
+                                                       trem < run + vin);
+    if (vh) {
+      const int vc = __ffs(vh) - 1;
+      vsel = base + vc;
+      tin = fmaxf(trem - run - __shfl_sync(0xffffffffu, vex, vc), 0.f);
+    }
+    run += __shfl_sync(0xffffffffu, vin, 31);
+  }
+  if (vsel < 0) {  // rounding left the target beyond the group: its last positive vector
+    if (vlast < 0) return -1;
+    vsel = vlast;
+    take_last = true;
+  }
+  // the element, on one lane
+  int found = -1;
+  if (lane == 0) {
+    f2 p[NP], qf[NP], r[NP];
+    slice_vector_masses<T, DS>(ga, gb, gt, vsel, beta2, L2, nA2, nS2, p, qf, r);
+    float cum = 0.f;
+    int pick = -1, last = -1;
+#pragma unroll
+    for (int h = 0; h < NP; ++h) {
+      float m0, m1;
+      upk(use_r ? r[h] : qf[h], m0, m1);
+      if (m0 > 0.f) last = 2 * h;
+      cum += m0;
+      if (!take_last && pick < 0 && cum > tin) pick = 2 * h;
+      if (m1 > 0.f) last = 2 * h + 1;
+      cum += m1;
+      if (!take_last && pick < 0 && cum > tin) pick = 2 * h + 1;
+    }
+    if (pick < 0) pick = last;
+    if (pick >= 0) found = lo + vsel * VE + pick;
+  }
+  return __shfl_sync(0xffffffffu, found, 0);
 }
 
 // ---------------------------------------------------------------- the kernel
@@ -1471,7 +1599,7 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
         const float tau_local = fmaxf(tau - (incl_o - mass_o), 0.f);
         const int lo_o = owner * P.W;
         const int nv_o = max(0, min(P.W, P.V - lo_o)) / VE;
-        const int ng_o = ((nv_o + kTThreads - 1) / kTThreads) * kTWarps;
+        const int ng_o = ((nv_o + P.tma_threads - 1) / P.tma_threads) * (P.tma_threads / 32);
         const size_t off = static_cast<size_t>(row) * P.V + lo_o;
         // the group masses are residual ones for draft rows and fused ones for
         // the bonus row; the other kind (a draft row whose residual is zero)
@@ -1483,7 +1611,12 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
         const float* gm = P.group_mass + (row * C + owner) * P.group_stride;
         const float A2 = st.lse[0] * kLog2e, S2 = st.lse[3] * kLog2e;
         const bool stored = r_ok == stored_r;
-        if (P.delta_src == ASYMSPEC_DELTA_A)
+        if (P.row_blocks) {
+          // fuse_verify_row: one group per warp block (delta = a - b)
+          const int nw = P.tma_threads / 32;
+          sample = block_walk<T>(ga, gb, gt, nv_o, lo_o, nw, row_block_vectors(nv_o, nw), P.beta,
+                                 gm, stored, r_ok, A2, S2, tau_local);
+        } else if (P.delta_src == ASYMSPEC_DELTA_A)
           sample = group_walk<T, true, ASYMSPEC_DELTA_A>(ga, gb, gt, nv_o, lo_o, ng_o, P.beta, gm,
                                                          stored, r_ok, A2, S2, tau_local);
         else if (P.delta_src == ASYMSPEC_DELTA_TB)

@@ -30,13 +30,16 @@ def device_inputs(batch, torch, device="cuda"):
 
 def run_gpu(batch, torch, *, mode, divergence=A.DIV_JSD, gamma=0.5, beta=1.0, lam=0.1,
             fuse_bonus=False, cluster_size=0, logprobs=True, inputs=None, kernel=0, full=True,
-            delta_source=A.DELTA_AB):
+            delta_source=A.DELTA_AB, tokens=True, block_threads=0):
     """One call of asymspec_fuse_verify_ex through the binding; numpy results.
 
     full=True asks for every debug output (row statistics, fused log-probs),
     which runs the full per-row program; full=False asks only for the row
-    tokens, which keeps the production program the benchmark times.
+    tokens (tokens=True) or for nothing but the accepted lengths and next
+    tokens (tokens=False: the production program the benchmark times).
     """
+    if full == "row":  # the production program's outputs only
+        full, tokens = False, False
     x = inputs if inputs is not None else device_inputs(batch, torch)
     elt = 4 if batch.dtype == synth.FP32 else 2
     if kernel == A.KERNEL_TMA and (batch.V * elt) % 16:
@@ -44,8 +47,9 @@ def run_gpu(batch, torch, *, mode, divergence=A.DIV_JSD, gamma=0.5, beta=1.0, la
     fv = A.FuseVerify(batch.B, batch.K)
     res = fv(x["a"], x["b"], x["t"], x["tokens"], x["probs"], x["unif"], gamma=gamma, beta=beta,
              lam=lam, mode=mode, divergence=divergence, fuse_bonus=fuse_bonus,
-             row_stats=full, row_tokens=True, fused_logprobs=full and logprobs,
-             cluster_size=cluster_size, kernel=kernel, delta_source=delta_source)
+             row_stats=full, row_tokens=full or tokens, fused_logprobs=full and logprobs,
+             cluster_size=cluster_size, kernel=kernel, delta_source=delta_source,
+             block_threads=block_threads)
     torch.cuda.synchronize()
     out = {k: v.cpu().numpy() for k, v in res.items()}
     out["workspace_after"] = fv.workspace.cpu().numpy()
@@ -168,8 +172,15 @@ def compare(batch, g, o, *, mode, select=None, logprobs=True, check_stats=True,
     nflag = check_decisions(batch, sel, L, N, o, mode)
     params = getattr(o, "params", dict(beta=1.0, fuse_bonus=False, delta_source=A.DELTA_AB))
     K1 = batch.K + 1
-    rt = g["row_tokens"][sel]
     good = ~err
+    if "row_tokens" not in g:  # the production program: accept_len / next_token only
+        ngood = int(good.sum())
+        frac = nflag / ngood if ngood else 0.0
+        if max_flagged is not None:
+            assert frac <= max_flagged, f"{nflag} of {ngood} elements flagged ({frac:.1%})"
+        return dict(compared=int(ok.sum()), flagged=nflag, flagged_frac=frac,
+                    errors=int(err.sum()), logprob_err=None, rows=int(len(sel) * K1))
+    rt = g["row_tokens"][sel]
     # fused argmax: compared wherever the GPU computed it (-1 = not needed by
     # the production program, only the greedy bonus row); draft rows always
     # have it.  Near-ties: a valid argmax within the band.

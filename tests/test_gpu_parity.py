@@ -1,10 +1,12 @@
 """GPU path (through the C ABI) against the float64 oracle on the same inputs.
 
-Every case runs on the kernel the library picks (the one-shot TMA kernel
-for 16-byte aligned rows, the generic kernel otherwise) and on the generic
-kernel; with the production program (accept/next plus row tokens, the work
-the benchmark times) and with every debug output (row statistics, fused
-log-probs), which runs the full per-row program.
+Every case runs on the kernel the library picks (for 16-byte aligned rows
+the one-shot cluster kernels, the generic kernel otherwise) and on the
+generic kernel: with accepted lengths and next tokens only (the production
+program the benchmark times: in stochastic mode with the JSD gate, the
+production row kernel), with the per-row tokens as well, and with every
+debug output (row statistics, fused log-probs), which runs the full per-row
+program.
 """
 import numpy as np
 import pytest
@@ -18,10 +20,10 @@ pytestmark = pytest.mark.gpu
 
 GREEDY, STOCH = A.MODE_GREEDY, A.MODE_STOCHASTIC
 AUTO, GENERIC, TMA = A.KERNEL_AUTO, A.KERNEL_GENERIC, A.KERNEL_TMA
-# the automatic choice (the one-shot TMA kernel for aligned rows) and the
-# generic cluster kernel
-PATHS = [(AUTO, False), (AUTO, True), (GENERIC, True)]
-PATH_IDS = ["auto-prod", "auto-full", "generic-full"]
+# the automatic choice (the one-shot cluster kernels for aligned rows) and
+# the generic cluster kernel; "row": outputs of the production program only
+PATHS = [(AUTO, "row"), (AUTO, False), (AUTO, True), (GENERIC, True)]
+PATH_IDS = ["auto-row", "auto-prod", "auto-full", "generic-full"]
 
 
 @pytest.fixture(scope="module")
@@ -412,3 +414,43 @@ def test_copy_wait_timeout_marks_every_row(torch, mode, full):
     assert list(res["next_token"].cpu().numpy()) == [-1] * batch.B
     assert int(res["error_word"].cpu().numpy()[0]) & A.DATA_TIMEOUT
     check(batch, torch, mode, TMA, full)
+
+
+# ---------------------------------------------------------------- the production row kernel
+
+@pytest.mark.parametrize("nt", [224, 256])
+@pytest.mark.parametrize("cluster", [1, 2, 4, 8, 12, 16])
+def test_row_kernel_shapes(torch, nt, cluster):
+    # the production kernel of the stochastic JSD step in every CTA shape and
+    # cluster size the planner may take: several rounds, a ragged last round,
+    # bf16 and fp32 rows, slices down to a single vector
+    for B, K, V, dtype, seed in ((3, 3, 40000, synth.BF16, 61), (2, 2, 12288, synth.FP32, 62),
+                                 (4, 1, 8200, synth.BF16, 63), (2, 2, 8 * cluster, synth.BF16, 64),
+                                 (2, 3, 128256, synth.BF16, 65)):
+        if dtype == synth.FP32 and nt != 256:
+            continue
+        batch = small(B, K, V, dtype, seed)
+        try:
+            g = run_gpu(batch, torch, mode=STOCH, full="row", cluster_size=cluster,
+                        block_threads=nt)
+        except A.AsymSpecError as e:
+            # a slice that does not fit on chip at this shape (more than 10
+            # vectors per thread, or too much shared memory for the CTAs per
+            # SM the shape stands for) is refused by the planner
+            assert e.status in (A.ERR_TOO_LARGE, A.ERR_UNSUPPORTED)
+            vecs = -(-V // cluster) * (4 if dtype == synth.FP32 else 2) // 16
+            slice_bytes = 3 * vecs * 16
+            assert vecs > 10 * nt or slice_bytes > 70 * 1024
+            continue
+        o = run_oracle(batch, mode=STOCH, logprobs=False)
+        compare(batch, g, o, mode=STOCH, logprobs=False)
+
+
+def test_row_kernel_is_the_production_choice(torch):
+    for B, K, V, dtype in ((64, 7, 128256, synth.BF16), (8, 5, 151936, synth.BF16),
+                           (256, 4, 151936, synth.FP32)):
+        info = A.plan(B, K, V, dtype, A.gate_params(mode=STOCH))
+        assert info.kernel == A.KERNEL_TMA
+        if dtype == synth.BF16:      # three CTAs of 224 threads per SM
+            assert info.block_threads == 224 and info.smem_bytes * 3 <= 225 * 1024
+        assert info.max_active_clusters > 0
