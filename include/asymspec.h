@@ -111,7 +111,9 @@ typedef struct {
 /* Optional launch overrides (host struct); zero fields mean "automatic". */
 typedef struct {
   int32_t cluster_size;   /* CTAs per row triple: 1 to 16 */
-  int32_t block_threads;  /* reserved, must be 0 (256 threads per CTA) */
+  int32_t block_threads;  /* 0 automatic; 192, 224 or 256: threads per CTA of the production
+                             row kernel of ASYMSPEC_KERNEL_TMA (the stochastic JSD step
+                             without debug outputs); every other program runs 256 */
   int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC or ASYMSPEC_KERNEL_TMA */
   int32_t test_flags;     /* 0, or test hooks (ASYMSPEC_TEST_*); other bits reserved, 0 */
   /* Optional cudaEvent_t handles (or NULL): recorded on the call's stream

@@ -48,6 +48,7 @@ struct Plan {
   bool vector_path;
   bool row;          // the production row kernel (fuse_verify_row) runs
   int nt, minb;      // its CTA shape: threads, CTAs per SM (kTThreads, 2 otherwise)
+  int grid_y;        // the row kernel's grid is (C (K+1), B): grid_y = B (1 otherwise)
 };
 
 // Shared memory one SM offers its CTAs, and what each CTA costs beyond its
@@ -124,13 +125,15 @@ bool plan_row(int V, int dtype, int forced_C, int forced_nt, Plan* pl) {
   struct Shape {
     int nt, minb;
   };
-  const Shape shapes_bf16[] = {{224, 3}, {256, 3}, {256, 2}};
+  // (192 threads, four to an SM: on request only)
+  const Shape shapes_bf16[] = {{224, 3}, {256, 3}, {256, 2}, {192, 4}};
   const Shape shapes_f32[] = {{256, 2}};
   const Shape* shapes = dtype == ASYMSPEC_FP32 ? shapes_f32 : shapes_bf16;
-  const int nshapes = dtype == ASYMSPEC_FP32 ? 1 : 3;
+  const int nshapes = dtype == ASYMSPEC_FP32 ? 1 : 4;
   for (int si = 0; si < nshapes; ++si) {
     const Shape sh = shapes[si];
     if (forced_nt && sh.nt != forced_nt) continue;
+    if (!forced_nt && sh.nt == 192) continue;
     if (!row_kernel(dtype, sh.nt, sh.minb)) continue;
     for (int C : kClusterOrder) {
       if (forced_C && C != forced_C) continue;
@@ -180,7 +183,8 @@ TmaLayout tma_layout(int B, int K, int C, int group_stride = kGroupsMax) {
   L.stat = off;
   off += round_up(R * sizeof(RowStat), 256);
   L.p2rec = off;
-  off += round_up(R * C * sizeof(X2), 256);
+  // one record per CTA (fuse_verify_tma) or per warp (fuse_verify_row)
+  off += round_up(R * C * kRowMaxWarps * sizeof(X2), 256);
   L.groups = off;
   off += round_up(R * C * static_cast<size_t>(group_stride) * sizeof(float), 256);
   L.total = off;
@@ -204,14 +208,17 @@ int make_plan(int B, int K, int V, int dtype, const asymspec_launch_opts* opts, 
   pl->row = false;
   pl->nt = kTThreads;
   pl->minb = 2;
+  pl->grid_y = 1;
   if (ws_bytes < cluster_ws_bytes(B, K)) return ASYMSPEC_ERR_WORKSPACE;
   bool ok = false;
-  if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && prod_row &&
+  // (its grid is (C (K+1), B): B up to 65535)
+  if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && prod_row && B <= 65535 &&
       plan_row(V, dtype, forced_C, forced_nt, pl)) {
     if (ws_bytes >= tma_layout(B, K, pl->C).total) {
       pl->kernel = ASYMSPEC_KERNEL_TMA;
       pl->VE = 16 / elt;
       pl->row = true;
+      pl->grid_y = B;
       ok = true;
     } else if (forced_kernel == ASYMSPEC_KERNEL_TMA) {
       return ASYMSPEC_ERR_WORKSPACE;
@@ -294,7 +301,9 @@ cudaLaunchConfig_t launch_config(const Plan& pl, long long ctas, cudaStream_t st
   attr[0].val.clusterDim.x = pl.C;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.gridDim = dim3(static_cast<unsigned>(ctas));
+  cfg.gridDim = pl.grid_y > 1 ? dim3(static_cast<unsigned>(ctas / pl.grid_y),
+                                     static_cast<unsigned>(pl.grid_y))
+                              : dim3(static_cast<unsigned>(ctas));
   cfg.blockDim = dim3(pl.kernel == ASYMSPEC_KERNEL_GENERIC ? kThreads : pl.nt);
   cfg.dynamicSmemBytes = pl.smem;
   cfg.stream = stream;
@@ -316,7 +325,9 @@ cudaError_t active_clusters(KernelFn fn, const Plan& pl, int device, int* out) {
       }
   }
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = launch_config(pl, pl.C, nullptr, attr);
+  Plan one = pl;  // a grid of one cluster
+  one.grid_y = 1;
+  cudaLaunchConfig_t cfg = launch_config(one, pl.C, nullptr, attr);
   int n = 0;
   const cudaError_t e = cudaOccupancyMaxActiveClusters(&n, fn, &cfg);
   if (e != cudaSuccess) return e;
@@ -346,8 +357,8 @@ int check_params(const asymspec_gate_params* gp) {
 }
 
 int check_opts(const asymspec_launch_opts* opts) {
-  if (opts && opts->block_threads != 0 && opts->block_threads != 224 &&
-      opts->block_threads != 256)
+  if (opts && opts->block_threads != 0 && opts->block_threads != 192 &&
+      opts->block_threads != 224 && opts->block_threads != 256)
     return ASYMSPEC_ERR_INVALID_ARG;
   if (opts && (opts->test_flags & ~ASYMSPEC_TEST_COPY_GIVE_UP) != 0) return ASYMSPEC_ERR_INVALID_ARG;
   if (opts && ((opts->timing_begin == nullptr) != (opts->timing_end == nullptr)))

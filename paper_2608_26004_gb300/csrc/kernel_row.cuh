@@ -116,7 +116,6 @@ __device__ __forceinline__ f2 jsd_pair(f2 amb, f2 p, const ResConst& k, f2 jacc)
 
 // ---------------------------------------------------------------- layout
 
-constexpr int kRowMaxWarps = 8;
 constexpr int kRowChunks = 2;  // bulk-copy chunks per warp block
 
 // A warp's pass-1 record: the references (nats) and sums of
@@ -342,6 +341,24 @@ __device__ __forceinline__ void row_pass2(const T* ra, const T* rb, const T* rt,
 
 // ---------------------------------------------------------------- the kernel
 
+// The cluster's index in the grid: (row k of batch element bi) = (x, y).
+__device__ __forceinline__ unsigned cluster_id_x() {
+  unsigned r;
+  asm("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ unsigned cluster_id_y() {
+  unsigned r;
+  asm("mov.u32 %0, %%clusterid.y;" : "=r"(r));
+  return r;
+}
+
+// Grid: (C (K+1), B) CTAs in clusters of (C, 1, 1); cluster (k, bi) takes
+// row k of batch element bi.  What it leaves for the decision kernel: rank
+// 0's row statistics (the normalisers, data-error bits) and one pass-2 record
+// per warp of every CTA (KParams::pass2_rec, kRowMaxWarps records per CTA):
+// the warp's JSD sum, the residual and fused masses of its block (its
+// inverse-CDF group) and the timeout flag.
 template <typename T, int NT, int MINB>
 __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
   static_assert(NT % 32 == 0 && NT / 32 <= kRowMaxWarps, "at most kRowMaxWarps warps");
@@ -354,8 +371,10 @@ __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
   const int tid = static_cast<int>(threadIdx.x);
   const int lane = tid & 31, warp = tid >> 5;
   const int C = P.C;
-  const unsigned row32 = blockIdx.x / static_cast<unsigned>(C);
-  const unsigned K1 = static_cast<unsigned>(P.K) + 1u;
+  const int k = static_cast<int>(cluster_id_x());
+  const int bi = static_cast<int>(cluster_id_y());
+  const unsigned row32 = static_cast<unsigned>(bi) * static_cast<unsigned>(P.K + 1) +
+                         static_cast<unsigned>(k);
   const int W = P.W;
   const int lo = rank * W;
   const int n = max(0, min(W, P.V - lo));
@@ -368,8 +387,6 @@ __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
   T* sb = sa + W;
   T* st = sb + W;
   RowShared* sh = reinterpret_cast<RowShared*>(smem_row + P.sh_off);
-  const int bi = static_cast<int>(row32 / K1);
-  const int k = static_cast<int>(row32 - static_cast<unsigned>(bi) * K1);
   const bool draft = k < P.K;
 
   // each warp brings in its own block: no CTA barrier before the copies
@@ -384,9 +401,6 @@ __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
     sh->broken = 0;
     sh->wait_ns = P.copy_wait_ns;
   }
-  // warp 0 keeps the row's draft token, loaded while the slice is in flight
-  int dtok = -1;
-  if (warp == 0 && draft) dtok = P.tokens[static_cast<size_t>(bi) * P.K + k];
   __syncthreads();  // every warp's barriers and the shared flags are initialised
 
   // ---- pass 1: the row normalisers, combined over the cluster
@@ -419,39 +433,24 @@ __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
     if (draft) warp_reduce_x1<FD>(x);
     else warp_reduce_x1<F_LS>(x);
     x.bad = sh->broken;
-    if (dtok >= lo && dtok < lo + n) {  // this CTA's slice holds the draft token
-      x.da = to_f32(sa[dtok - lo]);
-      x.db = to_f32(sb[dtok - lo]);
-      x.dt = to_f32(st[dtok - lo]);
-    }
     push_record(x, sh->recv(), rank, C, cluster);
   }
   cluster_barrier(warp == 0);  // every CTA's pass-1 record is in every CTA
 
   if (warp == 0) {
-    float lse[4];
     X1 x = (lane < C) ? sh->recv()[lane] : x1_neutral();
     if (draft) warp_reduce_x1<FD>(x);
     else warp_reduce_x1<F_LS>(x);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) lse[q] = x.ref[q] + logf(x.s[q]);
     if (lane == 0) {
+      float lse[4];
+      lse[0] = draft ? x.ref[0] + logf(x.s[0]) : NAN;
+      lse[1] = draft ? x.ref[1] + logf(x.s[1]) : NAN;
+      lse[2] = NAN;
+      lse[3] = x.ref[3] + logf(x.s[3]);
 #pragma unroll
       for (int q = 0; q < 4; ++q) sh->lse[q] = lse[q];
-      // this slice's fused mass, from its own pass-1 record (the draw falls
-      // back to the fused masses when the row's whole residual is zero)
-      const X1& own = sh->recv()[rank];
-      sh->qown = own.s[3] * ex2((own.ref[3] - lse[3]) * kLog2e);
-      if (rank == 0) {
-        float ad = 0.f, bd = 0.f, td = 0.f;
-        if (dtok >= 0 && W > 0) {
-          const X1& o = sh->recv()[dtok / W < C ? dtok / W : 0];
-          ad = o.da;
-          bd = o.db;
-          td = o.dt;
-        }
-        store_row_stat(P, row32, lse, INT_MAX, INT_MAX, x.bad, dtok, ad, bd, td);
-      }
+      // the draft token's logits are read by the decision kernel itself
+      if (rank == 0) store_row_stat(P, row32, lse, INT_MAX, INT_MAX, x.bad, -1, 0.f, 0.f, 0.f);
     }
   }
   __syncthreads();
@@ -462,31 +461,21 @@ __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
   float jsum, msum;
   if (draft) row_pass2<T, true>(sa, sb, st, v0, v1, R, kc, jsum, msum);
   else row_pass2<T, false>(sa, sb, st, v0, v1, R, kc, jsum, msum);
-  const size_t slot = static_cast<size_t>(row32) * C + rank;
+  const bool broken = sh->broken != 0;
   if (lane == 0) {
-    // the warp's block is group `warp` of this CTA's slice
-    P.group_mass[slot * P.group_stride + warp] = msum;
-    X2 x = x2_zero();
-    x.j = jsum;  // 2 JSD in bits (the decision kernel adds msum = 0)
-    if (draft) x.R = msum;
-    else x.Q = msum;
-    sh->w2[warp] = x;
-  }
-  __syncthreads();
-  if (warp == 0) {
-    X2 x = (lane < NW) ? sh->w2[lane] : x2_zero();
-    warp_reduce_x2<G_JSD | G_RES>(x);
-    x.msum = 0.f;
-    if (draft) x.Q = sh->qown;
-    if (sh->broken) x.pad[0] = __uint_as_float(kBadTimeout);
-    float4* rec = reinterpret_cast<float4*>(P.pass2_rec + slot * 8);
-    if (lane == 0) rec[0] = make_float4(x.j, x.msum, x.kl, x.R);
-    if (lane == 1) rec[1] = make_float4(x.Q, x.pad[0], x.pad[1], x.pad[2]);
+    // this warp's record: its block is one inverse-CDF group of the row.  A
+    // draft row's fused mass (the draw's fallback when the row's whole
+    // residual is zero) comes from the warp's pass-1 sum.
+    const float qf = draft ? e.s[2] * ex2(e.ref[2] * kLog2e - S2) : msum;
+    float4* rec = reinterpret_cast<float4*>(
+        P.pass2_rec + ((static_cast<size_t>(row32) * C + rank) * kRowMaxWarps + warp) * 8);
+    rec[0] = make_float4(jsum, 0.f, 0.f, draft ? msum : 0.f);
+    rec[1] = make_float4(qf, broken ? __uint_as_float(kBadTimeout) : 0.f, 0.f, 0.f);
   }
 
   // a copy that timed out may still land: wait for it (bounded, always with
   // the normal limit) before the CTA exits
-  if (lane == 0 && sh->broken) {
+  if (lane == 0 && broken) {
     mbar_wait_bounded(&sh->bar[warp][0], 0u, kCopyTimeoutNs);
     mbar_wait_bounded(&sh->bar[warp][1], 0u, kCopyTimeoutNs);
   }

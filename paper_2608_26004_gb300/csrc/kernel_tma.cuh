@@ -1156,70 +1156,43 @@ __host__ __device__ __forceinline__ int row_block_vectors(int nv, int nw) {
   return (nv + nw - 1) / nw;
 }
 
-// The inverse-CDF draw inside one slice whose groups are warp blocks (the
-// layout of fuse_verify_row): group g is vectors [g bw, min(nvec, (g+1) bw))
-// of the slice, its mass gm[g] (stored: pass 2's sums; else recomputed here,
-// the rare fallback to the fused masses of a draft row whose residual is
-// zero).  One warp: lane g takes group g (ngroups <= 32), the lane holding
-// the target walks its group 32 vectors per step (recomputed from global
-// memory exactly as pass 2 forms them), then the element inside the vector.
-// Same conventions as group_walk: the smallest index whose cumulative mass
-// exceeds tau, else the last index with positive mass; -1 when the slice
-// holds no mass.
-template <typename T, int DS = ASYMSPEC_DELTA_AB>
-__device__ __noinline__ int block_walk(const T* ga, const T* gb, const T* gt, int nvec, int lo,
-                                       int ngroups, int bw, float beta, const float* gm,
-                                       bool stored, bool use_r, float A2, float S2, float tau) {
+// The inverse-CDF draw inside vectors [b0, b1) of a slice (one group of
+// fuse_verify_row: a warp's block), by one warp: the smallest index whose
+// cumulative residual (use_r) or fused mass exceeds trem, or with take_last
+// (rounding left the target at or beyond the group's mass) the last index
+// with positive mass.  Every vector mass of the group is loaded first
+// (independent loads, one round trip), then scanned 32 vectors at a time in
+// index order; the masses are formed exactly as the row kernel's pass 2
+// forms them.  Returns the index within the row, or -1 if the group holds
+// no mass.
+template <typename T>
+__device__ __noinline__ int walk_vectors(const T* ga, const T* gb, const T* gt, int b0, int b1,
+                                         int lo, float beta, bool use_r, float A2, float S2,
+                                         float trem, bool take_last) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
   const int lane = threadIdx.x & 31;
   const f2 beta2 = pk(beta, beta), L2 = pk(kLog2e, kLog2e);
   const f2 nA2 = pk(-A2, -A2), nS2 = pk(-S2, -S2);
-  auto vmass = [&](int v) {
-    f2 p[NP], qf[NP], r[NP];
-    slice_vector_masses<T, DS>(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
-    return vsum(use_r ? r : qf);
-  };
-  // the group masses, one per lane
-  float gmass = 0.f;
-  if (stored) {
-    if (lane < ngroups) gmass = __ldcg(gm + lane);
-  } else {
-    for (int g = 0; g < ngroups; ++g) {
-      const int b0 = g * bw, b1 = min(nvec, b0 + bw);
-      float m = 0.f;
-      for (int v = b0 + lane; v < b1; v += 32) m += vmass(v);
-      m = warp_sum(m);
-      if (lane == g) gmass = m;
+  float mvs[kMaxRounds];
+#pragma unroll
+  for (int s = 0; s < kMaxRounds; ++s) {
+    const int v = b0 + 32 * s + lane;
+    mvs[s] = 0.f;
+    if (v < b1) {
+      f2 p[NP], qf[NP], r[NP];
+      slice_vector_masses<T>(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
+      mvs[s] = vsum(use_r ? r : qf);
     }
   }
-  float incl = gmass;
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const float v = __shfl_up_sync(0xffffffffu, incl, off);
-    if (lane >= off) incl += v;
-  }
-  const float excl = incl - gmass;
-  bool take_last = false;
-  const unsigned hit = __ballot_sync(0xffffffffu, gmass > 0.f && excl <= tau && tau < incl);
-  int gc;
-  if (hit) {
-    gc = __ffs(hit) - 1;
-  } else {
-    const unsigned pos = __ballot_sync(0xffffffffu, gmass > 0.f);
-    if (!pos) return -1;
-    gc = 31 - __clz(pos);
-    take_last = true;
-  }
-  const float trem = fmaxf(tau - __shfl_sync(0xffffffffu, excl, gc), 0.f);
-  // the vector, 32 at a time in index order
-  const int b0 = gc * bw, b1 = min(nvec, b0 + bw);
   float run = 0.f;
   int vsel = -1, vlast = -1;
   float tin = 0.f;  // the target's offset inside the selected vector
-  for (int base = b0; base < b1 && vsel < 0; base += 32) {
-    const int v = base + lane;
-    const float mv = v < b1 ? vmass(v) : 0.f;
+#pragma unroll
+  for (int s = 0; s < kMaxRounds; ++s) {
+    const int base = b0 + 32 * s;
+    if (base >= b1 || vsel >= 0) break;
+    const float mv = mvs[s];
     float vin = mv;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
@@ -1243,11 +1216,10 @@ __device__ __noinline__ int block_walk(const T* ga, const T* gb, const T* gt, in
     vsel = vlast;
     take_last = true;
   }
-  // the element, on one lane
   int found = -1;
   if (lane == 0) {
     f2 p[NP], qf[NP], r[NP];
-    slice_vector_masses<T, DS>(ga, gb, gt, vsel, beta2, L2, nA2, nS2, p, qf, r);
+    slice_vector_masses<T>(ga, gb, gt, vsel, beta2, L2, nA2, nS2, p, qf, r);
     float cum = 0.f;
     int pick = -1, last = -1;
 #pragma unroll
@@ -1533,6 +1505,144 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
 
 constexpr int kDecideThreads = 256;  // at most 8 warps; each takes rows k, k + 8, ...
 
+// ---- rows of fuse_verify_row (kernel_row.cuh): one pass-2 record per warp
+// block, each block one inverse-CDF group
+
+constexpr int kRowMaxWarps = 8;  // warps per CTA of fuse_verify_row; records per CTA
+
+// What the decision of row (bi, k) needs from the kernel's inputs (not from
+// the row kernel): the draft token, its three logits, the row's scalars.
+// Loaded before griddepcontrol.wait, so that the loads overlap the row
+// kernel's last CTAs.
+struct RowInputs {
+  int dtok;
+  float ad, bd, td;
+  RowScalars sc;
+};
+
+template <typename T>
+__device__ __forceinline__ RowInputs load_row_inputs(const KParams& P, int bi, int k) {
+  RowInputs d;
+  d.dtok = -1;
+  d.ad = d.bd = d.td = 0.f;
+  d.sc = load_row_scalars(P, bi, k);
+  if (k < P.K) {
+    d.dtok = P.tokens[static_cast<size_t>(bi) * P.K + k];
+    if (d.dtok >= 0 && d.dtok < P.V) {
+      const size_t o = (static_cast<size_t>(bi) * (P.K + 1) + k) * P.V + d.dtok;
+      d.ad = to_f32(static_cast<const T*>(P.a)[o]);
+      d.bd = to_f32(static_cast<const T*>(P.b)[o]);
+      d.td = to_f32(static_cast<const T*>(P.t)[o]);
+    }
+  }
+  return d;
+}
+
+// The row's results from its C x NW warp records (one warp): the divergence
+// of Eq. 3 and the inverse-CDF draw at u_K (the residual's groups, or the
+// fused masses when the whole residual is zero and on the bonus row).  Lane
+// l takes groups 4l .. 4l + 3 (group g = warp g % NW of rank g / NW, in index
+// order), the lane holding the target picks the group, walk_vectors the
+// element.
+template <typename T>
+__device__ __forceinline__ RowResult block_row_result(const KParams& P, int k, long long row,
+                                                      const RowScalars& sc) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  const int lane = threadIdx.x & 31;
+  const int C = P.C, NW = P.tma_threads / 32, ng = C * NW;
+  const bool bonus = (k == P.K);
+  const RowStat st = static_cast<const RowStat*>(P.row_stat)[row];
+  float j = 0.f, Rm[4], Qm[4];
+  bool late = false;
+#pragma unroll
+  for (int h = 0; h < 4; ++h) {
+    const int g = 4 * lane + h;
+    Rm[h] = Qm[h] = 0.f;
+    if (g < ng) {
+      const int r = g / NW, w = g - r * NW;
+      const float4* rec = reinterpret_cast<const float4*>(
+          P.pass2_rec + ((static_cast<size_t>(row) * C + r) * kRowMaxWarps + w) * 8);
+      const float4 x0 = __ldcg(rec), x1 = __ldcg(rec + 1);
+      j += x0.x;
+      Rm[h] = x0.w;
+      Qm[h] = x1.x;
+      late = late || __float_as_uint(x1.y) != 0u;
+    }
+  }
+  RowResult rr;
+  rr.lse_a = bonus ? NAN : st.lse[0];
+  rr.lse_b = bonus ? NAN : st.lse[1];
+  rr.lse_t = NAN;
+  rr.lse_s = st.lse[3];
+  rr.D = bonus ? 0.f : 0.5f * kLn2 * warp_sum(j);  // j sums 2 JSD in bits
+  rr.is = rr.it = INT_MAX;
+  rr.bad = st.bad | (__any_sync(0xffffffffu, late) ? kBadTimeout : 0u);
+  rr.have_lse_t = false;
+  const float Rl = (Rm[0] + Rm[1]) + (Rm[2] + Rm[3]), Ql = (Qm[0] + Qm[1]) + (Qm[2] + Qm[3]);
+  const float R_all = warp_sum(Rl), Q_all = warp_sum(Ql);
+  const bool r_ok = !bonus && R_all > 0.f;
+  const float ml = r_ok ? Rl : Ql, total = r_ok ? R_all : Q_all;
+  rr.mass = total;
+  const float tau = sc.u_last * total;
+  float incl = ml;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const float v = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += v;
+  }
+  const float excl = incl - ml;
+  bool take_last = false;
+  const unsigned hit = __ballot_sync(0xffffffffu, ml > 0.f && excl <= tau && tau < incl);
+  int lc;
+  if (hit) {
+    lc = __ffs(hit) - 1;
+  } else {
+    const unsigned pos = __ballot_sync(0xffffffffu, ml > 0.f);
+    if (!pos) {
+      rr.sample = -1;
+      return rr;
+    }
+    lc = 31 - __clz(pos);
+    take_last = true;
+  }
+  // the group, inside lane lc's four
+  int gsel = -1, glast = -1;
+  float trem = 0.f;
+  if (lane == lc) {
+    float cum = excl;
+#pragma unroll
+    for (int h = 0; h < 4; ++h) {
+      const float m = r_ok ? Rm[h] : Qm[h];
+      if (m > 0.f) glast = 4 * lane + h;
+      if (!take_last && gsel < 0) {
+        if (m > 0.f && cum + m > tau) {
+          gsel = 4 * lane + h;
+          trem = fmaxf(tau - cum, 0.f);
+        } else {
+          cum += m;
+        }
+      }
+    }
+    if (gsel < 0) {
+      gsel = glast;
+      take_last = true;
+    }
+  }
+  gsel = __shfl_sync(0xffffffffu, gsel, lc);
+  trem = __shfl_sync(0xffffffffu, trem, lc);
+  take_last = __shfl_sync(0xffffffffu, take_last ? 1 : 0, lc) != 0;
+  const int r = gsel / NW, w = gsel - r * NW;
+  const int lo_r = r * P.W;
+  const int nv_r = max(0, min(P.W, P.V - lo_r)) / VE;
+  const int bw = row_block_vectors(nv_r, NW);
+  const int b0 = min(nv_r, w * bw), b1 = min(nv_r, b0 + bw);
+  const size_t off = static_cast<size_t>(row) * P.V + lo_r;
+  rr.sample = walk_vectors<T>(static_cast<const T*>(P.a) + off, static_cast<const T*>(P.b) + off,
+                              static_cast<const T*>(P.t) + off, b0, b1, lo_r, P.beta, r_ok,
+                              st.lse[0] * kLog2e, st.lse[3] * kLog2e, trem, take_last);
+  return rr;
+}
+
 // The decisions of one batch element's K+1 rows (one CTA per element, one
 // warp per row) from what fuse_verify_tma left in the workspace, then
 // Algorithm 1's scan over them in shared memory.  Per row: the divergence
@@ -1543,16 +1653,28 @@ constexpr int kDecideThreads = 256;  // at most 8 warps; each takes rows k, k + 
 template <typename T, bool STOCH>
 __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
-  // launched as a programmatic dependent of the row kernel: its CTAs may
-  // start early; nothing of the workspace is read before that kernel is done
-  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int bi = blockIdx.x;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
   const int K = P.K, K1 = K + 1, C = P.C;
   const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
   const bool klg = P.divergence == ASYMSPEC_DIV_KL;
+  // the kernel inputs of this warp's first row, loaded before the wait
+  RowInputs pre{-1, 0.f, 0.f, 0.f, RowScalars{0.f, 0.f, 0.f}};
+  if (STOCH && P.row_blocks && warp < K1) pre = load_row_inputs<T>(P, bi, warp);
+  // launched as a programmatic dependent of the row kernel: its CTAs may
+  // start early; nothing of the workspace is read before that kernel is done
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   for (int k = warp; k < K1; k += nw) {
     const long long row = static_cast<long long>(bi) * K1 + k;
+    if constexpr (STOCH) {
+      if (P.row_blocks) {  // a row of fuse_verify_row
+        const RowInputs din = (k == warp) ? pre : load_row_inputs<T>(P, bi, k);
+        const RowResult rr = block_row_result<T>(P, k, row, din.sc);
+        if (lane == 0)
+          P.recs[row] = row_record<true>(P, row, k, rr, din.dtok, din.ad, din.bd, din.td, din.sc);
+        continue;
+      }
+    }
     const bool bonus = (k == K);
     const bool pass2 = STOCH || P.full || (!bonus && (jsd || klg));
     RowStat st = static_cast<const RowStat*>(P.row_stat)[row];
@@ -1611,12 +1733,7 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
         const float* gm = P.group_mass + (row * C + owner) * P.group_stride;
         const float A2 = st.lse[0] * kLog2e, S2 = st.lse[3] * kLog2e;
         const bool stored = r_ok == stored_r;
-        if (P.row_blocks) {
-          // fuse_verify_row: one group per warp block (delta = a - b)
-          const int nw = P.tma_threads / 32;
-          sample = block_walk<T>(ga, gb, gt, nv_o, lo_o, nw, row_block_vectors(nv_o, nw), P.beta,
-                                 gm, stored, r_ok, A2, S2, tau_local);
-        } else if (P.delta_src == ASYMSPEC_DELTA_A)
+        if (P.delta_src == ASYMSPEC_DELTA_A)
           sample = group_walk<T, true, ASYMSPEC_DELTA_A>(ga, gb, gt, nv_o, lo_o, ng_o, P.beta, gm,
                                                          stored, r_ok, A2, S2, tau_local);
         else if (P.delta_src == ASYMSPEC_DELTA_TB)

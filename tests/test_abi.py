@@ -57,11 +57,11 @@ def _up(n):
 
 
 def tma_bytes(B, K, C):
-    """Records and tickets, then the TMA kernel's per-row results: a 48-byte
-    row record of pass 1, and per CTA a 32-byte pass-2 record and 80 group
-    masses."""
+    """Records and tickets, then the cluster kernels' per-row results: a
+    48-byte row record of pass 1, and per CTA room for eight 32-byte pass-2
+    records (one per warp of the production row kernel) and 80 group masses."""
     R = B * (K + 1)
-    return _up(R * 16) + _up(B * 4) + _up(R * 48) + _up(R * C * 32) + _up(R * C * 80 * 4)
+    return _up(R * 16) + _up(B * 4) + _up(R * 48) + _up(R * C * 8 * 32) + _up(R * C * 80 * 4)
 
 
 def test_workspace_size():

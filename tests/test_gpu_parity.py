@@ -132,7 +132,15 @@ def test_large_workloads_sampled(torch, cfg, mode):
     check_decisions(batch, sel, L[sel], N[sel], o, mode)
     for full in (False, True):
         g = run_gpu(batch, torch, mode=mode, inputs=x, full=full)
-        assert np.array_equal(g["accept_len"], L) and np.array_equal(g["next_token"], N)
+        # the production kernel and the full-program kernel sum in different
+        # orders: they may differ only on elements where both are correct
+        # emissions, checked against the oracle (near-ties of a few 1e-7)
+        diff = np.nonzero((g["accept_len"] != L) | (g["next_token"] != N))[0]
+        assert diff.size <= 2, f"{diff.size} elements differ between the kernels"
+        if diff.size:
+            od = run_oracle(batch, mode=mode, select=diff, logprobs=False)
+            check_decisions(batch, diff, L[diff], N[diff], od, mode)
+            check_decisions(batch, diff, g["accept_len"][diff], g["next_token"][diff], od, mode)
         compare(batch, g, o, mode=mode, select=sel)
 
 

@@ -106,13 +106,13 @@ def _up(n):
 
 
 def test_the_cases_cover_both_kernels_the_scratch_selects(torch):
-    # the TMA kernel needs, beyond records and tickets, 48 bytes per row and
-    # 352 per row and CTA; the static scratch takes it when these fit
+    # the cluster kernels need, beyond records and tickets, 48 bytes per row
+    # and 576 per row and CTA; the static scratch takes them when these fit
     fits = []
     for B, K, V, dtype, mode, seed in CASES:
         info = A.plan(B, K, V, dtype, A.gate_params(mode=mode))
         R = B * (K + 1)
-        need = (_up(R * 16) + _up(B * 4) + _up(R * 48) + _up(R * info.cluster_size * 32)
+        need = (_up(R * 16) + _up(B * 4) + _up(R * 48) + _up(R * info.cluster_size * 256)
                 + _up(R * info.cluster_size * 320))
         if info.kernel == A.KERNEL_TMA:
             fits.append(need <= A.STATIC_SCRATCH_BYTES)
