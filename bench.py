@@ -3,8 +3,8 @@
 One step = one pass of the whole path over one batch: the C-ABI call
 asymspec_fuse_verify_ex in stochastic mode (row normalisers, delta fusion,
 JSD gate, acceptance tests, residual inverse-CDF draws and the per-element
-accept scan), which is two kernel launches: the fused row kernel and the
-decision kernel.  The workload is B=64, K=7, V=128256 bf16 logits with the
+accept scan): two launches, the production row kernel and the decision
+kernel.  The workload is B=64, K=7, V=128256 bf16 logits with the
 Zipf-profile recipe (512 verify rows, 394 MB of logits per step, larger than
 the 129 MB L2; four resident input sets are rotated).
 
@@ -37,12 +37,12 @@ WORKLOAD_CFG = 2
 FALLBACK_HBM_GBS = 6800.0
 CSRC = os.path.join(ROOT, "paper_2608_26004_gb300", "csrc")
 KERNEL_SRCS = ("asymspec.cu", "device_common.cuh", "kernel_generic.cuh", "kernel_tma.cuh",
-               "kernels.h", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu",
+               "kernel_row.cuh", "kernels.h", "k_generic.cu", "k_tma_bf16.cu", "k_tma_f32.cu",
                "k_tma_bf16_prod.cu", "k_tma_f32_prod.cu", "k_tma_bf16_any_s.cu",
-               "k_tma_f32_any_s.cu")
+               "k_tma_f32_any_s.cu", "k_row_bf16.cu", "k_row_f32.cu")
 N_SETS = 4          # resident input sets rotated between steps (4 x 394 MB, each > L2)
 DIST_MIN_S = 1.0    # the per-step distribution loop runs at least this long
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fuse_verify_tma_B64_K7_V128256_bf16_traffic.txt")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fuse_verify_B64_K7_V128256_bf16_traffic.txt")
 REASON_BITS = {
     0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
     0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
@@ -80,6 +80,13 @@ def peaks():
         return float(d["hbm_gbs"]), "measured"
     except Exception:
         return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_name(A, info) -> str:
+    """The row kernel a call launches (the roofline's kernel)."""
+    if info.kernel == A.KERNEL_TMA:
+        return "fuse_verify_row" if info.row_kernel else "fuse_verify_tma"
+    return "fuse_verify_generic" if info.kernel == A.KERNEL_GENERIC else str(info.kernel)
 
 
 def kernel_hash() -> str:
@@ -571,10 +578,10 @@ def main():
     clocks = clk.summary()
     ms_step = ms / args.steps
     value = aggregate_rows_per_s(world, rows, ms_step)
-    # a step is the fused row kernel and its decision kernel; the roofline is
-    # the fused row kernel's own: its mean duration between the events the
-    # library recorded around it in every step of the distribution loop
-    launches_per_step = 2 if info.kernel == A.KERNEL_TMA else 1
+    # the roofline is the fused row kernel's own: its mean duration between
+    # the events the library recorded around it in every step of the
+    # distribution loop (the decision kernel that follows it is not included)
+    launches_per_step = info.launches
     kernel_ms = float(np.mean(kern_us)) * 1e-3
     launch_s = kernel_ms * 1e-3
     hbm_peak, peak_kind = peaks()
@@ -658,7 +665,7 @@ def main():
                      "frac": achieved / hbm_peak, "peak_kind": peak_kind,
                      "traffic": measured_traffic(args.mode),
                      "algorithmic_bytes_per_launch": alg_bytes,
-                     "kernel": "fuse_verify_tma" if info.kernel == A.KERNEL_TMA else str(info.kernel),
+                     "kernel": kernel_name(A, info),
                      "launch_us": kernel_ms * 1e3,
                      "launch_us_pct": percentiles(kern_us),
                      "timing": "CUDA events the library records around the fused row kernel "

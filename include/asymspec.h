@@ -149,6 +149,11 @@ typedef struct {
   int32_t vector_path;     /* 1 if rows qualify for 16-byte copies (V * element size % 16 == 0) */
   int32_t max_active_clusters; /* clusters the device can hold at once (0 if unknown) */
   int32_t kernel;          /* ASYMSPEC_KERNEL_GENERIC or ASYMSPEC_KERNEL_TMA */
+  int32_t launches;        /* kernel launches of one call: 1 (the generic kernel) or 2
+                              (a cluster row kernel and its decision kernel) */
+  int32_t row_kernel;      /* 1 if ASYMSPEC_KERNEL_TMA runs its production row kernel
+                              (fuse_verify_row: the stochastic JSD step without debug
+                              outputs), 0 otherwise */
 } asymspec_launch_info;
 
 /* Fills *p with the paper's defaults: gamma 0.5, beta 1.0, lambda 0.1,

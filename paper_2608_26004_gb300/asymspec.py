@@ -95,7 +95,8 @@ class LaunchInfo(ctypes.Structure):
     _fields_ = [("cluster_size", ctypes.c_int32), ("block_threads", ctypes.c_int32),
                 ("slice_elems", ctypes.c_int32), ("smem_bytes", ctypes.c_int32),
                 ("ctas", ctypes.c_int64), ("vector_path", ctypes.c_int32),
-                ("max_active_clusters", ctypes.c_int32), ("kernel", ctypes.c_int32)]
+                ("max_active_clusters", ctypes.c_int32), ("kernel", ctypes.c_int32),
+                ("launches", ctypes.c_int32), ("row_kernel", ctypes.c_int32)]
 
 
 class AsymSpecError(RuntimeError):

@@ -521,6 +521,8 @@ int asymspec_plan(int B, int K, int V, int dtype, const asymspec_gate_params* ga
   out->vector_path = vec_ok ? 1 : 0;
   out->max_active_clusters = 0;
   out->kernel = pl.kernel;
+  out->launches = pl.kernel == ASYMSPEC_KERNEL_TMA ? 2 : 1;
+  out->row_kernel = pl.row ? 1 : 0;
   int device = 0;
   if (cudaGetDevice(&device) == cudaSuccess) {
     const bool st_mode = gp.mode == ASYMSPEC_MODE_STOCHASTIC;

@@ -1551,7 +1551,15 @@ __device__ __forceinline__ RowResult block_row_result(const KParams& P, int k, l
   const int lane = threadIdx.x & 31;
   const int C = P.C, NW = P.tma_threads / 32, ng = C * NW;
   const bool bonus = (k == P.K);
-  const RowStat st = static_cast<const RowStat*>(P.row_stat)[row];
+  // (read from L2: another CTA wrote it during this launch)
+  RowStat st;
+  {
+    const float4* src = reinterpret_cast<const float4*>(static_cast<const RowStat*>(P.row_stat) + row);
+    float4* dst = reinterpret_cast<float4*>(&st);
+    dst[0] = __ldcg(src);
+    dst[1] = __ldcg(src + 1);
+    dst[2] = __ldcg(src + 2);
+  }
   float j = 0.f, Rm[4], Qm[4];
   bool late = false;
 #pragma unroll

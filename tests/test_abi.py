@@ -217,6 +217,11 @@ def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
     assert info.kernel == A.KERNEL_TMA and info.cluster_size == 4
     info = A.plan(2, 2, 4099, A.BF16)
     assert info.vector_path == 0 and info.kernel == A.KERNEL_GENERIC
+    assert info.launches == 1 and info.row_kernel == 0
+    info = A.plan(64, 7, 128256, A.BF16, A.gate_params(mode=A.MODE_STOCHASTIC))
+    assert info.launches == 2 and info.row_kernel == 1
+    info = A.plan(64, 7, 128256, A.BF16, A.gate_params(mode=A.MODE_GREEDY))
+    assert info.launches == 2 and info.row_kernel == 0
     with pytest.raises(A.AsymSpecError):
         A.plan(1, 1, 2_000_000, A.FP32)
     info = A.plan(2, 2, 100, A.FP32, opts=A.LaunchOpts(16, 0, 0))
