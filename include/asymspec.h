@@ -60,7 +60,7 @@ extern "C" {
 #define ASYMSPEC_ERR_MISALIGNED (-3)    /* a pointer not aligned to its element size */
 #define ASYMSPEC_ERR_WORKSPACE (-4)     /* workspace missing or smaller than asymspec_workspace_bytes() */
 #define ASYMSPEC_ERR_CUDA (-5)          /* a CUDA call failed; see asymspec_last_cuda_error() */
-#define ASYMSPEC_ERR_TOO_LARGE (-6)     /* V too large for the on-chip row slices (see asymspec_plan) */
+#define ASYMSPEC_ERR_TOO_LARGE (-6)     /* V too large for the row slices of any cluster (see asymspec_plan) */
 #define ASYMSPEC_ERR_SCRATCH_LIMIT (-7) /* B*(K+1) above ASYMSPEC_STATIC_MAX_ROWS (asymspec_fuse_verify_static) */
 
 /* ---- device error-word bits (data errors, per batch element) ----------- */
@@ -111,9 +111,8 @@ typedef struct {
 /* Optional launch overrides (host struct); zero fields mean "automatic". */
 typedef struct {
   int32_t cluster_size;   /* CTAs per row triple: 1 to 16 */
-  int32_t block_threads;  /* 0 automatic; 192, 224 or 256: threads per CTA of the production
-                             row kernel of ASYMSPEC_KERNEL_TMA (the stochastic JSD step
-                             without debug outputs); every other program runs 256 */
+  int32_t block_threads;  /* 0 (automatic) or 256: every kernel runs 256-thread CTAs;
+                             other values are reserved (ASYMSPEC_ERR_INVALID_ARG) */
   int32_t kernel;         /* 0 automatic; ASYMSPEC_KERNEL_GENERIC or ASYMSPEC_KERNEL_TMA */
   int32_t test_flags;     /* 0, or test hooks (ASYMSPEC_TEST_*); other bits reserved, 0 */
   /* Optional cudaEvent_t handles (or NULL): recorded on the call's stream
@@ -125,25 +124,30 @@ typedef struct {
 } asymspec_launch_opts;
 
 /* Test hook (asymspec_launch_opts.test_flags), for tests of the timeout
- * path only: every bulk-copy wait of ASYMSPEC_KERNEL_TMA gives up at once,
- * as if its time limit (200 ms) had passed, while the copies still land.
+ * path only: every bulk-copy wait of the staged row kernel of
+ * ASYMSPEC_KERNEL_TMA (fuse_verify_tma) gives up at once, as if its time
+ * limit (200 ms) had passed, while the copies still land.
  * Each CTA then takes its timeout branch: it marks its row, still reaches
  * every cluster barrier, and before it exits waits (with the normal limit)
  * for its copies in flight; every batch element comes back as a data error
  * (accept_len = next_token = -1) with ASYMSPEC_DATA_TIMEOUT in the error
- * word.  The generic kernel has no bounded waits and ignores it. */
+ * word.  The generic kernel and the production row kernel (fuse_verify_row)
+ * wait on no copies and ignore it. */
 #define ASYMSPEC_TEST_COPY_GIVE_UP 1
 
 /* Kernels (asymspec_launch_opts.kernel, asymspec_launch_info.kernel). */
 #define ASYMSPEC_KERNEL_GENERIC 1  /* one cluster per row; any element-aligned input */
-#define ASYMSPEC_KERNEL_TMA 2      /* one cluster per row, chunked 1-D bulk copies, per-row
-                                      programs, then a decision kernel; rows 16-byte aligned */
+#define ASYMSPEC_KERNEL_TMA 2      /* one cluster per row, then a decision kernel; rows
+                                      16-byte aligned.  The stochastic JSD step without debug
+                                      outputs runs the production row kernel (slices read
+                                      from HBM, then again from the L2); every other program
+                                      stages its slices by chunked 1-D bulk copies */
 
 /* What a launch would use (filled by asymspec_plan). */
 typedef struct {
   int32_t cluster_size;    /* CTAs that split one row triple, combined over DSMEM */
   int32_t block_threads;   /* threads per CTA */
-  int32_t slice_elems;     /* vocabulary entries held on chip per CTA */
+  int32_t slice_elems;     /* vocabulary entries per CTA (its slice of each row) */
   int32_t smem_bytes;      /* dynamic shared memory per CTA */
   int64_t ctas;            /* CTAs in the grid */
   int32_t vector_path;     /* 1 if rows qualify for 16-byte copies (V * element size % 16 == 0) */

@@ -6,8 +6,9 @@
 //                        programs; the default for 16-byte aligned rows.  Its
 //                        rows are decided, and Algorithm 1's scan run, by
 //                        decide_rows, a second launch.
-//   fuse_verify_row      (kernel_row.cuh) the same decomposition with a CTA
-//                        shape chosen per workload and the lean per-entry
+//   fuse_verify_row      (kernel_row.cuh) the same decomposition with no
+//                        slice in shared memory (pass 1 from HBM, pass 2 from
+//                        the L2, four CTAs per SM) and the lean per-entry
 //                        arithmetic: the production program of the
 //                        stochastic JSD step (no debug outputs, delta = a - b).
 //   fuse_verify_generic  (kernel_generic.cuh) one cluster per row, any
@@ -47,7 +48,7 @@ struct Plan {
   long long ctas;  // grid size
   bool vector_path;
   bool row;          // the production row kernel (fuse_verify_row) runs
-  int nt, minb;      // its CTA shape: threads, CTAs per SM (kTThreads, 2 otherwise)
+  int nt;            // threads per CTA (kRowThreads or kTThreads)
   int grid_y;        // the row kernel's grid is (C (K+1), B): grid_y = B (1 otherwise)
 };
 
@@ -56,8 +57,8 @@ struct Plan {
 constexpr int kSmemPerSm = 228 * 1024;
 constexpr int kSmemPerCta = 1024;
 
-const void* row_kernel(int dtype, int nt, int minb) {
-  return dtype == ASYMSPEC_FP32 ? row_kernel_f32(nt, minb) : row_kernel_bf16(nt, minb);
+const void* row_kernel(int dtype) {
+  return dtype == ASYMSPEC_FP32 ? row_kernel_f32() : row_kernel_bf16();
 }
 
 
@@ -113,46 +114,27 @@ bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
   return false;
 }
 
-// The production row kernel: CTA shapes in order of preference (bf16: 224
-// threads three to an SM, else 256 threads two to an SM; fp32: 256 threads
-// two to an SM), each with the smallest cluster (1, 2, 4, 8, 10, 12, 16)
-// whose slice and shared state fit that many CTAs per SM and whose slice
-// takes at most kMaxRounds vectors per thread.  forced_nt, forced_C: the
+// The production row kernel: the first cluster size (8, 12, 16, 4, 10, 2,
+// 1; 8 packs GB300's GPCs best at four CTAs per SM) whose warp blocks take
+// at most kMaxRounds steps (the decision kernel's walk loads a whole block
+// at once).  Only the pass-1 records live in shared memory.  forced_C: the
 // caller's asymspec_launch_opts.
-bool plan_row(int V, int dtype, int forced_C, int forced_nt, Plan* pl) {
+bool plan_row(int V, int dtype, int forced_C, Plan* pl) {
   const int elt = elt_size(dtype);
   const int VE = 16 / elt;
-  struct Shape {
-    int nt, minb;
-  };
-  // (192 threads, four to an SM: on request only)
-  const Shape shapes_bf16[] = {{224, 3}, {256, 3}, {256, 2}, {192, 4}};
-  const Shape shapes_f32[] = {{256, 2}};
-  const Shape* shapes = dtype == ASYMSPEC_FP32 ? shapes_f32 : shapes_bf16;
-  const int nshapes = dtype == ASYMSPEC_FP32 ? 1 : 4;
-  for (int si = 0; si < nshapes; ++si) {
-    const Shape sh = shapes[si];
-    if (forced_nt && sh.nt != forced_nt) continue;
-    if (!forced_nt && sh.nt == 192) continue;
-    if (!row_kernel(dtype, sh.nt, sh.minb)) continue;
-    for (int C : kClusterOrder) {
-      if (forced_C && C != forced_C) continue;
-      const long long per = (static_cast<long long>(V) + C - 1) / C;
-      const long long W = round_up_ll(per, VE);
-      const long long sh_off = round_up_ll(3 * W * elt, 128);
-      const long long smem = sh_off + row_shared_bytes(C);
-      if (W / VE > static_cast<long long>(kMaxRounds) * sh.nt) continue;
-      if (sh.minb * (smem + kSmemPerCta) > kSmemPerSm) continue;
-      if (sh.minb == 2 && smem > kTmaPreferredSmem) continue;
-      pl->C = C;
-      pl->W = static_cast<int>(W);
-      pl->sh_off = static_cast<int>(sh_off);
-      pl->smem = static_cast<int>(smem);
-      pl->group_stride = kGroupsMax;
-      pl->nt = sh.nt;
-      pl->minb = sh.minb;
-      return true;
-    }
+  constexpr int kRowClusters[] = {8, 12, 16, 4, 10, 2, 1};
+  for (int C : kRowClusters) {
+    if (forced_C && C != forced_C) continue;
+    const long long per = (static_cast<long long>(V) + C - 1) / C;
+    const long long W = round_up_ll(per, VE);
+    if (W / VE > static_cast<long long>(kMaxRounds) * kRowThreads) continue;
+    pl->C = C;
+    pl->W = static_cast<int>(W);
+    pl->sh_off = 0;
+    pl->smem = row_shared_bytes(C);
+    pl->group_stride = kGroupsMax;
+    pl->nt = kRowThreads;
+    return true;
   }
   return false;
 }
@@ -198,7 +180,6 @@ int make_plan(int B, int K, int V, int dtype, const asymspec_launch_opts* opts, 
   const int elt = elt_size(dtype);
   const int forced_C = (opts && opts->cluster_size > 0) ? opts->cluster_size : 0;
   const int forced_kernel = opts ? opts->kernel : 0;
-  const int forced_nt = opts ? opts->block_threads : 0;
   if (forced_C < 0 || forced_C > 16) return ASYMSPEC_ERR_INVALID_ARG;
   if (forced_kernel != 0 && forced_kernel != ASYMSPEC_KERNEL_GENERIC &&
       forced_kernel != ASYMSPEC_KERNEL_TMA)
@@ -207,13 +188,12 @@ int make_plan(int B, int K, int V, int dtype, const asymspec_launch_opts* opts, 
   pl->vector_path = vec_ok;
   pl->row = false;
   pl->nt = kTThreads;
-  pl->minb = 2;
   pl->grid_y = 1;
   if (ws_bytes < cluster_ws_bytes(B, K)) return ASYMSPEC_ERR_WORKSPACE;
   bool ok = false;
   // (its grid is (C (K+1), B): B up to 65535)
   if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && prod_row && B <= 65535 &&
-      plan_row(V, dtype, forced_C, forced_nt, pl)) {
+      plan_row(V, dtype, forced_C, pl)) {
     if (ws_bytes >= tma_layout(B, K, pl->C).total) {
       pl->kernel = ASYMSPEC_KERNEL_TMA;
       pl->VE = 16 / elt;
@@ -224,8 +204,6 @@ int make_plan(int B, int K, int V, int dtype, const asymspec_launch_opts* opts, 
       return ASYMSPEC_ERR_WORKSPACE;
     }
   }
-  // other shapes than 256 threads exist for the production row kernel only
-  if (!ok && forced_nt != 0 && forced_nt != kTThreads) return ASYMSPEC_ERR_UNSUPPORTED;
   if (ok) {
     // the production row kernel
   } else if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && plan_tma(V, elt, forced_C, pl)) {
@@ -255,7 +233,7 @@ using KernelFn = const void*;  // a __global__ function taking KParams (or SPara
 
 // sel: the TMA kernel's program set (tma_program_set; 0 = run-time dispatch)
 KernelFn pick_kernel(const Plan& pl, int dtype, bool stoch, int sel = 0) {
-  if (pl.row) return row_kernel(dtype, pl.nt, pl.minb);
+  if (pl.row) return row_kernel(dtype);
   if (pl.kernel == ASYMSPEC_KERNEL_TMA)
     return dtype == ASYMSPEC_FP32 ? tma_kernel_f32(stoch, sel) : tma_kernel_bf16(stoch, sel);
   return generic_kernel(dtype, pl.vector_path, stoch);
@@ -357,8 +335,8 @@ int check_params(const asymspec_gate_params* gp) {
 }
 
 int check_opts(const asymspec_launch_opts* opts) {
-  if (opts && opts->block_threads != 0 && opts->block_threads != 192 &&
-      opts->block_threads != 224 && opts->block_threads != 256)
+  // every kernel runs 256-thread CTAs
+  if (opts && opts->block_threads != 0 && opts->block_threads != 256)
     return ASYMSPEC_ERR_INVALID_ARG;
   if (opts && (opts->test_flags & ~ASYMSPEC_TEST_COPY_GIVE_UP) != 0) return ASYMSPEC_ERR_INVALID_ARG;
   if (opts && ((opts->timing_begin == nullptr) != (opts->timing_end == nullptr)))

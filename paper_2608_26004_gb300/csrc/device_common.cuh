@@ -410,6 +410,12 @@ __device__ __forceinline__ void bulk_load_hint(void* dst, const void* src, unsig
       : "memory");
 }
 
+// Bulk prefetch of [src, src + bytes) into the L2 (no completion to wait
+// for); src 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, unsigned bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // Plain arrive (one count) on an mbarrier of this CTA.
 __device__ __forceinline__ void mbar_arrive(unsigned long long* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");

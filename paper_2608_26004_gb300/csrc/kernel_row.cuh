@@ -3,30 +3,35 @@
 //
 // Same decomposition as fuse_verify_tma (kernel_tma.cuh), whose records it
 // leaves for the same decision kernel: one cluster of C CTAs per row triple
-// (a_k, b_k, t_k); CTA r brings entries [r W, (r+1) W) of the three rows
-// into shared memory with 1-D bulk copies in kChunks chunks, each on its own
-// mbarrier; pass 1 (the normalisers of Eqs. 1-3) streams the slice as the
-// chunks land; the CTAs exchange pass-1 records through distributed shared
-// memory and one cluster barrier; pass 2 reads the slice again from shared
-// memory.  Each logit row is read from HBM once.
+// (a_k, b_k, t_k), CTA r taking entries [r W, (r+1) W) of the three rows;
+// pass 1 (the normalisers of Eqs. 1-3) over the slice; the CTAs exchange
+// pass-1 records through distributed shared memory and one cluster barrier;
+// pass 2 (the divergence of Eq. 3 and the masses of the fused and residual
+// distributions) over the slice again.
 //
-// What differs from fuse_verify_tma is the shape of the work, chosen for
-// the instruction budget (the arithmetic alone is about 27 instructions per
-// vocabulary entry against 6 bytes read, so every instruction a CTA spends
-// once per row counts):
-//   * the CTA shape is a template parameter: NT threads, MINB CTAs per SM
-//     (the register cap of __launch_bounds__);
-//   * each warp owns a contiguous block of the slice: its lane 0 issues the
-//     block's bulk copies (two chunks, each on the warp's own mbarrier), the
-//     warp waits for its own data only, and each step reads 32 consecutive
-//     16-byte vectors per stream (no bank conflicts);
+// What differs from fuse_verify_tma is where the slice lives between the
+// passes and the shape of the work:
+//   * no slice is held in shared memory.  Each warp owns a contiguous block
+//     of the slice; its lane 0 starts with a bulk prefetch of the block's
+//     three streams into the L2, pass 1 reads the block from global memory
+//     (16-byte loads, 32 consecutive vectors per warp and step) and pass 2
+//     reads it again, which the L2 serves.  The rows in flight at once (one
+//     per resident cluster: 74 clusters of 8 CTAs on GB300, 57 MB for
+//     V = 128256 bf16) sit well inside the 129 MB L2, so each logit row
+//     still comes from HBM once.  With only the pass-1 records in shared
+//     memory, four 256-thread CTAs fit on an SM (the register file is the
+//     limit), against three when the slice is staged in shared memory; the
+//     extra warps hide the load latency and the cluster barrier, which is
+//     what bounds this kernel (about 1 warp instruction per vocabulary entry
+//     against 6 bytes read);
 //   * the block of a warp is one inverse-CDF group: its mass is the warp's
 //     residual (or fused) sum, which the warp reduces anyway, so pass 2 needs
 //     no per-step group reductions (the decision kernel walks the group's
 //     vectors);
 //   * one 16-byte vector per stream per step, unpacked pair by pair from the
 //     raw words (bf16 -> fp32 is a shift or a mask), two fp32 lanes per
-//     add/sub/mul/fma instruction;
+//     add/sub/mul/fma instruction, loads issued in batches of kRowBatch
+//     steps;
 //   * the divergence of Eq. 3 in one product per pair.  With p = softmax(a),
 //     q = softmax(b) in log2 units, e = q/p = 2^d (d = log2 q - log2 p) and
 //     w = 1 + e, each entry contributes to 2 JSD (in bits)
@@ -36,10 +41,8 @@
 //     are formed exactly as the decision kernel's inverse-CDF walk forms
 //     them (res_pair), so the group masses and the walk agree bit for bit.
 //
-// Every wait is bounded as in fuse_verify_tma: a chunk that does not land in
-// time (KParams::copy_wait_ns) marks the row ASYMSPEC_DATA_TIMEOUT, the CTA
-// still reaches the cluster barrier, and thread 0 drains its copies
-// (bounded) before the CTA exits.
+// The kernel waits on nothing but the hardware cluster barrier (no copies
+// complete on mbarriers), so it never reports ASYMSPEC_DATA_TIMEOUT.
 #pragma once
 
 #include "kernel_tma.cuh"
@@ -65,10 +68,11 @@ struct RawVec<float> {
   float4 v;
   __device__ __forceinline__ f2 pair(int h) const { return h == 0 ? pk(v.x, v.y) : pk(v.z, v.w); }
 };
+// A vector from global memory (read-only for the kernel's lifetime).
 template <typename T>
-__device__ __forceinline__ RawVec<T> raw_load(const T* p) {
+__device__ __forceinline__ RawVec<T> raw_ldg(const T* p) {
   RawVec<T> r;
-  r.v = *reinterpret_cast<const decltype(r.v)*>(p);
+  r.v = __ldg(reinterpret_cast<const decltype(r.v)*>(p));
   return r;
 }
 
@@ -113,10 +117,12 @@ __device__ __forceinline__ f2 jsd_pair(f2 amb, f2 p, const ResConst& k, f2 jacc)
   return fma2(p, fma2(w, x, mul2(e, d)), jacc);
 }
 
-
 // ---------------------------------------------------------------- layout
 
-constexpr int kRowChunks = 2;  // bulk-copy chunks per warp block
+constexpr int kRowThreads = 256;  // threads per CTA of the row kernel
+constexpr int kRowMinBlocks = 4;  // CTAs per SM (64 registers a thread)
+constexpr int kRowBatch = 2;      // steps whose loads a warp issues together
+static_assert(kRowThreads / 32 <= kRowMaxWarps, "one pass-2 record slot per warp");
 
 // A warp's pass-1 record: the references (nats) and sums of
 // 2^((x - ref) log2 e) of a, b and the fused score, and its data-error bits.
@@ -126,74 +132,50 @@ struct __align__(16) W1 {
   float pad;
 };
 
-// Fixed shared state of the row kernel; the C pass-1 records pushed by the
+// Shared state of the row kernel; the C pass-1 records pushed by the
 // cluster follow it (recv()).
 struct __align__(16) RowShared {
-  unsigned long long bar[kRowMaxWarps][kRowChunks];  // per warp and chunk
-  union {                                            // per-warp records, one pass at a time
-    W1 w1[kRowMaxWarps];
-    X2 w2[kRowMaxWarps];
-  };
-  float lse[4];                 // the row's normalisers (a, b, -, s)
-  unsigned broken;              // a chunk copy timed out
-  float qown;                   // this slice's fused mass (draft rows), from pass 1
-  unsigned long long wait_ns;   // limit of each chunk wait (KParams::copy_wait_ns)
+  W1 w1[kRowMaxWarps];  // per-warp pass-1 records
+  float lse[4];         // the row's normalisers (a, b, -, s)
   __device__ X1* recv() { return reinterpret_cast<X1*>(this + 1); }
 };
-static_assert(sizeof(W1) == 32 && sizeof(X2) == 32, "warp records share storage");
+static_assert(sizeof(W1) == 32, "one warp record is two 16-byte words");
 static_assert(sizeof(RowShared) % 16 == 0, "records after RowShared stay 16-byte aligned");
 
 __host__ __device__ constexpr int row_shared_bytes(int C) {
   return static_cast<int>(sizeof(RowShared) + C * sizeof(X1));
 }
 
-// Lane 0 of warp w: the bulk copies of the warp's block [v0, v1) of the
-// slice (vectors), in two chunks (the first ceil(R/2) steps, then the rest),
-// each completing on the warp's own mbarrier.
-template <typename T>
-__device__ __forceinline__ void issue_block(const KParams& P, RowShared* sh, int w, size_t off,
-                                            int v0, int v1, int split, T* sa, T* sb, T* st) {
-  constexpr int VE = 16 / static_cast<int>(sizeof(T));
-#pragma unroll
-  for (int q = 0; q < kRowChunks; ++q) {
-    const int c0 = q == 0 ? v0 : min(v1, split), c1 = q == 0 ? min(v1, split) : v1;
-    const unsigned bytes = static_cast<unsigned>(max(0, c1 - c0)) * 16u;
-    mbar_arrive_expect_tx(&sh->bar[w][q], 3u * bytes);
-    if (bytes) {
-      const int e0 = c0 * VE;
-      bulk_load(sa + e0, static_cast<const T*>(P.a) + off + e0, bytes, &sh->bar[w][q]);
-      bulk_load(sb + e0, static_cast<const T*>(P.b) + off + e0, bytes, &sh->bar[w][q]);
-      bulk_load(st + e0, static_cast<const T*>(P.t) + off + e0, bytes, &sh->bar[w][q]);
-    }
-  }
-}
-
 // ---------------------------------------------------------------- pass 1
 
-// Pass 1 over the warp's block [v0, v1) (R steps, chunk 1 from step R1 on)
-// with one fixed reference per warp and stream.  DRAFT: the normalisers of
-// a, b and the fused score s; the bonus row needs s only.  Returns true when
-// a lane's sum reached 2^100 or is not finite (the CTA then redoes its slice
-// with a running maximum).  Every lane ends with the warp's record.
+// Pass 1 over the warp's block [v0, v1) of the slice (ga, gb, gt: the
+// slice's first entries in global memory; R steps), with one fixed reference
+// per warp and stream: the largest of the first pairs of the lanes' first
+// vectors.  DRAFT: the normalisers of a, b and the fused score s; the bonus
+// row needs s only.  Returns true when a lane's sum reached 2^100 or is not
+// finite (the CTA then redoes its slice with a running maximum).  Every lane
+// ends with the warp's record.
 template <typename T, bool DRAFT>
-__device__ __forceinline__ bool row_pass1(const T* ra, const T* rb, const T* rt, int v0, int v1,
-                                          int R, int R1, float beta, RowShared* sh, int w,
-                                          W1& e) {
+__device__ __forceinline__ bool row_pass1(const T* ga, const T* gb, const T* gt, int v0, int v1,
+                                          int R, float beta, W1& e) {
   constexpr int NP = RawVec<T>::NP;
   constexpr int VE = 2 * NP;
+  constexpr int U = kRowBatch;
   const int lane = static_cast<int>(threadIdx.x & 31);
-  if (!sh->broken && !mbar_wait_bounded(&sh->bar[w][0], 0u, sh->wait_ns))
-    atomicOr(&sh->broken, kBadTimeout);
   const f2 L2 = pk(kLog2e, kLog2e);
   const float bl = beta * kLog2e;
   const f2 bL2 = pk(bl, bl);
-  // references (nats): the largest of the warp's first pairs of a, b and the
-  // fused score (every lane's first vector is in chunk 0)
-  float ra0 = -INFINITY, rb0 = -INFINITY, rs0 = -INFINITY;
   const int i0 = v0 + lane;
-  if (i0 < v1) {
-    const f2 a2 = first_pair(ra + i0 * VE), b2 = first_pair(rb + i0 * VE);
-    const f2 t2 = first_pair(rt + i0 * VE);
+  const bool have0 = i0 < v1;
+  RawVec<T> va0 = {}, vb0 = {}, vt0 = {};
+  if (have0) {
+    va0 = raw_ldg(ga + i0 * VE);
+    vb0 = raw_ldg(gb + i0 * VE);
+    vt0 = raw_ldg(gt + i0 * VE);
+  }
+  float ra0 = -INFINITY, rb0 = -INFINITY, rs0 = -INFINITY;
+  if (have0) {
+    const f2 a2 = va0.pair(0), b2 = vb0.pair(0), t2 = vt0.pair(0);
     const f2 s2 = fma2(pk(beta, beta), sub2(a2, b2), t2);
     ra0 = fmaxf(lo_of(a2), hi_of(a2));
     rb0 = fmaxf(lo_of(b2), hi_of(b2));
@@ -207,9 +189,7 @@ __device__ __forceinline__ bool row_pass1(const T* ra, const T* rb, const T* rt,
   const float nA = -ra0 * kLog2e, nB = -rb0 * kLog2e, nS = -rs0 * kLog2e;
   const f2 nA2 = pk(nA, nA), nB2 = pk(nB, nB), nS2 = pk(nS, nS);
   f2 acc_a = 0ull, acc_b = 0ull, acc_s = 0ull;
-  auto step = [&](int i) {
-    const RawVec<T> va = raw_load(ra + i * VE), vb = raw_load(rb + i * VE);
-    const RawVec<T> vt = raw_load(rt + i * VE);
+  auto body = [&](const RawVec<T>& va, const RawVec<T>& vb, const RawVec<T>& vt) {
 #pragma unroll
     for (int h = 0; h < NP; ++h) {
       const f2 a2 = va.pair(h), b2 = vb.pair(h), t2 = vt.pair(h);
@@ -220,18 +200,24 @@ __device__ __forceinline__ bool row_pass1(const T* ra, const T* rb, const T* rt,
       acc_s = add2(acc_s, ex2_2(fma2(t2, L2, fma2(bL2, sub2(a2, b2), nS2))));
     }
   };
-  int r = 0;
-#pragma unroll 2
-  for (; r < R1; ++r) {
-    const int i = i0 + 32 * r;
-    if (i < v1) step(i);
-  }
-  if (!sh->broken && !mbar_wait_bounded(&sh->bar[w][1], 0u, sh->wait_ns))
-    atomicOr(&sh->broken, kBadTimeout);
-#pragma unroll 2
-  for (; r < R; ++r) {
-    const int i = i0 + 32 * r;
-    if (i < v1) step(i);
+  if (have0) body(va0, vb0, vt0);
+  // the other steps in batches of U, each batch's loads issued together
+  for (int r0 = 1; r0 < R; r0 += U) {
+    RawVec<T> xa[U], xb[U], xt[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + 32 * (r0 + u);
+      if (r0 + u < R && i < v1) {
+        xa[u] = raw_ldg(ga + i * VE);
+        xb[u] = raw_ldg(gb + i * VE);
+        xt[u] = raw_ldg(gt + i * VE);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + 32 * (r0 + u);
+      if (r0 + u < R && i < v1) body(xa[u], xb[u], xt[u]);
+    }
   }
   float sa = DRAFT ? hsum2(acc_a) : 0.f, sb = DRAFT ? hsum2(acc_b) : 0.f, ss = hsum2(acc_s);
   const bool ovf = !(ss < kSumLimit) || (DRAFT && (!(sa < kSumLimit) || !(sb < kSumLimit)));
@@ -251,10 +237,9 @@ __device__ __forceinline__ bool row_pass1(const T* ra, const T* rb, const T* rt,
 
 // Fallback of row_pass1 (a sum reached 2^100, or non-finite data): each lane
 // keeps a running maximum per stream over its vectors of the warp's block,
-// rescaling its sum when the maximum rises; the lanes then merge.  The block
-// is in shared memory (its chunks have landed, or the warp gave up waiting).
+// rescaling its sum when the maximum rises; the lanes then merge.
 template <typename T, bool DRAFT>
-__device__ __forceinline__ void row_pass1_online(const T* ra, const T* rb, const T* rt, int v0,
+__device__ __forceinline__ void row_pass1_online(const T* ga, const T* gb, const T* gt, int v0,
                                                  int v1, float beta, W1& e) {
   constexpr int NP = RawVec<T>::NP;
   constexpr int VE = 2 * NP;
@@ -262,8 +247,8 @@ __device__ __forceinline__ void row_pass1_online(const T* ra, const T* rb, const
   float m[3] = {-INFINITY, -INFINITY, -INFINITY};  // running maxima of a, b, s (nats)
   float s[3] = {0.f, 0.f, 0.f};                    // sums of 2^((x - m) log2 e)
   for (int i = v0 + lane; i < v1; i += 32) {
-    const RawVec<T> va = raw_load(ra + i * VE), vb = raw_load(rb + i * VE);
-    const RawVec<T> vt = raw_load(rt + i * VE);
+    const RawVec<T> va = raw_ldg(ga + i * VE), vb = raw_ldg(gb + i * VE);
+    const RawVec<T> vt = raw_ldg(gt + i * VE);
 #pragma unroll
     for (int h = 0; h < NP; ++h) {
       const f2 a2 = va.pair(h), b2 = vb.pair(h), t2 = vt.pair(h);
@@ -302,35 +287,47 @@ __device__ __forceinline__ void row_pass1_online(const T* ra, const T* rb, const
 
 // ---------------------------------------------------------------- pass 2
 
-// Pass 2 over the warp's block: DRAFT, the JSD terms (see the header) and
-// the residual masses; the bonus row, the fused masses.  Returns through
-// jsum / msum the warp's sums (every lane ends with them): msum is the mass
-// of the warp's inverse-CDF group.
+// Pass 2 over the warp's block (from the L2, where pass 1 left it): DRAFT,
+// the JSD terms (see the header) and the residual masses; the bonus row, the
+// fused masses.  Returns through jsum / msum the warp's sums (every lane
+// ends with them): msum is the mass of the warp's inverse-CDF group.
 template <typename T, bool DRAFT>
-__device__ __forceinline__ void row_pass2(const T* ra, const T* rb, const T* rt, int v0, int v1,
+__device__ __forceinline__ void row_pass2(const T* ga, const T* gb, const T* gt, int v0, int v1,
                                           int R, const ResConst& k, float& jsum, float& msum) {
   constexpr int NP = RawVec<T>::NP;
   constexpr int VE = 2 * NP;
+  constexpr int U = kRowBatch;
   const int lane = static_cast<int>(threadIdx.x & 31);
   f2 jacc = 0ull, macc = 0ull;
   const int i0 = v0 + lane;
-#pragma unroll 2
-  for (int r = 0; r < R; ++r) {
-    const int i = i0 + 32 * r;
-    if (i < v1) {
-      const RawVec<T> va = raw_load(ra + i * VE), vb = raw_load(rb + i * VE);
-      const RawVec<T> vt = raw_load(rt + i * VE);
+  auto body = [&](const RawVec<T>& va, const RawVec<T>& vb, const RawVec<T>& vt) {
 #pragma unroll
-      for (int h = 0; h < NP; ++h) {
-        f2 amb, p, qf, rr;
-        res_pair(va.pair(h), vb.pair(h), vt.pair(h), k, amb, p, qf, rr);
-        if (DRAFT) {
-          macc = add2(macc, rr);
-          jacc = jsd_pair(amb, p, k, jacc);
-        } else {
-          macc = add2(macc, qf);
-        }
+    for (int h = 0; h < NP; ++h) {
+      f2 amb, p, qf, rr;
+      res_pair(va.pair(h), vb.pair(h), vt.pair(h), k, amb, p, qf, rr);
+      if (DRAFT) {
+        macc = add2(macc, rr);
+        jacc = jsd_pair(amb, p, k, jacc);
+      } else {
+        macc = add2(macc, qf);
       }
+    }
+  };
+  for (int r0 = 0; r0 < R; r0 += U) {
+    RawVec<T> xa[U], xb[U], xt[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + 32 * (r0 + u);
+      if (r0 + u < R && i < v1) {
+        xa[u] = raw_ldg(ga + i * VE);
+        xb[u] = raw_ldg(gb + i * VE);
+        xt[u] = raw_ldg(gt + i * VE);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + 32 * (r0 + u);
+      if (r0 + u < R && i < v1) body(xa[u], xb[u], xt[u]);
     }
   }
   float j = hsum2(jacc), m = hsum2(macc), z0 = 0.f, z1 = 0.f;
@@ -353,16 +350,15 @@ __device__ __forceinline__ unsigned cluster_id_y() {
   return r;
 }
 
-// Grid: (C (K+1), B) CTAs in clusters of (C, 1, 1); cluster (k, bi) takes
-// row k of batch element bi.  What it leaves for the decision kernel: rank
-// 0's row statistics (the normalisers, data-error bits) and one pass-2 record
-// per warp of every CTA (KParams::pass2_rec, kRowMaxWarps records per CTA):
-// the warp's JSD sum, the residual and fused masses of its block (its
-// inverse-CDF group) and the timeout flag.
-template <typename T, int NT, int MINB>
-__global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
-  static_assert(NT % 32 == 0 && NT / 32 <= kRowMaxWarps, "at most kRowMaxWarps warps");
-  constexpr int NW = NT / 32;
+// Grid: (C (K+1), B) CTAs of kRowThreads threads in clusters of (C, 1, 1);
+// cluster (k, bi) takes row k of batch element bi.  What it leaves for the
+// decision kernel: rank 0's row statistics (the normalisers, data-error
+// bits) and one pass-2 record per warp of every CTA (KParams::pass2_rec,
+// kRowMaxWarps records per CTA): the warp's JSD sum, the residual and fused
+// masses of its block (its inverse-CDF group).
+template <typename T>
+__global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(const KParams P) {
+  constexpr int NW = kRowThreads / 32;
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr unsigned FD = F_LA | F_LB | F_LS;
   extern __shared__ __align__(128) unsigned char smem_row[];
@@ -379,40 +375,36 @@ __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
   const int lo = rank * W;
   const int n = max(0, min(W, P.V - lo));
   const int nv = n / VE;
-  // this warp's block of the slice, its steps, and the step chunk 1 starts at
+  // this warp's block of the slice (vectors) and its steps
   const int bw = row_block_vectors(nv, NW);
   const int v0 = min(nv, warp * bw), v1 = min(nv, v0 + bw);
-  const int R = (v1 - v0 + 31) / 32, R1 = (R + 1) / 2;
-  T* sa = reinterpret_cast<T*>(smem_row);
-  T* sb = sa + W;
-  T* st = sb + W;
-  RowShared* sh = reinterpret_cast<RowShared*>(smem_row + P.sh_off);
+  const int R = (v1 - v0 + 31) / 32;
+  const size_t off = static_cast<size_t>(row32) * P.V + lo;
+  const T* ga = static_cast<const T*>(P.a) + off;
+  const T* gb = static_cast<const T*>(P.b) + off;
+  const T* gt = static_cast<const T*>(P.t) + off;
+  RowShared* sh = reinterpret_cast<RowShared*>(smem_row);
   const bool draft = k < P.K;
 
-  // each warp brings in its own block: no CTA barrier before the copies
-  if (lane == 0) {
-    mbar_init(&sh->bar[warp][0], 1);
-    mbar_init(&sh->bar[warp][1], 1);
-    fence_mbar_init();
-    issue_block<T>(P, sh, warp, static_cast<size_t>(row32) * P.V + lo, v0, v1, v0 + 32 * R1, sa,
-                   sb, st);
+  // the warp's block of the three rows into the L2 (16-byte aligned: the
+  // host takes this kernel only for rows of a multiple of 16 bytes)
+  if (lane == 0 && v1 > v0) {
+    const unsigned bytes = static_cast<unsigned>(v1 - v0) * 16u;
+    bulk_prefetch_l2(ga + v0 * VE, bytes);
+    bulk_prefetch_l2(gb + v0 * VE, bytes);
+    bulk_prefetch_l2(gt + v0 * VE, bytes);
   }
-  if (tid == 0) {
-    sh->broken = 0;
-    sh->wait_ns = P.copy_wait_ns;
-  }
-  __syncthreads();  // every warp's barriers and the shared flags are initialised
 
   // ---- pass 1: the row normalisers, combined over the cluster
   W1 e;
-  const bool ovf = draft ? row_pass1<T, true>(sa, sb, st, v0, v1, R, R1, P.beta, sh, warp, e)
-                         : row_pass1<T, false>(sa, sb, st, v0, v1, R, R1, P.beta, sh, warp, e);
+  const bool ovf = draft ? row_pass1<T, true>(ga, gb, gt, v0, v1, R, P.beta, e)
+                         : row_pass1<T, false>(ga, gb, gt, v0, v1, R, P.beta, e);
   if (lane == 0) sh->w1[warp] = e;
   if (__syncthreads_or(ovf)) {
     // an entry far above its warp's reference (or non-finite data): redo the
     // slice with running maxima
-    if (draft) row_pass1_online<T, true>(sa, sb, st, v0, v1, P.beta, e);
-    else row_pass1_online<T, false>(sa, sb, st, v0, v1, P.beta, e);
+    if (draft) row_pass1_online<T, true>(ga, gb, gt, v0, v1, P.beta, e);
+    else row_pass1_online<T, false>(ga, gb, gt, v0, v1, P.beta, e);
     e.bad = 0u;
     e.pad = 0.f;
     if (lane == 0) sh->w1[warp] = e;
@@ -432,7 +424,7 @@ __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
     }
     if (draft) warp_reduce_x1<FD>(x);
     else warp_reduce_x1<F_LS>(x);
-    x.bad = sh->broken;
+    x.bad = 0u;
     push_record(x, sh->recv(), rank, C, cluster);
   }
   cluster_barrier(warp == 0);  // every CTA's pass-1 record is in every CTA
@@ -459,9 +451,8 @@ __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
   const float A2 = sh->lse[0] * kLog2e, B2 = sh->lse[1] * kLog2e, S2 = sh->lse[3] * kLog2e;
   const ResConst kc = res_const(P.beta, A2, B2, S2);
   float jsum, msum;
-  if (draft) row_pass2<T, true>(sa, sb, st, v0, v1, R, kc, jsum, msum);
-  else row_pass2<T, false>(sa, sb, st, v0, v1, R, kc, jsum, msum);
-  const bool broken = sh->broken != 0;
+  if (draft) row_pass2<T, true>(ga, gb, gt, v0, v1, R, kc, jsum, msum);
+  else row_pass2<T, false>(ga, gb, gt, v0, v1, R, kc, jsum, msum);
   if (lane == 0) {
     // this warp's record: its block is one inverse-CDF group of the row.  A
     // draft row's fused mass (the draw's fallback when the row's whole
@@ -470,14 +461,7 @@ __global__ void __launch_bounds__(NT, MINB) fuse_verify_row(const KParams P) {
     float4* rec = reinterpret_cast<float4*>(
         P.pass2_rec + ((static_cast<size_t>(row32) * C + rank) * kRowMaxWarps + warp) * 8);
     rec[0] = make_float4(jsum, 0.f, 0.f, draft ? msum : 0.f);
-    rec[1] = make_float4(qf, broken ? __uint_as_float(kBadTimeout) : 0.f, 0.f, 0.f);
-  }
-
-  // a copy that timed out may still land: wait for it (bounded, always with
-  // the normal limit) before the CTA exits
-  if (lane == 0 && broken) {
-    mbar_wait_bounded(&sh->bar[warp][0], 0u, kCopyTimeoutNs);
-    mbar_wait_bounded(&sh->bar[warp][1], 0u, kCopyTimeoutNs);
+    rec[1] = make_float4(qf, 0.f, 0.f, 0.f);
   }
 }
 

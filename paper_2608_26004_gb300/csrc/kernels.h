@@ -16,10 +16,10 @@ const void* tma_kernel_bf16_any_stoch();  // k_tma_bf16_any_s.cu
 const void* tma_kernel_f32_any_stoch();   // k_tma_f32_any_s.cu
 const void* tma_kernel_bf16(bool stoch, int sel);
 const void* tma_kernel_f32(bool stoch, int sel);
-// fuse_verify_row<T, NT, MINB>, the production kernel of the stochastic JSD
-// step (k_row_bf16.cu, k_row_f32.cu); nullptr for a shape not instantiated
-const void* row_kernel_bf16(int nt, int minb);
-const void* row_kernel_f32(int nt, int minb);
+// fuse_verify_row<T>, the production kernel of the stochastic JSD step
+// (k_row_bf16.cu, k_row_f32.cu)
+const void* row_kernel_bf16();
+const void* row_kernel_f32();
 // decide_rows<T, STOCH>, launched after fuse_verify_tma or fuse_verify_row (k_tma_*.cu)
 const void* decide_kernel_bf16(bool stoch);
 const void* decide_kernel_f32(bool stoch);

@@ -403,8 +403,7 @@ def test_entries_far_above_the_first_vector(torch, kernel, mode):
 
 # ---------------------------------------------------------------- bounded waits
 
-@pytest.mark.parametrize("mode", [GREEDY, STOCH])
-@pytest.mark.parametrize("full", [False, True])
+@pytest.mark.parametrize("mode,full", [(GREEDY, False), (GREEDY, True), (STOCH, True)])
 def test_copy_wait_timeout_marks_every_row(torch, mode, full):
     # the test hook makes every bulk-copy wait give up at once while the copies
     # still land: each CTA takes its timeout branch (marks its row, reaches every
@@ -424,41 +423,54 @@ def test_copy_wait_timeout_marks_every_row(torch, mode, full):
     check(batch, torch, mode, TMA, full)
 
 
+def test_copy_wait_hook_ignored_by_the_production_row_kernel(torch):
+    # the production row kernel waits on no copies: the hook changes nothing
+    batch = small(3, 2, 40000, synth.BF16, seed=18)
+    x = device_inputs(batch, torch)
+    fv = A.FuseVerify(batch.B, batch.K)
+    res = fv(x["a"], x["b"], x["t"], x["tokens"], x["probs"], x["unif"], mode=STOCH,
+             kernel=TMA, test_flags=A.TEST_COPY_GIVE_UP)
+    ref = fv(x["a"], x["b"], x["t"], x["tokens"], x["probs"], x["unif"], mode=STOCH, kernel=TMA)
+    torch.cuda.synchronize()
+    assert A.plan(3, 2, 40000, A.BF16, A.gate_params(mode=STOCH)).row_kernel == 1
+    for key in ("accept_len", "next_token", "error_word"):
+        assert np.array_equal(res[key].cpu().numpy(), ref[key].cpu().numpy())
+    assert int(res["error_word"].cpu().numpy()[0]) == 0
+
+
 # ---------------------------------------------------------------- the production row kernel
 
-@pytest.mark.parametrize("nt", [224, 256])
-@pytest.mark.parametrize("cluster", [1, 2, 4, 8, 12, 16])
-def test_row_kernel_shapes(torch, nt, cluster):
-    # the production kernel of the stochastic JSD step in every CTA shape and
-    # cluster size the planner may take: several rounds, a ragged last round,
-    # bf16 and fp32 rows, slices down to a single vector
+@pytest.mark.parametrize("cluster", [1, 2, 4, 8, 10, 12, 16])
+def test_row_kernel_shapes(torch, cluster):
+    # the production kernel of the stochastic JSD step at every cluster size
+    # the planner may take: several steps per warp, a ragged last step, bf16
+    # and fp32 rows, warp blocks down to a single vector, empty warp blocks
     for B, K, V, dtype, seed in ((3, 3, 40000, synth.BF16, 61), (2, 2, 12288, synth.FP32, 62),
                                  (4, 1, 8200, synth.BF16, 63), (2, 2, 8 * cluster, synth.BF16, 64),
                                  (2, 3, 128256, synth.BF16, 65)):
-        if dtype == synth.FP32 and nt != 256:
-            continue
         batch = small(B, K, V, dtype, seed)
+        # a warp block of more than 10 steps (the decision kernel's walk loads a
+        # whole block at once) is not taken by the row kernel: the staged kernel
+        # takes the row if its slice fits on chip, else the planner refuses it
+        vecs = -(-V // cluster) * (4 if dtype == synth.FP32 else 2) // 16
         try:
-            g = run_gpu(batch, torch, mode=STOCH, full="row", cluster_size=cluster,
-                        block_threads=nt)
+            g = run_gpu(batch, torch, mode=STOCH, full="row", cluster_size=cluster)
         except A.AsymSpecError as e:
-            # a slice that does not fit on chip at this shape (more than 10
-            # vectors per thread, or too much shared memory for the CTAs per
-            # SM the shape stands for) is refused by the planner
-            assert e.status in (A.ERR_TOO_LARGE, A.ERR_UNSUPPORTED)
-            vecs = -(-V // cluster) * (4 if dtype == synth.FP32 else 2) // 16
-            slice_bytes = 3 * vecs * 16
-            assert vecs > 10 * nt or slice_bytes > 70 * 1024
+            assert e.status == A.ERR_TOO_LARGE and vecs > 10 * 256
             continue
+        info = A.plan(B, K, V, A.FP32 if dtype == synth.FP32 else A.BF16,
+                      A.gate_params(mode=STOCH), A.LaunchOpts(cluster, 0, 0))
+        assert info.row_kernel == (1 if vecs <= 10 * 256 else 0)
         o = run_oracle(batch, mode=STOCH, logprobs=False)
         compare(batch, g, o, mode=STOCH, logprobs=False)
 
 
 def test_row_kernel_is_the_production_choice(torch):
-    for B, K, V, dtype in ((64, 7, 128256, synth.BF16), (8, 5, 151936, synth.BF16),
-                           (256, 4, 151936, synth.FP32)):
+    for B, K, V, dtype, C in ((64, 7, 128256, A.BF16, 8), (8, 5, 151936, A.BF16, 8),
+                              (256, 4, 151936, A.FP32, 16), (1, 4, 32000, A.FP32, 8)):
         info = A.plan(B, K, V, dtype, A.gate_params(mode=STOCH))
-        assert info.kernel == A.KERNEL_TMA
-        if dtype == synth.BF16:      # three CTAs of 224 threads per SM
-            assert info.block_threads == 224 and info.smem_bytes * 3 <= 225 * 1024
+        assert info.kernel == A.KERNEL_TMA and info.row_kernel == 1 and info.launches == 2
+        # 256-thread CTAs with only the cluster's pass-1 records in shared memory
+        assert info.block_threads == 256 and info.cluster_size == C
+        assert info.smem_bytes <= 2048
         assert info.max_active_clusters > 0
