@@ -358,6 +358,10 @@ __device__ __forceinline__ unsigned cluster_id_y() {
 // masses of its block (its inverse-CDF group).
 template <typename T>
 __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(const KParams P) {
+  // the decision kernel (a programmatic dependent) may be scheduled once
+  // every CTA of this grid has started; it waits for this grid's completion
+  // before it reads anything the grid writes
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   constexpr int NW = kRowThreads / 32;
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr unsigned FD = F_LA | F_LB | F_LS;

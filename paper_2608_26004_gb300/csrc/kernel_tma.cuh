@@ -1407,6 +1407,10 @@ __host__ __device__ constexpr int tma_program_set(bool stoch, int divergence, bo
 // takes entries [r W, (r+1) W) of the row.
 template <typename T, bool STOCH, int SEL>
 __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P) {
+  // the decision kernel (a programmatic dependent) may be scheduled once
+  // every CTA of this grid has started; it waits for this grid's completion
+  // before it reads anything the grid writes
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   extern __shared__ __align__(128) unsigned char smem_tma[];
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
@@ -1503,7 +1507,8 @@ __global__ void __launch_bounds__(kTThreads, 2) fuse_verify_tma(const KParams P)
 
 // ---------------------------------------------------------------- row decisions
 
-constexpr int kDecideThreads = 256;  // at most 8 warps; each takes rows k, k + 8, ...
+constexpr int kDecideThreads = 512;  // at most 16 warps; each takes rows k, k + 16, ...
+constexpr int kDecideSmemRows = 64;  // rows of an element whose records the scan reads from shared memory
 
 // ---- rows of fuse_verify_row (kernel_row.cuh): one pass-2 record per warp
 // block, each block one inverse-CDF group
@@ -1666,6 +1671,7 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
   const int K = P.K, K1 = K + 1, C = P.C;
   const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
   const bool klg = P.divergence == ASYMSPEC_DIV_KL;
+  __shared__ int4 srec[kDecideSmemRows];  // the element's records (K + 1 <= kDecideSmemRows)
   // the kernel inputs of this warp's first row, loaded before the wait
   RowInputs pre{-1, 0.f, 0.f, 0.f, RowScalars{0.f, 0.f, 0.f}};
   if (STOCH && P.row_blocks && warp < K1) pre = load_row_inputs<T>(P, bi, warp);
@@ -1678,8 +1684,11 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
       if (P.row_blocks) {  // a row of fuse_verify_row
         const RowInputs din = (k == warp) ? pre : load_row_inputs<T>(P, bi, k);
         const RowResult rr = block_row_result<T>(P, k, row, din.sc);
-        if (lane == 0)
-          P.recs[row] = row_record<true>(P, row, k, rr, din.dtok, din.ad, din.bd, din.td, din.sc);
+        if (lane == 0) {
+          const int4 rec = row_record<true>(P, row, k, rr, din.dtok, din.ad, din.bd, din.td, din.sc);
+          P.recs[row] = rec;
+          if (k < kDecideSmemRows) srec[k] = rec;
+        }
         continue;
       }
     }
@@ -1766,10 +1775,15 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
     r.mass = mass_total;
     r.bad = st.bad;
     r.have_lse_t = has_t;
-    if (lane == 0) P.recs[row] = row_record<STOCH>(P, row, k, r, st.dtok, st.da, st.db, st.dt, sc);
+    if (lane == 0) {
+      const int4 rec = row_record<STOCH>(P, row, k, r, st.dtok, st.da, st.db, st.dt, sc);
+      P.recs[row] = rec;
+      if (k < kDecideSmemRows) srec[k] = rec;
+    }
   }
   __syncthreads();  // the element's records are visible to the block
   const int4* recs = P.recs + static_cast<size_t>(bi) * K1;
+  const bool in_smem = K1 <= kDecideSmemRows;
   if (warp != 0) return;
   // Algorithm 1: the first rejected draft, or K if none; any data error voids the element
   bool any_err = false;
@@ -1777,7 +1791,7 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
   for (int base = 0; base < K1; base += 32) {
     const int j = base + lane;
     int4 v = make_int4(1, -1, 0, 0);
-    if (j < K1) v = __ldcg(&recs[j]);
+    if (j < K1) v = in_smem ? srec[j] : __ldcg(&recs[j]);
     any_err |= __any_sync(0xffffffffu, v.z != 0);
     if (len < 0) {
       const unsigned rej = __ballot_sync(0xffffffffu, j < K && v.x == 0);
