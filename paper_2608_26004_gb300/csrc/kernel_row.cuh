@@ -30,8 +30,7 @@
 //     vectors);
 //   * one 16-byte vector per stream per step, unpacked pair by pair from the
 //     raw words (bf16 -> fp32 is a shift or a mask), two fp32 lanes per
-//     add/sub/mul/fma instruction, loads issued in batches of kRowBatch
-//     steps;
+//     add/sub/mul/fma instruction, two steps of loads in flight per warp;
 //   * the divergence of Eq. 3 in one product per pair.  With p = softmax(a),
 //     q = softmax(b) in log2 units, e = q/p = 2^d (d = log2 q - log2 p) and
 //     w = 1 + e, each entry contributes to 2 JSD (in bits)
@@ -121,7 +120,6 @@ __device__ __forceinline__ f2 jsd_pair(f2 amb, f2 p, const ResConst& k, f2 jacc)
 
 constexpr int kRowThreads = 256;  // threads per CTA of the row kernel
 constexpr int kRowMinBlocks = 4;  // CTAs per SM (64 registers a thread)
-constexpr int kRowBatch = 2;      // steps whose loads a warp issues together
 static_assert(kRowThreads / 32 <= kRowMaxWarps, "one pass-2 record slot per warp");
 
 // A warp's pass-1 record: the references (nats) and sums of
@@ -160,7 +158,6 @@ __device__ __forceinline__ bool row_pass1(const T* ga, const T* gb, const T* gt,
                                           int R, float beta, W1& e) {
   constexpr int NP = RawVec<T>::NP;
   constexpr int VE = 2 * NP;
-  constexpr int U = kRowBatch;
   const int lane = static_cast<int>(threadIdx.x & 31);
   const f2 L2 = pk(kLog2e, kLog2e);
   const float bl = beta * kLog2e;
@@ -201,23 +198,10 @@ __device__ __forceinline__ bool row_pass1(const T* ga, const T* gb, const T* gt,
     }
   };
   if (have0) body(va0, vb0, vt0);
-  // the other steps in batches of U, each batch's loads issued together
-  for (int r0 = 1; r0 < R; r0 += U) {
-    RawVec<T> xa[U], xb[U], xt[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + 32 * (r0 + u);
-      if (r0 + u < R && i < v1) {
-        xa[u] = raw_ldg(ga + i * VE);
-        xb[u] = raw_ldg(gb + i * VE);
-        xt[u] = raw_ldg(gt + i * VE);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + 32 * (r0 + u);
-      if (r0 + u < R && i < v1) body(xa[u], xb[u], xt[u]);
-    }
+#pragma unroll 2
+  for (int r = 1; r < R; ++r) {
+    const int i = i0 + 32 * r;
+    if (i < v1) body(raw_ldg(ga + i * VE), raw_ldg(gb + i * VE), raw_ldg(gt + i * VE));
   }
   float sa = DRAFT ? hsum2(acc_a) : 0.f, sb = DRAFT ? hsum2(acc_b) : 0.f, ss = hsum2(acc_s);
   const bool ovf = !(ss < kSumLimit) || (DRAFT && (!(sa < kSumLimit) || !(sb < kSumLimit)));
@@ -296,7 +280,6 @@ __device__ __forceinline__ void row_pass2(const T* ga, const T* gb, const T* gt,
                                           int R, const ResConst& k, float& jsum, float& msum) {
   constexpr int NP = RawVec<T>::NP;
   constexpr int VE = 2 * NP;
-  constexpr int U = kRowBatch;
   const int lane = static_cast<int>(threadIdx.x & 31);
   f2 jacc = 0ull, macc = 0ull;
   const int i0 = v0 + lane;
@@ -313,22 +296,10 @@ __device__ __forceinline__ void row_pass2(const T* ga, const T* gb, const T* gt,
       }
     }
   };
-  for (int r0 = 0; r0 < R; r0 += U) {
-    RawVec<T> xa[U], xb[U], xt[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + 32 * (r0 + u);
-      if (r0 + u < R && i < v1) {
-        xa[u] = raw_ldg(ga + i * VE);
-        xb[u] = raw_ldg(gb + i * VE);
-        xt[u] = raw_ldg(gt + i * VE);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + 32 * (r0 + u);
-      if (r0 + u < R && i < v1) body(xa[u], xb[u], xt[u]);
-    }
+#pragma unroll 2
+  for (int r = 0; r < R; ++r) {
+    const int i = i0 + 32 * r;
+    if (i < v1) body(raw_ldg(ga + i * VE), raw_ldg(gb + i * VE), raw_ldg(gt + i * VE));
   }
   float j = hsum2(jacc), m = hsum2(macc), z0 = 0.f, z1 = 0.f;
   warp_sum4(j, m, z0, z1);
