@@ -272,6 +272,20 @@ cudaError_t prepare_kernel(KernelFn fn, int device) {
   return cudaSuccess;
 }
 
+// The decision kernel: dynamic shared memory (walk staging) up to what its
+// static records leave of the per-CTA limit; no clusters.
+cudaError_t prepare_decide(KernelFn fn, int device) {
+  std::lock_guard<std::mutex> lock(g_mu);
+  const void* f = fn;
+  for (int i = 0; i < g_attr_count; ++i)
+    if (g_attr_done[i].fn == f && g_attr_done[i].device == device) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kMaxSmem - kDecideSmemRows * 16);
+  if (e != cudaSuccess) return e;
+  if (g_attr_count < 64) g_attr_done[g_attr_count++] = {f, device};
+  return cudaSuccess;
+}
+
 cudaLaunchConfig_t launch_config(const Plan& pl, long long ctas, cudaStream_t stream,
                                  cudaLaunchAttribute* attr) {
   cudaLaunchConfig_t cfg = {};
@@ -599,6 +613,7 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
   P.tma_threads = pl.nt;
   P.row_blocks = pl.row ? 1 : 0;
   // the chunk waits of the TMA kernel: bounded, or (test hook) giving up at once
+  P.walk_stage = 0;
   P.copy_wait_ns =
       (opts && (opts->test_flags & ASYMSPEC_TEST_COPY_GIVE_UP)) ? 0ull : kCopyTimeoutNs;
   P.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) +
@@ -633,18 +648,31 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
     // the rows' decisions and Algorithm 1's scan: one CTA per batch element
     // as a programmatic dependent launch: its launch overlaps the row
     // kernel's last CTAs, and it waits (griddepcontrol.wait) for that kernel
-    const int warps = std::min(K + 1, kDecideThreads / 32);
+    int warps = std::min(K + 1, kDecideThreads / 32);
+    // rows of the production row kernel: each warp stages the vectors of the
+    // inverse-CDF group it walks (at most one warp block: 3 streams x 32
+    // vectors per step) in shared memory
+    P.walk_stage = 0;
+    if (pl.row) {
+      const int nv = pl.W / pl.VE;
+      const int steps = (row_block_vectors(nv, pl.nt / 32) + 31) / 32;
+      P.walk_stage = 3 * steps * 32 * 16;
+      warps = std::min(warps, (kMaxSmem - kDecideSmemRows * 16) / P.walk_stage);
+    }
+    const KernelFn dfn = pick_decide(dtype, stoch);
+    e = prepare_decide(dfn, device);
+    if (e != cudaSuccess) return cuda_fail(e);
     cudaLaunchConfig_t dcfg = {};
     cudaLaunchAttribute dattr[1];
     dattr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     dattr[0].val.programmaticStreamSerializationAllowed = 1;
     dcfg.gridDim = dim3(static_cast<unsigned>(B));
     dcfg.blockDim = dim3(32 * warps);
-    dcfg.dynamicSmemBytes = 0;
+    dcfg.dynamicSmemBytes = static_cast<size_t>(warps) * P.walk_stage;
     dcfg.stream = static_cast<cudaStream_t>(stream);
     dcfg.attrs = dattr;
     dcfg.numAttrs = 1;
-    e = cudaLaunchKernelExC(&dcfg, pick_decide(dtype, stoch), args);
+    e = cudaLaunchKernelExC(&dcfg, dfn, args);
     if (e != cudaSuccess) return cuda_fail(e);
   }
   return ASYMSPEC_OK;

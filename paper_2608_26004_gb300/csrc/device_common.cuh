@@ -453,6 +453,7 @@ struct KParams {
   int tma_threads;      // threads per CTA of the row kernel (its group layout)
   int row_blocks;       // 1: fuse_verify_row's layout, one inverse-CDF group per warp block
   unsigned long long copy_wait_ns;  // limit of each bulk-copy wait (0: give up at once)
+  int walk_stage;       // decide_rows on fuse_verify_row's rows: staging bytes per warp
 };
 
 // What pass 1 leaves for the decision of a row: the normalisers, the

@@ -1160,28 +1160,42 @@ __host__ __device__ __forceinline__ int row_block_vectors(int nv, int nw) {
 // fuse_verify_row: a warp's block), by one warp: the smallest index whose
 // cumulative residual (use_r) or fused mass exceeds trem, or with take_last
 // (rounding left the target at or beyond the group's mass) the last index
-// with positive mass.  Every vector mass of the group is loaded first
-// (independent loads, one round trip), then scanned 32 vectors at a time in
-// index order; the masses are formed exactly as the row kernel's pass 2
-// forms them.  Returns the index within the row, or -1 if the group holds
-// no mass.
+// with positive mass.  The group's vectors of the three rows are first
+// copied into the warp's staging area `stg` (16-byte cp.async, all in
+// flight at once: one round trip; 3 x 32 ceil((b1 - b0) / 32) vectors), then
+// their masses are scanned 32 vectors at a time in index order; the masses
+// are formed exactly as the row kernel's pass 2 forms them.  Returns the
+// index within the row, or -1 if the group holds no mass.
 template <typename T>
 __device__ __noinline__ int walk_vectors(const T* ga, const T* gb, const T* gt, int b0, int b1,
                                          int lo, float beta, bool use_r, float A2, float S2,
-                                         float trem, bool take_last) {
+                                         float trem, bool take_last, uint4* stg) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   constexpr int NP = VE / 2;
   const int lane = threadIdx.x & 31;
   const f2 beta2 = pk(beta, beta), L2 = pk(kLog2e, kLog2e);
   const f2 nA2 = pk(-A2, -A2), nS2 = pk(-S2, -S2);
+  // staging: vector j of the group (vector b0 + j of the slice) of stream
+  // a, b, t at stg[j], stg[cap + j], stg[2 cap + j]
+  const int nvb = max(0, b1 - b0), cap = (nvb + 31) & ~31;
+  T* sa = reinterpret_cast<T*>(stg);
+  T* sb = reinterpret_cast<T*>(stg + cap);
+  T* st = reinterpret_cast<T*>(stg + 2 * cap);
+  for (int j = lane; j < nvb; j += 32) {
+    cp_async16(sa + j * VE, ga + (b0 + j) * VE);
+    cp_async16(sb + j * VE, gb + (b0 + j) * VE);
+    cp_async16(st + j * VE, gt + (b0 + j) * VE);
+  }
+  cp_async_wait_all();
+  __syncwarp();
   float mvs[kMaxRounds];
 #pragma unroll
   for (int s = 0; s < kMaxRounds; ++s) {
-    const int v = b0 + 32 * s + lane;
+    const int j = 32 * s + lane;
     mvs[s] = 0.f;
-    if (v < b1) {
+    if (j < nvb) {
       f2 p[NP], qf[NP], r[NP];
-      slice_vector_masses<T>(ga, gb, gt, v, beta2, L2, nA2, nS2, p, qf, r);
+      slice_vector_masses<T>(sa, sb, st, j, beta2, L2, nA2, nS2, p, qf, r);
       mvs[s] = vsum(use_r ? r : qf);
     }
   }
@@ -1219,7 +1233,7 @@ __device__ __noinline__ int walk_vectors(const T* ga, const T* gb, const T* gt, 
   int found = -1;
   if (lane == 0) {
     f2 p[NP], qf[NP], r[NP];
-    slice_vector_masses<T>(ga, gb, gt, vsel, beta2, L2, nA2, nS2, p, qf, r);
+    slice_vector_masses<T>(sa, sb, st, vsel - b0, beta2, L2, nA2, nS2, p, qf, r);
     float cum = 0.f;
     int pick = -1, last = -1;
 #pragma unroll
@@ -1551,7 +1565,7 @@ __device__ __forceinline__ RowInputs load_row_inputs(const KParams& P, int bi, i
 // element.
 template <typename T>
 __device__ __forceinline__ RowResult block_row_result(const KParams& P, int k, long long row,
-                                                      const RowScalars& sc) {
+                                                      const RowScalars& sc, uint4* stg) {
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
   const int lane = threadIdx.x & 31;
   const int C = P.C, NW = P.tma_threads / 32, ng = C * NW;
@@ -1652,7 +1666,7 @@ __device__ __forceinline__ RowResult block_row_result(const KParams& P, int k, l
   const size_t off = static_cast<size_t>(row) * P.V + lo_r;
   rr.sample = walk_vectors<T>(static_cast<const T*>(P.a) + off, static_cast<const T*>(P.b) + off,
                               static_cast<const T*>(P.t) + off, b0, b1, lo_r, P.beta, r_ok,
-                              st.lse[0] * kLog2e, st.lse[3] * kLog2e, trem, take_last);
+                              st.lse[0] * kLog2e, st.lse[3] * kLog2e, trem, take_last, stg);
   return rr;
 }
 
@@ -1672,6 +1686,9 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
   const bool jsd = P.divergence == ASYMSPEC_DIV_JSD;
   const bool klg = P.divergence == ASYMSPEC_DIV_KL;
   __shared__ int4 srec[kDecideSmemRows];  // the element's records (K + 1 <= kDecideSmemRows)
+  // rows of fuse_verify_row: each warp's staging area for its walks
+  extern __shared__ uint4 walk_stage[];
+  uint4* stg = walk_stage + static_cast<size_t>(warp) * (P.walk_stage / 16);
   // the kernel inputs of this warp's first row, loaded before the wait
   RowInputs pre{-1, 0.f, 0.f, 0.f, RowScalars{0.f, 0.f, 0.f}};
   if (STOCH && P.row_blocks && warp < K1) pre = load_row_inputs<T>(P, bi, warp);
@@ -1683,7 +1700,7 @@ __global__ void __launch_bounds__(kDecideThreads) decide_rows(const KParams P) {
     if constexpr (STOCH) {
       if (P.row_blocks) {  // a row of fuse_verify_row
         const RowInputs din = (k == warp) ? pre : load_row_inputs<T>(P, bi, k);
-        const RowResult rr = block_row_result<T>(P, k, row, din.sc);
+        const RowResult rr = block_row_result<T>(P, k, row, din.sc, stg);
         if (lane == 0) {
           const int4 rec = row_record<true>(P, row, k, rr, din.dtok, din.ad, din.bd, din.td, din.sc);
           P.recs[row] = rec;
