@@ -374,17 +374,22 @@ int asymspec_draft_sample(const void* logits, int rows, int V, int dtype, int mo
  *   ASYMSPEC_DATA_BAD_MAP in *out_error_word and a map-error word in the
  *   scratch.  Without one, an entry outside its vocabulary is still never
  *   dereferenced (its values read NaN, and ASYMSPEC_DATA_BAD_MAP is set) but
- *   a repeated token is not detected.  Each pair is read through the maps
- *   (one thread per pair and row).  One launch on `stream` (three with a
- *   scratch), nothing allocated.  Host-detectable errors:
+ *   a repeated token is not detected.  a and b are read through map_d (one
+ *   thread per pair and row).  With a scratch, logits_ver 16-byte aligned,
+ *   V_v * element size a multiple of 16 and S * element size at most
+ *   227 KB, t is gathered by a second kernel, one CTA per row, that builds
+ *   the restricted row in shared memory through the inverse map of the
+ *   check, so that a map_v in any order costs no DRAM sector per entry;
+ *   otherwise t too is read through map_v by the first kernel.  One launch
+ *   on `stream` (four with a scratch), nothing allocated.  Host-detectable errors:
  *   ASYMSPEC_ERR_INVALID_ARG (a null pointer, rows < 0, S < 2, V_d < 1,
  *   V_v < 1), ASYMSPEC_ERR_UNSUPPORTED (dtype), ASYMSPEC_ERR_MISALIGNED,
  *   ASYMSPEC_ERR_WORKSPACE (scratch unaligned or too small),
  *   ASYMSPEC_ERR_TOO_LARGE (rows above 524,280).
  *
- * asymspec_fuse_verify_xvocab: map check, gather, step and emission, five
- *   or six launches on `stream` (two for the map check, the gather, the
- *   step's one or two, the emission): logits_full, logits_comp
+ * asymspec_fuse_verify_xvocab: map check, gather, step and emission, up to
+ *   seven launches on `stream` (the gather's four, the step's one or two,
+ *   the emission): logits_full, logits_comp
  *   [B, K+1, V_d]; logits_ver [B, K+1, V_v]; draft_index [B, K] int32 pair indices; draft_probs,
  *   uniforms, gate_params as for asymspec_fuse_verify (draft_probs[b][k] is
  *   the drafter's probability of pair draft_index[b][k] under the restricted

@@ -272,15 +272,16 @@ cudaError_t prepare_kernel(KernelFn fn, int device) {
   return cudaSuccess;
 }
 
-// The decision kernel: dynamic shared memory (walk staging) up to what its
-// static records leave of the per-CTA limit; no clusters.
-cudaError_t prepare_decide(KernelFn fn, int device) {
+// A kernel without clusters whose dynamic shared memory may reach max_bytes
+// (the decision kernel's walk staging: what its static records leave of the
+// per-CTA limit; the gather's restricted row of t).
+cudaError_t prepare_plain_kernel(KernelFn fn, int device, int max_bytes) {
   std::lock_guard<std::mutex> lock(g_mu);
   const void* f = fn;
   for (int i = 0; i < g_attr_count; ++i)
     if (g_attr_done[i].fn == f && g_attr_done[i].device == device) return cudaSuccess;
-  const cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kMaxSmem - kDecideSmemRows * 16);
+  const cudaError_t e =
+      cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, max_bytes);
   if (e != cudaSuccess) return e;
   if (g_attr_count < 64) g_attr_done[g_attr_count++] = {f, device};
   return cudaSuccess;
@@ -660,7 +661,7 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
       warps = std::min(warps, (kMaxSmem - kDecideSmemRows * 16) / P.walk_stage);
     }
     const KernelFn dfn = pick_decide(dtype, stoch);
-    e = prepare_decide(dfn, device);
+    e = prepare_plain_kernel(dfn, device, kMaxSmem - kDecideSmemRows * 16);
     if (e != cudaSuccess) return cuda_fail(e);
     cudaLaunchConfig_t dcfg = {};
     cudaLaunchAttribute dattr[1];
@@ -991,6 +992,9 @@ int asymspec_xvocab_gather(const void* logits_full, const void* logits_comp, int
     if (e != cudaSuccess) return cuda_fail(e);
   }
   XGatherParams P;
+  P.inv_v = scratch ? reinterpret_cast<const int*>(static_cast<char*>(scratch) + XL.inv_v) : nullptr;
+  P.map_err =
+      scratch ? reinterpret_cast<const unsigned*>(static_cast<char*>(scratch) + XL.err) : nullptr;
   P.a = logits_full;
   P.b = logits_comp;
   P.t = logits_ver;
@@ -1007,7 +1011,43 @@ int asymspec_xvocab_gather(const void* logits_full, const void* logits_comp, int
   const dim3 grid(static_cast<unsigned>((S + kXThreads * kXJ - 1) / (kXThreads * kXJ)),
                   static_cast<unsigned>(ycount));
   void* args[] = {&P};
-  e = cudaLaunchKernel(xvocab_gather_ptr(dtype), grid, dim3(kXThreads), args, 0, st);
+  // t built in shared memory through the inverse map (its map may be in any
+  // order) when the caller gave the scratch (where the map check builds the
+  // inverse map), every row of t starts on a 16-byte boundary and a
+  // restricted row fits in one CTA's shared memory; a and b (and otherwise
+  // t) through global memory
+  // (one CTA per row; a restricted row larger than a CTA's shared memory is
+  // cut into parts, each CTA reading the whole row of t for its part)
+  int parts = 1;
+  while (parts < 16 && ((static_cast<size_t>(S) + parts - 1) / parts + 8) * elt >
+                           static_cast<size_t>(kMaxSmem))
+    ++parts;
+  const size_t row_out = ((static_cast<size_t>(S) + parts - 1) / parts + 8) * elt;
+  const bool inv_t = scratch && row_out <= static_cast<size_t>(kMaxSmem) &&
+                     aligned(logits_ver, 16) && (static_cast<size_t>(V_v) * elt) % 16 == 0;
+  e = cudaLaunchKernel(xvocab_gather_ptr(dtype, !inv_t), grid, dim3(kXThreads), args, 0, st);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (inv_t) {
+    const KernelFn fn = xvocab_gather_inv_ptr(dtype);
+    int device = 0;
+    e = cudaGetDevice(&device);
+    if (e == cudaSuccess) e = prepare_plain_kernel(fn, device, kMaxSmem);
+    if (e == cudaSuccess) {
+      // a programmatic dependent of the a/b gather, which it does not read:
+      // the two gathers overlap (the map check before them is complete)
+      cudaLaunchConfig_t cfg = {};
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+      attr[0].val.programmaticStreamSerializationAllowed = 1;
+      cfg.gridDim = dim3(static_cast<unsigned>(rows), static_cast<unsigned>(parts));
+      cfg.blockDim = dim3(kXInvThreads);
+      cfg.dynamicSmemBytes = round_up(row_out, 16);
+      cfg.stream = st;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      e = cudaLaunchKernelExC(&cfg, fn, args);
+    }
+  }
   return e == cudaSuccess ? ASYMSPEC_OK : cuda_fail(e);
 }
 

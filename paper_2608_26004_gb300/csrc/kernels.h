@@ -25,9 +25,10 @@ const void* decide_kernel_bf16(bool stoch);
 const void* decide_kernel_f32(bool stoch);
 // draft_kernel<T, VE, STOCH>, the drafter's draw (k_draft.cu)
 const void* draft_kernel_ptr(int dtype, bool vector_path, bool stoch);
-// the cross-family vocabulary map (k_xvocab.cu): xvocab_gather<T>, xvocab_inv_fill,
-// xvocab_inv_build, xvocab_emit
-const void* xvocab_gather_ptr(int dtype);
+// the cross-family vocabulary map (k_xvocab.cu): xvocab_gather<T, WITH_T>,
+// xvocab_gather_inv<T>, xvocab_inv_fill, xvocab_inv_build, xvocab_emit
+const void* xvocab_gather_ptr(int dtype, bool with_t);
+const void* xvocab_gather_inv_ptr(int dtype);
 const void* xvocab_inv_fill_ptr();
 const void* xvocab_inv_build_ptr();
 const void* xvocab_emit_ptr();

@@ -243,8 +243,8 @@ def test_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):
 
 def test_xvocab_workspace_layout_and_validation(lib):
     # the restricted rows a', b', t' ([B, K+1, S] each), the emitted pair
-    # indices, the gather's scratch (inverse maps and the map-error word),
-    # then the step's workspace for a vocabulary of S entries
+    # indices, the gather's scratch (inverse maps and the map-error word), then
+    # the step's workspace for a vocabulary of S entries
     for B, K, S, V_d, V_v, dtype, elt in ((64, 7, 109568, 151936, 128256, A.BF16, 2),
                                           (3, 2, 37, 50, 41, A.FP32, 4)):
         R = B * (K + 1)
