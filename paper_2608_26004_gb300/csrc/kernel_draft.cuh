@@ -6,7 +6,8 @@
 // One cluster of C CTAs (1 <= C <= 8) per row: CTA c owns the vectors
 // [c W, (c + 1) W) of the row (VE elements each; the last slice may be
 // shorter or empty).  In a slice, vector v0 + r kDThreads + t is handled by
-// thread t in round r, kDUnroll rounds' loads issued before any is used.
+// thread t in round r, kDUnroll rounds' loads issued before any is used (in
+// sampling, the next kDUnroll rounds' too).
 // Each CTA reads its slice once from HBM and pushes a summary (reference,
 // mass relative to it, finiteness sum, argmax index) into every CTA of the
 // cluster; after one cluster barrier every CTA combines the C summaries
@@ -291,35 +292,45 @@ __device__ __forceinline__ DSlice slice_greedy(const T* a, int v0, int v1, DShar
 
 // -------------------------------------------------------------- sampling slice
 
+// Loads of rounds [r, r + kDUnroll) of the slice (vectors past v1 skipped).
+template <typename T, int VE>
+__device__ __forceinline__ void dld_batch(const T* a, int v0, int v1, int r,
+                                          DRaw<T, VE> (&raw)[kDUnroll]) {
+#pragma unroll
+  for (int u = 0; u < kDUnroll; ++u) {
+    const int v = v0 + (r + u) * kDThreads + threadIdx.x;
+    if (v < v1) dld(a, v, raw[u]);
+  }
+}
+
 // Group masses of the slice against the warp reference `ref`: gm[r kDWarps +
 // warp] = the mass of vectors v0 + r kDThreads + warp 32 + [0, 32), summed
-// kDUnroll rounds at a time.  Adds the thread's share to tot (and, when FIN,
-// its finiteness sum to fin); returns true if a group's mass reached kDGuard
-// (or is not a number).
+// kDUnroll rounds at a time.  `cur` holds the first batch's loads (rounds
+// 0 .. kDUnroll - 1); each next batch is loaded before the current one is
+// used, so a slice of two batches costs one memory round trip.  Adds the
+// thread's share to tot (and, when FIN, its finiteness sum to fin); returns
+// true if a group's mass reached kDGuard (or is not a number).
 template <typename T, int VE, bool FIN>
 __device__ __forceinline__ bool slice_masses(const T* a, int v0, int v1, float ref, float* gm,
-                                             float& tot, DFin<T, VE>& fin) {
+                                             float& tot, DFin<T, VE>& fin,
+                                             DRaw<T, VE> (&cur)[kDUnroll]) {
   static_assert(kDUnroll == 4, "dwarp_sum4 sums four rounds");
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int rounds = (v1 - v0 + kDThreads - 1) / kDThreads;
   const float nm2 = -ref * kLog2e;
   bool over = false;
   for (int r = 0; r < rounds; r += kDUnroll) {
-    DRaw<T, VE> raw[kDUnroll];
-#pragma unroll
-    for (int u = 0; u < kDUnroll; ++u) {
-      const int v = v0 + (r + u) * kDThreads + tid;
-      if (v < v1) dld(a, v, raw[u]);  // v < v1 implies r + u < rounds
-    }
+    DRaw<T, VE> nxt[kDUnroll];
+    if (r + kDUnroll < rounds) dld_batch<T, VE>(a, v0, v1, r + kDUnroll, nxt);
     float mv[kDUnroll];
 #pragma unroll
     for (int u = 0; u < kDUnroll; ++u) {
       mv[u] = 0.f;
-      if (v0 + (r + u) * kDThreads + tid < v1) {
+      if (v0 + (r + u) * kDThreads + tid < v1) {  // implies r + u < rounds
         float x[VE];
-        dwiden(raw[u], x);
+        dwiden(cur[u], x);
         mv[u] = dmass(x, nm2);
-        if (FIN) fin.add(raw[u]);
+        if (FIN) fin.add(cur[u]);
       }
       tot += mv[u];
     }
@@ -327,6 +338,8 @@ __device__ __forceinline__ bool slice_masses(const T* a, int v0, int v1, float r
     over |= !(g < kDGuard);
     const int q = lane >> 3;  // lanes 0, 8, 16, 24 hold rounds r .. r + 3
     if ((lane & 7) == 0 && r + q < rounds) gm[(r + q) * kDWarps + warp] = g;
+#pragma unroll
+    for (int u = 0; u < kDUnroll; ++u) cur[u] = nxt[u];
   }
   return over;
 }
@@ -334,23 +347,23 @@ __device__ __forceinline__ bool slice_masses(const T* a, int v0, int v1, float r
 template <typename T, int VE>
 __device__ __forceinline__ DSlice slice_sample(const T* a, int v0, int v1, float* gm, DShared& sh) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // the warp reference: the maximum of the warp's first-round vectors (-inf if none)
+  // the first batch of rounds; the warp reference: the maximum of the
+  // warp's first-round vectors (-inf if none)
+  DRaw<T, VE> first[kDUnroll];
+  dld_batch<T, VE>(a, v0, v1, 0, first);
   float ref;
   {
-    const int v = v0 + tid;
     float r0 = -INFINITY;
-    if (v < v1) {
-      DRaw<T, VE> raw;
-      dld(a, v, raw);
+    if (v0 + tid < v1) {
       float x[VE];
-      dwiden(raw, x);
+      dwiden(first[0], x);
       r0 = dvmax(x);
     }
     ref = dwarp_max(r0);
   }
   float tot = 0.f;
   DFin<T, VE> fin;
-  const bool over = slice_masses<T, VE, true>(a, v0, v1, ref, gm, tot, fin);
+  const bool over = slice_masses<T, VE, true>(a, v0, v1, ref, gm, tot, fin, first);
   if (__syncthreads_or(over)) {
     // an entry far above its warp's reference: the exact slice maximum, then
     // every group again against it
@@ -372,7 +385,8 @@ __device__ __forceinline__ DSlice slice_sample(const T* a, int v0, int v1, float
     ref = dwarp_max(lane < kDWarps ? sh.red[lane] : -INFINITY);
     tot = 0.f;
     DFin<T, VE> unused;
-    slice_masses<T, VE, false>(a, v0, v1, ref, gm, tot, unused);
+    dld_batch<T, VE>(a, v0, v1, 0, first);
+    slice_masses<T, VE, false>(a, v0, v1, ref, gm, tot, unused, first);
     __syncthreads();  // every warp has read sh.red
   }
   const float wt = dwarp_sum(tot), wf = dwarp_sum(fin.value());
