@@ -1,4 +1,6 @@
-// Fast fuse-and-verify kernel for 16-byte aligned rows.
+// Staged fuse-and-verify kernel for 16-byte aligned rows (every program
+// but the production stochastic JSD step, which fuse_verify_row in
+// kernel_row.cuh runs), and the decision kernel both row kernels feed.
 //
 // One cluster of C CTAs per row triple (one launch of the cluster per row;
 // the hardware hands out rows as clusters finish).  CTA r owns vocabulary
@@ -21,20 +23,21 @@
 // (f32x2); exponentials and logarithms use ex2.approx / lg2.approx.
 //
 // Normalisers: each thread sums 2^((x - ref) log2 e) against one fixed
-// reference per stream, the maximum of its first vector, so an entry costs
-// one FMA, one ex2 and one add; partial sums are rescaled only where they
-// meet (warp, CTA, cluster).  A thread whose sum reaches 2^100 (an entry
-// more than ~69 nats above its reference, or non-finite data) makes the CTA
-// redo its slice with a running maximum (pass1_online).
+// reference per stream and warp (the warp's largest of its threads' first
+// two entries), so an entry costs one FMA, one ex2 and one add; the warps'
+// references meet only in the reductions.  A thread whose sum reaches 2^100
+// (an entry more than ~69 nats above its reference, or non-finite data)
+// makes the CTA redo its slice with a running maximum (pass1_online).
 //
 // Reductions: warp maxima with redux.sync, sums with shuffles; warp -> CTA in
-// shared memory.  Each CTA pushes its record into every peer's shared memory
-// (DSMEM stores) before a cluster barrier, so after the barrier every CTA
-// combines local copies, identically.  Two cluster barriers per row (one
-// when no pass 2 is needed).  Once the last barrier has passed, only the
-// warp that finishes the row stays: warp 0 of rank 0 (greedy), or warp 0 of
-// the CTA whose slice holds the inverse-CDF target (stochastic), which walks
-// its slice and then decides the row itself.
+// shared memory.  Each CTA pushes its pass-1 record into every peer's shared
+// memory (DSMEM stores) before one cluster barrier, so after the barrier
+// every CTA combines local copies, identically.  After pass 2 each CTA
+// stores its row statistics (rank 0), its pass-2 record and its inverse-CDF
+// group masses in the workspace and exits; decide_rows (below), a second
+// launch with one CTA per batch element, decides every row from those
+// records (the divergence, the walk to the drawn element, the acceptance
+// test) and runs Algorithm 1's scan.
 //
 // Every wait is bounded: a chunk that does not land within 200 ms marks the
 // row with ASYMSPEC_DATA_TIMEOUT; the CTA still reaches every cluster
