@@ -130,8 +130,8 @@ bool plan_row(int V, int dtype, int forced_C, Plan* pl) {
     if (W / VE > static_cast<long long>(kMaxRounds) * kRowThreads) continue;
     pl->C = C;
     pl->W = static_cast<int>(W);
-    pl->sh_off = 0;
-    pl->smem = row_shared_bytes(C);
+    pl->sh_off = row_shared_bytes(C);  // the warps' rings follow the fixed state
+    pl->smem = row_shared_bytes(C) + kRingBytes;
     pl->group_stride = kGroupsMax;
     pl->nt = kRowThreads;
     return true;

@@ -7,4 +7,5 @@ namespace asymspec_impl {
 
 const void* row_kernel_bf16() { return reinterpret_cast<const void*>(&fuse_verify_row<__nv_bfloat16>); }
 
+
 }  // namespace asymspec_impl

@@ -7,4 +7,5 @@ namespace asymspec_impl {
 
 const void* row_kernel_f32() { return reinterpret_cast<const void*>(&fuse_verify_row<float>); }
 
+
 }  // namespace asymspec_impl

@@ -12,25 +12,24 @@
 // What differs from fuse_verify_tma is where the slice lives between the
 // passes and the shape of the work:
 //   * no slice is held in shared memory.  Each warp owns a contiguous block
-//     of the slice; its lane 0 starts with a bulk prefetch of the block's
-//     three streams into the L2, pass 1 reads the block from global memory
-//     (16-byte loads, 32 consecutive vectors per warp and step) and pass 2
-//     reads it again, which the L2 serves.  The rows in flight at once (one
-//     per resident cluster: 74 clusters of 8 CTAs on GB300, 57 MB for
-//     V = 128256 bf16) sit well inside the 129 MB L2, so each logit row
-//     still comes from HBM once.  With only the pass-1 records in shared
-//     memory, four 256-thread CTAs fit on an SM (the register file is the
-//     limit), against three when the slice is staged in shared memory; the
-//     extra warps hide the load latency and the cluster barrier, which is
-//     what bounds this kernel (about 1 warp instruction per vocabulary entry
-//     against 6 bytes read);
+//     of the slice and reads it twice through a small ring in shared memory
+//     (kRing steps of 32 consecutive 16-byte vectors per stream, filled with
+//     cp.async): pass 1 from HBM, pass 2 from the L2, where pass 1 just
+//     brought it.  The rows in flight at once (one per resident cluster: 74
+//     clusters of 8 CTAs on GB300, 57 MB for V = 128256 bf16) sit well inside
+//     the 129 MB L2, so each logit row still comes from HBM once.  With 48 KB
+//     of rings and the pass-1 records in shared memory, four 256-thread CTAs
+//     fit on an SM (the register file is the limit), against three when the
+//     slice is staged whole; the ring keeps four steps of every warp in
+//     flight without holding registers, and pass 2's first steps are issued
+//     before the cluster barrier;
 //   * the block of a warp is one inverse-CDF group: its mass is the warp's
 //     residual (or fused) sum, which the warp reduces anyway, so pass 2 needs
 //     no per-step group reductions (the decision kernel walks the group's
 //     vectors);
 //   * one 16-byte vector per stream per step, unpacked pair by pair from the
 //     raw words (bf16 -> fp32 is a shift or a mask), two fp32 lanes per
-//     add/sub/mul/fma instruction, two steps of loads in flight per warp;
+//     add/sub/mul/fma instruction;
 //   * the divergence of Eq. 3 in one product per pair.  With p = softmax(a),
 //     q = softmax(b) in log2 units, e = q/p = 2^d (d = log2 q - log2 p) and
 //     w = 1 + e, each entry contributes to 2 JSD (in bits)
@@ -40,8 +39,9 @@
 //     are formed exactly as the decision kernel's inverse-CDF walk forms
 //     them (res_pair), so the group masses and the walk agree bit for bit.
 //
-// The kernel waits on nothing but the hardware cluster barrier (no copies
-// complete on mbarriers), so it never reports ASYMSPEC_DATA_TIMEOUT.
+// The kernel waits on nothing but the hardware cluster barrier, CTA
+// barriers and its own cp.async groups (no copies complete on mbarriers), so
+// it never reports ASYMSPEC_DATA_TIMEOUT.
 #pragma once
 
 #include "kernel_tma.cuh"
@@ -144,35 +144,89 @@ __host__ __device__ constexpr int row_shared_bytes(int C) {
   return static_cast<int>(sizeof(RowShared) + C * sizeof(X1));
 }
 
+// ---------------------------------------------------------------- the rings
+
+// Each warp reads its block through a ring of kRing steps in shared memory:
+// lane l copies its vector of the three streams for a step into the step's
+// slot with 16-byte cp.async (one commit group per step) and later reads
+// back only what it copied itself, so no barrier is needed; kRing steps of
+// every warp are in flight without holding registers.
+constexpr int kRing = 4;
+constexpr int kRingBytes = (kRowThreads / 32) * kRing * 3 * 32 * 16;  // per CTA (48 KB)
+
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Lane's vector i of the three streams into ring slot `slot` (one commit
+// group per step, committed by the caller).
+template <typename T>
+__device__ __forceinline__ void ring_issue(uint4* ring, int slot, const T* ga, const T* gb,
+                                           const T* gt, int i) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
+  uint4* d = ring + slot * 96 + (threadIdx.x & 31);
+  cp_async16(d, ga + i * VE);
+  cp_async16(d + 32, gb + i * VE);
+  cp_async16(d + 64, gt + i * VE);
+}
+template <typename T>
+__device__ __forceinline__ void ring_read(const uint4* ring, int slot, RawVec<T>& va,
+                                          RawVec<T>& vb, RawVec<T>& vt) {
+  using V = decltype(va.v);
+  const V* d = reinterpret_cast<const V*>(ring + slot * 96 + (threadIdx.x & 31));
+  va.v = d[0];
+  vb.v = d[32];
+  vt.v = d[64];
+}
+// Before step r (r >= 1) reads its slot: step r + kRing - 1 into the slot
+// step r - 1 used.  That slot's values were consumed by instructions this
+// thread has already issued, so the copy cannot overwrite unread data.
+template <typename T>
+__device__ __forceinline__ void ring_refill(uint4* ring, const T* ga, const T* gb, const T* gt,
+                                            int i0, int v1, int R, int r) {
+  const int q = r + kRing - 1;
+  const int i = i0 + 32 * q;
+  if (q < R && i < v1) ring_issue<T>(ring, (r - 1) & (kRing - 1), ga, gb, gt, i);
+  cp_async_commit();
+}
+// The first kRing steps of a pass into the ring (one group each, empty past R).
+template <typename T>
+__device__ __forceinline__ void ring_prologue(uint4* ring, const T* ga, const T* gb, const T* gt,
+                                              int v0, int v1, int R) {
+  const int i0 = v0 + static_cast<int>(threadIdx.x & 31);
+#pragma unroll
+  for (int q = 0; q < kRing; ++q) {
+    const int i = i0 + 32 * q;
+    if (q < R && i < v1) ring_issue<T>(ring, q, ga, gb, gt, i);
+    cp_async_commit();
+  }
+}
+
 // ---------------------------------------------------------------- pass 1
 
 // Pass 1 over the warp's block [v0, v1) of the slice (ga, gb, gt: the
-// slice's first entries in global memory; R steps), with one fixed reference
+// slice's first entries in global memory; R steps), its vectors read through
+// the warp's ring (the caller issued the prologue), with one fixed reference
 // per warp and stream: the largest of the first pairs of the lanes' first
 // vectors.  DRAFT: the normalisers of a, b and the fused score s; the bonus
 // row needs s only.  Returns true when a lane's sum reached 2^100 or is not
 // finite (the CTA then redoes its slice with a running maximum).  Every lane
 // ends with the warp's record.
 template <typename T, bool DRAFT>
-__device__ __forceinline__ bool row_pass1(const T* ga, const T* gb, const T* gt, int v0, int v1,
-                                          int R, float beta, W1& e) {
+__device__ __forceinline__ bool row_pass1(uint4* ring, const T* ga, const T* gb, const T* gt,
+                                           int v0, int v1, int R, float beta, W1& e) {
   constexpr int NP = RawVec<T>::NP;
-  constexpr int VE = 2 * NP;
   const int lane = static_cast<int>(threadIdx.x & 31);
   const f2 L2 = pk(kLog2e, kLog2e);
   const float bl = beta * kLog2e;
   const f2 bL2 = pk(bl, bl);
   const int i0 = v0 + lane;
-  const bool have0 = i0 < v1;
-  RawVec<T> va0 = {}, vb0 = {}, vt0 = {};
-  if (have0) {
-    va0 = raw_ldg(ga + i0 * VE);
-    vb0 = raw_ldg(gb + i0 * VE);
-    vt0 = raw_ldg(gt + i0 * VE);
-  }
   float ra0 = -INFINITY, rb0 = -INFINITY, rs0 = -INFINITY;
-  if (have0) {
-    const f2 a2 = va0.pair(0), b2 = vb0.pair(0), t2 = vt0.pair(0);
+  cp_async_wait<kRing - 1>();  // step 0 (this lane's own copies)
+  RawVec<T> va, vb, vt;
+  if (i0 < v1) {
+    ring_read<T>(ring, 0, va, vb, vt);
+    const f2 a2 = va.pair(0), b2 = vb.pair(0), t2 = vt.pair(0);
     const f2 s2 = fma2(pk(beta, beta), sub2(a2, b2), t2);
     ra0 = fmaxf(lo_of(a2), hi_of(a2));
     rb0 = fmaxf(lo_of(b2), hi_of(b2));
@@ -186,26 +240,27 @@ __device__ __forceinline__ bool row_pass1(const T* ga, const T* gb, const T* gt,
   const float nA = -ra0 * kLog2e, nB = -rb0 * kLog2e, nS = -rs0 * kLog2e;
   const f2 nA2 = pk(nA, nA), nB2 = pk(nB, nB), nS2 = pk(nS, nS);
   f2 acc_a = 0ull, acc_b = 0ull, acc_s = 0ull;
-  auto body = [&](const RawVec<T>& va, const RawVec<T>& vb, const RawVec<T>& vt) {
-#pragma unroll
-    for (int h = 0; h < NP; ++h) {
-      const f2 a2 = va.pair(h), b2 = vb.pair(h), t2 = vt.pair(h);
-      if (DRAFT) {
-        acc_a = add2(acc_a, ex2_2(fma2(a2, L2, nA2)));
-        acc_b = add2(acc_b, ex2_2(fma2(b2, L2, nB2)));
-      }
-      acc_s = add2(acc_s, ex2_2(fma2(t2, L2, fma2(bL2, sub2(a2, b2), nS2))));
-    }
-  };
-  if (have0) body(va0, vb0, vt0);
-#pragma unroll 2
-  for (int r = 1; r < R; ++r) {
+  for (int r = 0; r < R; ++r) {
     const int i = i0 + 32 * r;
-    if (i < v1) body(raw_ldg(ga + i * VE), raw_ldg(gb + i * VE), raw_ldg(gt + i * VE));
+    if (r > 0) {
+      ring_refill<T>(ring, ga, gb, gt, i0, v1, R, r);
+      cp_async_wait<kRing - 1>();
+    }
+    if (i < v1) {
+      if (r > 0) ring_read<T>(ring, r & (kRing - 1), va, vb, vt);
+#pragma unroll
+      for (int h = 0; h < NP; ++h) {
+        const f2 a2 = va.pair(h), b2 = vb.pair(h), t2 = vt.pair(h);
+        if (DRAFT) {
+          acc_a = add2(acc_a, ex2_2(fma2(a2, L2, nA2)));
+          acc_b = add2(acc_b, ex2_2(fma2(b2, L2, nB2)));
+        }
+        acc_s = add2(acc_s, ex2_2(fma2(t2, L2, fma2(bL2, sub2(a2, b2), nS2))));
+      }
+    }
   }
   float sa = DRAFT ? hsum2(acc_a) : 0.f, sb = DRAFT ? hsum2(acc_b) : 0.f, ss = hsum2(acc_s);
   const bool ovf = !(ss < kSumLimit) || (DRAFT && (!(sa < kSumLimit) || !(sb < kSumLimit)));
-  // the warp's sums (its references are equal across lanes)
   float z = 0.f;
   warp_sum4(sa, sb, ss, z);
   e.ref[0] = ra0;
@@ -271,35 +326,38 @@ __device__ __forceinline__ void row_pass1_online(const T* ga, const T* gb, const
 
 // ---------------------------------------------------------------- pass 2
 
-// Pass 2 over the warp's block (from the L2, where pass 1 left it): DRAFT,
-// the JSD terms (see the header) and the residual masses; the bonus row, the
-// fused masses.  Returns through jsum / msum the warp's sums (every lane
-// ends with them): msum is the mass of the warp's inverse-CDF group.
+// Pass 2 over the warp's block (from the L2, where pass 1 left it), through
+// the warp's ring (the caller issued the prologue): DRAFT, the JSD terms
+// (see the header) and the residual masses; the bonus row, the fused
+// masses.  Returns through jsum / msum the warp's sums (every lane ends with
+// them): msum is the mass of the warp's inverse-CDF group.
 template <typename T, bool DRAFT>
-__device__ __forceinline__ void row_pass2(const T* ga, const T* gb, const T* gt, int v0, int v1,
-                                          int R, const ResConst& k, float& jsum, float& msum) {
+__device__ __forceinline__ void row_pass2(uint4* ring, const T* ga, const T* gb, const T* gt,
+                                           int v0, int v1, int R, const ResConst& k, float& jsum,
+                                           float& msum) {
   constexpr int NP = RawVec<T>::NP;
-  constexpr int VE = 2 * NP;
   const int lane = static_cast<int>(threadIdx.x & 31);
   f2 jacc = 0ull, macc = 0ull;
   const int i0 = v0 + lane;
-  auto body = [&](const RawVec<T>& va, const RawVec<T>& vb, const RawVec<T>& vt) {
-#pragma unroll
-    for (int h = 0; h < NP; ++h) {
-      f2 amb, p, qf, rr;
-      res_pair(va.pair(h), vb.pair(h), vt.pair(h), k, amb, p, qf, rr);
-      if (DRAFT) {
-        macc = add2(macc, rr);
-        jacc = jsd_pair(amb, p, k, jacc);
-      } else {
-        macc = add2(macc, qf);
-      }
-    }
-  };
-#pragma unroll 2
   for (int r = 0; r < R; ++r) {
     const int i = i0 + 32 * r;
-    if (i < v1) body(raw_ldg(ga + i * VE), raw_ldg(gb + i * VE), raw_ldg(gt + i * VE));
+    if (r > 0) ring_refill<T>(ring, ga, gb, gt, i0, v1, R, r);
+    cp_async_wait<kRing - 1>();
+    if (i < v1) {
+      RawVec<T> va, vb, vt;
+      ring_read<T>(ring, r & (kRing - 1), va, vb, vt);
+#pragma unroll
+      for (int h = 0; h < NP; ++h) {
+        f2 amb, p, qf, rr;
+        res_pair(va.pair(h), vb.pair(h), vt.pair(h), k, amb, p, qf, rr);
+        if (DRAFT) {
+          macc = add2(macc, rr);
+          jacc = jsd_pair(amb, p, k, jacc);
+        } else {
+          macc = add2(macc, qf);
+        }
+      }
+    }
   }
   float j = hsum2(jacc), m = hsum2(macc), z0 = 0.f, z1 = 0.f;
   warp_sum4(j, m, z0, z1);
@@ -326,12 +384,12 @@ __device__ __forceinline__ unsigned cluster_id_y() {
 // decision kernel: rank 0's row statistics (the normalisers, data-error
 // bits) and one pass-2 record per warp of every CTA (KParams::pass2_rec,
 // kRowMaxWarps records per CTA): the warp's JSD sum, the residual and fused
-// masses of its block (its inverse-CDF group).
+// masses of its block (its inverse-CDF group).  Dynamic shared memory: the
+// fixed state and pushed records (row_shared_bytes(C)), then the warps'
+// rings (kRingBytes) at KParams::sh_off.  Pass 2's first kRing steps are
+// issued before the cluster barrier: they do not depend on the normalisers.
 template <typename T>
 __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(const KParams P) {
-  // the decision kernel (a programmatic dependent) may be scheduled once
-  // every CTA of this grid has started; it waits for this grid's completion
-  // before it reads anything the grid writes
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   constexpr int NW = kRowThreads / 32;
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
@@ -350,7 +408,6 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
   const int lo = rank * W;
   const int n = max(0, min(W, P.V - lo));
   const int nv = n / VE;
-  // this warp's block of the slice (vectors) and its steps
   const int bw = row_block_vectors(nv, NW);
   const int v0 = min(nv, warp * bw), v1 = min(nv, v0 + bw);
   const int R = (v1 - v0 + 31) / 32;
@@ -359,21 +416,17 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
   const T* gb = static_cast<const T*>(P.b) + off;
   const T* gt = static_cast<const T*>(P.t) + off;
   RowShared* sh = reinterpret_cast<RowShared*>(smem_row);
+  uint4* ring = reinterpret_cast<uint4*>(smem_row + P.sh_off) + warp * (kRing * 96);
   const bool draft = k < P.K;
-
-  // the warp's block of the three rows into the L2 (16-byte aligned: the
-  // host takes this kernel only for rows of a multiple of 16 bytes)
-  if (lane == 0 && v1 > v0) {
-    const unsigned bytes = static_cast<unsigned>(v1 - v0) * 16u;
-    bulk_prefetch_l2(ga + v0 * VE, bytes);
-    bulk_prefetch_l2(gb + v0 * VE, bytes);
-    bulk_prefetch_l2(gt + v0 * VE, bytes);
-  }
+  ring_prologue<T>(ring, ga, gb, gt, v0, v1, R);
 
   // ---- pass 1: the row normalisers, combined over the cluster
   W1 e;
-  const bool ovf = draft ? row_pass1<T, true>(ga, gb, gt, v0, v1, R, P.beta, e)
-                         : row_pass1<T, false>(ga, gb, gt, v0, v1, R, P.beta, e);
+  const bool ovf = draft ? row_pass1<T, true>(ring, ga, gb, gt, v0, v1, R, P.beta, e)
+                         : row_pass1<T, false>(ring, ga, gb, gt, v0, v1, R, P.beta, e);
+  cp_async_wait<0>();  // the pass's trailing (empty) groups; the ring is free
+  // pass 2's first steps do not depend on the normalisers
+  ring_prologue<T>(ring, ga, gb, gt, v0, v1, R);
   if (lane == 0) sh->w1[warp] = e;
   if (__syncthreads_or(ovf)) {
     // an entry far above its warp's reference (or non-finite data): redo the
@@ -403,7 +456,6 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
     push_record(x, sh->recv(), rank, C, cluster);
   }
   cluster_barrier(warp == 0);  // every CTA's pass-1 record is in every CTA
-
   if (warp == 0) {
     X1 x = (lane < C) ? sh->recv()[lane] : x1_neutral();
     if (draft) warp_reduce_x1<FD>(x);
@@ -426,8 +478,9 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
   const float A2 = sh->lse[0] * kLog2e, B2 = sh->lse[1] * kLog2e, S2 = sh->lse[3] * kLog2e;
   const ResConst kc = res_const(P.beta, A2, B2, S2);
   float jsum, msum;
-  if (draft) row_pass2<T, true>(ga, gb, gt, v0, v1, R, kc, jsum, msum);
-  else row_pass2<T, false>(ga, gb, gt, v0, v1, R, kc, jsum, msum);
+  if (draft) row_pass2<T, true>(ring, ga, gb, gt, v0, v1, R, kc, jsum, msum);
+  else row_pass2<T, false>(ring, ga, gb, gt, v0, v1, R, kc, jsum, msum);
+  cp_async_wait<0>();
   if (lane == 0) {
     // this warp's record: its block is one inverse-CDF group of the row.  A
     // draft row's fused mass (the draw's fallback when the row's whole

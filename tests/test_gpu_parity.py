@@ -470,7 +470,8 @@ def test_row_kernel_is_the_production_choice(torch):
                               (256, 4, 151936, A.FP32, 16), (1, 4, 32000, A.FP32, 8)):
         info = A.plan(B, K, V, dtype, A.gate_params(mode=STOCH))
         assert info.kernel == A.KERNEL_TMA and info.row_kernel == 1 and info.launches == 2
-        # 256-thread CTAs with only the cluster's pass-1 records in shared memory
+        # 256-thread CTAs, four to an SM: the warps' 48 KB of load rings and the
+        # cluster's pass-1 records in shared memory, no slice
         assert info.block_threads == 256 and info.cluster_size == C
-        assert info.smem_bytes <= 2048
+        assert 4 * (info.smem_bytes + 1024) <= 228 * 1024
         assert info.max_active_clusters > 0
