@@ -179,14 +179,21 @@ __device__ __forceinline__ void ring_read(const uint4* ring, int slot, RawVec<T>
   vt.v = d[64];
 }
 // Before step r (r >= 1) reads its slot: step r + kRing - 1 into the slot
-// step r - 1 used.  That slot's values were consumed by instructions this
-// thread has already issued, so the copy cannot overwrite unread data.
+// step r - 1 used (slot `slot`, a constant once the loops are unrolled).  That slot's values were consumed by instructions this thread has
+// already issued, so the copy cannot overwrite unread data.  pa, pb, pt: the
+// lane's vector of step 0 of each stream.
 template <typename T>
-__device__ __forceinline__ void ring_refill(uint4* ring, const T* ga, const T* gb, const T* gt,
-                                            int i0, int v1, int R, int r) {
+__device__ __forceinline__ void ring_refill(uint4* ring, int slot, const T* pa, const T* pb,
+                                            const T* pt, int i0, int v1, int r) {
+  constexpr int VE = 16 / static_cast<int>(sizeof(T));
   const int q = r + kRing - 1;
-  const int i = i0 + 32 * q;
-  if (q < R && i < v1) ring_issue<T>(ring, (r - 1) & (kRing - 1), ga, gb, gt, i);
+  if (i0 + 32 * q < v1) {
+    uint4* d = ring + slot * 96 + (threadIdx.x & 31);
+    const size_t o = static_cast<size_t>(q) * 32 * VE;
+    cp_async16(d, pa + o);
+    cp_async16(d + 32, pb + o);
+    cp_async16(d + 64, pt + o);
+  }
   cp_async_commit();
 }
 // The first kRing steps of a pass into the ring (one group each, empty past R).
@@ -240,22 +247,31 @@ __device__ __forceinline__ bool row_pass1(uint4* ring, const T* ga, const T* gb,
   const float nA = -ra0 * kLog2e, nB = -rb0 * kLog2e, nS = -rs0 * kLog2e;
   const f2 nA2 = pk(nA, nA), nB2 = pk(nB, nB), nS2 = pk(nS, nS);
   f2 acc_a = 0ull, acc_b = 0ull, acc_s = 0ull;
-  for (int r = 0; r < R; ++r) {
-    const int i = i0 + 32 * r;
-    if (r > 0) {
-      ring_refill<T>(ring, ga, gb, gt, i0, v1, R, r);
-      cp_async_wait<kRing - 1>();
-    }
-    if (i < v1) {
-      if (r > 0) ring_read<T>(ring, r & (kRing - 1), va, vb, vt);
+  constexpr int VE = 2 * NP;
+  const T* pa = ga + static_cast<size_t>(i0) * VE;
+  const T* pb = gb + static_cast<size_t>(i0) * VE;
+  const T* pt = gt + static_cast<size_t>(i0) * VE;
+  // unrolled by the ring's depth, so that every slot is a constant
+  for (int r0 = 0; r0 < R; r0 += kRing) {
 #pragma unroll
-      for (int h = 0; h < NP; ++h) {
-        const f2 a2 = va.pair(h), b2 = vb.pair(h), t2 = vt.pair(h);
-        if (DRAFT) {
-          acc_a = add2(acc_a, ex2_2(fma2(a2, L2, nA2)));
-          acc_b = add2(acc_b, ex2_2(fma2(b2, L2, nB2)));
+    for (int u = 0; u < kRing; ++u) {
+      const int r = r0 + u;
+      if (r >= R) break;
+      if (r > 0) {
+        ring_refill<T>(ring, (u + kRing - 1) % kRing, pa, pb, pt, i0, v1, r);
+        cp_async_wait<kRing - 1>();
+      }
+      if (i0 + 32 * r < v1) {
+        if (r > 0) ring_read<T>(ring, u, va, vb, vt);
+#pragma unroll
+        for (int h = 0; h < NP; ++h) {
+          const f2 a2 = va.pair(h), b2 = vb.pair(h), t2 = vt.pair(h);
+          if (DRAFT) {
+            acc_a = add2(acc_a, ex2_2(fma2(a2, L2, nA2)));
+            acc_b = add2(acc_b, ex2_2(fma2(b2, L2, nB2)));
+          }
+          acc_s = add2(acc_s, ex2_2(fma2(t2, L2, fma2(bL2, sub2(a2, b2), nS2))));
         }
-        acc_s = add2(acc_s, ex2_2(fma2(t2, L2, fma2(bL2, sub2(a2, b2), nS2))));
       }
     }
   }
@@ -339,22 +355,30 @@ __device__ __forceinline__ void row_pass2(uint4* ring, const T* ga, const T* gb,
   const int lane = static_cast<int>(threadIdx.x & 31);
   f2 jacc = 0ull, macc = 0ull;
   const int i0 = v0 + lane;
-  for (int r = 0; r < R; ++r) {
-    const int i = i0 + 32 * r;
-    if (r > 0) ring_refill<T>(ring, ga, gb, gt, i0, v1, R, r);
-    cp_async_wait<kRing - 1>();
-    if (i < v1) {
-      RawVec<T> va, vb, vt;
-      ring_read<T>(ring, r & (kRing - 1), va, vb, vt);
+  constexpr int VE = 2 * NP;
+  const T* pa = ga + static_cast<size_t>(i0) * VE;
+  const T* pb = gb + static_cast<size_t>(i0) * VE;
+  const T* pt = gt + static_cast<size_t>(i0) * VE;
+  for (int r0 = 0; r0 < R; r0 += kRing) {
 #pragma unroll
-      for (int h = 0; h < NP; ++h) {
-        f2 amb, p, qf, rr;
-        res_pair(va.pair(h), vb.pair(h), vt.pair(h), k, amb, p, qf, rr);
-        if (DRAFT) {
-          macc = add2(macc, rr);
-          jacc = jsd_pair(amb, p, k, jacc);
-        } else {
-          macc = add2(macc, qf);
+    for (int u = 0; u < kRing; ++u) {
+      const int r = r0 + u;
+      if (r >= R) break;
+      if (r > 0) ring_refill<T>(ring, (u + kRing - 1) % kRing, pa, pb, pt, i0, v1, r);
+      cp_async_wait<kRing - 1>();
+      if (i0 + 32 * r < v1) {
+        RawVec<T> va, vb, vt;
+        ring_read<T>(ring, u, va, vb, vt);
+#pragma unroll
+        for (int h = 0; h < NP; ++h) {
+          f2 amb, p, qf, rr;
+          res_pair(va.pair(h), vb.pair(h), vt.pair(h), k, amb, p, qf, rr);
+          if (DRAFT) {
+            macc = add2(macc, rr);
+            jacc = jsd_pair(amb, p, k, jacc);
+          } else {
+            macc = add2(macc, qf);
+          }
         }
       }
     }
