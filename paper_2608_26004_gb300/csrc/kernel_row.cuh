@@ -135,6 +135,8 @@ struct __align__(16) W1 {
 struct __align__(16) RowShared {
   W1 w1[kRowMaxWarps];  // per-warp pass-1 records
   float lse[4];         // the row's normalisers (a, b, -, s)
+  unsigned long long xbar;  // completes when the cluster's C records have landed
+  unsigned long long pad2;
   __device__ X1* recv() { return reinterpret_cast<X1*>(this + 1); }
 };
 static_assert(sizeof(W1) == 32, "one warp record is two 16-byte words");
@@ -391,6 +393,43 @@ __device__ __forceinline__ void row_pass2(uint4* ring, const T* ga, const T* gb,
 
 // ---------------------------------------------------------------- the kernel
 
+// 16 bytes into CTA `rank`'s copy of the shared variable at `local`,
+// completing 16 bytes of the transaction count of that CTA's copy of `bar`.
+__device__ __forceinline__ void st_async16(const void* local, unsigned rank,
+                                           unsigned long long* bar, float4 v) {
+  unsigned ra, rb;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(rb) : "r"(smem_u32(bar)), "r"(rank));
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(ra),
+      "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rb)
+      : "memory");
+}
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+}
+// The record combine of warp_reduce_x1 over lanes 0-7 only (the others hold
+// the neutral record): three butterfly levels.
+template <unsigned F>
+__device__ __forceinline__ void warp_reduce_x1_8(X1& e) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const unsigned bit = q == 0 ? F_LA : q == 1 ? F_LB : q == 2 ? F_LT : F_LS;
+    if (F & bit) {
+      const float M = warp_max(e.ref[q]);
+      float s = (e.s[q] == 0.f || e.ref[q] == M) ? e.s[q] : e.s[q] * ex2((e.ref[q] - M) * kLog2e);
+#pragma unroll
+      for (int off = 4; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+      e.ref[q] = M;
+      e.s[q] = s;
+    }
+  }
+  e.bad = __reduce_or_sync(0xffffffffu, e.bad);
+}
+
 // The cluster's index in the grid: (row k of batch element bi) = (x, y).
 __device__ __forceinline__ unsigned cluster_id_x() {
   unsigned r;
@@ -442,6 +481,13 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
   RowShared* sh = reinterpret_cast<RowShared*>(smem_row);
   uint4* ring = reinterpret_cast<uint4*>(smem_row + P.sh_off) + warp * (kRing * 96);
   const bool draft = k < P.K;
+  const bool m3 = C <= 8;  // the cluster's records fit in lanes 0-7
+  if (tid == 0) {
+    mbar_init(&sh->xbar, 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(&sh->xbar, static_cast<unsigned>(C * sizeof(X1)));
+  }
+  cluster_arrive_relaxed();  // waited for before the first push
   ring_prologue<T>(ring, ga, gb, gt, v0, v1, R);
 
   // ---- pass 1: the row normalisers, combined over the cluster
@@ -462,6 +508,8 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
     if (lane == 0) sh->w1[warp] = e;
     __syncthreads();
   }
+  // every CTA's mbarrier was initialised before any push (completes at once)
+  cluster_wait();
   if (warp == 0) {
     // the CTA's record: the warps' records merged (their references differ)
     X1 x = x1_neutral();
@@ -474,16 +522,36 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
       x.s[1] = r.s[1];
       x.s[3] = r.s[2];
     }
-    if (draft) warp_reduce_x1<FD>(x);
-    else warp_reduce_x1<F_LS>(x);
+    if (m3) {
+      if (draft) warp_reduce_x1_8<FD>(x);
+      else warp_reduce_x1_8<F_LS>(x);
+    } else {
+      if (draft) warp_reduce_x1<FD>(x);
+      else warp_reduce_x1<F_LS>(x);
+    }
     x.bad = 0u;
-    push_record(x, sh->recv(), rank, C, cluster);
+    if (lane < C) {
+      const float4* src = reinterpret_cast<const float4*>(&x);
+      X1* slot = sh->recv() + rank;
+#pragma unroll
+      for (int w = 0; w < static_cast<int>(sizeof(X1) / 16); ++w)
+        st_async16(reinterpret_cast<const float4*>(slot) + w, static_cast<unsigned>(lane), &sh->xbar,
+                   src[w]);
+    }
   }
-  cluster_barrier(warp == 0);  // every CTA's pass-1 record is in every CTA
+  cluster_arrive_relaxed();  // waited for before the CTA exits
   if (warp == 0) {
+    // every CTA's pass-1 record is in this CTA once the barrier completes
+    const bool got = mbar_wait_cluster_bounded(&sh->xbar, 0, kCopyTimeoutNs);
     X1 x = (lane < C) ? sh->recv()[lane] : x1_neutral();
-    if (draft) warp_reduce_x1<FD>(x);
-    else warp_reduce_x1<F_LS>(x);
+    if (m3) {
+      if (draft) warp_reduce_x1_8<FD>(x);
+      else warp_reduce_x1_8<F_LS>(x);
+    } else {
+      if (draft) warp_reduce_x1<FD>(x);
+      else warp_reduce_x1<F_LS>(x);
+    }
+    if (!got) x.bad |= kBadTimeout;
     if (lane == 0) {
       float lse[4];
       lse[0] = draft ? x.ref[0] + logf(x.s[0]) : NAN;
@@ -515,6 +583,7 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
     rec[0] = make_float4(jsum, 0.f, 0.f, draft ? msum : 0.f);
     rec[1] = make_float4(qf, 0.f, 0.f, 0.f);
   }
+  cluster_wait();  // no CTA exits while a push to it may be in flight
 }
 
 }  // namespace asymspec_impl
