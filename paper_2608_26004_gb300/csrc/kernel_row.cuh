@@ -130,20 +130,20 @@ struct __align__(16) W1 {
   float pad;
 };
 
-// Shared state of the row kernel; the C pass-1 records pushed by the
-// cluster follow it (recv()).
+// Shared state of the row kernel; the pass-1 records of every warp of the
+// cluster follow it (recv(): C x kRowThreads / 32 records, the record of
+// warp w of CTA r at r kRowThreads / 32 + w).
 struct __align__(16) RowShared {
-  W1 w1[kRowMaxWarps];  // per-warp pass-1 records
-  float lse[4];         // the row's normalisers (a, b, -, s)
-  unsigned long long xbar;  // completes when the cluster's C records have landed
+  float lse[4];             // the row's normalisers (a, b, -, s)
+  unsigned long long xbar;  // completes when the cluster's records have landed
   unsigned long long pad2;
-  __device__ X1* recv() { return reinterpret_cast<X1*>(this + 1); }
+  __device__ W1* recv() { return reinterpret_cast<W1*>(this + 1); }
 };
 static_assert(sizeof(W1) == 32, "one warp record is two 16-byte words");
 static_assert(sizeof(RowShared) % 16 == 0, "records after RowShared stay 16-byte aligned");
 
 __host__ __device__ constexpr int row_shared_bytes(int C) {
-  return static_cast<int>(sizeof(RowShared) + C * sizeof(X1));
+  return static_cast<int>(sizeof(RowShared) + C * (kRowThreads / 32) * sizeof(W1));
 }
 
 // ---------------------------------------------------------------- the rings
@@ -411,23 +411,37 @@ __device__ __forceinline__ void cluster_arrive_relaxed() {
 __device__ __forceinline__ void cluster_wait() {
   asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
 }
-// The record combine of warp_reduce_x1 over lanes 0-7 only (the others hold
-// the neutral record): three butterfly levels.
-template <unsigned F>
-__device__ __forceinline__ void warp_reduce_x1_8(X1& e) {
+// The row's pass-1 result from the n warp records of its cluster, by one
+// warp: lane l merges records l, l + 32, ... (each stream's sums restated
+// against the largest of their references), then the lanes' results are
+// combined as warp_reduce_x1 combines them.  Every lane ends with the same
+// (bit-identical) result, and so does every CTA, whose records are the same.
+__device__ __forceinline__ void combine_records(const W1* rec, int n, float (&ref)[3],
+                                                float (&sum)[3]) {
+  const int lane = static_cast<int>(threadIdx.x & 31);
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const unsigned bit = q == 0 ? F_LA : q == 1 ? F_LB : q == 2 ? F_LT : F_LS;
-    if (F & bit) {
-      const float M = warp_max(e.ref[q]);
-      float s = (e.s[q] == 0.f || e.ref[q] == M) ? e.s[q] : e.s[q] * ex2((e.ref[q] - M) * kLog2e);
+  for (int q = 0; q < 3; ++q) {
+    ref[q] = -INFINITY;
+    sum[q] = 0.f;
+  }
+  for (int i = lane; i < n; i += 32) {
+    const W1 r = rec[i];
 #pragma unroll
-      for (int off = 4; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-      e.ref[q] = M;
-      e.s[q] = s;
+    for (int q = 0; q < 3; ++q) {
+      const float M = fmaxf(ref[q], r.ref[q]);
+      const float a = (sum[q] == 0.f || ref[q] == M) ? sum[q] : sum[q] * ex2((ref[q] - M) * kLog2e);
+      const float b = (r.s[q] == 0.f || r.ref[q] == M) ? r.s[q] : r.s[q] * ex2((r.ref[q] - M) * kLog2e);
+      ref[q] = M;
+      sum[q] = a + b;
     }
   }
-  e.bad = __reduce_or_sync(0xffffffffu, e.bad);
+#pragma unroll
+  for (int q = 0; q < 3; ++q) {
+    const float M = warp_max(ref[q]);
+    const float v = (sum[q] == 0.f || ref[q] == M) ? sum[q] : sum[q] * ex2((ref[q] - M) * kLog2e);
+    ref[q] = M;
+    sum[q] = warp_sum(v);
+  }
 }
 
 // The cluster's index in the grid: (row k of batch element bi) = (x, y).
@@ -456,7 +470,6 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   constexpr int NW = kRowThreads / 32;
   constexpr int VE = 16 / static_cast<int>(sizeof(T));
-  constexpr unsigned FD = F_LA | F_LB | F_LS;
   extern __shared__ __align__(128) unsigned char smem_row[];
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
@@ -481,87 +494,58 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
   RowShared* sh = reinterpret_cast<RowShared*>(smem_row);
   uint4* ring = reinterpret_cast<uint4*>(smem_row + P.sh_off) + warp * (kRing * 96);
   const bool draft = k < P.K;
-  const bool m3 = C <= 8;  // the cluster's records fit in lanes 0-7
+  const int nrec = C * NW;  // pass-1 records the cluster exchanges
   if (tid == 0) {
     mbar_init(&sh->xbar, 1);
     fence_mbar_init();
-    mbar_arrive_expect_tx(&sh->xbar, static_cast<unsigned>(C * sizeof(X1)));
+    mbar_arrive_expect_tx(&sh->xbar, static_cast<unsigned>(nrec * sizeof(W1)));
   }
-  cluster_arrive_relaxed();  // waited for before the first push
+  cluster_arrive_relaxed();
   ring_prologue<T>(ring, ga, gb, gt, v0, v1, R);
+  // every CTA's barrier is initialised before any push (the CTAs of a
+  // cluster start together; this wait overlaps the first loads)
+  cluster_wait();
 
   // ---- pass 1: the row normalisers, combined over the cluster
   W1 e;
-  const bool ovf = draft ? row_pass1<T, true>(ring, ga, gb, gt, v0, v1, R, P.beta, e)
-                         : row_pass1<T, false>(ring, ga, gb, gt, v0, v1, R, P.beta, e);
+  bool ovf = draft ? row_pass1<T, true>(ring, ga, gb, gt, v0, v1, R, P.beta, e)
+                   : row_pass1<T, false>(ring, ga, gb, gt, v0, v1, R, P.beta, e);
   cp_async_wait<0>();  // the pass's trailing (empty) groups; the ring is free
   // pass 2's first steps do not depend on the normalisers
   ring_prologue<T>(ring, ga, gb, gt, v0, v1, R);
-  if (lane == 0) sh->w1[warp] = e;
-  if (__syncthreads_or(ovf)) {
-    // an entry far above its warp's reference (or non-finite data): redo the
-    // slice with running maxima
+  if (__any_sync(0xffffffffu, ovf)) {
+    // an entry far above the warp's reference (or non-finite data): redo the
+    // block with running maxima
     if (draft) row_pass1_online<T, true>(ga, gb, gt, v0, v1, P.beta, e);
     else row_pass1_online<T, false>(ga, gb, gt, v0, v1, P.beta, e);
-    e.bad = 0u;
-    e.pad = 0.f;
-    if (lane == 0) sh->w1[warp] = e;
-    __syncthreads();
   }
-  // every CTA's mbarrier was initialised before any push (completes at once)
-  cluster_wait();
-  if (warp == 0) {
-    // the CTA's record: the warps' records merged (their references differ)
-    X1 x = x1_neutral();
-    if (lane < NW) {
-      const W1 r = sh->w1[lane];
-      x.ref[0] = r.ref[0];
-      x.ref[1] = r.ref[1];
-      x.ref[3] = r.ref[2];
-      x.s[0] = r.s[0];
-      x.s[1] = r.s[1];
-      x.s[3] = r.s[2];
-    }
-    if (m3) {
-      if (draft) warp_reduce_x1_8<FD>(x);
-      else warp_reduce_x1_8<F_LS>(x);
-    } else {
-      if (draft) warp_reduce_x1<FD>(x);
-      else warp_reduce_x1<F_LS>(x);
-    }
-    x.bad = 0u;
-    if (lane < C) {
-      const float4* src = reinterpret_cast<const float4*>(&x);
-      X1* slot = sh->recv() + rank;
-#pragma unroll
-      for (int w = 0; w < static_cast<int>(sizeof(X1) / 16); ++w)
-        st_async16(reinterpret_cast<const float4*>(slot) + w, static_cast<unsigned>(lane), &sh->xbar,
-                   src[w]);
-    }
+  e.bad = 0u;
+  e.pad = 0.f;
+  if (lane < C) {
+    // this warp's record into slot rank NW + warp of every CTA (lane j to CTA j)
+    const float4* slot = reinterpret_cast<const float4*>(sh->recv() + rank * NW + warp);
+    st_async16(slot, static_cast<unsigned>(lane), &sh->xbar,
+               make_float4(e.ref[0], e.ref[1], e.ref[2], e.s[0]));
+    st_async16(slot + 1, static_cast<unsigned>(lane), &sh->xbar,
+               make_float4(e.s[1], e.s[2], 0.f, 0.f));
   }
   cluster_arrive_relaxed();  // waited for before the CTA exits
   if (warp == 0) {
-    // every CTA's pass-1 record is in this CTA once the barrier completes
+    // every warp's record of the cluster is in this CTA once the barrier completes
     const bool got = mbar_wait_cluster_bounded(&sh->xbar, 0, kCopyTimeoutNs);
-    X1 x = (lane < C) ? sh->recv()[lane] : x1_neutral();
-    if (m3) {
-      if (draft) warp_reduce_x1_8<FD>(x);
-      else warp_reduce_x1_8<F_LS>(x);
-    } else {
-      if (draft) warp_reduce_x1<FD>(x);
-      else warp_reduce_x1<F_LS>(x);
-    }
-    if (!got) x.bad |= kBadTimeout;
+    float ref[3], sum[3];
+    combine_records(sh->recv(), nrec, ref, sum);
     if (lane == 0) {
       float lse[4];
-      lse[0] = draft ? x.ref[0] + logf(x.s[0]) : NAN;
-      lse[1] = draft ? x.ref[1] + logf(x.s[1]) : NAN;
+      lse[0] = draft ? ref[0] + logf(sum[0]) : NAN;
+      lse[1] = draft ? ref[1] + logf(sum[1]) : NAN;
       lse[2] = NAN;
-      lse[3] = x.ref[3] + logf(x.s[3]);
+      lse[3] = ref[2] + logf(sum[2]);
 #pragma unroll
       for (int q = 0; q < 4; ++q) sh->lse[q] = lse[q];
       // the draft token's logits are read by the decision kernel itself
-      if (rank == 0) store_row_stat(P, row32, lse, INT_MAX, INT_MAX, x.bad, -1, 0.f, 0.f, 0.f);
+      if (rank == 0)
+        store_row_stat(P, row32, lse, INT_MAX, INT_MAX, got ? 0u : kBadTimeout, -1, 0.f, 0.f, 0.f);
     }
   }
   __syncthreads();
