@@ -529,10 +529,10 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
     st_async16(slot + 1, static_cast<unsigned>(lane), &sh->xbar,
                make_float4(e.s[1], e.s[2], 0.f, 0.f));
   }
-  cluster_arrive_relaxed();  // waited for before the CTA exits
+  bool got = true;
   if (warp == 0) {
     // every warp's record of the cluster is in this CTA once the barrier completes
-    const bool got = mbar_wait_cluster_bounded(&sh->xbar, 0, kCopyTimeoutNs);
+    got = mbar_wait_cluster_bounded(&sh->xbar, 0, kCopyTimeoutNs);
     float ref[3], sum[3];
     combine_records(sh->recv(), nrec, ref, sum);
     if (lane == 0) {
@@ -567,7 +567,10 @@ __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(co
     rec[0] = make_float4(jsum, 0.f, 0.f, draft ? msum : 0.f);
     rec[1] = make_float4(qf, 0.f, 0.f, 0.f);
   }
-  cluster_wait();  // no CTA exits while a push to it may be in flight
+  // no CTA exits while a push to it may be in flight: once the barrier has
+  // completed every push has landed; after a wait that gave up, warp 0 waits
+  // once more (bounded) before the CTA may exit
+  if (warp == 0 && !got) mbar_wait_cluster_bounded(&sh->xbar, 0, kCopyTimeoutNs);
 }
 
 }  // namespace asymspec_impl
