@@ -68,8 +68,10 @@ extern "C" {
 #define ASYMSPEC_DATA_NONFINITE 0x2u    /* a non-finite normaliser or divergence (NaN/inf logits) */
 #define ASYMSPEC_DATA_BAD_PROB 0x4u     /* stochastic: draft probability outside (0, 1] */
 #define ASYMSPEC_DATA_BAD_UNIFORM 0x8u  /* stochastic: uniform outside [0, 1) */
-#define ASYMSPEC_DATA_TIMEOUT 0x10u     /* a bulk copy into shared memory did not complete within
-                                           its time limit (the kernel gave up instead of hanging) */
+#define ASYMSPEC_DATA_TIMEOUT 0x10u     /* a bulk copy into shared memory (staged row kernel) or the
+                                           exchange of the cluster's pass-1 records (production row
+                                           kernel) did not complete within its time limit (the
+                                           kernel gave up instead of hanging) */
 #define ASYMSPEC_DATA_BAD_MAP 0x20u     /* cross-family step: a map entry outside its vocabulary */
 
 typedef enum { ASYMSPEC_FP32 = 0, ASYMSPEC_BF16 = 1 } asymspec_dtype_t;
@@ -131,8 +133,9 @@ typedef struct {
  * every cluster barrier, and before it exits waits (with the normal limit)
  * for its copies in flight; every batch element comes back as a data error
  * (accept_len = next_token = -1) with ASYMSPEC_DATA_TIMEOUT in the error
- * word.  The generic kernel and the production row kernel (fuse_verify_row)
- * wait on no copies and ignore it. */
+ * word.  The generic kernel waits on no copies and ignores it; so does the
+ * production row kernel (fuse_verify_row), whose one bounded wait (the
+ * record exchange, 200 ms) the hook does not shorten. */
 #define ASYMSPEC_TEST_COPY_GIVE_UP 1
 
 /* Kernels (asymspec_launch_opts.kernel, asymspec_launch_info.kernel). */
@@ -140,7 +143,9 @@ typedef struct {
 #define ASYMSPEC_KERNEL_TMA 2      /* one cluster per row, then a decision kernel; rows
                                       16-byte aligned.  The stochastic JSD step without debug
                                       outputs runs the production row kernel (slices read
-                                      from HBM, then again from the L2); every other program
+                                      from HBM, then again from the L2; C chosen so that the
+                                      rows in flight stay within an L2 budget once a batch
+                                      fills a wave of clusters of 8); every other program
                                       stages its slices by chunked 1-D bulk copies */
 
 /* What a launch would use (filled by asymspec_plan). */

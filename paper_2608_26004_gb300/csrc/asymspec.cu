@@ -114,29 +114,98 @@ bool plan_tma(int V, int elt, int forced_C, Plan* pl) {
   return false;
 }
 
-// The production row kernel: the first cluster size (8, 12, 16, 4, 10, 2,
-// 1; 8 packs GB300's GPCs best at four CTAs per SM) whose warp blocks take
-// at most kMaxRounds steps (the decision kernel's walk loads a whole block
-// at once).  Only the pass-1 records live in shared memory.  forced_C: the
-// caller's asymspec_launch_opts.
-bool plan_row(int V, int dtype, int forced_C, Plan* pl) {
+// The production row kernel.  Pass 2 re-reads each row from the L2, so the
+// rows in flight (one per resident cluster) must stay well inside it, while
+// fewer CTAs per row give each warp a longer block over which the fixed
+// costs of a CTA (its launch, the first loads, the exchange of the pass-1
+// records) are spread.  With at least one wave of clusters of 8 (rows x 8 >=
+// 4 CTAs x SMs): the smallest C of kRowClusters whose resident clusters
+// hold at most kRowL2Budget of rows.  Measured on GB300 (kernel time, rows
+// in flight):
+//   B=64, K=7, V=128256 bf16:  C=5 103.4 us (90 MB), C=6 97.3 us (75 MB), C=8 102.4 us (57 MB)
+//   B=32, K=8, V=151936 bf16:  C=6 70.7 us (88 MB), C=7 71.7 us (74 MB), C=8 75.8 us (67 MB)
+//   B=128, K=4, V=151936 fp32: C=12 207.9 us (84 MB), C=16 247.8 us (60 MB)
+// Smaller batches take C = 8.  A warp's block takes at most kWalkRounds
+// steps (the decision kernel's walk loads a whole block at once).  Only the
+// pass-1 records live in shared memory.  forced_C: the caller's
+// asymspec_launch_opts.
+constexpr int kRowClusters[] = {4, 5, 6, 7, 8, 10, 12, 16};
+constexpr double kRowL2Budget = 86.0e6;
+
+struct DeviceShape {
+  int device, sms;
+  bool ok;
+};
+DeviceShape device_shape() {
+  DeviceShape d{0, 152, false};  // GB300 when no device answers
+  int n = 0;
+  if (cudaGetDevice(&d.device) == cudaSuccess &&
+      cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, d.device) == cudaSuccess && n > 0) {
+    d.sms = n;
+    d.ok = true;
+  }
+  cudaGetLastError();
+  return d;
+}
+
+const void* row_kernel(int dtype);
+cudaError_t prepare_kernel(const void* fn, int device);
+cudaError_t active_clusters(const void* fn, const Plan& pl, int device, int* out);
+
+bool plan_row(int V, int dtype, int forced_C, long long rows, Plan* pl) {
   const int elt = elt_size(dtype);
   const int VE = 16 / elt;
-  constexpr int kRowClusters[] = {8, 12, 16, 4, 10, 2, 1};
-  for (int C : kRowClusters) {
-    if (forced_C && C != forced_C) continue;
+  auto width = [&](int C) {
     const long long per = (static_cast<long long>(V) + C - 1) / C;
-    const long long W = round_up_ll(per, VE);
-    if (W / VE > static_cast<long long>(kMaxRounds) * kRowThreads) continue;
-    pl->C = C;
-    pl->W = static_cast<int>(W);
-    pl->sh_off = row_shared_bytes(C);  // the warps' rings follow the fixed state
-    pl->smem = row_shared_bytes(C) + kRingBytes;
-    pl->group_stride = kGroupsMax;
-    pl->nt = kRowThreads;
-    return true;
+    return round_up_ll(per, VE);
+  };
+  auto fits = [&](int C) {
+    return width(C) / VE <= static_cast<long long>(kWalkRounds) * kRowThreads;
+  };
+  int C = 0;
+  if (forced_C) {
+    if (fits(forced_C)) C = forced_C;
+  } else {
+    const DeviceShape dev = device_shape();
+    const long long slots = static_cast<long long>(dev.sms) * kRowMinBlocks;
+    const double row_bytes = 3.0 * V * elt;
+    if (rows * 8 < slots) {
+      if (fits(8)) C = 8;
+    } else {
+      const void* fn = row_kernel(dtype);
+      const bool query = dev.ok && prepare_kernel(fn, dev.device) == cudaSuccess;
+      for (int c : kRowClusters) {
+        if (!fits(c)) continue;
+        // the clusters the device holds at once (an estimate without a device)
+        long long resident = slots / c;
+        Plan q = *pl;
+        q.C = c;
+        q.smem = row_shared_bytes(c) + kRingBytes;
+        q.nt = kRowThreads;
+        q.kernel = ASYMSPEC_KERNEL_TMA;
+        q.grid_y = 1;
+        int n = 0;
+        if (query && active_clusters(fn, q, dev.device, &n) == cudaSuccess && n > 0) resident = n;
+        cudaGetLastError();
+        if (static_cast<double>(std::min(rows, resident)) * row_bytes <= kRowL2Budget) {
+          C = c;
+          break;
+        }
+      }
+    }
+    if (!C) {  // nothing within the budget (or no full wave): the largest cluster that fits
+      for (int c : kRowClusters)
+        if (fits(c)) C = c;
+    }
   }
-  return false;
+  if (!C) return false;
+  pl->C = C;
+  pl->W = static_cast<int>(width(C));
+  pl->sh_off = row_shared_bytes(C);  // the warps' rings follow the fixed state
+  pl->smem = row_shared_bytes(C) + kRingBytes;
+  pl->group_stride = kGroupsMax;
+  pl->nt = kRowThreads;
+  return true;
 }
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -193,7 +262,7 @@ int make_plan(int B, int K, int V, int dtype, const asymspec_launch_opts* opts, 
   bool ok = false;
   // (its grid is (C (K+1), B): B up to 65535)
   if (forced_kernel != ASYMSPEC_KERNEL_GENERIC && vec_ok && prod_row && B <= 65535 &&
-      plan_row(V, dtype, forced_C, pl)) {
+      plan_row(V, dtype, forced_C, static_cast<long long>(B) * (K + 1), pl)) {
     if (ws_bytes >= tma_layout(B, K, pl->C).total) {
       pl->kernel = ASYMSPEC_KERNEL_TMA;
       pl->VE = 16 / elt;

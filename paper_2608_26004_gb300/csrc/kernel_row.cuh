@@ -4,10 +4,11 @@
 // Same decomposition as fuse_verify_tma (kernel_tma.cuh), whose records it
 // leaves for the same decision kernel: one cluster of C CTAs per row triple
 // (a_k, b_k, t_k), CTA r taking entries [r W, (r+1) W) of the three rows;
-// pass 1 (the normalisers of Eqs. 1-3) over the slice; the CTAs exchange
-// pass-1 records through distributed shared memory and one cluster barrier;
-// pass 2 (the divergence of Eq. 3 and the masses of the fused and residual
-// distributions) over the slice again.
+// pass 1 (the normalisers of Eqs. 1-3) over the slice; every warp pushes its
+// pass-1 record into every CTA of the cluster (distributed shared memory,
+// st.async completing on the receiver's mbarrier); pass 2 (the divergence of
+// Eq. 3 and the masses of the fused and residual distributions) over the
+// slice again.
 //
 // What differs from fuse_verify_tma is where the slice lives between the
 // passes and the shape of the work:
@@ -15,14 +16,19 @@
 //     of the slice and reads it twice through a small ring in shared memory
 //     (kRing steps of 32 consecutive 16-byte vectors per stream, filled with
 //     cp.async): pass 1 from HBM, pass 2 from the L2, where pass 1 just
-//     brought it.  The rows in flight at once (one per resident cluster: 74
-//     clusters of 8 CTAs on GB300, 57 MB for V = 128256 bf16) sit well inside
-//     the 129 MB L2, so each logit row still comes from HBM once.  With 48 KB
-//     of rings and the pass-1 records in shared memory, four 256-thread CTAs
+//     brought it.  The rows in flight at once (one per resident cluster:
+//     97 clusters of 6 CTAs on GB300 for V = 128256 bf16, 75 MB; the host
+//     picks C so that they stay within its L2 budget) sit inside the 129 MB
+//     L2, so each logit row comes from HBM about once.  With 48 KB of rings
+//     and the cluster's pass-1 records in shared memory, four 256-thread CTAs
 //     fit on an SM (the register file is the limit), against three when the
 //     slice is staged whole; the ring keeps four steps of every warp in
 //     flight without holding registers, and pass 2's first steps are issued
-//     before the cluster barrier;
+//     while the records are exchanged;
+//   * no CTA or cluster barrier between the passes but the one __syncthreads
+//     after warp 0 has combined the records: a warp pushes its record as soon
+//     as its block is done, and the exchange completes on each receiver's
+//     mbarrier when the last record of the cluster lands;
 //   * the block of a warp is one inverse-CDF group: its mass is the warp's
 //     residual (or fused) sum, which the warp reduces anyway, so pass 2 needs
 //     no per-step group reductions (the decision kernel walks the group's
@@ -39,9 +45,11 @@
 //     are formed exactly as the decision kernel's inverse-CDF walk forms
 //     them (res_pair), so the group masses and the walk agree bit for bit.
 //
-// The kernel waits on nothing but the hardware cluster barrier, CTA
-// barriers and its own cp.async groups (no copies complete on mbarriers), so
-// it never reports ASYMSPEC_DATA_TIMEOUT.
+// Waits: one cluster barrier at the start (every CTA's mbarrier is
+// initialised before the first push), CTA barriers, its own cp.async groups,
+// and the record exchange's mbarrier, bounded by %globaltimer: a wait that
+// gives up reports ASYMSPEC_DATA_TIMEOUT for the row, and is waited for once
+// more (bounded) before the CTA exits, so that a late push finds it alive.
 #pragma once
 
 #include "kernel_tma.cuh"
@@ -464,7 +472,8 @@ __device__ __forceinline__ unsigned cluster_id_y() {
 // masses of its block (its inverse-CDF group).  Dynamic shared memory: the
 // fixed state and pushed records (row_shared_bytes(C)), then the warps'
 // rings (kRingBytes) at KParams::sh_off.  Pass 2's first kRing steps are
-// issued before the cluster barrier: they do not depend on the normalisers.
+// issued before the records are exchanged: they do not depend on the
+// normalisers.
 template <typename T>
 __global__ void __launch_bounds__(kRowThreads, kRowMinBlocks) fuse_verify_row(const KParams P) {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");

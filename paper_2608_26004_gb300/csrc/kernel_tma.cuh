@@ -54,6 +54,7 @@ namespace asymspec_impl {
 constexpr int kTThreads = 256;
 constexpr int kTWarps = kTThreads / 32;
 constexpr int kMaxRounds = 10;  // 16-byte vectors per thread per slice
+constexpr int kWalkRounds = 16;  // steps of 32 vectors in a group the walk takes
 constexpr int kChunks = 4;      // bulk-copy chunks per slice
 constexpr unsigned long long kCopyTimeoutNs = 200ull * 1000ull * 1000ull;
 constexpr float kSumLimit = 1.2676506e30f;  // 2^100: pass1_fast's overflow guard
@@ -1191,9 +1192,9 @@ __device__ __noinline__ int walk_vectors(const T* ga, const T* gb, const T* gt, 
   }
   cp_async_wait_all();
   __syncwarp();
-  float mvs[kMaxRounds];
+  float mvs[kWalkRounds];
 #pragma unroll
-  for (int s = 0; s < kMaxRounds; ++s) {
+  for (int s = 0; s < kWalkRounds; ++s) {
     const int j = 32 * s + lane;
     mvs[s] = 0.f;
     if (j < nvb) {
@@ -1206,7 +1207,7 @@ __device__ __noinline__ int walk_vectors(const T* ga, const T* gb, const T* gt, 
   int vsel = -1, vlast = -1;
   float tin = 0.f;  // the target's offset inside the selected vector
 #pragma unroll
-  for (int s = 0; s < kMaxRounds; ++s) {
+  for (int s = 0; s < kWalkRounds; ++s) {
     const int base = b0 + 32 * s;
     if (base >= b1 || vsel >= 0) break;
     const float mv = mvs[s];
