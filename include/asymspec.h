@@ -246,8 +246,9 @@ int asymspec_fuse_verify_ex(const void* logits_full, const void* logits_comp,
  * kernel's records and tickets for B*(K+1) <= 8192 rows (16 bytes per row
  * and 4 per batch element); larger batches return ASYMSPEC_ERR_SCRATCH_LIMIT
  * before anything is enqueued.  Aligned rows run ASYMSPEC_KERNEL_TMA when
- * the array also holds its per-row results (about 1400 rows in clusters of
- * 8), else the generic kernel.  Each call enqueues on `stream` a zero fill
+ * the array also holds its per-row results (48 + 576 C bytes a row for
+ * clusters of C: about 890 rows at C = 8, 1190 at C = 6), else the generic
+ * kernel.  Each call enqueues on `stream` a zero fill
  * of the B tickets (the only part that must start at zero), then the
  * launches of asymspec_fuse_verify_ex.  Nothing is allocated: no
  * cudaMalloc, cudaMallocAsync, cudaFree or library call that allocates.
