@@ -220,6 +220,12 @@ def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
     assert info.launches == 1 and info.row_kernel == 0
     info = A.plan(64, 7, 128256, A.BF16, A.gate_params(mode=A.MODE_STOCHASTIC))
     assert info.launches == 2 and info.row_kernel == 1
+    # the production row kernel: clusters of 6 keep ~97 rows of 770 KB in flight
+    # (within the L2 budget; clusters of 5 would hold ~117); warp blocks of 334 vectors
+    assert info.cluster_size == 6 and info.slice_elems == 21376 and info.ctas == 512 * 6
+    # fewer rows than a wave of clusters of 8: clusters of 8
+    small = A.plan(8, 5, 151936, A.BF16, A.gate_params(mode=A.MODE_STOCHASTIC))
+    assert small.row_kernel == 1 and small.cluster_size == 8
     info = A.plan(64, 7, 128256, A.BF16, A.gate_params(mode=A.MODE_GREEDY))
     assert info.launches == 2 and info.row_kernel == 0
     with pytest.raises(A.AsymSpecError):
