@@ -438,8 +438,9 @@ cudaError_t record_timing(const asymspec_launch_opts* opts, bool begin, cudaStre
 // uses any workspace.  The generic kernel needs records for
 // ASYMSPEC_STATIC_MAX_ROWS rows and tickets for the largest batch that can
 // have that many rows (K >= 1, so B <= ASYMSPEC_STATIC_MAX_ROWS / 2): 144 KiB.
-// 4 MiB also holds the TMA kernel's per-row results for about 1400 rows in
-// clusters of 8 (2880 bytes a row); larger batches take the generic kernel.
+// 4 MiB also holds the cluster kernels' per-row results (48 + 576 C bytes a
+// row for clusters of C: about 890 rows at C = 8, 1190 at C = 6); larger
+// batches take the generic kernel.
 constexpr size_t kStaticScratchBytes = ASYMSPEC_STATIC_SCRATCH_BYTES;
 static_assert(kStaticScratchBytes >= static_cast<size_t>(ASYMSPEC_STATIC_MAX_ROWS) * sizeof(int4) +
                                          static_cast<size_t>(ASYMSPEC_STATIC_MAX_ROWS / 2) *
