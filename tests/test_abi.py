@@ -240,6 +240,33 @@ def test_plan_picks_kernels_and_clusters_that_fit_on_chip(lib):
         A.plan(2, 2, 4099, A.BF16, opts=A.LaunchOpts(0, 0, A.KERNEL_TMA))
 
 
+def test_row_kernel_plans_fit_on_chip_across_shapes(lib):
+    # the production row kernel's plan over batch sizes, row widths and dtypes:
+    # a cluster size the planner offers, warp blocks the decision kernel's walk
+    # can stage (16 steps of 32 vectors), four CTAs an SM, one cluster per row;
+    # a batch smaller than a wave of clusters of 8 keeps 8 whenever it fits
+    S = A.gate_params(mode=A.MODE_STOCHASTIC)
+    for dtype, elt in ((A.BF16, 2), (A.FP32, 4)):
+        ve = 16 // elt
+        for V in (4096, 32000, 50000, 109568, 128256, 151936, 200000):
+            for B, K in ((1, 4), (8, 5), (32, 8), (64, 7), (256, 4)):
+                try:
+                    info = A.plan(B, K, V, dtype, S)
+                except A.AsymSpecError as e:
+                    assert e.status == A.ERR_TOO_LARGE
+                    continue
+                if not info.row_kernel:
+                    continue
+                C, W = info.cluster_size, info.slice_elems
+                assert C in (4, 5, 6, 7, 8, 10, 12, 16), (dtype, V, B, K, C)
+                assert C * W >= V and W % ve == 0 and W - (V + C - 1) // C < ve
+                assert -(-(W // ve) // 8) <= 16 * 32
+                assert 4 * (info.smem_bytes + 1024) <= 228 * 1024
+                assert info.ctas == B * (K + 1) * C and info.block_threads == 256
+                if B * (K + 1) * 8 < 152 * 4 and (V + 7) // 8 <= 16 * 256 * ve:
+                    assert C == 8
+
+
 def test_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):
     monkeypatch.setattr(A, "_lib", None)
     monkeypatch.setattr(A, "LIB_PATH", str(tmp_path / "missing.so"))
